@@ -1,0 +1,550 @@
+/*
+ * wm_oracle.c -- plain CPU oracle for the RLFlow world-model dream path.
+ *
+ * TEST INFRASTRUCTURE ONLY (see wm_oracle.h).  Straight loops, fp64, no
+ * blocking, fusion or reordering beyond the step order below:
+ *
+ *   for t = 0..T-1, for every episode independently:
+ *     a1  controller logits   l = W_c^T [z_t; h_t] + b_c           (Sec. 3.5)
+ *     a2  mask + select       invalid logits -> -inf; argmax or a
+ *                             tempered-softmax draw                 (Sec. 3.1.3)
+ *     a3  LSTM gates          G = W^T [z_t; onehot(a_t); h_t] + b   (Sec. 3.4.3)
+ *     a4  cell update         c' = f c + i g, h' = o tanh(c')
+ *     a5  heads               MDN params, reward, done logit on h'  (Sec. 3.4.3, 4.7)
+ *     a6  mixture weights     log softmax(logit / tau)              (temperature eq.)
+ *     a7  sample z_{t+1}      component by inverse CDF, then mu + sigma*eps
+ *     a8  done / freeze       done = logit > 0; frozen episodes stay put
+ *   a9  teacher-forced NLL  sum_t sum_d -log sum_k pi N(z_{t+1,d}; mu, sigma)  (Sec. 4.7)
+ *
+ * Readings where the paper is silent (all fixed here, mirrored by the kernels):
+ *   - the state (z, h, c) is carried in fp32 between steps; inside a step the
+ *     oracle computes in fp64;
+ *   - per-latent-dim 1-D mixtures, K logits per dim (3KZ head outputs);
+ *   - gate column order i,f,g,o, no implicit forget bias;
+ *   - masked logits become -inf (the paper "zeroes" them, which could not keep
+ *     a zeroed logit from winning an argmax);
+ *   - ties: lowest index; inverse CDF: first k with u < C_k, else K-1;
+ *   - tau = 0: argmax component, z = mu (the paper's "deterministic" limit);
+ *   - reward / done are linear heads on h_{t+1}; done = (logit > 0).
+ *
+ * Random numbers: Philox-4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11),
+ * key = (seed lo, seed hi), counter = (episode lo, step, purpose<<24 | block,
+ * episode hi).  Purpose 0: component uniforms (4 dims per block); purpose 1:
+ * normals by Box-Muller (4 dims per block, words (0,1) and (2,3) are pairs);
+ * purpose 2: the controller's sampling uniform (word 0 of block 0).
+ */
+#include "wm_oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifndef M_PI
+#define M_PI 3.14159265358979323846
+#endif
+
+/* ------------------------------------------------------------------------- */
+/* Philox-4x32-10, written from the round function of Salmon et al. (SC'11): */
+/* two 32x32->64 multiplies per round on words 0 and 2, the high halves are   */
+/* xored with the other words and the round key, the key is bumped by the     */
+/* Weyl constants between rounds.                                             */
+/* ------------------------------------------------------------------------- */
+void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4])
+{
+    uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+    uint32_t k0 = key[0], k1 = key[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+        uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+        uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+        uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+        uint32_t n0 = hi1 ^ c1 ^ k0;
+        uint32_t n1 = lo1;
+        uint32_t n2 = hi0 ^ c3 ^ k1;
+        uint32_t n3 = lo0;
+        c0 = n0; c1 = n1; c2 = n2; c3 = n3;
+    }
+    out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* u in [0,1): the top 24 bits scaled by 2^-24 (exact in fp32 and fp64). */
+double orc_uniform(uint32_t x)
+{
+    return (double)(x >> 8) * (1.0 / 16777216.0);
+}
+
+/* Box-Muller (1958): r = sqrt(-2 ln(1-u1)), theta = 2 pi u2. */
+void orc_box_muller(uint32_t x1, uint32_t x2, double *e0, double *e1)
+{
+    double u1 = orc_uniform(x1), u2 = orc_uniform(x2);
+    double r = sqrt(-2.0 * log(1.0 - u1));
+    double th = 2.0 * M_PI * u2;
+    *e0 = r * cos(th);
+    *e1 = r * sin(th);
+}
+
+void orc_draw(uint64_t seed, uint64_t episode, uint32_t step, uint32_t purpose,
+              uint32_t block, uint32_t out[4])
+{
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t ctr[4] = {(uint32_t)episode, step, (purpose << 24) | block,
+                       (uint32_t)(episode >> 32)};
+    orc_philox4x32_10(ctr, key, out);
+}
+
+/* fp32 -> bf16 round-to-nearest-even, returned widened to fp32. */
+float orc_bf16(float x)
+{
+    uint32_t u;
+    memcpy(&u, &x, 4);
+    uint32_t r;
+    if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu) != 0u) {
+        r = 0x7FC00000u;                          /* canonical quiet NaN */
+    } else {
+        uint32_t lsb = (u >> 16) & 1u;
+        r = ((u + 0x7FFFu + lsb) >> 16) << 16;   /* ties go to even */
+    }
+    float y;
+    memcpy(&y, &r, 4);
+    return y;
+}
+
+static double sigmoid(double v) { return 1.0 / (1.0 + exp(-v)); }
+
+/* a4: gates = [i | f | g | o] pre-activations, each H long. */
+void orc_lstm_cell(int H, const double *gates, const double *c_in,
+                   double *c_out, double *h_out)
+{
+    for (int u = 0; u < H; ++u) {
+        double ig = sigmoid(gates[u]);
+        double fg = sigmoid(gates[H + u]);
+        double gg = tanh(gates[2 * H + u]);
+        double og = sigmoid(gates[3 * H + u]);
+        double c = fg * c_in[u] + ig * gg;
+        c_out[u] = c;
+        h_out[u] = og * tanh(c);
+    }
+}
+
+/* a9 for one latent dim: -log sum_k softmax(logits)_k N(x; mu_k, exp(logsig_k)). */
+double orc_mixture_nll_1d(int K, const double *logits, const double *mu,
+                          const double *logsig, double x)
+{
+    double lmax = -INFINITY;
+    for (int k = 0; k < K; ++k) if (logits[k] > lmax) lmax = logits[k];
+    double s = 0.0;
+    for (int k = 0; k < K; ++k) s += exp(logits[k] - lmax);
+    double logz = lmax + log(s);
+    double terms[64];
+    double tmax = -INFINITY;
+    for (int k = 0; k < K; ++k) {
+        double zsc = (x - mu[k]) * exp(-logsig[k]);
+        double lp = (logits[k] - logz) - 0.5 * zsc * zsc - logsig[k] - 0.5 * log(2.0 * M_PI);
+        terms[k] = lp;
+        if (lp > tmax) tmax = lp;
+    }
+    double acc = 0.0;
+    for (int k = 0; k < K; ++k) acc += exp(terms[k] - tmax);
+    return -(tmax + log(acc));
+}
+
+/*
+ * a6 + a7 for one latent dim.  logits are the fp32-rounded head outputs.
+ * tau > 0: pi = softmax(logit / tau), k = first index with u < C_k (else K-1),
+ *          z = mu_k + sigma_k * s * eps with s = sqrt(tau) if sigma_sqrt_tau.
+ *          margin = min_k<K-1 |u - C_k|.
+ * tau = 0: k = argmax logit (lowest index), z = mu_k; margin = top-2 gap.
+ * Returns k.
+ */
+int orc_sample_dim(int K, double tau, int sigma_sqrt_tau, const float *logits,
+                   const double *mu, const double *logsig, double u, double eps,
+                   double *z, double *margin)
+{
+    if (tau <= 0.0) {
+        int best = 0;
+        for (int k = 1; k < K; ++k) if (logits[k] > logits[best]) best = k;
+        double gap = INFINITY;
+        for (int k = 0; k < K; ++k)
+            if (k != best && (double)logits[best] - (double)logits[k] < gap)
+                gap = (double)logits[best] - (double)logits[k];
+        *z = mu[best];
+        *margin = gap;
+        return best;
+    }
+    double lmax = -INFINITY;
+    for (int k = 0; k < K; ++k) if ((double)logits[k] / tau > lmax) lmax = (double)logits[k] / tau;
+    double p[64], s = 0.0;
+    for (int k = 0; k < K; ++k) { p[k] = exp((double)logits[k] / tau - lmax); s += p[k]; }
+    int chosen = K - 1;
+    double cum = 0.0, mg = INFINITY;
+    for (int k = 0; k < K; ++k) {
+        cum += p[k] / s;
+        if (k < K - 1) {
+            double d = fabs(u - cum);
+            if (d < mg) mg = d;
+        }
+        if (chosen == K - 1 && k < K - 1 && u < cum) chosen = k;
+    }
+    double scale = sigma_sqrt_tau ? sqrt(tau) : 1.0;
+    *z = mu[chosen] + exp(logsig[chosen]) * scale * eps;
+    *margin = mg;
+    return chosen;
+}
+
+static int bit_set(const uint32_t *words, int j)
+{
+    return (int)((words[j >> 5] >> (j & 31)) & 1u);
+}
+
+/*
+ * a2: masked action choice.  mask_words == NULL means every action is valid.
+ * argmax mode (ctrl_sample == 0 or ctrl_tau == 0): lowest index among the
+ * valid maxima; margin = top-2 gap among valid logits.
+ * sample mode: w_j = exp((l_j - l_max)/tau) on valid j, S = sum w, pick the
+ * first valid j with u*S < cumsum_j (else the last valid one);
+ * margin = min_j |u*S - cumsum_j| / S.
+ * Returns -1 when no action is valid.
+ */
+int orc_select_action(int A, const float *logits, const uint32_t *mask_words,
+                      int ctrl_sample, double ctrl_tau, double u, double *margin)
+{
+    int nvalid = 0, best = -1, last = -1;
+    for (int j = 0; j < A; ++j) {
+        if (mask_words && !bit_set(mask_words, j)) continue;
+        ++nvalid;
+        last = j;
+        if (best < 0 || logits[j] > logits[best]) best = j;
+    }
+    *margin = INFINITY;
+    if (nvalid == 0) return -1;
+    if (!ctrl_sample || ctrl_tau <= 0.0) {
+        double gap = INFINITY;
+        for (int j = 0; j < A; ++j) {
+            if (j == best || (mask_words && !bit_set(mask_words, j))) continue;
+            double g = (double)logits[best] - (double)logits[j];
+            if (g < gap) gap = g;
+        }
+        *margin = gap;
+        return best;
+    }
+    double lmax = (double)logits[best];
+    double S = 0.0;
+    for (int j = 0; j < A; ++j) {
+        if (mask_words && !bit_set(mask_words, j)) continue;
+        S += exp(((double)logits[j] - lmax) / ctrl_tau);
+    }
+    double target = u * S, cum = 0.0, mg = INFINITY;
+    int chosen = -1;
+    for (int j = 0; j < A; ++j) {
+        if (mask_words && !bit_set(mask_words, j)) continue;
+        cum += exp(((double)logits[j] - lmax) / ctrl_tau);
+        if (j != last) {
+            double d = fabs(target - cum) / S;
+            if (d < mg) mg = d;
+        }
+        if (chosen < 0 && target < cum) chosen = j;
+    }
+    if (chosen < 0) chosen = last;
+    *margin = mg;
+    return chosen;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Weights widened to fp64 (rounded to bf16 first in bf16 mode).             */
+/* ------------------------------------------------------------------------- */
+typedef struct {
+    double *W_lstm, *b_lstm, *W_mdn, *b_mdn, *w_rew, *w_done, *W_ctrl, *b_ctrl;
+    double b_rew, b_done;
+} wts64;
+
+static double *widen(const float *src, size_t n, int round_bf16)
+{
+    double *dst = (double *)malloc(n * sizeof(double));
+    if (!dst) return NULL;
+    for (size_t i = 0; i < n; ++i) dst[i] = round_bf16 ? (double)orc_bf16(src[i]) : (double)src[i];
+    return dst;
+}
+
+static void free_wts(wts64 *v)
+{
+    free(v->W_lstm); free(v->b_lstm); free(v->W_mdn); free(v->b_mdn);
+    free(v->w_rew); free(v->w_done); free(v->W_ctrl); free(v->b_ctrl);
+}
+
+static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need_ctrl)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
+    const int rb = cfg->bf16;
+    memset(v, 0, sizeof(*v));
+    v->W_lstm = widen(w->W_lstm, (size_t)(Z + A + H) * 4 * H, rb);
+    v->b_lstm = widen(w->b_lstm, (size_t)4 * H, 0);
+    v->W_mdn = widen(w->W_mdn, (size_t)H * 3 * K * Z, rb);
+    v->b_mdn = widen(w->b_mdn, (size_t)3 * K * Z, 0);
+    v->w_rew = widen(w->w_rew, (size_t)H, rb);
+    v->w_done = widen(w->w_done, (size_t)H, rb);
+    v->b_rew = (double)w->b_rew;
+    v->b_done = (double)w->b_done;
+    if (need_ctrl) {
+        v->W_ctrl = widen(w->W_ctrl, (size_t)(Z + H) * A, rb);
+        v->b_ctrl = widen(w->b_ctrl, (size_t)A, 0);
+    }
+    if (!v->W_lstm || !v->b_lstm || !v->W_mdn || !v->b_mdn || !v->w_rew || !v->w_done ||
+        (need_ctrl && (!v->W_ctrl || !v->b_ctrl))) {
+        free_wts(v);
+        return -1;
+    }
+    return 0;
+}
+
+/* GEMM A-operand: bf16-rounded through fp32 in bf16 mode, else fp32 value. */
+static double opnd(const orc_cfg *cfg, double v)
+{
+    float f = (float)v;
+    return cfg->bf16 ? (double)orc_bf16(f) : (double)f;
+}
+
+static int check_cfg(const orc_cfg *c)
+{
+    if (c->z_dim <= 0 || c->a_dim <= 0 || c->h_dim <= 0 || c->k_mix <= 0 || c->k_mix > 64) return -1;
+    if (!(c->mdn_tau >= 0.0) || !(c->ctrl_tau >= 0.0)) return -1;
+    return 0;
+}
+
+/* a3 + a4: one LSTM step for one episode.  x = [op(z); op(h)] of length Z+H. */
+static void lstm_step(const orc_cfg *cfg, const wts64 *v, const double *x, int a,
+                      double *gates, double *c, double *h)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, N4 = 4 * H;
+    for (int n = 0; n < N4; ++n) {
+        double g = v->b_lstm[n];
+        for (int i = 0; i < Z; ++i) g += x[i] * v->W_lstm[(size_t)i * N4 + n];
+        if (a >= 0) g += v->W_lstm[(size_t)(Z + a) * N4 + n];
+        for (int i = 0; i < H; ++i) g += x[Z + i] * v->W_lstm[(size_t)(Z + A + i) * N4 + n];
+        gates[n] = g;
+    }
+    orc_lstm_cell(H, gates, c, c, h);
+    /* the recurrent state is carried in fp32 between steps */
+    for (int u = 0; u < H; ++u) {
+        c[u] = (double)(float)c[u];
+        h[u] = (double)(float)h[u];
+    }
+}
+
+/* a5: MDN head outputs on y = op(h'). */
+static void mdn_head(const orc_cfg *cfg, const wts64 *v, const double *y, double *mdn)
+{
+    const int H = cfg->h_dim, M = 3 * cfg->k_mix * cfg->z_dim;
+    for (int m = 0; m < M; ++m) {
+        double s = v->b_mdn[m];
+        for (int i = 0; i < H; ++i) s += y[i] * v->W_mdn[(size_t)i * M + m];
+        mdn[m] = s;
+    }
+}
+
+#define INF_F ((float)INFINITY)
+
+static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int T,
+                           uint64_t episode_offset, uint32_t t0,
+                           const float *z0, const float *h0, const float *c0,
+                           const uint8_t *done0, const uint32_t *mask,
+                           float *z_out, int32_t *actions, float *rewards, uint8_t *done,
+                           float *h_final, float *c_final,
+                           float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
+                           float *ctrl_margin, float *comp_margin, float *done_margin)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
+    const int M = 3 * K * Z, W = (A + 31) / 32;
+    const uint64_t e = episode_offset + (uint64_t)b;
+    double *z = malloc(sizeof(double) * Z), *h = malloc(sizeof(double) * H);
+    double *c = malloc(sizeof(double) * H), *x = malloc(sizeof(double) * (Z + H));
+    double *g = malloc(sizeof(double) * 4 * H), *y = malloc(sizeof(double) * H);
+    double *mdn = malloc(sizeof(double) * M), *znew = malloc(sizeof(double) * Z);
+    float *lg = malloc(sizeof(float) * (A > K ? A : K));
+    if (!z || !h || !c || !x || !g || !y || !mdn || !znew || !lg) {
+        free(z); free(h); free(c); free(x); free(g); free(y); free(mdn); free(znew); free(lg);
+        return -1;
+    }
+    for (int i = 0; i < Z; ++i) z[i] = z0[(size_t)b * Z + i];
+    for (int i = 0; i < H; ++i) {
+        h[i] = h0 ? h0[(size_t)b * H + i] : 0.0;
+        c[i] = c0 ? c0[(size_t)b * H + i] : 0.0;
+    }
+    int frozen = done0 ? (done0[b] != 0) : 0;
+    for (int i = 0; i < Z; ++i) z_out[(size_t)b * Z + i] = (float)z[i];
+
+    for (int t = 0; t < T; ++t) {
+        const uint32_t s = t0 + (uint32_t)t;
+        const size_t tb = (size_t)t * B + b;
+        if (frozen) {
+            actions[tb] = -1; rewards[tb] = 0.0f; done[tb] = 1;
+            for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
+            if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
+            if (c_seq) for (int i = 0; i < H; ++i) c_seq[tb * H + i] = (float)c[i];
+            if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = 0.0f;
+            if (comp_seq) for (int d = 0; d < Z; ++d) comp_seq[tb * Z + d] = 255;
+            if (ctrl_margin) ctrl_margin[tb] = INF_F;
+            if (done_margin) done_margin[tb] = INF_F;
+            if (comp_margin) for (int d = 0; d < Z; ++d) comp_margin[tb * Z + d] = INF_F;
+            continue;
+        }
+        for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z[i]);
+        for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
+
+        /* a1: controller logits, rounded to fp32 for the decision */
+        for (int j = 0; j < A; ++j) {
+            double l = v->b_ctrl[j];
+            for (int i = 0; i < Z + H; ++i) l += x[i] * v->W_ctrl[(size_t)i * A + j];
+            lg[j] = (float)l;
+        }
+        /* a2: mask + select */
+        double u_ctrl = 0.0;
+        if (cfg->ctrl_sample && cfg->ctrl_tau > 0.0) {
+            uint32_t r4[4];
+            orc_draw(cfg->seed, e, s, 2u, 0u, r4);
+            u_ctrl = orc_uniform(r4[0]);
+        }
+        double cm;
+        const uint32_t *mw = mask ? mask + tb * W : NULL;
+        int a = orc_select_action(A, lg, mw, cfg->ctrl_sample, cfg->ctrl_tau, u_ctrl, &cm);
+        actions[tb] = a;
+        if (ctrl_margin) ctrl_margin[tb] = (float)cm;
+
+        /* a3 + a4 */
+        lstm_step(cfg, v, x, a, g, c, h);
+        if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
+        if (c_seq) for (int i = 0; i < H; ++i) c_seq[tb * H + i] = (float)c[i];
+
+        /* a5: heads on op(h') */
+        for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h[i]);
+        mdn_head(cfg, v, y, mdn);
+        if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = (float)mdn[m];
+        double r = v->b_rew, dl = v->b_done;
+        for (int i = 0; i < H; ++i) { r += y[i] * v->w_rew[i]; dl += y[i] * v->w_done[i]; }
+        rewards[tb] = (float)r;
+        float dlf = (float)dl;
+        if (done_margin) done_margin[tb] = fabsf(dlf);
+        int is_noop = cfg->noop_terminates && a == A - 1;
+        int dn = (dlf > 0.0f) || is_noop;
+        done[tb] = (uint8_t)dn;
+
+        /* a6 + a7: per-dim mixture sample */
+        for (int d = 0; d < Z; ++d) {
+            double u = 0.0, eps = 0.0;
+            if (cfg->mdn_tau > 0.0) {
+                uint32_t ru[4], rn[4];
+                orc_draw(cfg->seed, e, s, 0u, (uint32_t)(d / 4), ru);
+                u = orc_uniform(ru[d % 4]);
+                orc_draw(cfg->seed, e, s, 1u, (uint32_t)(d / 4), rn);
+                double e0, e1;
+                int pair = (d % 4) / 2;
+                orc_box_muller(rn[2 * pair], rn[2 * pair + 1], &e0, &e1);
+                eps = (d % 2 == 0) ? e0 : e1;
+            }
+            for (int k = 0; k < K; ++k) lg[k] = (float)mdn[d * K + k];
+            double zd, mg;
+            int k = orc_sample_dim(K, cfg->mdn_tau, cfg->sigma_sqrt_tau, lg,
+                                   mdn + K * Z + d * K, mdn + 2 * K * Z + d * K, u, eps, &zd, &mg);
+            znew[d] = zd;
+            if (comp_seq) comp_seq[tb * Z + d] = (uint8_t)k;
+            if (comp_margin) comp_margin[tb * Z + d] = (float)mg;
+        }
+        for (int d = 0; d < Z; ++d) {
+            z[d] = (double)(float)znew[d];   /* fp32 latent state */
+            z_out[((size_t)(t + 1) * B + b) * Z + d] = (float)z[d];
+        }
+        /* a8 */
+        if ((cfg->done_terminates && dlf > 0.0f) || is_noop) frozen = 1;
+    }
+    if (h_final) for (int i = 0; i < H; ++i) h_final[(size_t)b * H + i] = (float)h[i];
+    if (c_final) for (int i = 0; i < H; ++i) c_final[(size_t)b * H + i] = (float)c[i];
+    free(z); free(h); free(c); free(x); free(g); free(y); free(mdn); free(znew); free(lg);
+    return 0;
+}
+
+int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
+                uint64_t episode_offset, uint32_t t0,
+                const float *z0, const float *h0, const float *c0,
+                const uint8_t *done0, const uint32_t *mask,
+                float *z_out, int32_t *actions, float *rewards, uint8_t *done,
+                float *h_final, float *c_final,
+                float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
+                float *ctrl_margin, float *comp_margin, float *done_margin)
+{
+    if (check_cfg(cfg) || B < 0 || T < 0 || !z0 || !z_out || !actions || !rewards || !done)
+        return -1;
+    wts64 v;
+    if (load_wts(cfg, w, &v, 1)) return -2;
+    int bad = 0;
+    int nt = cfg->nthreads > 0 ? cfg->nthreads : 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nt) reduction(| : bad)
+    for (int b = 0; b < B; ++b) {
+        bad |= rollout_episode(cfg, &v, b, B, T, episode_offset, t0, z0, h0, c0, done0, mask,
+                               z_out, actions, rewards, done, h_final, c_final,
+                               h_seq, c_seq, mdn_seq, comp_seq,
+                               ctrl_margin, comp_margin, done_margin) ? 1 : 0;
+    }
+    free_wts(&v);
+    return bad ? -2 : 0;
+}
+
+static int nll_sequence(const orc_cfg *cfg, const wts64 *v, int n, int N, int T,
+                        const float *z_seq, const int32_t *actions, int len,
+                        double *nll, float *h_seq, float *c_seq, float *mdn_seq)
+{
+    const int Z = cfg->z_dim, H = cfg->h_dim, K = cfg->k_mix, M = 3 * K * Z;
+    double *h = calloc((size_t)H, sizeof(double)), *c = calloc((size_t)H, sizeof(double));
+    double *x = malloc(sizeof(double) * (Z + H)), *g = malloc(sizeof(double) * 4 * H);
+    double *y = malloc(sizeof(double) * H), *mdn = malloc(sizeof(double) * M);
+    if (!h || !c || !x || !g || !y || !mdn) {
+        free(h); free(c); free(x); free(g); free(y); free(mdn);
+        return -1;
+    }
+    double total = 0.0;
+    for (int t = 0; t < T; ++t) {
+        const size_t tn = (size_t)t * N + n;
+        for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z_seq[tn * Z + i]);
+        for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
+        lstm_step(cfg, v, x, actions[tn], g, c, h);
+        for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h[i]);
+        mdn_head(cfg, v, y, mdn);
+        if (h_seq) for (int i = 0; i < H; ++i) h_seq[tn * H + i] = (float)h[i];
+        if (c_seq) for (int i = 0; i < H; ++i) c_seq[tn * H + i] = (float)c[i];
+        if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tn * M + m] = (float)mdn[m];
+        if (t < len) {
+            const float *target = z_seq + ((size_t)(t + 1) * N + n) * Z;
+            for (int d = 0; d < Z; ++d)
+                total += orc_mixture_nll_1d(K, mdn + d * K, mdn + K * Z + d * K,
+                                            mdn + 2 * K * Z + d * K, (double)target[d]);
+        }
+    }
+    nll[n] = total;
+    free(h); free(c); free(x); free(g); free(y); free(mdn);
+    return 0;
+}
+
+int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
+                const float *z_seq, const int32_t *actions, const int32_t *lengths,
+                double *nll, float *h_seq, float *c_seq, float *mdn_seq)
+{
+    if (check_cfg(cfg) || N < 0 || T < 0 || !z_seq || !actions || !nll) return -1;
+    for (size_t i = 0; i < (size_t)N * T; ++i)
+        if (actions[i] >= cfg->a_dim) return -1;
+    if (lengths)
+        for (int n = 0; n < N; ++n)
+            if (lengths[n] < 0 || lengths[n] > T) return -1;
+    wts64 v;
+    if (load_wts(cfg, w, &v, 0)) return -2;
+    int bad = 0;
+    int nt = cfg->nthreads > 0 ? cfg->nthreads : 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nt) reduction(| : bad)
+    for (int n = 0; n < N; ++n) {
+        int len = lengths ? lengths[n] : T;
+        bad |= nll_sequence(cfg, &v, n, N, T, z_seq, actions, len, nll, h_seq, c_seq, mdn_seq) ? 1 : 0;
+    }
+    free_wts(&v);
+    return bad ? -2 : 0;
+}

@@ -1,0 +1,91 @@
+/*
+ * wm_oracle.h -- plain, slow, obviously-correct CPU oracle for the RLFlow
+ * world-model "dream" path (MDN-RNN world model + linear controller).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and
+ * bench.py's cpu_baseline / reference arm may load or call this code.  The
+ * CUDA product path shares no code, header, table or helper with it.
+ *
+ * Arithmetic is fp64 throughout.  Where a floating-point value decides an
+ * integer (controller argmax, mixture-component choice, done threshold) the
+ * deciding value is first rounded to fp32, the precision the kernels decide
+ * in.  A "bf16" mode emulates the bf16 operand rounding points of the GPU
+ * bf16 path (weights, and the GEMM A-operands [z_t; h_t] and h_{t+1}).
+ *
+ * Paper anchors (RLFlow, SIGMOD'22): MDN-RNN models P(z_{t+1}|a_t,z_t,h_t)
+ * (Sec. 3.4.3); mixture weights = softmax(logits / tau) (Sec. 3.4.3, the
+ * temperature equation); linear controller a_t = W_c[z_t,h_t] + b_c
+ * (Sec. 3.5); invalid-action masking of the logits (Sec. 3.1.3); padding and
+ * masking of sequences (Sec. 3.4.2); world-model log-likelihood loss
+ * (Sec. 4.7).
+ */
+#ifndef WM_ORACLE_H
+#define WM_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct {
+    int z_dim, a_dim, h_dim, k_mix;
+    int bf16;             /* 1: emulate bf16 operand rounding              */
+    double mdn_tau;       /* mixture temperature, >= 0                       */
+    int sigma_sqrt_tau;   /* 1: sigma scaled by sqrt(tau)                    */
+    int ctrl_sample;      /* 0: masked argmax, 1: tempered softmax sample    */
+    double ctrl_tau;      /* controller temperature (sample mode), >= 0      */
+    int done_terminates;  /* done head (logit > 0) freezes the episode       */
+    int noop_terminates;  /* action a_dim-1 (NO-OP) freezes the episode      */
+    uint64_t seed;        /* Philox key                                      */
+    int nthreads;         /* OpenMP threads over episodes (<=0: 1)           */
+} orc_cfg;
+
+typedef struct {
+    const float *W_lstm;  /* [Z+A+H, 4H]  rows z | a | h, cols i | f | g | o  */
+    const float *b_lstm;  /* [4H]                                            */
+    const float *W_mdn;   /* [H, 3KZ]  cols logit | mu | logsigma, d*K+k      */
+    const float *b_mdn;   /* [3KZ]                                           */
+    const float *w_rew;   /* [H]                                             */
+    float b_rew;
+    const float *w_done;  /* [H]                                             */
+    float b_done;
+    const float *W_ctrl;  /* [Z+H, A]                                        */
+    const float *b_ctrl;  /* [A]                                             */
+} orc_weights;
+
+/* ---- building blocks (exported so tests can pin each one) ---------------- */
+void     orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
+double   orc_uniform(uint32_t x);
+void     orc_box_muller(uint32_t x1, uint32_t x2, double *e0, double *e1);
+void     orc_draw(uint64_t seed, uint64_t episode, uint32_t step, uint32_t purpose,
+                  uint32_t block, uint32_t out[4]);
+float    orc_bf16(float x);
+void     orc_lstm_cell(int H, const double *gates, const double *c_in,
+                       double *c_out, double *h_out);
+double   orc_mixture_nll_1d(int K, const double *logits, const double *mu,
+                            const double *logsig, double x);
+int      orc_sample_dim(int K, double tau, int sigma_sqrt_tau, const float *logits,
+                        const double *mu, const double *logsig, double u, double eps,
+                        double *z, double *margin);
+int      orc_select_action(int A, const float *logits, const uint32_t *mask_words,
+                           int ctrl_sample, double ctrl_tau, double u, double *margin);
+
+/* ---- the two operations of the path --------------------------------------- */
+int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
+                uint64_t episode_offset, uint32_t t0,
+                const float *z0, const float *h0, const float *c0,
+                const uint8_t *done0, const uint32_t *mask,
+                float *z_out, int32_t *actions, float *rewards, uint8_t *done,
+                float *h_final, float *c_final,
+                float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
+                float *ctrl_margin, float *comp_margin, float *done_margin);
+
+int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
+                const float *z_seq, const int32_t *actions, const int32_t *lengths,
+                double *nll, float *h_seq, float *c_seq, float *mdn_seq);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
