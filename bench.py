@@ -1,0 +1,352 @@
+#!/usr/bin/env python3
+"""Dream-rollout throughput on GB300: env-steps/s of wm_rollout, with its roofline.
+
+One "step" is one wm_rollout call over the whole workload: T dream steps of B
+independent episodes (controller, mask + action choice, LSTM, mixture head,
+sampling, reward / done).  Default workload: the small-batch latency regime,
+B=1024 episodes x T=50 steps, Z=32, A=128 (30% valid mask), H=256, K=5, bf16
+operands / fp32 state (``synth.WORKLOADS['small_bf16']``).
+
+Timing: W untimed warm-ups, then K steps each bracketed by CUDA events on the
+launching stream, with a 512 MiB write between steps to flush the 129 MB L2.
+N GPUs (torchrun): every rank runs its own B episodes (episode_offset =
+rank * B), no data-path collective, max time over ranks -> weak scaling.
+
+``--impl reference`` times the CPU oracle (the plain C definition of the same
+steps) on the host cores instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+           "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+           "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def flops_per_env_step(cfg: dict) -> float:
+    """Algorithmic FLOPs of one (episode, step): the three contractions plus heads.
+
+    controller [Z+H] x [Z+H, A], gates [Z+H] x [Z+H, 4H] (the one-hot action
+    row is a gather, not FLOPs), mixture head [H] x [H, 3KZ], reward and done.
+    """
+    Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
+    return 2.0 * ((Z + H) * A + (Z + H) * 4 * H + H * 3 * K * Z + 2 * H)
+
+
+def bytes_per_env_step(cfg: dict) -> float:
+    """Algorithmic HBM bytes of one (episode, step) with the state kept on chip:
+    the mask words read, z_{t+1}, action, reward and done written."""
+    Z, A = cfg["z_dim"], cfg["a_dim"]
+    return 4.0 * ((A + 31) // 32) + 4.0 * Z + 4 + 4 + 1
+
+
+def weight_bytes(cfg: dict) -> float:
+    Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
+    el = 2 if cfg["precision"] == "bf16" else 4
+    return el * ((Z + A + H) * 4 * H + H * (3 * K * Z + 2) + (Z + H) * A)
+
+
+def load_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def fp32_simt_peak_tflops() -> float:
+    # 152 SMs x 128 fp32 FMA lanes x 2 FLOP x 2.07 GHz (maximum SM clock)
+    return 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def kernel_source_sha(path_name: str) -> str:
+    src = {"fused": "wm_fused.cu", "stepwise": "wm_step.cu"}.get(path_name, "wm_step.cu")
+    with open(os.path.join(ROOT, "paper_2205_01435_gb300", "csrc", src), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel_key: str, sha: str):
+    """DRAM bytes per launch from a committed ncu capture of this exact kernel source."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel_key)
+    if not e or e.get("source_sha") != sha:
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            self.path = f"/tmp/wm_clocks_{os.getpid()}.csv"
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={CLOCK_Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self) -> dict:
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_ours(args) -> None:
+    import torch
+    import torch.distributed as dist
+
+    import paper_2205_01435_gb300 as pkg
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    wm = pkg.load()
+    name = args.workload
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
+    if args.path:
+        cfg["path"] = args.path
+    model = wm.WorldModel(cfg, w, device=local)
+    dev = torch.device("cuda", local)
+    zc = torch.from_numpy(z0).to(dev)
+    mc = torch.from_numpy(mask).to(dev)
+    ep0 = rank * B
+    out = {"z": torch.empty((T + 1, B, cfg["z_dim"]), device=dev),
+           "actions": torch.empty((T, B), dtype=torch.int32, device=dev),
+           "rewards": torch.empty((T, B), device=dev),
+           "done": torch.empty((T, B), dtype=torch.uint8, device=dev)}
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    def step():
+        return model.rollout(zc, T, mask=mc, episode_offset=ep0, want_final=False, out=out,
+                             stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    path_name = model.last_path
+    launches = model.last_launches
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    times = [a.elapsed_time(b) for a, b in ev]  # ms, each one launch of the step
+    total_ms = sum(times)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if ws > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    env_steps = B * T * ws
+    value = env_steps / (ms_per_step / 1e3)
+
+    # e2e: the same call through the C ABI with pinned HOST buffers, copies timed.
+    zh = torch.from_numpy(z0).pin_memory()
+    mh = torch.from_numpy(mask).pin_memory()
+    hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
+            "actions": torch.empty((T, B), dtype=torch.int32, pin_memory=True),
+            "rewards": torch.empty((T, B), pin_memory=True),
+            "done": torch.empty((T, B), dtype=torch.uint8, pin_memory=True)}
+    for _ in range(2):
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+    torch.cuda.synchronize()
+    e2e_t = []
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_s = torch.tensor([sum(e2e_t) / len(e2e_t)], dtype=torch.float64, device=dev)
+    if ws > 1:
+        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
+    e2e_value = env_steps / float(e2e_s.item())
+    h2d = zh.numel() * 4 + mh.numel() * 4
+    d2h = sum(v.numel() * v.element_size() for v in hout.values())
+
+    peaks = load_peaks()
+    fl = flops_per_env_step(cfg) * B * T
+    if path_name == "fused":
+        kernel_key = f"wm_fused_rollout/{name}"
+        bound, peak, unit = "tensor", peaks["bf16_tflops"], "TFLOP/s"
+        achieved = fl / (ms_per_step / 1e3) / 1e12
+    else:
+        kernel_key = f"wm_step/{name}"
+        bound, peak, unit = "alu", fp32_simt_peak_tflops(), "TFLOP/s"
+        achieved = fl / (ms_per_step / 1e3) / 1e12
+    sha = kernel_source_sha(path_name)
+    traffic = ncu_traffic(kernel_key, sha)
+    roof = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
+            "frac": round(achieved / peak, 5), "traffic": traffic,
+            "peak_source": peaks["source"] if bound == "tensor" else "derived: 152 SM x 128 FMA x 2.07 GHz",
+            "kernel": kernel_key, "algorithmic_flops_per_launch": fl,
+            "algorithmic_hbm_bytes_per_launch": bytes_per_env_step(cfg) * B * T + weight_bytes(cfg)}
+
+    line = {"metric": "dream env-steps/s (wm_rollout)", "value": round(value, 1),
+            "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if cfg["precision"] == "bf16" else "f32",
+            "data": "synthetic (seeded: weights N(0,0.05^2), z0 N(0,1), Bernoulli masks)",
+            "config": {"workload": name, "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
+                       "H": cfg["h_dim"], "K": cfg["k_mix"],
+                       "mask_density": synth.WORKLOADS[name]["mask_density"],
+                       "precision": cfg["precision"], "kernel_path": path_name,
+                       "l2": "flushed between timed steps (512 MiB write)",
+                       "parallelism": f"episodes sharded over {ws} GPU(s), no collective"},
+            "e2e": {"value": round(e2e_value, 1), "unit": "env-steps/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches * args.steps,
+            "roofline": roof, "clocks": clk.summary()}
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def cpu_baseline(name: str, episodes: int, threads: int | None = None) -> dict:
+    import oracle
+
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
+    n = min(episodes, B)
+    threads = threads or os.cpu_count() or 1
+    t0 = time.perf_counter()
+    oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+    dt = time.perf_counter() - t0
+    return {"value": round(n * T / dt, 2), "unit": "env-steps/s", "cores": threads,
+            "kind": "oracle", "sample": f"{n} of {B} episodes x {T} steps of {name}, "
+                                        f"{threads} threads, {dt:.1f} s"}
+
+
+def run_reference(args) -> None:
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+
+    name = args.workload
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
+    n = min(args.ref_episodes, B)
+    threads = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+        times.append(time.perf_counter() - t0)
+    per = sum(times) / len(times)
+    value = n * T / per
+    sample = f"{n} of {B} episodes x {T} steps of {name} per step, {threads} threads"
+    line = {"impl": "reference", "metric": "dream env-steps/s (wm_rollout)",
+            "value": round(value, 2), "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(per * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64 (bf16 operand emulation)" if cfg["precision"] == "bf16" else "f64",
+            "data": "synthetic (seeded: weights N(0,0.05^2), z0 N(0,1), Bernoulli masks)",
+            "config": {"workload": name, "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
+                       "H": cfg["h_dim"], "K": cfg["k_mix"], "precision": cfg["precision"]},
+            "cpu_baseline": {"value": round(value, 2), "unit": "env-steps/s", "cores": threads,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 2), "unit": "env-steps/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="small_bf16",
+                    choices=[k for k in synth.WORKLOADS if k != "nll"])
+    ap.add_argument("--path", choices=["auto", "stepwise", "fused"], default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-episodes", type=int, default=1024)
+    ap.add_argument("--ref-episodes", type=int, default=96)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,182 @@
+/*
+ * wm.h -- C ABI of the GB300 world-model "dream" engine.
+ *
+ * The engine runs batched rollouts inside the world model of RLFlow
+ * (Mitchell et al., "RLFlow: Optimising Neural Network Subgraph
+ * Transformation with World Models", SIGMOD'22) and scores teacher-forced
+ * sequences under its mixture-density head.  The world model is an MDN-RNN
+ * (Sec. 3.3.1 "Recurrent Neural Networks", Sec. 3.3.2 "MDN-RNN") driven by the
+ * linear controller a_t = W_c [z_t, h_t] + b_c (Sec. 3.4 "Action Controller");
+ * one wm_rollout step is the imagined-environment analogue of the Gym
+ * step(action) -> (next_state, reward, terminal, info) of Sec. 3.1.1.
+ *
+ * Notation: B episodes, T steps, Z latent size, A actions, H LSTM hidden size,
+ * K mixture components, M = 3*K*Z mixture-head outputs, W = ceil(A/32).
+ *
+ * Per episode and step t (all episodes independent):
+ *   a1  l   = W_c^T [z_t; h_t] + b_c                               (Sec. 3.4)
+ *   a2  l_j = -inf where action j is invalid (Sec. 3.1.3); a_t = lowest-index
+ *       argmax, or a draw from softmax(l / ctrl_tau); -1 if nothing is valid
+ *   a3  G   = W_lstm^T [z_t; onehot(a_t); h_t] + b_lstm, columns i|f|g|o
+ *   a4  c'  = sig(f) c + sig(i) tanh(g);  h' = sig(o) tanh(c')       (Sec. 3.3.2)
+ *   a5  [logit | mu | log sigma] = W_mdn^T h' + b_mdn;  r = w_rew.h' + b_rew;
+ *       d = w_done.h' + b_done
+ *   a6  pi_d = softmax(logit_d / mdn_tau) per latent dim d   (temperature eq., Sec. 3.3.2)
+ *   a7  k ~ pi_d (inverse CDF on a Philox uniform), z'_d = mu_dk + sigma_dk eps_d
+ *   a8  done = d > 0 (or NO-OP when noop_terminates); with done_terminates a
+ *       done episode is frozen: later steps give a = -1, r = 0, done = 1 and
+ *       repeat z, h, c.
+ *   a9  (wm_mdn_nll) NLL_n = sum_{t<len_n} sum_d -log sum_k pi N(z_{t+1,d}; mu, sigma)
+ *       with tau = 1 -- the world-model log-likelihood loss of Sec. 4.7.
+ *
+ * Random numbers: Philox-4x32-10 (Salmon et al., SC'11) with key = seed and
+ * counter = (episode lo32, t0 + t, purpose << 24 | block, episode hi32), where
+ * episode = episode_offset + b.  Purpose 0: component uniforms (4 dims per
+ * block); 1: Box-Muller normals (4 dims per block); 2: controller uniform.
+ * A uniform is (x >> 8) * 2^-24.  Results therefore do not depend on how the
+ * episodes are split across calls or devices.
+ *
+ * Precision: WM_FP32 computes in fp32.  WM_BF16 rounds every weight matrix to
+ * bf16 (RNE) at wm_create and rounds the GEMM operands [z_t; h_t] and h' to
+ * bf16; biases, accumulation, nonlinearities, state and sampling stay fp32.
+ *
+ * Memory: every array argument below may be device memory (cudaMalloc'd,
+ * managed) or host memory (pinned or pageable); the library tells them apart
+ * with cudaPointerGetAttributes.  Host arrays are staged through device
+ * buffers owned by the handle, on the call's stream; if any output is host
+ * memory the call synchronises the stream before it returns.  All arrays are
+ * dense, row-major, in the layouts given, and owned by the caller.
+ *
+ * Errors: argument errors are returned synchronously and leave outputs
+ * untouched.  Device-side errors (a bounded wait that gave up) are recorded in
+ * a device status word and returned by wm_sync.  wm_last_error gives a
+ * message for the last failing call on a handle.
+ *
+ * Threading: a handle is not thread-safe; use one handle per host thread.
+ * Calls on one handle must not overlap on the GPU (they share workspace):
+ * issue them on one stream, or synchronise between streams.
+ */
+#ifndef WM_H
+#define WM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    WM_OK = 0,
+    WM_ERR_INVALID_ARG = 1,
+    WM_ERR_CUDA = 2,
+    WM_ERR_UNSUPPORTED = 3,
+    WM_ERR_TIMEOUT = 4,
+    WM_ERR_OOM = 5
+} wm_status;
+
+enum { WM_FP32 = 0, WM_BF16 = 1 };
+
+/* Kernel family.  AUTO picks by batch size and model size; the others force
+ * one (WM_ERR_UNSUPPORTED if it cannot run the model). */
+enum { WM_PATH_AUTO = 0, WM_PATH_STEPWISE = 1, WM_PATH_FUSED = 2, WM_PATH_TENSOR = 3 };
+
+typedef struct {
+    int z_dim, a_dim, h_dim, k_mix;   /* Z, A, H, K (K <= 32)                      */
+    int precision;                    /* WM_FP32 or WM_BF16                        */
+    float mdn_tau;                    /* >= 0; 0 = argmax component, z = mu        */
+    int sigma_sqrt_tau;               /* 1: sigma scaled by sqrt(mdn_tau)          */
+    int ctrl_sample;                  /* 0: masked argmax; 1: tempered draw        */
+    float ctrl_tau;                   /* >= 0; 0 behaves as argmax                 */
+    int done_terminates;              /* done head freezes the episode             */
+    int noop_terminates;              /* action A-1 (NO-OP, Sec. 3.1.3) freezes it */
+    unsigned long long seed;          /* Philox key                                */
+    int path;                         /* WM_PATH_*                                 */
+} wm_config;
+
+/* Canonical fp32 weights, row-major, HOST memory; copied (and packed) by
+ * wm_create, so the caller may free them afterwards. */
+typedef struct {
+    const float *W_lstm;  /* [Z+A+H, 4H]: rows z | a | h; cols i | f | g | o      */
+    const float *b_lstm;  /* [4H]                                                 */
+    const float *W_mdn;   /* [H, 3KZ]: cols logit | mu | log sigma, index d*K + k  */
+    const float *b_mdn;   /* [3KZ]                                                */
+    const float *w_rew;   /* [H]                                                  */
+    float b_rew;
+    const float *w_done;  /* [H]                                                  */
+    float b_done;
+    const float *W_ctrl;  /* [Z+H, A]: rows z | h                                 */
+    const float *b_ctrl;  /* [A]                                                  */
+} wm_weights;
+
+typedef struct wm_handle wm_handle;
+
+/* Inputs and outputs of one wm_rollout call (see the memory rules above). */
+typedef struct {
+    const float *z0;             /* [B,Z]   required: z_{t0} of every episode        */
+    const float *h0;             /* [B,H]   or NULL = zeros                          */
+    const float *c0;             /* [B,H]   or NULL = zeros                          */
+    const uint8_t *done0;        /* [B]     or NULL; nonzero = episode already frozen */
+    const uint32_t *mask;        /* [T,B,W] or NULL = all valid; bit j of word w
+                                    set = action 32w+j valid at that step            */
+    float *z_out;                /* [T+1,B,Z] required; z_out[0] = z0                */
+    int32_t *actions;            /* [T,B]   required; -1 = no action                 */
+    float *rewards;              /* [T,B]   required                                 */
+    uint8_t *done;               /* [T,B]   required                                 */
+    float *h_final;              /* [B,H]   optional                                 */
+    float *c_final;              /* [B,H]   optional                                 */
+    float *h_seq;                /* [T,B,H] optional: h after each step              */
+    float *c_seq;                /* [T,B,H] optional                                 */
+    float *mdn_seq;              /* [T,B,M] optional: raw head outputs (0 if frozen) */
+    uint8_t *comp_seq;           /* [T,B,Z] optional: chosen component (255 if frozen)*/
+} wm_rollout_io;
+
+/* Copies and packs the weights onto the current CUDA device.  The handle owns
+ * that device memory until wm_destroy.  Returns WM_ERR_INVALID_ARG for bad
+ * sizes (any dim <= 0, K > 32, negative temperatures) or NULL weights. */
+wm_status wm_create(const wm_config *cfg, const wm_weights *weights, wm_handle **out);
+
+/* Runs T dream steps (a1..a8 above) for B independent episodes, asynchronously
+ * on cuda_stream (a cudaStream_t; NULL = legacy default stream).  Episode b is
+ * keyed to Philox as episode_offset + b and its steps as t0 + t, so a rollout
+ * split over calls (resume: pass z_out[T], h_final, c_final, done[T-1]) or over
+ * devices (shard: episode_offset) reproduces the unsplit one bit for bit.
+ * B = 0 or T = 0 are valid (T = 0 only copies z0 to z_out[0]). */
+wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offset,
+                     unsigned int t0, const wm_rollout_io *io, void *cuda_stream);
+
+/* Teacher-forced scoring (a9): runs the LSTM over the given latents and
+ * actions from h = c = 0 and returns the per-sequence mixture NLL in nats.
+ *   z_seq   [T+1,N,Z] latents; step t reads z_seq[t] and scores z_seq[t+1]
+ *   actions [T,N]     in [0,A) or negative for no action row
+ *   lengths [N]       in [0,T], or NULL = T: only steps t < lengths[n] count
+ *                     (Sec. 3.3.1 padding); the recurrence still runs all T
+ *   nll     [N]       output
+ *   h_seq, c_seq [T,N,H], mdn_seq [T,N,M]: optional per-step outputs.
+ * An action >= A or a length outside [0,T] is an argument error, detected on
+ * the host only when the array is host memory; on device memory the kernels
+ * treat an out-of-range action as no action and clamp lengths. */
+wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                     const int32_t *lengths, float *nll, float *h_seq, float *c_seq,
+                     float *mdn_seq, void *cuda_stream);
+
+/* Synchronises the device and returns the first device-side error since the
+ * last wm_sync (WM_ERR_TIMEOUT if a bounded wait gave up), then clears it. */
+wm_status wm_sync(wm_handle *h);
+
+/* Message for the last failing call on h (never NULL; "" if none). */
+const char *wm_last_error(const wm_handle *h);
+
+/* Kernel family the last wm_rollout / wm_mdn_nll call ran (WM_PATH_*). */
+int wm_last_path(const wm_handle *h);
+
+/* Number of kernels the last wm_rollout / wm_mdn_nll call launched (staging
+ * copies not counted). */
+int wm_last_launches(const wm_handle *h);
+
+/* Frees everything the handle owns.  NULL is a no-op. */
+void wm_destroy(wm_handle *h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* WM_H */

@@ -6,9 +6,9 @@ package.  It shares no code with the CUDA product path
 (``paper_2205_01435_gb300``) and never imports it.
 
 Every function follows the paper's statement of the world model (RLFlow,
-SIGMOD'22): the MDN-RNN that models P(z_{t+1} | a_t, z_t, h_t) (Sec. 3.4.3),
-the temperature softmax of the mixture weights (Sec. 3.4.3), the linear
-controller a_t = W_c [z_t, h_t] + b_c (Sec. 3.5), invalid-action masking
+SIGMOD'22): the MDN-RNN that models P(z_{t+1} | a_t, z_t, h_t) (Sec. 3.3.2),
+the temperature softmax of the mixture weights (Sec. 3.3.2), the linear
+controller a_t = W_c [z_t, h_t] + b_c (Sec. 3.4), invalid-action masking
 (Sec. 3.1.3) and the world-model log-likelihood loss (Sec. 4.7).  The
 arithmetic lives in ``wm_oracle.c``; this module only marshals arguments.
 """

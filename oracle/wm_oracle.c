@@ -5,12 +5,12 @@
  * blocking, fusion or reordering beyond the step order below:
  *
  *   for t = 0..T-1, for every episode independently:
- *     a1  controller logits   l = W_c^T [z_t; h_t] + b_c           (Sec. 3.5)
+ *     a1  controller logits   l = W_c^T [z_t; h_t] + b_c           (Sec. 3.4)
  *     a2  mask + select       invalid logits -> -inf; argmax or a
  *                             tempered-softmax draw                 (Sec. 3.1.3)
- *     a3  LSTM gates          G = W^T [z_t; onehot(a_t); h_t] + b   (Sec. 3.4.3)
+ *     a3  LSTM gates          G = W^T [z_t; onehot(a_t); h_t] + b   (Sec. 3.3.2)
  *     a4  cell update         c' = f c + i g, h' = o tanh(c')
- *     a5  heads               MDN params, reward, done logit on h'  (Sec. 3.4.3, 4.7)
+ *     a5  heads               MDN params, reward, done logit on h'  (Sec. 3.3.2, 4.7)
  *     a6  mixture weights     log softmax(logit / tau)              (temperature eq.)
  *     a7  sample z_{t+1}      component by inverse CDF, then mu + sigma*eps
  *     a8  done / freeze       done = logit > 0; frozen episodes stay put

@@ -13,10 +13,10 @@
  * bf16 path (weights, and the GEMM A-operands [z_t; h_t] and h_{t+1}).
  *
  * Paper anchors (RLFlow, SIGMOD'22): MDN-RNN models P(z_{t+1}|a_t,z_t,h_t)
- * (Sec. 3.4.3); mixture weights = softmax(logits / tau) (Sec. 3.4.3, the
+ * (Sec. 3.3.2); mixture weights = softmax(logits / tau) (Sec. 3.3.2, the
  * temperature equation); linear controller a_t = W_c[z_t,h_t] + b_c
- * (Sec. 3.5); invalid-action masking of the logits (Sec. 3.1.3); padding and
- * masking of sequences (Sec. 3.4.2); world-model log-likelihood loss
+ * (Sec. 3.4); invalid-action masking of the logits (Sec. 3.1.3); padding and
+ * masking of sequences (Sec. 3.3.1); world-model log-likelihood loss
  * (Sec. 4.7).
  */
 #ifndef WM_ORACLE_H

@@ -1,0 +1,333 @@
+// wm_api.cu -- the C ABI of include/wm.h: argument checks, weight packing,
+// host<->device staging of caller arrays, and dispatch to a kernel family.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+#include <string>
+#include <vector>
+
+#include "wm_internal.h"
+
+// ---- kernel families implemented in other translation units ---------------
+int wm_fused_supported(const wm_handle *h, int B);
+cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w);
+void wm_fused_free(wm_handle *h);
+cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaStream_t s);
+cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s);
+size_t wm_fused_nll_ws(const wm_handle *h, int N);
+
+namespace {
+
+wm_status fail(wm_handle *h, wm_status st, const std::string &msg) {
+    if (h) h->err = msg;
+    return st;
+}
+
+wm_status cuda_fail(wm_handle *h, cudaError_t e, const char *where) {
+    std::string m = std::string(where) + ": " + cudaGetErrorString(e);
+    return fail(h, e == cudaErrorMemoryAllocation ? WM_ERR_OOM : WM_ERR_CUDA, m);
+}
+
+bool is_host_ptr(const void *p) {
+    cudaPointerAttributes at;
+    cudaError_t e = cudaPointerGetAttributes(&at, p);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return true;
+    }
+    return at.type == cudaMemoryTypeHost || at.type == cudaMemoryTypeUnregistered;
+}
+
+float bf16_round_host(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+cudaError_t grow(void **buf, size_t *have, size_t need) {
+    if (need <= *have) return cudaSuccess;
+    if (*buf) {
+        cudaError_t e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return e;
+        cudaFree(*buf);
+        *buf = nullptr;
+        *have = 0;
+    }
+    size_t n = need + need / 8;
+    cudaError_t e = cudaMalloc(buf, n);
+    if (e != cudaSuccess) return e;
+    *have = n;
+    return cudaSuccess;
+}
+
+template <class T>
+cudaError_t upload(T **dst, const std::vector<T> &src) {
+    cudaError_t e = cudaMalloc((void **)dst, src.size() * sizeof(T));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpy(*dst, src.data(), src.size() * sizeof(T), cudaMemcpyHostToDevice);
+}
+
+// One caller array that may need staging.
+struct Stage {
+    void **dev;        // where the device pointer goes
+    const void *user;  // caller pointer
+    size_t bytes;
+    bool out;
+    size_t off;
+};
+
+struct Stager {
+    std::vector<Stage> items;
+    size_t total = 0;
+    bool any_host_out = false;
+    void add(void **dev, const void *user, size_t bytes, bool out) {
+        *dev = const_cast<void *>(user);
+        if (!user || bytes == 0 || !is_host_ptr(user)) return;
+        items.push_back({dev, user, bytes, out, total});
+        total += (bytes + 255) & ~(size_t)255;
+        if (out) any_host_out = true;
+    }
+    cudaError_t begin(wm_handle *h, cudaStream_t s) {
+        if (items.empty()) return cudaSuccess;
+        cudaError_t e = grow(&h->stage, &h->stage_bytes, total);
+        if (e != cudaSuccess) return e;
+        for (auto &it : items) {
+            *it.dev = (char *)h->stage + it.off;
+            if (!it.out) {
+                e = cudaMemcpyAsync(*it.dev, it.user, it.bytes, cudaMemcpyHostToDevice, s);
+                if (e != cudaSuccess) return e;
+            }
+        }
+        return cudaSuccess;
+    }
+    cudaError_t end(cudaStream_t s) {
+        for (auto &it : items) {
+            if (!it.out) continue;
+            cudaError_t e = cudaMemcpyAsync(const_cast<void *>(it.user), *it.dev, it.bytes,
+                                            cudaMemcpyDeviceToHost, s);
+            if (e != cudaSuccess) return e;
+        }
+        if (any_host_out) return cudaStreamSynchronize(s);
+        return cudaSuccess;
+    }
+};
+
+bool valid_cfg(const wm_config *c) {
+    return c && c->z_dim > 0 && c->a_dim > 0 && c->h_dim > 0 && c->k_mix > 0 && c->k_mix <= 32 &&
+           (c->precision == WM_FP32 || c->precision == WM_BF16) && c->mdn_tau >= 0.f &&
+           c->ctrl_tau >= 0.f && c->path >= WM_PATH_AUTO && c->path <= WM_PATH_TENSOR &&
+           c->z_dim <= 4096 && c->a_dim <= 65536 && c->h_dim <= 16384;
+}
+
+cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
+    const wm_config &c = h->cfg;
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, N1 = 4 * H + A;
+    const bool rb = c.precision == WM_BF16;
+    auto wv = [&](float x) { return rb ? bf16_round_host(x) : x; };
+    std::vector<float> Wg((Z + H) * N1), Wa(A * 4 * H), bg(N1), Wh(H * (M + 2)), bh(M + 2);
+    for (size_t r = 0; r < Z + H; ++r) {
+        const size_t src = r < Z ? r : r + A;  // skip the action rows
+        for (size_t n = 0; n < 4 * H; ++n) Wg[r * N1 + n] = wv(w->W_lstm[src * 4 * H + n]);
+        for (size_t j = 0; j < A; ++j) Wg[r * N1 + 4 * H + j] = wv(w->W_ctrl[r * A + j]);
+    }
+    for (size_t a = 0; a < A; ++a)
+        for (size_t n = 0; n < 4 * H; ++n) Wa[a * 4 * H + n] = wv(w->W_lstm[(Z + a) * 4 * H + n]);
+    for (size_t n = 0; n < 4 * H; ++n) bg[n] = w->b_lstm[n];
+    for (size_t j = 0; j < A; ++j) bg[4 * H + j] = w->b_ctrl[j];
+    for (size_t i = 0; i < H; ++i) {
+        for (size_t m = 0; m < M; ++m) Wh[i * (M + 2) + m] = wv(w->W_mdn[i * M + m]);
+        Wh[i * (M + 2) + M] = wv(w->w_rew[i]);
+        Wh[i * (M + 2) + M + 1] = wv(w->w_done[i]);
+    }
+    for (size_t m = 0; m < M; ++m) bh[m] = w->b_mdn[m];
+    bh[M] = w->b_rew;
+    bh[M + 1] = w->b_done;
+    cudaError_t e;
+    if ((e = upload(&h->step.Wg, Wg)) != cudaSuccess) return e;
+    if ((e = upload(&h->step.Wa, Wa)) != cudaSuccess) return e;
+    if ((e = upload(&h->step.bg, bg)) != cudaSuccess) return e;
+    if ((e = upload(&h->step.Wh, Wh)) != cudaSuccess) return e;
+    return upload(&h->step.bh, bh);
+}
+
+}  // namespace
+
+extern "C" {
+
+wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) {
+    if (!out) return WM_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!valid_cfg(cfg)) return WM_ERR_INVALID_ARG;
+    if (!w || !w->W_lstm || !w->b_lstm || !w->W_mdn || !w->b_mdn || !w->w_rew || !w->w_done ||
+        !w->W_ctrl || !w->b_ctrl)
+        return WM_ERR_INVALID_ARG;
+    wm_handle *h = new (std::nothrow) wm_handle();
+    if (!h) return WM_ERR_OOM;
+    h->cfg = *cfg;
+    h->M = 3 * cfg->k_mix * cfg->z_dim;
+    memset(&h->step, 0, sizeof(h->step));
+    memset(&h->fused, 0, sizeof(h->fused));
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e == cudaSuccess) e = pack_step(h, w);
+    if (e == cudaSuccess) e = wm_fused_pack(h, w);
+    if (e == cudaSuccess) e = cudaMalloc((void **)&h->status, sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(h->status, 0, sizeof(int));
+    if (e != cudaSuccess) {
+        wm_status st = e == cudaErrorMemoryAllocation ? WM_ERR_OOM : WM_ERR_CUDA;
+        cudaGetLastError();
+        wm_destroy(h);
+        return st;
+    }
+    *out = h;
+    return WM_OK;
+}
+
+void wm_destroy(wm_handle *h) {
+    if (!h) return;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    cudaSetDevice(h->device);
+    cudaDeviceSynchronize();
+    cudaFree(h->step.Wg);
+    cudaFree(h->step.Wa);
+    cudaFree(h->step.bg);
+    cudaFree(h->step.Wh);
+    cudaFree(h->step.bh);
+    wm_fused_free(h);
+    cudaFree(h->ws);
+    cudaFree(h->stage);
+    cudaFree(h->status);
+    if (prev >= 0) cudaSetDevice(prev);
+    delete h;
+}
+
+const char *wm_last_error(const wm_handle *h) { return h ? h->err.c_str() : "null handle"; }
+
+int wm_last_path(const wm_handle *h) { return h ? h->last_path : 0; }
+
+int wm_last_launches(const wm_handle *h) { return h ? h->last_launches : 0; }
+
+wm_status wm_sync(wm_handle *h) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(h, e, "wm_sync");
+    int st = 0;
+    e = cudaMemcpy(&st, h->status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(h, e, "wm_sync status");
+    if (st != 0) {
+        cudaMemset(h->status, 0, sizeof(int));
+        return fail(h, (wm_status)st, "device-side error reported by a kernel");
+    }
+    return WM_OK;
+}
+
+wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offset, unsigned int t0,
+                     const wm_rollout_io *io, void *cuda_stream) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->err.clear();
+    if (!io) return fail(h, WM_ERR_INVALID_ARG, "io is NULL");
+    if (B < 0 || T < 0 || B > (1 << 22)) return fail(h, WM_ERR_INVALID_ARG, "B must be in [0, 2^22], T >= 0");
+    if (B > 0 && (!io->z0 || !io->z_out || (T > 0 && (!io->actions || !io->rewards || !io->done))))
+        return fail(h, WM_ERR_INVALID_ARG, "z0, z_out, actions, rewards and done are required");
+    if ((unsigned long long)t0 + (unsigned long long)T > 0x100000000ull)
+        return fail(h, WM_ERR_INVALID_ARG, "t0 + T overflows the 32-bit Philox step counter");
+    const wm_config &c = h->cfg;
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, W = (A + 31) / 32;
+    const size_t b = (size_t)B, t = (size_t)T;
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    cudaError_t e = cudaSetDevice(h->device);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+
+    wm_rollout_dev a{};
+    a.B = B; a.T = T; a.ep0 = episode_offset; a.t0 = t0;
+    Stager st;
+    st.add((void **)&a.z0, io->z0, b * Z * 4, false);
+    st.add((void **)&a.h0, io->h0, b * H * 4, false);
+    st.add((void **)&a.c0, io->c0, b * H * 4, false);
+    st.add((void **)&a.done0, io->done0, b, false);
+    st.add((void **)&a.mask, io->mask, t * b * W * 4, false);
+    st.add((void **)&a.z_out, io->z_out, (t + 1) * b * Z * 4, true);
+    st.add((void **)&a.actions, io->actions, t * b * 4, true);
+    st.add((void **)&a.rewards, io->rewards, t * b * 4, true);
+    st.add((void **)&a.done, io->done, t * b, true);
+    st.add((void **)&a.h_final, io->h_final, b * H * 4, true);
+    st.add((void **)&a.c_final, io->c_final, b * H * 4, true);
+    st.add((void **)&a.h_seq, io->h_seq, t * b * H * 4, true);
+    st.add((void **)&a.c_seq, io->c_seq, t * b * H * 4, true);
+    st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true);
+    st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true);
+
+    int path = c.path;
+    if (path == WM_PATH_AUTO) path = wm_fused_supported(h, B) ? WM_PATH_FUSED : WM_PATH_STEPWISE;
+    if (path == WM_PATH_FUSED && !wm_fused_supported(h, B))
+        return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
+    if (path == WM_PATH_TENSOR) return fail(h, WM_ERR_UNSUPPORTED, "the tensor family is not built for rollouts");
+
+    if (path == WM_PATH_STEPWISE) {
+        e = grow(&h->ws, &h->ws_bytes, wm_step_rollout_ws(h, B));
+        if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
+    }
+    if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    if (path == WM_PATH_FUSED)
+        e = wm_fused_rollout(h, a, s);
+    else
+        e = wm_step_rollout(h, a, h->ws, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "rollout launch");
+    h->last_path = path;
+    if (path == WM_PATH_STEPWISE)
+        h->last_launches = B == 0 ? 0 : 1 + 4 * T + ((a.h_final || a.c_final) ? 1 : 0);
+    if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
+    return WM_OK;
+}
+
+wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                     const int32_t *lengths, float *nll, float *h_seq, float *c_seq, float *mdn_seq,
+                     void *cuda_stream) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->err.clear();
+    if (N < 0 || T < 0 || N > (1 << 22)) return fail(h, WM_ERR_INVALID_ARG, "N must be in [0, 2^22], T >= 0");
+    if (N > 0 && (!z_seq || !nll || (T > 0 && !actions)))
+        return fail(h, WM_ERR_INVALID_ARG, "z_seq, actions and nll are required");
+    const wm_config &c = h->cfg;
+    const size_t Z = c.z_dim, H = c.h_dim, M = h->M, n = (size_t)N, t = (size_t)T;
+    if (actions && is_host_ptr(actions))
+        for (size_t i = 0; i < n * t; ++i)
+            if (actions[i] >= c.a_dim) return fail(h, WM_ERR_INVALID_ARG, "action index >= A");
+    if (lengths && is_host_ptr(lengths))
+        for (size_t i = 0; i < n; ++i)
+            if (lengths[i] < 0 || lengths[i] > T) return fail(h, WM_ERR_INVALID_ARG, "length outside [0, T]");
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    cudaError_t e = cudaSetDevice(h->device);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+
+    wm_nll_dev a{};
+    a.N = N; a.T = T;
+    Stager st;
+    st.add((void **)&a.z_seq, z_seq, (t + 1) * n * Z * 4, false);
+    st.add((void **)&a.actions, actions, t * n * 4, false);
+    st.add((void **)&a.lengths, lengths, n * 4, false);
+    st.add((void **)&a.nll, nll, n * 4, true);
+    st.add((void **)&a.h_seq, h_seq, t * n * H * 4, true);
+    st.add((void **)&a.c_seq, c_seq, t * n * H * 4, true);
+    st.add((void **)&a.mdn_seq, mdn_seq, t * n * M * 4, true);
+
+    int path = c.path;
+    if (path == WM_PATH_AUTO) path = wm_fused_supported(h, N) ? WM_PATH_FUSED : WM_PATH_STEPWISE;
+    if (path == WM_PATH_FUSED && !wm_fused_supported(h, N))
+        return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
+    if (path == WM_PATH_TENSOR) return fail(h, WM_ERR_UNSUPPORTED, "the tensor family is not built for scoring");
+    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : wm_step_nll_ws(h, N);
+    e = grow(&h->ws, &h->ws_bytes, need);
+    if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
+    if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    if (path == WM_PATH_FUSED)
+        e = wm_fused_nll(h, a, h->ws, s);
+    else
+        e = wm_step_nll(h, a, h->ws, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "nll launch");
+    h->last_path = path;
+    if (path == WM_PATH_STEPWISE) h->last_launches = N == 0 ? 0 : 2 + 4 * T;
+    if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
+    return WM_OK;
+}
+
+}  // extern "C"

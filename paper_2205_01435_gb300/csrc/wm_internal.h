@@ -1,0 +1,76 @@
+// wm_internal.h -- handle layout and kernel-family launchers behind the C ABI
+// of include/wm.h.  Not part of the public interface.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "wm.h"
+
+// Device pointers of one rollout call (after host arrays were staged).
+struct wm_rollout_dev {
+    int B, T;
+    unsigned long long ep0;
+    unsigned int t0;
+    const float *z0, *h0, *c0;
+    const uint8_t *done0;
+    const uint32_t *mask;
+    float *z_out;
+    int32_t *actions;
+    float *rewards;
+    uint8_t *done;
+    float *h_final, *c_final, *h_seq, *c_seq, *mdn_seq;
+    uint8_t *comp_seq;
+};
+
+// Device pointers of one teacher-forced scoring call.
+struct wm_nll_dev {
+    int N, T;
+    const float *z_seq;
+    const int32_t *actions;
+    const int32_t *lengths;
+    float *nll, *h_seq, *c_seq, *mdn_seq;
+};
+
+// Weights of the stepwise (SIMT) family: fp32 values (bf16-rounded in WM_BF16).
+struct wm_step_weights {
+    float *Wg;   // [Z+H, 4H+A]  rows z | h; cols gates i|f|g|o then controller
+    float *Wa;   // [A, 4H]      action rows of the gate matrix
+    float *bg;   // [4H+A]       gate bias then controller bias
+    float *Wh;   // [H, M+2]     mixture head, reward, done
+    float *bh;   // [M+2]
+};
+
+// Weights of the fused single-launch family (bf16 tensor-core operand images).
+struct wm_fused_weights {
+    void *img;         // packed per-CTA shared-memory images, see wm_fused.cu
+    size_t img_bytes;
+    void *wa;          // action rows, bf16, [A, 4H] in the fused gate-column order
+    float *bias;       // fp32 biases in the fused column order
+    int ok;            // 1 if the model fits this family
+    int cluster;       // CTAs per cluster
+};
+
+struct wm_handle {
+    wm_config cfg;
+    int device;
+    int M;                       // 3 K Z
+    wm_step_weights step;
+    wm_fused_weights fused;
+    void *ws = nullptr;          // workspace (grows on demand)
+    size_t ws_bytes = 0;
+    void *stage = nullptr;       // staging for host arrays (grows on demand)
+    size_t stage_bytes = 0;
+    int *status = nullptr;       // device status word (WM_ERR_TIMEOUT etc.)
+    int last_path = 0;
+    mutable int last_launches = 0;   // kernels launched by the last call
+    std::string err;
+};
+
+// ---- stepwise family (wm_step.cu) -------------------------------------------
+size_t wm_step_rollout_ws(const wm_handle *h, int B);
+size_t wm_step_nll_ws(const wm_handle *h, int N);
+cudaError_t wm_step_rollout(const wm_handle *h, const wm_rollout_dev &a, void *ws, cudaStream_t s);
+cudaError_t wm_step_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s);

@@ -1,0 +1,242 @@
+"""Thin Python binding of the C ABI in include/wm.h (ctypes, argument marshalling only).
+
+Every step of the dream path runs in the CUDA kernels of ``libwm.so``; this
+module only turns torch tensors into pointers and the call's stream.  There is
+no CPU fallback: if ``libwm.so`` is missing, importing the binding fails.
+
+Names mirror the C entry points: ``wm_create``, ``wm_rollout``, ``wm_mdn_nll``,
+``wm_sync``, ``wm_destroy``, ``wm_last_error``, ``wm_last_path``.  The
+``WorldModel`` class wraps them for convenience.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libwm.so")
+
+WM_OK, WM_ERR_INVALID_ARG, WM_ERR_CUDA, WM_ERR_UNSUPPORTED, WM_ERR_TIMEOUT, WM_ERR_OOM = range(6)
+WM_FP32, WM_BF16 = 0, 1
+PATHS = {"auto": 0, "stepwise": 1, "fused": 2, "tensor": 3}
+PATH_NAMES = {v: k for k, v in PATHS.items()}
+
+
+class WMError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"wm status {status}: {msg}")
+        self.status = status
+
+
+class wm_config(C.Structure):
+    _fields_ = [("z_dim", C.c_int), ("a_dim", C.c_int), ("h_dim", C.c_int), ("k_mix", C.c_int),
+                ("precision", C.c_int), ("mdn_tau", C.c_float), ("sigma_sqrt_tau", C.c_int),
+                ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_float), ("done_terminates", C.c_int),
+                ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int)]
+
+
+class wm_weights(C.Structure):
+    _fields_ = [("W_lstm", C.c_void_p), ("b_lstm", C.c_void_p), ("W_mdn", C.c_void_p),
+                ("b_mdn", C.c_void_p), ("w_rew", C.c_void_p), ("b_rew", C.c_float),
+                ("w_done", C.c_void_p), ("b_done", C.c_float), ("W_ctrl", C.c_void_p),
+                ("b_ctrl", C.c_void_p)]
+
+
+class wm_rollout_io(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "z0", "h0", "c0", "done0", "mask", "z_out", "actions", "rewards", "done", "h_final",
+        "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq")]
+
+
+def _load():
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(f"{_LIB_PATH} is missing: build it with "
+                          "`python -c 'import __graft_entry__ as g; g.build()'` (no CPU fallback)")
+    lib = C.CDLL(_LIB_PATH)
+    P = C.c_void_p
+    lib.wm_create.argtypes = [C.POINTER(wm_config), C.POINTER(wm_weights), C.POINTER(P)]
+    lib.wm_create.restype = C.c_int
+    lib.wm_rollout.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_uint,
+                               C.POINTER(wm_rollout_io), P]
+    lib.wm_rollout.restype = C.c_int
+    lib.wm_mdn_nll.argtypes = [P, C.c_int, C.c_int] + [P] * 7 + [P]
+    lib.wm_mdn_nll.restype = C.c_int
+    lib.wm_sync.argtypes = [P]
+    lib.wm_sync.restype = C.c_int
+    lib.wm_last_error.argtypes = [P]
+    lib.wm_last_error.restype = C.c_char_p
+    lib.wm_last_path.argtypes = [P]
+    lib.wm_last_path.restype = C.c_int
+    lib.wm_last_launches.argtypes = [P]
+    lib.wm_last_launches.restype = C.c_int
+    lib.wm_destroy.argtypes = [P]
+    lib.wm_destroy.restype = None
+    return lib
+
+
+_lib = _load()
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, torch.Tensor):
+        if not t.is_contiguous():
+            raise ValueError("tensors passed to the engine must be contiguous")
+        return C.c_void_p(t.data_ptr())
+    return C.c_void_p(int(t))
+
+
+def _check(h, st: int, what: str):
+    if st != WM_OK:
+        msg = _lib.wm_last_error(h).decode() if h else ""
+        raise WMError(st, f"{what}: {msg}")
+
+
+# ------------------------------------------------------------------ the C names
+def wm_create(cfg: dict, weights: dict):
+    """wm_create: copies + packs the fp32 host weights onto the current CUDA device."""
+    c = wm_config(int(cfg["z_dim"]), int(cfg["a_dim"]), int(cfg["h_dim"]), int(cfg["k_mix"]),
+                  WM_BF16 if cfg.get("precision", "fp32") == "bf16" else WM_FP32,
+                  float(cfg.get("mdn_tau", 1.0)), int(cfg.get("sigma_sqrt_tau", 0)),
+                  int(cfg.get("ctrl_sample", 0)), float(cfg.get("ctrl_tau", 1.0)),
+                  int(cfg.get("done_terminates", 0)), int(cfg.get("noop_terminates", 0)),
+                  int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF,
+                  PATHS[cfg.get("path", "auto")] if isinstance(cfg.get("path", "auto"), str)
+                  else int(cfg["path"]))
+    keep = {k: torch.as_tensor(weights[k], dtype=torch.float32).contiguous().cpu()
+            for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl")}
+    w = wm_weights(_ptr(keep["W_lstm"]), _ptr(keep["b_lstm"]), _ptr(keep["W_mdn"]),
+                   _ptr(keep["b_mdn"]), _ptr(keep["w_rew"]), float(weights["b_rew"]),
+                   _ptr(keep["w_done"]), float(weights["b_done"]), _ptr(keep["W_ctrl"]),
+                   _ptr(keep["b_ctrl"]))
+    h = C.c_void_p()
+    st = _lib.wm_create(C.byref(c), C.byref(w), C.byref(h))
+    if st != WM_OK:
+        raise WMError(st, "wm_create failed (invalid sizes or CUDA error)")
+    return h
+
+
+def wm_rollout(h, B: int, T: int, episode_offset: int, t0: int, io: dict, stream: int = 0):
+    s = wm_rollout_io(*[_ptr(io.get(n)) for n, _ in wm_rollout_io._fields_])
+    _check(h, _lib.wm_rollout(h, B, T, episode_offset, t0, C.byref(s), C.c_void_p(stream)),
+           "wm_rollout")
+
+
+def wm_mdn_nll(h, N: int, T: int, z_seq, actions, lengths, nll, h_seq=None, c_seq=None,
+               mdn_seq=None, stream: int = 0):
+    _check(h, _lib.wm_mdn_nll(h, N, T, _ptr(z_seq), _ptr(actions), _ptr(lengths), _ptr(nll),
+                              _ptr(h_seq), _ptr(c_seq), _ptr(mdn_seq), C.c_void_p(stream)),
+           "wm_mdn_nll")
+
+
+def wm_sync(h):
+    _check(h, _lib.wm_sync(h), "wm_sync")
+
+
+def wm_last_path(h) -> str:
+    return PATH_NAMES.get(_lib.wm_last_path(h), "?")
+
+
+def wm_last_launches(h) -> int:
+    return int(_lib.wm_last_launches(h))
+
+
+def wm_destroy(h):
+    _lib.wm_destroy(h)
+
+
+# ------------------------------------------------------------------ convenience wrapper
+class WorldModel:
+    """Owns one wm_handle on one CUDA device."""
+
+    def __init__(self, cfg: dict, weights: dict, device: int | torch.device | None = None):
+        self.cfg = dict(cfg)
+        self.Z, self.A, self.H, self.K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
+        self.M = 3 * self.K * self.Z
+        self.device = torch.device("cuda", torch.cuda.current_device() if device is None
+                                   else torch.device("cuda", device).index if isinstance(device, int)
+                                   else torch.device(device).index)
+        with torch.cuda.device(self.device):
+            self.h = wm_create(cfg, weights)
+
+    def close(self):
+        if getattr(self, "h", None):
+            wm_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _stream(self, stream):
+        if stream is not None:
+            return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+        return torch.cuda.current_stream(self.device).cuda_stream
+
+    def _alloc(self, like: torch.Tensor, shape, dtype):
+        if like.is_cuda:
+            return torch.empty(shape, dtype=dtype, device=like.device)
+        return torch.empty(shape, dtype=dtype, pin_memory=like.is_pinned())
+
+    def rollout(self, z0: torch.Tensor, T: int, mask: torch.Tensor | None = None,
+                episode_offset: int = 0, t0: int = 0, h0=None, c0=None, done0=None,
+                want_final: bool = True, want_seq: bool = False, out: dict | None = None,
+                stream=None) -> dict:
+        """wm_rollout on B = z0.shape[0] episodes; returns the output tensors (device of z0)."""
+        B = int(z0.shape[0])
+        o = dict(out or {})
+        for name, shape, dt in (("z", (T + 1, B, self.Z), torch.float32),
+                                ("actions", (T, B), torch.int32),
+                                ("rewards", (T, B), torch.float32),
+                                ("done", (T, B), torch.uint8)):
+            if name not in o:
+                o[name] = self._alloc(z0, shape, dt)
+        if want_final:
+            for name in ("h_final", "c_final"):
+                if name not in o:
+                    o[name] = self._alloc(z0, (B, self.H), torch.float32)
+        if want_seq:
+            o.setdefault("h_seq", self._alloc(z0, (T, B, self.H), torch.float32))
+            o.setdefault("c_seq", self._alloc(z0, (T, B, self.H), torch.float32))
+            o.setdefault("mdn_seq", self._alloc(z0, (T, B, self.M), torch.float32))
+            o.setdefault("comp_seq", self._alloc(z0, (T, B, self.Z), torch.uint8))
+        io = {"z0": z0, "h0": h0, "c0": c0, "done0": done0, "mask": mask, "z_out": o["z"],
+              "actions": o["actions"], "rewards": o["rewards"], "done": o["done"],
+              "h_final": o.get("h_final"), "c_final": o.get("c_final"), "h_seq": o.get("h_seq"),
+              "c_seq": o.get("c_seq"), "mdn_seq": o.get("mdn_seq"), "comp_seq": o.get("comp_seq")}
+        with torch.cuda.device(self.device):
+            wm_rollout(self.h, B, T, episode_offset, t0, io, self._stream(stream))
+        return o
+
+    def mdn_nll(self, z_seq: torch.Tensor, actions: torch.Tensor, lengths=None,
+                want_seq: bool = False, stream=None) -> dict:
+        T = int(z_seq.shape[0]) - 1
+        N = int(z_seq.shape[1])
+        o = {"nll": self._alloc(z_seq, (N,), torch.float32)}
+        if want_seq:
+            o["h_seq"] = self._alloc(z_seq, (T, N, self.H), torch.float32)
+            o["c_seq"] = self._alloc(z_seq, (T, N, self.H), torch.float32)
+            o["mdn_seq"] = self._alloc(z_seq, (T, N, self.M), torch.float32)
+        with torch.cuda.device(self.device):
+            wm_mdn_nll(self.h, N, T, z_seq, actions, lengths, o["nll"], o.get("h_seq"),
+                       o.get("c_seq"), o.get("mdn_seq"), self._stream(stream))
+        return o
+
+    def sync(self):
+        wm_sync(self.h)
+
+    @property
+    def last_path(self) -> str:
+        return wm_last_path(self.h)
+
+    @property
+    def last_launches(self) -> int:
+        return wm_last_launches(self.h)

@@ -1,0 +1,249 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs and Philox noise.  Rules and tolerances: tests/parity.py."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from parity import check_rollout, check_teacher, np_
+
+pytestmark = pytest.mark.gpu
+NT = os.cpu_count() or 1
+
+
+@pytest.fixture(scope="module")
+def wm():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    import paper_2205_01435_gb300 as pkg
+    return pkg.load()
+
+
+def _cuda(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _spread(B, n):
+    """n episode indices spread over [0, B), always including the first and last."""
+    if n >= B:
+        return np.arange(B)
+    return np.unique(np.linspace(0, B - 1, n).round().astype(np.int64))
+
+
+def _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=False):
+    """Oracle rollout of episodes idx (Philox keyed by their global index)."""
+    outs = []
+    idx = list(idx)
+    # contiguous runs share one call
+    start = 0
+    while start < len(idx):
+        end = start
+        while end + 1 < len(idx) and idx[end + 1] == idx[end] + 1:
+            end += 1
+        lo, hi = idx[start], idx[end] + 1
+        outs.append(orc.rollout(cfg, w, z0[lo:hi], None if mask is None else mask[:, lo:hi], T,
+                                episode_offset=lo, want_seq=want_seq, nthreads=NT))
+        start = end + 1
+    cat = {}
+    for k in outs[0]:
+        ax = 0 if k in ("h_final", "c_final") else 1
+        cat[k] = np.concatenate([o[k] for o in outs], axis=ax)
+    return cat
+
+
+PATHS_SMALL = ["stepwise", "auto"]
+
+
+# ------------------------------------------------------------------ teacher-forced
+TEACHER = [("tiny_fp32", None, 16, 20), ("small_bf16", None, 64, 50), ("mid_bf16", None, 32, 40),
+           ("nll", "fp32", 512, 128), ("nll", "bf16", 512, 128), ("large_bf16", None, 8, 12)]
+
+
+@pytest.mark.parametrize("name,prec,N,T", TEACHER)
+@pytest.mark.parametrize("path", PATHS_SMALL)
+def test_teacher_forced_parity(wm, orc, name, prec, N, T, path):
+    cfg = synth.model_config(name)
+    if prec:
+        cfg["precision"] = prec
+    w = synth.weights(cfg)
+    zs, acts, _ = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=3)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.mdn_nll(_cuda(zs), _cuda(acts), want_seq=True)
+    torch.cuda.synchronize()
+    idx = _spread(N, 96)
+    o = orc.mdn_nll(cfg, w, zs[:, idx], acts[:, idx], want_seq=True, nthreads=NT)
+    gs = {k: np_(v)[:, idx] if k != "nll" else np_(v)[idx] for k, v in g.items()}
+    check_teacher(gs, o, cfg["precision"])
+    if cfg["precision"] == "bf16":
+        # the bf16 path also stays within 2e-2 of the plain fp32 oracle
+        o32 = orc.mdn_nll(dict(cfg, precision="fp32"), w, zs[:, idx], acts[:, idx],
+                          want_seq=True, nthreads=NT)
+        for k in ("h_seq", "c_seq", "mdn_seq"):
+            assert float(np.abs(gs[k] - o32[k]).max()) <= 2e-2
+
+
+def test_teacher_forced_ragged_lengths_and_no_action(wm, orc):
+    cfg = dict(synth.model_config("tiny_fp32"), z_dim=7, a_dim=45, h_dim=40, k_mix=3)
+    w = synth.weights(cfg, seed=4)
+    zs, acts, lens = synth.teacher_inputs(37, 9, 7, 45, seed=4, ragged=True)
+    acts[::3, ::2] = -1
+    lens[0], lens[1] = 0, 9
+    for path in PATHS_SMALL:
+        m = wm.WorldModel(dict(cfg, path=path), w)
+        g = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+        o = orc.mdn_nll(cfg, w, zs, acts, lengths=lens, want_seq=True)
+        check_teacher({k: np_(v) for k, v in g.items()}, o, "fp32")
+
+
+# ------------------------------------------------------------------ free-running rollouts
+@pytest.mark.parametrize("path", PATHS_SMALL)
+def test_rollout_tiny_full(wm, orc, path):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
+    r = check_rollout(g, o, cfg)
+    assert r["clean_episodes"] >= B - 2
+
+
+@pytest.mark.parametrize("path", PATHS_SMALL)
+def test_rollout_small_bf16(wm, orc, path):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16")
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    idx = _spread(B, 48)
+    o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
+    check_rollout(g, o, cfg, idx)
+
+
+def _rollout_sampled(wm, orc, name, n_oracle, path="auto"):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    comp = torch.empty((T, B, cfg["z_dim"]), dtype=torch.uint8, device="cuda")
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), out={"comp_seq": comp})
+    torch.cuda.synchronize()
+    idx = _spread(B, n_oracle)
+    o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
+    return check_rollout(g, o, cfg, idx)
+
+
+def test_rollout_mid_bf16_sampled(wm, orc):
+    r = _rollout_sampled(wm, orc, "mid_bf16", 24)
+    print("mid_bf16 parity:", r)
+
+
+def test_rollout_large_bf16_sampled(wm, orc):
+    r = _rollout_sampled(wm, orc, "large_bf16", 24)
+    print("large_bf16 parity:", r)
+
+
+# ------------------------------------------------------------------ edge cases
+@pytest.mark.parametrize("path", PATHS_SMALL)
+def test_ragged_shapes_and_flags(wm, orc, path):
+    cfg = dict(synth.model_config("tiny_fp32"), z_dim=5, a_dim=33, h_dim=24, k_mix=3,
+               noop_terminates=1, done_terminates=1)
+    w = synth.weights(cfg, seed=9, std=0.3)
+    B, T = 37, 7
+    z0 = synth.z0(B, 5, seed=9)
+    mask = synth.mask(T, B, 33, 0.4, seed=9)
+    mask[2, 5] = 0  # all masked at one step
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=123456789012, t0=77,
+                  want_seq=True)
+    o = orc.rollout(cfg, w, z0, mask, T, episode_offset=123456789012, t0=77, want_seq=True)
+    check_rollout(g, o, cfg)
+
+
+@pytest.mark.parametrize("tau,sq", [(0.0, 0), (0.5, 1), (1.7, 0)])
+def test_mixture_temperature(wm, orc, tau, sq):
+    cfg = dict(synth.model_config("tiny_fp32"), mdn_tau=tau, sigma_sqrt_tau=sq)
+    cfg2, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32", T=8)
+    m = wm.WorldModel(dict(cfg, path="auto"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
+    check_rollout(g, o, cfg)
+
+
+def test_sampled_controller(wm, orc):
+    cfg = dict(synth.model_config("tiny_fp32"), ctrl_sample=1, ctrl_tau=0.8)
+    _, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
+    for path in PATHS_SMALL:
+        m = wm.WorldModel(dict(cfg, path=path), w)
+        g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+        o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
+        check_rollout(g, o, cfg)
+
+
+def test_empty_and_zero_length(wm):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
+    m = wm.WorldModel(cfg, w)
+    g = m.rollout(_cuda(z0[:0]), T, mask=_cuda(mask[:, :0]))
+    assert g["z"].shape == (T + 1, 0, cfg["z_dim"])
+    h0 = torch.randn(B, cfg["h_dim"], device="cuda")
+    g = m.rollout(_cuda(z0), 0, h0=h0)
+    torch.cuda.synchronize()
+    assert torch.equal(g["z"][0].cpu(), torch.from_numpy(z0))
+    assert torch.equal(g["h_final"], h0)
+    n = m.mdn_nll(_cuda(np.zeros((1, 0, cfg["z_dim"]), np.float32)),
+                  _cuda(np.zeros((0, 0), np.int32)))
+    assert n["nll"].numel() == 0
+
+
+def test_invalid_arguments(wm):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
+    m = wm.WorldModel(cfg, w)
+    with pytest.raises(wm.WMError) as ei:
+        wm.wm_rollout(m.h, -1, T, 0, 0, {"z0": _cuda(z0)})
+    assert ei.value.status == wm.WM_ERR_INVALID_ARG
+    with pytest.raises(wm.WMError):
+        wm.wm_rollout(m.h, B, T, 0, 0, {"z0": _cuda(z0)})  # outputs missing
+    zs, acts, _ = synth.teacher_inputs(4, 3, cfg["z_dim"], cfg["a_dim"])
+    acts[0, 0] = cfg["a_dim"]
+    with pytest.raises(wm.WMError):
+        m.mdn_nll(torch.from_numpy(zs), torch.from_numpy(acts))  # host actions are checked
+
+
+# ------------------------------------------------------------------ invariants of the GPU path
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_sharding_is_bit_exact(wm, name):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, T=12)
+    m = wm.WorldModel(cfg, w)
+    zc, mc = _cuda(z0), _cuda(mask)
+    full = m.rollout(zc, T, mask=mc)
+    cut = B // 3
+    lo = m.rollout(zc[:cut].contiguous(), T, mask=mc[:, :cut].contiguous())
+    hi = m.rollout(zc[cut:].contiguous(), T, mask=mc[:, cut:].contiguous(), episode_offset=cut)
+    for k in ("z", "actions", "rewards", "done"):
+        assert torch.equal(torch.cat([lo[k], hi[k]], 1), full[k]), k
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_resume_is_bit_exact(wm, name):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, T=10)
+    cfg["done_terminates"] = 1
+    m = wm.WorldModel(cfg, w)
+    zc, mc = _cuda(z0), _cuda(mask)
+    full = m.rollout(zc, T, mask=mc)
+    a = m.rollout(zc, 4, mask=mc[:4].contiguous())
+    b = m.rollout(a["z"][4].contiguous(), T - 4, mask=mc[4:].contiguous(), t0=4,
+                  h0=a["h_final"], c0=a["c_final"], done0=a["done"][3].contiguous())
+    assert torch.equal(torch.cat([a["z"], b["z"][1:]]), full["z"])
+    for k in ("actions", "rewards", "done"):
+        assert torch.equal(torch.cat([a[k], b[k]]), full[k]), k
+
+
+@pytest.mark.parametrize("kind", ["pinned", "pageable"])
+def test_host_buffers_match_device_buffers(wm, kind):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", T=6)
+    m = wm.WorldModel(cfg, w)
+    dev = m.rollout(_cuda(z0), T, mask=_cuda(mask))
+    zh, mh = torch.from_numpy(z0), torch.from_numpy(mask)
+    if kind == "pinned":
+        zh, mh = zh.pin_memory(), mh.pin_memory()
+    host = m.rollout(zh, T, mask=mh)  # outputs allocated on the host, call syncs
+    for k in ("z", "actions", "rewards", "done", "h_final", "c_final"):
+        assert not host[k].is_cuda
+        assert torch.equal(host[k], dev[k].cpu()), k
