@@ -116,18 +116,30 @@ def test_rollout_small_bf16(wm, orc, path):
     torch.cuda.synchronize()
     idx = _spread(B, 48)
     o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
-    check_rollout(g, o, cfg, idx)
+    check_rollout(g, o, cfg, idx, weights=w)
 
 
 def _rollout_sampled(wm, orc, name, n_oracle, path="auto"):
+    """Full-size GPU rollout; the sampled episodes are re-run alone on the GPU (bit-exact
+    against the full batch, since episodes are independent) to get their per-step
+    sequences, then compared with the oracle."""
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
     m = wm.WorldModel(dict(cfg, path=path), w)
     comp = torch.empty((T, B, cfg["z_dim"]), dtype=torch.uint8, device="cuda")
-    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), out={"comp_seq": comp})
+    full = m.rollout(_cuda(z0), T, mask=_cuda(mask), out={"comp_seq": comp})
     torch.cuda.synchronize()
     idx = _spread(B, n_oracle)
+    parts = []
+    for b in idx:
+        one = m.rollout(_cuda(z0[b:b + 1]), T, mask=_cuda(mask[:, b:b + 1]), episode_offset=int(b),
+                        want_seq=True)
+        for k in ("z", "actions", "rewards", "done", "comp_seq"):
+            assert torch.equal(one[k][:, 0], full[k][:, int(b)]), (k, int(b))
+        parts.append({k: np_(v) for k, v in one.items()})
+    g = {k: np.concatenate([p[k] for p in parts], axis=0 if k in ("h_final", "c_final") else 1)
+         for k in parts[0]}
     o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
-    return check_rollout(g, o, cfg, idx)
+    return check_rollout(g, o, cfg, weights=w)
 
 
 def test_rollout_mid_bf16_sampled(wm, orc):
