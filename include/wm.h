@@ -159,6 +159,35 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
                      const int32_t *lengths, float *nll, float *h_seq, float *c_seq,
                      float *mdn_seq, void *cuda_stream);
 
+/* wm_rollout without any device allocation.  The paper has no counterpart:
+ * this entry point exists for callers that cannot call cudaMalloc/cudaFree
+ * while they run -- work issued during CUDA stream capture, real-time loops
+ * where an allocation (and the device-wide synchronisation cudaFree implies)
+ * would stall other work, or hosts whose GPU memory belongs entirely to
+ * another allocator.  wm_rollout may grow its per-handle workspace (and stage
+ * host arrays) on demand; this call never does.
+ *
+ * Same arguments, results and Philox keying as wm_rollout, always on the
+ * stepwise kernel family.  Differences:
+ *   - every array must be device or managed memory (host memory is rejected
+ *     with WM_ERR_INVALID_ARG, since it would need staging buffers);
+ *   - its scratch (gate and head buffers, h, c, frozen flags) is a fixed
+ *     WM_NOALLOC_SCRATCH_BYTES array inside the library, which every GPU that
+ *     loads the library holds until the process exits; a batch whose scratch
+ *     would exceed it is rejected with WM_ERR_INVALID_ARG (at Z=32, A=128,
+ *     H=256, K=5 that allows about 1950 episodes);
+ *   - all calls share that array, so calls that overlap on the GPU (on any
+ *     handle of the process, on different streams) race and corrupt each
+ *     other: serialise them.  Each call re-initialises the state it needs;
+ *   - the first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with the handle's device made current) and
+ *     caches it, so make that first call before any stream capture begins.
+ * The handle itself (wm_create) still holds the packed weights allocated at
+ * set-up time. */
+#define WM_NOALLOC_SCRATCH_BYTES (16u << 20)
+wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned long long episode_offset,
+                             unsigned int t0, const wm_rollout_io *io, void *cuda_stream);
+
 /* Synchronises the device and returns the first device-side error since the
  * last wm_sync (WM_ERR_TIMEOUT if a bounded wait gave up), then clears it. */
 wm_status wm_sync(wm_handle *h);

@@ -60,6 +60,9 @@ def _load():
     lib.wm_rollout.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_uint,
                                C.POINTER(wm_rollout_io), P]
     lib.wm_rollout.restype = C.c_int
+    lib.wm_rollout_noalloc.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_uint,
+                                       C.POINTER(wm_rollout_io), P]
+    lib.wm_rollout_noalloc.restype = C.c_int
     lib.wm_mdn_nll.argtypes = [P, C.c_int, C.c_int] + [P] * 7 + [P]
     lib.wm_mdn_nll.restype = C.c_int
     lib.wm_sync.argtypes = [P]
@@ -126,6 +129,14 @@ def wm_rollout(h, B: int, T: int, episode_offset: int, t0: int, io: dict, stream
     s = wm_rollout_io(*[_ptr(io.get(n)) for n, _ in wm_rollout_io._fields_])
     _check(h, _lib.wm_rollout(h, B, T, episode_offset, t0, C.byref(s), C.c_void_p(stream)),
            "wm_rollout")
+
+
+def wm_rollout_noalloc(h, B: int, T: int, episode_offset: int, t0: int, io: dict,
+                       stream: int = 0):
+    """wm_rollout_noalloc: device arrays only; scratch from the library's fixed array."""
+    s = wm_rollout_io(*[_ptr(io.get(n)) for n, _ in wm_rollout_io._fields_])
+    _check(h, _lib.wm_rollout_noalloc(h, B, T, episode_offset, t0, C.byref(s),
+                                      C.c_void_p(stream)), "wm_rollout_noalloc")
 
 
 def wm_mdn_nll(h, N: int, T: int, z_seq, actions, lengths, nll, h_seq=None, c_seq=None,
