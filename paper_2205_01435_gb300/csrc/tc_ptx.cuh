@@ -67,6 +67,10 @@ __device__ __forceinline__ void fence_after_sync() {
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// same, for generic-proxy stores into other CTAs' shared memory (DSMEM)
+__device__ __forceinline__ void fence_proxy_async_cluster() {
+    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+}
 
 // TMEM allocation: one full warp executes these.
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_saddr, uint32_t ncols) {

@@ -51,6 +51,7 @@ struct wm_fused_weights {
     float *bias;       // fp32 biases in the fused column order
     int ok;            // 1 if the model fits this family
     int cluster;       // CTAs per cluster
+    int max_clusters;  // clusters of this size that can be resident at once
 };
 
 struct wm_handle {

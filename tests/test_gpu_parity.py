@@ -259,3 +259,55 @@ def test_host_buffers_match_device_buffers(wm, kind):
     for k in ("z", "actions", "rewards", "done", "h_final", "c_final"):
         assert not host[k].is_cuda
         assert torch.equal(host[k], dev[k].cpu()), k
+
+
+# ------------------------------------------------------------------ the fused single-launch family
+@pytest.mark.parametrize("flags", [dict(), dict(done_terminates=1, noop_terminates=1),
+                                   dict(mdn_tau=0.0), dict(mdn_tau=0.5, sigma_sqrt_tau=1)])
+def test_fused_against_oracle(wm, orc, flags):
+    """Two clusters (the second one partly filled), resumed state, offsets, flags."""
+    cfg = dict(synth.model_config("small_bf16"), **flags)
+    w = synth.weights(cfg, seed=5)
+    B, T = 200, 9
+    z0 = synth.z0(B, cfg["z_dim"], seed=5)
+    mask = synth.mask(T, B, cfg["a_dim"], 0.3, seed=5)
+    mask[3, 17] = 0  # no valid action for one episode at one step
+    rng = np.random.default_rng(5)
+    h0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    c0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    done0 = (np.arange(B) % 37 == 0).astype(np.uint8)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=77, t0=3, h0=_cuda(h0),
+                  c0=_cuda(c0), done0=_cuda(done0), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    o = orc.rollout(cfg, w, z0, mask, T, episode_offset=77, t0=3, h0=h0, c0=c0, done0=done0,
+                    want_seq=True, nthreads=NT)
+    r = check_rollout(g, o, cfg, weights=w, h0=h0)
+    print("fused", flags, r)
+
+
+def test_fused_teacher_forced_ragged(wm, orc):
+    cfg = synth.model_config("small_bf16")
+    w = synth.weights(cfg, seed=6)
+    zs, acts, lens = synth.teacher_inputs(300, 11, cfg["z_dim"], cfg["a_dim"], seed=6, ragged=True)
+    acts[2, ::5] = -1
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    o = orc.mdn_nll(cfg, w, zs, acts, lengths=lens, want_seq=True, nthreads=NT)
+    check_teacher({k: np_(v) for k, v in g.items()}, o, "bf16")
+
+
+def test_fused_matches_stepwise_closely(wm):
+    """Same model through both families: equal decisions and close values until an
+    episode's first near-tie flip (the two families round differently)."""
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", T=20)
+    a = wm.WorldModel(dict(cfg, path="fused"), w).rollout(_cuda(z0), T, mask=_cuda(mask))
+    b = wm.WorldModel(dict(cfg, path="stepwise"), w).rollout(_cuda(z0), T, mask=_cuda(mask))
+    torch.cuda.synchronize()
+    act_eq = (a["actions"] == b["actions"]).cpu().numpy()             # [T, B]
+    z_eq = ((a["z"][1:] - b["z"][1:]).abs().amax(-1) < 2e-2).cpu().numpy()
+    ok = np.cumprod(act_eq & z_eq, axis=0)                           # 1 until first divergence
+    assert ok.mean() > 0.95, ok.mean()
