@@ -118,6 +118,11 @@ __device__ __forceinline__ uint32_t mbar_try_wait(uint32_t saddr, uint32_t parit
         : "=r"(ok) : "r"(saddr), "r"(parity) : "memory");
     return ok;
 }
+// Arrive once on the current phase and add `bytes` to the transaction count it waits for.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t saddr, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(saddr), "r"(bytes)
+                 : "memory");
+}
 // Bounded wait: returns false if the phase did not complete within max_iter polls.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t saddr, uint32_t parity, uint32_t max_iter) {
     for (uint32_t i = 0; i < max_iter; ++i)
@@ -140,6 +145,15 @@ __device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
     uint32_t r;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
     return r;
+}
+// Bulk copy (TMA engine) of `bytes` from this CTA's shared memory into the shared memory
+// of a CTA of the cluster; the destination's mbarrier counts the bytes on arrival.
+// Addresses 16-byte aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
+                                                  uint32_t mbar_cluster) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        :: "r"(dst_cluster), "r"(src_cta), "r"(bytes), "r"(mbar_cluster) : "memory");
 }
 __device__ __forceinline__ void st_cluster_v4(uint32_t caddr, uint4 v) {
     asm volatile("st.shared::cluster.v4.b32 [%0], {%1,%2,%3,%4};"
