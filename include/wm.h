@@ -91,6 +91,8 @@ typedef struct {
     int noop_terminates;              /* action A-1 (NO-OP, Sec. 3.1.3) freezes it */
     unsigned long long seed;          /* Philox key                                */
     int path;                         /* WM_PATH_*                                 */
+    int fused_cluster;                /* fused family: CTAs per cluster, 8 or 16;
+                                         0 = choose per call (fewest waves)        */
 } wm_config;
 
 /* Canonical fp32 weights, row-major, HOST memory; copied (and packed) by

@@ -155,6 +155,14 @@ __device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t
         "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
         :: "r"(dst_cluster), "r"(src_cta), "r"(bytes), "r"(mbar_cluster) : "memory");
 }
+// Bulk copy (TMA engine) of `bytes` from global memory into this CTA's shared memory,
+// counted on this CTA's mbarrier.  Addresses 16-byte aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_load_global(uint32_t dst_cta, const void *src, uint32_t bytes,
+                                                 uint32_t mbar_cta) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        :: "r"(dst_cta), "l"(src), "r"(bytes), "r"(mbar_cta) : "memory");
+}
 __device__ __forceinline__ void st_cluster_v4(uint32_t caddr, uint4 v) {
     asm volatile("st.shared::cluster.v4.b32 [%0], {%1,%2,%3,%4};"
                  :: "r"(caddr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");

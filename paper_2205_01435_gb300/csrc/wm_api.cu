@@ -115,7 +115,8 @@ bool valid_cfg(const wm_config *c) {
     return c && c->z_dim > 0 && c->a_dim > 0 && c->h_dim > 0 && c->k_mix > 0 && c->k_mix <= 32 &&
            (c->precision == WM_FP32 || c->precision == WM_BF16) && c->mdn_tau >= 0.f &&
            c->ctrl_tau >= 0.f && c->path >= WM_PATH_AUTO && c->path <= WM_PATH_TENSOR &&
-           c->z_dim <= 4096 && c->a_dim <= 65536 && c->h_dim <= 16384;
+           c->z_dim <= 4096 && c->a_dim <= 65536 && c->h_dim <= 16384 &&
+           (c->fused_cluster == 0 || c->fused_cluster == 8 || c->fused_cluster == 16);
 }
 
 cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
@@ -168,6 +169,7 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) 
     memset(&h->fused, 0, sizeof(h->fused));
     cudaError_t e = cudaGetDevice(&h->device);
     if (e == cudaSuccess) e = pack_step(h, w);
+    h->fused.force_cluster = cfg->fused_cluster;
     if (e == cudaSuccess) e = wm_fused_pack(h, w);
     if (e == cudaSuccess) e = cudaMalloc((void **)&h->status, sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, sizeof(int));

@@ -1,33 +1,48 @@
 // wm_fused.cu -- the fused kernel family: one launch runs all T dream steps.
 //
-// Layout of the work.  One thread-block cluster of CL = 16 CTAs owns a tile of
-// 128 episodes (the M = 128 of a tcgen05 MMA; thread i of every CTA is episode
-// i of the tile and TMEM lane i).  The weights are split by output column across
-// the 16 CTAs and stay resident in shared memory for the whole rollout:
-//   rank r owns hidden units [rU, rU+U)  -> 4U gate columns (i|f|g|o)   (a3)
-//              actions [r*AC, r*AC+AC)   -> controller columns          (a1)
-//              latent dims [r*ZD, r*ZD+ZD) -> 3*ZD*K mixture columns     (a5)
-//   and every rank also computes the reward and done columns (2 columns), so
-//   the done decision needs no exchange.
+// Layout of the work.  One thread-block cluster of CL CTAs (CL = 16 or 8) owns a
+// tile of 128 episodes (the M = 128 of a tcgen05 MMA; TMEM lane i = episode i of
+// the tile).  The weights are split by output column across the CL CTAs:
+//   rank r owns hidden units [rU, rU+U), U = H/CL -> 4U gate columns      (a3)
+//              actions [r*AC, r*AC+AC), AC = A/CL -> controller columns   (a1)
+//              latent dims [r*ZD, r*ZD+ZD), ZD = Z/CL -> 16 head columns
+//              per dim (K logits, K means, K log-sigmas, one spare)       (a5)
+//   and the spare columns of its first two dims carry the reward and done heads,
+//   so every CTA knows the done decision without an exchange.
 // Each CTA holds the full GEMM operand tile X = [z_t | h_t] (128 x (Z+H) bf16,
-// K-major core-matrix layout).  Per step:
-//   MMA1  X x W1_r -> TMEM (gate and controller pre-activations)
-//   each CTA: masked local argmax over its actions; (value, index) partials are
-//         written into every CTA (DSMEM)                               -- barrier 1
-//   every CTA reduces the 16 partials (same order everywhere) -> a_t (a2);
-//   gates + bias + W_a[a_t] row (shared-memory gather), LSTM cell with c kept
-//         in registers (a4); h' (bf16) is written into every CTA's X    -- barrier 2
-//   MMA2  X_h x W2_r -> TMEM (mixture head, reward, done)
-//   per owned dim: temperature softmax, inverse-CDF component, Box-Muller
-//         (a6, a7); z' (bf16) is written into every CTA's X; done/freeze (a8)
-//                                                                       -- barrier 3
-// In teacher-forced mode (a9) the actions and z come from the inputs, every CTA
-// loads z_{t+1} itself, and each rank accumulates the NLL of its dims; a small
-// kernel adds the 16 partials per sequence in a fixed order.
+// K-major core-matrix layout), its gate/controller weights W1 and the biases.
+// W_a (the action rows of the gate matrix, used by the cell update) and W2 (the
+// head weights, used by MMA2) are needed at disjoint moments of a step, so they
+// share one shared-memory buffer that TMA bulk loads refill from L2 each step
+// while the exchanges run.  Per step:
+//   MMA1  X x W1 -> TMEM: gate and controller pre-activations (the h part of it
+//         was issued at the end of the previous step, the z part now)
+//   masked local argmax over the rank's actions; (value, index) partials go to
+//         every CTA                                                  (a2)
+//   the CL partials are reduced in rank order -> a_t; gates + bias + the W_a
+//         row, LSTM cell with c in registers; h' (bf16) goes into every CTA's X
+//                                                                    (a3, a4)
+//   MMA2  X_h x W2 -> TMEM: mixture head, reward, done
+//   per owned dim: temperature softmax, inverse-CDF component, Box-Muller (a6,
+//         a7); z' (bf16) goes to every CTA; done / freeze (a8)
+// Exchanges: a CTA writes its slice into its own shared memory, then the TMA
+// engine copies it into the same offset of every other CTA of the cluster
+// (cp.async.bulk shared::cluster), completing on the receiver's mbarrier.  No
+// cluster barrier runs inside the step loop: the data dependencies order every
+// reuse of a buffer (the partials certify that every CTA's MMA1 has finished
+// reading X before any h' lands in it; h' -> MMA2 -> z' certifies that the
+// z staging area was consumed).
+// Threads: 512 compute threads per CTA, 4 per episode row (TMEM lets warps w,
+// w+4, w+8, w+12 read the same 32 lanes); group g = warp/4 owns U/4 hidden units
+// and, if g < ZD, one latent dim.  A 17th warp issues every MMA and weight load,
+// so the tensor core is fed while the compute warps work.
+// In teacher-forced mode (a9) actions and z come from the inputs, every CTA
+// loads z_{t+1} itself, and each latent dim keeps its NLL partial; a small
+// kernel adds the partials per sequence in a fixed order.
 //
-// Waits on MMA completion are bounded: on expiry the kernel records
-// WM_ERR_TIMEOUT in the status word, stops issuing MMAs and waiting, and still
-// runs every cluster barrier so that all CTAs finish.
+// All waits are bounded: on expiry the kernel records WM_ERR_TIMEOUT in the
+// status word, stops issuing MMAs and waiting, and still reaches the final
+// cluster barrier, so that every CTA finishes.
 #include <cuda_bf16.h>
 #include <math.h>
 #include <string.h>
@@ -42,30 +57,36 @@ using namespace wmk;
 
 namespace {
 
-constexpr int CL = 16;     // CTAs per cluster
-constexpr int TILE = 128;  // episodes per cluster = MMA M = threads per CTA
+constexpr int TILE = 128;              // episodes per cluster = MMA M
+constexpr int NT = 4 * TILE;           // compute threads per CTA: 4 per episode row
+constexpr int NGRP = NT / TILE;        // thread groups per row
+constexpr int NTHREADS = NT + 32;      // + one warp that issues MMAs and weight loads
+constexpr int MMA_WARP = NT / 32;
 constexpr uint32_t WAIT_POLLS = 1u << 26;
+constexpr uint32_t D2_COL = 160;       // TMEM column of the MMA2 accumulator
 
-template <int U_, int ZD_, int KM_>
+template <int CL_, int U_, int ZD_, int KM_>
 struct Shape {
-    static constexpr int U = U_, ZD = ZD_, KM = KM_;
+    static constexpr int CL = CL_, U = U_, ZD = ZD_, KM = KM_;
+    static constexpr int UG = U / NGRP;                    // units per thread
     static constexpr int NG = 4 * U;                       // gate columns
     static constexpr int NA = 16;                          // controller columns (padded)
     static constexpr int N1 = NG + NA;                     // MMA1 N (rollout)
-    static constexpr int NH = 3 * ZD * KM;                 // mixture-head columns
-    static constexpr int N2 = (NH + 2 + 15) / 16 * 16;     // MMA2 N (+ reward, done)
+    static constexpr int N2 = 16 * ZD;                     // MMA2 N
     static constexpr int WA_STRIDE = NG * 2 + 16;          // bytes per action row of W_a
-    static_assert(N1 % 16 == 0 && N1 <= 256, "MMA1 N");
-    static_assert(N2 % 16 == 0 && N2 <= 128, "MMA2 N");
+    static_assert(UG == 4 || UG == 8, "4 or 8 units per thread");
+    static_assert(ZD >= 2 && ZD <= NGRP && 3 * KM + 1 <= 16, "head column groups");
+    static_assert(N1 % 16 == 0 && N1 <= (int)D2_COL && N2 <= 256 - (int)D2_COL, "TMEM columns");
 };
 
-// The one shape instantiated: Z = 32, H = 256, K = 5 (A = 16 * AC, AC <= 16).
-using S0 = Shape<16, 2, 5>;
-static_assert(S0::ZD == 2, "the z' exchange packs two bf16 dims per rank into one word");
+// Z = 32, H = 256, K = 5: 16 CTAs of 16 units / 2 dims, or 8 CTAs of 32 units / 4 dims.
+using S16 = Shape<16, 16, 2, 5>;
+using S8 = Shape<8, 32, 4, 5>;
 
-struct Geo {  // byte layout of a rank's weight image / of shared memory
-    size_t w1, w2, wa, b1, b2, img;  // image sections (offsets) and total
-    size_t x, part, zst, smem;       // shared-memory extras and total
+struct Geo {               // byte layout of a rank's weight image and of shared memory
+    size_t w1, b1, b2;     // resident part (same offsets in the image and in smem)
+    size_t iwa, iw2, img;  // streamed sections of the image, image size
+    size_t buf, buf_bytes, x, part, zst, smem;
 };
 
 __host__ __device__ inline size_t a128(size_t x) { return (x + 127) & ~(size_t)127; }
@@ -75,15 +96,18 @@ __host__ __device__ Geo geometry(int Z, int A, int H) {
     Geo g{};
     const size_t K1 = Z + H;
     g.w1 = 0;
-    g.w2 = a128(g.w1 + (size_t)S::N1 * K1 * 2);
-    g.wa = a128(g.w2 + (size_t)S::N2 * H * 2);
-    g.b1 = a128(g.wa + (size_t)A * S::WA_STRIDE);
+    g.b1 = a128(g.w1 + (size_t)S::N1 * K1 * 2);
     g.b2 = a128(g.b1 + (size_t)S::N1 * 4);
-    g.img = a128(g.b2 + (size_t)S::N2 * 4);
-    g.x = (g.img + 1023) & ~(size_t)1023;
+    g.iwa = a128(g.b2 + (size_t)S::N2 * 4);
+    g.iw2 = a128(g.iwa + (size_t)A * S::WA_STRIDE);
+    g.img = a128(g.iw2 + (size_t)S::N2 * H * 2);
+    const size_t wa_bytes = (size_t)A * S::WA_STRIDE, w2_bytes = (size_t)S::N2 * H * 2;
+    g.buf = g.iwa;
+    g.buf_bytes = wa_bytes > w2_bytes ? wa_bytes : w2_bytes;
+    g.x = (g.buf + g.buf_bytes + 1023) & ~(size_t)1023;
     g.part = a128(g.x + (size_t)TILE * K1 * 2);
-    g.zst = a128(g.part + (size_t)CL * TILE * 8);
-    g.smem = a128(g.zst + (size_t)CL * TILE * 4);
+    g.zst = a128(g.part + (size_t)S::CL * TILE * 8);
+    g.smem = a128(g.zst + (size_t)S::CL * TILE * S::ZD * 2);
     return g;
 }
 
@@ -107,7 +131,7 @@ struct FusedParams {
     uint8_t *comp_seq;
     const float *z_seq;
     const int32_t *act_in, *lengths;
-    float *nll_part;  // [CL, B]
+    float *nll_part;  // [Z, B]: one partial per latent dim
     int *status;
 };
 
@@ -126,11 +150,9 @@ __device__ __forceinline__ void x_store8(unsigned char *sx, int r, int k, const 
     *reinterpret_cast<uint4 *>(sx + tc::kmajor_offset(r, k, TILE)) = q;
 }
 
-constexpr int NT = 4 * TILE;  // 4 threads per episode row
-constexpr int NGRP = NT / TILE;
-
 // Push this CTA's block at shared address `src` (same offset in every CTA) to the
-// 15 other CTAs of the cluster; lane 0 of warp w < nwarps serves peers w, w + nwarps, ...
+// other CTAs of the cluster; lane 0 of warp w < nwarps serves peers w, w + nwarps, ...
+template <int CL>
 __device__ __forceinline__ void push_to_peers(uint32_t src, uint32_t bytes, uint32_t mbar, uint32_t rank,
                                               int warp, int lane, int nwarps) {
     if (lane == 0 && warp < nwarps)
@@ -139,80 +161,81 @@ __device__ __forceinline__ void push_to_peers(uint32_t src, uint32_t bytes, uint
                 tc::bulk_copy_to_peer(tc::map_rank(src, q), src, bytes, tc::map_rank(mbar, q));
 }
 
-// barrier over the first 12 warps (the sampling side); warps 12..15 may be issuing MMAs
-__device__ __forceinline__ void sync_sampling_warps() { asm volatile("bar.sync 1, 384;" ::: "memory"); }
+// barrier over the 16 compute warps (the MMA warp may still be issuing)
+__device__ __forceinline__ void sync_compute_warps() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
-__device__ __forceinline__ float fast_sigmoid(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
-__device__ __forceinline__ float fast_tanh(float x) { return 2.f * fast_sigmoid(2.f * x) - 1.f; }
+// Gate nonlinearities on the hardware tanh (one MUFU op each; relative error about
+// 2^-11, far inside the bf16 path's tolerance): sigmoid(x) = (1 + tanh(x/2)) / 2.
+__device__ __forceinline__ float fast_tanh(float x) {
+    float y;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float fast_sigmoid(float x) { return fmaf(0.5f, fast_tanh(0.5f * x), 0.5f); }
 
-// Thread roles.  row = 32*(warp%4) + lane is the episode (TMEM lane); grp = warp/4.
-//   gates: group g owns hidden units [4g, 4g+4) of this rank (its 16 MMA1 columns
-//          are i|f|g|o of those units); group 0 also owns the controller columns.
-//   heads: group i < ZD owns latent dim rank*ZD + i (its 16 MMA2 columns are the
-//          K logits, K means, K log-sigmas, then reward (group 0) / done (group 1)).
-//   MMA issue: thread 0 issues MMA2; thread 384 issues MMA1 (so the h part of the
-//          next step's MMA1 runs while the other warps sample).
 template <class S>
-__global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
-    static_assert(S::U == 4 * NGRP && S::ZD == 2 && 3 * S::KM + 1 <= 16, "fused thread mapping");
+__global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
+    constexpr int CL = S::CL, UG = S::UG, ZD = S::ZD, KM = S::KM;
     extern __shared__ __align__(1024) unsigned char smem[];
-    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in
-    __shared__ __align__(8) uint64_t mbar[5];
+    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in, 5 W_a/W2 buffer
+    __shared__ __align__(8) uint64_t mbar[6];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     __shared__ float s_done_logit[TILE];
 
     const Geo g = geometry<S>(p.Z, p.A, p.H);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int row = 32 * (warp & 3) + lane, grp = warp >> 2;
+    const bool mma_warp = warp == MMA_WARP;
+    const int row = 32 * (warp & 3) + lane, grp = mma_warp ? 0 : warp >> 2;
     const uint32_t rank = tc::cluster_rank();
     const int tile = blockIdx.x / CL;
     const int b = tile * TILE + row;
-    const bool live = b < p.B;
-    const int Z = p.Z, H = p.H, A = p.A, K1 = Z + H, KZ = S::KM * Z;
-    const int U = S::U, NG = S::NG;
+    const bool live = b < p.B && !mma_warp;
+    const int Z = p.Z, H = p.H, A = p.A, K1 = Z + H, KZ = KM * Z;
     const int W = (A + 31) >> 5;
-    const int u0 = 4 * grp;                   // first owned unit (within this rank)
-    const int dim = (int)rank * S::ZD + grp;  // owned latent dim (groups 0, 1)
-    const bool has_dim = grp < S::ZD;
-    const int MMA1_THREAD = 3 * TILE;         // warp 12, lane 0
+    const int u0 = UG * grp;               // first owned unit (within this rank)
+    const int dim = (int)rank * ZD + grp;  // owned latent dim (groups < ZD)
+    const bool has_dim = grp < ZD;
 
-    unsigned char *sW1 = smem + g.w1, *sW2 = smem + g.w2;
-    const __nv_bfloat16 *sWa = reinterpret_cast<const __nv_bfloat16 *>(smem + g.wa);
+    unsigned char *sW1 = smem + g.w1, *sBuf = smem + g.buf;
     const float *sB1 = reinterpret_cast<const float *>(smem + g.b1);
     const float *sB2 = reinterpret_cast<const float *>(smem + g.b2);
     unsigned char *sX = smem + g.x;
     uint64_t *part = reinterpret_cast<uint64_t *>(smem + g.part);
     uint16_t *zst = reinterpret_cast<uint16_t *>(smem + g.zst);
 
-    const uint32_t PART_BYTES = TILE * 8, H_BYTES = TILE * S::U * 2, Z_BYTES = TILE * 4;
+    const uint32_t PART_BYTES = TILE * 8, H_BYTES = TILE * S::U * 2, Z_BYTES = TILE * ZD * 2;
+    const uint32_t WA_BYTES = (uint32_t)A * S::WA_STRIDE, W2_BYTES = (uint32_t)S::N2 * H * 2;
     const uint32_t mb = tc::smem_u32(&mbar[0]);
-    const uint32_t MB_MMA1 = mb, MB_MMA2 = mb + 8, MB_PART = mb + 16, MB_H = mb + 24, MB_Z = mb + 32;
+    const uint32_t MB_MMA1 = mb, MB_MMA2 = mb + 8, MB_PART = mb + 16, MB_H = mb + 24, MB_Z = mb + 32,
+                   MB_W = mb + 40;
+    const unsigned char *img = p.img + rank * p.img_stride;
+    const uint32_t buf_u32 = tc::smem_u32(sBuf);
 
-    // ---- load this rank's weight image --------------------------------------
+    // ---- resident part of this rank's weight image (W1, biases) ---------------
     {
-        const uint4 *src = reinterpret_cast<const uint4 *>(p.img + rank * p.img_stride);
+        const uint4 *src = reinterpret_cast<const uint4 *>(img);
         uint4 *dst = reinterpret_cast<uint4 *>(smem);
-        for (size_t i = tid; i < g.img / 16; i += NT) dst[i] = src[i];
+        for (size_t i = tid; i < g.iwa / 16; i += NTHREADS) dst[i] = src[i];
     }
     // ---- initial operand tile and register state -----------------------------
-    float c[4], hs[4], zs = 0.f;
+    float c[UG], hs[UG], zs = 0.f;
     bool frozen = false;
     {
         const float *zsrc = p.teacher ? p.z_seq : p.z0;
-        for (int k0 = 8 * grp; k0 < Z; k0 += 8 * NGRP) {
+        for (int k0 = 8 * grp; k0 < Z && !mma_warp; k0 += 8 * NGRP) {
             float v[8];
             for (int j = 0; j < 8; ++j) v[j] = live ? zsrc[(size_t)b * Z + k0 + j] : 0.f;
             x_store8(sX, row, k0, v);
         }
-        for (int k0 = 8 * grp; k0 < H; k0 += 8 * NGRP) {
+        for (int k0 = 8 * grp; k0 < H && !mma_warp; k0 += 8 * NGRP) {
             float v[8];
             for (int j = 0; j < 8; ++j) v[j] = (live && p.h0) ? p.h0[(size_t)b * H + k0 + j] : 0.f;
             x_store8(sX, row, Z + k0, v);
         }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const size_t i = (size_t)b * H + rank * U + u0 + j;
+        for (int j = 0; j < UG; ++j) {
+            const size_t i = (size_t)b * H + rank * S::U + u0 + j;
             c[j] = (live && p.c0) ? p.c0[i] : 0.f;
             hs[j] = (live && p.h0) ? p.h0[i] : 0.f;
         }
@@ -220,12 +243,14 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
         frozen = live && p.done0 && p.done0[b] != 0;
     }
     if (tid == 0) {
-        for (int i = 0; i < 5; ++i) tc::mbar_init(mb + 8 * i, 1);
+        for (int i = 0; i < 6; ++i) tc::mbar_init(mb + 8 * i, 1);
         tc::fence_mbar_init();
-        // arm the exchange barriers for step 0
+        // arm the exchange barriers for step 0; start the first W_a load
         tc::mbar_arrive_expect_tx(MB_PART, (CL - 1) * PART_BYTES);
         tc::mbar_arrive_expect_tx(MB_H, (CL - 1) * H_BYTES);
         tc::mbar_arrive_expect_tx(MB_Z, (CL - 1) * Z_BYTES);
+        tc::mbar_arrive_expect_tx(MB_W, WA_BYTES);
+        tc::bulk_load_global(buf_u32, img + g.iwa, WA_BYTES, MB_W);
         s_abort = 0;
     }
     if (warp == 0) tc::tmem_alloc(tc::smem_u32(&tmem_base), 256);
@@ -236,17 +261,17 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
     const uint32_t tm = tmem_base;
     const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
     const uint32_t x_u32 = tc::smem_u32(sX);
-    const uint32_t w1_u32 = tc::smem_u32(sW1), w2_u32 = tc::smem_u32(sW2);
+    const uint32_t w1_u32 = tc::smem_u32(sW1);
     const uint32_t part_u32 = tc::smem_u32(part), zst_u32 = tc::smem_u32(zst);
 
     const uint32_t idesc1 = tc::idesc_bf16_f32(128, p.teacher ? S::NG : S::N1);
     const uint32_t idesc2 = tc::idesc_bf16_f32(128, S::N2);
     const uint32_t lboX = TILE * 16, lbo1 = S::N1 * 16, lbo2 = S::N2 * 16;
+    // descriptor start addresses advance by 2 core matrices along K: 2*lbo bytes (>> 4)
+    const uint64_t dX0 = tc::smem_desc(x_u32, lboX, 128), dW10 = tc::smem_desc(w1_u32, lbo1, 128);
+    const uint64_t dW20 = tc::smem_desc(buf_u32, lbo2, 128);
     // MMA1 over k-blocks [kb0, kb1) of 16: z part is [0, Z/16), h part [Z/16, K1/16).
     // Every step accumulates the h part first, then the z part.
-    // (descriptor start addresses advance by 2 core matrices along K: 2*lbo bytes, >> 4)
-    const uint64_t dX0 = tc::smem_desc(x_u32, lboX, 128), dW10 = tc::smem_desc(w1_u32, lbo1, 128);
-    const uint64_t dW20 = tc::smem_desc(w2_u32, lbo2, 128);
     auto mma1 = [&](int kb0, int kb1, bool acc_first) {
         uint64_t da = dX0 + (uint64_t)kb0 * (2 * lboX >> 4), db = dW10 + (uint64_t)kb0 * (2 * lbo1 >> 4);
         for (int kb = kb0; kb < kb1; ++kb) {
@@ -255,13 +280,18 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
             db += 2 * lbo1 >> 4;
         }
     };
-    auto wait_bar = [&](uint32_t bar, uint32_t parity) {
+    // bounded waits: wait_one by a single thread, wait_bar by whole warps
+    auto wait_one = [&](uint32_t bar, uint32_t parity) {
         if (!s_abort && !tc::mbar_wait_bounded(bar, parity, WAIT_POLLS)) {
             s_abort = 1;
             atomicExch(p.status, (int)WM_ERR_TIMEOUT);
         }
+    };
+    auto wait_bar = [&](uint32_t bar, uint32_t parity) {
+        wait_one(bar, parity);
         __syncwarp();
     };
+    const bool issuer = mma_warp && lane == 0;
 
     float nll_acc = 0.f;
     const int len = p.teacher ? (p.lengths ? min(max(p.lengths[live ? b : 0], 0), p.T) : p.T) : 0;
@@ -272,12 +302,13 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
     uint32_t mword = 0xFFFFFFFFu;
     if (!p.teacher && grp == 0 && p.mask && live && p.T > 0) mword = __ldg(p.mask + (size_t)b * W + (a0 >> 5));
 
-    if (tid == MMA1_THREAD) {  // MMA1 of step 0
+    if (issuer) {  // MMA1 of step 0
         tc::fence_after_sync();
         mma1(Z / 16, K1 / 16, false);
         mma1(0, Z / 16, true);
         tc::mma_commit(MB_MMA1);
     }
+    __syncwarp();  // the MMA warp reconverges before the next aligned barrier
 
     for (int t = 0; t < p.T; ++t) {
         const uint32_t step = p.t0 + (uint32_t)t;
@@ -286,22 +317,24 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
         const bool last = t + 1 == p.T;
 
         // ---------------- gates + controller pre-activations ------------------
-        wait_bar(MB_MMA1, parity);
-        tc::fence_after_sync();
-        float gv[16];
-        {
-            uint32_t r[16];
-            TC_LD16(tm + lane_base + 16 * grp, r);
+        float gv[4 * UG];
+        uint32_t rc[16];  // controller columns (group 0)
+        if (!mma_warp) {
+            wait_bar(MB_MMA1, parity);
+            tc::fence_after_sync();
+            uint32_t rg[4 * UG];
+            // all loads in flight before a single wait
+#pragma unroll
+            for (int c0 = 0; c0 < 4 * UG; c0 += 16) TC_LD16(tm + lane_base + 4 * UG * grp + c0, (rg + c0));
+            if (grp == 0 && !p.teacher) TC_LD16(tm + lane_base + S::NG, rc);
             tc::tmem_ld_wait();
 #pragma unroll
-            for (int j = 0; j < 16; ++j) gv[j] = __uint_as_float(r[j]);
+            for (int j = 0; j < 4 * UG; ++j) gv[j] = __uint_as_float(rg[j]);
         }
-        if (grp == 0) {
+        if (grp == 0 && !mma_warp) {
             uint64_t rec = 0xFFFFFFFF00000000ull;  // index -1: nothing valid here
             if (!p.teacher) {
-                uint32_t r[16];
-                TC_LD16(tm + lane_base + S::NG, r);
-                tc::tmem_ld_wait();
+                const uint32_t *r = rc;
                 // local masked argmax over this rank's actions (lowest index on ties)
                 float bv = -INFINITY;
                 int bi = -1;
@@ -321,12 +354,14 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
         tc::fence_proxy_async_smem();
         tc::fence_before_sync();
         __syncthreads();
-        push_to_peers(part_u32 + rank * PART_BYTES, PART_BYTES, MB_PART, rank, warp, lane, NT / 32);
+        push_to_peers<CL>(part_u32 + rank * PART_BYTES, PART_BYTES, MB_PART, rank, warp, lane, NT / 32);
+        float hn[UG];
+        int a = -1;
+        if (!mma_warp) {
         wait_bar(MB_PART, parity);
         if (tid == 0) tc::mbar_arrive_expect_tx(MB_PART, (CL - 1) * PART_BYTES);
 
         // ---------------- action (a2) ----------------------------------------
-        int a = -1;
         if (p.teacher) {
             if (live) {
                 a = p.act_in[tb];
@@ -343,35 +378,32 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
         }
         if (!p.teacher && rank == 0 && grp == 0 && live) p.actions[tb] = a;
 
-        // ---------------- LSTM cell (a3, a4): 4 units per thread --------------
-        float hn[4];
+        // ---------------- LSTM cell (a3, a4): UG units per thread -------------
+        wait_bar(MB_W, 0);  // W_a is in the buffer
         {
-            // W_a row of a_t: this group's 16 bf16 (i|f|g|o of 4 units) as two 16-byte loads
-            float wa[16];
-            if (a >= 0) {
-                const uint4 *src = reinterpret_cast<const uint4 *>(
-                    reinterpret_cast<const unsigned char *>(sWa) + (size_t)a * S::WA_STRIDE + 32 * grp);
-                const uint4 q0 = src[0], q1 = src[1];
-                const uint32_t wv[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+            const float *bb = sB1 + 4 * UG * grp;
+            const uint4 *src = reinterpret_cast<const uint4 *>(sBuf + (size_t)(a >= 0 ? a : 0) * S::WA_STRIDE +
+                                                               8 * UG * grp);
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&wv[j]);
-                    wa[2 * j] = __low2float(v2);
-                    wa[2 * j + 1] = __high2float(v2);
+            for (int q = 0; q < UG / 2; ++q) {  // 8 bf16 per 16-byte load
+                const uint4 w4 = src[q];
+                const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&wv[e]);
+                    const int col = 8 * q + 2 * e;
+                    const float w0 = a >= 0 ? __low2float(v2) : 0.f, w1 = a >= 0 ? __high2float(v2) : 0.f;
+                    gv[col] += bb[col] + w0;
+                    gv[col + 1] += bb[col + 1] + w1;
                 }
-            } else {
-#pragma unroll
-                for (int j = 0; j < 16; ++j) wa[j] = 0.f;
             }
-            const float *bb = sB1 + 16 * grp;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < UG; ++j) {
                 if (frozen) {
                     hn[j] = hs[j];
                     continue;
                 }
-                const float gi = gv[j] + bb[j] + wa[j], gf = gv[4 + j] + bb[4 + j] + wa[4 + j];
-                const float gg = gv[8 + j] + bb[8 + j] + wa[8 + j], go = gv[12 + j] + bb[12 + j] + wa[12 + j];
+                const float gi = gv[j], gf = gv[UG + j], gg = gv[2 * UG + j], go = gv[3 * UG + j];
                 c[j] = fast_sigmoid(gf) * c[j] + fast_sigmoid(gi) * fast_tanh(gg);
                 hn[j] = fast_sigmoid(go) * fast_tanh(c[j]);
                 hs[j] = hn[j];
@@ -379,115 +411,136 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
         }
         // h' (bf16) into this CTA's own tile; the rank's U/8 k-blocks are one contiguous block
         {
-            uint2 v;
-            v.x = pack_bf16x2(hn[0], hn[1]);
-            v.y = pack_bf16x2(hn[2], hn[3]);
-            *reinterpret_cast<uint2 *>(sX + tc::kmajor_offset(row, Z + rank * U + u0, TILE)) = v;
+            unsigned char *dst = sX + tc::kmajor_offset(row, Z + rank * S::U + u0, TILE);
+            uint32_t pk[UG / 2];
+#pragma unroll
+            for (int j = 0; j < UG / 2; ++j) pk[j] = pack_bf16x2(hn[2 * j], hn[2 * j + 1]);
+            if constexpr (UG == 4) {
+                *reinterpret_cast<uint2 *>(dst) = make_uint2(pk[0], pk[1]);
+            } else {
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            }
         }
+        }  // !mma_warp
         tc::fence_proxy_async_smem();
-        tc::fence_before_sync();
-        __syncthreads();
-        const uint32_t hblk = x_u32 + tc::kmajor_offset(0, Z + rank * U, TILE);
-        push_to_peers(hblk, H_BYTES, MB_H, rank, warp, lane, NT / 32);
-        if (live) {
-            const size_t o = tb * H + rank * U + u0;
-            if (p.h_seq)
-                for (int j = 0; j < 4; ++j) p.h_seq[o + j] = hs[j];
-            if (p.c_seq)
-                for (int j = 0; j < 4; ++j) p.c_seq[o + j] = c[j];
+        __syncthreads();  // every W_a read and h' write of this CTA is done
+        if (issuer) {      // W2 replaces W_a in the buffer while h' travels
+            tc::mbar_arrive_expect_tx(MB_W, W2_BYTES);
+            tc::bulk_load_global(buf_u32, img + g.iw2, W2_BYTES, MB_W);
         }
+        __syncwarp();
+        const uint32_t hblk = x_u32 + tc::kmajor_offset(0, Z + rank * S::U, TILE);
+        push_to_peers<CL>(hblk, H_BYTES, MB_H, rank, warp, lane, NT / 32);
+        if (live) {
+            const size_t o = tb * H + rank * S::U + u0;
+            if (p.h_seq)
+                for (int j = 0; j < UG; ++j) p.h_seq[o + j] = hs[j];
+            if (p.c_seq)
+                for (int j = 0; j < UG; ++j) p.c_seq[o + j] = c[j];
+        }
+        // this step's random numbers do not depend on the data: draw them while h' travels
+        float u_dim = 0.f, eps_dim = 0.f;
+        if (!mma_warp && has_dim && !p.teacher && !frozen && p.mdn_tau > 0.f) {
+            u_dim = uniform_for_dim(p.seed, ep, step, dim);
+            eps_dim = normal_for_dim(p.seed, ep, step, dim);
+        }
+
+        // ---------------- MMA2: heads (a5); then the h part of the next MMA1 ---
+        if (issuer) {
+            wait_one(MB_H, parity);  // h' of every rank is in X
+            wait_one(MB_W, 1);       // W2 is in the buffer
+            if (!s_abort) {
+                tc::fence_after_sync();
+                uint64_t da = dX0 + ((uint64_t)Z * 256u >> 4), db = dW20;  // X_h: Z/8 k-blocks in
+                for (int kb = 0; kb < H / 16; ++kb) {
+                    tc::mma_bf16(tm + D2_COL, da, db, idesc2, kb > 0);
+                    da += 2 * lboX >> 4;
+                    db += 2 * lbo2 >> 4;
+                }
+                tc::mma_commit(MB_MMA2);
+                // same issuing thread: runs after MMA2 and overlaps the sampling
+                if (!last) mma1(Z / 16, K1 / 16, false);
+            }
+            if (!last) {  // W_a back into the buffer once MMA2 has read W2
+                wait_one(MB_MMA2, parity);
+                tc::mbar_arrive_expect_tx(MB_W, WA_BYTES);
+                tc::bulk_load_global(buf_u32, img + g.iwa, WA_BYTES, MB_W);
+            }
+        }
+        __syncwarp();
+        float hv[16], zn = 0.f;
+        int kc = 0;
+        if (!mma_warp) {
         wait_bar(MB_H, parity);
         if (tid == 0) tc::mbar_arrive_expect_tx(MB_H, (CL - 1) * H_BYTES);
-
-        // ---------------- MMA2: heads (a5); the h part of the next MMA1 ------
-        if (tid == 0 && !s_abort) {
-            tc::fence_after_sync();
-            uint64_t da = dX0 + ((uint64_t)Z * 256u >> 4), db = dW20;  // X_h: Z/8 k-blocks in
-            for (int kb = 0; kb < H / 16; ++kb) {
-                tc::mma_bf16(tm + 128, da, db, idesc2, kb > 0);
-                da += 2 * lboX >> 4;
-                db += 2 * lbo2 >> 4;
-            }
-            tc::mma_commit(MB_MMA2);
-        }
         wait_bar(MB_MMA2, parity);
-        if (tid == MMA1_THREAD && !s_abort && !last) {
-            // the h part of the next step's MMA1 (h_{t+1} is in X) runs while warps 0..11 sample
-            tc::fence_after_sync();
-            mma1(Z / 16, K1 / 16, false);
-        }
         tc::fence_after_sync();
-        float hv[16];
         {
+            const int cg = has_dim ? grp : 0;
             uint32_t r[16];
-            TC_LD16(tm + 128 + lane_base + 16 * (has_dim ? grp : 0), r);
+            TC_LD16(tm + D2_COL + lane_base + 16 * cg, r);
             tc::tmem_ld_wait();
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] = __uint_as_float(r[j]) + sB2[16 * (has_dim ? grp : 0) + j];
+            for (int j = 0; j < 16; ++j) hv[j] = __uint_as_float(r[j]) + sB2[16 * cg + j];
         }
         // reward is column 15 of group 0, the done logit column 15 of group 1
         const float rew = hv[15];
 
         // ---------------- mixture sample / NLL (a6, a7, a9): one dim per thread
-        float zn = 0.f;
-        int kc = 0;
         if (has_dim) {
-            const float *lg = hv, *mu = hv + S::KM, *ls = hv + 2 * S::KM;
+            const float *lg = hv, *mu = hv + KM, *ls = hv + 2 * KM;
             if (p.teacher) {
                 const float x = live ? p.z_seq[((size_t)(t + 1) * p.B + b) * Z + dim] : 0.f;
                 float m = -INFINITY;
-                for (int k = 0; k < S::KM; ++k) m = fmaxf(m, lg[k]);
+                for (int k = 0; k < KM; ++k) m = fmaxf(m, lg[k]);
                 float s = 0.f;
-                for (int k = 0; k < S::KM; ++k) s += expf(lg[k] - m);
+                for (int k = 0; k < KM; ++k) s += expf(lg[k] - m);
                 const float lse = m + logf(s);
-                float lp[S::KM], tmax = -INFINITY;
-                for (int k = 0; k < S::KM; ++k) {
+                float lp[KM], tmax = -INFINITY;
+                for (int k = 0; k < KM; ++k) {
                     const float zsc = (x - mu[k]) * expf(-ls[k]);
                     lp[k] = (lg[k] - lse) - 0.5f * zsc * zsc - ls[k] - 0.91893853320467274178f;
                     tmax = fmaxf(tmax, lp[k]);
                 }
                 float acc = 0.f;
-                for (int k = 0; k < S::KM; ++k) acc += expf(lp[k] - tmax);
+                for (int k = 0; k < KM; ++k) acc += expf(lp[k] - tmax);
                 if (t < len) nll_acc += -(tmax + logf(acc));
                 zn = x;
             } else if (frozen) {
                 zn = zs;
             } else if (!(p.mdn_tau > 0.f)) {
-                for (int k = 1; k < S::KM; ++k) if (lg[k] > lg[kc]) kc = k;
+                for (int k = 1; k < KM; ++k) if (lg[k] > lg[kc]) kc = k;
                 zn = mu[kc];
             } else {
                 const float tau = p.mdn_tau;
                 float m = -INFINITY;
-                for (int k = 0; k < S::KM; ++k) m = fmaxf(m, lg[k] / tau);
-                float pk[S::KM], s = 0.f;
-                for (int k = 0; k < S::KM; ++k) { pk[k] = expf(lg[k] / tau - m); s += pk[k]; }
-                const float u = uniform_for_dim(p.seed, ep, step, dim);
-                kc = S::KM - 1;
+                const float itau = __fdividef(1.f, tau);
+                for (int k = 0; k < KM; ++k) m = fmaxf(m, lg[k] * itau);
+                float pk[KM], s = 0.f;
+                for (int k = 0; k < KM; ++k) { pk[k] = __expf(lg[k] * itau - m); s += pk[k]; }
+                const float u = u_dim, is = __fdividef(1.f, s);
+                kc = KM - 1;
                 float cum = 0.f;
-                for (int k = 0; k < S::KM - 1; ++k) {
-                    cum += pk[k] / s;
+                for (int k = 0; k < KM - 1; ++k) {
+                    cum += pk[k] * is;
                     if (u < cum) { kc = k; break; }
                 }
-                const float eps = normal_for_dim(p.seed, ep, step, dim);
                 const float scale = p.sigma_sqrt_tau ? sqrtf(tau) : 1.f;
-                zn = mu[kc] + expf(ls[kc]) * scale * eps;
+                zn = mu[kc] + __expf(ls[kc]) * scale * eps_dim;
             }
         }
         // ---------------- z' exchange, then the z part of the next MMA1 ------
         if (!p.teacher && has_dim) {
             __nv_bfloat16 zb = __float2bfloat16_rn(zn);
-            zst[(rank * TILE + row) * 2 + grp] = *reinterpret_cast<uint16_t *>(&zb);
+            zst[(rank * TILE + row) * ZD + grp] = *reinterpret_cast<uint16_t *>(&zb);
         }
         if (grp == 1) s_done_logit[row] = hv[15];
         tc::fence_proxy_async_smem();
         tc::fence_before_sync();
-        float dl = 0.f;
-        if (grp < 3) {
-            sync_sampling_warps();  // z' staged, done logit published
-            if (!last && !p.teacher)
-                push_to_peers(zst_u32 + rank * Z_BYTES, Z_BYTES, MB_Z, rank, warp, lane, 12);
-            dl = s_done_logit[row];
-        }
+        sync_compute_warps();  // z' staged, done logit published
+        if (!last && !p.teacher)
+            push_to_peers<CL>(zst_u32 + rank * Z_BYTES, Z_BYTES, MB_Z, rank, warp, lane, NT / 32);
+        const float dl = s_done_logit[row];
         // outputs of this step (overlap the exchange)
         if (live) {
             if (has_dim) {
@@ -498,10 +551,10 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
                 if (p.mdn_seq) {
                     float *ms = p.mdn_seq + tb * M;
                     const bool zero = frozen && !p.teacher;
-                    for (int k = 0; k < S::KM; ++k) {
-                        ms[dim * S::KM + k] = zero ? 0.f : hv[k];
-                        ms[KZ + dim * S::KM + k] = zero ? 0.f : hv[S::KM + k];
-                        ms[2 * KZ + dim * S::KM + k] = zero ? 0.f : hv[2 * S::KM + k];
+                    for (int k = 0; k < KM; ++k) {
+                        ms[dim * KM + k] = zero ? 0.f : hv[k];
+                        ms[KZ + dim * KM + k] = zero ? 0.f : hv[KM + k];
+                        ms[2 * KZ + dim * KM + k] = zero ? 0.f : hv[2 * KM + k];
                     }
                 }
             }
@@ -511,18 +564,25 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
                 if (grp == 1) p.done[tb] = (frozen || dl > 0.f || noop) ? 1 : 0;
             }
         }
+        }  // !mma_warp
         if (!last) {
-            if (!p.teacher) {
+            if (mma_warp) {
+            } else if (!p.teacher) {
                 wait_bar(MB_Z, parity);
                 if (tid == 0) tc::mbar_arrive_expect_tx(MB_Z, (CL - 1) * Z_BYTES);
-                // z' of all ranks -> this CTA's operand tile; group g packs k-block g
-                const uint32_t *zw = reinterpret_cast<const uint32_t *>(zst);
+                // z' of all ranks -> this CTA's operand tile; group g packs k-blocks g, g+4, ...
                 for (int k0 = 8 * grp; k0 < Z; k0 += 8 * NGRP) {
+                    uint16_t v[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const int d = k0 + j;
+                        v[j] = zst[((d / ZD) * TILE + row) * ZD + d % ZD];
+                    }
                     uint4 q;
-                    q.x = zw[(k0 / 2 + 0) * TILE + row];
-                    q.y = zw[(k0 / 2 + 1) * TILE + row];
-                    q.z = zw[(k0 / 2 + 2) * TILE + row];
-                    q.w = zw[(k0 / 2 + 3) * TILE + row];
+                    q.x = v[0] | ((uint32_t)v[1] << 16);
+                    q.y = v[2] | ((uint32_t)v[3] << 16);
+                    q.z = v[4] | ((uint32_t)v[5] << 16);
+                    q.w = v[6] | ((uint32_t)v[7] << 16);
                     *reinterpret_cast<uint4 *>(sX + tc::kmajor_offset(row, k0, TILE)) = q;
                 }
             } else {
@@ -536,13 +596,14 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
             tc::fence_proxy_async_smem();
             tc::fence_before_sync();
             __syncthreads();
-            if (tid == MMA1_THREAD && !s_abort) {
+            if (issuer && !s_abort) {
                 tc::fence_after_sync();
                 mma1(0, Z / 16, true);  // accumulate onto the h part issued after MMA2
                 tc::mma_commit(MB_MMA1);
             }
-            if (!p.teacher) {  // freezing (a8), now that every group can read the done logit
-                dl = s_done_logit[row];
+            __syncwarp();
+            if (!p.teacher && !mma_warp) {  // freezing (a8)
+                const float dl = s_done_logit[row];
                 if (!frozen) {
                     const bool noop = p.noop_terminates && a == A - 1;
                     if ((p.done_terminates && dl > 0.f) || noop) frozen = true;
@@ -553,19 +614,19 @@ __global__ void __launch_bounds__(NT, 1) k_fused(FusedParams p) {
     }
 
     if (live) {
-        const size_t o = (size_t)b * H + rank * U + u0;
+        const size_t o = (size_t)b * H + rank * S::U + u0;
         if (p.h_final)
-            for (int j = 0; j < 4; ++j) p.h_final[o + j] = hs[j];
+            for (int j = 0; j < UG; ++j) p.h_final[o + j] = hs[j];
         if (p.c_final)
-            for (int j = 0; j < 4; ++j) p.c_final[o + j] = c[j];
-        if (p.teacher && has_dim) p.nll_part[((size_t)rank * S::ZD + grp) * p.B + b] = nll_acc;
+            for (int j = 0; j < UG; ++j) p.c_final[o + j] = c[j];
+        if (p.teacher && has_dim) p.nll_part[(size_t)dim * p.B + b] = nll_acc;
     }
     tc::fence_before_sync();
     tc::cluster_sync();  // no CTA leaves while others may still write into it
     if (warp == 0) tc::tmem_dealloc(tm, 256);
 }
 
-// nll[n] = sum over the 32 (rank, dim) partials, in a fixed order.
+// nll[n] = sum over the Z per-dim partials, in dim order.
 __global__ void k_nll_reduce(int N, int parts, const float *part, float *nll) {
     const int n = blockIdx.x * blockDim.x + threadIdx.x;
     if (n >= N) return;
@@ -574,63 +635,51 @@ __global__ void k_nll_reduce(int N, int parts, const float *part, float *nll) {
     nll[n] = (float)s;
 }
 
-inline float bf16r(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+__global__ void k_copy_f32(size_t n, const float *src, float *dst) {
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+        dst[i] = src[i];
+}
+
+inline size_t host_kmajor(size_t r, size_t k, size_t R) {
+    return ((k >> 3) * (R >> 3) + (r >> 3)) * 128 + (r & 7) * 16 + (k & 7) * 2;
+}
+
+inline void put_bf16(unsigned char *base, size_t off, float v) {
+    __nv_bfloat16 q = __float2bfloat16_rn(v);
+    memcpy(base + off, &q, 2);
+}
 
 template <class S>
-bool shape_matches(const wm_config &c) {
-    return c.h_dim == CL * S::U && c.z_dim == CL * S::ZD && c.k_mix == S::KM;
+bool shape_fits(const wm_config &c) {
+    const int A = c.a_dim;
+    return c.h_dim == S::CL * S::U && c.z_dim == S::CL * S::ZD && c.k_mix == S::KM && A % S::CL == 0 &&
+           A / S::CL <= S::NA && 32 % (A / S::CL) == 0;  // a rank's actions sit in one mask word
 }
 
-}  // namespace
-
-// ---------------------------------------------------------------------------
-int wm_fused_supported(const wm_handle *h, int B) {
-    (void)B;
-    const wm_config &c = h->cfg;
-    if (!h->fused.ok) return 0;
-    if (c.ctrl_sample && c.ctrl_tau > 0.f) return 0;  // masked argmax only
-    return 1;
-}
-
-cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w) {
-    const wm_config &c = h->cfg;
-    h->fused.ok = 0;
-    if (c.precision != WM_BF16 || !shape_matches<S0>(c) || c.a_dim % CL != 0 || c.a_dim / CL > S0::NA ||
-        32 % (c.a_dim / CL) != 0)  // a rank's actions must sit in one mask word
-        return cudaSuccess;
-    using S = S0;
-    const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, K = c.k_mix, AC = A / CL, U = S::U;
+// Builds the per-rank weight images of shape S; returns the device buffer (or null).
+template <class S>
+void *pack_images(const wm_config &c, const wm_weights *w, size_t *img_bytes, cudaError_t *err) {
+    const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, K = c.k_mix, AC = A / S::CL, U = S::U, UG = S::UG;
     const size_t K1 = Z + H, M = (size_t)3 * K * Z;
     const Geo g = geometry<S>(Z, A, H);
-    int dev = 0, smem_optin = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    if ((size_t)smem_optin < g.smem + 64) return cudaSuccess;
-
-    std::vector<unsigned char> img(g.img * CL, 0);
-    auto put_bf16 = [&](unsigned char *base, size_t off, float v) {
-        __nv_bfloat16 q = __float2bfloat16_rn(v);
-        memcpy(base + off, &q, 2);
-    };
-    auto host_kmajor = [](size_t r, size_t k, size_t R) {
-        return ((k >> 3) * (R >> 3) + (r >> 3)) * 128 + (r & 7) * 16 + (k & 7) * 2;
-    };
-    for (int r = 0; r < CL; ++r) {
+    std::vector<unsigned char> img(g.img * S::CL, 0);
+    for (int r = 0; r < S::CL; ++r) {
         unsigned char *base = img.data() + (size_t)r * g.img;
         float *b1 = reinterpret_cast<float *>(base + g.b1);
         float *b2 = reinterpret_cast<float *>(base + g.b2);
-        // W1 rows: group gi (16 columns) = i|f|g|o of units 4gi..4gi+3, then the controller
+        // W1 rows: group gi (4*UG columns) = i|f|g|o of units UG*gi.., then the controller
         for (int n = 0; n < S::N1; ++n) {
             if (n < S::NG) {
-                const int gi = n / 16, within = n % 16, gate = within / 4, j = within % 4;
-                const size_t col = (size_t)gate * H + (size_t)r * U + 4 * gi + j;
+                const int gi = n / (4 * UG), within = n % (4 * UG), gate = within / UG, j = within % UG;
+                const size_t col = (size_t)gate * H + (size_t)r * U + UG * gi + j;
                 for (size_t k = 0; k < K1; ++k) {
                     const size_t src = k < (size_t)Z ? k : k + A;
                     put_bf16(base + g.w1, host_kmajor(n, k, S::N1), w->W_lstm[src * 4 * H + col]);
                 }
                 b1[n] = w->b_lstm[col];
                 for (int a = 0; a < A; ++a)
-                    put_bf16(base + g.wa, (size_t)a * S::WA_STRIDE + (size_t)n * 2, w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
+                    put_bf16(base + g.iwa, (size_t)a * S::WA_STRIDE + (size_t)n * 2,
+                             w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
             } else if (n - S::NG < AC) {
                 const size_t act = (size_t)r * AC + (n - S::NG);
                 for (size_t k = 0; k < K1; ++k)
@@ -651,7 +700,7 @@ cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w) {
                 col = (size_t)part * K * Z + (size_t)(r * S::ZD + i) * K + kk;
                 colsrc = w->W_mdn;
                 bias = w->b_mdn[col];
-            } else if (within == 15) {
+            } else if (within == 15 && i < 2) {
                 special = i == 0 ? 1 : 2;
                 bias = special == 1 ? w->b_rew : w->b_done;
             }
@@ -660,88 +709,139 @@ cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w) {
                 if (colsrc) v = colsrc[(size_t)k * M + col];
                 else if (special == 1) v = w->w_rew[k];
                 else if (special == 2) v = w->w_done[k];
-                put_bf16(base + g.w2, host_kmajor(n, k, S::N2), v);
+                put_bf16(base + g.iw2, host_kmajor(n, k, S::N2), v);
             }
             b2[n] = bias;
         }
     }
-    cudaError_t e = cudaMalloc(&h->fused.img, img.size());
-    if (e != cudaSuccess) return e;
-    e = cudaMemcpy(h->fused.img, img.data(), img.size(), cudaMemcpyHostToDevice);
-    if (e != cudaSuccess) return e;
-    h->fused.img_bytes = g.img;
-    e = cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        return cudaSuccess;  // the family stays unavailable; stepwise serves the model
+    void *d = nullptr;
+    *err = cudaMalloc(&d, img.size());
+    if (*err != cudaSuccess) return nullptr;
+    *err = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
+    if (*err != cudaSuccess) {
+        cudaFree(d);
+        return nullptr;
     }
-    // can one 16-CTA cluster of this size be resident at all?
+    *img_bytes = g.img;
+    return d;
+}
+
+// How many clusters of shape S can be resident at once (0 if none).
+template <class S>
+int max_clusters(const wm_config &c) {
+    const Geo g = geometry<S>(c.z_dim, c.a_dim, c.h_dim);
+    int dev = 0, optin = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if ((size_t)optin < g.smem + 2048) return 0;
+    if (cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem) != cudaSuccess ||
+        (S::CL > 8 && cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                          cudaSuccess)) {
+        cudaGetLastError();
+        return 0;
+    }
     cudaLaunchConfig_t lc = {};
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = CL;
+    at[0].val.clusterDim.x = S::CL;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
-    lc.gridDim = dim3(CL);
-    lc.blockDim = dim3(NT);
+    lc.gridDim = dim3(S::CL);
+    lc.blockDim = dim3(NTHREADS);
     lc.dynamicSmemBytes = g.smem;
     lc.attrs = at;
     lc.numAttrs = 1;
-    int nclusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&nclusters, k_fused<S>, &lc);
-    if (e != cudaSuccess || nclusters < 1) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_fused<S>, &lc) != cudaSuccess) {
         cudaGetLastError();
-        return cudaSuccess;
+        return 0;
     }
-    h->fused.cluster = CL;
-    h->fused.max_clusters = nclusters;
-    h->fused.ok = 1;
-    (void)bf16r;
-    return cudaSuccess;
+    return n;
 }
 
-void wm_fused_free(wm_handle *h) {
-    cudaFree(h->fused.img);
-    h->fused.img = nullptr;
-}
-
-static cudaError_t launch_fused(const wm_handle *h, FusedParams &p, cudaStream_t s) {
-    using S = S0;
+template <class S>
+cudaError_t launch_fused(const wm_handle *h, int slot, FusedParams &p, cudaStream_t s) {
     const Geo g = geometry<S>(p.Z, p.A, p.H);
     const int nclusters = (p.B + TILE - 1) / TILE;
     cudaLaunchConfig_t lc = {};
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = CL;
+    at[0].val.clusterDim.x = S::CL;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
-    lc.gridDim = dim3(nclusters * CL);
-    lc.blockDim = dim3(NT);
+    lc.gridDim = dim3(nclusters * S::CL);
+    lc.blockDim = dim3(NTHREADS);
     lc.dynamicSmemBytes = g.smem;
     lc.stream = s;
     lc.attrs = at;
     lc.numAttrs = 1;
-    p.img = (const unsigned char *)h->fused.img;
-    p.img_stride = h->fused.img_bytes;
+    p.img = (const unsigned char *)h->fused.img[slot];
+    p.img_stride = h->fused.img_bytes[slot];
+    p.AC = p.A / S::CL;
     p.status = h->status;
     return cudaLaunchKernelEx(&lc, k_fused<S>, p);
 }
 
-static FusedParams base(const wm_handle *h, int B, int T) {
+// slot 0: 16-CTA clusters, slot 1: 8-CTA clusters.  Fewer waves wins; ties go to 16.
+int choose_slot(const wm_handle *h, int B) {
+    const int tiles = (B + TILE - 1) / TILE;
+    const int m16 = h->fused.max_clusters[0], m8 = h->fused.max_clusters[1];
+    if (h->fused.force_cluster == 8 && m8 > 0) return 1;
+    if (h->fused.force_cluster == 16 && m16 > 0) return 0;
+    if (m16 <= 0) return 1;
+    if (m8 <= 0) return 0;
+    const int w16 = (tiles + m16 - 1) / m16, w8 = (tiles + m8 - 1) / m8;
+    return w8 < w16 ? 1 : 0;
+}
+
+cudaError_t launch_slot(const wm_handle *h, FusedParams &p, cudaStream_t s) {
+    return choose_slot(h, p.B) == 0 ? launch_fused<S16>(h, 0, p, s) : launch_fused<S8>(h, 1, p, s);
+}
+
+FusedParams base_params(const wm_handle *h, int B, int T) {
     const wm_config &c = h->cfg;
     FusedParams p{};
-    p.B = B; p.T = T; p.Z = c.z_dim; p.A = c.a_dim; p.H = c.h_dim; p.AC = c.a_dim / CL;
+    p.B = B; p.T = T; p.Z = c.z_dim; p.A = c.a_dim; p.H = c.h_dim;
     p.seed = c.seed; p.mdn_tau = c.mdn_tau; p.sigma_sqrt_tau = c.sigma_sqrt_tau;
     p.done_terminates = c.done_terminates; p.noop_terminates = c.noop_terminates;
     return p;
 }
 
-__global__ void k_copy_f32(size_t n, const float *src, float *dst) {
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
-        dst[i] = src[i];
+}  // namespace
+
+// ---------------------------------------------------------------------------
+int wm_fused_supported(const wm_handle *h, int B) {
+    (void)B;
+    const wm_config &c = h->cfg;
+    if (!h->fused.ok) return 0;
+    if (c.ctrl_sample && c.ctrl_tau > 0.f) return 0;  // masked argmax only
+    return 1;
 }
+
+cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w) {
+    const wm_config &c = h->cfg;
+    h->fused.ok = 0;
+    if (c.precision != WM_BF16 || !shape_fits<S16>(c) || !shape_fits<S8>(c)) return cudaSuccess;
+    h->fused.max_clusters[0] = max_clusters<S16>(c);
+    h->fused.max_clusters[1] = max_clusters<S8>(c);
+    if (h->fused.max_clusters[0] <= 0 && h->fused.max_clusters[1] <= 0) return cudaSuccess;
+    cudaError_t e = cudaSuccess;
+    h->fused.img[0] = pack_images<S16>(c, w, &h->fused.img_bytes[0], &e);
+    if (e != cudaSuccess) return e;
+    h->fused.img[1] = pack_images<S8>(c, w, &h->fused.img_bytes[1], &e);
+    if (e != cudaSuccess) return e;
+    h->fused.ok = 1;
+    return cudaSuccess;
+}
+
+void wm_fused_free(wm_handle *h) {
+    for (int i = 0; i < 2; ++i) {
+        cudaFree(h->fused.img[i]);
+        h->fused.img[i] = nullptr;
+    }
+}
+
+int wm_fused_cluster_size(const wm_handle *h, int B) { return choose_slot(h, B) == 0 ? S16::CL : S8::CL; }
 
 cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaStream_t s) {
     if (a.B == 0) { h->last_launches = 0; return cudaSuccess; }
@@ -762,19 +862,19 @@ cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaSt
         }
         return cudaGetLastError();
     }
-    FusedParams p = base(h, a.B, a.T);
+    FusedParams p = base_params(h, a.B, a.T);
     p.teacher = 0;
     p.ep0 = a.ep0; p.t0 = a.t0;
     p.z0 = a.z0; p.h0 = a.h0; p.c0 = a.c0; p.done0 = a.done0; p.mask = a.mask;
     p.z_out = a.z_out; p.actions = a.actions; p.rewards = a.rewards; p.done = a.done;
     p.h_final = a.h_final; p.c_final = a.c_final; p.h_seq = a.h_seq; p.c_seq = a.c_seq;
     p.mdn_seq = a.mdn_seq; p.comp_seq = a.comp_seq;
-    cudaError_t e = launch_fused(h, p, s);
+    cudaError_t e = launch_slot(h, p, s);
     h->last_launches = 2;
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-size_t wm_fused_nll_ws(const wm_handle *, int N) { return (size_t)CL * S0::ZD * N * 4 + 256; }
+size_t wm_fused_nll_ws(const wm_handle *h, int N) { return (size_t)h->cfg.z_dim * N * 4 + 256; }
 
 cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s) {
     if (a.N == 0) { h->last_launches = 0; return cudaSuccess; }
@@ -782,14 +882,14 @@ cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cuda
         h->last_launches = 0;
         return cudaMemsetAsync(a.nll, 0, (size_t)a.N * 4, s);
     }
-    FusedParams p = base(h, a.N, a.T);
+    FusedParams p = base_params(h, a.N, a.T);
     p.teacher = 1;
     p.z_seq = a.z_seq; p.act_in = a.actions; p.lengths = a.lengths;
     p.h_seq = a.h_seq; p.c_seq = a.c_seq; p.mdn_seq = a.mdn_seq;
     p.nll_part = (float *)ws;
-    cudaError_t e = launch_fused(h, p, s);
+    cudaError_t e = launch_slot(h, p, s);
     if (e != cudaSuccess) return e;
-    k_nll_reduce<<<(a.N + 127) / 128, 128, 0, s>>>(a.N, CL * S0::ZD, p.nll_part, a.nll);
+    k_nll_reduce<<<(a.N + 127) / 128, 128, 0, s>>>(a.N, h->cfg.z_dim, p.nll_part, a.nll);
     h->last_launches = 2;
     return cudaGetLastError();
 }

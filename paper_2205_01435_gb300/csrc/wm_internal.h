@@ -43,15 +43,14 @@ struct wm_step_weights {
     float *bh;   // [M+2]
 };
 
-// Weights of the fused single-launch family (bf16 tensor-core operand images).
+// Weights of the fused single-launch family: per cluster size (slot 0: 16 CTAs,
+// slot 1: 8 CTAs) one bf16 image per cluster rank, laid out as in wm_fused.cu.
 struct wm_fused_weights {
-    void *img;         // packed per-CTA shared-memory images, see wm_fused.cu
-    size_t img_bytes;
-    void *wa;          // action rows, bf16, [A, 4H] in the fused gate-column order
-    float *bias;       // fp32 biases in the fused column order
-    int ok;            // 1 if the model fits this family
-    int cluster;       // CTAs per cluster
-    int max_clusters;  // clusters of this size that can be resident at once
+    void *img[2];
+    size_t img_bytes[2];   // bytes per rank image
+    int max_clusters[2];   // clusters of that size that can be resident at once
+    int force_cluster;     // 0 = choose per call, else 8 or 16
+    int ok;                // 1 if the model fits this family
 };
 
 struct wm_handle {

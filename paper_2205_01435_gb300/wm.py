@@ -33,7 +33,8 @@ class wm_config(C.Structure):
     _fields_ = [("z_dim", C.c_int), ("a_dim", C.c_int), ("h_dim", C.c_int), ("k_mix", C.c_int),
                 ("precision", C.c_int), ("mdn_tau", C.c_float), ("sigma_sqrt_tau", C.c_int),
                 ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_float), ("done_terminates", C.c_int),
-                ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int)]
+                ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int),
+                ("fused_cluster", C.c_int)]
 
 
 class wm_weights(C.Structure):
@@ -111,7 +112,7 @@ def wm_create(cfg: dict, weights: dict):
                   int(cfg.get("done_terminates", 0)), int(cfg.get("noop_terminates", 0)),
                   int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF,
                   PATHS[cfg.get("path", "auto")] if isinstance(cfg.get("path", "auto"), str)
-                  else int(cfg["path"]))
+                  else int(cfg["path"]), int(cfg.get("fused_cluster", 0)))
     keep = {k: torch.as_tensor(weights[k], dtype=torch.float32).contiguous().cpu()
             for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl")}
     w = wm_weights(_ptr(keep["W_lstm"]), _ptr(keep["b_lstm"]), _ptr(keep["W_mdn"]),

@@ -262,11 +262,12 @@ def test_host_buffers_match_device_buffers(wm, kind):
 
 
 # ------------------------------------------------------------------ the fused single-launch family
+@pytest.mark.parametrize("cluster", [16, 8])
 @pytest.mark.parametrize("flags", [dict(), dict(done_terminates=1, noop_terminates=1),
                                    dict(mdn_tau=0.0), dict(mdn_tau=0.5, sigma_sqrt_tau=1)])
-def test_fused_against_oracle(wm, orc, flags):
+def test_fused_against_oracle(wm, orc, flags, cluster):
     """Two clusters (the second one partly filled), resumed state, offsets, flags."""
-    cfg = dict(synth.model_config("small_bf16"), **flags)
+    cfg = dict(synth.model_config("small_bf16"), fused_cluster=cluster, **flags)
     w = synth.weights(cfg, seed=5)
     B, T = 200, 9
     z0 = synth.z0(B, cfg["z_dim"], seed=5)
@@ -284,11 +285,12 @@ def test_fused_against_oracle(wm, orc, flags):
     o = orc.rollout(cfg, w, z0, mask, T, episode_offset=77, t0=3, h0=h0, c0=c0, done0=done0,
                     want_seq=True, nthreads=NT)
     r = check_rollout(g, o, cfg, weights=w, h0=h0)
-    print("fused", flags, r)
+    print("fused", cluster, flags, r)
 
 
-def test_fused_teacher_forced_ragged(wm, orc):
-    cfg = synth.model_config("small_bf16")
+@pytest.mark.parametrize("cluster", [16, 8])
+def test_fused_teacher_forced_ragged(wm, orc, cluster):
+    cfg = dict(synth.model_config("small_bf16"), fused_cluster=cluster)
     w = synth.weights(cfg, seed=6)
     zs, acts, lens = synth.teacher_inputs(300, 11, cfg["z_dim"], cfg["a_dim"], seed=6, ragged=True)
     acts[2, ::5] = -1
