@@ -78,7 +78,7 @@ def fp32_simt_peak_tflops() -> float:
 
 
 def kernel_source_sha(path_name: str) -> str:
-    src = {"fused": "wm_fused.cu", "stepwise": "wm_step.cu"}.get(path_name, "wm_step.cu")
+    src = {"fused": "wm_fused.cu", "stepwise": "wm_step.cu", "tensor": "wm_tensor.cu"}[path_name]
     with open(os.path.join(ROOT, "paper_2205_01435_gb300", "csrc", src), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
@@ -152,6 +152,38 @@ def dist_env():
     return ws, rank, local
 
 
+def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg):
+    """The same rollout through the C ABI with pinned HOST arrays: copies are timed."""
+    import torch
+    import torch.distributed as dist
+
+    env_steps = B * T * ws
+    zh = torch.from_numpy(z0).pin_memory()
+    mh = torch.from_numpy(mask).pin_memory()
+    hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
+            "actions": torch.empty((T, B), dtype=torch.int32, pin_memory=True),
+            "rewards": torch.empty((T, B), pin_memory=True),
+            "done": torch.empty((T, B), dtype=torch.uint8, pin_memory=True)}
+    for _ in range(2):
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+    torch.cuda.synchronize()
+    e2e_t = []
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_s = torch.tensor([sum(e2e_t) / len(e2e_t)], dtype=torch.float64, device=dev)
+    if ws > 1:
+        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
+    e2e_value = env_steps / float(e2e_s.item())
+    h2d = zh.numel() * 4 + mh.numel() * 4
+    d2h = sum(v.numel() * v.element_size() for v in hout.values())
+
+    return e2e_value, h2d, d2h
+
+
 def run_ours(args) -> None:
     import torch
     import torch.distributed as dist
@@ -213,34 +245,18 @@ def run_ours(args) -> None:
     value = env_steps / (ms_per_step / 1e3)
 
     # e2e: the same call through the C ABI with pinned HOST buffers, copies timed.
-    zh = torch.from_numpy(z0).pin_memory()
-    mh = torch.from_numpy(mask).pin_memory()
-    hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
-            "actions": torch.empty((T, B), dtype=torch.int32, pin_memory=True),
-            "rewards": torch.empty((T, B), pin_memory=True),
-            "done": torch.empty((T, B), dtype=torch.uint8, pin_memory=True)}
-    for _ in range(2):
-        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
-    torch.cuda.synchronize()
-    e2e_t = []
-    for i in range(args.steps):
-        flush.fill_(float(i))
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
-        e2e_t.append(time.perf_counter() - t0)
-    e2e_s = torch.tensor([sum(e2e_t) / len(e2e_t)], dtype=torch.float64, device=dev)
-    if ws > 1:
-        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
-    e2e_value = env_steps / float(e2e_s.item())
-    h2d = zh.numel() * 4 + mh.numel() * 4
-    d2h = sum(v.numel() * v.element_size() for v in hout.values())
+    if args.no_e2e:
+        e2e_value, h2d, d2h = None, 0, 0
+    else:
+        e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg)
 
     peaks = load_peaks()
     fl = flops_per_env_step(cfg) * B * T
-    if path_name == "fused":
-        kernel_key = f"wm_fused_rollout/{name}"
-        bound, peak, unit = "tensor", peaks["bf16_tflops"], "TFLOP/s"
+    if path_name in ("fused", "tensor"):
+        # fused: the call is one kernel; tensor: 3 GEMM kernels per step, counted together
+        kernel_key = f"wm_{path_name}_rollout/{name}"
+        bound, unit = "tensor", "TFLOP/s"
+        peak = peaks["bf16_tflops"] if path_name == "fused" else peaks["bf16_tflops_sustained"]
         achieved = fl / (ms_per_step / 1e3) / 1e12
     else:
         kernel_key = f"wm_step/{name}"
@@ -250,7 +266,8 @@ def run_ours(args) -> None:
     traffic = ncu_traffic(kernel_key, sha)
     roof = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
             "frac": round(achieved / peak, 5), "traffic": traffic,
-            "peak_source": peaks["source"] if bound == "tensor" else "derived: 152 SM x 128 FMA x 2.07 GHz",
+            "peak_source": (peaks["source"] + (" bf16 burst" if path_name == "fused" else " bf16 sustained"))
+            if bound == "tensor" else "derived: 152 SM x 128 FMA x 2.07 GHz",
             "kernel": kernel_key, "algorithmic_flops_per_launch": fl,
             "algorithmic_hbm_bytes_per_launch": bytes_per_env_step(cfg) * B * T + weight_bytes(cfg)}
 
@@ -265,8 +282,9 @@ def run_ours(args) -> None:
                        "precision": cfg["precision"], "kernel_path": path_name,
                        "l2": "flushed between timed steps (512 MiB write)",
                        "parallelism": f"episodes sharded over {ws} GPU(s), no collective"},
-            "e2e": {"value": round(e2e_value, 1), "unit": "env-steps/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": None if e2e_value is None else
+            {"value": round(e2e_value, 1), "unit": "env-steps/s",
+             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches * args.steps,
             "roofline": roof, "clocks": clk.summary()}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -278,11 +296,18 @@ def run_ours(args) -> None:
         dist.destroy_process_group()
 
 
-def cpu_baseline(name: str, episodes: int, threads: int | None = None) -> dict:
+def oracle_episodes(name: str, flop_budget: float) -> int:
+    """Episodes whose whole rollout costs about flop_budget algorithmic FLOPs (bounded sample)."""
+    w = synth.WORKLOADS[name]
+    per = flops_per_env_step(synth.model_config(name)) * w["T"]
+    return int(max(8, min(w["B"], flop_budget // per)))
+
+
+def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) -> dict:
     import oracle
 
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
-    n = min(episodes, B)
+    n = min(episodes or oracle_episodes(name, 2e11), B)
     threads = threads or os.cpu_count() or 1
     t0 = time.perf_counter()
     oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
@@ -300,7 +325,7 @@ def run_reference(args) -> None:
 
     name = args.workload
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
-    n = min(args.ref_episodes, B)
+    n = min(args.ref_episodes or oracle_episodes(name, 2e10), B)
     threads = os.cpu_count() or 1
     for _ in range(args.warmup):
         oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
@@ -335,10 +360,13 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="small_bf16",
                     choices=[k for k in synth.WORKLOADS if k != "nll"])
-    ap.add_argument("--path", choices=["auto", "stepwise", "fused"], default=None)
+    ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-episodes", type=int, default=1024)
-    ap.add_argument("--ref-episodes", type=int, default=96)
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer leg (profiling runs)")
+    ap.add_argument("--cpu-episodes", type=int, default=None,
+                    help="oracle sample size (default: about 2e11 FLOPs of the workload)")
+    ap.add_argument("--ref-episodes", type=int, default=None,
+                    help="oracle episodes per reference step (default: about 2e10 FLOPs)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -150,6 +150,17 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
     return upload(&h->step.bh, bh);
 }
 
+// AUTO: the fused single-launch family for batches that fit one wave of clusters,
+// the tensor-core family for large bf16 batches, the stepwise family otherwise.
+int pick_path(const wm_handle *h, int B) {
+    const int p = h->cfg.path;
+    if (p != WM_PATH_AUTO) return p;
+    if (wm_fused_supported(h, B) && B <= 2048) return WM_PATH_FUSED;
+    if (wm_tc_supported(h) && B >= 256) return WM_PATH_TENSOR;
+    if (wm_fused_supported(h, B)) return WM_PATH_FUSED;
+    return WM_PATH_STEPWISE;
+}
+
 }  // namespace
 
 extern "C" {
@@ -167,10 +178,12 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) 
     h->M = 3 * cfg->k_mix * cfg->z_dim;
     memset(&h->step, 0, sizeof(h->step));
     memset(&h->fused, 0, sizeof(h->fused));
+    memset(&h->tc, 0, sizeof(h->tc));
     cudaError_t e = cudaGetDevice(&h->device);
     if (e == cudaSuccess) e = pack_step(h, w);
     h->fused.force_cluster = cfg->fused_cluster;
     if (e == cudaSuccess) e = wm_fused_pack(h, w);
+    if (e == cudaSuccess) e = wm_tc_pack(h, w);
     if (e == cudaSuccess) e = cudaMalloc((void **)&h->status, sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, sizeof(int));
     if (e != cudaSuccess) {
@@ -195,6 +208,7 @@ void wm_destroy(wm_handle *h) {
     cudaFree(h->step.Wh);
     cudaFree(h->step.bh);
     wm_fused_free(h);
+    wm_tc_free(h);
     cudaFree(h->ws);
     cudaFree(h->stage);
     cudaFree(h->status);
@@ -258,19 +272,22 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true);
     st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true);
 
-    int path = c.path;
-    if (path == WM_PATH_AUTO) path = wm_fused_supported(h, B) ? WM_PATH_FUSED : WM_PATH_STEPWISE;
+    int path = pick_path(h, B);
     if (path == WM_PATH_FUSED && !wm_fused_supported(h, B))
         return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
-    if (path == WM_PATH_TENSOR) return fail(h, WM_ERR_UNSUPPORTED, "the tensor family is not built for rollouts");
+    if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
+        return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
 
-    if (path == WM_PATH_STEPWISE) {
-        e = grow(&h->ws, &h->ws_bytes, wm_step_rollout_ws(h, B));
+    size_t need = path == WM_PATH_STEPWISE ? wm_step_rollout_ws(h, B) : path == WM_PATH_TENSOR ? wm_tc_ws(h, B) : 0;
+    if (need) {
+        e = grow(&h->ws, &h->ws_bytes, need);
         if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
     }
     if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
     if (path == WM_PATH_FUSED)
         e = wm_fused_rollout(h, a, s);
+    else if (path == WM_PATH_TENSOR)
+        e = wm_tc_rollout(h, a, h->ws, s);
     else
         e = wm_step_rollout(h, a, h->ws, s);
     if (e != cudaSuccess) return cuda_fail(h, e, "rollout launch");
@@ -312,17 +329,20 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
     st.add((void **)&a.c_seq, c_seq, t * n * H * 4, true);
     st.add((void **)&a.mdn_seq, mdn_seq, t * n * M * 4, true);
 
-    int path = c.path;
-    if (path == WM_PATH_AUTO) path = wm_fused_supported(h, N) ? WM_PATH_FUSED : WM_PATH_STEPWISE;
+    int path = pick_path(h, N);
     if (path == WM_PATH_FUSED && !wm_fused_supported(h, N))
         return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
-    if (path == WM_PATH_TENSOR) return fail(h, WM_ERR_UNSUPPORTED, "the tensor family is not built for scoring");
-    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : wm_step_nll_ws(h, N);
+    if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
+        return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
+    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N)
+                                                                                      : wm_step_nll_ws(h, N);
     e = grow(&h->ws, &h->ws_bytes, need);
     if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
     if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
     if (path == WM_PATH_FUSED)
         e = wm_fused_nll(h, a, h->ws, s);
+    else if (path == WM_PATH_TENSOR)
+        e = wm_tc_nll(h, a, h->ws, s);
     else
         e = wm_step_nll(h, a, h->ws, s);
     if (e != cudaSuccess) return cuda_fail(h, e, "nll launch");

@@ -53,12 +53,22 @@ struct wm_fused_weights {
     int ok;                // 1 if the model fits this family
 };
 
+// Weights of the tensor-core family (bf16, K-major; orders in wm_tensor.cu).
+struct wm_tc_weights {
+    void *wc, *wg, *wa, *wh;  // W_c^T [A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
+    float *bc, *bg, *bh;
+    int dims_per_tile, n_head_tiles, rd_tile, rd_col;
+    int sms;
+    int ok;
+};
+
 struct wm_handle {
     wm_config cfg;
     int device;
     int M;                       // 3 K Z
     wm_step_weights step;
     wm_fused_weights fused;
+    wm_tc_weights tc;
     void *ws = nullptr;          // workspace (grows on demand)
     size_t ws_bytes = 0;
     void *stage = nullptr;       // staging for host arrays (grows on demand)
@@ -68,6 +78,14 @@ struct wm_handle {
     mutable int last_launches = 0;   // kernels launched by the last call
     std::string err;
 };
+
+// ---- tensor-core family (wm_tensor.cu) ----------------------------------------
+int wm_tc_supported(const wm_handle *h);
+size_t wm_tc_ws(const wm_handle *h, int B);
+cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w);
+void wm_tc_free(wm_handle *h);
+cudaError_t wm_tc_rollout(const wm_handle *h, const wm_rollout_dev &a, void *ws, cudaStream_t s);
+cudaError_t wm_tc_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s);
 
 // ---- stepwise family (wm_step.cu) -------------------------------------------
 size_t wm_step_rollout_ws(const wm_handle *h, int B);

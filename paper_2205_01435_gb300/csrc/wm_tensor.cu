@@ -1,0 +1,858 @@
+// wm_tensor.cu -- the tensor-core family for large batches: three persistent
+// tcgen05 GEMMs per dream step, each with the step's math fused into its epilogue.
+//
+//   controller  [B, Z+H] x W_c^T [A, Z+H]   -> masked argmax / tempered draw    (a1, a2)
+//   gates       [B, Z+H] x W_g^T [4H, Z+H]  -> + W_a[a_t] row, LSTM cell         (a3, a4)
+//   heads       [B, H]   x W_h^T [Nh, H]    -> mixture sample (or NLL), reward,
+//                                              done, freeze                       (a5..a9)
+//
+// Operands: bf16, K-major, loaded by TMA into 128-byte-swizzled shared-memory
+// tiles (box 64 K x rows), consumed by tcgen05.mma (cta_group::1, M = 128) with
+// fp32 accumulators in TMEM.  Each GEMM kernel is persistent (one CTA per SM,
+// tiles in N-fastest order so that concurrently running CTAs share the A rows in
+// L2) and warp-specialised:
+//   warp 0      TMA producer: a ring of STAGES (A, B) tiles guarded by full /
+//               empty mbarriers,
+//   warp 1      owns TMEM (512 columns) and issues the MMAs; accumulators are
+//               double-buffered when a tile is at most 256 columns wide, so the
+//               epilogue of one tile overlaps the MMAs of the next,
+//   warps 2..5  the epilogue: one thread per accumulator row (TMEM lane).
+// The operand X = [z_t | h_t] (bf16) is ping-ponged between two buffers: the
+// gate epilogue writes h_{t+1} and the head epilogue z_{t+1} into the other one.
+// The carried state c, h (fp32) lives in HBM.  All waits are bounded; on expiry a
+// kernel records WM_ERR_TIMEOUT and stops waiting.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <math.h>
+#include <string.h>
+
+#include <vector>
+
+#include "tc_ptx.cuh"
+#include "wm_device.cuh"
+#include "wm_internal.h"
+
+using namespace wmk;
+
+namespace {
+
+constexpr int BM = 128;          // rows per tile (MMA M)
+constexpr int BK = 64;           // K per stage: one 128-byte swizzle row of bf16
+constexpr int EPI_WARPS = 16;      // 4 per TMEM lane quadrant
+constexpr int GEMM_THREADS = 64 + 32 * EPI_WARPS;
+constexpr uint32_t POLLS = 1u << 26;
+constexpr int HEAD_TILE = 240;   // head columns per tile (a multiple of 16 and of 24)
+
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)1u << 16;            // leading byte offset: unused for swizzled K-major
+    d |= (uint64_t)(1024u >> 4) << 32;  // stride byte offset: 8 rows x 128 B
+    d |= (uint64_t)1u << 46;            // descriptor version
+    d |= (uint64_t)2u << 61;            // 128-byte swizzle
+    return d;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t mbar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        :: "r"(dst), "l"(map), "r"(x), "r"(y), "r"(mbar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t mbar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(mbar) : "memory");
+}
+
+// Gate nonlinearities from the fast exponential (relative error ~1e-6).
+__device__ __forceinline__ float sigmoid_hw(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+__device__ __forceinline__ float tanh_hw(float x) { return fmaf(2.f, sigmoid_hw(2.f * x), -1.f); }
+
+struct GemmGrid {
+    int m_tiles, n_tiles, k_steps;
+    int a_col0;   // first K column of A (the heads read X from column Z)
+    int *status;
+};
+
+// ---------------------------------------------------------------------------
+// Epilogue parameters (device pointers; one step)
+struct StepIO {
+    int B, Z, A, H, K, T, t;
+    uint32_t step;
+    unsigned long long ep0, seed;
+    int teacher, ctrl_sample, sigma_sqrt_tau, done_terminates, noop_terminates;
+    float ctrl_tau, mdn_tau;
+    // state
+    __nv_bfloat16 *x_cur, *x_next;  // [B, Z+H]
+    float *c, *h32;                 // [B, H]
+    int32_t *act;                   // [B] the step's action
+    const uint8_t *fz_cur;
+    uint8_t *fz_next;
+    // weights (packed orders, see wm_tc_pack)
+    const float *b_ctrl, *b_gate, *b_head;
+    const __nv_bfloat16 *wa;        // [A, 4H] gate-tile column order
+    // head tiles
+    int dims_per_tile, rd_tile, rd_col;  // reward / done columns: tile, first column
+    // inputs / outputs
+    const uint32_t *mask;           // [T, B, W] or null
+    const int32_t *act_in;          // teacher: [T, B]
+    const float *z_seq;             // teacher: [T+1, B, Z]
+    const int32_t *lengths;
+    float *z_out;                   // [T+1, B, Z]
+    int32_t *actions;
+    float *rewards;
+    uint8_t *done;
+    float *h_seq, *c_seq, *mdn_seq;
+    uint8_t *comp_seq;
+    float *nll_part;                // [n_head_tiles, B]
+};
+
+// Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
+// quadrant w%4) and owns column group cg = (w-2)/4 of the tile.  The 4 groups of a
+// quadrant cooperate through shared memory and a named barrier (ids 1..4).
+struct EpiCtx {
+    int quad, cg, lane, row;
+    float *red;  // [4 quad][4 group][32 lane][2] scratch for cross-group reductions
+    __device__ void sync() const { asm volatile("bar.sync %0, 128;" :: "r"(1 + quad) : "memory"); }
+    __device__ float *slot(int g) const { return red + ((quad * 4 + g) * 32 + lane) * 2; }
+};
+
+// ---- controller epilogue: A columns in TMEM, A/4 per column group ---------------
+// Every thread of a warp issues the same TMEM loads (they are warp-collective);
+// rows past B only skip their memory accesses.
+struct EpiCtrl {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+        (void)n;
+        const int b = m * BM + x.row;
+        const bool valid = b < p.B;
+        const int A = p.A, W = (A + 31) >> 5, CW = A / 4, c_lo = x.cg * CW;
+        const uint32_t *mw = (valid && p.mask) ? p.mask + ((size_t)p.t * p.B + b) * W : nullptr;
+        const bool live = valid && !p.fz_cur[b];
+        auto bits_at = [&](int c0) -> uint32_t { return mw ? (mw[c0 >> 5] >> (c0 & 31)) : 0xFFFFu; };
+        // pass 1: masked argmax over this group's columns (lowest index on ties)
+        int a = -1, last_v = -1;
+        float bv = -INFINITY;
+        for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
+            uint32_t r[16];
+            TC_LD16(tacc + c0, r);
+            tc::tmem_ld_wait();
+            const uint32_t bits = live ? bits_at(c0) : 0u;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                if (!((bits >> j) & 1u)) continue;
+                const float v = __uint_as_float(r[j]) + p.b_ctrl[c0 + j];
+                last_v = c0 + j;
+                if (a < 0 || v > bv) { bv = v; a = c0 + j; }
+            }
+        }
+        float *my = x.slot(x.cg);
+        my[0] = bv;
+        my[1] = __int_as_float(a);
+        x.sync();
+        int ga = -1;
+        float gbv = -INFINITY;
+        for (int g = 0; g < 4; ++g) {  // groups in column order: ties keep the lower index
+            const float *o = x.slot(g);
+            const int i = __float_as_int(o[1]);
+            if (i >= 0 && (ga < 0 || o[0] > gbv)) { gbv = o[0]; ga = i; }
+        }
+        if (p.ctrl_sample && p.ctrl_tau > 0.f) {  // uniform over the warp
+            const bool draw = live && ga >= 0;
+            const float itau = __fdividef(1.f, p.ctrl_tau);
+            float S = 0.f;
+            for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
+                uint32_t r[16];
+                TC_LD16(tacc + c0, r);
+                tc::tmem_ld_wait();
+                const uint32_t bits = draw ? bits_at(c0) : 0u;
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    if ((bits >> j) & 1u) S += __expf((__uint_as_float(r[j]) + p.b_ctrl[c0 + j] - gbv) * itau);
+            }
+            x.sync();  // everyone has read the argmax partials
+            my[0] = S;
+            my[1] = __int_as_float(last_v);
+            x.sync();
+            float total = 0.f, prefix = 0.f;
+            int glast = -1;
+            for (int g = 0; g < 4; ++g) {
+                const float *o = x.slot(g);
+                if (g < x.cg) prefix += o[0];
+                total += o[0];
+                glast = max(glast, __float_as_int(o[1]));
+            }
+            const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x) : 0.f;
+            const float target = u * total;
+            int chosen = -1;
+            float cum = prefix;
+            const bool mine = draw && target >= prefix && target < prefix + S;
+            for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
+                uint32_t r[16];
+                TC_LD16(tacc + c0, r);
+                tc::tmem_ld_wait();
+                const uint32_t bits = mine ? bits_at(c0) : 0u;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    if (!((bits >> j) & 1u) || chosen >= 0) continue;
+                    cum += __expf((__uint_as_float(r[j]) + p.b_ctrl[c0 + j] - gbv) * itau);
+                    if (target < cum) chosen = c0 + j;
+                }
+            }
+            x.sync();  // everyone has read the sum partials
+            my[1] = __int_as_float(chosen);
+            x.sync();
+            int pick = -1;
+            for (int g = 0; g < 4; ++g) pick = max(pick, __float_as_int(x.slot(g)[1]));
+            if (draw) ga = pick >= 0 ? pick : glast;  // rounding past the last valid action
+        }
+        x.sync();  // the scratch is reused by the next tile
+        if (!valid || x.cg != 0) return;
+        if (!live) ga = -1;
+        p.act[b] = ga;
+        p.actions[(size_t)p.t * p.B + b] = ga;
+    }
+};
+
+// ---- gate epilogue: 64 units per tile, columns [i | f | g | o] x 64; 16 units per group
+struct EpiGates {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+        const int b = m * BM + x.row;
+        const bool valid = b < p.B;
+        const int bb = valid ? b : 0;  // rows past B compute on row 0 and store nothing
+        const int H = p.H, KX = p.Z + p.H;
+        const bool fz = p.fz_cur[bb] != 0;
+        int a = p.act[bb];
+        if (p.teacher) {
+            a = p.act_in[(size_t)p.t * p.B + bb];
+            if (a < 0 || a >= p.A) a = -1;
+        }
+        const int q = x.cg;             // 16-unit chunk of the tile
+        const __nv_bfloat16 *war = a >= 0 ? p.wa + (size_t)a * 4 * H + 256 * n + 16 * q : nullptr;
+        const float *bg = p.b_gate + 256 * n + 16 * q;
+        for (int half = 0; half < 2; ++half) {  // 8 units at a time keeps the registers in bounds
+            const int j0 = 8 * half, u0 = 64 * n + 16 * q + j0;
+            uint32_t r[4][8];
+#pragma unroll
+            for (int gate = 0; gate < 4; ++gate) TC_LD8(tacc + 64 * gate + 16 * q + j0, r[gate]);
+            tc::tmem_ld_wait();
+            float4 *c4 = reinterpret_cast<float4 *>(p.c + (size_t)bb * H + u0);
+            float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)bb * H + u0);
+            float cv[8], hv[8];
+            if (fz) {
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const float4 cc = c4[k], hh = h4[k];
+                    cv[4 * k] = cc.x; cv[4 * k + 1] = cc.y; cv[4 * k + 2] = cc.z; cv[4 * k + 3] = cc.w;
+                    hv[4 * k] = hh.x; hv[4 * k + 1] = hh.y; hv[4 * k + 2] = hh.z; hv[4 * k + 3] = hh.w;
+                }
+            } else {
+                float gv[4][8];
+#pragma unroll
+                for (int gate = 0; gate < 4; ++gate) {
+                    float w8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                    if (war) {
+                        const uint4 w4 = *reinterpret_cast<const uint4 *>(war + 64 * gate + j0);
+                        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&wv[e]);
+                            w8[2 * e] = __low2float(v2);
+                            w8[2 * e + 1] = __high2float(v2);
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        gv[gate][j] = __uint_as_float(r[gate][j]) + bg[64 * gate + j0 + j] + w8[j];
+                }
+                const float4 ca = c4[0], cb = c4[1];
+                const float cold[8] = {ca.x, ca.y, ca.z, ca.w, cb.x, cb.y, cb.z, cb.w};
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float cn = sigmoid_hw(gv[1][j]) * cold[j] + sigmoid_hw(gv[0][j]) * tanh_hw(gv[2][j]);
+                    cv[j] = cn;
+                    hv[j] = sigmoid_hw(gv[3][j]) * tanh_hw(cn);
+                }
+                if (valid) {
+                    c4[0] = make_float4(cv[0], cv[1], cv[2], cv[3]);
+                    c4[1] = make_float4(cv[4], cv[5], cv[6], cv[7]);
+                    h4[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
+                    h4[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
+                }
+            }
+            if (!valid) continue;
+            uint32_t pk[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                __nv_bfloat162 v = __floats2bfloat162_rn(hv[2 * j], hv[2 * j + 1]);
+                pk[j] = *reinterpret_cast<uint32_t *>(&v);
+            }
+            *reinterpret_cast<uint4 *>(p.x_next + (size_t)b * KX + p.Z + u0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            const size_t o = ((size_t)p.t * p.B + b) * H + u0;
+            if (p.h_seq)
+                for (int j = 0; j < 8; ++j) p.h_seq[o + j] = hv[j];
+            if (p.c_seq)
+                for (int j = 0; j < 8; ++j) p.c_seq[o + j] = cv[j];
+        }
+    }
+};
+
+// ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
+struct EpiHeads {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+        const int b0 = m * BM + x.row;
+        const bool valid = b0 < p.B;
+        const int b = valid ? b0 : 0;  // rows past B compute on row 0 and store nothing
+        const int Z = p.Z, K = p.K, KZ = K * Z, M = 3 * KZ, KX = Z + p.H;
+        const int DS = (3 * K + 7) & ~7;  // columns per latent dim (8-aligned TMEM loads)
+        const bool fz = p.fz_cur[b] != 0;
+        const size_t tb = (size_t)p.t * p.B + b;
+        const unsigned long long ep = p.ep0 + b;
+        const int d0 = n * p.dims_per_tile;
+        const int nd = min(p.dims_per_tile, Z - d0);
+        const int per = (nd + 3) / 4;  // dims per column group, contiguous
+        const int i_lo = min(nd, x.cg * per), i_hi = min(nd, i_lo + per);
+        const float *bh = p.b_head + (size_t)n * HEAD_TILE;
+        float nll = 0.f;
+        u32x4 ru = {0, 0, 0, 0}, rn = {0, 0, 0, 0};
+        int rblock = -1;
+        for (int i = i_lo; i < i_hi; ++i) {
+            const int d = d0 + i;
+            float v[24];
+            {
+                uint32_t r0[8], r1[8], r2[8];
+                TC_LD8(tacc + DS * i, r0);
+                TC_LD8(tacc + DS * i + 8, r1);
+                TC_LD8(tacc + DS * i + 16, r2);  // past the dim when 3K <= 16: unused
+                tc::tmem_ld_wait();
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    v[j] = __uint_as_float(r0[j]);
+                    v[8 + j] = __uint_as_float(r1[j]);
+                    v[16 + j] = __uint_as_float(r2[j]);
+                }
+            }
+            float lg[8], mu[8], ls[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                if (k < K) {
+                    lg[k] = v[k] + bh[DS * i + k];
+                    mu[k] = v[K + k] + bh[DS * i + K + k];
+                    ls[k] = v[2 * K + k] + bh[DS * i + 2 * K + k];
+                }
+            }
+            if (!valid) continue;
+            if (p.mdn_seq) {
+                float *ms = p.mdn_seq + tb * M;
+                const bool zero = fz && !p.teacher;
+                for (int k = 0; k < K; ++k) {
+                    ms[d * K + k] = zero ? 0.f : lg[k];
+                    ms[KZ + d * K + k] = zero ? 0.f : mu[k];
+                    ms[2 * KZ + d * K + k] = zero ? 0.f : ls[k];
+                }
+            }
+            float zn;
+            if (p.teacher) {
+                const float xv = p.z_seq[((size_t)(p.t + 1) * p.B + b) * Z + d];
+                float mx = -INFINITY;
+                for (int k = 0; k < K; ++k) mx = fmaxf(mx, lg[k]);
+                float s = 0.f;
+                for (int k = 0; k < K; ++k) s += expf(lg[k] - mx);
+                const float lse = mx + logf(s);
+                float lp[8], tmax = -INFINITY;
+                for (int k = 0; k < K; ++k) {
+                    const float zs = (xv - mu[k]) * expf(-ls[k]);
+                    lp[k] = (lg[k] - lse) - 0.5f * zs * zs - ls[k] - 0.91893853320467274178f;
+                    tmax = fmaxf(tmax, lp[k]);
+                }
+                float acc = 0.f;
+                for (int k = 0; k < K; ++k) acc += expf(lp[k] - tmax);
+                nll += -(tmax + logf(acc));
+                zn = xv;
+            } else if (fz) {
+                zn = p.z_out[tb * Z + d];
+                if (p.comp_seq) p.comp_seq[tb * Z + d] = 255;
+            } else {
+                int kc = 0;
+                if (!(p.mdn_tau > 0.f)) {
+                    for (int k = 1; k < K; ++k) if (lg[k] > lg[kc]) kc = k;
+                    zn = mu[kc];
+                } else {
+                    if ((d >> 2) != rblock) {
+                        rblock = d >> 2;
+                        ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)rblock);
+                        rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)rblock);
+                    }
+                    const float itau = __fdividef(1.f, p.mdn_tau);
+                    float mx = -INFINITY;
+                    for (int k = 0; k < K; ++k) mx = fmaxf(mx, lg[k] * itau);
+                    float pk[8], s = 0.f;
+                    for (int k = 0; k < K; ++k) { pk[k] = __expf(lg[k] * itau - mx); s += pk[k]; }
+                    const float u = to_uniform(u32x4_get(ru, d & 3)), is = __fdividef(1.f, s);
+                    kc = K - 1;
+                    float cum = 0.f;
+                    for (int k = 0; k < K - 1; ++k) {
+                        cum += pk[k] * is;
+                        if (u < cum) { kc = k; break; }
+                    }
+                    const int pair = (d & 3) >> 1;
+                    const float eps = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
+                    const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
+                    zn = mu[kc] + __expf(ls[kc]) * scale * eps;
+                }
+                if (p.comp_seq) p.comp_seq[tb * Z + d] = (uint8_t)kc;
+            }
+            if (!p.teacher) p.z_out[(tb + p.B) * Z + d] = zn;
+            p.x_next[(size_t)b * KX + d] = __float2bfloat16_rn(zn);
+        }
+        if (p.teacher && valid) {
+            const int len = p.lengths ? p.lengths[b] : p.T;
+            if (p.t < len) p.nll_part[((size_t)n * 4 + x.cg) * p.B + b] += nll;
+        }
+        if (n == p.rd_tile) {
+            uint32_t r[2];
+            asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
+                         : "=r"(r[0]), "=r"(r[1]) : "r"(tacc + p.rd_col));
+            tc::tmem_ld_wait();
+            if (!p.teacher && valid && x.cg == 0) {
+                const float rew = __uint_as_float(r[0]) + bh[p.rd_col];
+                const float dl = __uint_as_float(r[1]) + bh[p.rd_col + 1];
+                const int a = p.act[b];
+                const bool noop = p.noop_terminates && a == p.A - 1;
+                p.rewards[tb] = fz ? 0.f : rew;
+                p.done[tb] = (fz || dl > 0.f || noop) ? 1 : 0;
+                p.fz_next[b] = (fz || (p.done_terminates && dl > 0.f) || noop) ? 1 : 0;
+            }
+        }
+    }
+};
+
+// ---------------------------------------------------------------------------
+// The persistent warp-specialised GEMM.  TILE_N = BN * NSUB columns per tile.
+template <int BN, int NSUB, int STAGES, class Epi>
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmGrid g,
+              StepIO io) {
+    constexpr int TILE_N = BN * NSUB;
+    constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BN * BK * 2, B_BYTES = B_SUB * NSUB;
+    constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    constexpr int NACC = TILE_N <= 256 ? 2 : 1;
+    constexpr uint32_t ACC_COLS = 256;
+    static_assert(BN % 16 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2];
+    __shared__ uint32_t tmem_base;
+    __shared__ int s_abort;
+    __shared__ float epi_red[4 * 4 * 32 * 2];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t smem_u = tc::smem_u32(smem);
+    auto full_b = [&](int s) { return tc::smem_u32(&bar_full[s]); };
+    auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            tc::mbar_init(full_b(s), 1);
+            tc::mbar_init(empty_b(s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            tc::mbar_init(tc::smem_u32(&bar_accf[a]), 1);
+            tc::mbar_init(tc::smem_u32(&bar_acce[a]), EPI_WARPS * 32);
+        }
+        tc::fence_mbar_init();
+        s_abort = 0;
+    }
+    if (warp == 1) tc::tmem_alloc(tc::smem_u32(&tmem_base), 512);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tm = tmem_base;
+    const int ntiles = g.m_tiles * g.n_tiles;
+    auto wait = [&](uint32_t bar, uint32_t parity) {
+        if (!s_abort && !tc::mbar_wait_bounded(bar, parity, POLLS)) {
+            s_abort = 1;
+            atomicExch(g.status, (int)WM_ERR_TIMEOUT);
+        }
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {  // ---- TMA producer
+            int stage = 0;
+            uint32_t phase = 0;
+            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+                const int m = tile / g.n_tiles, n = tile % g.n_tiles;
+                for (int ks = 0; ks < g.k_steps; ++ks) {
+                    wait(empty_b(stage), phase ^ 1u);
+                    if (s_abort) break;
+                    const uint32_t sa = smem_u + stage * STAGE_BYTES;
+                    tc::mbar_arrive_expect_tx(full_b(stage), STAGE_BYTES);
+                    tma_load_2d(sa, &tmA, g.a_col0 + ks * BK, m * BM, full_b(stage));
+#pragma unroll
+                    for (int s = 0; s < NSUB; ++s)
+                        tma_load_2d(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN, full_b(stage));
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // ---- MMA issuer
+            int stage = 0, acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            const uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+                wait(tc::smem_u32(&bar_acce[acc]), acc_phase ^ 1u);
+                tc::fence_after_sync();
+                const uint32_t dcol = tm + acc * ACC_COLS;
+                for (int ks = 0; ks < g.k_steps; ++ks) {
+                    wait(full_b(stage), phase);
+                    if (s_abort) break;
+                    tc::fence_after_sync();
+                    const uint32_t sa = smem_u + stage * STAGE_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t da = desc_sw128(sa + 32 * kk);
+#pragma unroll
+                        for (int s = 0; s < NSUB; ++s)
+                            tc::mma_bf16(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
+                                         (ks > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc::mma_commit(empty_b(stage));  // the stage is free once these MMAs are done
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+                tc::mma_commit(tc::smem_u32(&bar_accf[acc]));
+                if (NACC == 2) {
+                    acc ^= 1;
+                    if (acc == 0) acc_phase ^= 1u;
+                } else {
+                    acc_phase ^= 1u;
+                }
+            }
+        }
+    } else {  // ---- epilogue warps 2..17: 4 column groups per TMEM lane quadrant
+        const int quad = warp & 3;
+        EpiCtx x{quad, (warp - 2) >> 2, lane, 32 * quad + lane, epi_red};
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+            const int m = tile / g.n_tiles, n = tile % g.n_tiles;
+            wait(tc::smem_u32(&bar_accf[acc]), acc_phase);
+            __syncwarp();
+            tc::fence_after_sync();
+            const uint32_t tacc = tm + ((uint32_t)(32 * quad) << 16) + acc * ACC_COLS;
+            // always run: the epilogues use per-quadrant named barriers, so every thread of a
+            // quadrant must take the same path (after an abort the results are just unused)
+            Epi::run(io, tacc, m, n, x);
+            __syncwarp();
+            tc::fence_before_sync();
+            mbar_arrive(tc::smem_u32(&bar_acce[acc]));
+            if (NACC == 2) {
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1u;
+            } else {
+                acc_phase ^= 1u;
+            }
+        }
+    }
+    __syncwarp();
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 1) tc::tmem_dealloc(tm, 512);
+}
+
+// ---------------------------------------------------------------------------
+__global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const float *c0, const uint8_t *done0,
+                          __nv_bfloat16 *x0, uint8_t *fz0, uint8_t *fz1, int n_head_tiles) {
+    const int KX = p.Z + p.H;
+    const size_t nx = (size_t)p.B * KX;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nx; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t b = i / KX, k = i % KX;
+        float v;
+        if (k < (size_t)p.Z) v = p.teacher ? p.z_seq[b * p.Z + k] : z0[b * p.Z + k];
+        else v = h0 ? h0[b * p.H + (k - p.Z)] : 0.f;
+        x0[i] = __float2bfloat16_rn(v);
+        if (k >= (size_t)p.Z) {
+            const size_t j = b * p.H + (k - p.Z);
+            p.h32[j] = h0 ? h0[j] : 0.f;
+            p.c[j] = c0 ? c0[j] : 0.f;
+        } else if (!p.teacher) {
+            p.z_out[b * p.Z + k] = z0[b * p.Z + k];
+        }
+    }
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)p.B; i += (size_t)gridDim.x * blockDim.x) {
+        fz0[i] = fz1[i] = done0 ? (done0[i] != 0) : 0;
+        if (p.teacher)
+            for (int t = 0; t < 4 * n_head_tiles; ++t) p.nll_part[(size_t)t * p.B + i] = 0.f;
+    }
+}
+
+__global__ void k_tc_finish(int B, int H, const float *h32, const float *c, float *h_final, float *c_final,
+                            const float *nll_part, int n_parts, float *nll) {
+    const size_t n = (size_t)B * H;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+        if (h_final) h_final[i] = h32[i];
+        if (c_final) c_final[i] = c[i];
+    }
+    if (nll)
+        for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)B; i += (size_t)gridDim.x * blockDim.x) {
+            double s = 0.0;
+            for (int t = 0; t < n_parts; ++t) s += (double)nll_part[(size_t)t * B + i];
+            nll[i] = (float)s;
+        }
+}
+
+// ---------------------------------------------------------------------------
+typedef CUresult (*encode_fn_t)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+encode_fn_t get_encode() {
+    static encode_fn_t fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            fn = (encode_fn_t)p;
+    }
+    return fn;
+}
+
+// 2-D bf16 map over a row-major [rows, cols] matrix, box = 64 columns x box_rows, 128B swizzle.
+bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    encode_fn_t enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {cols, rows}, strides[1] = {cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows}, es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int NSUB, int STAGES, class Epi>
+size_t gemm_smem() {
+    return 1024 + (size_t)STAGES * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2);
+}
+
+template <int BN, int NSUB, int STAGES, class Epi>
+cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, GemmGrid g, const StepIO &io, int sms,
+                        cudaStream_t s) {
+    const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi>();
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN, NSUB, STAGES, Epi>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    const int tiles = g.m_tiles * g.n_tiles;
+    const int grid = tiles < sms ? tiles : sms;
+    k_tc_gemm<BN, NSUB, STAGES, Epi><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, g, io);
+    return cudaGetLastError();
+}
+
+inline size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+struct TcWs {
+    __nv_bfloat16 *x[2];
+    float *c, *h32, *nll_part;
+    int32_t *act;
+    uint8_t *fz[2];
+};
+
+TcWs carve_ws(const wm_handle *h, int B, void *ws) {
+    const wm_config &c = h->cfg;
+    const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
+    char *p = (char *)ws;
+    TcWs w{};
+    for (int i = 0; i < 2; ++i) { w.x[i] = (__nv_bfloat16 *)p; p += a256((size_t)B * KX * 2); }
+    w.c = (float *)p; p += a256((size_t)B * H * 4);
+    w.h32 = (float *)p; p += a256((size_t)B * H * 4);
+    w.act = (int32_t *)p; p += a256((size_t)B * 4);
+    for (int i = 0; i < 2; ++i) { w.fz[i] = (uint8_t *)p; p += a256((size_t)B); }
+    w.nll_part = (float *)p;
+    return w;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Host side: packing, support test, per-call orchestration.
+
+int wm_tc_supported(const wm_handle *h) { return h->tc.ok; }
+
+size_t wm_tc_ws(const wm_handle *h, int B) {
+    const wm_config &c = h->cfg;
+    const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
+    return 2 * a256((size_t)B * KX * 2) + 2 * a256((size_t)B * H * 4) + a256((size_t)B * 4) + 2 * a256(B) +
+           a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256;
+}
+
+cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
+    const wm_config &c = h->cfg;
+    wm_tc_weights &T = h->tc;
+    memset(&T, 0, sizeof(T));
+    const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, K = c.k_mix, KX = Z + H;
+    if (c.precision != WM_BF16 || H % 64 != 0 || A % 64 != 0 || (A > 256 && A != 512) || K > 8 || Z % 8 != 0 ||
+        !get_encode())
+        return cudaSuccess;
+    const int DS = (3 * K + 7) & ~7;  // head columns per latent dim
+    const int dpt = HEAD_TILE / DS;
+    int nht = (Z + dpt - 1) / dpt;
+    const int last_dims = Z - (nht - 1) * dpt;
+    int rd_tile = nht - 1, rd_col = DS * last_dims;
+    if (rd_col + 2 > HEAD_TILE) {  // reward / done get a tile of their own
+        rd_tile = nht;
+        rd_col = 0;
+        ++nht;
+    }
+    T.dims_per_tile = dpt;
+    T.n_head_tiles = nht;
+    T.rd_tile = rd_tile;
+    T.rd_col = rd_col;
+    auto bf = [](float v) { return __float2bfloat16_rn(v); };
+    // controller: W_c^T [A, KX]
+    std::vector<__nv_bfloat16> wc((size_t)A * KX), wg((size_t)4 * H * KX), wa((size_t)A * 4 * H),
+        wh((size_t)nht * HEAD_TILE * H, bf(0.f));
+    std::vector<float> bc(A), bg(4 * H), bh((size_t)nht * HEAD_TILE, 0.f);
+    for (int a = 0; a < A; ++a) {
+        for (int k = 0; k < KX; ++k) wc[(size_t)a * KX + k] = bf(w->W_ctrl[(size_t)k * A + a]);
+        bc[a] = w->b_ctrl[a];
+    }
+    // gates: row n = 256*j + 64*gate + u  <->  canonical column gate*H + 64*j + u
+    for (int n = 0; n < 4 * H; ++n) {
+        const int j = n / 256, gate = (n % 256) / 64, u = n % 64;
+        const size_t col = (size_t)gate * H + 64 * j + u;
+        for (int k = 0; k < KX; ++k) {
+            const size_t src = k < Z ? k : k + A;
+            wg[(size_t)n * KX + k] = bf(w->W_lstm[src * 4 * H + col]);
+        }
+        bg[n] = w->b_lstm[col];
+        for (int a = 0; a < A; ++a) wa[(size_t)a * 4 * H + n] = bf(w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
+    }
+    // heads: tile j, local dim i, part p, component k -> row j*240 + 3K*i + K*p + k
+    const size_t M = (size_t)3 * K * Z;
+    for (int d = 0; d < Z; ++d)
+        for (int part = 0; part < 3; ++part)
+            for (int k = 0; k < K; ++k) {
+                const size_t row = (size_t)(d / dpt) * HEAD_TILE + DS * (d % dpt) + K * part + k;
+                const size_t col = (size_t)part * K * Z + (size_t)d * K + k;
+                for (int i = 0; i < H; ++i) wh[row * H + i] = bf(w->W_mdn[(size_t)i * M + col]);
+                bh[row] = w->b_mdn[col];
+            }
+    {
+        const size_t rr = (size_t)rd_tile * HEAD_TILE + rd_col;
+        for (int i = 0; i < H; ++i) {
+            wh[rr * H + i] = bf(w->w_rew[i]);
+            wh[(rr + 1) * H + i] = bf(w->w_done[i]);
+        }
+        bh[rr] = w->b_rew;
+        bh[rr + 1] = w->b_done;
+    }
+    cudaError_t e;
+    auto up = [&](void **dst, const void *src, size_t bytes) {
+        cudaError_t r = cudaMalloc(dst, bytes);
+        if (r == cudaSuccess) r = cudaMemcpy(*dst, src, bytes, cudaMemcpyHostToDevice);
+        return r;
+    };
+    if ((e = up(&T.wc, wc.data(), wc.size() * 2)) != cudaSuccess) return e;
+    if ((e = up(&T.wg, wg.data(), wg.size() * 2)) != cudaSuccess) return e;
+    if ((e = up(&T.wa, wa.data(), wa.size() * 2)) != cudaSuccess) return e;
+    if ((e = up(&T.wh, wh.data(), wh.size() * 2)) != cudaSuccess) return e;
+    if ((e = up((void **)&T.bc, bc.data(), bc.size() * 4)) != cudaSuccess) return e;
+    if ((e = up((void **)&T.bg, bg.data(), bg.size() * 4)) != cudaSuccess) return e;
+    if ((e = up((void **)&T.bh, bh.data(), bh.size() * 4)) != cudaSuccess) return e;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&T.sms, cudaDevAttrMultiProcessorCount, dev);
+    T.ok = 1;
+    return cudaSuccess;
+}
+
+void wm_tc_free(wm_handle *h) {
+    wm_tc_weights &T = h->tc;
+    cudaFree(T.wc); cudaFree(T.wg); cudaFree(T.wa); cudaFree(T.wh);
+    cudaFree(T.bc); cudaFree(T.bg); cudaFree(T.bh);
+    memset(&T, 0, sizeof(T));
+}
+
+// One call: rollout (teacher = 0) or teacher-forced scoring (teacher = 1).
+static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev *ra, const wm_nll_dev *na,
+                          void *ws, cudaStream_t s) {
+    const wm_config &c = h->cfg;
+    const wm_tc_weights &T = h->tc;
+    const int B = teacher ? na->N : ra->B, Tn = teacher ? na->T : ra->T;
+    const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, KX = Z + H;
+    if (B == 0) { h->last_launches = 0; return cudaSuccess; }
+    TcWs w = carve_ws(h, B, ws);
+    StepIO io{};
+    io.B = B; io.Z = Z; io.A = A; io.H = H; io.K = c.k_mix; io.T = Tn;
+    io.seed = c.seed; io.teacher = teacher;
+    io.ctrl_sample = c.ctrl_sample; io.ctrl_tau = c.ctrl_tau; io.mdn_tau = c.mdn_tau;
+    io.sigma_sqrt_tau = c.sigma_sqrt_tau; io.done_terminates = c.done_terminates;
+    io.noop_terminates = c.noop_terminates;
+    io.c = w.c; io.h32 = w.h32; io.act = w.act;
+    io.b_ctrl = T.bc; io.b_gate = T.bg; io.b_head = T.bh;
+    io.wa = (const __nv_bfloat16 *)T.wa;
+    io.dims_per_tile = T.dims_per_tile; io.rd_tile = T.rd_tile; io.rd_col = T.rd_col;
+    io.nll_part = w.nll_part;
+    if (teacher) {
+        io.act_in = na->actions; io.z_seq = na->z_seq; io.lengths = na->lengths;
+        io.h_seq = na->h_seq; io.c_seq = na->c_seq; io.mdn_seq = na->mdn_seq;
+    } else {
+        io.ep0 = ra->ep0;
+        io.mask = ra->mask; io.z_out = ra->z_out; io.actions = ra->actions; io.rewards = ra->rewards;
+        io.done = ra->done; io.h_seq = ra->h_seq; io.c_seq = ra->c_seq; io.mdn_seq = ra->mdn_seq;
+        io.comp_seq = ra->comp_seq;
+    }
+    int launches = 0;
+    const int init_grid = 1024;
+    io.fz_cur = w.fz[0];
+    k_tc_init<<<init_grid, 256, 0, s>>>(io, teacher ? nullptr : ra->z0, teacher ? nullptr : ra->h0,
+                                        teacher ? nullptr : ra->c0, teacher ? nullptr : ra->done0, w.x[0], w.fz[0],
+                                        w.fz[1], T.n_head_tiles);
+    ++launches;
+    CUtensorMap mx[2], mwc, mwg, mwh;
+    const uint32_t ctrl_box = A > 128 ? 256u : 128u;  // the instantiated BN; rows past A read as zero
+    if (!make_map(&mx[0], w.x[0], B, KX, BM) || !make_map(&mx[1], w.x[1], B, KX, BM) ||
+        !make_map(&mwc, T.wc, A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 256) ||
+        !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE))
+        return cudaErrorInvalidValue;
+    const int m_tiles = (B + BM - 1) / BM;
+    cudaError_t e = cudaSuccess;
+    for (int t = 0; t < Tn && e == cudaSuccess; ++t) {
+        io.t = t;
+        io.step = teacher ? (uint32_t)t : ra->t0 + (uint32_t)t;
+        io.x_cur = w.x[t & 1];
+        io.x_next = w.x[(t + 1) & 1];
+        io.fz_cur = w.fz[t & 1];
+        io.fz_next = w.fz[(t + 1) & 1];
+        const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status};
+        if (!teacher) {
+            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
+            else if (A > 128) e = launch_gemm<256, 1, 4, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
+            else e = launch_gemm<128, 1, 4, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
+            ++launches;
+            if (e != cudaSuccess) break;
+        }
+        const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
+        e = launch_gemm<256, 1, 4, EpiGates>(mx[t & 1], mwg, g2, io, T.sms, s);
+        ++launches;
+        if (e != cudaSuccess) break;
+        const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
+        e = launch_gemm<HEAD_TILE, 1, 4, EpiHeads>(mx[(t + 1) & 1], mwh, g3, io, T.sms, s);
+        ++launches;
+    }
+    if (e != cudaSuccess) return e;
+    k_tc_finish<<<init_grid, 256, 0, s>>>(B, H, w.h32, w.c, teacher ? nullptr : ra->h_final,
+                                          teacher ? nullptr : ra->c_final, w.nll_part, 4 * T.n_head_tiles,
+                                          teacher ? na->nll : nullptr);
+    ++launches;
+    h->last_launches = launches;
+    return cudaGetLastError();
+}
+
+cudaError_t wm_tc_rollout(const wm_handle *h, const wm_rollout_dev &a, void *ws, cudaStream_t s) {
+    return tc_run(h, 0, &a, nullptr, ws, s);
+}
+
+cudaError_t wm_tc_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s) {
+    return tc_run(h, 1, nullptr, &a, ws, s);
+}

@@ -136,20 +136,23 @@ def _rollout_sampled(wm, orc, name, n_oracle, path="auto"):
         for k in ("z", "actions", "rewards", "done", "comp_seq"):
             assert torch.equal(one[k][:, 0], full[k][:, int(b)]), (k, int(b))
         parts.append({k: np_(v) for k, v in one.items()})
+    assert m.last_path == path  # the re-runs used the same kernel family as the full batch
     g = {k: np.concatenate([p[k] for p in parts], axis=0 if k in ("h_final", "c_final") else 1)
          for k in parts[0]}
     o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
-    return check_rollout(g, o, cfg, weights=w)
+    return check_rollout(g, o, cfg, weights=w, mask=mask[:, idx])
 
 
-def test_rollout_mid_bf16_sampled(wm, orc):
-    r = _rollout_sampled(wm, orc, "mid_bf16", 24)
-    print("mid_bf16 parity:", r)
+@pytest.mark.parametrize("path", ["tensor", "stepwise"])
+def test_rollout_mid_bf16_sampled(wm, orc, path):
+    r = _rollout_sampled(wm, orc, "mid_bf16", 24, path=path)
+    print("mid_bf16 parity:", path, r)
 
 
-def test_rollout_large_bf16_sampled(wm, orc):
-    r = _rollout_sampled(wm, orc, "large_bf16", 24)
-    print("large_bf16 parity:", r)
+@pytest.mark.parametrize("path", ["tensor", "stepwise"])
+def test_rollout_large_bf16_sampled(wm, orc, path):
+    r = _rollout_sampled(wm, orc, "large_bf16", 24, path=path)
+    print("large_bf16 parity:", path, r)
 
 
 # ------------------------------------------------------------------ edge cases
@@ -313,3 +316,51 @@ def test_fused_matches_stepwise_closely(wm):
     z_eq = ((a["z"][1:] - b["z"][1:]).abs().amax(-1) < 2e-2).cpu().numpy()
     ok = np.cumprod(act_eq & z_eq, axis=0)                           # 1 until first divergence
     assert ok.mean() > 0.95, ok.mean()
+
+
+# ------------------------------------------------------------------ the tensor-core family
+@pytest.mark.parametrize("name,flags", [("mid_bf16", dict()), ("large_bf16", dict()),
+                                        ("small_bf16", dict(mdn_tau=0.0)),
+                                        ("small_bf16", dict(mdn_tau=0.6, sigma_sqrt_tau=1,
+                                                            noop_terminates=1, done_terminates=1)),
+                                        ("mid_bf16", dict(ctrl_sample=1, ctrl_tau=0.7))])
+def test_tensor_against_oracle(wm, orc, name, flags):
+    """Two row tiles (the second partly filled), resumed state, offsets, flags."""
+    cfg = dict(synth.model_config(name), **flags)
+    w = synth.weights(cfg, seed=7)
+    B, T = 200, 6
+    z0 = synth.z0(B, cfg["z_dim"], seed=7)
+    mask = synth.mask(T, B, cfg["a_dim"], synth.WORKLOADS[name]["mask_density"], seed=7)
+    mask[2, 9] = 0
+    rng = np.random.default_rng(7)
+    h0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    c0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    done0 = (np.arange(B) % 41 == 0).astype(np.uint8)
+    m = wm.WorldModel(dict(cfg, path="tensor"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=99, t0=11, h0=_cuda(h0),
+                  c0=_cuda(c0), done0=_cuda(done0), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "tensor"
+    o = orc.rollout(cfg, w, z0, mask, T, episode_offset=99, t0=11, h0=h0, c0=c0, done0=done0,
+                    want_seq=True, nthreads=NT)
+    r = check_rollout(g, o, cfg, weights=w, h0=h0, mask=mask)
+    print("tensor", name, flags, r)
+
+
+@pytest.mark.parametrize("name,prec,N,T", [("mid_bf16", None, 300, 9), ("nll", "bf16", 512, 128),
+                                           ("large_bf16", None, 130, 5)])
+def test_tensor_teacher_forced(wm, orc, name, prec, N, T):
+    cfg = synth.model_config(name)
+    if prec:
+        cfg["precision"] = prec
+    w = synth.weights(cfg, seed=8)
+    zs, acts, lens = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=8, ragged=True)
+    acts[1, ::7] = -1
+    m = wm.WorldModel(dict(cfg, path="tensor"), w)
+    g = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "tensor"
+    idx = _spread(N, 96)
+    o = orc.mdn_nll(cfg, w, zs[:, idx], acts[:, idx], lengths=lens[idx], want_seq=True, nthreads=NT)
+    gs = {k: np_(v)[:, idx] if k != "nll" else np_(v)[idx] for k, v in g.items()}
+    check_teacher(gs, o, "bf16")
