@@ -48,19 +48,6 @@ def flops_per_env_step(cfg: dict) -> float:
     return 2.0 * ((Z + H) * A + (Z + H) * 4 * H + H * 3 * K * Z + 2 * H)
 
 
-def bytes_per_env_step(cfg: dict) -> float:
-    """Algorithmic HBM bytes of one (episode, step) with the state kept on chip:
-    the mask words read, z_{t+1}, action, reward and done written."""
-    Z, A = cfg["z_dim"], cfg["a_dim"]
-    return 4.0 * ((A + 31) // 32) + 4.0 * Z + 4 + 4 + 1
-
-
-def weight_bytes(cfg: dict) -> float:
-    Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
-    el = 2 if cfg["precision"] == "bf16" else 4
-    return el * ((Z + A + H) * 4 * H + H * (3 * K * Z + 2) + (Z + H) * A)
-
-
 def load_peaks() -> dict:
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -77,8 +64,33 @@ def fp32_simt_peak_tflops() -> float:
     return 152 * 128 * 2 * 2.07e9 / 1e12
 
 
-def kernel_source_sha(path_name: str) -> str:
-    src = {"fused": "wm_fused.cu", "stepwise": "wm_step.cu", "tensor": "wm_tensor.cu"}[path_name]
+# kernel class -> (kernel as the profiler names it, source file)
+KERNELS = {"fused": ("k_fused", "wm_fused.cu"),
+           "tc_ctrl": ("k_tc_gemm<EpiCtrl>", "wm_tensor.cu"),
+           "tc_gates": ("k_tc_gemm<EpiGates>", "wm_tensor.cu"),
+           "tc_heads": ("k_tc_gemm<EpiHeads>", "wm_tensor.cu"),
+           "step_gemm": ("k_gemm", "wm_step.cu"),
+           "step_cell": ("k_select_cell", "wm_step.cu"),
+           "step_sample": ("k_sample", "wm_step.cu")}
+
+
+def kernel_flops(cls: str, cfg: dict, B: int, T: int, launches: int) -> float:
+    """Algorithmic FLOPs of one launch of a kernel class (its contraction)."""
+    Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
+    if cls == "fused":
+        return flops_per_env_step(cfg) * B * T
+    if cls == "tc_ctrl":
+        return 2.0 * B * (Z + H) * A
+    if cls == "tc_gates":
+        return 2.0 * B * (Z + H) * 4 * H
+    if cls == "tc_heads":
+        return 2.0 * B * H * (3 * K * Z + 2)
+    if cls == "step_gemm":  # two GEMMs per step: gates + controller, then heads
+        return 2.0 * B * ((Z + H) * (4 * H + A) + H * (3 * K * Z + 2)) / 2
+    return 0.0
+
+
+def kernel_source_sha(src: str) -> str:
     with open(os.path.join(ROOT, "paper_2205_01435_gb300", "csrc", src), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
@@ -196,7 +208,7 @@ def run_ours(args) -> None:
     torch.cuda.set_device(local)
     wm = pkg.load()
     name = args.workload
-    cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=args.batch)
     if args.path:
         cfg["path"] = args.path
     model = wm.WorldModel(cfg, w, device=local)
@@ -220,6 +232,7 @@ def run_ours(args) -> None:
     torch.cuda.synchronize()
     path_name = model.last_path
     launches = model.last_launches
+    model.set_timing(True)  # each kernel bracketed by CUDA events on the launching stream
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -235,6 +248,8 @@ def run_ours(args) -> None:
     if ws > 1:
         dist.barrier()
     times = [a.elapsed_time(b) for a, b in ev]  # ms, each one launch of the step
+    kt = model.kernel_times()
+    model.set_timing(False)
     total_ms = sum(times)
     t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
     if ws > 1:
@@ -250,33 +265,43 @@ def run_ours(args) -> None:
     else:
         e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg)
 
+    # roofline of the dominant kernel: its algorithmic FLOPs per launch over its own
+    # event-timed average launch duration inside the timed region
     peaks = load_peaks()
-    fl = flops_per_env_step(cfg) * B * T
-    if path_name in ("fused", "tensor"):
-        # fused: the call is one kernel; tensor: 3 GEMM kernels per step, counted together
-        kernel_key = f"wm_{path_name}_rollout/{name}"
-        bound, unit = "tensor", "TFLOP/s"
-        peak = peaks["bf16_tflops"] if path_name == "fused" else peaks["bf16_tflops_sustained"]
-        achieved = fl / (ms_per_step / 1e3) / 1e12
+    timed = {k: v for k, v in kt.items() if k in KERNELS}
+    dom = max(timed, key=lambda k: timed[k][0])
+    dom_ms, dom_n = timed[dom]
+    launch_ms = dom_ms / dom_n
+    fl = kernel_flops(dom, cfg, B, T, dom_n)
+    achieved = fl / (launch_ms / 1e3) / 1e12
+    unit = "TFLOP/s"
+    if cfg["precision"] == "bf16" and dom in ("fused", "tc_ctrl", "tc_gates", "tc_heads"):
+        bound = "tensor"
+        # a call of the fused family is one short kernel (burst); the tensor family's kernels
+        # run back to back inside a long call (sustained)
+        burst = dom == "fused"
+        peak = peaks["bf16_tflops"] if burst else peaks["bf16_tflops_sustained"]
+        peak_source = f"{peaks['source']} bf16 {'burst' if burst else 'sustained'}"
     else:
-        kernel_key = f"wm_step/{name}"
-        bound, peak, unit = "alu", fp32_simt_peak_tflops(), "TFLOP/s"
-        achieved = fl / (ms_per_step / 1e3) / 1e12
-    sha = kernel_source_sha(path_name)
-    traffic = ncu_traffic(kernel_key, sha)
+        bound, peak = "alu", fp32_simt_peak_tflops()
+        peak_source = "derived: 152 SM x 128 fp32 FMA x 2 FLOP x 2.07 GHz"
+    kname, ksrc = KERNELS[dom]
+    kernel_key = f"{kname}/{name}" + ("" if args.batch is None else f"@B{B}")
+    traffic = ncu_traffic(kernel_key, kernel_source_sha(ksrc))
+    all_ms = sum(v[0] for v in kt.values())
     roof = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": unit,
-            "frac": round(achieved / peak, 5), "traffic": traffic,
-            "peak_source": (peaks["source"] + (" bf16 burst" if path_name == "fused" else " bf16 sustained"))
-            if bound == "tensor" else "derived: 152 SM x 128 FMA x 2.07 GHz",
-            "kernel": kernel_key, "algorithmic_flops_per_launch": fl,
-            "algorithmic_hbm_bytes_per_launch": bytes_per_env_step(cfg) * B * T + weight_bytes(cfg)}
+            "frac": round(achieved / peak, 5), "traffic": traffic, "peak_source": peak_source,
+            "kernel": kernel_key, "launch_ms": round(launch_ms, 5), "launches": dom_n,
+            "algorithmic_flops_per_launch": fl,
+            "kernel_shares": {k: round(v[0] / all_ms, 4) for k, v in sorted(kt.items())}}
 
     line = {"metric": "dream env-steps/s (wm_rollout)", "value": round(value, 1),
             "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if cfg["precision"] == "bf16" else "f32",
             "data": "synthetic (seeded: weights N(0,0.05^2), z0 N(0,1), Bernoulli masks)",
-            "config": {"workload": name, "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
+            "config": {"workload": name if args.batch is None else f"{name} with B overridden",
+                       "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
                        "H": cfg["h_dim"], "K": cfg["k_mix"],
                        "mask_density": synth.WORKLOADS[name]["mask_density"],
                        "precision": cfg["precision"], "kernel_path": path_name,
@@ -363,6 +388,8 @@ def main():
     ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer leg (profiling runs)")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="episodes per call instead of the workload's B (profiling runs only)")
     ap.add_argument("--cpu-episodes", type=int, default=None,
                     help="oracle sample size (default: about 2e11 FLOPs of the workload)")
     ap.add_argument("--ref-episodes", type=int, default=None,

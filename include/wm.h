@@ -204,6 +204,33 @@ int wm_last_path(const wm_handle *h);
  * copies not counted). */
 int wm_last_launches(const wm_handle *h);
 
+/* Per-kernel timing.  The paper has no counterpart: this is instrumentation
+ * that splits a call's device time by kernel.  While timing is enabled, every
+ * kernel the handle launches is bracketed by two CUDA events recorded on the
+ * call's stream (no synchronisation is added).  wm_kernel_time waits for the
+ * events recorded so far, folds their elapsed times into per-class totals and
+ * returns the totals (milliseconds, launches) since timing was last enabled.
+ * Calls made during CUDA stream capture must not be timed. */
+enum {
+    WM_KERNEL_STEP_GEMM = 0,    /* stepwise: gate / controller and head GEMMs     */
+    WM_KERNEL_STEP_CELL = 1,    /* stepwise: action selection and LSTM cell       */
+    WM_KERNEL_STEP_SAMPLE = 2,  /* stepwise: mixture sampling or NLL              */
+    WM_KERNEL_FUSED = 3,        /* fused: the single rollout / scoring kernel      */
+    WM_KERNEL_TC_CTRL = 4,      /* tensor: controller GEMM with action selection   */
+    WM_KERNEL_TC_GATES = 5,     /* tensor: gate GEMM with the LSTM cell            */
+    WM_KERNEL_TC_HEADS = 6,     /* tensor: head GEMM with sampling or NLL          */
+    WM_KERNEL_AUX = 7,          /* state set-up, finishing copies, reductions      */
+    WM_KERNEL_CLASSES = 8
+};
+
+/* enable != 0 turns timing on and clears the totals; 0 turns it off (events
+ * already recorded can still be read). */
+wm_status wm_set_timing(wm_handle *h, int enable);
+
+/* Totals of one class (WM_KERNEL_*) since timing was enabled.  Either output
+ * may be NULL.  WM_ERR_CUDA if an event cannot be read. */
+wm_status wm_kernel_time(wm_handle *h, int kernel_class, double *total_ms, long long *launches);
+
 /* Frees everything the handle owns.  NULL is a no-op. */
 void wm_destroy(wm_handle *h);
 

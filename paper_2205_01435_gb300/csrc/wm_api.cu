@@ -212,8 +212,91 @@ void wm_destroy(wm_handle *h) {
     cudaFree(h->ws);
     cudaFree(h->stage);
     cudaFree(h->status);
+    for (auto &r : h->timer.pending) {
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+    }
+    for (cudaEvent_t ev : h->timer.spare) cudaEventDestroy(ev);
     if (prev >= 0) cudaSetDevice(prev);
     delete h;
+}
+
+// ---- per-kernel timing --------------------------------------------------------
+static cudaEvent_t timer_event(wm_timer &t) {
+    if (!t.spare.empty()) {
+        cudaEvent_t ev = t.spare.back();
+        t.spare.pop_back();
+        return ev;
+    }
+    cudaEvent_t ev = nullptr;
+    if (cudaEventCreate(&ev) != cudaSuccess) return nullptr;
+    return ev;
+}
+
+wm_ktime::wm_ktime(const wm_handle *h, int cls, cudaStream_t s) : t_(nullptr), cls_(cls), s_(s) {
+    if (!h || !h->timer.on) return;
+    t_ = &h->timer;
+    a_ = timer_event(*t_);
+    if (a_ && cudaEventRecord(a_, s_) != cudaSuccess) {
+        t_->spare.push_back(a_);
+        a_ = nullptr;
+    }
+}
+
+wm_ktime::~wm_ktime() {
+    if (!t_ || !a_) return;
+    cudaEvent_t b = timer_event(*t_);
+    if (b && cudaEventRecord(b, s_) == cudaSuccess) {
+        t_->pending.push_back({cls_, a_, b});
+        return;
+    }
+    t_->spare.push_back(a_);
+    if (b) t_->spare.push_back(b);
+}
+
+wm_status wm_set_timing(wm_handle *h, int enable) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    wm_timer &t = h->timer;
+    if (enable) {
+        for (auto &r : t.pending) {  // discard what was recorded before
+            cudaEventSynchronize(r.b);
+            t.spare.push_back(r.a);
+            t.spare.push_back(r.b);
+        }
+        t.pending.clear();
+        for (int i = 0; i < WM_KERNEL_CLASSES; ++i) {
+            t.ms[i] = 0.0;
+            t.launches[i] = 0;
+        }
+    }
+    t.on = enable != 0;
+    return WM_OK;
+}
+
+wm_status wm_kernel_time(wm_handle *h, int kernel_class, double *total_ms, long long *launches) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    if (kernel_class < 0 || kernel_class >= WM_KERNEL_CLASSES)
+        return fail(h, WM_ERR_INVALID_ARG, "kernel class out of range");
+    wm_timer &t = h->timer;
+    cudaError_t err = cudaSuccess;
+    for (auto &r : t.pending) {
+        float ms = 0.f;
+        cudaError_t e = cudaEventSynchronize(r.b);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, r.a, r.b);
+        if (e == cudaSuccess) {
+            t.ms[r.cls] += ms;
+            t.launches[r.cls] += 1;
+        } else if (err == cudaSuccess) {
+            err = e;
+        }
+        t.spare.push_back(r.a);
+        t.spare.push_back(r.b);
+    }
+    t.pending.clear();
+    if (err != cudaSuccess) return cuda_fail(h, err, "wm_kernel_time");
+    if (total_ms) *total_ms = t.ms[kernel_class];
+    if (launches) *launches = t.launches[kernel_class];
+    return WM_OK;
 }
 
 const char *wm_last_error(const wm_handle *h) { return h ? h->err.c_str() : "null handle"; }

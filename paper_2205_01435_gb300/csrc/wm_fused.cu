@@ -847,11 +847,15 @@ cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaSt
     if (a.B == 0) { h->last_launches = 0; return cudaSuccess; }
     // z_out[0] = z0
     const size_t nz = (size_t)a.B * h->cfg.z_dim;
-    k_copy_f32<<<(int)((nz + 255) / 256 < 1024 ? (nz + 255) / 256 : 1024), 256, 0, s>>>(nz, a.z0, a.z_out);
+    {
+        wm_ktime kt(h, WM_KERNEL_AUX, s);
+        k_copy_f32<<<(int)((nz + 255) / 256 < 1024 ? (nz + 255) / 256 : 1024), 256, 0, s>>>(nz, a.z0, a.z_out);
+    }
     h->last_launches = 1;
     if (a.T == 0) {
         const size_t nh = (size_t)a.B * h->cfg.h_dim;
         int grid = (int)((nh + 255) / 256 < 1024 ? (nh + 255) / 256 : 1024);
+        wm_ktime kt(h, WM_KERNEL_AUX, s);
         if (a.h_final) {
             if (a.h0) k_copy_f32<<<grid, 256, 0, s>>>(nh, a.h0, a.h_final);
             else cudaMemsetAsync(a.h_final, 0, nh * 4, s);
@@ -869,7 +873,11 @@ cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaSt
     p.z_out = a.z_out; p.actions = a.actions; p.rewards = a.rewards; p.done = a.done;
     p.h_final = a.h_final; p.c_final = a.c_final; p.h_seq = a.h_seq; p.c_seq = a.c_seq;
     p.mdn_seq = a.mdn_seq; p.comp_seq = a.comp_seq;
-    cudaError_t e = launch_slot(h, p, s);
+    cudaError_t e;
+    {
+        wm_ktime kt(h, WM_KERNEL_FUSED, s);
+        e = launch_slot(h, p, s);
+    }
     h->last_launches = 2;
     return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -887,9 +895,16 @@ cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cuda
     p.z_seq = a.z_seq; p.act_in = a.actions; p.lengths = a.lengths;
     p.h_seq = a.h_seq; p.c_seq = a.c_seq; p.mdn_seq = a.mdn_seq;
     p.nll_part = (float *)ws;
-    cudaError_t e = launch_slot(h, p, s);
+    cudaError_t e;
+    {
+        wm_ktime kt(h, WM_KERNEL_FUSED, s);
+        e = launch_slot(h, p, s);
+    }
     if (e != cudaSuccess) return e;
-    k_nll_reduce<<<(a.N + 127) / 128, 128, 0, s>>>(a.N, h->cfg.z_dim, p.nll_part, a.nll);
+    {
+        wm_ktime kt(h, WM_KERNEL_AUX, s);
+        k_nll_reduce<<<(a.N + 127) / 128, 128, 0, s>>>(a.N, h->cfg.z_dim, p.nll_part, a.nll);
+    }
     h->last_launches = 2;
     return cudaGetLastError();
 }

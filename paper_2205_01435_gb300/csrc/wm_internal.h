@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <vector>
 
 #include "wm.h"
 
@@ -62,6 +63,20 @@ struct wm_tc_weights {
     int ok;
 };
 
+// Per-kernel timing (wm_set_timing): event pairs recorded on the launching
+// stream, folded into per-class totals when read.
+struct wm_timer {
+    struct Rec {
+        int cls;
+        cudaEvent_t a, b;
+    };
+    bool on = false;
+    std::vector<Rec> pending;
+    std::vector<cudaEvent_t> spare;
+    double ms[WM_KERNEL_CLASSES] = {};
+    long long launches[WM_KERNEL_CLASSES] = {};
+};
+
 struct wm_handle {
     wm_config cfg;
     int device;
@@ -76,7 +91,24 @@ struct wm_handle {
     int *status = nullptr;       // device status word (WM_ERR_TIMEOUT etc.)
     int last_path = 0;
     mutable int last_launches = 0;   // kernels launched by the last call
+    mutable wm_timer timer;
     std::string err;
+};
+
+// Brackets the kernel launches of its scope with CUDA events on stream s when
+// timing is on for h; does nothing otherwise.
+class wm_ktime {
+  public:
+    wm_ktime(const wm_handle *h, int cls, cudaStream_t s);
+    ~wm_ktime();
+    wm_ktime(const wm_ktime &) = delete;
+    wm_ktime &operator=(const wm_ktime &) = delete;
+
+  private:
+    wm_timer *t_;
+    int cls_;
+    cudaStream_t s_;
+    cudaEvent_t a_ = nullptr;
 };
 
 // ---- tensor-core family (wm_tensor.cu) ----------------------------------------

@@ -394,8 +394,10 @@ StepWs carve(const wm_handle *hd, int B, void *ws, bool teacher) {
     return w;
 }
 
-void launch_gemm(bool round, int M, int N, int K1, int K2, const float *A1, long lda1, const float *A2,
-                 long lda2, const float *W, long ldw, const float *bias, float *C, long ldc, cudaStream_t s) {
+void launch_gemm(const wm_handle *hd, bool round, int M, int N, int K1, int K2, const float *A1, long lda1,
+                 const float *A2, long lda2, const float *W, long ldw, const float *bias, float *C, long ldc,
+                 cudaStream_t s) {
+    wm_ktime kt(hd, WM_KERNEL_STEP_GEMM, s);
     dim3 grid((N + GBN - 1) / GBN, (M + GBM - 1) / GBM);
     if (round)
         k_gemm<true><<<grid, 256, 0, s>>>(M, N, K1, K2, A1, lda1, A2, lda2, W, ldw, bias, C, ldc);
@@ -435,8 +437,11 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
     if (B == 0) return cudaSuccess;
     StepWs w = carve(hd, B, ws, false);
     const bool round = c.precision == WM_BF16;
-    k_init_state<<<grid_1d((size_t)B * H), 256, 0, s>>>(B, H, Z, a.h0, a.c0, a.done0, a.z0, w.h, w.c,
-                                                         w.frozen, a.z_out, nullptr);
+    {
+        wm_ktime kt(hd, WM_KERNEL_AUX, s);
+        k_init_state<<<grid_1d((size_t)B * H), 256, 0, s>>>(B, H, Z, a.h0, a.c0, a.done0, a.z0, w.h, w.c,
+                                                             w.frozen, a.z_out, nullptr);
+    }
     StepParams p = base_params(hd, B, T, w);
     p.teacher = 0;
     p.ep0 = a.ep0;
@@ -449,15 +454,23 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
         p.step = a.t0 + (uint32_t)t;
         p.z_cur = a.z_out + (size_t)t * B * Z;
         p.z_next = a.z_out + (size_t)(t + 1) * B * Z;
-        launch_gemm(round, B, 4 * H + A, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A, hd->step.bg,
+        launch_gemm(hd, round, B, 4 * H + A, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A, hd->step.bg,
                     w.G, 4L * H + A, s);
-        k_select_cell<<<B, 256, 0, s>>>(p);
-        launch_gemm(round, B, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
+        {
+            wm_ktime kt(hd, WM_KERNEL_STEP_CELL, s);
+            k_select_cell<<<B, 256, 0, s>>>(p);
+        }
+        launch_gemm(hd, round, B, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
                     w.heads, hd->M + 2, s);
-        k_sample<<<B, 128, 0, s>>>(p);
+        {
+            wm_ktime kt(hd, WM_KERNEL_STEP_SAMPLE, s);
+            k_sample<<<B, 128, 0, s>>>(p);
+        }
     }
-    if (a.h_final || a.c_final)
+    if (a.h_final || a.c_final) {
+        wm_ktime kt(hd, WM_KERNEL_AUX, s);
         k_finish<<<grid_1d((size_t)B * H), 256, 0, s>>>(B, H, w.h, w.c, a.h_final, a.c_final, nullptr, nullptr);
+    }
     return cudaGetLastError();
 }
 
@@ -467,8 +480,11 @@ cudaError_t wm_step_nll(const wm_handle *hd, const wm_nll_dev &a, void *ws, cuda
     if (N == 0) return cudaSuccess;
     StepWs w = carve(hd, N, ws, true);
     const bool round = c.precision == WM_BF16;
-    k_init_state<<<grid_1d((size_t)N * H), 256, 0, s>>>(N, H, Z, nullptr, nullptr, nullptr, nullptr, w.h,
-                                                         w.c, w.frozen, nullptr, w.nll_acc);
+    {
+        wm_ktime kt(hd, WM_KERNEL_AUX, s);
+        k_init_state<<<grid_1d((size_t)N * H), 256, 0, s>>>(N, H, Z, nullptr, nullptr, nullptr, nullptr, w.h,
+                                                             w.c, w.frozen, nullptr, w.nll_acc);
+    }
     StepParams p = base_params(hd, N, T, w);
     p.teacher = 1;
     p.act_in = a.actions;
@@ -479,13 +495,22 @@ cudaError_t wm_step_nll(const wm_handle *hd, const wm_nll_dev &a, void *ws, cuda
         p.t = t;
         p.z_cur = a.z_seq + (size_t)t * N * Z;
         p.z_target = a.z_seq + (size_t)(t + 1) * N * Z;
-        launch_gemm(round, N, 4 * H, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A, hd->step.bg, w.G,
+        launch_gemm(hd, round, N, 4 * H, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A, hd->step.bg, w.G,
                     4L * H + A, s);
-        k_select_cell<<<N, 256, 0, s>>>(p);
-        launch_gemm(round, N, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
+        {
+            wm_ktime kt(hd, WM_KERNEL_STEP_CELL, s);
+            k_select_cell<<<N, 256, 0, s>>>(p);
+        }
+        launch_gemm(hd, round, N, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
                     w.heads, hd->M + 2, s);
-        k_sample<<<N, 128, 0, s>>>(p);
+        {
+            wm_ktime kt(hd, WM_KERNEL_STEP_SAMPLE, s);
+            k_sample<<<N, 128, 0, s>>>(p);
+        }
     }
-    k_finish<<<grid_1d((size_t)N * H), 256, 0, s>>>(N, H, w.h, w.c, nullptr, nullptr, w.nll_acc, a.nll);
+    {
+        wm_ktime kt(hd, WM_KERNEL_AUX, s);
+        k_finish<<<grid_1d((size_t)N * H), 256, 0, s>>>(N, H, w.h, w.c, nullptr, nullptr, w.nll_acc, a.nll);
+    }
     return cudaGetLastError();
 }

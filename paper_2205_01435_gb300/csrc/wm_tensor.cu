@@ -59,6 +59,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         :: "r"(dst), "l"(map), "r"(x), "r"(y), "r"(mbar) : "memory");
 }
 
+// TMA store of a box from shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x, int y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+                 :: "l"(map), "r"(x), "r"(y), "r"(src) : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// the shared-memory sources of this thread's committed stores have been read
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// ... and the stores are complete
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ void mbar_arrive(uint32_t mbar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(mbar) : "memory");
 }
@@ -80,6 +91,7 @@ struct StepIO {
     uint32_t step;
     unsigned long long ep0, seed;
     int teacher, ctrl_sample, sigma_sqrt_tau, done_terminates, noop_terminates;
+    int h32_mode;                   // when h (fp32) is stored: 0 never, 1 last step, 2 every step
     float ctrl_tau, mdn_tau;
     // state
     __nv_bfloat16 *x_cur, *x_next;  // [B, Z+H]
@@ -92,6 +104,7 @@ struct StepIO {
     const __nv_bfloat16 *wa;        // [A, 4H] gate-tile column order
     // head tiles
     int dims_per_tile, rd_tile, rd_col;  // reward / done columns: tile, first column
+    int gates_n_tiles;                   // H / 64
     // inputs / outputs
     const uint32_t *mask;           // [T, B, W] or null
     const int32_t *act_in;          // teacher: [T, B]
@@ -109,18 +122,47 @@ struct StepIO {
 // Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
 // quadrant w%4) and owns column group cg = (w-2)/4 of the tile.  The 4 groups of a
 // quadrant cooperate through shared memory and a named barrier (ids 1..4).
+//
+// An epilogue may also stage data in a slab of shared memory per quadrant
+// (QUAD_STAGE bytes, 1024-aligned): the quadrant's leader fills it by TMA
+// (prefetch, signalled on the quadrant's mbarrier) and stores it back by TMA.
 struct EpiCtx {
     int quad, cg, lane, row;
     float *red;  // [4 quad][4 group][32 lane][2] scratch for cross-group reductions
+    unsigned char *stage;
+    uint32_t stage_u, stage_bar, stage_phase;
+    bool leader;        // lane 0 of the quadrant's first warp: issues the quadrant's TMA copies
+    bool pending;       // leader: a prefetch not yet waited for (parity pending_phase)
+    uint32_t pending_phase;
+    const CUtensorMap *tm_c, *tm_xs;
+    int *abort_flag, *status;
     __device__ void sync() const { asm volatile("bar.sync %0, 128;" :: "r"(1 + quad) : "memory"); }
     __device__ float *slot(int g) const { return red + ((quad * 4 + g) * 32 + lane) * 2; }
+    __device__ void wait_stage() {
+        if (!*abort_flag) {
+            if (tc::mbar_wait_bounded(stage_bar, stage_phase, POLLS)) {
+                pending = false;
+            } else {
+                *abort_flag = 1;
+                atomicExch(status, (int)WM_ERR_TIMEOUT);
+            }
+        }
+        stage_phase ^= 1u;
+    }
+    __device__ void note_prefetch() {
+        pending = true;
+        pending_phase = stage_phase;
+    }
 };
 
 // ---- controller epilogue: A columns in TMEM, A/4 per column group ---------------
 // Every thread of a warp issues the same TMEM loads (they are warp-collective);
 // rows past B only skip their memory accesses.
 struct EpiCtrl {
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+    static constexpr uint32_t QUAD_STAGE = 0;
+    static constexpr uint32_t RED_BYTES = 4 * 4 * 32 * 2 * 4;
+    static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int) {
         (void)n;
         const int b = m * BM + x.row;
         const bool valid = b < p.B;
@@ -213,91 +255,138 @@ struct EpiCtrl {
 };
 
 // ---- gate epilogue: 64 units per tile, columns [i | f | g | o] x 64; 16 units per group
+// The quadrant's c rows (32 x 64 fp32) and h' rows (32 x 64 bf16) go through
+// shared memory in the 128-byte-swizzled layout of TMA boxes 128 bytes wide,
+// so that every global access of the cell is a full-row TMA box instead of 32
+// rows per instruction: c is loaded by TMA, updated in place and stored back by
+// TMA; h' is stored by TMA into X_next.  The next tile's c is loaded as soon as
+// the stores have read the slab.  (Separate in- and out-slabs, refilled
+// mid-tile, measured slower: the extra quadrant barrier costs more than the
+// load latency it hides.)
 struct EpiGates {
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+    static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
+    static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
+    static constexpr uint32_t QUAD_STAGE = C_SLAB + X_SLAB;  // c (in place) | h' out
+    static constexpr uint32_t RED_BYTES = 0;
+
+    // byte offset of (row r, 16-byte chunk j) in a 128-byte-swizzled box
+    static __device__ __forceinline__ uint32_t sw(int r, int j) { return r * 128 + ((j ^ (r & 7)) << 4); }
+
+    static __device__ void prefetch(const StepIO &, int m, int n, EpiCtx &x) {
+        x.note_prefetch();
+        tc::mbar_arrive_expect_tx(x.stage_bar, C_SLAB);
+        for (int bx = 0; bx < 2; ++bx)
+            tma_load_2d(x.stage_u + bx * 4096, x.tm_c, 64 * n + 32 * bx, m * BM + 32 * x.quad, x.stage_bar);
+    }
+
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int next) {
         const int b = m * BM + x.row;
         const bool valid = b < p.B;
-        const int bb = valid ? b : 0;  // rows past B compute on row 0 and store nothing
-        const int H = p.H, KX = p.Z + p.H;
+        const int bb = valid ? b : 0;  // rows past B compute on row 0; TMA stores clip them
+        const int H = p.H, r = x.lane, q = x.cg;
         const bool fz = p.fz_cur[bb] != 0;
         int a = p.act[bb];
         if (p.teacher) {
             a = p.act_in[(size_t)p.t * p.B + bb];
             if (a < 0 || a >= p.A) a = -1;
         }
-        const int q = x.cg;             // 16-unit chunk of the tile
-        const __nv_bfloat16 *war = a >= 0 ? p.wa + (size_t)a * 4 * H + 256 * n + 16 * q : nullptr;
+        // the action's W_a row segment, an L2 gather (a row per lane): the first half is
+        // issued before any wait, the second while the first is computed
+        const bool gather = a >= 0 && !fz;
+        const uint4 *war = reinterpret_cast<const uint4 *>(p.wa + (size_t)(gather ? a : 0) * 4 * H + 256 * n + 16 * q);
+        uint4 wv[4];
+#pragma unroll
+        for (int gate = 0; gate < 4; ++gate) wv[gate] = gather ? war[8 * gate] : make_uint4(0, 0, 0, 0);
         const float *bg = p.b_gate + 256 * n + 16 * q;
+        const bool store_h32 = valid && !fz && (p.h32_mode == 2 || (p.h32_mode == 1 && p.t == p.T - 1));
+        unsigned char *cs = x.stage, *xs = x.stage + C_SLAB;
+        x.wait_stage();  // the quadrant's c rows have landed
+#pragma unroll 1
         for (int half = 0; half < 2; ++half) {  // 8 units at a time keeps the registers in bounds
-            const int j0 = 8 * half, u0 = 64 * n + 16 * q + j0;
-            uint32_t r[4][8];
+            const int j0 = 8 * half, ut = 16 * q + j0, u0 = 64 * n + ut;
+            if (half == 1) {
 #pragma unroll
-            for (int gate = 0; gate < 4; ++gate) TC_LD8(tacc + 64 * gate + 16 * q + j0, r[gate]);
+                for (int gate = 0; gate < 4; ++gate) wv[gate] = gather ? war[8 * gate + 1] : make_uint4(0, 0, 0, 0);
+            }
+            uint32_t rr[4][8];
+#pragma unroll
+            for (int gate = 0; gate < 4; ++gate) TC_LD8(tacc + 64 * gate + ut, rr[gate]);
             tc::tmem_ld_wait();
-            float4 *c4 = reinterpret_cast<float4 *>(p.c + (size_t)bb * H + u0);
-            float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)bb * H + u0);
-            float cv[8], hv[8];
-            if (fz) {
-#pragma unroll
-                for (int k = 0; k < 2; ++k) {
-                    const float4 cc = c4[k], hh = h4[k];
-                    cv[4 * k] = cc.x; cv[4 * k + 1] = cc.y; cv[4 * k + 2] = cc.z; cv[4 * k + 3] = cc.w;
-                    hv[4 * k] = hh.x; hv[4 * k + 1] = hh.y; hv[4 * k + 2] = hh.z; hv[4 * k + 3] = hh.w;
-                }
+            const uint32_t o0 = (ut >> 5) * 4096 + sw(r, (ut & 31) >> 2), o1 = (ut >> 5) * 4096 + sw(r, ((ut & 31) >> 2) + 1);
+            const float4 ca = *reinterpret_cast<const float4 *>(cs + o0), cb = *reinterpret_cast<const float4 *>(cs + o1);
+            float cv[8] = {ca.x, ca.y, ca.z, ca.w, cb.x, cb.y, cb.z, cb.w}, hv[8];
+            if (fz) {  // frozen: c stays, h is the carried one
+                const float4 *h4 = reinterpret_cast<const float4 *>(p.h32 + (size_t)bb * H + u0);
+                const float4 ha = h4[0], hb = h4[1];
+                hv[0] = ha.x; hv[1] = ha.y; hv[2] = ha.z; hv[3] = ha.w;
+                hv[4] = hb.x; hv[5] = hb.y; hv[6] = hb.z; hv[7] = hb.w;
             } else {
                 float gv[4][8];
 #pragma unroll
                 for (int gate = 0; gate < 4; ++gate) {
-                    float w8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-                    if (war) {
-                        const uint4 w4 = *reinterpret_cast<const uint4 *>(war + 64 * gate + j0);
-                        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+                    const uint32_t w4[4] = {wv[gate].x, wv[gate].y, wv[gate].z, wv[gate].w};
+                    const float4 b0 = *reinterpret_cast<const float4 *>(bg + 64 * gate + j0);
+                    const float4 b1 = *reinterpret_cast<const float4 *>(bg + 64 * gate + j0 + 4);
+                    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&wv[e]);
-                            w8[2 * e] = __low2float(v2);
-                            w8[2 * e + 1] = __high2float(v2);
-                        }
+                    for (int e = 0; e < 4; ++e) {
+                        const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&w4[e]);
+                        gv[gate][2 * e] = __uint_as_float(rr[gate][2 * e]) + bv[2 * e] + __low2float(v2);
+                        gv[gate][2 * e + 1] = __uint_as_float(rr[gate][2 * e + 1]) + bv[2 * e + 1] + __high2float(v2);
                     }
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        gv[gate][j] = __uint_as_float(r[gate][j]) + bg[64 * gate + j0 + j] + w8[j];
                 }
-                const float4 ca = c4[0], cb = c4[1];
-                const float cold[8] = {ca.x, ca.y, ca.z, ca.w, cb.x, cb.y, cb.z, cb.w};
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    const float cn = sigmoid_hw(gv[1][j]) * cold[j] + sigmoid_hw(gv[0][j]) * tanh_hw(gv[2][j]);
+                    const float cn = sigmoid_hw(gv[1][j]) * cv[j] + sigmoid_hw(gv[0][j]) * tanh_hw(gv[2][j]);
                     cv[j] = cn;
                     hv[j] = sigmoid_hw(gv[3][j]) * tanh_hw(cn);
                 }
-                if (valid) {
-                    c4[0] = make_float4(cv[0], cv[1], cv[2], cv[3]);
-                    c4[1] = make_float4(cv[4], cv[5], cv[6], cv[7]);
-                    h4[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
-                    h4[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
-                }
             }
-            if (!valid) continue;
+            *reinterpret_cast<float4 *>(cs + o0) = make_float4(cv[0], cv[1], cv[2], cv[3]);
+            *reinterpret_cast<float4 *>(cs + o1) = make_float4(cv[4], cv[5], cv[6], cv[7]);
             uint32_t pk[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 __nv_bfloat162 v = __floats2bfloat162_rn(hv[2 * j], hv[2 * j + 1]);
                 pk[j] = *reinterpret_cast<uint32_t *>(&v);
             }
-            *reinterpret_cast<uint4 *>(p.x_next + (size_t)b * KX + p.Z + u0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4 *>(xs + sw(r, ut >> 3)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            if (store_h32) {
+                float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)b * H + u0);
+                h4[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
+                h4[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
+            }
+            if (!valid) continue;
             const size_t o = ((size_t)p.t * p.B + b) * H + u0;
             if (p.h_seq)
                 for (int j = 0; j < 8; ++j) p.h_seq[o + j] = hv[j];
             if (p.c_seq)
                 for (int j = 0; j < 8; ++j) p.c_seq[o + j] = cv[j];
         }
+        // the slab's generic-proxy reads and writes are ordered before the TMA (async-proxy)
+        // stores and the refill by this fence and the barrier
+        tc::fence_proxy_async_smem();
+        x.sync();
+        if (x.leader) {
+            const int y = m * BM + 32 * x.quad;
+            if (y < p.B) {  // rows past B are clipped by the stores; a slab wholly past B is skipped
+                tma_store_2d(x.tm_c, 64 * n, y, x.stage_u);
+                tma_store_2d(x.tm_c, 64 * n + 32, y, x.stage_u + 4096);
+                tma_store_2d(x.tm_xs, p.Z + 64 * n, y, x.stage_u + C_SLAB);
+                bulk_commit();
+                bulk_wait_read();  // the slab may be refilled
+            }
+            if (next >= 0) prefetch(p, next / p.gates_n_tiles, next % p.gates_n_tiles, x);
+        }
     }
 };
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
 struct EpiHeads {
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, const EpiCtx &x) {
+    static constexpr uint32_t QUAD_STAGE = 0;
+    static constexpr uint32_t RED_BYTES = 0;
+    static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int) {
         const int b0 = m * BM + x.row;
         const bool valid = b0 < p.B;
         const int b = valid ? b0 : 0;  // rows past B compute on row 0 and store nothing
@@ -330,41 +419,51 @@ struct EpiHeads {
                     v[16 + j] = __uint_as_float(r2[j]);
                 }
             }
+            // columns of a dim are component-interleaved (logit, mu, log sigma) so that every
+            // register index below is static: no local-memory arrays
             float lg[8], mu[8], ls[8];
+            const float *bhd = bh + DS * i;
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-                if (k < K) {
-                    lg[k] = v[k] + bh[DS * i + k];
-                    mu[k] = v[K + k] + bh[DS * i + K + k];
-                    ls[k] = v[2 * K + k] + bh[DS * i + 2 * K + k];
-                }
+                lg[k] = k < K ? v[3 * k] + bhd[3 * k] : -INFINITY;
+                mu[k] = k < K ? v[3 * k + 1] + bhd[3 * k + 1] : 0.f;
+                ls[k] = k < K ? v[3 * k + 2] + bhd[3 * k + 2] : 0.f;
             }
             if (!valid) continue;
             if (p.mdn_seq) {
                 float *ms = p.mdn_seq + tb * M;
                 const bool zero = fz && !p.teacher;
-                for (int k = 0; k < K; ++k) {
-                    ms[d * K + k] = zero ? 0.f : lg[k];
-                    ms[KZ + d * K + k] = zero ? 0.f : mu[k];
-                    ms[2 * KZ + d * K + k] = zero ? 0.f : ls[k];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    if (k < K) {
+                        ms[d * K + k] = zero ? 0.f : lg[k];
+                        ms[KZ + d * K + k] = zero ? 0.f : mu[k];
+                        ms[2 * KZ + d * K + k] = zero ? 0.f : ls[k];
+                    }
                 }
             }
             float zn;
             if (p.teacher) {
                 const float xv = p.z_seq[((size_t)(p.t + 1) * p.B + b) * Z + d];
                 float mx = -INFINITY;
-                for (int k = 0; k < K; ++k) mx = fmaxf(mx, lg[k]);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k]);
                 float s = 0.f;
-                for (int k = 0; k < K; ++k) s += expf(lg[k] - mx);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) if (k < K) s += expf(lg[k] - mx);
                 const float lse = mx + logf(s);
                 float lp[8], tmax = -INFINITY;
-                for (int k = 0; k < K; ++k) {
-                    const float zs = (xv - mu[k]) * expf(-ls[k]);
-                    lp[k] = (lg[k] - lse) - 0.5f * zs * zs - ls[k] - 0.91893853320467274178f;
-                    tmax = fmaxf(tmax, lp[k]);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    if (k < K) {
+                        const float zs = (xv - mu[k]) * expf(-ls[k]);
+                        lp[k] = (lg[k] - lse) - 0.5f * zs * zs - ls[k] - 0.91893853320467274178f;
+                        tmax = fmaxf(tmax, lp[k]);
+                    }
                 }
                 float acc = 0.f;
-                for (int k = 0; k < K; ++k) acc += expf(lp[k] - tmax);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) if (k < K) acc += expf(lp[k] - tmax);
                 nll += -(tmax + logf(acc));
                 zn = xv;
             } else if (fz) {
@@ -373,8 +472,11 @@ struct EpiHeads {
             } else {
                 int kc = 0;
                 if (!(p.mdn_tau > 0.f)) {
-                    for (int k = 1; k < K; ++k) if (lg[k] > lg[kc]) kc = k;
-                    zn = mu[kc];
+                    float best = lg[0];
+                    zn = mu[0];
+#pragma unroll
+                    for (int k = 1; k < 8; ++k)
+                        if (k < K && lg[k] > best) { best = lg[k]; kc = k; zn = mu[k]; }
                 } else {
                     if ((d >> 2) != rblock) {
                         rblock = d >> 2;
@@ -383,20 +485,31 @@ struct EpiHeads {
                     }
                     const float itau = __fdividef(1.f, p.mdn_tau);
                     float mx = -INFINITY;
-                    for (int k = 0; k < K; ++k) mx = fmaxf(mx, lg[k] * itau);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k] * itau);
                     float pk[8], s = 0.f;
-                    for (int k = 0; k < K; ++k) { pk[k] = __expf(lg[k] * itau - mx); s += pk[k]; }
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        pk[k] = k < K ? __expf(lg[k] * itau - mx) : 0.f;
+                        s += pk[k];
+                    }
                     const float u = to_uniform(u32x4_get(ru, d & 3)), is = __fdividef(1.f, s);
+                    // first k with u < C_k (the last component when rounding leaves u >= C_{K-2})
                     kc = K - 1;
-                    float cum = 0.f;
-                    for (int k = 0; k < K - 1; ++k) {
-                        cum += pk[k] * is;
-                        if (u < cum) { kc = k; break; }
+                    float cum = 0.f, muc = 0.f, lsc = 0.f;
+                    bool found = false;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        if (k < K - 1 && !found) {
+                            cum += pk[k] * is;
+                            if (u < cum) { kc = k; found = true; }
+                        }
+                        if (k == kc) { muc = mu[k]; lsc = ls[k]; }
                     }
                     const int pair = (d & 3) >> 1;
                     const float eps = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
                     const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
-                    zn = mu[kc] + __expf(ls[kc]) * scale * eps;
+                    zn = muc + __expf(lsc) * scale * eps;
                 }
                 if (p.comp_seq) p.comp_seq[tb * Z + d] = (uint8_t)kc;
             }
@@ -429,7 +542,8 @@ struct EpiHeads {
 // The persistent warp-specialised GEMM.  TILE_N = BN * NSUB columns per tile.
 template <int BN, int NSUB, int STAGES, class Epi>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
-    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmGrid g,
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmXs, GemmGrid g,
               StepIO io) {
     constexpr int TILE_N = BN * NSUB;
     constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BN * BK * 2, B_BYTES = B_SUB * NSUB;
@@ -439,10 +553,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     static_assert(BN % 16 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2];
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
-    __shared__ float epi_red[4 * 4 * 32 * 2];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t smem_u = tc::smem_u32(smem);
     auto full_b = [&](int s) { return tc::smem_u32(&bar_full[s]); };
@@ -457,6 +570,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             tc::mbar_init(tc::smem_u32(&bar_accf[a]), 1);
             tc::mbar_init(tc::smem_u32(&bar_acce[a]), EPI_WARPS * 32);
         }
+        for (int q = 0; q < 4; ++q) tc::mbar_init(tc::smem_u32(&bar_stage[q]), 1);
         tc::fence_mbar_init();
         s_abort = 0;
     }
@@ -528,18 +642,37 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
     } else {  // ---- epilogue warps 2..17: 4 column groups per TMEM lane quadrant
         const int quad = warp & 3;
-        EpiCtx x{quad, (warp - 2) >> 2, lane, 32 * quad + lane, epi_red};
+        EpiCtx x;
+        x.quad = quad;
+        x.cg = (warp - 2) >> 2;
+        x.lane = lane;
+        x.row = 32 * quad + lane;
+        x.red = reinterpret_cast<float *>(smem + STAGES * STAGE_BYTES + 4 * Epi::QUAD_STAGE);
+        x.stage = smem + STAGES * STAGE_BYTES + quad * Epi::QUAD_STAGE;
+        x.stage_u = tc::smem_u32(x.stage);
+        x.stage_bar = tc::smem_u32(&bar_stage[quad]);
+        x.stage_phase = 0;
+        x.leader = x.cg == 0 && lane == 0;
+        x.pending = false;
+        x.pending_phase = 0;
+        x.tm_c = &tmC;
+        x.tm_xs = &tmXs;
+        x.abort_flag = &s_abort;
+        x.status = g.status;
         int acc = 0;
         uint32_t acc_phase = 0;
+        if (Epi::QUAD_STAGE > 0 && x.leader && (int)blockIdx.x < ntiles)
+            Epi::prefetch(io, blockIdx.x / g.n_tiles, blockIdx.x % g.n_tiles, x);
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
             const int m = tile / g.n_tiles, n = tile % g.n_tiles;
+            const int next = tile + (int)gridDim.x < ntiles ? tile + (int)gridDim.x : -1;
             wait(tc::smem_u32(&bar_accf[acc]), acc_phase);
             __syncwarp();
             tc::fence_after_sync();
             const uint32_t tacc = tm + ((uint32_t)(32 * quad) << 16) + acc * ACC_COLS;
             // always run: the epilogues use per-quadrant named barriers, so every thread of a
             // quadrant must take the same path (after an abort the results are just unused)
-            Epi::run(io, tacc, m, n, x);
+            Epi::run(io, tacc, m, n, x, next);
             __syncwarp();
             tc::fence_before_sync();
             mbar_arrive(tc::smem_u32(&bar_acce[acc]));
@@ -549,6 +682,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             } else {
                 acc_phase ^= 1u;
             }
+        }
+        if (Epi::QUAD_STAGE > 0 && x.leader) {
+            bulk_wait_all();  // the TMA stores have completed
+            // after an abort a prefetch may still be in flight: let it land before the CTA exits
+            if (x.pending) tc::mbar_wait_bounded(x.stage_bar, x.pending_phase, POLLS);
         }
     }
     __syncwarp();
@@ -615,25 +753,30 @@ encode_fn_t get_encode() {
     return fn;
 }
 
-// 2-D bf16 map over a row-major [rows, cols] matrix, box = 64 columns x box_rows, 128B swizzle.
-bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+// 2-D map over a row-major [rows, cols] matrix of bf16 (or fp32), box = 128 bytes of a row x
+// box_rows rows, 128-byte swizzle.  Rows past `rows` read as zero and are not written.
+bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+              bool fp32 = false) {
     encode_fn_t enc = get_encode();
     if (!enc) return false;
-    cuuint64_t dims[2] = {cols, rows}, strides[1] = {cols * 2};
-    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows}, es[2] = {1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    const uint64_t es_bytes = fp32 ? 4 : 2;
+    cuuint64_t dims[2] = {cols, rows}, strides[1] = {cols * es_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)(128 / es_bytes), box_rows}, es[2] = {1, 1};
+    return enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+               const_cast<void *>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int BN, int NSUB, int STAGES, class Epi>
 size_t gemm_smem() {
-    return 1024 + (size_t)STAGES * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2);
+    return 1024 + (size_t)STAGES * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2) + 4 * (size_t)Epi::QUAD_STAGE +
+           Epi::RED_BYTES;
 }
 
 template <int BN, int NSUB, int STAGES, class Epi>
-cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, GemmGrid g, const StepIO &io, int sms,
-                        cudaStream_t s) {
+cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
+                        const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s) {
     const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi>();
     static bool attr = false;
     if (!attr) {
@@ -644,7 +787,7 @@ cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, GemmGrid g
     }
     const int tiles = g.m_tiles * g.n_tiles;
     const int grid = tiles < sms ? tiles : sms;
-    k_tc_gemm<BN, NSUB, STAGES, Epi><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, g, io);
+    k_tc_gemm<BN, NSUB, STAGES, Epi><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, mc, mxs, g, io);
     return cudaGetLastError();
 }
 
@@ -727,12 +870,12 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         bg[n] = w->b_lstm[col];
         for (int a = 0; a < A; ++a) wa[(size_t)a * 4 * H + n] = bf(w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
     }
-    // heads: tile j, local dim i, part p, component k -> row j*240 + 3K*i + K*p + k
+    // heads: tile j, local dim i, component k, part p -> row j*240 + DS*i + 3k + p
     const size_t M = (size_t)3 * K * Z;
     for (int d = 0; d < Z; ++d)
         for (int part = 0; part < 3; ++part)
             for (int k = 0; k < K; ++k) {
-                const size_t row = (size_t)(d / dpt) * HEAD_TILE + DS * (d % dpt) + K * part + k;
+                const size_t row = (size_t)(d / dpt) * HEAD_TILE + DS * (d % dpt) + 3 * k + part;
                 const size_t col = (size_t)part * K * Z + (size_t)d * K + k;
                 for (int i = 0; i < H; ++i) wh[row * H + i] = bf(w->W_mdn[(size_t)i * M + col]);
                 bh[row] = w->b_mdn[col];
@@ -792,6 +935,10 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     io.b_ctrl = T.bc; io.b_gate = T.bg; io.b_head = T.bh;
     io.wa = (const __nv_bfloat16 *)T.wa;
     io.dims_per_tile = T.dims_per_tile; io.rd_tile = T.rd_tile; io.rd_col = T.rd_col;
+    io.gates_n_tiles = H / 64;
+    // h (fp32) is read back only by frozen episodes and for h_final: with no way to freeze
+    // during the call it is needed after the last step only
+    io.h32_mode = teacher ? 0 : (c.done_terminates || c.noop_terminates) ? 2 : 1;
     io.nll_part = w.nll_part;
     if (teacher) {
         io.act_in = na->actions; io.z_seq = na->z_seq; io.lengths = na->lengths;
@@ -805,13 +952,18 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     int launches = 0;
     const int init_grid = 1024;
     io.fz_cur = w.fz[0];
-    k_tc_init<<<init_grid, 256, 0, s>>>(io, teacher ? nullptr : ra->z0, teacher ? nullptr : ra->h0,
-                                        teacher ? nullptr : ra->c0, teacher ? nullptr : ra->done0, w.x[0], w.fz[0],
-                                        w.fz[1], T.n_head_tiles);
+    {
+        wm_ktime kt(h, WM_KERNEL_AUX, s);
+        k_tc_init<<<init_grid, 256, 0, s>>>(io, teacher ? nullptr : ra->z0, teacher ? nullptr : ra->h0,
+                                            teacher ? nullptr : ra->c0, teacher ? nullptr : ra->done0, w.x[0],
+                                            w.fz[0], w.fz[1], T.n_head_tiles);
+    }
     ++launches;
-    CUtensorMap mx[2], mwc, mwg, mwh;
+    CUtensorMap mx[2], mxs[2], mwc, mwg, mwh, mc;
     const uint32_t ctrl_box = A > 128 ? 256u : 128u;  // the instantiated BN; rows past A read as zero
     if (!make_map(&mx[0], w.x[0], B, KX, BM) || !make_map(&mx[1], w.x[1], B, KX, BM) ||
+        !make_map(&mxs[0], w.x[0], B, KX, 32) || !make_map(&mxs[1], w.x[1], B, KX, 32) ||
+        !make_map(&mc, w.c, B, H, 32, true) ||
         !make_map(&mwc, T.wc, A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 256) ||
         !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE))
         return cudaErrorInvalidValue;
@@ -826,24 +978,34 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         io.fz_next = w.fz[(t + 1) & 1];
         const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status};
         if (!teacher) {
-            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
-            else if (A > 128) e = launch_gemm<256, 1, 4, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
-            else e = launch_gemm<128, 1, 4, EpiCtrl>(mx[t & 1], mwc, g1, io, T.sms, s);
+            wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
+            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            else if (A > 128) e = launch_gemm<256, 1, 4, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            else e = launch_gemm<128, 1, 4, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
             ++launches;
             if (e != cudaSuccess) break;
         }
         const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
-        e = launch_gemm<256, 1, 4, EpiGates>(mx[t & 1], mwg, g2, io, T.sms, s);
+        {
+            wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
+            e = launch_gemm<256, 1, 3, EpiGates>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s);
+        }
         ++launches;
         if (e != cudaSuccess) break;
         const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
-        e = launch_gemm<HEAD_TILE, 1, 4, EpiHeads>(mx[(t + 1) & 1], mwh, g3, io, T.sms, s);
+        {
+            wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
+            e = launch_gemm<HEAD_TILE, 1, 4, EpiHeads>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
+        }
         ++launches;
     }
     if (e != cudaSuccess) return e;
-    k_tc_finish<<<init_grid, 256, 0, s>>>(B, H, w.h32, w.c, teacher ? nullptr : ra->h_final,
-                                          teacher ? nullptr : ra->c_final, w.nll_part, 4 * T.n_head_tiles,
-                                          teacher ? na->nll : nullptr);
+    {
+        wm_ktime kt(h, WM_KERNEL_AUX, s);
+        k_tc_finish<<<init_grid, 256, 0, s>>>(B, H, w.h32, w.c, teacher ? nullptr : ra->h_final,
+                                              teacher ? nullptr : ra->c_final, w.nll_part, 4 * T.n_head_tiles,
+                                              teacher ? na->nll : nullptr);
+    }
     ++launches;
     h->last_launches = launches;
     return cudaGetLastError();

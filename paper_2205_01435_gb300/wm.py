@@ -5,7 +5,8 @@ module only turns torch tensors into pointers and the call's stream.  There is
 no CPU fallback: if ``libwm.so`` is missing, importing the binding fails.
 
 Names mirror the C entry points: ``wm_create``, ``wm_rollout``, ``wm_mdn_nll``,
-``wm_sync``, ``wm_destroy``, ``wm_last_error``, ``wm_last_path``.  The
+``wm_sync``, ``wm_destroy``, ``wm_last_error``, ``wm_last_path``, ``wm_last_launches``,
+``wm_set_timing``, ``wm_kernel_time``.  The
 ``WorldModel`` class wraps them for convenience.
 """
 from __future__ import annotations
@@ -21,6 +22,8 @@ WM_OK, WM_ERR_INVALID_ARG, WM_ERR_CUDA, WM_ERR_UNSUPPORTED, WM_ERR_TIMEOUT, WM_E
 WM_FP32, WM_BF16 = 0, 1
 PATHS = {"auto": 0, "stepwise": 1, "fused": 2, "tensor": 3}
 PATH_NAMES = {v: k for k, v in PATHS.items()}
+KERNEL_CLASSES = ("step_gemm", "step_cell", "step_sample", "fused", "tc_ctrl", "tc_gates",
+                  "tc_heads", "aux")  # WM_KERNEL_* in order
 
 
 class WMError(RuntimeError):
@@ -74,6 +77,10 @@ def _load():
     lib.wm_last_path.restype = C.c_int
     lib.wm_last_launches.argtypes = [P]
     lib.wm_last_launches.restype = C.c_int
+    lib.wm_set_timing.argtypes = [P, C.c_int]
+    lib.wm_set_timing.restype = C.c_int
+    lib.wm_kernel_time.argtypes = [P, C.c_int, C.POINTER(C.c_double), C.POINTER(C.c_longlong)]
+    lib.wm_kernel_time.restype = C.c_int
     lib.wm_destroy.argtypes = [P]
     lib.wm_destroy.restype = None
     return lib
@@ -157,6 +164,17 @@ def wm_last_path(h) -> str:
 
 def wm_last_launches(h) -> int:
     return int(_lib.wm_last_launches(h))
+
+
+def wm_set_timing(h, enable: bool):
+    _check(h, _lib.wm_set_timing(h, int(bool(enable))), "wm_set_timing")
+
+
+def wm_kernel_time(h, kernel_class: int) -> tuple[float, int]:
+    """(total milliseconds, launches) of one WM_KERNEL_* class since timing was enabled."""
+    ms, n = C.c_double(0.0), C.c_longlong(0)
+    _check(h, _lib.wm_kernel_time(h, int(kernel_class), C.byref(ms), C.byref(n)), "wm_kernel_time")
+    return float(ms.value), int(n.value)
 
 
 def wm_destroy(h):
@@ -252,3 +270,16 @@ class WorldModel:
     @property
     def last_launches(self) -> int:
         return wm_last_launches(self.h)
+
+    def set_timing(self, enable: bool = True):
+        """Bracket every kernel of later calls with CUDA events (clears the totals)."""
+        wm_set_timing(self.h, enable)
+
+    def kernel_times(self) -> dict:
+        """{class name: (total ms, launches)} for the classes that launched since set_timing."""
+        out = {}
+        for i, name in enumerate(KERNEL_CLASSES):
+            ms, n = wm_kernel_time(self.h, i)
+            if n:
+                out[name] = (ms, n)
+        return out

@@ -38,8 +38,18 @@ def test_every_declared_symbol_is_exported(lib):
 def test_binding_loads_and_mirrors_names():
     import paper_2205_01435_gb300 as pkg
     wm = pkg.load()
-    for n in ("wm_create", "wm_rollout", "wm_mdn_nll", "wm_sync", "wm_destroy", "wm_last_path"):
+    for n in ("wm_create", "wm_rollout", "wm_mdn_nll", "wm_sync", "wm_destroy", "wm_last_path",
+              "wm_last_launches", "wm_rollout_noalloc", "wm_set_timing", "wm_kernel_time"):
         assert callable(getattr(wm, n))
+
+
+def test_timing_entry_points_reject_null_handle(lib):
+    lib.wm_set_timing.argtypes = [C.c_void_p, C.c_int]
+    lib.wm_kernel_time.argtypes = [C.c_void_p, C.c_int, C.POINTER(C.c_double), C.POINTER(C.c_longlong)]
+    assert lib.wm_set_timing(None, 1) == 1
+    ms, n = C.c_double(-1.0), C.c_longlong(-1)
+    assert lib.wm_kernel_time(None, 0, C.byref(ms), C.byref(n)) == 1
+    assert ms.value == -1.0 and n.value == -1  # outputs untouched on error
 
 
 def test_invalid_config_rejected_on_host():
