@@ -157,6 +157,17 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def max_over_ranks(value: float, ws: int, device=None) -> float:
+    """The maximum of a per-rank value over all ranks (the slowest rank's time)."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if ws > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -167,7 +178,6 @@ def dist_env():
 def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg):
     """The same rollout through the C ABI with pinned HOST arrays: copies are timed."""
     import torch
-    import torch.distributed as dist
 
     env_steps = B * T * ws
     zh = torch.from_numpy(z0).pin_memory()
@@ -186,10 +196,7 @@ def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg):
         t0 = time.perf_counter()
         model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
         e2e_t.append(time.perf_counter() - t0)
-    e2e_s = torch.tensor([sum(e2e_t) / len(e2e_t)], dtype=torch.float64, device=dev)
-    if ws > 1:
-        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
-    e2e_value = env_steps / float(e2e_s.item())
+    e2e_value = env_steps / max_over_ranks(sum(e2e_t) / len(e2e_t), ws, dev)
     h2d = zh.numel() * 4 + mh.numel() * 4
     d2h = sum(v.numel() * v.element_size() for v in hout.values())
 
@@ -208,7 +215,8 @@ def run_ours(args) -> None:
     torch.cuda.set_device(local)
     wm = pkg.load()
     name = args.workload
-    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=args.batch)
+    # rank r runs shard r of the global batch: its own z0 and masks, Philox episodes r*B + b
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=args.batch, shard=rank)
     if args.path:
         cfg["path"] = args.path
     model = wm.WorldModel(cfg, w, device=local)
@@ -250,11 +258,7 @@ def run_ours(args) -> None:
     times = [a.elapsed_time(b) for a, b in ev]  # ms, each one launch of the step
     kt = model.kernel_times()
     model.set_timing(False)
-    total_ms = sum(times)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if ws > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(times), ws, dev)
     ms_per_step = total_ms / args.steps
     env_steps = B * T * ws
     value = env_steps / (ms_per_step / 1e3)

@@ -16,6 +16,11 @@ available, so these stand in for them.  Recipe (per workload below):
 * teacher-forced sequences: z ~ N(0, 1) for all T+1 frames, actions uniform
   on [0, A).
 
+Sharding: a run over S shards of B episodes (one shard per GPU) draws shard
+r's z_0 and masks from streams of their own; shard 0's are exactly the
+unsharded workload's.  The global batch is the concatenation of the shards,
+global episode r*B + b being episode b of shard r (its Philox episode index).
+
 The five workloads follow the world-model hyper-parameters the paper uses
 (256 hidden units, a handful of Gaussians, Sec. 4.7) scaled to the regimes
 that matter on one GPU.
@@ -50,6 +55,13 @@ def _rng(seed: int, stream: int, sub: int = 0) -> np.random.Generator:
     return np.random.default_rng(np.random.SeedSequence([int(seed), int(stream), int(sub)]))
 
 
+def _shard_rng(seed: int, stream: int, sub: int, shard: int) -> np.random.Generator:
+    """Shard 0 uses the unsharded streams; shard r > 0 a disjoint family of its own."""
+    if shard == 0:
+        return _rng(seed, stream, sub)
+    return _rng(seed, 1000 + stream, int(shard) * 65536 + sub)
+
+
 def model_config(name: str, **over) -> dict:
     """The wm_config-style dict of a workload (sizes, precision, flags)."""
     w = dict(WORKLOADS[name])
@@ -75,8 +87,8 @@ def weights(cfg: dict, seed: int = 0, std: float = 0.05) -> dict:
     return out
 
 
-def z0(B: int, Z: int, seed: int = 0) -> np.ndarray:
-    return _rng(seed, _STREAM["z0"]).standard_normal((B, Z), dtype=np.float32)
+def z0(B: int, Z: int, seed: int = 0, shard: int = 0) -> np.ndarray:
+    return _shard_rng(seed, _STREAM["z0"], 0, shard).standard_normal((B, Z), dtype=np.float32)
 
 
 def pack_mask(valid: np.ndarray) -> np.ndarray:
@@ -91,13 +103,13 @@ def pack_mask(valid: np.ndarray) -> np.ndarray:
     return np.ascontiguousarray(by).view("<u4").astype(np.uint32, copy=False)
 
 
-def mask(T: int, B: int, A: int, density: float, seed: int = 0) -> np.ndarray:
+def mask(T: int, B: int, A: int, density: float, seed: int = 0, shard: int = 0) -> np.ndarray:
     """Bernoulli(density) valid-action bits, packed [T, B, ceil(A/32)] uint32."""
     W = (A + 31) // 32
     out = np.empty((T, B, W), dtype=np.uint32)
     thr = np.float32(density)
     for t in range(T):
-        r = _rng(seed, _STREAM["mask"], t)
+        r = _shard_rng(seed, _STREAM["mask"], t, shard)
         out[t] = pack_mask(r.random((B, A), dtype=np.float32) < thr)
     return out
 
@@ -112,13 +124,15 @@ def teacher_inputs(N: int, T: int, Z: int, A: int, seed: int = 0, ragged: bool =
     return zs, acts, lens
 
 
-def rollout_inputs(name: str, seed: int = 0, B: int | None = None, T: int | None = None):
-    """(cfg, weights, z0, mask, B, T) for a rollout workload."""
+def rollout_inputs(name: str, seed: int = 0, B: int | None = None, T: int | None = None,
+                   shard: int = 0):
+    """(cfg, weights, z0, mask, B, T) for a rollout workload; `shard` picks the shard's
+    episodes (the weights are the same for every shard)."""
     w = WORKLOADS[name]
     cfg = model_config(name)
     B = w["B"] if B is None else B
     T = w["T"] if T is None else T
     wts = weights(cfg, seed)
-    z = z0(B, cfg["z_dim"], seed)
-    m = mask(T, B, cfg["a_dim"], w["mask_density"], seed)
+    z = z0(B, cfg["z_dim"], seed, shard)
+    m = mask(T, B, cfg["a_dim"], w["mask_density"], seed, shard)
     return cfg, wts, z, m, B, T
