@@ -159,6 +159,7 @@ struct EpiCtx {
 // Every thread of a warp issues the same TMEM loads (they are warp-collective);
 // rows past B only skip their memory accesses.
 struct EpiCtrl {
+    static constexpr bool TMA_STAGE = false;
     static constexpr uint32_t QUAD_STAGE = 0;
     static constexpr uint32_t RED_BYTES = 4 * 4 * 32 * 2 * 4;
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
@@ -254,6 +255,7 @@ struct EpiCtrl {
     }
 };
 
+
 // ---- gate epilogue: 64 units per tile, columns [i | f | g | o] x 64; 16 units per group
 // The quadrant's c rows (32 x 64 fp32) and h' rows (32 x 64 bf16) go through
 // shared memory in the 128-byte-swizzled layout of TMA boxes 128 bytes wide,
@@ -267,6 +269,7 @@ struct EpiGates {
     static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
     static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
     static constexpr uint32_t QUAD_STAGE = C_SLAB + X_SLAB;  // c (in place) | h' out
+    static constexpr bool TMA_STAGE = true;
     static constexpr uint32_t RED_BYTES = 0;
 
     // byte offset of (row r, 16-byte chunk j) in a 128-byte-swizzled box
@@ -382,8 +385,15 @@ struct EpiGates {
 };
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
+// Column group g takes the dims of Philox blocks first + g, first + g + 4, ... (4 dims
+// per block), so each block's two draws are made once per row.  The quadrant's z'
+// values are staged in shared memory ([32 rows][33], conflict-free) and stored by all
+// 128 threads in row-major order, so a warp's stores cover a few contiguous row
+// segments instead of 32 rows.
 struct EpiHeads {
-    static constexpr uint32_t QUAD_STAGE = 0;
+    static constexpr bool TMA_STAGE = false;
+    static constexpr int ZS_PITCH = 33;
+    static constexpr uint32_t QUAD_STAGE = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
     static constexpr uint32_t RED_BYTES = 0;
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int) {
@@ -397,124 +407,124 @@ struct EpiHeads {
         const unsigned long long ep = p.ep0 + b;
         const int d0 = n * p.dims_per_tile;
         const int nd = min(p.dims_per_tile, Z - d0);
-        const int per = (nd + 3) / 4;  // dims per column group, contiguous
-        const int i_lo = min(nd, x.cg * per), i_hi = min(nd, i_lo + per);
         const float *bh = p.b_head + (size_t)n * HEAD_TILE;
+        float *zs = reinterpret_cast<float *>(x.stage);
+        const bool draw = !p.teacher && !fz && p.mdn_tau > 0.f;
         float nll = 0.f;
-        u32x4 ru = {0, 0, 0, 0}, rn = {0, 0, 0, 0};
-        int rblock = -1;
-        for (int i = i_lo; i < i_hi; ++i) {
-            const int d = d0 + i;
-            float v[24];
-            {
-                uint32_t r0[8], r1[8], r2[8];
-                TC_LD8(tacc + DS * i, r0);
-                TC_LD8(tacc + DS * i + 8, r1);
-                TC_LD8(tacc + DS * i + 16, r2);  // past the dim when 3K <= 16: unused
-                tc::tmem_ld_wait();
+        for (int blk = (d0 >> 2) + x.cg; 4 * blk < d0 + nd; blk += 4) {  // warp-uniform bounds
+            u32x4 ru = {0, 0, 0, 0}, rn = {0, 0, 0, 0};
+            if (draw) {
+                ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)blk);
+                rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)blk);
+            }
+            const int lo = max(d0, 4 * blk), hi = min(d0 + nd, 4 * blk + 4);
+            for (int d = lo; d < hi; ++d) {
+                const int i = d - d0;
+                float v[24];
+                {
+                    uint32_t r0[8], r1[8], r2[8];
+                    TC_LD8(tacc + DS * i, r0);
+                    TC_LD8(tacc + DS * i + 8, r1);
+                    TC_LD8(tacc + DS * i + 16, r2);  // past the dim when 3K <= 16: unused
+                    tc::tmem_ld_wait();
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    v[j] = __uint_as_float(r0[j]);
-                    v[8 + j] = __uint_as_float(r1[j]);
-                    v[16 + j] = __uint_as_float(r2[j]);
+                    for (int j = 0; j < 8; ++j) {
+                        v[j] = __uint_as_float(r0[j]);
+                        v[8 + j] = __uint_as_float(r1[j]);
+                        v[16 + j] = __uint_as_float(r2[j]);
+                    }
                 }
-            }
-            // columns of a dim are component-interleaved (logit, mu, log sigma) so that every
-            // register index below is static: no local-memory arrays
-            float lg[8], mu[8], ls[8];
-            const float *bhd = bh + DS * i;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                lg[k] = k < K ? v[3 * k] + bhd[3 * k] : -INFINITY;
-                mu[k] = k < K ? v[3 * k + 1] + bhd[3 * k + 1] : 0.f;
-                ls[k] = k < K ? v[3 * k + 2] + bhd[3 * k + 2] : 0.f;
-            }
-            if (!valid) continue;
-            if (p.mdn_seq) {
-                float *ms = p.mdn_seq + tb * M;
-                const bool zero = fz && !p.teacher;
+                // columns of a dim are component-interleaved (logit, mu, log sigma) so that every
+                // register index below is static: no local-memory arrays
+                float lg[8], mu[8], ls[8];
+                const float *bhd = bh + DS * i;
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
-                    if (k < K) {
-                        ms[d * K + k] = zero ? 0.f : lg[k];
-                        ms[KZ + d * K + k] = zero ? 0.f : mu[k];
-                        ms[2 * KZ + d * K + k] = zero ? 0.f : ls[k];
+                    lg[k] = k < K ? v[3 * k] + bhd[3 * k] : -INFINITY;
+                    mu[k] = k < K ? v[3 * k + 1] + bhd[3 * k + 1] : 0.f;
+                    ls[k] = k < K ? v[3 * k + 2] + bhd[3 * k + 2] : 0.f;
+                }
+                if (!valid) continue;
+                if (p.mdn_seq) {
+                    float *ms = p.mdn_seq + tb * M;
+                    const bool zero = fz && !p.teacher;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        if (k < K) {
+                            ms[d * K + k] = zero ? 0.f : lg[k];
+                            ms[KZ + d * K + k] = zero ? 0.f : mu[k];
+                            ms[2 * KZ + d * K + k] = zero ? 0.f : ls[k];
+                        }
                     }
                 }
-            }
-            float zn;
-            if (p.teacher) {
-                const float xv = p.z_seq[((size_t)(p.t + 1) * p.B + b) * Z + d];
-                float mx = -INFINITY;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k]);
-                float s = 0.f;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) if (k < K) s += expf(lg[k] - mx);
-                const float lse = mx + logf(s);
-                float lp[8], tmax = -INFINITY;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    if (k < K) {
-                        const float zs = (xv - mu[k]) * expf(-ls[k]);
-                        lp[k] = (lg[k] - lse) - 0.5f * zs * zs - ls[k] - 0.91893853320467274178f;
-                        tmax = fmaxf(tmax, lp[k]);
-                    }
-                }
-                float acc = 0.f;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) if (k < K) acc += expf(lp[k] - tmax);
-                nll += -(tmax + logf(acc));
-                zn = xv;
-            } else if (fz) {
-                zn = p.z_out[tb * Z + d];
-                if (p.comp_seq) p.comp_seq[tb * Z + d] = 255;
-            } else {
-                int kc = 0;
-                if (!(p.mdn_tau > 0.f)) {
-                    float best = lg[0];
-                    zn = mu[0];
-#pragma unroll
-                    for (int k = 1; k < 8; ++k)
-                        if (k < K && lg[k] > best) { best = lg[k]; kc = k; zn = mu[k]; }
-                } else {
-                    if ((d >> 2) != rblock) {
-                        rblock = d >> 2;
-                        ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)rblock);
-                        rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)rblock);
-                    }
-                    const float itau = __fdividef(1.f, p.mdn_tau);
+                float zn;
+                if (p.teacher) {
+                    const float xv = p.z_seq[((size_t)(p.t + 1) * p.B + b) * Z + d];
                     float mx = -INFINITY;
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k] * itau);
-                    float pk[8], s = 0.f;
+                    for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k]);
+                    float s = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) if (k < K) s += expf(lg[k] - mx);
+                    const float lse = mx + logf(s);
+                    float lp[8], tmax = -INFINITY;
 #pragma unroll
                     for (int k = 0; k < 8; ++k) {
-                        pk[k] = k < K ? __expf(lg[k] * itau - mx) : 0.f;
-                        s += pk[k];
-                    }
-                    const float u = to_uniform(u32x4_get(ru, d & 3)), is = __fdividef(1.f, s);
-                    // first k with u < C_k (the last component when rounding leaves u >= C_{K-2})
-                    kc = K - 1;
-                    float cum = 0.f, muc = 0.f, lsc = 0.f;
-                    bool found = false;
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        if (k < K - 1 && !found) {
-                            cum += pk[k] * is;
-                            if (u < cum) { kc = k; found = true; }
+                        if (k < K) {
+                            const float zsd = (xv - mu[k]) * expf(-ls[k]);
+                            lp[k] = (lg[k] - lse) - 0.5f * zsd * zsd - ls[k] - 0.91893853320467274178f;
+                            tmax = fmaxf(tmax, lp[k]);
                         }
-                        if (k == kc) { muc = mu[k]; lsc = ls[k]; }
                     }
-                    const int pair = (d & 3) >> 1;
-                    const float eps = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
-                    const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
-                    zn = muc + __expf(lsc) * scale * eps;
+                    float acc = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) if (k < K) acc += expf(lp[k] - tmax);
+                    nll += -(tmax + logf(acc));
+                    zn = xv;
+                } else if (fz) {
+                    zn = p.z_out[tb * Z + d];
+                    if (p.comp_seq) p.comp_seq[tb * Z + d] = 255;
+                } else {
+                    int kc = 0;
+                    if (!(p.mdn_tau > 0.f)) {
+                        float best = lg[0];
+                        zn = mu[0];
+#pragma unroll
+                        for (int k = 1; k < 8; ++k)
+                            if (k < K && lg[k] > best) { best = lg[k]; kc = k; zn = mu[k]; }
+                    } else {
+                        const float itau = __fdividef(1.f, p.mdn_tau);
+                        float mx = -INFINITY;
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k] * itau);
+                        float pk[8], s = 0.f;
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) {
+                            pk[k] = k < K ? __expf(lg[k] * itau - mx) : 0.f;
+                            s += pk[k];
+                        }
+                        const float u = to_uniform(u32x4_get(ru, d & 3)), is = __fdividef(1.f, s);
+                        // first k with u < C_k (the last component when rounding leaves u >= C_{K-2})
+                        kc = K - 1;
+                        float cum = 0.f, muc = 0.f, lsc = 0.f;
+                        bool found = false;
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) {
+                            if (k < K - 1 && !found) {
+                                cum += pk[k] * is;
+                                if (u < cum) { kc = k; found = true; }
+                            }
+                            if (k == kc) { muc = mu[k]; lsc = ls[k]; }
+                        }
+                        const int pair = (d & 3) >> 1;
+                        const float eps = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
+                        const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
+                        zn = muc + __expf(lsc) * scale * eps;
+                    }
+                    if (p.comp_seq) p.comp_seq[tb * Z + d] = (uint8_t)kc;
                 }
-                if (p.comp_seq) p.comp_seq[tb * Z + d] = (uint8_t)kc;
+                zs[x.lane * ZS_PITCH + i] = zn;
             }
-            if (!p.teacher) p.z_out[(tb + p.B) * Z + d] = zn;
-            p.x_next[(size_t)b * KX + d] = __float2bfloat16_rn(zn);
         }
         if (p.teacher && valid) {
             const int len = p.lengths ? p.lengths[b] : p.T;
@@ -535,6 +545,17 @@ struct EpiHeads {
                 p.fz_next[b] = (fz || (p.done_terminates && dl > 0.f) || noop) ? 1 : 0;
             }
         }
+        // the quadrant's 32 x nd block of z', stored row-major by its 128 threads
+        x.sync();
+        const int y0 = m * BM + 32 * x.quad, nrow = min(32, p.B - y0);
+        for (int e = x.cg * 32 + x.lane; e < nrow * nd; e += 128) {
+            const int rr = e / nd, i = e - rr * nd;
+            const size_t bb = (size_t)(y0 + rr);
+            const float zn = zs[rr * ZS_PITCH + i];
+            if (!p.teacher) p.z_out[((size_t)(p.t + 1) * p.B + bb) * Z + d0 + i] = zn;
+            p.x_next[bb * KX + d0 + i] = __float2bfloat16_rn(zn);
+        }
+        x.sync();  // the staging may be rewritten by the next tile
     }
 };
 
@@ -661,7 +682,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x.status = g.status;
         int acc = 0;
         uint32_t acc_phase = 0;
-        if (Epi::QUAD_STAGE > 0 && x.leader && (int)blockIdx.x < ntiles)
+        if (Epi::TMA_STAGE && x.leader && (int)blockIdx.x < ntiles)
             Epi::prefetch(io, blockIdx.x / g.n_tiles, blockIdx.x % g.n_tiles, x);
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
             const int m = tile / g.n_tiles, n = tile % g.n_tiles;
@@ -683,7 +704,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 acc_phase ^= 1u;
             }
         }
-        if (Epi::QUAD_STAGE > 0 && x.leader) {
+        if (Epi::TMA_STAGE && x.leader) {
             bulk_wait_all();  // the TMA stores have completed
             // after an abort a prefetch may still be in flight: let it land before the CTA exits
             if (x.pending) tc::mbar_wait_bounded(x.stage_bar, x.pending_phase, POLLS);

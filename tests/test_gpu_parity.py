@@ -323,7 +323,10 @@ def test_fused_matches_stepwise_closely(wm):
                                         ("small_bf16", dict(mdn_tau=0.0)),
                                         ("small_bf16", dict(mdn_tau=0.6, sigma_sqrt_tau=1,
                                                             noop_terminates=1, done_terminates=1)),
-                                        ("mid_bf16", dict(ctrl_sample=1, ctrl_tau=0.7))])
+                                        ("mid_bf16", dict(ctrl_sample=1, ctrl_tau=0.7)),
+                                        # column groups starting mid-word of the action mask
+                                        ("small_bf16", dict(a_dim=192, ctrl_sample=1, ctrl_tau=0.8)),
+                                        ("small_bf16", dict(a_dim=64))])
 def test_tensor_against_oracle(wm, orc, name, flags):
     """Two row tiles (the second partly filled), resumed state, offsets, flags."""
     cfg = dict(synth.model_config(name), **flags)
