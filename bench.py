@@ -299,6 +299,15 @@ def run_ours(args) -> None:
             "algorithmic_flops_per_launch": fl,
             "kernel_shares": {k: round(v[0] / all_ms, 4) for k, v in sorted(kt.items())}}
 
+    live = None
+    if cfg.get("done_terminates") or cfg.get("noop_terminates"):
+        # episode b is live at step t unless it was done at an earlier step (then frozen)
+        d = out["done"].to(torch.int32)
+        frozen = torch.zeros_like(d)
+        frozen[1:] = (torch.cumsum(d, dim=0)[:-1] > 0).to(torch.int32)
+        live_steps = int((frozen == 0).sum().item()) * ws
+        live = {"live_env_steps_per_s": round(live_steps / (ms_per_step / 1e3), 1),
+                "live_fraction": round(live_steps / (B * T * ws), 4)}
     line = {"metric": "dream env-steps/s (wm_rollout)", "value": round(value, 1),
             "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
@@ -316,6 +325,8 @@ def run_ours(args) -> None:
              "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches * args.steps,
             "roofline": roof, "clocks": clk.summary()}
+    if live is not None:
+        line["live_steps"] = live  # frozen (done) episode-steps are executed but not live
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes)
     if rank == 0:
@@ -333,6 +344,8 @@ def oracle_episodes(name: str, flop_budget: float) -> int:
 
 
 def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) -> dict:
+    """The oracle on the host cores (all of them), plus a one-thread figure on a tenth of the
+    sample (episodes are independent, so throughput per episode-step is comparable)."""
     import oracle
 
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
@@ -341,9 +354,15 @@ def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) ->
     t0 = time.perf_counter()
     oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
     dt = time.perf_counter() - t0
+    n1 = max(1, n // 10)
+    t1 = time.perf_counter()
+    oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1)
+    dt1 = time.perf_counter() - t1
     return {"value": round(n * T / dt, 2), "unit": "env-steps/s", "cores": threads,
             "kind": "oracle", "sample": f"{n} of {B} episodes x {T} steps of {name}, "
-                                        f"{threads} threads, {dt:.1f} s"}
+                                        f"{threads} threads, {dt:.1f} s",
+            "value_1thread": round(n1 * T / dt1, 2),
+            "sample_1thread": f"{n1} episodes x {T} steps, 1 thread, {dt1:.1f} s"}
 
 
 def run_reference(args) -> None:
