@@ -560,33 +560,34 @@ struct EpiHeads {
 };
 
 // ---------------------------------------------------------------------------
-// The persistent warp-specialised GEMM.  TILE_N = BN * NSUB columns per tile.
-template <int BN, int NSUB, int STAGES, class Epi>
+// The persistent warp-specialised GEMM.  TILE_N = BN * NSUB columns per tile.  A ring
+// stage holds KPS k-steps of BK: the MMA thread waits for a stage once and issues all its
+// MMAs back to back (any wait on the issuing thread lets the tensor pipe drain), and each
+// k-step of a stage has its own "empty" barrier so that refills still go k-step by k-step.
+template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmXs, GemmGrid g,
               StepIO io) {
     constexpr int TILE_N = BN * NSUB;
     constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BN * BK * 2, B_BYTES = B_SUB * NSUB;
-    constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    constexpr uint32_t KSTEP_BYTES = A_BYTES + B_BYTES, STAGE_BYTES = KPS * KSTEP_BYTES;
     constexpr int NACC = TILE_N <= 256 ? 2 : 1;
     constexpr uint32_t ACC_COLS = 256;
     static_assert(BN % 16 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4];
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES * KPS], bar_accf[2], bar_acce[2], bar_stage[4];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t smem_u = tc::smem_u32(smem);
     auto full_b = [&](int s) { return tc::smem_u32(&bar_full[s]); };
-    auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };
+    auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };  // s = stage * KPS + k-step
 
     if (tid == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            tc::mbar_init(full_b(s), 1);
-            tc::mbar_init(empty_b(s), 1);
-        }
+        for (int s = 0; s < STAGES; ++s) tc::mbar_init(full_b(s), 1);
+        for (int s = 0; s < STAGES * KPS; ++s) tc::mbar_init(empty_b(s), 1);
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(tc::smem_u32(&bar_accf[a]), 1);
             tc::mbar_init(tc::smem_u32(&bar_acce[a]), EPI_WARPS * 32);
@@ -614,15 +615,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             uint32_t phase = 0;
             for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
                 const int m = tile / g.n_tiles, n = tile % g.n_tiles;
-                for (int ks = 0; ks < g.k_steps; ++ks) {
-                    wait(empty_b(stage), phase ^ 1u);
-                    if (s_abort) break;
-                    const uint32_t sa = smem_u + stage * STAGE_BYTES;
-                    tc::mbar_arrive_expect_tx(full_b(stage), STAGE_BYTES);
-                    tma_load_2d(sa, &tmA, g.a_col0 + ks * BK, m * BM, full_b(stage));
+                for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
+                    const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;  // k-steps in this stage
+                    for (int h = 0; h < nk; ++h) {
+                        const int ks = ks0 + h;
+                        wait(empty_b(stage * KPS + h), phase ^ 1u);
+                        if (s_abort) break;
+                        const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
+                        if (h == 0) tc::mbar_arrive_expect_tx(full_b(stage), nk * KSTEP_BYTES);
+                        tma_load_2d(sa, &tmA, g.a_col0 + ks * BK, m * BM, full_b(stage));
 #pragma unroll
-                    for (int s = 0; s < NSUB; ++s)
-                        tma_load_2d(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN, full_b(stage));
+                        for (int s = 0; s < NSUB; ++s)
+                            tma_load_2d(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN, full_b(stage));
+                    }
+                    if (s_abort) break;
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
             }
@@ -636,20 +642,24 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 wait(tc::smem_u32(&bar_acce[acc]), acc_phase ^ 1u);
                 tc::fence_after_sync();
                 const uint32_t dcol = tm + acc * ACC_COLS;
-                for (int ks = 0; ks < g.k_steps; ++ks) {
+                for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
+                    const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;
                     wait(full_b(stage), phase);
                     if (s_abort) break;
                     tc::fence_after_sync();
-                    const uint32_t sa = smem_u + stage * STAGE_BYTES;
+                    for (int h = 0; h < nk; ++h) {
+                        const int ks = ks0 + h;
+                        const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk) {
-                        const uint64_t da = desc_sw128(sa + 32 * kk);
+                        for (int kk = 0; kk < BK / 16; ++kk) {
+                            const uint64_t da = desc_sw128(sa + 32 * kk);
 #pragma unroll
-                        for (int s = 0; s < NSUB; ++s)
-                            tc::mma_bf16(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
-                                         (ks > 0 || kk > 0) ? 1u : 0u);
+                            for (int s = 0; s < NSUB; ++s)
+                                tc::mma_bf16(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
+                                             (ks > 0 || kk > 0) ? 1u : 0u);
+                        }
+                        tc::mma_commit(empty_b(stage * KPS + h));  // this k-step's slot is free once its MMAs are done
                     }
-                    tc::mma_commit(empty_b(stage));  // the stage is free once these MMAs are done
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 tc::mma_commit(tc::smem_u32(&bar_accf[acc]));
@@ -789,26 +799,26 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, ui
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int NSUB, int STAGES, class Epi>
+template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 size_t gemm_smem() {
-    return 1024 + (size_t)STAGES * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2) + 4 * (size_t)Epi::QUAD_STAGE +
+    return 1024 + (size_t)STAGES * KPS * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2) + 4 * (size_t)Epi::QUAD_STAGE +
            Epi::RED_BYTES;
 }
 
-template <int BN, int NSUB, int STAGES, class Epi>
+template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
                         const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s) {
-    const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi>();
+    const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi, KPS>();
     static bool attr = false;
     if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN, NSUB, STAGES, Epi>,
+        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN, NSUB, STAGES, Epi, KPS>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         attr = true;
     }
     const int tiles = g.m_tiles * g.n_tiles;
     const int grid = tiles < sms ? tiles : sms;
-    k_tc_gemm<BN, NSUB, STAGES, Epi><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, mc, mxs, g, io);
+    k_tc_gemm<BN, NSUB, STAGES, Epi, KPS><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, mc, mxs, g, io);
     return cudaGetLastError();
 }
 
@@ -1016,7 +1026,8 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
-            e = launch_gemm<HEAD_TILE, 1, 4, EpiHeads>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
+            // two k-steps per stage: half the waits on the MMA-issuing thread (same ring bytes)
+            e = launch_gemm<HEAD_TILE, 1, 2, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
         }
         ++launches;
     }
