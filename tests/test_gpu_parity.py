@@ -207,6 +207,28 @@ def test_empty_and_zero_length(wm):
     assert n["nll"].numel() == 0
 
 
+@pytest.mark.parametrize("path", ["fused", "tensor"])
+def test_empty_and_zero_length_on_each_family(wm, path):
+    """B = 0, T = 0 (state passes through unchanged) and N = 0 / T = 0 scoring on the
+    fused and tensor-core families, which the small tiny_fp32 case above does not reach."""
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=40, T=3)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0[:0]), T, mask=_cuda(mask[:, :0]))
+    torch.cuda.synchronize()
+    assert g["z"].shape == (T + 1, 0, cfg["z_dim"])
+    h0 = torch.randn(B, cfg["h_dim"], device="cuda")
+    c0 = torch.randn(B, cfg["h_dim"], device="cuda")
+    g = m.rollout(_cuda(z0), 0, h0=h0, c0=c0)
+    torch.cuda.synchronize()
+    assert torch.equal(g["z"][0].cpu(), torch.from_numpy(z0))
+    assert torch.equal(g["h_final"], h0) and torch.equal(g["c_final"], c0)
+    zs = np.zeros((1, 4, cfg["z_dim"]), np.float32)
+    n = m.mdn_nll(_cuda(zs), _cuda(np.zeros((0, 4), np.int32)))
+    torch.cuda.synchronize()
+    assert torch.equal(n["nll"].cpu(), torch.zeros(4))
+    m.sync()
+
+
 def test_invalid_arguments(wm):
     cfg, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
     m = wm.WorldModel(cfg, w)
