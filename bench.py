@@ -74,19 +74,31 @@ KERNELS = {"fused": ("k_fused", "wm_fused.cu"),
            "step_sample": ("k_sample", "wm_step.cu")}
 
 
+def nll_flops_per_step(cfg: dict) -> float:
+    """Algorithmic FLOPs of one teacher-forced (sequence, step): gates and mixture head."""
+    Z, H, K = cfg["z_dim"], cfg["h_dim"], cfg["k_mix"]
+    return 2.0 * ((Z + H) * 4 * H + H * (3 * K * Z + 2))
+
+
+def nll_inputs(cfg: dict, rank: int = 0):
+    """(z_seq, actions) of the scoring workload; rank r scores its own sequences."""
+    w = synth.WORKLOADS["nll"]
+    return synth.teacher_inputs(w["N"], w["T"], cfg["z_dim"], cfg["a_dim"], seed=rank)[:2]
+
+
 def kernel_flops(cls: str, cfg: dict, B: int, T: int, launches: int) -> float:
     """Algorithmic FLOPs of one launch of a kernel class (its contraction)."""
     Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
     if cls == "fused":
-        return flops_per_env_step(cfg) * B * T
+        return (nll_flops_per_step(cfg) if cfg.get("teacher") else flops_per_env_step(cfg)) * B * T
     if cls == "tc_ctrl":
         return 2.0 * B * (Z + H) * A
     if cls == "tc_gates":
         return 2.0 * B * (Z + H) * 4 * H
     if cls == "tc_heads":
         return 2.0 * B * H * (3 * K * Z + 2)
-    if cls == "step_gemm":  # two GEMMs per step: gates + controller, then heads
-        return 2.0 * B * ((Z + H) * (4 * H + A) + H * (3 * K * Z + 2)) / 2
+    if cls == "step_gemm":  # two GEMMs per step: gates (+ controller), then heads
+        return 2.0 * B * ((Z + H) * (4 * H + (0 if cfg.get("teacher") else A)) + H * (3 * K * Z + 2)) / 2
     return 0.0
 
 
@@ -203,6 +215,116 @@ def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg):
     return e2e_value, h2d, d2h
 
 
+def kernel_timing_pass(model, step, flush, stream, steps: int) -> dict:
+    import torch
+
+    torch.cuda.synchronize()
+    model.set_timing(True)
+    for i in range(steps):
+        flush.fill_(float(i))
+        step()
+    torch.cuda.synchronize()
+    kt = model.kernel_times()
+    model.set_timing(False)
+    return kt
+
+
+def run_nll(args) -> None:
+    """Teacher-forced scoring (wm_mdn_nll) of the nll workload: scored (sequence, step)
+    pairs per second, same timing, e2e, roofline and CPU-baseline rules as the rollouts."""
+    import torch
+
+    import paper_2205_01435_gb300 as pkg
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    wm = pkg.load()
+    cfg = synth.model_config("nll", precision=args.precision or "bf16")
+    if args.path:
+        cfg["path"] = args.path
+    w = synth.weights(cfg)
+    zs, acts = nll_inputs(cfg, rank)
+    T, N = acts.shape
+    model = wm.WorldModel(cfg, w, device=local)
+    dev = torch.device("cuda", local)
+    zc, ac = torch.from_numpy(zs).to(dev), torch.from_numpy(acts).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    for _ in range(args.warmup):
+        model.mdn_nll(zc, ac, stream=stream)
+    torch.cuda.synchronize()
+    path_name, launches = model.last_path, model.last_launches
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            ev[i][0].record(stream)
+            model.mdn_nll(zc, ac, stream=stream)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+    kt = kernel_timing_pass(model, lambda: model.mdn_nll(zc, ac, stream=stream), flush, stream, args.steps)
+    ms_per_step = max_over_ranks(sum(a.elapsed_time(b) for a, b in ev), ws, dev) / args.steps
+    value = N * T * ws / (ms_per_step / 1e3)
+    # e2e: pinned host inputs and output
+    zh, ah = torch.from_numpy(zs).pin_memory(), torch.from_numpy(acts).pin_memory()
+    model.mdn_nll(zh, ah)
+    e2e_t = []
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        r = model.mdn_nll(zh, ah)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_value = N * T * ws / max_over_ranks(sum(e2e_t) / len(e2e_t), ws, dev)
+    peaks = load_peaks()
+    tcfg = dict(cfg, teacher=1)
+    timed = {k: v for k, v in kt.items() if k in KERNELS}
+    dom = max(timed, key=lambda k: timed[k][0])
+    dom_ms, dom_n = timed[dom]
+    fl = kernel_flops(dom, tcfg, N, T, dom_n)
+    achieved = fl / (dom_ms / dom_n / 1e3) / 1e12
+    if cfg["precision"] == "bf16" and dom in ("fused", "tc_gates", "tc_heads"):
+        bound, peak, psrc = "tensor", peaks["bf16_tflops"], peaks["source"] + " bf16 burst"
+    else:
+        bound, peak, psrc = "alu", fp32_simt_peak_tflops(), "derived: 152 SM x 128 fp32 FMA x 2 FLOP x 2.07 GHz"
+    kname, ksrc = KERNELS[dom]
+    call_fl = nll_flops_per_step(cfg) * N * T
+    roof = {"bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 5),
+            "traffic": ncu_traffic(f"{kname}/nll_{cfg['precision']}", kernel_source_sha(ksrc)),
+            "peak_source": psrc, "kernel": f"{kname}/nll_{cfg['precision']}",
+            "launch_ms": round(dom_ms / dom_n, 5), "launches": dom_n, "algorithmic_flops_per_launch": fl,
+            "kernel_shares": {k: round(v[0] / sum(x[0] for x in kt.values()), 4) for k, v in sorted(kt.items())},
+            "call_frac_of_tensor_roofline": round(call_fl / (ms_per_step / 1e3) / 1e12 / peaks["bf16_tflops"], 5)}
+    line = {"metric": "teacher-forced scored steps/s (wm_mdn_nll)", "value": round(value, 1),
+            "unit": "scored-steps/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if cfg["precision"] == "bf16" else "f32",
+            "data": "synthetic (seeded: weights N(0,0.05^2), z ~ N(0,1), actions uniform)",
+            "config": {"workload": f"nll_{cfg['precision']}", "N": N, "T": T, "z": cfg["z_dim"],
+                       "A": cfg["a_dim"], "H": cfg["h_dim"], "K": cfg["k_mix"], "kernel_path": path_name,
+                       "l2": "flushed between timed steps (512 MiB write)",
+                       "parallelism": f"sequences sharded over {ws} GPU(s), no collective"},
+            "e2e": {"value": round(e2e_value, 1), "unit": "scored-steps/s",
+                    "h2d_bytes_per_step": zh.numel() * 4 + ah.numel() * 4, "d2h_bytes_per_step": N * 4},
+            "gpu_launches": launches * args.steps, "roofline": roof, "clocks": clk.summary()}
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        import oracle
+        n = max(8, min(N, args.cpu_episodes or N // 4))
+        threads = os.cpu_count() or 1
+        t0 = time.perf_counter()
+        oracle.mdn_nll(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": round(n * T / dt, 2), "unit": "scored-steps/s", "cores": threads,
+                                "kind": "oracle", "sample": f"{n} of {N} sequences x {T} steps, {threads} threads, {dt:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+
+
 def run_ours(args) -> None:
     import torch
     import torch.distributed as dist
@@ -240,7 +362,6 @@ def run_ours(args) -> None:
     torch.cuda.synchronize()
     path_name = model.last_path
     launches = model.last_launches
-    model.set_timing(True)  # each kernel bracketed by CUDA events on the launching stream
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -256,8 +377,10 @@ def run_ours(args) -> None:
     if ws > 1:
         dist.barrier()
     times = [a.elapsed_time(b) for a, b in ev]  # ms, each one launch of the step
-    kt = model.kernel_times()
-    model.set_timing(False)
+    # per-kernel durations: a second, identical timed pass with every kernel bracketed by CUDA
+    # events on the launching stream (kept out of the pass above: the extra event records slow
+    # calls made of many short launches)
+    kt = kernel_timing_pass(model, step, flush, stream, args.steps)
     total_ms = max_over_ranks(sum(times), ws, dev)
     ms_per_step = total_ms / args.steps
     env_steps = B * T * ws
@@ -372,6 +495,36 @@ def run_reference(args) -> None:
     import oracle
 
     name = args.workload
+    if name == "nll":
+        cfg = synth.model_config("nll", precision=args.precision or "bf16")
+        w = synth.weights(cfg)
+        zs, acts = nll_inputs(cfg)
+        T, N = acts.shape
+        n = max(8, min(N, args.ref_episodes or N // 16))
+        threads = os.cpu_count() or 1
+        for _ in range(args.warmup):
+            oracle.mdn_nll(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+        times = []
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            oracle.mdn_nll(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+            times.append(time.perf_counter() - t0)
+        per = sum(times) / len(times)
+        value = n * T / per
+        line = {"impl": "reference", "metric": "teacher-forced scored steps/s (wm_mdn_nll)",
+                "value": round(value, 2), "unit": "scored-steps/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": round(per * 1e3, 3), "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None,
+                "dtype": "f64 (bf16 operand emulation)" if cfg["precision"] == "bf16" else "f64",
+                "data": "synthetic (seeded: weights N(0,0.05^2), z ~ N(0,1), actions uniform)",
+                "config": {"workload": f"nll_{cfg['precision']}", "N": N, "T": T, "z": cfg["z_dim"],
+                           "A": cfg["a_dim"], "H": cfg["h_dim"], "K": cfg["k_mix"]},
+                "cpu_baseline": {"value": round(value, 2), "unit": "scored-steps/s", "cores": threads,
+                                 "kind": "oracle", "sample": f"{n} of {N} sequences x {T} steps, {threads} threads"},
+                "e2e": {"value": round(value, 2), "unit": "scored-steps/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
     n = min(args.ref_episodes or oracle_episodes(name, 2e10), B)
     threads = os.cpu_count() or 1
@@ -406,8 +559,10 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="small_bf16",
-                    choices=[k for k in synth.WORKLOADS if k != "nll"])
+    ap.add_argument("--workload", default="small_bf16", choices=list(synth.WORKLOADS),
+                    help="a rollout workload, or nll (teacher-forced scoring)")
+    ap.add_argument("--precision", choices=["fp32", "bf16"], default=None,
+                    help="nll workload only: fp32 or bf16 path (default bf16)")
     ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer leg (profiling runs)")
@@ -422,6 +577,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "nll":
+        run_nll(args)
     else:
         run_ours(args)
 
