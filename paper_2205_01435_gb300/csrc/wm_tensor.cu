@@ -59,6 +59,41 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         :: "r"(dst), "l"(map), "r"(x), "r"(y), "r"(mbar) : "memory");
 }
 
+// ---- CTA-pair (2-SM) forms: a pair computes a 256-row tile with one MMA stream issued
+// by the leader CTA (cluster rank 0); each CTA holds its 128 rows of A and half of the B
+// rows in its shared memory, and its 128 accumulator rows in its own TMEM.
+__device__ __forceinline__ void tma_load_2sm(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                             uint32_t mbar_cluster) {  // completes on the leader's mbarrier
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        :: "r"(dst), "l"(map), "r"(x), "r"(y), "r"(mbar_cluster) : "memory");
+}
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+// arrive (once) on the mbarrier at this shared-memory offset in both CTAs of the pair when
+// the leader's MMAs issued so far have completed
+__device__ __forceinline__ void mma_commit_pair(uint32_t mbar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+        :: "r"(mbar), "h"((uint16_t)0x3) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_saddr, uint32_t ncols) {  // a warp of each CTA
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" :: "r"(dst_saddr), "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t mbar_cluster) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" :: "r"(mbar_cluster) : "memory");
+}
+
 // TMA store of a box from shared memory (bulk-group completion).
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x, int y, uint32_t src) {
     asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
@@ -104,7 +139,6 @@ struct StepIO {
     const __nv_bfloat16 *wa;        // [A, 4H] gate-tile column order
     // head tiles
     int dims_per_tile, rd_tile, rd_col;  // reward / done columns: tile, first column
-    int gates_n_tiles;                   // H / 64
     // inputs / outputs
     const uint32_t *mask;           // [T, B, W] or null
     const int32_t *act_in;          // teacher: [T, B]
@@ -163,7 +197,7 @@ struct EpiCtrl {
     static constexpr uint32_t QUAD_STAGE = 0;
     static constexpr uint32_t RED_BYTES = 4 * 4 * 32 * 2 * 4;
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int) {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int, int) {
         (void)n;
         const int b = m * BM + x.row;
         const bool valid = b < p.B;
@@ -275,6 +309,7 @@ struct EpiGates {
     // byte offset of (row r, 16-byte chunk j) in a 128-byte-swizzled box
     static __device__ __forceinline__ uint32_t sw(int r, int j) { return r * 128 + ((j ^ (r & 7)) << 4); }
 
+    // leader of a quadrant: TMA load of the c rows of 128-row block m, unit tile n
     static __device__ void prefetch(const StepIO &, int m, int n, EpiCtx &x) {
         x.note_prefetch();
         tc::mbar_arrive_expect_tx(x.stage_bar, C_SLAB);
@@ -282,7 +317,7 @@ struct EpiGates {
             tma_load_2d(x.stage_u + bx * 4096, x.tm_c, 64 * n + 32 * bx, m * BM + 32 * x.quad, x.stage_bar);
     }
 
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int next) {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int next_m, int next_n) {
         const int b = m * BM + x.row;
         const bool valid = b < p.B;
         const int bb = valid ? b : 0;  // rows past B compute on row 0; TMA stores clip them
@@ -379,7 +414,7 @@ struct EpiGates {
                 bulk_commit();
                 bulk_wait_read();  // the slab may be refilled
             }
-            if (next >= 0) prefetch(p, next / p.gates_n_tiles, next % p.gates_n_tiles, x);
+            if (next_m >= 0) prefetch(p, next_m, next_n, x);
         }
     }
 };
@@ -396,7 +431,7 @@ struct EpiHeads {
     static constexpr uint32_t QUAD_STAGE = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
     static constexpr uint32_t RED_BYTES = 0;
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int) {
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int, int) {
         const int b0 = m * BM + x.row;
         const bool valid = b0 < p.B;
         const int b = valid ? b0 : 0;  // rows past B compute on row 0 and store nothing
@@ -560,48 +595,54 @@ struct EpiHeads {
 };
 
 // ---------------------------------------------------------------------------
-// The persistent warp-specialised GEMM.  TILE_N = BN * NSUB columns per tile.  A ring
-// stage holds KPS k-steps of BK: the MMA thread waits for a stage once and issues all its
-// MMAs back to back (any wait on the issuing thread lets the tensor pipe drain), and each
-// k-step of a stage has its own "empty" barrier so that refills still go k-step by k-step.
+// The persistent warp-specialised GEMM on CTA pairs.  A pair computes 256-row tiles of
+// TILE_N = BN * NSUB columns with M = 256 tcgen05 MMAs (cta_group::2) issued by the leader
+// CTA: each CTA loads its 128 rows of A and BN/2 rows of each BN-wide slice of B, and runs
+// the epilogue on its own 128 accumulator rows.  (One M = 256 MMA does twice the work of an
+// M = 128 one in about 0.6 of its time, per SM.)  A ring stage holds KPS k-steps of BK: the
+// MMA thread waits for a stage once and issues all its MMAs back to back (any wait on the
+// issuing thread lets the tensor pipe drain), and each k-step has its own "empty" barrier so
+// that refills still go k-step by k-step.
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmXs, GemmGrid g,
               StepIO io) {
-    constexpr int TILE_N = BN * NSUB;
-    constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BN * BK * 2, B_BYTES = B_SUB * NSUB;
-    constexpr uint32_t KSTEP_BYTES = A_BYTES + B_BYTES, STAGE_BYTES = KPS * KSTEP_BYTES;
+    constexpr int TILE_N = BN * NSUB, BNH = BN / 2;
+    constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BNH * BK * 2, B_BYTES = B_SUB * NSUB;
+    constexpr uint32_t KSTEP_BYTES = A_BYTES + B_BYTES, STAGE_BYTES = KPS * KSTEP_BYTES;  // per CTA
     constexpr int NACC = TILE_N <= 256 ? 2 : 1;
     constexpr uint32_t ACC_COLS = 256;
-    static_assert(BN % 16 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
+    static_assert(BN % 16 == 0 && BNH % 8 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES * KPS], bar_accf[2], bar_acce[2], bar_stage[4];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t rank = tc::cluster_rank();  // 0: the pair's leader
+    const int pair = (int)(blockIdx.x >> 1), npairs = (int)(gridDim.x >> 1);
     const uint32_t smem_u = tc::smem_u32(smem);
     auto full_b = [&](int s) { return tc::smem_u32(&bar_full[s]); };
     auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };  // s = stage * KPS + k-step
 
     if (tid == 0) {
-        for (int s = 0; s < STAGES; ++s) tc::mbar_init(full_b(s), 1);
-        for (int s = 0; s < STAGES * KPS; ++s) tc::mbar_init(empty_b(s), 1);
+        for (int s = 0; s < STAGES; ++s) tc::mbar_init(full_b(s), 1);             // the leader's: both CTAs' bytes
+        for (int s = 0; s < STAGES * KPS; ++s) tc::mbar_init(empty_b(s), 1);      // the leader's commit, multicast
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(tc::smem_u32(&bar_accf[a]), 1);
-            tc::mbar_init(tc::smem_u32(&bar_acce[a]), EPI_WARPS * 32);
+            tc::mbar_init(tc::smem_u32(&bar_acce[a]), 2 * EPI_WARPS);  // the leader's: both CTAs' warps
         }
         for (int q = 0; q < 4; ++q) tc::mbar_init(tc::smem_u32(&bar_stage[q]), 1);
         tc::fence_mbar_init();
         s_abort = 0;
     }
-    if (warp == 1) tc::tmem_alloc(tc::smem_u32(&tmem_base), 512);
+    if (warp == 1) tmem_alloc_pair(tc::smem_u32(&tmem_base), 512);
     tc::fence_before_sync();
-    __syncthreads();
+    tc::cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrive
     tc::fence_after_sync();
     const uint32_t tm = tmem_base;
-    const int ntiles = g.m_tiles * g.n_tiles;
+    const int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
     auto wait = [&](uint32_t bar, uint32_t parity) {
         if (!s_abort && !tc::mbar_wait_bounded(bar, parity, POLLS)) {
             s_abort = 1;
@@ -610,23 +651,25 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     };
 
     if (warp == 0) {
-        if (lane == 0) {  // ---- TMA producer
+        if (lane == 0) {  // ---- TMA producer (both CTAs)
             int stage = 0;
             uint32_t phase = 0;
-            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+            for (int tile = pair; tile < ntiles; tile += npairs) {
                 const int m = tile / g.n_tiles, n = tile % g.n_tiles;
                 for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
                     const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;  // k-steps in this stage
+                    const uint32_t full_ldr = tc::map_rank(full_b(stage), 0);
                     for (int h = 0; h < nk; ++h) {
                         const int ks = ks0 + h;
                         wait(empty_b(stage * KPS + h), phase ^ 1u);
                         if (s_abort) break;
                         const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
-                        if (h == 0) tc::mbar_arrive_expect_tx(full_b(stage), nk * KSTEP_BYTES);
-                        tma_load_2d(sa, &tmA, g.a_col0 + ks * BK, m * BM, full_b(stage));
+                        if (h == 0 && rank == 0) tc::mbar_arrive_expect_tx(full_b(stage), 2 * nk * KSTEP_BYTES);
+                        tma_load_2sm(sa, &tmA, g.a_col0 + ks * BK, (2 * m + (int)rank) * BM, full_ldr);
 #pragma unroll
                         for (int s = 0; s < NSUB; ++s)
-                            tma_load_2d(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN, full_b(stage));
+                            tma_load_2sm(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN + (int)rank * BNH,
+                                         full_ldr);
                     }
                     if (s_abort) break;
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -634,11 +677,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {  // ---- MMA issuer
+        if (lane == 0 && rank == 0) {  // ---- MMA issuer (the leader only)
             int stage = 0, acc = 0;
             uint32_t phase = 0, acc_phase = 0;
-            const uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
-            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+            const uint32_t idesc = tc::idesc_bf16_f32(2 * BM, BN);
+            for (int tile = pair; tile < ntiles; tile += npairs) {
                 wait(tc::smem_u32(&bar_acce[acc]), acc_phase ^ 1u);
                 tc::fence_after_sync();
                 const uint32_t dcol = tm + acc * ACC_COLS;
@@ -655,14 +698,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                             const uint64_t da = desc_sw128(sa + 32 * kk);
 #pragma unroll
                             for (int s = 0; s < NSUB; ++s)
-                                tc::mma_bf16(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
-                                             (ks > 0 || kk > 0) ? 1u : 0u);
+                                mma_bf16_pair(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
+                                              (ks > 0 || kk > 0) ? 1u : 0u);
                         }
-                        tc::mma_commit(empty_b(stage * KPS + h));  // this k-step's slot is free once its MMAs are done
+                        mma_commit_pair(empty_b(stage * KPS + h));  // both CTAs' slot is free once these are done
                     }
+                    // the unused slots of a partial stage (k_steps not a multiple of KPS) complete
+                    // their phase too: every slot's barrier then advances once per pass of the
+                    // ring, in step with the stage parity the producer waits on
+                    for (int h = nk; h < KPS; ++h) mma_commit_pair(empty_b(stage * KPS + h));
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
-                tc::mma_commit(tc::smem_u32(&bar_accf[acc]));
+                mma_commit_pair(tc::smem_u32(&bar_accf[acc]));
                 if (NACC == 2) {
                     acc ^= 1;
                     if (acc == 0) acc_phase ^= 1u;
@@ -671,7 +718,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 }
             }
         }
-    } else {  // ---- epilogue warps 2..17: 4 column groups per TMEM lane quadrant
+    } else {  // ---- epilogue warps 2..17: 4 column groups per TMEM lane quadrant (both CTAs)
         const int quad = warp & 3;
         EpiCtx x;
         x.quad = quad;
@@ -679,7 +726,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x.lane = lane;
         x.row = 32 * quad + lane;
         x.red = reinterpret_cast<float *>(smem + STAGES * STAGE_BYTES + 4 * Epi::QUAD_STAGE);
-        x.stage = smem + STAGES * STAGE_BYTES + quad * Epi::QUAD_STAGE;
+        x.stage = smem + STAGES * STAGE_BYTES + quad * Epi::QUAD_STAGE;  // past the ring
         x.stage_u = tc::smem_u32(x.stage);
         x.stage_bar = tc::smem_u32(&bar_stage[quad]);
         x.stage_phase = 0;
@@ -692,21 +739,22 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x.status = g.status;
         int acc = 0;
         uint32_t acc_phase = 0;
-        if (Epi::TMA_STAGE && x.leader && (int)blockIdx.x < ntiles)
-            Epi::prefetch(io, blockIdx.x / g.n_tiles, blockIdx.x % g.n_tiles, x);
-        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-            const int m = tile / g.n_tiles, n = tile % g.n_tiles;
-            const int next = tile + (int)gridDim.x < ntiles ? tile + (int)gridDim.x : -1;
+        // this CTA's 128-row block of 256-row tile `tile`
+        auto mblock = [&](int tile) { return 2 * (tile / g.n_tiles) + (int)rank; };
+        if (Epi::TMA_STAGE && x.leader && pair < ntiles) Epi::prefetch(io, mblock(pair), pair % g.n_tiles, x);
+        for (int tile = pair; tile < ntiles; tile += npairs) {
+            const int mb = mblock(tile), n = tile % g.n_tiles;
+            const int next = tile + npairs < ntiles ? tile + npairs : -1;
             wait(tc::smem_u32(&bar_accf[acc]), acc_phase);
             __syncwarp();
             tc::fence_after_sync();
             const uint32_t tacc = tm + ((uint32_t)(32 * quad) << 16) + acc * ACC_COLS;
             // always run: the epilogues use per-quadrant named barriers, so every thread of a
             // quadrant must take the same path (after an abort the results are just unused)
-            Epi::run(io, tacc, m, n, x, next);
+            Epi::run(io, tacc, mb, n, x, next >= 0 ? mblock(next) : -1, next >= 0 ? next % g.n_tiles : 0);
             __syncwarp();
             tc::fence_before_sync();
-            mbar_arrive(tc::smem_u32(&bar_acce[acc]));
+            if (lane == 0) mbar_arrive_cluster(tc::map_rank(tc::smem_u32(&bar_acce[acc]), 0));
             if (NACC == 2) {
                 acc ^= 1;
                 if (acc == 0) acc_phase ^= 1u;
@@ -722,8 +770,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     __syncwarp();
     tc::fence_before_sync();
-    __syncthreads();
-    if (warp == 1) tc::tmem_dealloc(tm, 512);
+    tc::cluster_sync();  // the leader's MMAs into this CTA's TMEM and shared memory are done
+    if (warp == 1) tmem_dealloc_pair(tm, 512);
 }
 
 // ---------------------------------------------------------------------------
@@ -801,25 +849,41 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, ui
 
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 size_t gemm_smem() {
-    return 1024 + (size_t)STAGES * KPS * (BM * BK * 2 + (size_t)BN * NSUB * BK * 2) + 4 * (size_t)Epi::QUAD_STAGE +
-           Epi::RED_BYTES;
+    // per CTA: its A rows and half of each B slice per k-step
+    return 1024 + (size_t)STAGES * KPS * (BM * BK * 2 + (size_t)(BN / 2) * NSUB * BK * 2) +
+           4 * (size_t)Epi::QUAD_STAGE + Epi::RED_BYTES;
 }
 
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
                         const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s) {
     const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi, KPS>();
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN, NSUB, STAGES, Epi, KPS>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kern = k_tc_gemm<BN, NSUB, STAGES, Epi, KPS>;
+    cudaLaunchConfig_t lc = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;  // a CTA pair per 256-row tile
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    lc.blockDim = dim3(GEMM_THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = s;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    static int max_pairs = 0;  // pairs resident at once (the grid is persistent)
+    if (!max_pairs) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        attr = true;
+        lc.gridDim = dim3(sms & ~1);
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, kern, &lc);
+        if (e != cudaSuccess) return e;
+        max_pairs = n > 0 ? n : 1;
     }
     const int tiles = g.m_tiles * g.n_tiles;
-    const int grid = tiles < sms ? tiles : sms;
-    k_tc_gemm<BN, NSUB, STAGES, Epi, KPS><<<grid, GEMM_THREADS, smem, s>>>(ma, mb, mc, mxs, g, io);
-    return cudaGetLastError();
+    const int pairs = tiles < max_pairs ? tiles : max_pairs;
+    lc.gridDim = dim3(2 * pairs);
+    return cudaLaunchKernelEx(&lc, kern, ma, mb, mc, mxs, g, io);
 }
 
 inline size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -966,7 +1030,6 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     io.b_ctrl = T.bc; io.b_gate = T.bg; io.b_head = T.bh;
     io.wa = (const __nv_bfloat16 *)T.wa;
     io.dims_per_tile = T.dims_per_tile; io.rd_tile = T.rd_tile; io.rd_col = T.rd_col;
-    io.gates_n_tiles = H / 64;
     // h (fp32) is read back only by frozen episodes and for h_final: with no way to freeze
     // during the call it is needed after the last step only
     io.h32_mode = teacher ? 0 : (c.done_terminates || c.noop_terminates) ? 2 : 1;
@@ -991,14 +1054,16 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     }
     ++launches;
     CUtensorMap mx[2], mxs[2], mwc, mwg, mwh, mc;
-    const uint32_t ctrl_box = A > 128 ? 256u : 128u;  // the instantiated BN; rows past A read as zero
+    // B-operand boxes are half an instantiated BN (each CTA of a pair loads half the rows;
+    // rows past A read as zero)
+    const uint32_t ctrl_box = A > 128 ? 128u : 64u;
     if (!make_map(&mx[0], w.x[0], B, KX, BM) || !make_map(&mx[1], w.x[1], B, KX, BM) ||
         !make_map(&mxs[0], w.x[0], B, KX, 32) || !make_map(&mxs[1], w.x[1], B, KX, 32) ||
         !make_map(&mc, w.c, B, H, 32, true) ||
-        !make_map(&mwc, T.wc, A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 256) ||
-        !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE))
+        !make_map(&mwc, T.wc, A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 128) ||
+        !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE / 2))
         return cudaErrorInvalidValue;
-    const int m_tiles = (B + BM - 1) / BM;
+    const int m_tiles = (B + 2 * BM - 1) / (2 * BM);  // 256-row tiles, one per CTA pair
     cudaError_t e = cudaSuccess;
     for (int t = 0; t < Tn && e == cudaSuccess; ++t) {
         io.t = t;
@@ -1010,24 +1075,23 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status};
         if (!teacher) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
-            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
-            else if (A > 128) e = launch_gemm<256, 1, 4, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
-            else e = launch_gemm<128, 1, 4, EpiCtrl>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
             ++launches;
             if (e != cudaSuccess) break;
         }
         const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
-            e = launch_gemm<256, 1, 3, EpiGates>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s);
+            e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s);
         }
         ++launches;
         if (e != cudaSuccess) break;
         const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
-            // two k-steps per stage: half the waits on the MMA-issuing thread (same ring bytes)
-            e = launch_gemm<HEAD_TILE, 1, 2, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
+            e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
         }
         ++launches;
     }

@@ -348,7 +348,9 @@ def test_fused_matches_stepwise_closely(wm):
                                         ("mid_bf16", dict(ctrl_sample=1, ctrl_tau=0.7)),
                                         # column groups starting mid-word of the action mask
                                         ("small_bf16", dict(a_dim=192, ctrl_sample=1, ctrl_tau=0.8)),
-                                        ("small_bf16", dict(a_dim=64))])
+                                        ("small_bf16", dict(a_dim=64)),
+                                        # an odd number of k-steps in the head GEMM (H / 64 = 5)
+                                        ("small_bf16", dict(h_dim=320))])
 def test_tensor_against_oracle(wm, orc, name, flags):
     """Two row tiles (the second partly filled), resumed state, offsets, flags."""
     cfg = dict(synth.model_config(name), **flags)
@@ -391,11 +393,16 @@ def test_tensor_teacher_forced(wm, orc, name, prec, N, T):
     check_teacher(gs, o, "bf16")
 
 
-@pytest.mark.parametrize("name,T", [("large_bf16", 4), ("mid_bf16", 8)])
-def test_tensor_full_batch_is_deterministic(wm, name, T):
+@pytest.mark.parametrize("name,T,B,flags", [("large_bf16", 4, None, {}), ("mid_bf16", 8, None, {}),
+                                            # odd k-step counts: gates (Z + H) / 64 = 6, heads H / 64 = 5
+                                            ("small_bf16", 4, 16384, dict(h_dim=320))])
+def test_tensor_full_batch_is_deterministic(wm, name, T, B, flags):
     """Repeated full-batch calls are bit-identical (the persistent kernels' shared-memory
-    staging has no race: a missing ordering there shows up as run-to-run differences)."""
-    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, T=T)
+    staging and operand ring have no race: a missing ordering there shows up as run-to-run
+    differences).  Each CTA pair runs several tiles, so every ring slot is reused."""
+    cfg, _, z0, mask, B, T = synth.rollout_inputs(name, B=B, T=T)
+    cfg = dict(cfg, **flags)
+    w = synth.weights(cfg, seed=3)
     m = wm.WorldModel(dict(cfg, path="tensor"), w)
     zc, mc = _cuda(z0), _cuda(mask)
     first = m.rollout(zc, T, mask=mc)
