@@ -191,34 +191,74 @@ struct EpiCtx {
 
 // ---- controller epilogue: A columns in TMEM, A/4 per column group ---------------
 // Every thread of a warp issues the same TMEM loads (they are warp-collective);
-// rows past B only skip their memory accesses.
+// rows past B only skip their memory accesses.  The column group's columns are
+// taken 16 at a time ("chunks"; A % 64 == 0 puts each chunk inside one mask word).
+// The row's mask bits and frozen flag are loaded before the accumulator wait, and
+// the bias is read from a copy in shared memory.  The tempered draw keeps each
+// chunk's sum of weights, so only the chunk that holds the drawn point is read a
+// third time.
 struct EpiCtrl {
     static constexpr bool TMA_STAGE = false;
     static constexpr uint32_t QUAD_STAGE = 0;
-    static constexpr uint32_t RED_BYTES = 4 * 4 * 32 * 2 * 4;
+    static constexpr int MAX_A = 512, NCH = MAX_A / 4 / 16;  // chunks per column group, at most
+    static constexpr uint32_t RED_FLOATS = 4 * 4 * 32 * 2;
+    static constexpr uint32_t RED_BYTES = (RED_FLOATS + MAX_A) * 4;  // reductions | bias
+    struct Pre {
+        uint32_t bits[NCH];  // the chunk's 16 mask bits (0 for rows that do not act)
+        bool live;           // a row of the batch whose episode is not frozen
+    };
+    // once per CTA, by all 512 epilogue threads (e = 0..511), before the first tile
+    static __device__ void init(const StepIO &p, EpiCtx &x, int e) {
+        for (int i = e; i < p.A; i += 32 * EPI_WARPS) x.red[RED_FLOATS + i] = p.b_ctrl[i];
+    }
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int, int) {
+    static __device__ void pre(const StepIO &p, int m, int, EpiCtx &x, Pre &q) {
+        const int b = m * BM + x.row;
+        q.live = b < p.B && !p.fz_cur[b];
+        const int A = p.A, W = (A + 31) >> 5, CW = A / 4, c_lo = x.cg * CW;
+        const uint32_t *mw = (q.live && p.mask) ? p.mask + ((size_t)p.t * p.B + b) * W : nullptr;
+#pragma unroll
+        for (int k = 0; k < NCH; ++k) {
+            const int c0 = c_lo + 16 * k;
+            q.bits[k] = (!q.live || 16 * k >= CW) ? 0u : mw ? (mw[c0 >> 5] >> (c0 & 31)) & 0xFFFFu : 0xFFFFu;
+        }
+    }
+    // logits of chunk k (accumulator + bias)
+    static __device__ __forceinline__ void chunk(uint32_t tacc, const float *bs, int c0, float (&v)[16]) {
+        uint32_t r[16];
+        TC_LD16(tacc + c0, r);
+        const float4 *b4 = reinterpret_cast<const float4 *>(bs + c0);
+        float bb[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float4 t = b4[i];
+            bb[4 * i] = t.x; bb[4 * i + 1] = t.y; bb[4 * i + 2] = t.z; bb[4 * i + 3] = t.w;
+        }
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]) + bb[j];
+    }
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &q, int, int) {
         (void)n;
         const int b = m * BM + x.row;
-        const bool valid = b < p.B;
-        const int A = p.A, W = (A + 31) >> 5, CW = A / 4, c_lo = x.cg * CW;
-        const uint32_t *mw = (valid && p.mask) ? p.mask + ((size_t)p.t * p.B + b) * W : nullptr;
-        const bool live = valid && !p.fz_cur[b];
-        auto bits_at = [&](int c0) -> uint32_t { return mw ? (mw[c0 >> 5] >> (c0 & 31)) : 0xFFFFu; };
+        const bool valid = b < p.B, live = q.live;
+        const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
+        const float *bs = x.red + RED_FLOATS;
         // pass 1: masked argmax over this group's columns (lowest index on ties)
         int a = -1, last_v = -1;
         float bv = -INFINITY;
-        for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
-            uint32_t r[16];
-            TC_LD16(tacc + c0, r);
-            tc::tmem_ld_wait();
-            const uint32_t bits = live ? bits_at(c0) : 0u;
+#pragma unroll
+        for (int k = 0; k < NCH; ++k) {
+            if (k >= nch) break;
+            const int c0 = c_lo + 16 * k;
+            float v[16];
+            chunk(tacc, bs, c0, v);
+            const uint32_t bits = q.bits[k];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 if (!((bits >> j) & 1u)) continue;
-                const float v = __uint_as_float(r[j]) + p.b_ctrl[c0 + j];
                 last_v = c0 + j;
-                if (a < 0 || v > bv) { bv = v; a = c0 + j; }
+                if (a < 0 || v[j] > bv) { bv = v[j]; a = c0 + j; }
             }
         }
         float *my = x.slot(x.cg);
@@ -235,15 +275,21 @@ struct EpiCtrl {
         if (p.ctrl_sample && p.ctrl_tau > 0.f) {  // uniform over the warp
             const bool draw = live && ga >= 0;
             const float itau = __fdividef(1.f, p.ctrl_tau);
-            float S = 0.f;
-            for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
-                uint32_t r[16];
-                TC_LD16(tacc + c0, r);
-                tc::tmem_ld_wait();
-                const uint32_t bits = draw ? bits_at(c0) : 0u;
+            // pass 2: the group's sum of tempered weights, chunk by chunk
+            float cs[NCH], S = 0.f;
+#pragma unroll
+            for (int k = 0; k < NCH; ++k) {
+                cs[k] = 0.f;
+                if (k >= nch) continue;
+                float v[16];
+                chunk(tacc, bs, c_lo + 16 * k, v);
+                const uint32_t bits = draw ? q.bits[k] : 0u;
+                float sk = 0.f;
 #pragma unroll
                 for (int j = 0; j < 16; ++j)
-                    if ((bits >> j) & 1u) S += __expf((__uint_as_float(r[j]) + p.b_ctrl[c0 + j] - gbv) * itau);
+                    if ((bits >> j) & 1u) sk += __expf((v[j] - gbv) * itau);
+                cs[k] = sk;
+                S += sk;
             }
             x.sync();  // everyone has read the argmax partials
             my[0] = S;
@@ -259,20 +305,46 @@ struct EpiCtrl {
             }
             const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x) : 0.f;
             const float target = u * total;
-            int chosen = -1;
-            float cum = prefix;
             const bool mine = draw && target >= prefix && target < prefix + S;
-            for (int c0 = c_lo; c0 < c_lo + CW; c0 += 16) {
-                uint32_t r[16];
-                TC_LD16(tacc + c0, r);
-                tc::tmem_ld_wait();
-                const uint32_t bits = mine ? bits_at(c0) : 0u;
+            // the chunk holding the drawn point (the group's last chunk with a valid
+            // action if rounding carries the running sum past the target)
+            int kc = -1, klast = -1;
+            float base = prefix;
+#pragma unroll
+            for (int k = 0; k < NCH; ++k) {
+                if (k >= nch || !mine) continue;
+                if (q.bits[k]) klast = k;
+                if (kc < 0) {
+                    if (target < base + cs[k]) kc = k;
+                    else base += cs[k];
+                }
+            }
+            if (mine && kc < 0) {
+                kc = klast;
+                base = prefix;
+                for (int k = 0; k < NCH; ++k)
+                    if (k < klast) base += cs[k];
+            }
+            // pass 3: only chunks some row of the warp needs
+            int chosen = -1;
+#pragma unroll
+            for (int k = 0; k < NCH; ++k) {
+                if (k >= nch) break;
+                if (!__any_sync(0xffffffffu, kc == k)) continue;
+                float v[16];
+                chunk(tacc, bs, c_lo + 16 * k, v);
+                if (kc != k) continue;
+                const uint32_t bits = q.bits[k];
+                float cum = base;
+                int lastc = -1;
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     if (!((bits >> j) & 1u) || chosen >= 0) continue;
-                    cum += __expf((__uint_as_float(r[j]) + p.b_ctrl[c0 + j] - gbv) * itau);
-                    if (target < cum) chosen = c0 + j;
+                    cum += __expf((v[j] - gbv) * itau);
+                    lastc = c_lo + 16 * k + j;
+                    if (target < cum) chosen = lastc;
                 }
+                if (chosen < 0) chosen = lastc;  // rounding: the chunk's last valid action
             }
             x.sync();  // everyone has read the sum partials
             my[1] = __int_as_float(chosen);
@@ -298,7 +370,8 @@ struct EpiCtrl {
 // TMA; h' is stored by TMA into X_next.  The next tile's c is loaded as soon as
 // the stores have read the slab.  (Separate in- and out-slabs, refilled
 // mid-tile, measured slower: the extra quadrant barrier costs more than the
-// load latency it hides.)
+// load latency it hides.)  The cell is formed gate by gate over the thread's 16
+// units, so that each gate's W_a segment is one 256-bit load.
 struct EpiGates {
     static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
     static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
@@ -317,89 +390,144 @@ struct EpiGates {
             tma_load_2d(x.stage_u + bx * 4096, x.tm_c, 64 * n + 32 * bx, m * BM + 32 * x.quad, x.stage_bar);
     }
 
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int next_m, int next_n) {
+    struct Pre {
+        uint32_t wi[8], wg[8];  // the W_a row segments of gates i and g (16 units, bf16)
+        int a;                  // the action (-1: none)
+        bool fz;                // frozen episode
+    };
+    static __device__ void init(const StepIO &, EpiCtx &, int) {}
+    // one gate's W_a segment for the thread's 16 units: a single 32-byte sector, read with
+    // one 256-bit load (half the L1 wavefronts of two 16-byte loads: each lane reads
+    // another row, so every load instruction touches 32 lines)
+    static __device__ __forceinline__ void ld_wa(const StepIO &p, int a, int n, int q, int gate, uint32_t (&w)[8]) {
+        if (a < 0) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[i] = 0u;
+            return;
+        }
+        const __nv_bfloat16 *src = p.wa + (size_t)a * 4 * p.H + 256 * n + 64 * gate + 16 * q;
+        asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                     : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+                     : "l"(src));
+    }
+    // before the accumulator wait: the row's action and the W_a segments of gates i and g
+    // (L2 gathers), so that their latency overlaps the mainloop
+    static __device__ void pre(const StepIO &p, int m, int n, EpiCtx &x, Pre &pr) {
         const int b = m * BM + x.row;
-        const bool valid = b < p.B;
-        const int bb = valid ? b : 0;  // rows past B compute on row 0; TMA stores clip them
-        const int H = p.H, r = x.lane, q = x.cg;
-        const bool fz = p.fz_cur[bb] != 0;
+        const int bb = b < p.B ? b : 0;
+        pr.fz = p.fz_cur[bb] != 0;
         int a = p.act[bb];
         if (p.teacher) {
             a = p.act_in[(size_t)p.t * p.B + bb];
             if (a < 0 || a >= p.A) a = -1;
         }
-        // the action's W_a row segment, an L2 gather (a row per lane): the first half is
-        // issued before any wait, the second while the first is computed
-        const bool gather = a >= 0 && !fz;
-        const uint4 *war = reinterpret_cast<const uint4 *>(p.wa + (size_t)(gather ? a : 0) * 4 * H + 256 * n + 16 * q);
-        uint4 wv[4];
+        pr.a = (a >= 0 && !pr.fz) ? a : -1;
+        ld_wa(p, pr.a, n, x.cg, 0, pr.wi);
+        ld_wa(p, pr.a, n, x.cg, 2, pr.wg);
+    }
+    // pre-activations of one gate for the thread's 16 units: accumulator + bias + W_a[a]
+    static __device__ __forceinline__ void gate_pre(uint32_t tacc, const float *bg, int gate, int ut,
+                                                    const uint32_t (&w)[8], float (&g)[16]) {
 #pragma unroll
-        for (int gate = 0; gate < 4; ++gate) wv[gate] = gather ? war[8 * gate] : make_uint4(0, 0, 0, 0);
+        for (int h = 0; h < 2; ++h) {  // 8 columns per TMEM load: fewer registers held
+            uint32_t r[8];
+            TC_LD8(tacc + 64 * gate + ut + 8 * h, r);
+            tc::tmem_ld_wait();
+            // the bias is read after the wait (an L1 hit), so that it is not held across it
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const float4 t = *reinterpret_cast<const float4 *>(bg + 64 * gate + 8 * h + 4 * i);
+                const float bv[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int k = 8 * h + 4 * i + 2 * e;  // unit (column) index in 0..15
+                    const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&w[k / 2]);
+                    g[k] = __uint_as_float(r[4 * i + 2 * e]) + bv[2 * e] + __low2float(v2);
+                    g[k + 1] = __uint_as_float(r[4 * i + 2 * e + 1]) + bv[2 * e + 1] + __high2float(v2);
+                }
+            }
+        }
+    }
+
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &pr, int next_m,
+                               int next_n) {
+        const int b = m * BM + x.row;
+        const bool valid = b < p.B;
+        const int bb = valid ? b : 0;  // rows past B compute on row 0; TMA stores clip them
+        const int H = p.H, r = x.lane, q = x.cg;
+        const bool fz = pr.fz;
+        const int ut = 16 * q, u0 = 64 * n + ut;  // the thread's first unit: in the tile, in H
+        // gates f and o: loaded while i and g are computed
+        uint32_t wf[8], wo[8];
+        ld_wa(p, pr.a, n, q, 1, wf);
+        ld_wa(p, pr.a, n, q, 3, wo);
         const float *bg = p.b_gate + 256 * n + 16 * q;
         const bool store_h32 = valid && !fz && (p.h32_mode == 2 || (p.h32_mode == 1 && p.t == p.T - 1));
         unsigned char *cs = x.stage, *xs = x.stage + C_SLAB;
+        // the thread's 16 c values: 4 chunks of the swizzled box that holds units ut..ut+15
+        const uint32_t cbox = (ut >> 5) * 4096, cch = (ut & 31) >> 2;
+        // Every lane forms all four gates: the TMEM loads are warp-collective, and the rows
+        // of a warp may be frozen or not; a frozen row keeps its c and its carried h.
+        float cv[16], hv[16];
+        {  // hv = sigma(i) * tanh(g), one gate's pre-activations live at a time
+            float g[16];
+            gate_pre(tacc, bg, 0, ut, pr.wi, g);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]);
+            gate_pre(tacc, bg, 2, ut, pr.wg, g);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) hv[j] *= tanh_hw(g[j]);
+        }
         x.wait_stage();  // the quadrant's c rows have landed
-#pragma unroll 1
-        for (int half = 0; half < 2; ++half) {  // 8 units at a time keeps the registers in bounds
-            const int j0 = 8 * half, ut = 16 * q + j0, u0 = 64 * n + ut;
-            if (half == 1) {
 #pragma unroll
-                for (int gate = 0; gate < 4; ++gate) wv[gate] = gather ? war[8 * gate + 1] : make_uint4(0, 0, 0, 0);
+        for (int i = 0; i < 4; ++i) {
+            const float4 t = *reinterpret_cast<const float4 *>(cs + cbox + sw(r, cch + i));
+            cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
+        }
+        {
+            float g[16];
+            gate_pre(tacc, bg, 1, ut, wf, g);
+            if (!fz) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) cv[j] = sigmoid_hw(g[j]) * cv[j] + hv[j];
             }
-            uint32_t rr[4][8];
+            gate_pre(tacc, bg, 3, ut, wo, g);
 #pragma unroll
-            for (int gate = 0; gate < 4; ++gate) TC_LD8(tacc + 64 * gate + ut, rr[gate]);
-            tc::tmem_ld_wait();
-            const uint32_t o0 = (ut >> 5) * 4096 + sw(r, (ut & 31) >> 2), o1 = (ut >> 5) * 4096 + sw(r, ((ut & 31) >> 2) + 1);
-            const float4 ca = *reinterpret_cast<const float4 *>(cs + o0), cb = *reinterpret_cast<const float4 *>(cs + o1);
-            float cv[8] = {ca.x, ca.y, ca.z, ca.w, cb.x, cb.y, cb.z, cb.w}, hv[8];
-            if (fz) {  // frozen: c stays, h is the carried one
-                const float4 *h4 = reinterpret_cast<const float4 *>(p.h32 + (size_t)bb * H + u0);
-                const float4 ha = h4[0], hb = h4[1];
-                hv[0] = ha.x; hv[1] = ha.y; hv[2] = ha.z; hv[3] = ha.w;
-                hv[4] = hb.x; hv[5] = hb.y; hv[6] = hb.z; hv[7] = hb.w;
-            } else {
-                float gv[4][8];
+            for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]) * tanh_hw(cv[j]);
+        }
+        if (fz) {  // frozen: h is the carried one
+            const float4 *h4 = reinterpret_cast<const float4 *>(p.h32 + (size_t)bb * H + u0);
 #pragma unroll
-                for (int gate = 0; gate < 4; ++gate) {
-                    const uint32_t w4[4] = {wv[gate].x, wv[gate].y, wv[gate].z, wv[gate].w};
-                    const float4 b0 = *reinterpret_cast<const float4 *>(bg + 64 * gate + j0);
-                    const float4 b1 = *reinterpret_cast<const float4 *>(bg + 64 * gate + j0 + 4);
-                    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&w4[e]);
-                        gv[gate][2 * e] = __uint_as_float(rr[gate][2 * e]) + bv[2 * e] + __low2float(v2);
-                        gv[gate][2 * e + 1] = __uint_as_float(rr[gate][2 * e + 1]) + bv[2 * e + 1] + __high2float(v2);
-                    }
-                }
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    const float cn = sigmoid_hw(gv[1][j]) * cv[j] + sigmoid_hw(gv[0][j]) * tanh_hw(gv[2][j]);
-                    cv[j] = cn;
-                    hv[j] = sigmoid_hw(gv[3][j]) * tanh_hw(cn);
-                }
+            for (int i = 0; i < 4; ++i) {
+                const float4 t = h4[i];
+                hv[4 * i] = t.x; hv[4 * i + 1] = t.y; hv[4 * i + 2] = t.z; hv[4 * i + 3] = t.w;
             }
-            *reinterpret_cast<float4 *>(cs + o0) = make_float4(cv[0], cv[1], cv[2], cv[3]);
-            *reinterpret_cast<float4 *>(cs + o1) = make_float4(cv[4], cv[5], cv[6], cv[7]);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            *reinterpret_cast<float4 *>(cs + cbox + sw(r, cch + i)) =
+                make_float4(cv[4 * i], cv[4 * i + 1], cv[4 * i + 2], cv[4 * i + 3]);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
             uint32_t pk[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                __nv_bfloat162 v = __floats2bfloat162_rn(hv[2 * j], hv[2 * j + 1]);
+                __nv_bfloat162 v = __floats2bfloat162_rn(hv[8 * i + 2 * j], hv[8 * i + 2 * j + 1]);
                 pk[j] = *reinterpret_cast<uint32_t *>(&v);
             }
-            *reinterpret_cast<uint4 *>(xs + sw(r, ut >> 3)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            if (store_h32) {
-                float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)b * H + u0);
-                h4[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
-                h4[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
-            }
-            if (!valid) continue;
+            *reinterpret_cast<uint4 *>(xs + sw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+        if (store_h32) {
+            float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)b * H + u0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) h4[i] = make_float4(hv[4 * i], hv[4 * i + 1], hv[4 * i + 2], hv[4 * i + 3]);
+        }
+        if (valid) {
             const size_t o = ((size_t)p.t * p.B + b) * H + u0;
             if (p.h_seq)
-                for (int j = 0; j < 8; ++j) p.h_seq[o + j] = hv[j];
+                for (int j = 0; j < 16; ++j) p.h_seq[o + j] = hv[j];
             if (p.c_seq)
-                for (int j = 0; j < 8; ++j) p.c_seq[o + j] = cv[j];
+                for (int j = 0; j < 16; ++j) p.c_seq[o + j] = cv[j];
         }
         // the slab's generic-proxy reads and writes are ordered before the TMA (async-proxy)
         // stores and the refill by this fence and the barrier
@@ -430,8 +558,11 @@ struct EpiHeads {
     static constexpr int ZS_PITCH = 33;
     static constexpr uint32_t QUAD_STAGE = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
     static constexpr uint32_t RED_BYTES = 0;
+    struct Pre {};
+    static __device__ void init(const StepIO &, EpiCtx &, int) {}
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
-    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, int, int) {
+    static __device__ void pre(const StepIO &, int, int, EpiCtx &, Pre &) {}
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &, int, int) {
         const int b0 = m * BM + x.row;
         const bool valid = b0 < p.B;
         const int b = valid ? b0 : 0;  // rows past B compute on row 0 and store nothing
@@ -741,17 +872,21 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         uint32_t acc_phase = 0;
         // this CTA's 128-row block of 256-row tile `tile`
         auto mblock = [&](int tile) { return 2 * (tile / g.n_tiles) + (int)rank; };
+        Epi::init(io, x, tid - 64);
+        asm volatile("bar.sync 5, %0;" :: "n"(32 * EPI_WARPS) : "memory");  // the epilogue warps' set-up is done
         if (Epi::TMA_STAGE && x.leader && pair < ntiles) Epi::prefetch(io, mblock(pair), pair % g.n_tiles, x);
         for (int tile = pair; tile < ntiles; tile += npairs) {
             const int mb = mblock(tile), n = tile % g.n_tiles;
             const int next = tile + npairs < ntiles ? tile + npairs : -1;
+            typename Epi::Pre pr;
+            Epi::pre(io, mb, n, x, pr);  // loads that do not need the accumulator
             wait(tc::smem_u32(&bar_accf[acc]), acc_phase);
             __syncwarp();
             tc::fence_after_sync();
             const uint32_t tacc = tm + ((uint32_t)(32 * quad) << 16) + acc * ACC_COLS;
             // always run: the epilogues use per-quadrant named barriers, so every thread of a
             // quadrant must take the same path (after an abort the results are just unused)
-            Epi::run(io, tacc, mb, n, x, next >= 0 ? mblock(next) : -1, next >= 0 ? next % g.n_tiles : 0);
+            Epi::run(io, tacc, mb, n, x, pr, next >= 0 ? mblock(next) : -1, next >= 0 ? next % g.n_tiles : 0);
             __syncwarp();
             tc::fence_before_sync();
             if (lane == 0) mbar_arrive_cluster(tc::map_rank(tc::smem_u32(&bar_acce[acc]), 0));
