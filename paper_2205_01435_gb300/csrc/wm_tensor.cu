@@ -731,9 +731,9 @@ struct EpiHeads {
 // CTA: each CTA loads its 128 rows of A and BN/2 rows of each BN-wide slice of B, and runs
 // the epilogue on its own 128 accumulator rows.  (One M = 256 MMA does twice the work of an
 // M = 128 one in about 0.6 of its time, per SM.)  A ring stage holds KPS k-steps of BK: the
-// MMA thread waits for a stage once and issues all its MMAs back to back (any wait on the
-// issuing thread lets the tensor pipe drain), and each k-step has its own "empty" barrier so
-// that refills still go k-step by k-step.
+// MMA thread waits for a stage once, issues all its MMAs back to back and commits once, to
+// the stage's "empty" barrier: any wait or commit on the issuing thread lets the tensor
+// pipe drain, and a pair's multicast commit costs more than one k-step's MMAs can hide.
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -747,7 +747,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     static_assert(BN % 16 == 0 && BNH % 8 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES * KPS], bar_accf[2], bar_acce[2], bar_stage[4];
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -755,11 +755,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int pair = (int)(blockIdx.x >> 1), npairs = (int)(gridDim.x >> 1);
     const uint32_t smem_u = tc::smem_u32(smem);
     auto full_b = [&](int s) { return tc::smem_u32(&bar_full[s]); };
-    auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };  // s = stage * KPS + k-step
+    auto empty_b = [&](int s) { return tc::smem_u32(&bar_empty[s]); };
 
     if (tid == 0) {
         for (int s = 0; s < STAGES; ++s) tc::mbar_init(full_b(s), 1);             // the leader's: both CTAs' bytes
-        for (int s = 0; s < STAGES * KPS; ++s) tc::mbar_init(empty_b(s), 1);      // the leader's commit, multicast
+        for (int s = 0; s < STAGES; ++s) tc::mbar_init(empty_b(s), 1);            // the leader's commit, multicast
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(tc::smem_u32(&bar_accf[a]), 1);
             tc::mbar_init(tc::smem_u32(&bar_acce[a]), 2 * EPI_WARPS);  // the leader's: both CTAs' warps
@@ -790,10 +790,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
                     const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;  // k-steps in this stage
                     const uint32_t full_ldr = tc::map_rank(full_b(stage), 0);
+                    wait(empty_b(stage), phase ^ 1u);  // the stage's previous MMAs are done
+                    if (s_abort) break;
                     for (int h = 0; h < nk; ++h) {
                         const int ks = ks0 + h;
-                        wait(empty_b(stage * KPS + h), phase ^ 1u);
-                        if (s_abort) break;
                         const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
                         if (h == 0 && rank == 0) tc::mbar_arrive_expect_tx(full_b(stage), 2 * nk * KSTEP_BYTES);
                         tma_load_2sm(sa, &tmA, g.a_col0 + ks * BK, (2 * m + (int)rank) * BM, full_ldr);
@@ -832,12 +832,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                                 mma_bf16_pair(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
                                               (ks > 0 || kk > 0) ? 1u : 0u);
                         }
-                        mma_commit_pair(empty_b(stage * KPS + h));  // both CTAs' slot is free once these are done
                     }
-                    // the unused slots of a partial stage (k_steps not a multiple of KPS) complete
-                    // their phase too: every slot's barrier then advances once per pass of the
-                    // ring, in step with the stage parity the producer waits on
-                    for (int h = nk; h < KPS; ++h) mma_commit_pair(empty_b(stage * KPS + h));
+                    mma_commit_pair(empty_b(stage));  // both CTAs' stage is free once these are done
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 mma_commit_pair(tc::smem_u32(&bar_accf[acc]));
