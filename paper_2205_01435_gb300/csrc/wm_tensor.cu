@@ -552,16 +552,27 @@ struct EpiGates {
 // per block), so each block's two draws are made once per row.  The quadrant's z'
 // values are staged in shared memory ([32 rows][33], conflict-free) and stored by all
 // 128 threads in row-major order, so a warp's stores cover a few contiguous row
-// segments instead of 32 rows.
+// segments instead of 32 rows.  The tile's bias is copied into the quadrant's shared
+// memory before the accumulator wait and read as float4 broadcasts.
 struct EpiHeads {
     static constexpr bool TMA_STAGE = false;
     static constexpr int ZS_PITCH = 33;
-    static constexpr uint32_t QUAD_STAGE = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
+    static constexpr uint32_t ZS_BYTES = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
+    static constexpr uint32_t ZS_ALIGNED = (ZS_BYTES + 15) & ~15u;
+    // z' | the tile's bias (+ 16 floats: a dim's six float4 reads pass the tile's end by up to
+    // 16 when 3K < 24)
+    static constexpr uint32_t QUAD_STAGE = ZS_ALIGNED + (HEAD_TILE + 16) * 4;
     static constexpr uint32_t RED_BYTES = 0;
     struct Pre {};
     static __device__ void init(const StepIO &, EpiCtx &, int) {}
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
-    static __device__ void pre(const StepIO &, int, int, EpiCtx &, Pre &) {}
+    // the tile's HEAD_TILE bias values, by the quadrant's 128 threads (the previous tile's
+    // readers are past its closing barrier)
+    static __device__ void pre(const StepIO &p, int, int n, EpiCtx &x, Pre &) {
+        float *bq = reinterpret_cast<float *>(x.stage + ZS_ALIGNED);
+        const float *bh = p.b_head + (size_t)n * HEAD_TILE;
+        for (int i = x.cg * 32 + x.lane; i < HEAD_TILE; i += 128) bq[i] = bh[i];
+    }
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &, int, int) {
         const int b0 = m * BM + x.row;
         const bool valid = b0 < p.B;
@@ -573,10 +584,11 @@ struct EpiHeads {
         const unsigned long long ep = p.ep0 + b;
         const int d0 = n * p.dims_per_tile;
         const int nd = min(p.dims_per_tile, Z - d0);
-        const float *bh = p.b_head + (size_t)n * HEAD_TILE;
+        const float *bh = reinterpret_cast<const float *>(x.stage + ZS_ALIGNED);  // the tile's bias
         float *zs = reinterpret_cast<float *>(x.stage);
         const bool draw = !p.teacher && !fz && p.mdn_tau > 0.f;
         float nll = 0.f;
+        x.sync();  // the quadrant's copy of the bias is complete
         for (int blk = (d0 >> 2) + x.cg; 4 * blk < d0 + nd; blk += 4) {  // warp-uniform bounds
             u32x4 ru = {0, 0, 0, 0}, rn = {0, 0, 0, 0};
             if (draw) {
@@ -603,12 +615,20 @@ struct EpiHeads {
                 // columns of a dim are component-interleaved (logit, mu, log sigma) so that every
                 // register index below is static: no local-memory arrays
                 float lg[8], mu[8], ls[8];
-                const float *bhd = bh + DS * i;
+                {
+                    float bv[24];  // DS * i is a multiple of 8 floats: 16-byte aligned
+                    const float4 *b4 = reinterpret_cast<const float4 *>(bh + DS * i);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    lg[k] = k < K ? v[3 * k] + bhd[3 * k] : -INFINITY;
-                    mu[k] = k < K ? v[3 * k + 1] + bhd[3 * k + 1] : 0.f;
-                    ls[k] = k < K ? v[3 * k + 2] + bhd[3 * k + 2] : 0.f;
+                    for (int j = 0; j < 6; ++j) {
+                        const float4 t = b4[j];
+                        bv[4 * j] = t.x; bv[4 * j + 1] = t.y; bv[4 * j + 2] = t.z; bv[4 * j + 3] = t.w;
+                    }
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        lg[k] = k < K ? v[3 * k] + bv[3 * k] : -INFINITY;
+                        mu[k] = k < K ? v[3 * k + 1] + bv[3 * k + 1] : 0.f;
+                        ls[k] = k < K ? v[3 * k + 2] + bv[3 * k + 2] : 0.f;
+                    }
                 }
                 if (!valid) continue;
                 if (p.mdn_seq) {
