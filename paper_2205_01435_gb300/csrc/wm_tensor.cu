@@ -105,9 +105,6 @@ __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.w
 // ... and the stores are complete
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-__device__ __forceinline__ void mbar_arrive(uint32_t mbar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(mbar) : "memory");
-}
 
 // Gate nonlinearities from the fast exponential (relative error ~1e-6).
 __device__ __forceinline__ float sigmoid_hw(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
@@ -548,30 +545,50 @@ struct EpiGates {
 };
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
-// Column group g takes the dims of Philox blocks first + g, first + g + 4, ... (4 dims
-// per block), so each block's two draws are made once per row.  The quadrant's z'
-// values are staged in shared memory ([32 rows][33], conflict-free) and stored by all
-// 128 threads in row-major order, so a warp's stores cover a few contiguous row
-// segments instead of 32 rows.  The tile's bias is copied into the quadrant's shared
-// memory before the accumulator wait and read as float4 broadcasts.
+// Before the accumulator wait, the quadrant's 128 threads make the tile's random draws:
+// thread (row, g) takes Philox blocks first + g, first + g + 4, ... (4 dims per block, so
+// each block's two draws are made once per row) and leaves every (row, dim)'s uniform and
+// Box-Muller normal in shared memory; the tile's bias is copied there too.  After the
+// wait, column group g takes dims g, g + 4, ... (balanced: 10 dims go 3, 3, 2, 2).  The
+// quadrant's z' values are staged in shared memory ([32 rows][33], conflict-free) and
+// stored by all 128 threads in row-major order, so a warp's stores cover a few contiguous
+// row segments instead of 32 rows.
 struct EpiHeads {
     static constexpr bool TMA_STAGE = false;
     static constexpr int ZS_PITCH = 33;
-    static constexpr uint32_t ZS_BYTES = 32 * ZS_PITCH * 4;  // z' of the quadrant's 32 rows (<= 32 dims)
+    static constexpr uint32_t ZS_BYTES = 32 * ZS_PITCH * 4;  // [32 rows][<= 32 dims] floats
     static constexpr uint32_t ZS_ALIGNED = (ZS_BYTES + 15) & ~15u;
-    // z' | the tile's bias (+ 16 floats: a dim's six float4 reads pass the tile's end by up to
-    // 16 when 3K < 24)
-    static constexpr uint32_t QUAD_STAGE = ZS_ALIGNED + (HEAD_TILE + 16) * 4;
+    static constexpr uint32_t US_OFF = ZS_ALIGNED, BIAS_OFF = 2 * ZS_ALIGNED;
+    // normal draws, then z' | uniform draws | the tile's bias (+ 16 floats: a dim's six
+    // float4 reads pass the tile's end by up to 16 when 3K < 24)
+    static constexpr uint32_t QUAD_STAGE = BIAS_OFF + (HEAD_TILE + 16) * 4;
     static constexpr uint32_t RED_BYTES = 0;
     struct Pre {};
     static __device__ void init(const StepIO &, EpiCtx &, int) {}
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
     // the tile's HEAD_TILE bias values, by the quadrant's 128 threads (the previous tile's
     // readers are past its closing barrier)
-    static __device__ void pre(const StepIO &p, int, int n, EpiCtx &x, Pre &) {
-        float *bq = reinterpret_cast<float *>(x.stage + ZS_ALIGNED);
+    static __device__ void pre(const StepIO &p, int m, int n, EpiCtx &x, Pre &) {
+        float *bq = reinterpret_cast<float *>(x.stage + BIAS_OFF);
         const float *bh = p.b_head + (size_t)n * HEAD_TILE;
         for (int i = x.cg * 32 + x.lane; i < HEAD_TILE; i += 128) bq[i] = bh[i];
+        // the row's draws for the tile's dims (a5, a7): Philox blocks of 4 dims
+        const int b0 = m * BM + x.row;
+        const int b = b0 < p.B ? b0 : 0;
+        if (p.teacher || !(p.mdn_tau > 0.f) || p.fz_cur[b]) return;
+        const unsigned long long ep = p.ep0 + b;
+        const int d0 = n * p.dims_per_tile, nd = min(p.dims_per_tile, p.Z - d0);
+        float *es = reinterpret_cast<float *>(x.stage), *us = reinterpret_cast<float *>(x.stage + US_OFF);
+        for (int blk = (d0 >> 2) + x.cg; 4 * blk < d0 + nd; blk += 4) {
+            const u32x4 ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)blk);
+            const u32x4 rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)blk);
+            const int lo = max(d0, 4 * blk), hi = min(d0 + nd, 4 * blk + 4);
+            for (int d = lo; d < hi; ++d) {
+                const int pair = (d & 3) >> 1;
+                us[x.lane * ZS_PITCH + d - d0] = to_uniform(u32x4_get(ru, d & 3));
+                es[x.lane * ZS_PITCH + d - d0] = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
+            }
+        }
     }
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &, int, int) {
         const int b0 = m * BM + x.row;
@@ -581,23 +598,16 @@ struct EpiHeads {
         const int DS = (3 * K + 7) & ~7;  // columns per latent dim (8-aligned TMEM loads)
         const bool fz = p.fz_cur[b] != 0;
         const size_t tb = (size_t)p.t * p.B + b;
-        const unsigned long long ep = p.ep0 + b;
         const int d0 = n * p.dims_per_tile;
         const int nd = min(p.dims_per_tile, Z - d0);
-        const float *bh = reinterpret_cast<const float *>(x.stage + ZS_ALIGNED);  // the tile's bias
-        float *zs = reinterpret_cast<float *>(x.stage);
-        const bool draw = !p.teacher && !fz && p.mdn_tau > 0.f;
+        const float *bh = reinterpret_cast<const float *>(x.stage + BIAS_OFF);  // the tile's bias
+        float *zs = reinterpret_cast<float *>(x.stage);  // the normal draws, then z'
+        const float *us = reinterpret_cast<const float *>(x.stage + US_OFF);
         float nll = 0.f;
-        x.sync();  // the quadrant's copy of the bias is complete
-        for (int blk = (d0 >> 2) + x.cg; 4 * blk < d0 + nd; blk += 4) {  // warp-uniform bounds
-            u32x4 ru = {0, 0, 0, 0}, rn = {0, 0, 0, 0};
-            if (draw) {
-                ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)blk);
-                rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)blk);
-            }
-            const int lo = max(d0, 4 * blk), hi = min(d0 + nd, 4 * blk + 4);
-            for (int d = lo; d < hi; ++d) {
-                const int i = d - d0;
+        x.sync();  // the quadrant's bias copy and draws are complete
+        {
+            for (int i = x.cg; i < nd; i += 4) {  // warp-uniform bounds
+                const int d = d0 + i;
                 float v[24];
                 {
                     uint32_t r0[8], r1[8], r2[8];
@@ -689,7 +699,7 @@ struct EpiHeads {
                             pk[k] = k < K ? __expf(lg[k] * itau - mx) : 0.f;
                             s += pk[k];
                         }
-                        const float u = to_uniform(u32x4_get(ru, d & 3)), is = __fdividef(1.f, s);
+                        const float u = us[x.lane * ZS_PITCH + i], is = __fdividef(1.f, s);  // drawn in pre()
                         // first k with u < C_k (the last component when rounding leaves u >= C_{K-2})
                         kc = K - 1;
                         float cum = 0.f, muc = 0.f, lsc = 0.f;
@@ -702,8 +712,7 @@ struct EpiHeads {
                             }
                             if (k == kc) { muc = mu[k]; lsc = ls[k]; }
                         }
-                        const int pair = (d & 3) >> 1;
-                        const float eps = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
+                        const float eps = zs[x.lane * ZS_PITCH + i];  // drawn in pre()
                         const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
                         zn = muc + __expf(lsc) * scale * eps;
                     }
