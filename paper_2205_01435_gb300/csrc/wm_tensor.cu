@@ -235,13 +235,23 @@ struct EpiCtrl {
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]) + bb[j];
     }
+    // The per-column work is branch-free: each lane has its own mask bits, and a branch per
+    // column splits the warp at every column (the mask is sparse).
+    static __device__ __forceinline__ float ex2_approx(float x) {
+        float y;
+        asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+        return y;
+    }
+    // bit j of `bits` as an all-ones / all-zeros word
+    static __device__ __forceinline__ uint32_t lane_mask(uint32_t bits, int j) { return 0u - ((bits >> j) & 1u); }
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &q, int, int) {
         (void)n;
         const int b = m * BM + x.row;
         const bool valid = b < p.B, live = q.live;
         const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
         const float *bs = x.red + RED_FLOATS;
-        // pass 1: masked argmax over this group's columns (lowest index on ties)
+        // pass 1: masked argmax over this group's columns (lowest index on ties): per chunk,
+        // the maximum of the valid logits, then the lowest valid column that attains it
         int a = -1, last_v = -1;
         float bv = -INFINITY;
 #pragma unroll
@@ -251,12 +261,21 @@ struct EpiCtrl {
             float v[16];
             chunk(tacc, bs, c0, v);
             const uint32_t bits = q.bits[k];
+            float mx = -INFINITY;
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-                if (!((bits >> j) & 1u)) continue;
-                last_v = c0 + j;
-                if (a < 0 || v[j] > bv) { bv = v[j]; a = c0 + j; }
+                v[j] = __uint_as_float((__float_as_uint(v[j]) & lane_mask(bits, j)) |
+                                       (0xff800000u & ~lane_mask(bits, j)));  // -inf where masked
+                mx = fmaxf(mx, v[j]);
             }
+            uint32_t eq = 0u;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) eq |= (v[j] == mx ? 1u : 0u) << j;
+            eq &= bits;
+            const bool better = eq != 0u && (a < 0 || mx > bv);
+            bv = better ? mx : bv;
+            a = better ? c0 + __ffs(eq) - 1 : a;
+            last_v = bits ? c0 + 31 - __clz(bits) : last_v;
         }
         float *my = x.slot(x.cg);
         my[0] = bv;
@@ -271,7 +290,9 @@ struct EpiCtrl {
         }
         if (p.ctrl_sample && p.ctrl_tau > 0.f) {  // uniform over the warp
             const bool draw = live && ga >= 0;
-            const float itau = __fdividef(1.f, p.ctrl_tau);
+            // weight of logit v: exp((v - max) / tau) = 2^(v * s - max * s), s = log2(e) / tau;
+            // a masked column's weight is forced to +0 (its logit may exceed the maximum)
+            const float sc = 1.4426950408889634f / p.ctrl_tau, off = -gbv * sc;
             // pass 2: the group's sum of tempered weights, chunk by chunk
             float cs[NCH], S = 0.f;
 #pragma unroll
@@ -284,7 +305,7 @@ struct EpiCtrl {
                 float sk = 0.f;
 #pragma unroll
                 for (int j = 0; j < 16; ++j)
-                    if ((bits >> j) & 1u) sk += __expf((v[j] - gbv) * itau);
+                    sk += __uint_as_float(__float_as_uint(ex2_approx(fmaf(v[j], sc, off))) & lane_mask(bits, j));
                 cs[k] = sk;
                 S += sk;
             }
@@ -333,15 +354,15 @@ struct EpiCtrl {
                 if (kc != k) continue;
                 const uint32_t bits = q.bits[k];
                 float cum = base;
-                int lastc = -1;
+                uint32_t hit = 0u;  // valid columns at which the running sum has passed the target
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
-                    if (!((bits >> j) & 1u) || chosen >= 0) continue;
-                    cum += __expf((v[j] - gbv) * itau);
-                    lastc = c_lo + 16 * k + j;
-                    if (target < cum) chosen = lastc;
+                    cum += __uint_as_float(__float_as_uint(ex2_approx(fmaf(v[j], sc, off))) & lane_mask(bits, j));
+                    hit |= (target < cum ? 1u : 0u) << j;
                 }
-                if (chosen < 0) chosen = lastc;  // rounding: the chunk's last valid action
+                hit &= bits;
+                // the first such column; rounding: the chunk's last valid action
+                chosen = hit ? c_lo + 16 * k + __ffs(hit) - 1 : (bits ? c_lo + 16 * k + 31 - __clz(bits) : -1);
             }
             x.sync();  // everyone has read the sum partials
             my[1] = __int_as_float(chosen);
