@@ -721,17 +721,23 @@ struct EpiHeads {
                             s += pk[k];
                         }
                         const float u = us[x.lane * ZS_PITCH + i], is = __fdividef(1.f, s);  // drawn in pre()
-                        // first k with u < C_k (the last component when rounding leaves u >= C_{K-2})
-                        kc = K - 1;
-                        float cum = 0.f, muc = 0.f, lsc = 0.f;
-                        bool found = false;
+                        // first k with u < C_k (the last component when rounding leaves u >= C_{K-2}),
+                        // from a compare mask: no per-lane branches
+                        float cum = 0.f;
+                        uint32_t hit = 0u;
 #pragma unroll
                         for (int k = 0; k < 8; ++k) {
-                            if (k < K - 1 && !found) {
+                            if (k < K - 1) {  // uniform
                                 cum += pk[k] * is;
-                                if (u < cum) { kc = k; found = true; }
+                                hit |= (u < cum ? 1u : 0u) << k;
                             }
-                            if (k == kc) { muc = mu[k]; lsc = ls[k]; }
+                        }
+                        kc = hit ? __ffs(hit) - 1 : K - 1;
+                        float muc = mu[0], lsc = ls[0];
+#pragma unroll
+                        for (int k = 1; k < 8; ++k) {
+                            muc = (k < K && k == kc) ? mu[k] : muc;
+                            lsc = (k < K && k == kc) ? ls[k] : lsc;
                         }
                         const float eps = zs[x.lane * ZS_PITCH + i];  // drawn in pre()
                         const float scale = p.sigma_sqrt_tau ? sqrtf(p.mdn_tau) : 1.f;
