@@ -55,6 +55,16 @@ __device__ __forceinline__ float box_muller(uint32_t x1, uint32_t x2, bool secon
     return r * (second ? s : c);
 }
 
+// Both Box-Muller normals of a pair: c = r cos, s = r sin (the values box_muller returns).
+__device__ __forceinline__ void box_muller2(uint32_t x1, uint32_t x2, float &c_out, float &s_out) {
+    float u1 = to_uniform(x1), u2 = to_uniform(x2);
+    float r = sqrtf(-2.0f * logf(1.0f - u1));
+    float s, c;
+    sincospif(2.0f * u2, &s, &c);
+    c_out = r * c;
+    s_out = r * s;
+}
+
 // The normal of latent dim d at (episode, step).
 __device__ __forceinline__ float normal_for_dim(unsigned long long seed, unsigned long long ep,
                                                 uint32_t step, int d) {

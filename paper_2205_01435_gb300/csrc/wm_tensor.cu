@@ -90,8 +90,11 @@ __device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_saddr, uint32_t nco
 __device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
     asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols) : "memory");
 }
+// Relaxed: the epilogue's accumulator-empty arrive orders nothing in memory (the thread's
+// TMEM loads have completed at tcgen05.wait::ld), and a release at cluster scope stalled
+// the arriving thread for about 3K cycles per tile.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t mbar_cluster) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" :: "r"(mbar_cluster) : "memory");
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" :: "r"(mbar_cluster) : "memory");
 }
 
 // TMA store of a box from shared memory (bulk-group completion).
@@ -604,10 +607,14 @@ struct EpiHeads {
             const u32x4 ru = rng_draw(p.seed, ep, p.step, RNG_COMPONENT, (uint32_t)blk);
             const u32x4 rn = rng_draw(p.seed, ep, p.step, RNG_NORMAL, (uint32_t)blk);
             const int lo = max(d0, 4 * blk), hi = min(d0 + nd, 4 * blk + 4);
-            for (int d = lo; d < hi; ++d) {
-                const int pair = (d & 3) >> 1;
-                us[x.lane * ZS_PITCH + d - d0] = to_uniform(u32x4_get(ru, d & 3));
-                es[x.lane * ZS_PITCH + d - d0] = box_muller(pair ? rn.z : rn.x, pair ? rn.w : rn.y, (d & 1) != 0);
+            for (int d = lo; d < hi; ++d) us[x.lane * ZS_PITCH + d - d0] = to_uniform(u32x4_get(ru, d & 3));
+            for (int h = 0; h < 2; ++h) {  // the block's two Box-Muller pairs: dims da (cos), da + 1 (sin)
+                const int da = 4 * blk + 2 * h;
+                if (da + 1 < lo || da >= hi) continue;
+                float c, sn;
+                box_muller2(h ? rn.z : rn.x, h ? rn.w : rn.y, c, sn);
+                if (da >= lo) es[x.lane * ZS_PITCH + da - d0] = c;
+                if (da + 1 < hi) es[x.lane * ZS_PITCH + da + 1 - d0] = sn;
             }
         }
     }
@@ -877,15 +884,19 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     wait(full_b(stage), phase);
                     if (s_abort) break;
                     tc::fence_after_sync();
-                    for (int h = 0; h < nk; ++h) {
+                    // the issuing thread shares its SMSP with four epilogue warps: few instructions
+                    // between MMAs (descriptors built once per k-step, stepped by 32 bytes = 2)
+#pragma unroll
+                    for (int h = 0; h < KPS; ++h) {
+                        if (h >= nk) break;
                         const int ks = ks0 + h;
                         const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
+                        const uint64_t da0 = desc_sw128(sa), db0 = desc_sw128(sa + A_BYTES);
 #pragma unroll
                         for (int kk = 0; kk < BK / 16; ++kk) {
-                            const uint64_t da = desc_sw128(sa + 32 * kk);
 #pragma unroll
                             for (int s = 0; s < NSUB; ++s)
-                                mma_bf16_pair(dcol + s * BN, da, desc_sw128(sa + A_BYTES + s * B_SUB + 32 * kk), idesc,
+                                mma_bf16_pair(dcol + s * BN, da0 + 2 * kk, db0 + (s * B_SUB >> 4) + 2 * kk, idesc,
                                               (ks > 0 || kk > 0) ? 1u : 0u);
                         }
                     }
