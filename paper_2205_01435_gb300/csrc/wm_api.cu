@@ -67,47 +67,141 @@ cudaError_t upload(T **dst, const std::vector<T> &src) {
 }
 
 // One caller array that may need staging.
+// How a staged array meets the steps of a call.
+enum StageKind {
+    WHOLE = 0,    // copied whole: inputs before the call, outputs after it
+    STEP_IN = 1,  // input; slab t is first read by step t
+    STEP_OUT = 2, // output; slab t is final after step t
+    TRAJ_OUT = 3, // output of T + 1 slabs; slab 0 is final after the init kernel, slab t + 1 after step t
+};
+
 struct Stage {
     void **dev;        // where the device pointer goes
     const void *user;  // caller pointer
     size_t bytes;
     bool out;
     size_t off;
+    int kind;
+    size_t slab;       // bytes per step (per-step kinds)
 };
 
-struct Stager {
+// Copies caller host arrays through the handle's staging buffer.  With per-step
+// staging on (a family that launches step by step, pinned or pageable host memory,
+// a stream that is not capturing), step t's input slabs go up on copy_in ahead of the
+// steps and its output slabs come down on copy_out as soon as step t is done, so the
+// copies overlap the computation; otherwise everything is copied whole around the call.
+// Either way a call with host arrays returns once every copy is complete.
+struct Stager : wm_step_stage {
     std::vector<Stage> items;
     size_t total = 0;
-    bool any_host_out = false;
-    void add(void **dev, const void *user, size_t bytes, bool out) {
+    bool any_host = false, any_host_out = false;
+    bool stepped = false;
+    int T = 0;
+    wm_handle *h = nullptr;
+    cudaEvent_t *ev = nullptr;  // [0]: start, [1]: init done, [2 + t]: step t's inputs, [2 + T + t]: step t done
+    void add(void **dev, const void *user, size_t bytes, bool out, int kind = WHOLE, size_t slab = 0) {
         *dev = const_cast<void *>(user);
         if (!user || bytes == 0 || !is_host_ptr(user)) return;
-        items.push_back({dev, user, bytes, out, total});
+        items.push_back({dev, user, bytes, out, total, kind, slab});
         total += (bytes + 255) & ~(size_t)255;
+        any_host = true;
         if (out) any_host_out = true;
     }
-    cudaError_t begin(wm_handle *h, cudaStream_t s) {
+    cudaError_t copy_slab(const Stage &it, size_t i, cudaStream_t s) {
+        const size_t o = i * it.slab;
+        if (it.out)
+            return cudaMemcpyAsync((char *)const_cast<void *>(it.user) + o, (char *)*it.dev + o, it.slab,
+                                   cudaMemcpyDeviceToHost, s);
+        return cudaMemcpyAsync((char *)*it.dev + o, (const char *)it.user + o, it.slab, cudaMemcpyHostToDevice, s);
+    }
+    // step_wise: the family will call the wm_step_stage hooks
+    cudaError_t begin(wm_handle *hd, int steps, bool step_wise, cudaStream_t s) {
         if (items.empty()) return cudaSuccess;
+        h = hd;
+        T = steps;
         cudaError_t e = grow(&h->stage, &h->stage_bytes, total);
         if (e != cudaSuccess) return e;
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if ((e = cudaStreamIsCapturing(s, &cs)) != cudaSuccess) return e;
+        stepped = step_wise && T > 1 && cs == cudaStreamCaptureStatusNone;
+        if (stepped) {
+            if (!h->copy_in && (e = cudaStreamCreateWithFlags(&h->copy_in, cudaStreamNonBlocking)) != cudaSuccess)
+                return e;
+            if (!h->copy_out && (e = cudaStreamCreateWithFlags(&h->copy_out, cudaStreamNonBlocking)) != cudaSuccess)
+                return e;
+            const size_t need = 2 + 2 * (size_t)T;
+            while (h->events.size() < need) {
+                cudaEvent_t x;
+                if ((e = cudaEventCreateWithFlags(&x, cudaEventDisableTiming)) != cudaSuccess) return e;
+                h->events.push_back(x);
+            }
+            ev = h->events.data();
+        }
         for (auto &it : items) {
             *it.dev = (char *)h->stage + it.off;
-            if (!it.out) {
+            if (it.out) continue;
+            if (!stepped || it.kind == WHOLE) {
                 e = cudaMemcpyAsync(*it.dev, it.user, it.bytes, cudaMemcpyHostToDevice, s);
                 if (e != cudaSuccess) return e;
             }
         }
+        if (!stepped) return cudaSuccess;
+        // the copy streams start after the stream's earlier work (the staging buffer's
+        // previous users); step inputs go up in step order
+        if ((e = cudaEventRecord(ev[0], s)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(h->copy_in, ev[0], 0)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(h->copy_out, ev[0], 0)) != cudaSuccess) return e;
+        for (int t = 0; t < T; ++t) {
+            for (auto &it : items)
+                if (it.kind == STEP_IN && (e = copy_slab(it, (size_t)t, h->copy_in)) != cudaSuccess) return e;
+            if ((e = cudaEventRecord(ev[2 + t], h->copy_in)) != cudaSuccess) return e;
+        }
         return cudaSuccess;
+    }
+    cudaError_t after_init(cudaStream_t s) override {
+        if (!stepped) return cudaSuccess;
+        cudaError_t e = cudaEventRecord(ev[1], s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(h->copy_out, ev[1], 0);
+        for (auto &it : items)
+            if (e == cudaSuccess && it.kind == TRAJ_OUT) e = copy_slab(it, 0, h->copy_out);
+        return e;
+    }
+    cudaError_t before_step(int t, cudaStream_t s) override {
+        return stepped ? cudaStreamWaitEvent(s, ev[2 + t], 0) : cudaSuccess;
+    }
+    cudaError_t after_step(int t, cudaStream_t s) override {
+        if (!stepped) return cudaSuccess;
+        cudaEvent_t done = ev[2 + T + t];
+        cudaError_t e = cudaEventRecord(done, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(h->copy_out, done, 0);
+        for (auto &it : items) {
+            if (e != cudaSuccess) break;
+            if (it.kind == STEP_OUT) e = copy_slab(it, (size_t)t, h->copy_out);
+            else if (it.kind == TRAJ_OUT) e = copy_slab(it, (size_t)t + 1, h->copy_out);
+        }
+        return e;
     }
     cudaError_t end(cudaStream_t s) {
         for (auto &it : items) {
-            if (!it.out) continue;
+            if (!it.out || (stepped && it.kind != WHOLE)) continue;
             cudaError_t e = cudaMemcpyAsync(const_cast<void *>(it.user), *it.dev, it.bytes,
                                             cudaMemcpyDeviceToHost, s);
             if (e != cudaSuccess) return e;
         }
-        if (any_host_out) return cudaStreamSynchronize(s);
+        if (stepped) {
+            cudaError_t e = cudaStreamSynchronize(h->copy_in);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(h->copy_out);
+            if (e != cudaSuccess) return e;
+        }
+        if (any_host_out || stepped) return cudaStreamSynchronize(s);
         return cudaSuccess;
+    }
+    // an early return (an error) still waits for the copies that touch the caller's arrays
+    ~Stager() {
+        if (stepped && h) {
+            cudaStreamSynchronize(h->copy_in);
+            cudaStreamSynchronize(h->copy_out);
+        }
     }
 };
 
@@ -217,6 +311,9 @@ void wm_destroy(wm_handle *h) {
         cudaEventDestroy(r.b);
     }
     for (cudaEvent_t ev : h->timer.spare) cudaEventDestroy(ev);
+    for (cudaEvent_t ev : h->events) cudaEventDestroy(ev);
+    if (h->copy_in) cudaStreamDestroy(h->copy_in);
+    if (h->copy_out) cudaStreamDestroy(h->copy_out);
     if (prev >= 0) cudaSetDevice(prev);
     delete h;
 }
@@ -343,17 +440,17 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     st.add((void **)&a.h0, io->h0, b * H * 4, false);
     st.add((void **)&a.c0, io->c0, b * H * 4, false);
     st.add((void **)&a.done0, io->done0, b, false);
-    st.add((void **)&a.mask, io->mask, t * b * W * 4, false);
-    st.add((void **)&a.z_out, io->z_out, (t + 1) * b * Z * 4, true);
-    st.add((void **)&a.actions, io->actions, t * b * 4, true);
-    st.add((void **)&a.rewards, io->rewards, t * b * 4, true);
-    st.add((void **)&a.done, io->done, t * b, true);
+    st.add((void **)&a.mask, io->mask, t * b * W * 4, false, STEP_IN, b * W * 4);
+    st.add((void **)&a.z_out, io->z_out, (t + 1) * b * Z * 4, true, TRAJ_OUT, b * Z * 4);
+    st.add((void **)&a.actions, io->actions, t * b * 4, true, STEP_OUT, b * 4);
+    st.add((void **)&a.rewards, io->rewards, t * b * 4, true, STEP_OUT, b * 4);
+    st.add((void **)&a.done, io->done, t * b, true, STEP_OUT, b);
     st.add((void **)&a.h_final, io->h_final, b * H * 4, true);
     st.add((void **)&a.c_final, io->c_final, b * H * 4, true);
-    st.add((void **)&a.h_seq, io->h_seq, t * b * H * 4, true);
-    st.add((void **)&a.c_seq, io->c_seq, t * b * H * 4, true);
-    st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true);
-    st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true);
+    st.add((void **)&a.h_seq, io->h_seq, t * b * H * 4, true, STEP_OUT, b * H * 4);
+    st.add((void **)&a.c_seq, io->c_seq, t * b * H * 4, true, STEP_OUT, b * H * 4);
+    st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true, STEP_OUT, b * M * 4);
+    st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true, STEP_OUT, b * Z);
 
     int path = pick_path(h, B);
     if (path == WM_PATH_FUSED && !wm_fused_supported(h, B))
@@ -366,7 +463,9 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
         e = grow(&h->ws, &h->ws_bytes, need);
         if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
     }
-    if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    // the tensor family launches step by step: its host arrays are staged per step
+    if ((e = st.begin(h, T, path == WM_PATH_TENSOR && B > 0, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    a.stage = &st;
     if (path == WM_PATH_FUSED)
         e = wm_fused_rollout(h, a, s);
     else if (path == WM_PATH_TENSOR)
@@ -421,7 +520,7 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
                                                                                       : wm_step_nll_ws(h, N);
     e = grow(&h->ws, &h->ws_bytes, need);
     if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
-    if ((e = st.begin(h, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    if ((e = st.begin(h, T, false, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
     if (path == WM_PATH_FUSED)
         e = wm_fused_nll(h, a, h->ws, s);
     else if (path == WM_PATH_TENSOR)

@@ -11,7 +11,18 @@
 #include "wm.h"
 
 // Device pointers of one rollout call (after host arrays were staged).
+// Per-step staging of caller host arrays, for families that launch step by step: the
+// family calls these around its launches on stream s so that step t's inputs arrive
+// and its outputs leave on copy streams while other steps compute.
+struct wm_step_stage {
+    virtual cudaError_t after_init(cudaStream_t s) = 0;        // the init kernel is enqueued
+    virtual cudaError_t before_step(int t, cudaStream_t s) = 0;  // before step t's first launch
+    virtual cudaError_t after_step(int t, cudaStream_t s) = 0;   // after step t's last launch
+    virtual ~wm_step_stage() {}
+};
+
 struct wm_rollout_dev {
+    wm_step_stage *stage = nullptr;  // null: the arrays are whole on the device
     int B, T;
     unsigned long long ep0;
     unsigned int t0;
@@ -88,6 +99,8 @@ struct wm_handle {
     size_t ws_bytes = 0;
     void *stage = nullptr;       // staging for host arrays (grows on demand)
     size_t stage_bytes = 0;
+    cudaStream_t copy_in = nullptr, copy_out = nullptr;  // per-step staging copies (lazy)
+    std::vector<cudaEvent_t> events;                       // per-step staging events (grows)
     int *status = nullptr;       // device status word (WM_ERR_TIMEOUT etc.)
     int last_path = 0;
     mutable int last_launches = 0;   // kernels launched by the last call

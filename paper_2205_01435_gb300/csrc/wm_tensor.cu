@@ -1251,6 +1251,11 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
                                             w.fz[0], w.fz[1], T.n_head_tiles);
     }
     ++launches;
+    wm_step_stage *hooks = teacher ? nullptr : ra->stage;  // per-step staging of host arrays
+    if (hooks) {
+        cudaError_t he = hooks->after_init(s);
+        if (he != cudaSuccess) return he;
+    }
     CUtensorMap mx[2], mxs[2], mwc, mwg, mwh, mc;
     // B-operand boxes are half an instantiated BN (each CTA of a pair loads half the rows;
     // rows past A read as zero)
@@ -1271,6 +1276,7 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         io.fz_cur = w.fz[t & 1];
         io.fz_next = w.fz[(t + 1) & 1];
         const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status};
+        if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
         if (!teacher) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
             if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
@@ -1292,6 +1298,7 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
             e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
         }
         ++launches;
+        if (e == cudaSuccess && hooks) e = hooks->after_step(t, s);
     }
     if (e != cudaSuccess) return e;
     {

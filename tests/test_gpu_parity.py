@@ -273,17 +273,26 @@ def test_resume_is_bit_exact(wm, name):
 
 
 @pytest.mark.parametrize("kind", ["pinned", "pageable"])
-def test_host_buffers_match_device_buffers(wm, kind):
-    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", T=6)
-    m = wm.WorldModel(cfg, w)
-    dev = m.rollout(_cuda(z0), T, mask=_cuda(mask))
+@pytest.mark.parametrize("path,B,T,seq", [("auto", None, 6, False),   # fused: copied whole around the call
+                                          ("tensor", 700, 6, True),   # per-step staging, every output kind
+                                          ("tensor", 700, 1, False)])  # one step: copied whole
+def test_host_buffers_match_device_buffers(wm, kind, path, B, T, seq):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=B, T=T)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    dev = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=seq)
     zh, mh = torch.from_numpy(z0), torch.from_numpy(mask)
     if kind == "pinned":
         zh, mh = zh.pin_memory(), mh.pin_memory()
-    host = m.rollout(zh, T, mask=mh)  # outputs allocated on the host, call syncs
-    for k in ("z", "actions", "rewards", "done", "h_final", "c_final"):
-        assert not host[k].is_cuda
-        assert torch.equal(host[k], dev[k].cpu()), k
+    keys = ["z", "actions", "rewards", "done", "h_final", "c_final"]
+    if seq:
+        keys += ["h_seq", "c_seq", "mdn_seq", "comp_seq"]
+    for _ in range(2):  # the second call reuses the staging buffer and its events
+        host = m.rollout(zh, T, mask=mh, want_seq=seq)  # outputs allocated on the host, call syncs
+        if path == "tensor":
+            assert m.last_path == "tensor"
+        for k in keys:
+            assert not host[k].is_cuda
+            assert torch.equal(host[k], dev[k].cpu()), k
 
 
 # ------------------------------------------------------------------ the fused single-launch family
