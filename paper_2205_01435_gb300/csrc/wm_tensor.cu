@@ -836,6 +836,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     tc::cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrive
     tc::fence_after_sync();
     const uint32_t tm = tmem_base;
+    // Programmatic dependent launch (when the launch allows it): the set-up above may overlap
+    // the previous kernel of the stream; every read of its outputs comes after this wait.
+    // The next kernel may then be launched, its own set-up overlapping this one.  (Both
+    // return at once for a launch without programmatic serialization.)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
     auto wait = [&](uint32_t bar, uint32_t parity) {
         if (!s_abort && !tc::mbar_wait_bounded(bar, parity, POLLS)) {
@@ -1054,11 +1060,12 @@ size_t gemm_smem() {
 
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
-                        const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s) {
+                        const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s,
+                        bool pdl) {
     const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi, KPS>();
     auto kern = k_tc_gemm<BN, NSUB, STAGES, Epi, KPS>;
     cudaLaunchConfig_t lc = {};
-    cudaLaunchAttribute at[1];
+    cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = 2;  // a CTA pair per 256-row tile
     at[0].val.clusterDim.y = 1;
@@ -1067,7 +1074,9 @@ cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUte
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
     lc.attrs = at;
-    lc.numAttrs = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    lc.numAttrs = 2;
     static int max_pairs = 0;  // pairs resident at once (the grid is persistent)
     if (!max_pairs) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -1267,6 +1276,9 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE / 2))
         return cudaErrorInvalidValue;
     const int m_tiles = (B + 2 * BM - 1) / (2 * BM);  // 256-row tiles, one per CTA pair
+    // Programmatic dependent launch hides the ~4 us between consecutive launches (a fifth of
+    // a call at B = 8192), but made the long launches of B = 65536 3% slower: on below 32768.
+    const bool pdl = B < 32768;
     cudaError_t e = cudaSuccess;
     for (int t = 0; t < Tn && e == cudaSuccess; ++t) {
         io.t = t;
@@ -1279,23 +1291,23 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
         if (!teacher) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
-            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
-            else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
-            else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s);
+            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+            else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+            else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
             ++launches;
             if (e != cudaSuccess) break;
         }
         const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
-            e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s);
+            e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
         }
         ++launches;
         if (e != cudaSuccess) break;
         const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
-            e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s);
+            e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s, pdl);
         }
         ++launches;
         if (e == cudaSuccess && hooks) e = hooks->after_step(t, s);
