@@ -838,10 +838,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const uint32_t tm = tmem_base;
     // Programmatic dependent launch (when the launch allows it): the set-up above may overlap
     // the previous kernel of the stream; every read of its outputs comes after this wait.
-    // The next kernel may then be launched, its own set-up overlapping this one.  (Both
-    // return at once for a launch without programmatic serialization.)
+    // (It returns at once for a launch without programmatic serialization.)
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
     auto wait = [&](uint32_t bar, uint32_t parity) {
         if (!s_abort && !tc::mbar_wait_bounded(bar, parity, POLLS)) {
@@ -974,6 +972,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     __syncwarp();
     tc::fence_before_sync();
+    // this CTA's work is done: the next kernel may be launched (its set-up then overlaps
+    // the tail of this one; triggering at the start instead measured slower)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc::cluster_sync();  // the leader's MMAs into this CTA's TMEM and shared memory are done
     if (warp == 1) tmem_dealloc_pair(tm, 512);
 }
