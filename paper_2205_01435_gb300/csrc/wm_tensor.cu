@@ -110,8 +110,14 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 
 
 // Gate nonlinearities from the fast exponential (relative error ~1e-6).
-__device__ __forceinline__ float sigmoid_hw(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
-__device__ __forceinline__ float tanh_hw(float x) { return fmaf(2.f, sigmoid_hw(2.f * x), -1.f); }
+// The cell's nonlinearities on the hardware tanh (tanh.approx.f32: one MUFU op, relative
+// error about 2^-11); sigma(x) = (1 + tanh(x / 2)) / 2.
+__device__ __forceinline__ float tanh_hw(float x) {
+    float y;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float sigmoid_hw(float x) { return fmaf(0.5f, tanh_hw(0.5f * x), 0.5f); }
 
 struct GemmGrid {
     int m_tiles, n_tiles, k_steps;
