@@ -43,9 +43,15 @@
  * Memory: every array argument below may be device memory (cudaMalloc'd,
  * managed) or host memory (pinned or pageable); the library tells them apart
  * with cudaPointerGetAttributes.  Host arrays are staged through device
- * buffers owned by the handle, on the call's stream; if any output is host
- * memory the call synchronises the stream before it returns.  All arrays are
- * dense, row-major, in the layouts given, and owned by the caller.
+ * buffers owned by the handle.  In general they are copied whole on the call's
+ * stream, inputs before the kernels and outputs after them.  When the call runs
+ * step by step (wm_rollout on the tensor-core family, T > 1, a stream that is not
+ * capturing), per-step slabs move on two copy streams owned by the handle
+ * instead: the mask slab of step t goes up ahead of step t, and step t's output
+ * slabs come down as soon as step t is done, overlapping the other steps.  A call
+ * with a host output, or with per-step staging, returns only when every copy
+ * touching the caller's arrays is complete (also when it returns an error).  All
+ * arrays are dense, row-major, in the layouts given, and owned by the caller.
  *
  * Errors: argument errors are returned synchronously and leave outputs
  * untouched.  Device-side errors (a bounded wait that gave up) are recorded in
