@@ -7,16 +7,19 @@
 //                                              done, freeze                       (a5..a9)
 //
 // Operands: bf16, K-major, loaded by TMA into 128-byte-swizzled shared-memory
-// tiles (box 64 K x rows), consumed by tcgen05.mma (cta_group::1, M = 128) with
-// fp32 accumulators in TMEM.  Each GEMM kernel is persistent (one CTA per SM,
-// tiles in N-fastest order so that concurrently running CTAs share the A rows in
+// tiles (box 64 K x rows), consumed by tcgen05.mma.cta_group::2 (M = 256, a CTA
+// pair per tile, each CTA holding 128 A rows and half of the B rows) with fp32
+// accumulators in TMEM.  Each GEMM kernel is persistent (one CTA per SM, 256-row
+// tiles in N-fastest order so that concurrently running pairs share the A rows in
 // L2) and warp-specialised:
-//   warp 0      TMA producer: a ring of STAGES (A, B) tiles guarded by full /
-//               empty mbarriers,
-//   warp 1      owns TMEM (512 columns) and issues the MMAs; accumulators are
+//   warp 0      TMA producer (both CTAs): a ring of STAGES stages of KPS k-steps,
+//               one full and one empty mbarrier per stage,
+//   warp 1      owns TMEM (512 columns, pair allocation); in the leader CTA it
+//               issues the MMAs and commits once per stage; accumulators are
 //               double-buffered when a tile is at most 256 columns wide, so the
 //               epilogue of one tile overlaps the MMAs of the next,
-//   warps 2..5  the epilogue: one thread per accumulator row (TMEM lane).
+//   warps 2..17 the epilogue: four warps per TMEM lane quadrant (one accumulator
+//               row per thread), splitting the tile's columns.
 // The operand X = [z_t | h_t] (bf16) is ping-ponged between two buffers: the
 // gate epilogue writes h_{t+1} and the head epilogue z_{t+1} into the other one.
 // The carried state c, h (fp32) lives in HBM.  All waits are bounded; on expiry a
