@@ -79,6 +79,8 @@ def _load():
             lib.orc_select_action.restype = C.c_int
             lib.orc_rollout.argtypes = [P, P, C.c_int, C.c_int, C.c_uint64, C.c_uint32] + [P] * 18
             lib.orc_rollout.restype = C.c_int
+            lib.orc_step.argtypes = [P, P, C.c_int, P, C.c_uint32] + [P] * 19
+            lib.orc_step.restype = C.c_int
             lib.orc_mdn_nll.argtypes = [P, P, C.c_int, C.c_int] + [P] * 7
             lib.orc_mdn_nll.restype = C.c_int
             _lib = lib
@@ -226,6 +228,42 @@ def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset:
                          _ptr(out["comp_margin"]), _ptr(out["done_margin"]))
     if rc != 0:
         raise ValueError(f"orc_rollout failed ({rc})")
+    return out
+
+
+def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=None, mask=None,
+         a_use=None, h_use=None, k_use=None, nthreads: int = 1) -> dict:
+    """One dream step (a1..a8) of B = len(episodes) episodes started from the state
+    (z [B,Z], h [B,H], c [B,H], frozen [B]); episodes are global Philox indices.
+    a_use / h_use / k_use replace what flows downstream of the action, h' and
+    component decisions (the returned decisions and margins are the oracle's own)."""
+    lib = _load()
+    Z, A, H, K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
+    ep = np.ascontiguousarray(episodes, dtype=np.uint64).reshape(-1)
+    B = ep.shape[0]
+    W = (A + 31) // 32
+    z, h, c = _f32(z).reshape(B, Z), _f32(h).reshape(B, H), _f32(c).reshape(B, H)
+    fz = None if frozen is None else np.ascontiguousarray(frozen, dtype=np.uint8).reshape(B)
+    mk = None if mask is None else np.ascontiguousarray(mask, dtype=np.uint32).reshape(B, W)
+    au = None if a_use is None else np.ascontiguousarray(a_use, dtype=np.int32).reshape(B)
+    hu = None if h_use is None else _f32(h_use).reshape(B, H)
+    ku = None if k_use is None else np.ascontiguousarray(k_use, dtype=np.uint8).reshape(B, Z)
+    out = {"action": np.zeros(B, np.int32), "ctrl_margin": np.zeros(B, np.float32),
+           "h": np.zeros((B, H), np.float32), "c": np.zeros((B, H), np.float32),
+           "mdn": np.zeros((B, 3 * K * Z), np.float32), "reward": np.zeros(B, np.float32),
+           "done": np.zeros(B, np.uint8), "done_margin": np.zeros(B, np.float32),
+           "comp": np.zeros((B, Z), np.uint8), "comp_margin": np.zeros((B, Z), np.float32),
+           "z_next": np.zeros((B, Z), np.float32)}
+    w = _Weights(weights)
+    cs = _cfg(cfg, nthreads)
+    rc = lib.orc_step(C.byref(cs), C.byref(w.s), B, _ptr(ep), int(step_index) & 0xFFFFFFFF,
+                      _ptr(z), _ptr(h), _ptr(c), _ptr(fz), _ptr(mk), _ptr(au), _ptr(hu), _ptr(ku),
+                      _ptr(out["action"]), _ptr(out["ctrl_margin"]), _ptr(out["h"]), _ptr(out["c"]),
+                      _ptr(out["mdn"]), _ptr(out["reward"]), _ptr(out["done"]),
+                      _ptr(out["done_margin"]), _ptr(out["comp"]), _ptr(out["comp_margin"]),
+                      _ptr(out["z_next"]))
+    if rc != 0:
+        raise ValueError(f"orc_step failed ({rc})")
     return out
 
 

@@ -347,6 +347,121 @@ static void mdn_head(const orc_cfg *cfg, const wts64 *v, const double *y, double
 
 #define INF_F ((float)INFINITY)
 
+/* Per-episode work buffers of one step. */
+typedef struct {
+    double *x, *g, *y, *mdn, *znew;
+    float *lg;
+} step_buf;
+
+static int buf_alloc(const orc_cfg *cfg, step_buf *sb)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
+    sb->x = malloc(sizeof(double) * (Z + H));
+    sb->g = malloc(sizeof(double) * 4 * H);
+    sb->y = malloc(sizeof(double) * H);
+    sb->mdn = malloc(sizeof(double) * 3 * K * Z);
+    sb->znew = malloc(sizeof(double) * Z);
+    sb->lg = malloc(sizeof(float) * (A > K ? A : K));
+    return (sb->x && sb->g && sb->y && sb->mdn && sb->znew && sb->lg) ? 0 : -1;
+}
+
+static void buf_free(step_buf *sb)
+{
+    free(sb->x); free(sb->g); free(sb->y); free(sb->mdn); free(sb->znew); free(sb->lg);
+}
+
+/*
+ * One dream step (a1..a8) of one live episode e at global step s.  The state
+ * z [Z], h [H], c [H] enters as fp32 values held in doubles and leaves as
+ * (z_{t+1}, h', c'), again fp32 values.  mw: the step's mask words or NULL.
+ *
+ * Three optional overrides serve step-anchored checks, where the step is
+ * replayed with another implementation's decisions so that every later value
+ * stays comparable.  The oracle always reports its own decisions and margins;
+ * an override only replaces what flows downstream of a decision:
+ *   a_use (>= -1, or -2 for none) is the action row the LSTM takes (a3);
+ *   h_use (or NULL) is the h' the heads read (a5..a7);
+ *   k_use (or NULL) gives the component each dim's z_{t+1} is drawn from (a7).
+ * The done flag is formed from the action actually taken.  Returns 1 if the
+ * episode freezes after this step (a8).
+ */
+static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64_t e,
+                        uint32_t s, double *z, double *h, double *c, const uint32_t *mw,
+                        int a_use, const float *h_use, const uint8_t *k_use,
+                        int32_t *action, float *ctrl_margin, float *reward, uint8_t *done,
+                        float *done_margin, float *mdn_out, uint8_t *comp, float *comp_margin)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
+    double *x = sb->x, *g = sb->g, *y = sb->y, *mdn = sb->mdn, *znew = sb->znew;
+    float *lg = sb->lg;
+    for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z[i]);
+    for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
+
+    /* a1: controller logits, rounded to fp32 for the decision */
+    for (int j = 0; j < A; ++j) {
+        double l = v->b_ctrl[j];
+        for (int i = 0; i < Z + H; ++i) l += x[i] * v->W_ctrl[(size_t)i * A + j];
+        lg[j] = (float)l;
+    }
+    /* a2: mask + select */
+    double u_ctrl = 0.0;
+    if (cfg->ctrl_sample && cfg->ctrl_tau > 0.0) {
+        uint32_t r4[4];
+        orc_draw(cfg->seed, e, s, 2u, 0u, r4);
+        u_ctrl = orc_uniform(r4[0]);
+    }
+    double cm;
+    int a = orc_select_action(A, lg, mw, cfg->ctrl_sample, cfg->ctrl_tau, u_ctrl, &cm);
+    *action = a;
+    if (ctrl_margin) *ctrl_margin = (float)cm;
+    if (a_use >= -1) a = a_use;
+
+    /* a3 + a4 */
+    lstm_step(cfg, v, x, a, g, c, h);
+
+    /* a5: heads on op(h') */
+    for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h_use ? (double)h_use[i] : h[i]);
+    mdn_head(cfg, v, y, mdn);
+    if (mdn_out) for (int m = 0; m < 3 * K * Z; ++m) mdn_out[m] = (float)mdn[m];
+    double r = v->b_rew, dl = v->b_done;
+    for (int i = 0; i < H; ++i) { r += y[i] * v->w_rew[i]; dl += y[i] * v->w_done[i]; }
+    *reward = (float)r;
+    float dlf = (float)dl;
+    if (done_margin) *done_margin = fabsf(dlf);
+    int is_noop = cfg->noop_terminates && a == A - 1;
+    *done = (uint8_t)((dlf > 0.0f) || is_noop);
+
+    /* a6 + a7: per-dim mixture sample */
+    const double scale = cfg->sigma_sqrt_tau ? sqrt(cfg->mdn_tau) : 1.0;
+    for (int d = 0; d < Z; ++d) {
+        double u = 0.0, eps = 0.0;
+        if (cfg->mdn_tau > 0.0) {
+            uint32_t ru[4], rn[4];
+            orc_draw(cfg->seed, e, s, 0u, (uint32_t)(d / 4), ru);
+            u = orc_uniform(ru[d % 4]);
+            orc_draw(cfg->seed, e, s, 1u, (uint32_t)(d / 4), rn);
+            double e0, e1;
+            int pair = (d % 4) / 2;
+            orc_box_muller(rn[2 * pair], rn[2 * pair + 1], &e0, &e1);
+            eps = (d % 2 == 0) ? e0 : e1;
+        }
+        for (int k = 0; k < K; ++k) lg[k] = (float)mdn[d * K + k];
+        const double *mu = mdn + K * Z + d * K, *ls = mdn + 2 * K * Z + d * K;
+        double zd, mg;
+        int k = orc_sample_dim(K, cfg->mdn_tau, cfg->sigma_sqrt_tau, lg, mu, ls, u, eps, &zd, &mg);
+        if (comp) comp[d] = (uint8_t)k;
+        if (comp_margin) comp_margin[d] = (float)mg;
+        if (k_use && k_use[d] != k) {
+            int kf = k_use[d] < K ? k_use[d] : K - 1;
+            zd = cfg->mdn_tau > 0.0 ? mu[kf] + exp(ls[kf]) * scale * eps : mu[kf];
+        }
+        znew[d] = zd;
+    }
+    for (int d = 0; d < Z; ++d) z[d] = (double)(float)znew[d];   /* fp32 latent state */
+    /* a8 */
+    return (cfg->done_terminates && dlf > 0.0f) || is_noop;
+}
+
 static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int T,
                            uint64_t episode_offset, uint32_t t0,
                            const float *z0, const float *h0, const float *c0,
@@ -360,12 +475,11 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
     const int M = 3 * K * Z, W = (A + 31) / 32;
     const uint64_t e = episode_offset + (uint64_t)b;
     double *z = malloc(sizeof(double) * Z), *h = malloc(sizeof(double) * H);
-    double *c = malloc(sizeof(double) * H), *x = malloc(sizeof(double) * (Z + H));
-    double *g = malloc(sizeof(double) * 4 * H), *y = malloc(sizeof(double) * H);
-    double *mdn = malloc(sizeof(double) * M), *znew = malloc(sizeof(double) * Z);
-    float *lg = malloc(sizeof(float) * (A > K ? A : K));
-    if (!z || !h || !c || !x || !g || !y || !mdn || !znew || !lg) {
-        free(z); free(h); free(c); free(x); free(g); free(y); free(mdn); free(znew); free(lg);
+    double *c = malloc(sizeof(double) * H);
+    step_buf sb;
+    int ok = buf_alloc(cfg, &sb) == 0 && z && h && c;
+    if (!ok) {
+        free(z); free(h); free(c); buf_free(&sb);
         return -1;
     }
     for (int i = 0; i < Z; ++i) z[i] = z0[(size_t)b * Z + i];
@@ -381,87 +495,27 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
         const size_t tb = (size_t)t * B + b;
         if (frozen) {
             actions[tb] = -1; rewards[tb] = 0.0f; done[tb] = 1;
-            for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
-            if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
-            if (c_seq) for (int i = 0; i < H; ++i) c_seq[tb * H + i] = (float)c[i];
             if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = 0.0f;
             if (comp_seq) for (int d = 0; d < Z; ++d) comp_seq[tb * Z + d] = 255;
             if (ctrl_margin) ctrl_margin[tb] = INF_F;
             if (done_margin) done_margin[tb] = INF_F;
             if (comp_margin) for (int d = 0; d < Z; ++d) comp_margin[tb * Z + d] = INF_F;
-            continue;
+        } else {
+            frozen = step_episode(cfg, v, &sb, e, s, z, h, c, mask ? mask + tb * W : NULL,
+                                  -2, NULL, NULL, &actions[tb],
+                                  ctrl_margin ? &ctrl_margin[tb] : NULL, &rewards[tb], &done[tb],
+                                  done_margin ? &done_margin[tb] : NULL,
+                                  mdn_seq ? mdn_seq + tb * M : NULL,
+                                  comp_seq ? comp_seq + tb * Z : NULL,
+                                  comp_margin ? comp_margin + tb * Z : NULL);
         }
-        for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z[i]);
-        for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
-
-        /* a1: controller logits, rounded to fp32 for the decision */
-        for (int j = 0; j < A; ++j) {
-            double l = v->b_ctrl[j];
-            for (int i = 0; i < Z + H; ++i) l += x[i] * v->W_ctrl[(size_t)i * A + j];
-            lg[j] = (float)l;
-        }
-        /* a2: mask + select */
-        double u_ctrl = 0.0;
-        if (cfg->ctrl_sample && cfg->ctrl_tau > 0.0) {
-            uint32_t r4[4];
-            orc_draw(cfg->seed, e, s, 2u, 0u, r4);
-            u_ctrl = orc_uniform(r4[0]);
-        }
-        double cm;
-        const uint32_t *mw = mask ? mask + tb * W : NULL;
-        int a = orc_select_action(A, lg, mw, cfg->ctrl_sample, cfg->ctrl_tau, u_ctrl, &cm);
-        actions[tb] = a;
-        if (ctrl_margin) ctrl_margin[tb] = (float)cm;
-
-        /* a3 + a4 */
-        lstm_step(cfg, v, x, a, g, c, h);
+        for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
         if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
         if (c_seq) for (int i = 0; i < H; ++i) c_seq[tb * H + i] = (float)c[i];
-
-        /* a5: heads on op(h') */
-        for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h[i]);
-        mdn_head(cfg, v, y, mdn);
-        if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = (float)mdn[m];
-        double r = v->b_rew, dl = v->b_done;
-        for (int i = 0; i < H; ++i) { r += y[i] * v->w_rew[i]; dl += y[i] * v->w_done[i]; }
-        rewards[tb] = (float)r;
-        float dlf = (float)dl;
-        if (done_margin) done_margin[tb] = fabsf(dlf);
-        int is_noop = cfg->noop_terminates && a == A - 1;
-        int dn = (dlf > 0.0f) || is_noop;
-        done[tb] = (uint8_t)dn;
-
-        /* a6 + a7: per-dim mixture sample */
-        for (int d = 0; d < Z; ++d) {
-            double u = 0.0, eps = 0.0;
-            if (cfg->mdn_tau > 0.0) {
-                uint32_t ru[4], rn[4];
-                orc_draw(cfg->seed, e, s, 0u, (uint32_t)(d / 4), ru);
-                u = orc_uniform(ru[d % 4]);
-                orc_draw(cfg->seed, e, s, 1u, (uint32_t)(d / 4), rn);
-                double e0, e1;
-                int pair = (d % 4) / 2;
-                orc_box_muller(rn[2 * pair], rn[2 * pair + 1], &e0, &e1);
-                eps = (d % 2 == 0) ? e0 : e1;
-            }
-            for (int k = 0; k < K; ++k) lg[k] = (float)mdn[d * K + k];
-            double zd, mg;
-            int k = orc_sample_dim(K, cfg->mdn_tau, cfg->sigma_sqrt_tau, lg,
-                                   mdn + K * Z + d * K, mdn + 2 * K * Z + d * K, u, eps, &zd, &mg);
-            znew[d] = zd;
-            if (comp_seq) comp_seq[tb * Z + d] = (uint8_t)k;
-            if (comp_margin) comp_margin[tb * Z + d] = (float)mg;
-        }
-        for (int d = 0; d < Z; ++d) {
-            z[d] = (double)(float)znew[d];   /* fp32 latent state */
-            z_out[((size_t)(t + 1) * B + b) * Z + d] = (float)z[d];
-        }
-        /* a8 */
-        if ((cfg->done_terminates && dlf > 0.0f) || is_noop) frozen = 1;
     }
     if (h_final) for (int i = 0; i < H; ++i) h_final[(size_t)b * H + i] = (float)h[i];
     if (c_final) for (int i = 0; i < H; ++i) c_final[(size_t)b * H + i] = (float)c[i];
-    free(z); free(h); free(c); free(x); free(g); free(y); free(mdn); free(znew); free(lg);
+    free(z); free(h); free(c); buf_free(&sb);
     return 0;
 }
 
@@ -486,6 +540,73 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
                                z_out, actions, rewards, done, h_final, c_final,
                                h_seq, c_seq, mdn_seq, comp_seq,
                                ctrl_margin, comp_margin, done_margin) ? 1 : 0;
+    }
+    free_wts(&v);
+    return bad ? -2 : 0;
+}
+
+/*
+ * One dream step for B episodes from a given state: the step of orc_rollout,
+ * started from (z, h, c, frozen) instead of the previous step's results.
+ * episode[b] is episode b's global Philox index, step the global step index.
+ * The overrides a_use / h_use / k_use (see step_episode) may be NULL; a_use
+ * entries below -1 mean "no override" for that episode.  A frozen episode
+ * gives the frozen row (a = -1, r = 0, done = 1, state repeated, mdn 0,
+ * components 255, infinite margins).
+ */
+int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *episode,
+             uint32_t step, const float *z, const float *h, const float *c,
+             const uint8_t *frozen, const uint32_t *mask,
+             const int32_t *a_use, const float *h_use, const uint8_t *k_use,
+             int32_t *action, float *ctrl_margin, float *h_out, float *c_out, float *mdn_out,
+             float *reward, uint8_t *done, float *done_margin, uint8_t *comp,
+             float *comp_margin, float *z_next)
+{
+    if (check_cfg(cfg) || B < 0 || !episode || !z || !h || !c || !action || !ctrl_margin ||
+        !h_out || !c_out || !mdn_out || !reward || !done || !done_margin || !comp ||
+        !comp_margin || !z_next)
+        return -1;
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
+    const int M = 3 * K * Z, W = (A + 31) / 32;
+    wts64 v;
+    if (load_wts(cfg, w, &v, 1)) return -2;
+    int bad = 0;
+    int nt = cfg->nthreads > 0 ? cfg->nthreads : 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nt) reduction(| : bad)
+    for (int b = 0; b < B; ++b) {
+        double *zs = malloc(sizeof(double) * Z), *hs = malloc(sizeof(double) * H);
+        double *cs = malloc(sizeof(double) * H);
+        step_buf sb;
+        if (buf_alloc(cfg, &sb) || !zs || !hs || !cs) {
+            free(zs); free(hs); free(cs); buf_free(&sb);
+            bad |= 1;
+            continue;
+        }
+        for (int i = 0; i < Z; ++i) zs[i] = z[(size_t)b * Z + i];
+        for (int i = 0; i < H; ++i) { hs[i] = h[(size_t)b * H + i]; cs[i] = c[(size_t)b * H + i]; }
+        if (frozen && frozen[b]) {
+            action[b] = -1; ctrl_margin[b] = INF_F; reward[b] = 0.0f; done[b] = 1;
+            done_margin[b] = INF_F;
+            for (int m = 0; m < M; ++m) mdn_out[(size_t)b * M + m] = 0.0f;
+            for (int d = 0; d < Z; ++d) {
+                comp[(size_t)b * Z + d] = 255;
+                comp_margin[(size_t)b * Z + d] = INF_F;
+            }
+        } else {
+            step_episode(cfg, &v, &sb, episode[b], step, zs, hs, cs,
+                         mask ? mask + (size_t)b * W : NULL,
+                         a_use ? a_use[b] : -2, h_use ? h_use + (size_t)b * H : NULL,
+                         k_use ? k_use + (size_t)b * Z : NULL,
+                         &action[b], &ctrl_margin[b], &reward[b], &done[b], &done_margin[b],
+                         mdn_out + (size_t)b * M, comp + (size_t)b * Z,
+                         comp_margin + (size_t)b * Z);
+        }
+        for (int i = 0; i < Z; ++i) z_next[(size_t)b * Z + i] = (float)zs[i];
+        for (int i = 0; i < H; ++i) {
+            h_out[(size_t)b * H + i] = (float)hs[i];
+            c_out[(size_t)b * H + i] = (float)cs[i];
+        }
+        free(zs); free(hs); free(cs); buf_free(&sb);
     }
     free_wts(&v);
     return bad ? -2 : 0;

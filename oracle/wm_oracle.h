@@ -81,6 +81,23 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
                 float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
                 float *ctrl_margin, float *comp_margin, float *done_margin);
 
+/* One dream step for B episodes started from a given state (z, h, c, frozen):
+ * the step orc_rollout takes, for step-anchored comparisons.  episode[b] is the
+ * global Philox episode index of row b, step the global step index; mask is
+ * [B, ceil(A/32)] or NULL.  Optional overrides (NULL = none): a_use [B] is the
+ * action row the LSTM takes (entries < -1: none), h_use [B,H] the h' the heads
+ * read, k_use [B,Z] the components z_{t+1} is drawn from.  The outputs are the
+ * oracle's own decisions and margins and the values downstream of the
+ * overrides: action, ctrl_margin, reward, done, done_margin [B]; h_out, c_out
+ * [B,H]; mdn_out [B,3KZ]; comp, comp_margin, z_next [B,Z]. */
+int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *episode,
+             uint32_t step, const float *z, const float *h, const float *c,
+             const uint8_t *frozen, const uint32_t *mask,
+             const int32_t *a_use, const float *h_use, const uint8_t *k_use,
+             int32_t *action, float *ctrl_margin, float *h_out, float *c_out, float *mdn_out,
+             float *reward, uint8_t *done, float *done_margin, uint8_t *comp,
+             float *comp_margin, float *z_next);
+
 int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
                 const float *z_seq, const int32_t *actions, const int32_t *lengths,
                 double *nll, float *h_seq, float *c_seq, float *mdn_seq);
