@@ -1,29 +1,40 @@
 """Comparison rules shared by the GPU parity tests.
 
-Integer results (actions, done flags, mixture components) must match the
-oracle exactly, except where the oracle itself was within a hair of the
-decision boundary:
-  * controller argmax: top-2 logit gap < 1e-3;
-  * sampled controller action: |u*S - cumsum| < 1e-4 * S;
-  * mixture component: |u - C_k| < 1e-4 for some cumulative weight C_k;
-  * done: |done logit| < 1e-4.
-On the bf16 path the rounding of an operand to bf16 is itself a quantisation
-step: where the GPU's fp32 value and the oracle's value fall on two sides of a
-bf16 rounding midpoint, the two trajectories differ by one bf16 ulp from then
-on.  So on that path a flip is also excused when it is *explained*: the
-oracle's margin is smaller than the change of the deciding quantity recomputed
-from the GPU's own outputs (which must themselves be within tolerance).
-Flips must be < 0.1% of the draws, and an episode is compared no further after
-its first flip (its trajectory legitimately diverges).  Continuous values are
-compared with max-abs error <= 1e-4 (fp32 path) or <= 2e-2 (bf16 path) up to
-that point.
+Free-running rollouts are checked step by step against the oracle started from
+the GPU's own state (step-anchored parity).  For every step t of every checked
+episode, the oracle replays the step from the state the GPU entered it with
+(z_t, h_{t-1}, c_{t-1} and whether the episode was frozen), so every step is
+compared, however far the two trajectories would have drifted apart if each
+had run on its own:
+
+  * decisions (action, done, mixture component of every latent dim) must equal
+    the oracle's, except where the oracle's own margin puts it within a hair
+    of the decision boundary:
+      - controller argmax: top-2 logit gap < 1e-3;
+      - sampled controller action: |u*S - cumsum| / S < 1e-4;
+      - mixture component: |u - C_k| < 1e-4 for the nearest cumulative weight;
+      - done: |done logit| < 1e-4;
+    such excused flips must be < 0.1% of the draws;
+  * values (h', c', head outputs, reward, z_{t+1}) must be within max-abs 1e-4
+    (fp32 path) or 2e-2 (bf16 path) of the oracle's.  The bf16 path is held to
+    2e-2 of both the bf16-emulating oracle and the plain fp32 oracle.
+
+To keep every value comparable after an excused flip, the replay takes the
+GPU's decisions downstream of the oracle's own: its action row into the LSTM,
+its h' into the heads (the second state point inside a step) and its
+components into z_{t+1}.  The oracle still reports, and is judged on, its own
+decisions.  The teacher-forced check compares the GPU's whole chain with the
+oracle's directly.
 """
 from __future__ import annotations
+
+import os
 
 import numpy as np
 
 TOL = {"fp32": 1e-4, "bf16": 2e-2}
 CTRL_GAP, CTRL_SAMPLE_GAP, COMP_GAP, DONE_GAP = 1e-3, 1e-4, 1e-4, 1e-4
+NT = os.cpu_count() or 1
 
 
 def np_(x):
@@ -36,180 +47,142 @@ def np_(x):
     return np.asarray(x)
 
 
-def _bf16(x):
-    import torch
-    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16).double().numpy()
+def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=None, t0: int = 0,
+                  h0=None, c0=None, done0=None, orc=None, nthreads: int = NT) -> dict:
+    """Step-anchored parity of a GPU rollout of B episodes.
 
-
-class _Explain:
-    """Recomputes deciding quantities from the GPU's own outputs (fp64 math)."""
-
-    def __init__(self, cfg, w):
-        rb = cfg.get("precision") == "bf16"
-        self.conv = _bf16 if rb else (lambda a: np.asarray(a, np.float64))
-        self.Wc = self.conv(w["W_ctrl"])
-        self.bc = np.asarray(w["b_ctrl"], np.float64)
-        self.wd = self.conv(w["w_done"])
-        self.bd = float(w["b_done"])
-
-    def ctrl_logits(self, z, h):
-        x = np.concatenate([self.conv(z), self.conv(h)])
-        return x @ self.Wc + self.bc
-
-    def done_logit(self, h):
-        return float(self.conv(h) @ self.wd + self.bd)
-
-    @staticmethod
-    def ctrl_cdf(logits, valid, tau):
-        l = np.where(valid, np.asarray(logits, np.float64), -np.inf) / tau
-        p = np.exp(l - l[valid].max())
-        return np.cumsum(p / p.sum())
-
-    @staticmethod
-    def cum_weights(logits, tau):
-        l = np.asarray(logits, np.float64) / tau
-        p = np.exp(l - l.max())
-        return np.cumsum(p / p.sum())
-
-
-def check_rollout(g: dict, o: dict, cfg: dict, idx=None, check_final: bool = True,
-                  weights: dict | None = None, h0=None, mask=None) -> dict:
-    """g: GPU outputs (batch axis indexed by idx); o: oracle outputs for those episodes;
-    mask: the [T, B, W] action mask of the oracle's episodes (sampled-controller checks)."""
+    g: the GPU's outputs with their per-step sequences (z, actions, rewards, done,
+    h_seq, c_seq, mdn_seq, comp_seq; optional h_final, c_final), batch axis = the
+    checked episodes.  z0, mask [T, B, W], h0, c0, done0: the inputs of those
+    episodes.  episodes: their global Philox indices (default 0..B-1); t0: the
+    global index of step 0."""
+    if orc is None:
+        import oracle as orc
     prec = cfg.get("precision", "fp32")
     tol = TOL[prec]
     sampled = bool(cfg.get("ctrl_sample", 0)) and cfg.get("ctrl_tau", 1.0) > 0
     ctrl_thr = CTRL_SAMPLE_GAP if sampled else CTRL_GAP
-    tau = cfg.get("mdn_tau", 1.0)
-    K = cfg["k_mix"]
-    T, Bo = o["actions"].shape
-    idx = np.arange(Bo) if idx is None else np.asarray(idx)
-    ga = np_(g["actions"])[:, idx]
-    gd = np_(g["done"])[:, idx]
-    gr = np_(g["rewards"])[:, idx]
-    gz = np_(g["z"])[:, idx]
-    gcomp = np_(g["comp_seq"])[:, idx] if g.get("comp_seq") is not None else None
-    gh = np_(g["h_seq"])[:, idx] if g.get("h_seq") is not None else None
-    gc = np_(g["c_seq"])[:, idx] if g.get("c_seq") is not None else None
-    gm = np_(g["mdn_seq"])[:, idx] if g.get("mdn_seq") is not None else None
-    ex = _Explain(cfg, weights) if (prec == "bf16" and weights is not None and gh is not None) else None
-    Z = gz.shape[-1]
-    H = cfg["h_dim"]
-    assert np.array_equal(gz[0], o["z"][0])
-    stats = {"flips": 0, "explained_flips": 0, "draws": 0, "compared": 0, "worst": 0.0,
-             "kinds": {"action": 0, "done": 0, "component": 0}, "first_flip_steps": []}
-    clean = np.ones(Bo, bool)
+    Z, A, H, K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
+    ga, gd, gr = np_(g["actions"]), np_(g["done"]), np_(g["rewards"])
+    gz, gh, gc = np_(g["z"]), np_(g["h_seq"]), np_(g["c_seq"])
+    gm, gk = np_(g["mdn_seq"]), np_(g["comp_seq"])
+    T, B = ga.shape
+    ep = np.arange(B, dtype=np.uint64) if episodes is None else np.asarray(episodes, np.uint64)
+    assert np.array_equal(gz[0], np.asarray(z0, np.float32)), "z_out[0] must be z0"
+    h = np.zeros((B, H), np.float32) if h0 is None else np.asarray(h0, np.float32)
+    c = np.zeros((B, H), np.float32) if c0 is None else np.asarray(c0, np.float32)
+    frozen = np.zeros(B, bool) if done0 is None else np.asarray(done0).astype(bool)
+    refs = [(cfg, tol)]
+    if prec == "bf16":
+        refs.append((dict(cfg, precision="fp32"), TOL["bf16"]))
+    st = {"flips": 0, "draws": 0, "compared": 0, "frozen_steps": 0, "worst": 0.0,
+          "kinds": {"action": 0, "done": 0, "component": 0}, "flip_margins": []}
 
-    def flip(b, explained=False, kind="action", t=0):
-        stats["flips"] += 1
-        stats["explained_flips"] += int(explained)
-        stats["kinds"][kind] += 1
-        stats["first_flip_steps"].append(t)
-        clean[b] = False
+    def flip(kind, margin):
+        st["flips"] += 1
+        st["kinds"][kind] += 1
+        st["flip_margins"].append(float(margin))
 
-    for b in range(Bo):
+    last = None
+    for t in range(T):
+        mk = None if mask is None else np.asarray(mask)[t]
+        for ri, (rcfg, rtol) in enumerate(refs):
+            s = orc.step(rcfg, weights, ep, t0 + t, gz[t], h, c, frozen=frozen, mask=mk,
+                         a_use=ga[t], h_use=gh[t], k_use=gk[t], nthreads=nthreads)
+            if ri == 0:
+                last = s
+            live = ~frozen
+            where = f"t={t}"
+            # values downstream of the shared decisions
+            for key, gv, ov in (("h", gh[t], s["h"]), ("c", gc[t], s["c"]),
+                                ("mdn", gm[t], s["mdn"]), ("reward", gr[t], s["reward"]),
+                                ("z", gz[t + 1], s["z_next"])):
+                e = np.abs(gv.astype(np.float64) - ov.astype(np.float64))
+                e = e.reshape(B, -1).max(axis=1) if e.ndim > 1 else e
+                bad = np.nonzero(live & (e > rtol))[0]
+                assert not len(bad), (f"{key} {where} episodes {ep[bad][:8]} err {e[bad][:8]} "
+                                      f"(tol {rtol}, {rcfg['precision']} oracle)")
+                if ri == 0 and live.any():
+                    st["worst"] = max(st["worst"], float(e[live].max()))
+            if ri:
+                continue
+            # frozen rows are exact copies
+            fz = np.nonzero(frozen)[0]
+            if len(fz):
+                assert np.all(ga[t, fz] == -1) and np.all(gd[t, fz] == 1), where
+                assert np.all(gr[t, fz] == 0) and np.all(gk[t, fz] == 255), where
+                assert np.array_equal(gz[t + 1, fz], gz[t, fz]), where
+                assert np.array_equal(gh[t, fz], h[fz]) and np.array_equal(gc[t, fz], c[fz]), where
+                assert np.all(gm[t, fz] == 0), where
+                st["frozen_steps"] += len(fz)
+            # decisions: equal, or excused by the oracle's own margin
+            nl = int(live.sum())
+            st["draws"] += nl * (Z + 2)
+            st["compared"] += nl
+            for b in np.nonzero(live & (ga[t] != s["action"]))[0]:
+                m = s["ctrl_margin"][b]
+                assert m < ctrl_thr, (f"action {where} episode {ep[b]}: gpu {ga[t, b]} oracle "
+                                      f"{s['action'][b]} margin {m}")
+                flip("action", m)
+            for b in np.nonzero(live & (gd[t] != s["done"]))[0]:
+                m = s["done_margin"][b]
+                assert m < DONE_GAP, (f"done {where} episode {ep[b]}: gpu {gd[t, b]} oracle "
+                                      f"{s['done'][b]} margin {m}")
+                flip("done", m)
+            bb, dd = np.nonzero(live[:, None] & (gk[t] != s["comp"]))
+            for b, d in zip(bb, dd):
+                m = s["comp_margin"][b, d]
+                assert m < COMP_GAP, (f"component {where} episode {ep[b]} dim {d}: gpu "
+                                      f"{gk[t, b, d]} oracle {s['comp'][b, d]} margin {m}")
+                flip("component", m)
+        # the state the GPU carries into the next step
+        h, c = gh[t], gc[t]
+        if cfg.get("done_terminates"):
+            frozen = frozen | (gd[t] == 1)
+        if cfg.get("noop_terminates"):
+            frozen = frozen | (ga[t] == A - 1)
+    if T > 0 and g.get("h_final") is not None:
+        for key, gv in (("h_final", g["h_final"]), ("c_final", g["c_final"])):
+            e = float(np.abs(np_(gv).astype(np.float64)
+                             - last[key[0]].astype(np.float64)).max()) if B else 0.0
+            assert e <= tol, f"{key} err {e}"
+    f, d = st["flips"], st["draws"]
+    assert f <= max(1, 0.001 * d), f"{f} excused flips in {d} draws: {st['kinds']}"
+    return st
+
+
+def check_free_running(g: dict, o: dict, cfg: dict) -> dict:
+    """Compare a GPU rollout with the oracle's own free-running rollout o of the same
+    episodes, up to each episode's first decision mismatch, which must be excused by
+    the oracle's margin (after it the two trajectories legitimately differ).  Returns
+    how many (episode, step) pairs were compared before the first mismatch."""
+    tol = TOL[cfg.get("precision", "fp32")]
+    sampled = bool(cfg.get("ctrl_sample", 0)) and cfg.get("ctrl_tau", 1.0) > 0
+    ctrl_thr = CTRL_SAMPLE_GAP if sampled else CTRL_GAP
+    ga, gd, gr, gz = (np_(g[k]) for k in ("actions", "done", "rewards", "z"))
+    gk = np_(g["comp_seq"]) if g.get("comp_seq") is not None else None
+    T, B = ga.shape
+    st = {"compared": 0, "diverged": 0}
+    for b in range(B):
         for t in range(T):
-            stats["draws"] += Z + 1
-            if t == 0:
-                h_prev = np.zeros(H) if h0 is None else np_(h0)[idx[b]]
-            else:
-                h_prev = gh[t - 1, b] if gh is not None else None
             if ga[t, b] != o["actions"][t, b]:
-                m = o["ctrl_margin"][t, b]
-                if m < ctrl_thr:
-                    flip(b, False, "action", t)
-                    break
-                assert ex is not None and h_prev is not None, (
-                    f"action flip at t={t} b={idx[b]}: gpu {ga[t, b]} oracle {o['actions'][t, b]} "
-                    f"margin {m}")
-                lg = ex.ctrl_logits(gz[t, b], h_prev)
-                a_g, a_o = int(ga[t, b]), int(o["actions"][t, b])
-                if not sampled:
-                    # explained if, on the GPU's own values, the GPU's choice is at least as good
-                    assert a_g >= 0 and a_o >= 0 and lg[a_g] >= lg[a_o] - 1e-6 and m < 2e-2, (
-                        f"unexplained action flip t={t} b={idx[b]} margin {m}")
-                else:
-                    # explained if the CDF moved by more than the oracle's margin between the
-                    # GPU's own values and the oracle's
-                    assert mask is not None, "sampled-controller checks need the mask"
-                    A = lg.shape[0]
-                    valid = np.unpackbits(np.asarray(mask[t, b], np.uint32).view(np.uint8),
-                                          bitorder="little")[:A].astype(bool)
-                    ho = np.zeros(H) if t == 0 and h0 is None else (
-                        np_(h0)[idx[b]] if t == 0 else o["h_seq"][t - 1, b])
-                    lo = ex.ctrl_logits(o["z"][t, b], ho)
-                    tau_c = cfg.get("ctrl_tau", 1.0)
-                    shift = float(np.abs(ex.ctrl_cdf(lg, valid, tau_c)
-                                         - ex.ctrl_cdf(lo, valid, tau_c))[valid].max())
-                    assert m < max(CTRL_SAMPLE_GAP, shift + 1e-7) and m < 2e-2, (
-                        f"unexplained sampled-action flip t={t} b={idx[b]} margin {m} shift {shift}")
-                flip(b, True, "action", t)
+                assert o["ctrl_margin"][t, b] < ctrl_thr, (t, b, o["ctrl_margin"][t, b])
+                st["diverged"] += 1
                 break
             if gd[t, b] != o["done"][t, b]:
-                m = o["done_margin"][t, b]
-                if m < DONE_GAP:
-                    flip(b, False, "done", t)
-                    break
-                assert ex is not None, f"done flip at t={t} b={idx[b]} margin {m}"
-                dl = ex.done_logit(gh[t, b])
-                assert (dl > 0) == bool(gd[t, b]) and m < 2e-2, (
-                    f"unexplained done flip t={t} b={idx[b]} margin {m} gpu logit {dl}")
-                flip(b, True, "done", t)
+                assert o["done_margin"][t, b] < DONE_GAP, (t, b, o["done_margin"][t, b])
+                st["diverged"] += 1
                 break
-            err = abs(float(gr[t, b]) - float(o["rewards"][t, b]))
-            stats["worst"] = max(stats["worst"], err)
-            assert err <= tol, f"reward t={t} b={idx[b]} err {err}"
-            if gh is not None:
-                e = float(np.abs(gh[t, b] - o["h_seq"][t, b]).max())
-                stats["worst"] = max(stats["worst"], e)
-                assert e <= tol, f"h t={t} b={idx[b]} err {e}"
-                e = float(np.abs(gc[t, b] - o["c_seq"][t, b]).max())
-                assert e <= tol, f"c t={t} b={idx[b]} err {e}"
-            if gm is not None:
-                e = float(np.abs(gm[t, b] - o["mdn_seq"][t, b]).max())
-                stats["worst"] = max(stats["worst"], e)
-                assert e <= tol, f"mdn t={t} b={idx[b]} err {e}"
-            if gcomp is not None:
-                bad = np.nonzero(gcomp[t, b] != o["comp_seq"][t, b])[0]
-                if len(bad):
-                    m = o["comp_margin"][t, b, bad]
-                    if np.all(m < COMP_GAP):
-                        flip(b, False, "component", t)
-                        break
-                    assert ex is not None and gm is not None and tau > 0, (
-                        f"component flip at t={t} b={idx[b]} dims {bad} margins {m}")
-                    for d in bad:
-                        cg = ex.cum_weights(gm[t, b, d * K:(d + 1) * K], tau)
-                        co = ex.cum_weights(o["mdn_seq"][t, b, d * K:(d + 1) * K], tau)
-                        shift = float(np.abs(cg - co)[:-1].max())
-                        assert o["comp_margin"][t, b, d] < max(COMP_GAP, shift + 1e-7), (
-                            f"unexplained component flip t={t} b={idx[b]} d={d} "
-                            f"margin {o['comp_margin'][t, b, d]} weight shift {shift}")
-                    flip(b, True, "component", t)
-                    break
+            if gk is not None and not np.array_equal(gk[t, b], o["comp_seq"][t, b]):
+                dd = np.nonzero(gk[t, b] != o["comp_seq"][t, b])[0]
+                assert np.all(o["comp_margin"][t, b, dd] < COMP_GAP), (t, b, dd)
+                st["diverged"] += 1
+                break
+            assert abs(float(gr[t, b]) - float(o["rewards"][t, b])) <= tol, (t, b)
             e = float(np.abs(gz[t + 1, b] - o["z"][t + 1, b]).max())
-            if e > tol:
-                # a component flip without comp_seq shows up as a jump in z
-                d = int(np.argmax(np.abs(gz[t + 1, b] - o["z"][t + 1, b])))
-                assert gcomp is None and o["comp_margin"][t, b, d] < COMP_GAP, (
-                    f"z t={t + 1} b={idx[b]} dim {d} err {e} margin {o['comp_margin'][t, b, d]}")
-                flip(b, False, "component", t)
-                break
-            stats["worst"] = max(stats["worst"], e)
-            stats["compared"] += 1
-    if check_final and g.get("h_final") is not None and "h_final" in o:
-        hf = np_(g["h_final"])[idx]
-        cf = np_(g["c_final"])[idx]
-        for b in np.nonzero(clean)[0]:
-            assert float(np.abs(hf[b] - o["h_final"][b]).max()) <= tol
-            assert float(np.abs(cf[b] - o["c_final"][b]).max()) <= tol
-    f, d = stats["flips"], stats["draws"]
-    assert f < 0.001 * d or f <= 1, f"{f} flips in {d} draws"
-    # after a flip an episode legitimately diverges; still demand real coverage (a path that
-    # diverged systematically would flip within the first steps of every episode)
-    assert stats["compared"] >= 0.1 * T * Bo, f"only {stats['compared']} of {T * Bo} steps compared: {stats}"
-    stats["clean_episodes"] = int(clean.sum())
-    return stats
+            assert e <= tol, (t, b, e)
+            st["compared"] += 1
+    return st
 
 
 def check_teacher(g: dict, o: dict, precision: str, nll_rtol: float = 1e-3):

@@ -7,7 +7,7 @@ import pytest
 import torch
 
 import synth
-from parity import check_rollout, check_teacher, np_
+from parity import check_free_running, check_rollout, check_teacher, np_
 
 pytestmark = pytest.mark.gpu
 NT = os.cpu_count() or 1
@@ -31,25 +31,10 @@ def _spread(B, n):
     return np.unique(np.linspace(0, B - 1, n).round().astype(np.int64))
 
 
-def _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=False):
-    """Oracle rollout of episodes idx (Philox keyed by their global index)."""
-    outs = []
-    idx = list(idx)
-    # contiguous runs share one call
-    start = 0
-    while start < len(idx):
-        end = start
-        while end + 1 < len(idx) and idx[end + 1] == idx[end] + 1:
-            end += 1
-        lo, hi = idx[start], idx[end] + 1
-        outs.append(orc.rollout(cfg, w, z0[lo:hi], None if mask is None else mask[:, lo:hi], T,
-                                episode_offset=lo, want_seq=want_seq, nthreads=NT))
-        start = end + 1
-    cat = {}
-    for k in outs[0]:
-        ax = 0 if k in ("h_final", "c_final") else 1
-        cat[k] = np.concatenate([o[k] for o in outs], axis=ax)
-    return cat
+def _sub(g, idx):
+    """The batch columns idx of a rollout's outputs (as numpy)."""
+    return {k: (np_(v)[idx] if k in ("h_final", "c_final") else np_(v)[:, idx])
+            for k, v in g.items() if v is not None}
 
 
 PATHS_SMALL = ["stepwise", "auto"]
@@ -103,9 +88,12 @@ def test_rollout_tiny_full(wm, orc, path):
     m = wm.WorldModel(dict(cfg, path=path), w)
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
     torch.cuda.synchronize()
+    r = check_rollout(g, cfg, w, z0, mask, orc=orc)
+    assert r["compared"] == B * T
+    # the fp32 path also follows the oracle's own free-running trajectory
     o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
-    r = check_rollout(g, o, cfg)
-    assert r["clean_episodes"] >= B - 2
+    fr = check_free_running(g, o, cfg)
+    assert fr["diverged"] <= 2, fr
 
 
 @pytest.mark.parametrize("path", PATHS_SMALL)
@@ -115,8 +103,8 @@ def test_rollout_small_bf16(wm, orc, path):
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
     torch.cuda.synchronize()
     idx = _spread(B, 48)
-    o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
-    check_rollout(g, o, cfg, idx, weights=w)
+    r = check_rollout(_sub(g, idx), cfg, w, z0[idx], mask[:, idx], episodes=idx, orc=orc)
+    assert r["compared"] == len(idx) * T
 
 
 def _rollout_sampled(wm, orc, name, n_oracle, path="auto"):
@@ -139,8 +127,10 @@ def _rollout_sampled(wm, orc, name, n_oracle, path="auto"):
     assert m.last_path == path  # the re-runs used the same kernel family as the full batch
     g = {k: np.concatenate([p[k] for p in parts], axis=0 if k in ("h_final", "c_final") else 1)
          for k in parts[0]}
-    o = _oracle_subset(orc, cfg, w, z0, mask, T, idx, want_seq=True)
-    return check_rollout(g, o, cfg, weights=w, mask=mask[:, idx])
+    r = check_rollout(g, cfg, w, z0[idx], mask[:, idx], episodes=idx, orc=orc)
+    # every live step of every sampled episode is compared
+    assert r["compared"] + r["frozen_steps"] == len(idx) * T
+    return r
 
 
 @pytest.mark.parametrize("path", ["tensor", "stepwise"])
@@ -168,8 +158,9 @@ def test_ragged_shapes_and_flags(wm, orc, path):
     m = wm.WorldModel(dict(cfg, path=path), w)
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=123456789012, t0=77,
                   want_seq=True)
+    check_rollout(g, cfg, w, z0, mask, episodes=123456789012 + np.arange(B), t0=77, orc=orc)
     o = orc.rollout(cfg, w, z0, mask, T, episode_offset=123456789012, t0=77, want_seq=True)
-    check_rollout(g, o, cfg)
+    check_free_running(g, o, cfg)
 
 
 @pytest.mark.parametrize("tau,sq", [(0.0, 0), (0.5, 1), (1.7, 0)])
@@ -178,8 +169,9 @@ def test_mixture_temperature(wm, orc, tau, sq):
     cfg2, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32", T=8)
     m = wm.WorldModel(dict(cfg, path="auto"), w)
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    check_rollout(g, cfg, w, z0, mask, orc=orc)
     o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
-    check_rollout(g, o, cfg)
+    check_free_running(g, o, cfg)
 
 
 def test_sampled_controller(wm, orc):
@@ -188,8 +180,9 @@ def test_sampled_controller(wm, orc):
     for path in PATHS_SMALL:
         m = wm.WorldModel(dict(cfg, path=path), w)
         g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+        check_rollout(g, cfg, w, z0, mask, orc=orc)
         o = orc.rollout(cfg, w, z0, mask, T, want_seq=True)
-        check_rollout(g, o, cfg)
+        check_free_running(g, o, cfg)
 
 
 def test_empty_and_zero_length(wm):
@@ -316,9 +309,8 @@ def test_fused_against_oracle(wm, orc, flags, cluster):
                   c0=_cuda(c0), done0=_cuda(done0), want_seq=True)
     torch.cuda.synchronize()
     assert m.last_path == "fused"
-    o = orc.rollout(cfg, w, z0, mask, T, episode_offset=77, t0=3, h0=h0, c0=c0, done0=done0,
-                    want_seq=True, nthreads=NT)
-    r = check_rollout(g, o, cfg, weights=w, h0=h0)
+    r = check_rollout(g, cfg, w, z0, mask, episodes=77 + np.arange(B), t0=3, h0=h0, c0=c0,
+                      done0=done0, orc=orc)
     print("fused", cluster, flags, r)
 
 
@@ -377,9 +369,8 @@ def test_tensor_against_oracle(wm, orc, name, flags):
                   c0=_cuda(c0), done0=_cuda(done0), want_seq=True)
     torch.cuda.synchronize()
     assert m.last_path == "tensor"
-    o = orc.rollout(cfg, w, z0, mask, T, episode_offset=99, t0=11, h0=h0, c0=c0, done0=done0,
-                    want_seq=True, nthreads=NT)
-    r = check_rollout(g, o, cfg, weights=w, h0=h0, mask=mask)
+    r = check_rollout(g, cfg, w, z0, mask, episodes=99 + np.arange(B), t0=11, h0=h0, c0=c0,
+                      done0=done0, orc=orc)
     print("tensor", name, flags, r)
 
 
