@@ -3,9 +3,12 @@
 
 One "step" is one wm_rollout call over the whole workload: T dream steps of B
 independent episodes (controller, mask + action choice, LSTM, mixture head,
-sampling, reward / done).  Default workload: the small-batch latency regime,
-B=1024 episodes x T=50 steps, Z=32, A=128 (30% valid mask), H=256, K=5, bf16
-operands / fp32 state (``synth.WORKLOADS['small_bf16']``).
+sampling, reward / done).  Default workload: the large-batch tensor-core
+regime, B=65536 episodes x T=64 steps, Z=128, A=512 (10% valid mask), H=1024,
+K=8, bf16 operands / fp32 state, sampled controller at temperature 1
+(``synth.WORKLOADS['large_bf16']``), the largest configuration that fits one GPU.
+For workloads whose episodes end (done head or NO-OP), ``value`` counts live
+(episode, step) pairs only; frozen pairs are executed but not counted.
 
 Timing: W untimed warm-ups, then K steps each bracketed by CUDA events on the
 launching stream, with a 512 MiB write between steps to flush the 129 MB L2.
@@ -180,6 +183,17 @@ def max_over_ranks(value: float, ws: int, device=None) -> float:
     return float(t.item())
 
 
+def sum_over_ranks(value: float, ws: int, device=None) -> float:
+    """The sum of a per-rank count over all ranks."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if ws > 1:
+        dist.all_reduce(t)
+    return float(t.item())
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -187,11 +201,11 @@ def dist_env():
     return ws, rank, local
 
 
-def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg):
-    """The same rollout through the C ABI with pinned HOST arrays: copies are timed."""
+def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps):
+    """The same rollout through the C ABI with pinned HOST arrays: copies are timed.
+    env_steps: the (episode, step) pairs one call counts over all ranks."""
     import torch
 
-    env_steps = B * T * ws
     zh = torch.from_numpy(z0).pin_memory()
     mh = torch.from_numpy(mask).pin_memory()
     hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
@@ -384,13 +398,25 @@ def run_ours(args) -> None:
     total_ms = max_over_ranks(sum(times), ws, dev)
     ms_per_step = total_ms / args.steps
     env_steps = B * T * ws
+    live = None
+    if cfg.get("done_terminates") or cfg.get("noop_terminates"):
+        # episode b is live at step t unless it was done at an earlier step (then frozen);
+        # every timed call computes the same trajectories, so the last one's done flags count
+        d = out["done"].to(torch.int32)
+        frozen = torch.zeros_like(d)
+        frozen[1:] = (torch.cumsum(d, dim=0)[:-1] > 0).to(torch.int32)
+        live_steps = int(sum_over_ranks(int((frozen == 0).sum().item()), ws, dev))
+        live = {"live_env_steps": live_steps, "live_fraction": round(live_steps / env_steps, 4),
+                "all_pairs_env_steps_per_s": round(env_steps / (ms_per_step / 1e3), 1)}
+        env_steps = live_steps
     value = env_steps / (ms_per_step / 1e3)
 
     # e2e: the same call through the C ABI with pinned HOST buffers, copies timed.
     if args.no_e2e:
         e2e_value, h2d, d2h = None, 0, 0
     else:
-        e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg)
+        e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg,
+                                          env_steps)
 
     # roofline of the dominant kernel: its algorithmic FLOPs per launch over its own
     # event-timed average launch duration inside the timed region
@@ -422,15 +448,6 @@ def run_ours(args) -> None:
             "algorithmic_flops_per_launch": fl,
             "kernel_shares": {k: round(v[0] / all_ms, 4) for k, v in sorted(kt.items())}}
 
-    live = None
-    if cfg.get("done_terminates") or cfg.get("noop_terminates"):
-        # episode b is live at step t unless it was done at an earlier step (then frozen)
-        d = out["done"].to(torch.int32)
-        frozen = torch.zeros_like(d)
-        frozen[1:] = (torch.cumsum(d, dim=0)[:-1] > 0).to(torch.int32)
-        live_steps = int((frozen == 0).sum().item()) * ws
-        live = {"live_env_steps_per_s": round(live_steps / (ms_per_step / 1e3), 1),
-                "live_fraction": round(live_steps / (B * T * ws), 4)}
     line = {"metric": "dream env-steps/s (wm_rollout)", "value": round(value, 1),
             "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
@@ -449,7 +466,7 @@ def run_ours(args) -> None:
             "gpu_launches": launches * args.steps,
             "roofline": roof, "clocks": clk.summary()}
     if live is not None:
-        line["live_steps"] = live  # frozen (done) episode-steps are executed but not live
+        line["live_steps"] = live  # value counts live pairs; frozen pairs are executed too
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes)
     if rank == 0:
@@ -466,6 +483,17 @@ def oracle_episodes(name: str, flop_budget: float) -> int:
     return int(max(8, min(w["B"], flop_budget // per)))
 
 
+def counted_steps(cfg: dict, done) -> int:
+    """(episode, step) pairs a rollout counts: all of them, or the live ones when episodes
+    can end (an episode is live at step t unless it was done at an earlier step)."""
+    done = np.asarray(done)
+    if not (cfg.get("done_terminates") or cfg.get("noop_terminates")):
+        return int(done.size)
+    ended = np.zeros_like(done, dtype=bool)
+    ended[1:] = np.cumsum(done, axis=0)[:-1] > 0
+    return int((~ended).sum())
+
+
 def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) -> dict:
     """The oracle on the host cores (all of them), plus a one-thread figure on a tenth of the
     sample (episodes are independent, so throughput per episode-step is comparable)."""
@@ -475,16 +503,17 @@ def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) ->
     n = min(episodes or oracle_episodes(name, 2e11), B)
     threads = threads or os.cpu_count() or 1
     t0 = time.perf_counter()
-    oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+    o = oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
     dt = time.perf_counter() - t0
     n1 = max(1, n // 10)
     t1 = time.perf_counter()
-    oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1)
+    o1 = oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1)
     dt1 = time.perf_counter() - t1
-    return {"value": round(n * T / dt, 2), "unit": "env-steps/s", "cores": threads,
+    return {"value": round(counted_steps(cfg, o["done"]) / dt, 2), "unit": "env-steps/s",
+            "cores": threads,
             "kind": "oracle", "sample": f"{n} of {B} episodes x {T} steps of {name}, "
                                         f"{threads} threads, {dt:.1f} s",
-            "value_1thread": round(n1 * T / dt1, 2),
+            "value_1thread": round(counted_steps(cfg, o1["done"]) / dt1, 2),
             "sample_1thread": f"{n1} episodes x {T} steps, 1 thread, {dt1:.1f} s"}
 
 
@@ -533,10 +562,10 @@ def run_reference(args) -> None:
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+        o = oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
         times.append(time.perf_counter() - t0)
     per = sum(times) / len(times)
-    value = n * T / per
+    value = counted_steps(cfg, o["done"]) / per
     sample = f"{n} of {B} episodes x {T} steps of {name} per step, {threads} threads"
     line = {"impl": "reference", "metric": "dream env-steps/s (wm_rollout)",
             "value": round(value, 2), "unit": "env-steps/s", "n_gpus": ws, "steps": args.steps,
@@ -559,7 +588,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="small_bf16", choices=list(synth.WORKLOADS),
+    ap.add_argument("--workload", default="large_bf16", choices=list(synth.WORKLOADS),
                     help="a rollout workload, or nll (teacher-forced scoring)")
     ap.add_argument("--precision", choices=["fp32", "bf16"], default=None,
                     help="nll workload only: fp32 or bf16 path (default bf16)")
