@@ -138,9 +138,13 @@ typedef struct {
     uint8_t *comp_seq;           /* [T,B,Z] optional: chosen component (255 if frozen)*/
 } wm_rollout_io;
 
-/* Copies and packs the weights onto the current CUDA device.  The handle owns
- * that device memory until wm_destroy.  Returns WM_ERR_INVALID_ARG for bad
- * sizes (any dim <= 0, K > 32, negative temperatures) or NULL weights. */
+/* Creates a world model on the current CUDA device from the weights of the
+ * MDN-RNN (Sec. 3.3.1-3.3.2: the LSTM over [z_t, a_t] and the mixture head,
+ * plus the reward and done heads) and of the linear controller
+ * a_t = W_c [z_t, h_t] + b_c (Sec. 3.4).  Copies and packs the weights; the
+ * handle owns that device memory until wm_destroy.  Returns
+ * WM_ERR_INVALID_ARG for bad sizes (any dim <= 0, K > 32, negative
+ * temperatures) or NULL weights. */
 wm_status wm_create(const wm_config *cfg, const wm_weights *weights, wm_handle **out);
 
 /* Runs T dream steps (a1..a8 above) for B independent episodes, asynchronously
@@ -160,9 +164,11 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
  *                     (Sec. 3.3.1 padding); the recurrence still runs all T
  *   nll     [N]       output
  *   h_seq, c_seq [T,N,H], mdn_seq [T,N,M]: optional per-step outputs.
- * An action >= A or a length outside [0,T] is an argument error, detected on
- * the host only when the array is host memory; on device memory the kernels
- * treat an out-of-range action as no action and clamp lengths. */
+ * An action >= A or a length outside [0,T] is an argument error.  On host
+ * arrays it is returned by this call (outputs untouched); on device arrays the
+ * kernels find it, record WM_ERR_INVALID_ARG in the status word (returned by
+ * the next wm_sync) and go on with the action taken as no action and the
+ * length clamped to [0,T]. */
 wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
                      const int32_t *lengths, float *nll, float *h_seq, float *c_seq,
                      float *mdn_seq, void *cuda_stream);

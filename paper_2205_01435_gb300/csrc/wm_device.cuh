@@ -79,6 +79,12 @@ __device__ __forceinline__ float uniform_for_dim(unsigned long long seed, unsign
     return to_uniform(u32x4_get(v, d & 3));
 }
 
+// Records a device-side error in the status word unless one is already recorded
+// (wm_sync returns the first).
+__device__ __forceinline__ void report_status(int *status, int code) {
+    if (status) atomicCAS(status, 0, code);
+}
+
 __device__ __forceinline__ float round_bf16(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
 __device__ __forceinline__ float sigmoidf_(float x) { return 1.0f / (1.0f + expf(-x)); }

@@ -294,7 +294,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     const bool issuer = mma_warp && lane == 0;
 
     float nll_acc = 0.f;
-    const int len = p.teacher ? (p.lengths ? min(max(p.lengths[live ? b : 0], 0), p.T) : p.T) : 0;
+    const int len_in = p.teacher && p.lengths ? p.lengths[live ? b : 0] : p.T;
+    if (live && (len_in < 0 || len_in > p.T)) report_status(p.status, WM_ERR_INVALID_ARG);
+    const int len = p.teacher ? min(max(len_in, 0), p.T) : 0;
     const unsigned long long ep = p.ep0 + (unsigned long long)b;
     const int M = 3 * KZ;
     // the mask word holding this rank's actions, prefetched one step ahead
@@ -365,6 +367,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         if (p.teacher) {
             if (live) {
                 a = p.act_in[tb];
+                if (a >= A) report_status(p.status, WM_ERR_INVALID_ARG);
                 if (a < 0 || a >= A) a = -1;
             }
         } else if (!frozen) {

@@ -113,6 +113,7 @@ struct StepParams {
     uint8_t *comp_seq;
     const int32_t *lengths;
     double *nll_acc;
+    int *status;          // device status word (out-of-range teacher inputs)
 };
 
 __device__ __forceinline__ bool action_valid(const uint32_t *mw, int j) {
@@ -180,6 +181,7 @@ __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
             a = -1;
         } else if (p.teacher) {
             a = p.act_in[(size_t)p.t * p.B + b];
+            if (a >= p.A) report_status(p.status, WM_ERR_INVALID_ARG);
             if (a >= p.A || a < 0) a = -1;
         } else {
             a = select_action_warp(p, b);
@@ -311,6 +313,7 @@ __global__ void __launch_bounds__(128) k_sample(StepParams p) {
             float tot = 0.f;
             for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
             int len = p.lengths ? p.lengths[b] : p.T;
+            if (p.t == 0 && (len < 0 || len > p.T)) report_status(p.status, WM_ERR_INVALID_ARG);
             if (p.t < len) p.nll_acc[b] += (double)tot;
         }
         return;
@@ -423,6 +426,7 @@ StepParams base_params(const wm_handle *hd, int B, int T, const StepWs &w) {
     p.Wa = hd->step.Wa;
     p.h = w.h; p.c = w.c; p.frozen = w.frozen;
     p.heads = w.heads; p.ldh = hd->M + 2;
+    p.status = hd->status;
     return p;
 }
 

@@ -449,6 +449,7 @@ struct EpiGates {
         int a = p.act[bb];
         if (p.teacher) {
             a = p.act_in[(size_t)p.t * p.B + bb];
+            if (a >= p.A && b < p.B && n == 0 && x.cg == 0) report_status(x.status, WM_ERR_INVALID_ARG);
             if (a < 0 || a >= p.A) a = -1;
         }
         pr.a = (a >= 0 && !pr.fz) ? a : -1;
@@ -766,6 +767,8 @@ struct EpiHeads {
         }
         if (p.teacher && valid) {
             const int len = p.lengths ? p.lengths[b] : p.T;
+            if (p.t == 0 && n == 0 && x.cg == 0 && (len < 0 || len > p.T))
+                report_status(x.status, WM_ERR_INVALID_ARG);
             if (p.t < len) p.nll_part[((size_t)n * 4 + x.cg) * p.B + b] += nll;
         }
         if (n == p.rd_tile) {

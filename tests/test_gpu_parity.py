@@ -236,6 +236,34 @@ def test_invalid_arguments(wm):
         m.mdn_nll(torch.from_numpy(zs), torch.from_numpy(acts))  # host actions are checked
 
 
+@pytest.mark.parametrize("path", ["stepwise", "fused", "tensor"])
+def test_device_teacher_inputs_out_of_range_are_reported(wm, orc, path):
+    """On device arrays an action >= A or a length outside [0, T] is found by the kernels:
+    wm_sync reports WM_ERR_INVALID_ARG once, the action counts as no action, the length is
+    clamped, and the next call runs clean."""
+    cfg = synth.model_config("small_bf16")
+    w = synth.weights(cfg, seed=12)
+    N, T = 40, 5
+    zs, acts, _ = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=12)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    for bad_action in (True, False):
+        a2, lens = acts.copy(), np.full(N, T, np.int32)
+        if bad_action:
+            a2[1, 3] = cfg["a_dim"] + 7
+        else:
+            lens[5] = T + 2
+        g = m.mdn_nll(_cuda(zs), _cuda(a2), lengths=_cuda(lens))
+        with pytest.raises(wm.WMError) as ei:
+            m.sync()
+        assert ei.value.status == wm.WM_ERR_INVALID_ARG
+        assert m.last_path == path
+        fixed_a = np.where(a2 >= cfg["a_dim"], -1, a2)
+        o = orc.mdn_nll(cfg, w, zs, fixed_a, lengths=np.clip(lens, 0, T))
+        check_teacher({"nll": g["nll"]}, o, "bf16")
+        m.mdn_nll(_cuda(zs), _cuda(acts))
+        m.sync()  # the status was cleared
+
+
 # ------------------------------------------------------------------ invariants of the GPU path
 @pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
 def test_sharding_is_bit_exact(wm, name):
