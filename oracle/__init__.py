@@ -46,14 +46,22 @@ class _Cfg(C.Structure):
                 ("bf16", C.c_int), ("mdn_tau", C.c_double), ("sigma_sqrt_tau", C.c_int),
                 ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_double),
                 ("done_terminates", C.c_int), ("noop_terminates", C.c_int),
-                ("seed", C.c_uint64), ("nthreads", C.c_int)]
+                ("seed", C.c_uint64), ("nthreads", C.c_int), ("reward_mode", C.c_int),
+                ("reward_alpha", C.c_double), ("reward_beta", C.c_double),
+                ("invalid_reward", C.c_double)]
 
 
 class _W(C.Structure):
     _fields_ = [("W_lstm", C.c_void_p), ("b_lstm", C.c_void_p), ("W_mdn", C.c_void_p),
                 ("b_mdn", C.c_void_p), ("w_rew", C.c_void_p), ("b_rew", C.c_float),
                 ("w_done", C.c_void_p), ("b_done", C.c_float), ("W_ctrl", C.c_void_p),
-                ("b_ctrl", C.c_void_p)]
+                ("b_ctrl", C.c_void_p), ("w_rt", C.c_void_p), ("b_rt", C.c_float),
+                ("w_mem", C.c_void_p), ("b_mem", C.c_float)]
+
+
+class _Ext(C.Structure):
+    _fields_ = [("rt0", C.c_void_p), ("mem0", C.c_void_p), ("rt_seq", C.c_void_p),
+                ("mem_seq", C.c_void_p)]
 
 
 def _load():
@@ -77,9 +85,9 @@ def _load():
             lib.orc_sample_dim.restype = C.c_int
             lib.orc_select_action.argtypes = [C.c_int, P, P, C.c_int, C.c_double, C.c_double, P]
             lib.orc_select_action.restype = C.c_int
-            lib.orc_rollout.argtypes = [P, P, C.c_int, C.c_int, C.c_uint64, C.c_uint32] + [P] * 18
+            lib.orc_rollout.argtypes = [P, P, C.c_int, C.c_int, C.c_uint64, C.c_uint32] + [P] * 19
             lib.orc_rollout.restype = C.c_int
-            lib.orc_step.argtypes = [P, P, C.c_int, P, C.c_uint32] + [P] * 19
+            lib.orc_step.argtypes = [P, P, C.c_int, P, C.c_uint32] + [P] * 20
             lib.orc_step.restype = C.c_int
             lib.orc_mdn_nll.argtypes = [P, P, C.c_int, C.c_int] + [P] * 7
             lib.orc_mdn_nll.restype = C.c_int
@@ -101,7 +109,9 @@ def _cfg(cfg: dict, nthreads: int) -> _Cfg:
                 float(cfg.get("mdn_tau", 1.0)), int(cfg.get("sigma_sqrt_tau", 0)),
                 int(cfg.get("ctrl_sample", 0)), float(cfg.get("ctrl_tau", 1.0)),
                 int(cfg.get("done_terminates", 0)), int(cfg.get("noop_terminates", 0)),
-                int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(nthreads))
+                int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(nthreads),
+                int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
+                float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)))
 
 
 class _Weights:
@@ -109,11 +119,32 @@ class _Weights:
 
     def __init__(self, w: dict):
         self.arrs = {k: _f32(w[k]) for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew",
-                                               "w_done", "W_ctrl", "b_ctrl")}
+                                               "w_done", "W_ctrl", "b_ctrl", "w_rt", "w_mem")
+                     if w.get(k) is not None}
         a = self.arrs
         self.s = _W(_ptr(a["W_lstm"]), _ptr(a["b_lstm"]), _ptr(a["W_mdn"]), _ptr(a["b_mdn"]),
                     _ptr(a["w_rew"]), float(w["b_rew"]), _ptr(a["w_done"]), float(w["b_done"]),
-                    _ptr(a["W_ctrl"]), _ptr(a["b_ctrl"]))
+                    _ptr(a["W_ctrl"]), _ptr(a["b_ctrl"]), _ptr(a.get("w_rt")),
+                    float(w.get("b_rt", 0.0)), _ptr(a.get("w_mem")), float(w.get("b_mem", 0.0)))
+
+
+class _ExtArgs:
+    """The optional parts of a call (shaped-reward state); keeps the arrays alive."""
+
+    def __init__(self, cfg: dict, B: int, T: int, rt0=None, mem0=None):
+        self.out = {}
+        self.keep = []
+        self.s = None
+        if int(cfg.get("reward_mode", 0)) == 1:
+            if rt0 is None or mem0 is None:
+                raise ValueError("the shaped reward needs rt0 and mem0")
+            r, m = _f32(rt0).reshape(B), _f32(mem0).reshape(B)
+            self.out = {"rt_seq": np.zeros((T, B), np.float32), "mem_seq": np.zeros((T, B), np.float32)}
+            self.keep = [r, m]
+            self.s = _Ext(_ptr(r), _ptr(m), _ptr(self.out["rt_seq"]), _ptr(self.out["mem_seq"]))
+
+    def ref(self):
+        return None if self.s is None else C.byref(self.s)
 
 
 # ---------------------------------------------------------------- building blocks
@@ -195,8 +226,10 @@ def select_action(logits, mask_words=None, ctrl_sample: int = 0, ctrl_tau: float
 # ---------------------------------------------------------------- the path
 def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset: int = 0,
             t0: int = 0, h0=None, c0=None, done0=None, want_seq: bool = False,
-            nthreads: int = 1) -> dict:
-    """Free-running dream rollout of B = len(z0) episodes for T steps (a1..a8)."""
+            nthreads: int = 1, rt0=None, mem0=None) -> dict:
+    """Free-running dream rollout of B = len(z0) episodes for T steps (a1..a8).
+    With the shaped reward (reward_mode 1), rt0 / mem0 [B] are the predictions of the
+    current graphs and the result carries rt_seq / mem_seq [T, B]."""
     lib = _load()
     Z, A, H, K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
     z0 = _f32(z0).reshape(-1, Z)
@@ -219,24 +252,28 @@ def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset:
                    comp_seq=np.zeros((T, B, Z), np.uint8))
     w = _Weights(weights)
     cs = _cfg(cfg, nthreads)
+    ext = _ExtArgs(cfg, B, T, rt0, mem0)
+    out.update(ext.out)
     rc = lib.orc_rollout(C.byref(cs), C.byref(w.s), B, T, int(episode_offset), int(t0),
                          _ptr(z0), _ptr(h0), _ptr(c0), _ptr(d0), _ptr(mk),
                          _ptr(out["z"]), _ptr(out["actions"]), _ptr(out["rewards"]),
                          _ptr(out["done"]), _ptr(out["h_final"]), _ptr(out["c_final"]),
                          _ptr(out.get("h_seq")), _ptr(out.get("c_seq")), _ptr(out.get("mdn_seq")),
                          _ptr(out.get("comp_seq")), _ptr(out["ctrl_margin"]),
-                         _ptr(out["comp_margin"]), _ptr(out["done_margin"]))
+                         _ptr(out["comp_margin"]), _ptr(out["done_margin"]), ext.ref())
     if rc != 0:
         raise ValueError(f"orc_rollout failed ({rc})")
     return out
 
 
 def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=None, mask=None,
-         a_use=None, h_use=None, k_use=None, nthreads: int = 1) -> dict:
+         a_use=None, h_use=None, k_use=None, nthreads: int = 1, rt=None, mem=None) -> dict:
     """One dream step (a1..a8) of B = len(episodes) episodes started from the state
     (z [B,Z], h [B,H], c [B,H], frozen [B]); episodes are global Philox indices.
     a_use / h_use / k_use replace what flows downstream of the action, h' and
-    component decisions (the returned decisions and margins are the oracle's own)."""
+    component decisions (the returned decisions and margins are the oracle's own).
+    With the shaped reward, rt / mem [B] are the predictions entering the step and the
+    result carries the step's as "rt" / "mem"."""
     lib = _load()
     Z, A, H, K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
     ep = np.ascontiguousarray(episodes, dtype=np.uint64).reshape(-1)
@@ -256,14 +293,17 @@ def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=No
            "z_next": np.zeros((B, Z), np.float32)}
     w = _Weights(weights)
     cs = _cfg(cfg, nthreads)
+    ext = _ExtArgs(cfg, B, 1, rt, mem)
     rc = lib.orc_step(C.byref(cs), C.byref(w.s), B, _ptr(ep), int(step_index) & 0xFFFFFFFF,
                       _ptr(z), _ptr(h), _ptr(c), _ptr(fz), _ptr(mk), _ptr(au), _ptr(hu), _ptr(ku),
                       _ptr(out["action"]), _ptr(out["ctrl_margin"]), _ptr(out["h"]), _ptr(out["c"]),
                       _ptr(out["mdn"]), _ptr(out["reward"]), _ptr(out["done"]),
                       _ptr(out["done_margin"]), _ptr(out["comp"]), _ptr(out["comp_margin"]),
-                      _ptr(out["z_next"]))
+                      _ptr(out["z_next"]), ext.ref())
     if rc != 0:
         raise ValueError(f"orc_step failed ({rc})")
+    if ext.out:
+        out["rt"], out["mem"] = ext.out["rt_seq"][0], ext.out["mem_seq"][0]
     return out
 
 

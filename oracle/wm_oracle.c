@@ -257,8 +257,8 @@ int orc_select_action(int A, const float *logits, const uint32_t *mask_words,
 /* Weights widened to fp64 (rounded to bf16 first in bf16 mode).             */
 /* ------------------------------------------------------------------------- */
 typedef struct {
-    double *W_lstm, *b_lstm, *W_mdn, *b_mdn, *w_rew, *w_done, *W_ctrl, *b_ctrl;
-    double b_rew, b_done;
+    double *W_lstm, *b_lstm, *W_mdn, *b_mdn, *w_rew, *w_done, *W_ctrl, *b_ctrl, *w_rt, *w_mem;
+    double b_rew, b_done, b_rt, b_mem;
 } wts64;
 
 static double *widen(const float *src, size_t n, int round_bf16)
@@ -273,6 +273,7 @@ static void free_wts(wts64 *v)
 {
     free(v->W_lstm); free(v->b_lstm); free(v->W_mdn); free(v->b_mdn);
     free(v->w_rew); free(v->w_done); free(v->W_ctrl); free(v->b_ctrl);
+    free(v->w_rt); free(v->w_mem);
 }
 
 static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need_ctrl)
@@ -292,8 +293,19 @@ static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need
         v->W_ctrl = widen(w->W_ctrl, (size_t)(Z + H) * A, rb);
         v->b_ctrl = widen(w->b_ctrl, (size_t)A, 0);
     }
+    const int shaped = cfg->reward_mode == 1;
+    if (shaped) {
+        if (!w->w_rt || !w->w_mem) {
+            free_wts(v);
+            return -1;
+        }
+        v->w_rt = widen(w->w_rt, (size_t)H, rb);
+        v->w_mem = widen(w->w_mem, (size_t)H, rb);
+        v->b_rt = (double)w->b_rt;
+        v->b_mem = (double)w->b_mem;
+    }
     if (!v->W_lstm || !v->b_lstm || !v->W_mdn || !v->b_mdn || !v->w_rew || !v->w_done ||
-        (need_ctrl && (!v->W_ctrl || !v->b_ctrl))) {
+        (need_ctrl && (!v->W_ctrl || !v->b_ctrl)) || (shaped && (!v->w_rt || !v->w_mem))) {
         free_wts(v);
         return -1;
     }
@@ -311,6 +323,7 @@ static int check_cfg(const orc_cfg *c)
 {
     if (c->z_dim <= 0 || c->a_dim <= 0 || c->h_dim <= 0 || c->k_mix <= 0 || c->k_mix > 64) return -1;
     if (!(c->mdn_tau >= 0.0) || !(c->ctrl_tau >= 0.0)) return -1;
+    if (c->reward_mode != 0 && c->reward_mode != 1) return -1;
     return 0;
 }
 
@@ -382,12 +395,16 @@ static void buf_free(step_buf *sb)
  *   a_use (>= -1, or -2 for none) is the action row the LSTM takes (a3);
  *   h_use (or NULL) is the h' the heads read (a5..a7);
  *   k_use (or NULL) gives the component each dim's z_{t+1} is drawn from (a7).
- * The done flag is formed from the action actually taken.  Returns 1 if the
+ * The done flag is formed from the action actually taken.  With the shaped
+ * reward (reward_mode 1) rt, mem hold the predicted runtime and memory
+ * accesses entering the step (fp32 values) and leave with the step's; the
+ * reward is Eq. 2 of Sec. 3.1.4 on them when the action taken is valid (a
+ * row was taken, a >= 0), the invalid reward otherwise.  Returns 1 if the
  * episode freezes after this step (a8).
  */
 static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64_t e,
-                        uint32_t s, double *z, double *h, double *c, const uint32_t *mw,
-                        int a_use, const float *h_use, const uint8_t *k_use,
+                        uint32_t s, double *z, double *h, double *c, double *rt, double *mem,
+                        const uint32_t *mw, int a_use, const float *h_use, const uint8_t *k_use,
                         int32_t *action, float *ctrl_margin, float *reward, uint8_t *done,
                         float *done_margin, float *mdn_out, uint8_t *comp, float *comp_margin)
 {
@@ -425,6 +442,16 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
     if (mdn_out) for (int m = 0; m < 3 * K * Z; ++m) mdn_out[m] = (float)mdn[m];
     double r = v->b_rew, dl = v->b_done;
     for (int i = 0; i < H; ++i) { r += y[i] * v->w_rew[i]; dl += y[i] * v->w_done[i]; }
+    if (cfg->reward_mode == 1) {
+        double rt_new = v->b_rt, mem_new = v->b_mem;
+        for (int i = 0; i < H; ++i) { rt_new += y[i] * v->w_rt[i]; mem_new += y[i] * v->w_mem[i]; }
+        rt_new = (double)(float)rt_new;   /* predictions are carried in fp32 */
+        mem_new = (double)(float)mem_new;
+        r = a >= 0 ? cfg->reward_alpha * (*rt - rt_new) + cfg->reward_beta * (*mem - mem_new)
+                   : cfg->invalid_reward;
+        *rt = rt_new;
+        *mem = mem_new;
+    }
     *reward = (float)r;
     float dlf = (float)dl;
     if (done_margin) *done_margin = fabsf(dlf);
@@ -469,11 +496,14 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
                            float *z_out, int32_t *actions, float *rewards, uint8_t *done,
                            float *h_final, float *c_final,
                            float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
-                           float *ctrl_margin, float *comp_margin, float *done_margin)
+                           float *ctrl_margin, float *comp_margin, float *done_margin,
+                           const orc_ext *ext)
 {
     const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
     const int M = 3 * K * Z, W = (A + 31) / 32;
     const uint64_t e = episode_offset + (uint64_t)b;
+    const int shaped = cfg->reward_mode == 1;
+    double rt = shaped ? (double)ext->rt0[b] : 0.0, mem = shaped ? (double)ext->mem0[b] : 0.0;
     double *z = malloc(sizeof(double) * Z), *h = malloc(sizeof(double) * H);
     double *c = malloc(sizeof(double) * H);
     step_buf sb;
@@ -501,8 +531,8 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
             if (done_margin) done_margin[tb] = INF_F;
             if (comp_margin) for (int d = 0; d < Z; ++d) comp_margin[tb * Z + d] = INF_F;
         } else {
-            frozen = step_episode(cfg, v, &sb, e, s, z, h, c, mask ? mask + tb * W : NULL,
-                                  -2, NULL, NULL, &actions[tb],
+            frozen = step_episode(cfg, v, &sb, e, s, z, h, c, &rt, &mem,
+                                  mask ? mask + tb * W : NULL, -2, NULL, NULL, &actions[tb],
                                   ctrl_margin ? &ctrl_margin[tb] : NULL, &rewards[tb], &done[tb],
                                   done_margin ? &done_margin[tb] : NULL,
                                   mdn_seq ? mdn_seq + tb * M : NULL,
@@ -512,6 +542,8 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
         for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
         if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
         if (c_seq) for (int i = 0; i < H; ++i) c_seq[tb * H + i] = (float)c[i];
+        if (shaped && ext->rt_seq) ext->rt_seq[tb] = (float)rt;
+        if (shaped && ext->mem_seq) ext->mem_seq[tb] = (float)mem;
     }
     if (h_final) for (int i = 0; i < H; ++i) h_final[(size_t)b * H + i] = (float)h[i];
     if (c_final) for (int i = 0; i < H; ++i) c_final[(size_t)b * H + i] = (float)c[i];
@@ -526,10 +558,12 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
                 float *z_out, int32_t *actions, float *rewards, uint8_t *done,
                 float *h_final, float *c_final,
                 float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
-                float *ctrl_margin, float *comp_margin, float *done_margin)
+                float *ctrl_margin, float *comp_margin, float *done_margin,
+                const orc_ext *ext)
 {
     if (check_cfg(cfg) || B < 0 || T < 0 || !z0 || !z_out || !actions || !rewards || !done)
         return -1;
+    if (cfg->reward_mode == 1 && (!ext || !ext->rt0 || !ext->mem0)) return -1;
     wts64 v;
     if (load_wts(cfg, w, &v, 1)) return -2;
     int bad = 0;
@@ -539,7 +573,7 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
         bad |= rollout_episode(cfg, &v, b, B, T, episode_offset, t0, z0, h0, c0, done0, mask,
                                z_out, actions, rewards, done, h_final, c_final,
                                h_seq, c_seq, mdn_seq, comp_seq,
-                               ctrl_margin, comp_margin, done_margin) ? 1 : 0;
+                               ctrl_margin, comp_margin, done_margin, ext) ? 1 : 0;
     }
     free_wts(&v);
     return bad ? -2 : 0;
@@ -560,12 +594,14 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
              const int32_t *a_use, const float *h_use, const uint8_t *k_use,
              int32_t *action, float *ctrl_margin, float *h_out, float *c_out, float *mdn_out,
              float *reward, uint8_t *done, float *done_margin, uint8_t *comp,
-             float *comp_margin, float *z_next)
+             float *comp_margin, float *z_next, const orc_ext *ext)
 {
     if (check_cfg(cfg) || B < 0 || !episode || !z || !h || !c || !action || !ctrl_margin ||
         !h_out || !c_out || !mdn_out || !reward || !done || !done_margin || !comp ||
         !comp_margin || !z_next)
         return -1;
+    const int shaped = cfg->reward_mode == 1;
+    if (shaped && (!ext || !ext->rt0 || !ext->mem0)) return -1;
     const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
     const int M = 3 * K * Z, W = (A + 31) / 32;
     wts64 v;
@@ -584,6 +620,7 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
         }
         for (int i = 0; i < Z; ++i) zs[i] = z[(size_t)b * Z + i];
         for (int i = 0; i < H; ++i) { hs[i] = h[(size_t)b * H + i]; cs[i] = c[(size_t)b * H + i]; }
+        double rt = shaped ? (double)ext->rt0[b] : 0.0, mem = shaped ? (double)ext->mem0[b] : 0.0;
         if (frozen && frozen[b]) {
             action[b] = -1; ctrl_margin[b] = INF_F; reward[b] = 0.0f; done[b] = 1;
             done_margin[b] = INF_F;
@@ -593,7 +630,7 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
                 comp_margin[(size_t)b * Z + d] = INF_F;
             }
         } else {
-            step_episode(cfg, &v, &sb, episode[b], step, zs, hs, cs,
+            step_episode(cfg, &v, &sb, episode[b], step, zs, hs, cs, &rt, &mem,
                          mask ? mask + (size_t)b * W : NULL,
                          a_use ? a_use[b] : -2, h_use ? h_use + (size_t)b * H : NULL,
                          k_use ? k_use + (size_t)b * Z : NULL,
@@ -606,6 +643,8 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
             h_out[(size_t)b * H + i] = (float)hs[i];
             c_out[(size_t)b * H + i] = (float)cs[i];
         }
+        if (shaped && ext->rt_seq) ext->rt_seq[b] = (float)rt;
+        if (shaped && ext->mem_seq) ext->mem_seq[b] = (float)mem;
         free(zs); free(hs); free(cs); buf_free(&sb);
     }
     free_wts(&v);

@@ -39,6 +39,12 @@ typedef struct {
     int noop_terminates;  /* action a_dim-1 (NO-OP) freezes the episode      */
     uint64_t seed;        /* Philox key                                      */
     int nthreads;         /* OpenMP threads over episodes (<=0: 1)           */
+    /* reward (Sec. 3.1.4): 0 = the linear reward head; 1 = Eq. 2 on the
+     * predicted runtime and memory-access heads, alpha (RT_{t-1} - RT_t) +
+     * beta (M_{t-1} - M_t) for a valid action, invalid_reward otherwise
+     * (Eq. 1 is alpha = 1, beta = 0)                                       */
+    int reward_mode;
+    double reward_alpha, reward_beta, invalid_reward;
 } orc_cfg;
 
 typedef struct {
@@ -52,7 +58,20 @@ typedef struct {
     float b_done;
     const float *W_ctrl;  /* [Z+H, A]                                        */
     const float *b_ctrl;  /* [A]                                             */
+    const float *w_rt;    /* [H] runtime head (reward_mode 1), else NULL     */
+    float b_rt;
+    const float *w_mem;   /* [H] memory-access head (reward_mode 1)          */
+    float b_mem;
 } orc_weights;
+
+/* Inputs and outputs of the optional parts of a rollout (NULL = not used).
+ * Shaped reward (reward_mode 1): rt0, mem0 [B] are the predicted runtime and
+ * memory accesses of each episode's current graph (required); rt_seq,
+ * mem_seq [T,B] receive the predictions after each step. */
+typedef struct {
+    const float *rt0, *mem0;
+    float *rt_seq, *mem_seq;
+} orc_ext;
 
 /* ---- building blocks (exported so tests can pin each one) ---------------- */
 void     orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
@@ -79,7 +98,8 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
                 float *z_out, int32_t *actions, float *rewards, uint8_t *done,
                 float *h_final, float *c_final,
                 float *h_seq, float *c_seq, float *mdn_seq, uint8_t *comp_seq,
-                float *ctrl_margin, float *comp_margin, float *done_margin);
+                float *ctrl_margin, float *comp_margin, float *done_margin,
+                const orc_ext *ext);
 
 /* One dream step for B episodes started from a given state (z, h, c, frozen):
  * the step orc_rollout takes, for step-anchored comparisons.  episode[b] is the
@@ -89,14 +109,17 @@ int orc_rollout(const orc_cfg *cfg, const orc_weights *w, int B, int T,
  * read, k_use [B,Z] the components z_{t+1} is drawn from.  The outputs are the
  * oracle's own decisions and margins and the values downstream of the
  * overrides: action, ctrl_margin, reward, done, done_margin [B]; h_out, c_out
- * [B,H]; mdn_out [B,3KZ]; comp, comp_margin, z_next [B,Z]. */
+ * [B,H]; mdn_out [B,3KZ]; comp, comp_margin, z_next [B,Z].  ext (or NULL)
+ * carries the optional parts for this one step, with T = 1: ext->rt0/mem0
+ * are the predictions entering the step, ext->rt_seq/mem_seq [B] receive the
+ * step's. */
 int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *episode,
              uint32_t step, const float *z, const float *h, const float *c,
              const uint8_t *frozen, const uint32_t *mask,
              const int32_t *a_use, const float *h_use, const uint8_t *k_use,
              int32_t *action, float *ctrl_margin, float *h_out, float *c_out, float *mdn_out,
              float *reward, uint8_t *done, float *done_margin, uint8_t *comp,
-             float *comp_margin, float *z_next);
+             float *comp_margin, float *z_next, const orc_ext *ext);
 
 int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
                 const float *z_seq, const int32_t *actions, const int32_t *lengths,

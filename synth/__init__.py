@@ -14,7 +14,9 @@ available, so these stand in for them.  Recipe (per workload below):
   ``mask_density``, independently; packed little-endian into uint32 words
   ([T, B, ceil(A/32)], bit j of word w = action 32*w + j);
 * teacher-forced sequences: z ~ N(0, 1) for all T+1 frames, actions uniform
-  on [0, A).
+  on [0, A);
+* shaped-reward state: the predicted runtime and memory accesses of each
+  episode's current graph ~ N(0, 0.5^2).
 
 Sharding: a run over S shards of B episodes (one shard per GPU) draws shard
 r's z_0 and masks from streams of their own; shard 0's are exactly the
@@ -47,8 +49,9 @@ WORKLOADS = {
 }
 
 _STREAM = {"W_lstm": 1, "b_lstm": 2, "W_mdn": 3, "b_mdn": 4, "w_rew": 5, "b_rew": 6,
-           "w_done": 7, "b_done": 8, "W_ctrl": 9, "b_ctrl": 10,
-           "z0": 20, "mask": 21, "zseq": 22, "actions": 23, "lengths": 24}
+           "w_done": 7, "b_done": 8, "W_ctrl": 9, "b_ctrl": 10, "w_rt": 11, "b_rt": 12,
+           "w_mem": 13, "b_mem": 14,
+           "z0": 20, "mask": 21, "zseq": 22, "actions": 23, "lengths": 24, "rt0": 25, "mem0": 26}
 
 
 def _rng(seed: int, stream: int, sub: int = 0) -> np.random.Generator:
@@ -70,7 +73,9 @@ def model_config(name: str, **over) -> dict:
                precision=w.get("precision", "fp32"), mdn_tau=w.get("mdn_tau", 1.0),
                sigma_sqrt_tau=w.get("sigma_sqrt_tau", 0), ctrl_sample=w.get("ctrl_sample", 0),
                ctrl_tau=w.get("ctrl_tau", 1.0), done_terminates=w.get("done_terminates", 0),
-               noop_terminates=w.get("noop_terminates", 0), seed=w.get("seed", 0))
+               noop_terminates=w.get("noop_terminates", 0), seed=w.get("seed", 0),
+               reward_mode=w.get("reward_mode", 0), reward_alpha=w.get("reward_alpha", 0.8),
+               reward_beta=w.get("reward_beta", 0.2), invalid_reward=w.get("invalid_reward", -100.0))
     return cfg
 
 
@@ -79,12 +84,22 @@ def weights(cfg: dict, seed: int = 0, std: float = 0.05) -> dict:
     Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
     shapes = {"W_lstm": (Z + A + H, 4 * H), "b_lstm": (4 * H,), "W_mdn": (H, 3 * K * Z),
               "b_mdn": (3 * K * Z,), "w_rew": (H,), "b_rew": (), "w_done": (H,), "b_done": (),
-              "W_ctrl": (Z + H, A), "b_ctrl": (A,)}
+              "W_ctrl": (Z + H, A), "b_ctrl": (A,), "w_rt": (H,), "b_rt": (), "w_mem": (H,),
+              "b_mem": ()}
     out = {}
     for name, shp in shapes.items():
         v = _rng(seed, _STREAM[name]).standard_normal(shp, dtype=np.float32) * np.float32(std)
         out[name] = float(v) if shp == () else np.ascontiguousarray(v, dtype=np.float32)
     return out
+
+
+def shaping_state(B: int, seed: int = 0, shard: int = 0):
+    """(rt0, mem0) [B]: the predicted runtime and memory accesses of each episode's
+    current graph, for the shaped reward; ~ N(0, 0.5^2), the scale of the random-init
+    heads' outputs."""
+    rt = _shard_rng(seed, _STREAM["rt0"], 0, shard).standard_normal(B, dtype=np.float32) * np.float32(0.5)
+    mem = _shard_rng(seed, _STREAM["mem0"], 0, shard).standard_normal(B, dtype=np.float32) * np.float32(0.5)
+    return rt, mem
 
 
 def z0(B: int, Z: int, seed: int = 0, shard: int = 0) -> np.ndarray:
