@@ -99,7 +99,19 @@ typedef struct {
     int path;                         /* WM_PATH_*                                 */
     int fused_cluster;                /* fused family: CTAs per cluster, 8 or 16;
                                          0 = choose per call (fewest waves)        */
+    /* Reward (Sec. 3.1.4).  WM_REWARD_HEAD: r_t = w_rew . h' + b_rew.
+     * WM_REWARD_SHAPED: two more linear heads on h' predict the graph's runtime
+     * RT and memory accesses M, and r_t = alpha (RT_{t-1} - RT_t) +
+     * beta (M_{t-1} - M_t) (Eq. 2; Eq. 1 is alpha = 1, beta = 0) when an action
+     * was taken, invalid_reward when none was (a = -1).  Sec. 4.3 found
+     * alpha = 0.8, beta = 0.2 best; Eq. 1 / 2 give -100 for an invalid action.
+     * The stepwise and tensor-core families take it; the fused family does not. */
+    int reward_mode;                  /* WM_REWARD_HEAD or WM_REWARD_SHAPED         */
+    float reward_alpha, reward_beta;
+    float invalid_reward;
 } wm_config;
+
+enum { WM_REWARD_HEAD = 0, WM_REWARD_SHAPED = 1 };
 
 /* Canonical fp32 weights, row-major, HOST memory; copied (and packed) by
  * wm_create, so the caller may free them afterwards. */
@@ -114,6 +126,10 @@ typedef struct {
     float b_done;
     const float *W_ctrl;  /* [Z+H, A]: rows z | h                                 */
     const float *b_ctrl;  /* [A]                                                  */
+    const float *w_rt;    /* [H] predicted-runtime head (WM_REWARD_SHAPED only)   */
+    float b_rt;
+    const float *w_mem;   /* [H] predicted memory-access head (WM_REWARD_SHAPED)  */
+    float b_mem;
 } wm_weights;
 
 typedef struct wm_handle wm_handle;
@@ -136,6 +152,11 @@ typedef struct {
     float *c_seq;                /* [T,B,H] optional                                 */
     float *mdn_seq;              /* [T,B,M] optional: raw head outputs (0 if frozen) */
     uint8_t *comp_seq;           /* [T,B,Z] optional: chosen component (255 if frozen)*/
+    /* WM_REWARD_SHAPED only (ignored otherwise): */
+    const float *rt0, *mem0;     /* [B]     required: RT and M of each episode's graph
+                                    entering the call (resume: the last rt_seq / mem_seq) */
+    float *rt_seq, *mem_seq;     /* [T,B]   optional: RT_t, M_t after each step (frozen:
+                                    repeated)                                          */
 } wm_rollout_io;
 
 /* Creates a world model on the current CUDA device from the weights of the
@@ -144,7 +165,8 @@ typedef struct {
  * a_t = W_c [z_t, h_t] + b_c (Sec. 3.4).  Copies and packs the weights; the
  * handle owns that device memory until wm_destroy.  Returns
  * WM_ERR_INVALID_ARG for bad sizes (any dim <= 0, K > 32, negative
- * temperatures) or NULL weights. */
+ * temperatures) or NULL weights (w_rt and w_mem are needed with
+ * WM_REWARD_SHAPED only). */
 wm_status wm_create(const wm_config *cfg, const wm_weights *weights, wm_handle **out);
 
 /* Runs T dream steps (a1..a8 above) for B independent episodes, asynchronously

@@ -210,15 +210,16 @@ bool valid_cfg(const wm_config *c) {
            (c->precision == WM_FP32 || c->precision == WM_BF16) && c->mdn_tau >= 0.f &&
            c->ctrl_tau >= 0.f && c->path >= WM_PATH_AUTO && c->path <= WM_PATH_TENSOR &&
            c->z_dim <= 4096 && c->a_dim <= 65536 && c->h_dim <= 16384 &&
-           (c->fused_cluster == 0 || c->fused_cluster == 8 || c->fused_cluster == 16);
+           (c->fused_cluster == 0 || c->fused_cluster == 8 || c->fused_cluster == 16) &&
+           (c->reward_mode == WM_REWARD_HEAD || c->reward_mode == WM_REWARD_SHAPED);
 }
 
 cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
     const wm_config &c = h->cfg;
-    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, N1 = 4 * H + A;
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, N1 = 4 * H + A, NR = h->NR;
     const bool rb = c.precision == WM_BF16;
     auto wv = [&](float x) { return rb ? bf16_round_host(x) : x; };
-    std::vector<float> Wg((Z + H) * N1), Wa(A * 4 * H), bg(N1), Wh(H * (M + 2)), bh(M + 2);
+    std::vector<float> Wg((Z + H) * N1), Wa(A * 4 * H), bg(N1), Wh(H * (M + NR)), bh(M + NR);
     for (size_t r = 0; r < Z + H; ++r) {
         const size_t src = r < Z ? r : r + A;  // skip the action rows
         for (size_t n = 0; n < 4 * H; ++n) Wg[r * N1 + n] = wv(w->W_lstm[src * 4 * H + n]);
@@ -229,13 +230,21 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
     for (size_t n = 0; n < 4 * H; ++n) bg[n] = w->b_lstm[n];
     for (size_t j = 0; j < A; ++j) bg[4 * H + j] = w->b_ctrl[j];
     for (size_t i = 0; i < H; ++i) {
-        for (size_t m = 0; m < M; ++m) Wh[i * (M + 2) + m] = wv(w->W_mdn[i * M + m]);
-        Wh[i * (M + 2) + M] = wv(w->w_rew[i]);
-        Wh[i * (M + 2) + M + 1] = wv(w->w_done[i]);
+        for (size_t m = 0; m < M; ++m) Wh[i * (M + NR) + m] = wv(w->W_mdn[i * M + m]);
+        Wh[i * (M + NR) + M] = wv(w->w_rew[i]);
+        Wh[i * (M + NR) + M + 1] = wv(w->w_done[i]);
+        if (NR == 4) {
+            Wh[i * (M + NR) + M + 2] = wv(w->w_rt[i]);
+            Wh[i * (M + NR) + M + 3] = wv(w->w_mem[i]);
+        }
     }
     for (size_t m = 0; m < M; ++m) bh[m] = w->b_mdn[m];
     bh[M] = w->b_rew;
     bh[M + 1] = w->b_done;
+    if (NR == 4) {
+        bh[M + 2] = w->b_rt;
+        bh[M + 3] = w->b_mem;
+    }
     cudaError_t e;
     if ((e = upload(&h->step.Wg, Wg)) != cudaSuccess) return e;
     if ((e = upload(&h->step.Wa, Wa)) != cudaSuccess) return e;
@@ -266,10 +275,12 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) 
     if (!w || !w->W_lstm || !w->b_lstm || !w->W_mdn || !w->b_mdn || !w->w_rew || !w->w_done ||
         !w->W_ctrl || !w->b_ctrl)
         return WM_ERR_INVALID_ARG;
+    if (cfg->reward_mode == WM_REWARD_SHAPED && (!w->w_rt || !w->w_mem)) return WM_ERR_INVALID_ARG;
     wm_handle *h = new (std::nothrow) wm_handle();
     if (!h) return WM_ERR_OOM;
     h->cfg = *cfg;
     h->M = 3 * cfg->k_mix * cfg->z_dim;
+    h->NR = cfg->reward_mode == WM_REWARD_SHAPED ? 4 : 2;
     memset(&h->step, 0, sizeof(h->step));
     memset(&h->fused, 0, sizeof(h->fused));
     memset(&h->tc, 0, sizeof(h->tc));
@@ -427,6 +438,9 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     if ((unsigned long long)t0 + (unsigned long long)T > 0x100000000ull)
         return fail(h, WM_ERR_INVALID_ARG, "t0 + T overflows the 32-bit Philox step counter");
     const wm_config &c = h->cfg;
+    const bool shaped = c.reward_mode == WM_REWARD_SHAPED;
+    if (shaped && B > 0 && (!io->rt0 || !io->mem0))
+        return fail(h, WM_ERR_INVALID_ARG, "the shaped reward needs rt0 and mem0");
     const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, W = (A + 31) / 32;
     const size_t b = (size_t)B, t = (size_t)T;
     cudaStream_t s = (cudaStream_t)cuda_stream;
@@ -451,6 +465,12 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     st.add((void **)&a.c_seq, io->c_seq, t * b * H * 4, true, STEP_OUT, b * H * 4);
     st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true, STEP_OUT, b * M * 4);
     st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true, STEP_OUT, b * Z);
+    if (shaped) {
+        st.add((void **)&a.rt0, io->rt0, b * 4, false);
+        st.add((void **)&a.mem0, io->mem0, b * 4, false);
+        st.add((void **)&a.rt_seq, io->rt_seq, t * b * 4, true, STEP_OUT, b * 4);
+        st.add((void **)&a.mem_seq, io->mem_seq, t * b * 4, true, STEP_OUT, b * 4);
+    }
 
     int path = pick_path(h, B);
     if (path == WM_PATH_FUSED && !wm_fused_supported(h, B))

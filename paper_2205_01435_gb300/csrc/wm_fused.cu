@@ -818,6 +818,7 @@ int wm_fused_supported(const wm_handle *h, int B) {
     const wm_config &c = h->cfg;
     if (!h->fused.ok) return 0;
     if (c.ctrl_sample && c.ctrl_tau > 0.f) return 0;  // masked argmax only
+    if (c.reward_mode != WM_REWARD_HEAD) return 0;    // the linear reward head only
     return 1;
 }
 

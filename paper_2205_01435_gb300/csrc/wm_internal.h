@@ -35,6 +35,8 @@ struct wm_rollout_dev {
     uint8_t *done;
     float *h_final, *c_final, *h_seq, *c_seq, *mdn_seq;
     uint8_t *comp_seq;
+    const float *rt0, *mem0;   // shaped reward: predictions entering the call
+    float *rt_seq, *mem_seq;   // shaped reward: predictions after each step (optional)
 };
 
 // Device pointers of one teacher-forced scoring call.
@@ -51,8 +53,8 @@ struct wm_step_weights {
     float *Wg;   // [Z+H, 4H+A]  rows z | h; cols gates i|f|g|o then controller
     float *Wa;   // [A, 4H]      action rows of the gate matrix
     float *bg;   // [4H+A]       gate bias then controller bias
-    float *Wh;   // [H, M+2]     mixture head, reward, done
-    float *bh;   // [M+2]
+    float *Wh;   // [H, M+NR]    mixture head, reward, done (+ runtime, memory when shaped)
+    float *bh;   // [M+NR]
 };
 
 // Weights of the fused single-launch family: per cluster size (slot 0: 16 CTAs,
@@ -69,7 +71,7 @@ struct wm_fused_weights {
 struct wm_tc_weights {
     void *wc, *wg, *wa, *wh;  // W_c^T [A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
     float *bc, *bg, *bh;
-    int dims_per_tile, n_head_tiles, rd_tile, rd_col;
+    int dims_per_tile, n_head_tiles, rd_tile, rd_col;  // reward, done (, runtime, memory) columns
     int sms;
     int ok;
 };
@@ -92,6 +94,7 @@ struct wm_handle {
     wm_config cfg;
     int device;
     int M;                       // 3 K Z
+    int NR;                      // head columns after the mixture: reward, done (+ runtime, memory)
     wm_step_weights step;
     wm_fused_weights fused;
     wm_tc_weights tc;

@@ -76,9 +76,14 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
         return fail(h, WM_ERR_INVALID_ARG,
                     "batch too large for wm_rollout_noalloc: its scratch exceeds "
                     "WM_NOALLOC_SCRATCH_BYTES (use a smaller B, or wm_rollout)");
+    const bool shaped = h->cfg.reward_mode == WM_REWARD_SHAPED;
+    if (shaped && B > 0 && (!io->rt0 || !io->mem0))
+        return fail(h, WM_ERR_INVALID_ARG, "the shaped reward needs rt0 and mem0");
     const void *ptrs[] = {io->z0, io->h0, io->c0, io->done0, io->mask, io->z_out, io->actions,
                           io->rewards, io->done, io->h_final, io->c_final, io->h_seq, io->c_seq,
-                          io->mdn_seq, io->comp_seq};
+                          io->mdn_seq, io->comp_seq, shaped ? io->rt0 : nullptr,
+                          shaped ? io->mem0 : nullptr, shaped ? io->rt_seq : nullptr,
+                          shaped ? io->mem_seq : nullptr};
     for (const void *p : ptrs)
         if (!device_accessible(p))
             return fail(h, WM_ERR_INVALID_ARG,
@@ -95,6 +100,9 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
     a.z_out = io->z_out; a.actions = io->actions; a.rewards = io->rewards; a.done = io->done;
     a.h_final = io->h_final; a.c_final = io->c_final; a.h_seq = io->h_seq; a.c_seq = io->c_seq;
     a.mdn_seq = io->mdn_seq; a.comp_seq = io->comp_seq;
+    if (shaped) {
+        a.rt0 = io->rt0; a.mem0 = io->mem0; a.rt_seq = io->rt_seq; a.mem_seq = io->mem_seq;
+    }
     e = wm_step_rollout(h, a, scratch, (cudaStream_t)cuda_stream);
     if (e != cudaSuccess) return fail(h, WM_ERR_CUDA, "wm_rollout_noalloc launch failed");
     h->last_path = WM_PATH_STEPWISE;

@@ -114,6 +114,12 @@ struct StepParams {
     const int32_t *lengths;
     double *nll_acc;
     int *status;          // device status word (out-of-range teacher inputs)
+    // shaped reward (Sec. 3.1.4, Eq. 2): the heads' columns M+2, M+3 predict runtime and
+    // memory accesses; rt / mem carry each episode's last predictions
+    int reward_mode;
+    float alpha, beta, invalid_reward;
+    float *rt, *mem;
+    float *rt_seq, *mem_seq;
 };
 
 __device__ __forceinline__ bool action_valid(const uint32_t *mw, int j) {
@@ -320,23 +326,33 @@ __global__ void __launch_bounds__(128) k_sample(StepParams p) {
     }
     __syncthreads();  // every thread has read frozen[b] before it may change
     if (threadIdx.x == 0) {
+        const bool shaped = p.reward_mode == WM_REWARD_SHAPED;
         if (fz) {
             p.rewards[tb] = 0.f;
             p.done[tb] = 1;
         } else {
-            const float r = row[M], dl = row[M + 1];
+            float r = row[M];
+            const float dl = row[M + 1];
             const int a = p.act_out[tb];
             const bool noop = p.noop_terminates && a == p.A - 1;
+            if (shaped) {  // Eq. 2 on the predictions entering and leaving the step
+                const float rt = row[M + 2], mem = row[M + 3];
+                r = a >= 0 ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
+                p.rt[b] = rt;
+                p.mem[b] = mem;
+            }
             p.rewards[tb] = r;
             p.done[tb] = (dl > 0.f || noop) ? 1 : 0;
             if ((p.done_terminates && dl > 0.f) || noop) p.frozen[b] = 1;
         }
+        if (shaped && p.rt_seq) p.rt_seq[tb] = p.rt[b];
+        if (shaped && p.mem_seq) p.mem_seq[tb] = p.mem[b];
     }
 }
 
 __global__ void k_init_state(int B, int H, int Z, const float *h0, const float *c0, const uint8_t *done0,
                              const float *z0, float *h, float *c, uint8_t *frozen, float *z_out,
-                             double *nll_acc) {
+                             double *nll_acc, const float *rt0, const float *mem0, float *rt, float *mem) {
     const size_t n = (size_t)B * H;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
         h[i] = h0 ? h0[i] : 0.f;
@@ -345,6 +361,10 @@ __global__ void k_init_state(int B, int H, int Z, const float *h0, const float *
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)B; i += (size_t)gridDim.x * blockDim.x) {
         if (frozen) frozen[i] = done0 ? (done0[i] != 0) : 0;
         if (nll_acc) nll_acc[i] = 0.0;
+        if (rt0) {
+            rt[i] = rt0[i];
+            mem[i] = mem0[i];
+        }
     }
     if (z_out)
         for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)B * Z; i += (size_t)gridDim.x * blockDim.x)
@@ -367,17 +387,19 @@ inline size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct StepWs {
     float *G, *heads, *h, *c;
+    float *rt, *mem;  // shaped reward: each episode's last predictions
     uint8_t *frozen;
     double *nll_acc;
 };
 
 size_t step_ws_bytes(const wm_handle *hd, int B, bool teacher) {
     const wm_config &c = hd->cfg;
-    const size_t H = c.h_dim, A = c.a_dim, M = hd->M;
+    const size_t H = c.h_dim, A = c.a_dim, M = hd->M, NR = hd->NR;
     size_t s = 0;
     s += align_up((size_t)B * (4 * H + A) * 4);
-    s += align_up((size_t)B * (M + 2) * 4);
+    s += align_up((size_t)B * (M + NR) * 4);
     s += 2 * align_up((size_t)B * H * 4);
+    if (NR == 4) s += 2 * align_up((size_t)B * 4);
     s += align_up((size_t)B);
     if (teacher) s += align_up((size_t)B * 8);
     return s;
@@ -385,13 +407,17 @@ size_t step_ws_bytes(const wm_handle *hd, int B, bool teacher) {
 
 StepWs carve(const wm_handle *hd, int B, void *ws, bool teacher) {
     const wm_config &c = hd->cfg;
-    const size_t H = c.h_dim, A = c.a_dim, M = hd->M;
+    const size_t H = c.h_dim, A = c.a_dim, M = hd->M, NR = hd->NR;
     char *p = (char *)ws;
     StepWs w{};
     w.G = (float *)p; p += align_up((size_t)B * (4 * H + A) * 4);
-    w.heads = (float *)p; p += align_up((size_t)B * (M + 2) * 4);
+    w.heads = (float *)p; p += align_up((size_t)B * (M + NR) * 4);
     w.h = (float *)p; p += align_up((size_t)B * H * 4);
     w.c = (float *)p; p += align_up((size_t)B * H * 4);
+    if (NR == 4) {
+        w.rt = (float *)p; p += align_up((size_t)B * 4);
+        w.mem = (float *)p; p += align_up((size_t)B * 4);
+    }
     w.frozen = (uint8_t *)p; p += align_up((size_t)B);
     w.nll_acc = teacher ? (double *)p : nullptr;
     return w;
@@ -425,8 +451,11 @@ StepParams base_params(const wm_handle *hd, int B, int T, const StepWs &w) {
     p.G = w.G; p.ldg = 4L * c.h_dim + c.a_dim;
     p.Wa = hd->step.Wa;
     p.h = w.h; p.c = w.c; p.frozen = w.frozen;
-    p.heads = w.heads; p.ldh = hd->M + 2;
+    p.heads = w.heads; p.ldh = hd->M + hd->NR;
     p.status = hd->status;
+    p.reward_mode = c.reward_mode;
+    p.alpha = c.reward_alpha; p.beta = c.reward_beta; p.invalid_reward = c.invalid_reward;
+    p.rt = w.rt; p.mem = w.mem;
     return p;
 }
 
@@ -443,8 +472,11 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
     const bool round = c.precision == WM_BF16;
     {
         wm_ktime kt(hd, WM_KERNEL_AUX, s);
+        const bool shaped = c.reward_mode == WM_REWARD_SHAPED;
         k_init_state<<<grid_1d((size_t)B * H), 256, 0, s>>>(B, H, Z, a.h0, a.c0, a.done0, a.z0, w.h, w.c,
-                                                             w.frozen, a.z_out, nullptr);
+                                                             w.frozen, a.z_out, nullptr,
+                                                             shaped ? a.rt0 : nullptr, shaped ? a.mem0 : nullptr,
+                                                             w.rt, w.mem);
     }
     StepParams p = base_params(hd, B, T, w);
     p.teacher = 0;
@@ -453,6 +485,8 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
     p.act_out = a.actions;
     p.h_seq = a.h_seq; p.c_seq = a.c_seq;
     p.rewards = a.rewards; p.done = a.done; p.mdn_seq = a.mdn_seq; p.comp_seq = a.comp_seq;
+    p.rt_seq = a.rt_seq; p.mem_seq = a.mem_seq;
+    const int NH = hd->M + hd->NR;  // head GEMM columns
     for (int t = 0; t < T; ++t) {
         p.t = t;
         p.step = a.t0 + (uint32_t)t;
@@ -464,8 +498,7 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
             wm_ktime kt(hd, WM_KERNEL_STEP_CELL, s);
             k_select_cell<<<B, 256, 0, s>>>(p);
         }
-        launch_gemm(hd, round, B, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
-                    w.heads, hd->M + 2, s);
+        launch_gemm(hd, round, B, NH, H, 0, w.h, H, nullptr, 0, hd->step.Wh, NH, hd->step.bh, w.heads, NH, s);
         {
             wm_ktime kt(hd, WM_KERNEL_STEP_SAMPLE, s);
             k_sample<<<B, 128, 0, s>>>(p);
@@ -487,7 +520,8 @@ cudaError_t wm_step_nll(const wm_handle *hd, const wm_nll_dev &a, void *ws, cuda
     {
         wm_ktime kt(hd, WM_KERNEL_AUX, s);
         k_init_state<<<grid_1d((size_t)N * H), 256, 0, s>>>(N, H, Z, nullptr, nullptr, nullptr, nullptr, w.h,
-                                                             w.c, w.frozen, nullptr, w.nll_acc);
+                                                             w.c, w.frozen, nullptr, w.nll_acc, nullptr,
+                                                             nullptr, nullptr, nullptr);
     }
     StepParams p = base_params(hd, N, T, w);
     p.teacher = 1;
@@ -505,8 +539,8 @@ cudaError_t wm_step_nll(const wm_handle *hd, const wm_nll_dev &a, void *ws, cuda
             wm_ktime kt(hd, WM_KERNEL_STEP_CELL, s);
             k_select_cell<<<N, 256, 0, s>>>(p);
         }
-        launch_gemm(hd, round, N, hd->M + 2, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + 2, hd->step.bh,
-                    w.heads, hd->M + 2, s);
+        launch_gemm(hd, round, N, hd->M + hd->NR, H, 0, w.h, H, nullptr, 0, hd->step.Wh, hd->M + hd->NR,
+                    hd->step.bh, w.heads, hd->M + hd->NR, s);
         {
             wm_ktime kt(hd, WM_KERNEL_STEP_SAMPLE, s);
             k_sample<<<N, 128, 0, s>>>(p);

@@ -160,6 +160,12 @@ struct StepIO {
     float *h_seq, *c_seq, *mdn_seq;
     uint8_t *comp_seq;
     float *nll_part;                // [n_head_tiles, B]
+    // shaped reward (Sec. 3.1.4, Eq. 2): columns rd_col + 2, + 3 predict runtime and memory
+    // accesses; rt, mem carry each episode's last predictions
+    int reward_mode;
+    float alpha, beta, invalid_reward;
+    const float *rt0, *mem0;
+    float *rt, *mem, *rt_seq, *mem_seq;
 };
 
 // Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
@@ -772,15 +778,30 @@ struct EpiHeads {
             if (p.t < len) p.nll_part[((size_t)n * 4 + x.cg) * p.B + b] += nll;
         }
         if (n == p.rd_tile) {
-            uint32_t r[2];
+            const bool shaped = p.reward_mode == WM_REWARD_SHAPED;  // uniform
+            uint32_t r[2], q[2] = {0u, 0u};
             asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
                          : "=r"(r[0]), "=r"(r[1]) : "r"(tacc + p.rd_col));
+            if (shaped)
+                asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
+                             : "=r"(q[0]), "=r"(q[1]) : "r"(tacc + p.rd_col + 2));
             tc::tmem_ld_wait();
             if (!p.teacher && valid && x.cg == 0) {
-                const float rew = __uint_as_float(r[0]) + bh[p.rd_col];
+                float rew = __uint_as_float(r[0]) + bh[p.rd_col];
                 const float dl = __uint_as_float(r[1]) + bh[p.rd_col + 1];
                 const int a = p.act[b];
                 const bool noop = p.noop_terminates && a == p.A - 1;
+                if (shaped) {
+                    if (!fz) {  // Eq. 2 on the predictions entering and leaving the step
+                        const float rt = __uint_as_float(q[0]) + bh[p.rd_col + 2];
+                        const float mem = __uint_as_float(q[1]) + bh[p.rd_col + 3];
+                        rew = a >= 0 ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
+                        p.rt[b] = rt;
+                        p.mem[b] = mem;
+                    }
+                    if (p.rt_seq) p.rt_seq[tb] = p.rt[b];
+                    if (p.mem_seq) p.mem_seq[tb] = p.mem[b];
+                }
                 p.rewards[tb] = fz ? 0.f : rew;
                 p.done[tb] = (fz || dl > 0.f || noop) ? 1 : 0;
                 p.fz_next[b] = (fz || (p.done_terminates && dl > 0.f) || noop) ? 1 : 0;
@@ -1012,6 +1033,10 @@ __global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const floa
     }
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)p.B; i += (size_t)gridDim.x * blockDim.x) {
         fz0[i] = fz1[i] = done0 ? (done0[i] != 0) : 0;
+        if (p.rt0) {
+            p.rt[i] = p.rt0[i];
+            p.mem[i] = p.mem0[i];
+        }
         if (p.teacher)
             for (int t = 0; t < 4 * n_head_tiles; ++t) p.nll_part[(size_t)t * p.B + i] = 0.f;
     }
@@ -1110,7 +1135,7 @@ inline size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct TcWs {
     __nv_bfloat16 *x[2];
-    float *c, *h32, *nll_part;
+    float *c, *h32, *nll_part, *rt, *mem;
     int32_t *act;
     uint8_t *fz[2];
 };
@@ -1125,6 +1150,8 @@ TcWs carve_ws(const wm_handle *h, int B, void *ws) {
     w.h32 = (float *)p; p += a256((size_t)B * H * 4);
     w.act = (int32_t *)p; p += a256((size_t)B * 4);
     for (int i = 0; i < 2; ++i) { w.fz[i] = (uint8_t *)p; p += a256((size_t)B); }
+    w.rt = (float *)p; p += a256((size_t)B * 4);
+    w.mem = (float *)p; p += a256((size_t)B * 4);
     w.nll_part = (float *)p;
     return w;
 }
@@ -1140,7 +1167,7 @@ size_t wm_tc_ws(const wm_handle *h, int B) {
     const wm_config &c = h->cfg;
     const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
     return 2 * a256((size_t)B * KX * 2) + 2 * a256((size_t)B * H * 4) + a256((size_t)B * 4) + 2 * a256(B) +
-           a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256;
+           2 * a256((size_t)B * 4) + a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256;
 }
 
 cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
@@ -1156,7 +1183,7 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
     int nht = (Z + dpt - 1) / dpt;
     const int last_dims = Z - (nht - 1) * dpt;
     int rd_tile = nht - 1, rd_col = DS * last_dims;
-    if (rd_col + 2 > HEAD_TILE) {  // reward / done get a tile of their own
+    if (rd_col + h->NR > HEAD_TILE) {  // reward / done (/ runtime / memory) get a tile of their own
         rd_tile = nht;
         rd_col = 0;
         ++nht;
@@ -1203,6 +1230,14 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         }
         bh[rr] = w->b_rew;
         bh[rr + 1] = w->b_done;
+        if (h->NR == 4) {
+            for (int i = 0; i < H; ++i) {
+                wh[(rr + 2) * H + i] = bf(w->w_rt[i]);
+                wh[(rr + 3) * H + i] = bf(w->w_mem[i]);
+            }
+            bh[rr + 2] = w->b_rt;
+            bh[rr + 3] = w->b_mem;
+        }
     }
     cudaError_t e;
     auto up = [&](void **dst, const void *src, size_t bytes) {
@@ -1254,6 +1289,12 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     // during the call it is needed after the last step only
     io.h32_mode = teacher ? 0 : (c.done_terminates || c.noop_terminates) ? 2 : 1;
     io.nll_part = w.nll_part;
+    io.reward_mode = teacher ? WM_REWARD_HEAD : c.reward_mode;
+    io.alpha = c.reward_alpha; io.beta = c.reward_beta; io.invalid_reward = c.invalid_reward;
+    io.rt = w.rt; io.mem = w.mem;
+    if (!teacher && c.reward_mode == WM_REWARD_SHAPED) {
+        io.rt0 = ra->rt0; io.mem0 = ra->mem0; io.rt_seq = ra->rt_seq; io.mem_seq = ra->mem_seq;
+    }
     if (teacher) {
         io.act_in = na->actions; io.z_seq = na->z_seq; io.lengths = na->lengths;
         io.h_seq = na->h_seq; io.c_seq = na->c_seq; io.mdn_seq = na->mdn_seq;

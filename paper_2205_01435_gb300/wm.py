@@ -37,20 +37,22 @@ class wm_config(C.Structure):
                 ("precision", C.c_int), ("mdn_tau", C.c_float), ("sigma_sqrt_tau", C.c_int),
                 ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_float), ("done_terminates", C.c_int),
                 ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int),
-                ("fused_cluster", C.c_int)]
+                ("fused_cluster", C.c_int), ("reward_mode", C.c_int), ("reward_alpha", C.c_float),
+                ("reward_beta", C.c_float), ("invalid_reward", C.c_float)]
 
 
 class wm_weights(C.Structure):
     _fields_ = [("W_lstm", C.c_void_p), ("b_lstm", C.c_void_p), ("W_mdn", C.c_void_p),
                 ("b_mdn", C.c_void_p), ("w_rew", C.c_void_p), ("b_rew", C.c_float),
                 ("w_done", C.c_void_p), ("b_done", C.c_float), ("W_ctrl", C.c_void_p),
-                ("b_ctrl", C.c_void_p)]
+                ("b_ctrl", C.c_void_p), ("w_rt", C.c_void_p), ("b_rt", C.c_float),
+                ("w_mem", C.c_void_p), ("b_mem", C.c_float)]
 
 
 class wm_rollout_io(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "z0", "h0", "c0", "done0", "mask", "z_out", "actions", "rewards", "done", "h_final",
-        "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq")]
+        "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq", "rt0", "mem0", "rt_seq", "mem_seq")]
 
 
 def _load():
@@ -119,13 +121,17 @@ def wm_create(cfg: dict, weights: dict):
                   int(cfg.get("done_terminates", 0)), int(cfg.get("noop_terminates", 0)),
                   int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF,
                   PATHS[cfg.get("path", "auto")] if isinstance(cfg.get("path", "auto"), str)
-                  else int(cfg["path"]), int(cfg.get("fused_cluster", 0)))
+                  else int(cfg["path"]), int(cfg.get("fused_cluster", 0)),
+                  int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
+                  float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)))
     keep = {k: torch.as_tensor(weights[k], dtype=torch.float32).contiguous().cpu()
-            for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl")}
+            for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl",
+                      "w_rt", "w_mem") if weights.get(k) is not None}
     w = wm_weights(_ptr(keep["W_lstm"]), _ptr(keep["b_lstm"]), _ptr(keep["W_mdn"]),
                    _ptr(keep["b_mdn"]), _ptr(keep["w_rew"]), float(weights["b_rew"]),
                    _ptr(keep["w_done"]), float(weights["b_done"]), _ptr(keep["W_ctrl"]),
-                   _ptr(keep["b_ctrl"]))
+                   _ptr(keep["b_ctrl"]), _ptr(keep.get("w_rt")), float(weights.get("b_rt", 0.0)),
+                   _ptr(keep.get("w_mem")), float(weights.get("b_mem", 0.0)))
     h = C.c_void_p()
     st = _lib.wm_create(C.byref(c), C.byref(w), C.byref(h))
     if st != WM_OK:
@@ -219,8 +225,9 @@ class WorldModel:
     def rollout(self, z0: torch.Tensor, T: int, mask: torch.Tensor | None = None,
                 episode_offset: int = 0, t0: int = 0, h0=None, c0=None, done0=None,
                 want_final: bool = True, want_seq: bool = False, out: dict | None = None,
-                stream=None) -> dict:
-        """wm_rollout on B = z0.shape[0] episodes; returns the output tensors (device of z0)."""
+                stream=None, rt0=None, mem0=None) -> dict:
+        """wm_rollout on B = z0.shape[0] episodes; returns the output tensors (device of z0).
+        With the shaped reward, rt0 / mem0 are required and rt_seq / mem_seq are returned."""
         B = int(z0.shape[0])
         o = dict(out or {})
         for name, shape, dt in (("z", (T + 1, B, self.Z), torch.float32),
@@ -238,10 +245,14 @@ class WorldModel:
             o.setdefault("c_seq", self._alloc(z0, (T, B, self.H), torch.float32))
             o.setdefault("mdn_seq", self._alloc(z0, (T, B, self.M), torch.float32))
             o.setdefault("comp_seq", self._alloc(z0, (T, B, self.Z), torch.uint8))
+        if int(self.cfg.get("reward_mode", 0)) == 1:
+            o.setdefault("rt_seq", self._alloc(z0, (T, B), torch.float32))
+            o.setdefault("mem_seq", self._alloc(z0, (T, B), torch.float32))
         io = {"z0": z0, "h0": h0, "c0": c0, "done0": done0, "mask": mask, "z_out": o["z"],
               "actions": o["actions"], "rewards": o["rewards"], "done": o["done"],
               "h_final": o.get("h_final"), "c_final": o.get("c_final"), "h_seq": o.get("h_seq"),
-              "c_seq": o.get("c_seq"), "mdn_seq": o.get("mdn_seq"), "comp_seq": o.get("comp_seq")}
+              "c_seq": o.get("c_seq"), "mdn_seq": o.get("mdn_seq"), "comp_seq": o.get("comp_seq"),
+              "rt0": rt0, "mem0": mem0, "rt_seq": o.get("rt_seq"), "mem_seq": o.get("mem_seq")}
         with torch.cuda.device(self.device):
             wm_rollout(self.h, B, T, episode_offset, t0, io, self._stream(stream))
         return o

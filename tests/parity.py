@@ -48,14 +48,16 @@ def np_(x):
 
 
 def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=None, t0: int = 0,
-                  h0=None, c0=None, done0=None, orc=None, nthreads: int = NT) -> dict:
+                  h0=None, c0=None, done0=None, orc=None, nthreads: int = NT, rt0=None,
+                  mem0=None) -> dict:
     """Step-anchored parity of a GPU rollout of B episodes.
 
     g: the GPU's outputs with their per-step sequences (z, actions, rewards, done,
     h_seq, c_seq, mdn_seq, comp_seq; optional h_final, c_final), batch axis = the
     checked episodes.  z0, mask [T, B, W], h0, c0, done0: the inputs of those
     episodes.  episodes: their global Philox indices (default 0..B-1); t0: the
-    global index of step 0."""
+    global index of step 0.  With the shaped reward, rt0 / mem0 are the predictions
+    entering the call and g carries rt_seq / mem_seq."""
     if orc is None:
         import oracle as orc
     prec = cfg.get("precision", "fp32")
@@ -72,6 +74,10 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
     h = np.zeros((B, H), np.float32) if h0 is None else np.asarray(h0, np.float32)
     c = np.zeros((B, H), np.float32) if c0 is None else np.asarray(c0, np.float32)
     frozen = np.zeros(B, bool) if done0 is None else np.asarray(done0).astype(bool)
+    shaped = int(cfg.get("reward_mode", 0)) == 1
+    if shaped:
+        rt, mem = np.asarray(rt0, np.float32), np.asarray(mem0, np.float32)
+        g_rt, g_mem = np_(g["rt_seq"]), np_(g["mem_seq"])
     refs = [(cfg, tol)]
     if prec == "bf16":
         refs.append((dict(cfg, precision="fp32"), TOL["bf16"]))
@@ -87,16 +93,19 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
     for t in range(T):
         mk = None if mask is None else np.asarray(mask)[t]
         for ri, (rcfg, rtol) in enumerate(refs):
+            sk = dict(rt=rt, mem=mem) if shaped else {}
             s = orc.step(rcfg, weights, ep, t0 + t, gz[t], h, c, frozen=frozen, mask=mk,
-                         a_use=ga[t], h_use=gh[t], k_use=gk[t], nthreads=nthreads)
+                         a_use=ga[t], h_use=gh[t], k_use=gk[t], nthreads=nthreads, **sk)
             if ri == 0:
                 last = s
             live = ~frozen
             where = f"t={t}"
             # values downstream of the shared decisions
-            for key, gv, ov in (("h", gh[t], s["h"]), ("c", gc[t], s["c"]),
-                                ("mdn", gm[t], s["mdn"]), ("reward", gr[t], s["reward"]),
-                                ("z", gz[t + 1], s["z_next"])):
+            vals = [("h", gh[t], s["h"]), ("c", gc[t], s["c"]), ("mdn", gm[t], s["mdn"]),
+                    ("reward", gr[t], s["reward"]), ("z", gz[t + 1], s["z_next"])]
+            if shaped:
+                vals += [("rt", g_rt[t], s["rt"]), ("mem", g_mem[t], s["mem"])]
+            for key, gv, ov in vals:
                 e = np.abs(gv.astype(np.float64) - ov.astype(np.float64))
                 e = e.reshape(B, -1).max(axis=1) if e.ndim > 1 else e
                 bad = np.nonzero(live & (e > rtol))[0]
@@ -114,6 +123,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                 assert np.array_equal(gz[t + 1, fz], gz[t, fz]), where
                 assert np.array_equal(gh[t, fz], h[fz]) and np.array_equal(gc[t, fz], c[fz]), where
                 assert np.all(gm[t, fz] == 0), where
+                if shaped:
+                    assert np.array_equal(g_rt[t, fz], rt[fz]) and np.array_equal(g_mem[t, fz], mem[fz]), where
                 st["frozen_steps"] += len(fz)
             # decisions: equal, or excused by the oracle's own margin
             nl = int(live.sum())
@@ -137,6 +148,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                 flip("component", m)
         # the state the GPU carries into the next step
         h, c = gh[t], gc[t]
+        if shaped:
+            rt, mem = g_rt[t], g_mem[t]
         if cfg.get("done_terminates"):
             frozen = frozen | (gd[t] == 1)
         if cfg.get("noop_terminates"):

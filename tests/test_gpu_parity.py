@@ -440,3 +440,43 @@ def test_tensor_full_batch_is_deterministic(wm, name, T, B, flags):
         for k in ("z", "actions", "rewards", "done", "h_final", "c_final"):
             assert torch.equal(first[k], again[k]), k
     m.sync()
+
+
+# ------------------------------------------------------------------ shaped reward (Eq. 1 / Eq. 2)
+@pytest.mark.parametrize("path,name,flags", [("stepwise", "tiny_fp32", dict(done_terminates=1)),
+                                             ("auto", "small_bf16", dict()),
+                                             ("tensor", "small_bf16", dict(done_terminates=1)),
+                                             ("tensor", "large_bf16", dict()),
+                                             ("stepwise", "mid_bf16", dict(reward_alpha=1.0, reward_beta=0.0))])
+def test_shaped_reward_against_oracle(wm, orc, path, name, flags):
+    """Eq. 2 on the predicted runtime / memory heads, with an invalid step (-100), resumed
+    state, offsets and frozen episodes; AUTO never routes it to the fused family."""
+    cfg = dict(synth.model_config(name), reward_mode=1, **flags)
+    w = synth.weights(cfg, seed=13)
+    B, T = (16, 12) if name == "tiny_fp32" else (200, 6)
+    z0 = synth.z0(B, cfg["z_dim"], seed=13)
+    mask = synth.mask(T, B, cfg["a_dim"], synth.WORKLOADS[name]["mask_density"], seed=13)
+    mask[0, 9] = 0  # no valid action at the first step (episode 9 is live then)
+    rng = np.random.default_rng(13)
+    h0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    c0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    done0 = (np.arange(B) % 37 == 5).astype(np.uint8)
+    rt0, mem0 = synth.shaping_state(B, seed=13)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=55, t0=4, h0=_cuda(h0), c0=_cuda(c0),
+                  done0=_cuda(done0), rt0=_cuda(rt0), mem0=_cuda(mem0), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path != "fused" and (path == "auto" or m.last_path == path)
+    assert int(g["actions"][0, 9]) == -1 and float(g["rewards"][0, 9]) == -100.0
+    r = check_rollout(g, cfg, w, z0, mask, episodes=55 + np.arange(B), t0=4, h0=h0, c0=c0,
+                      done0=done0, orc=orc, rt0=rt0, mem0=mem0)
+    print("shaped", path, name, flags, r)
+    # resumed in two calls: bit for bit the same
+    a = m.rollout(_cuda(z0), 3, mask=_cuda(mask[:3]), episode_offset=55, t0=4, h0=_cuda(h0),
+                  c0=_cuda(c0), done0=_cuda(done0), rt0=_cuda(rt0), mem0=_cuda(mem0), want_seq=True)
+    d0b = torch.maximum(a["done"][2], _cuda(done0)) if cfg.get("done_terminates") else _cuda(done0)
+    b = m.rollout(a["z"][3].contiguous(), T - 3, mask=_cuda(mask[3:]), episode_offset=55, t0=7,
+                  h0=a["h_final"], c0=a["c_final"], done0=d0b,
+                  rt0=a["rt_seq"][2].contiguous(), mem0=a["mem_seq"][2].contiguous(), want_seq=True)
+    for k in ("rewards", "rt_seq", "mem_seq", "actions"):
+        assert torch.equal(torch.cat([a[k], b[k]]), g[k]), k

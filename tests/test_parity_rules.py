@@ -23,15 +23,22 @@ def _case(orc, precision="fp32", **flags):
     c0 = (0.3 * rng.standard_normal((B, 24))).astype(np.float32)
     done0 = (np.arange(B) == 5).astype(np.uint8)
     kw = dict(episode_offset=300, t0=9, h0=h0, c0=c0, done0=done0)
-    o = orc.rollout(cfg, w, z0, mask, T, want_seq=True, **kw)
-    g = {k: o[k].copy() for k in SEQ + ("h_final", "c_final")}
     ck = dict(episodes=300 + np.arange(B), t0=9, h0=h0, c0=c0, done0=done0, orc=orc)
+    keys = SEQ + ("h_final", "c_final")
+    if cfg.get("reward_mode"):
+        rt0, mem0 = synth.shaping_state(B, seed=41)
+        kw.update(rt0=rt0, mem0=mem0)
+        ck.update(rt0=rt0, mem0=mem0)
+        keys += ("rt_seq", "mem_seq")
+    o = orc.rollout(cfg, w, z0, mask, T, want_seq=True, **kw)
+    g = {k: o[k].copy() for k in keys}
     return cfg, w, z0, mask, g, o, ck
 
 
 @pytest.mark.parametrize("precision,flags", [("fp32", {}), ("bf16", {}),
                                              ("fp32", dict(done_terminates=1, noop_terminates=1)),
-                                             ("fp32", dict(ctrl_sample=1, ctrl_tau=0.8))])
+                                             ("fp32", dict(ctrl_sample=1, ctrl_tau=0.8)),
+                                             ("bf16", dict(reward_mode=1, done_terminates=1))])
 def test_oracle_trajectory_passes_without_flips(orc, precision, flags):
     cfg, w, z0, mask, g, o, ck = _case(orc, precision, **flags)
     r = check_rollout(g, cfg, w, z0, mask, **ck)
@@ -73,7 +80,8 @@ def test_tie_broken_the_other_way_is_one_excused_flip(orc):
 
 
 def _planted(orc, how):
-    cfg, w, z0, mask, g, o, ck = _case(orc, "fp32", done_terminates=1)
+    shaped = how in ("shaped_reward", "runtime")
+    cfg, w, z0, mask, g, o, ck = _case(orc, "fp32", done_terminates=1, reward_mode=int(shaped))
     T, B = g["actions"].shape
     live = np.argwhere(o["done"] == 0)
     t, b = (int(x) for x in live[len(live) // 2])
@@ -100,11 +108,15 @@ def _planted(orc, how):
     elif how == "frozen_z":
         fb = 5  # frozen from the start (done0)
         g["z"][t + 1, fb, 0] += 1e-6
+    elif how == "shaped_reward":
+        g["rewards"][t, b] += 5e-4
+    elif how == "runtime":
+        g["rt_seq"][t, b] -= 5e-4
     return cfg, w, z0, mask, g, ck
 
 
 @pytest.mark.parametrize("how", ["action", "component", "done", "z", "h", "mdn", "reward",
-                                 "frozen_z"])
+                                 "frozen_z", "shaped_reward", "runtime"])
 def test_planted_mistakes_fail(orc, how):
     cfg, w, z0, mask, g, ck = _planted(orc, how)
     with pytest.raises(AssertionError):
