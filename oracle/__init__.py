@@ -48,7 +48,8 @@ class _Cfg(C.Structure):
                 ("done_terminates", C.c_int), ("noop_terminates", C.c_int),
                 ("seed", C.c_uint64), ("nthreads", C.c_int), ("reward_mode", C.c_int),
                 ("reward_alpha", C.c_double), ("reward_beta", C.c_double),
-                ("invalid_reward", C.c_double)]
+                ("invalid_reward", C.c_double), ("pop_size", C.c_int), ("pop_group", C.c_int),
+                ("value_head", C.c_int)]
 
 
 class _W(C.Structure):
@@ -56,12 +57,13 @@ class _W(C.Structure):
                 ("b_mdn", C.c_void_p), ("w_rew", C.c_void_p), ("b_rew", C.c_float),
                 ("w_done", C.c_void_p), ("b_done", C.c_float), ("W_ctrl", C.c_void_p),
                 ("b_ctrl", C.c_void_p), ("w_rt", C.c_void_p), ("b_rt", C.c_float),
-                ("w_mem", C.c_void_p), ("b_mem", C.c_float)]
+                ("w_mem", C.c_void_p), ("b_mem", C.c_float), ("w_val", C.c_void_p),
+                ("b_val", C.c_float)]
 
 
 class _Ext(C.Structure):
     _fields_ = [("rt0", C.c_void_p), ("mem0", C.c_void_p), ("rt_seq", C.c_void_p),
-                ("mem_seq", C.c_void_p)]
+                ("mem_seq", C.c_void_p), ("logp_seq", C.c_void_p), ("value_seq", C.c_void_p)]
 
 
 def _load():
@@ -89,6 +91,9 @@ def _load():
             lib.orc_rollout.restype = C.c_int
             lib.orc_step.argtypes = [P, P, C.c_int, P, C.c_uint32] + [P] * 20
             lib.orc_step.restype = C.c_int
+            lib.orc_returns.argtypes = [C.c_int, C.c_int, C.c_double, C.c_int, P, P, P, P,
+                                        C.c_uint64, C.c_int, C.c_int, P]
+            lib.orc_returns.restype = C.c_int
             lib.orc_mdn_nll.argtypes = [P, P, C.c_int, C.c_int] + [P] * 7
             lib.orc_mdn_nll.restype = C.c_int
             _lib = lib
@@ -111,7 +116,9 @@ def _cfg(cfg: dict, nthreads: int) -> _Cfg:
                 int(cfg.get("done_terminates", 0)), int(cfg.get("noop_terminates", 0)),
                 int(cfg.get("seed", 0)) & 0xFFFFFFFFFFFFFFFF, int(nthreads),
                 int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
-                float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)))
+                float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)),
+                int(cfg.get("pop_size", 0)), int(cfg.get("pop_group", 1)),
+                int(cfg.get("value_head", 0)))
 
 
 class _Weights:
@@ -119,32 +126,37 @@ class _Weights:
 
     def __init__(self, w: dict):
         self.arrs = {k: _f32(w[k]) for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew",
-                                               "w_done", "W_ctrl", "b_ctrl", "w_rt", "w_mem")
-                     if w.get(k) is not None}
+                                               "w_done", "W_ctrl", "b_ctrl", "w_rt", "w_mem",
+                                               "w_val") if w.get(k) is not None}
         a = self.arrs
         self.s = _W(_ptr(a["W_lstm"]), _ptr(a["b_lstm"]), _ptr(a["W_mdn"]), _ptr(a["b_mdn"]),
                     _ptr(a["w_rew"]), float(w["b_rew"]), _ptr(a["w_done"]), float(w["b_done"]),
                     _ptr(a["W_ctrl"]), _ptr(a["b_ctrl"]), _ptr(a.get("w_rt")),
-                    float(w.get("b_rt", 0.0)), _ptr(a.get("w_mem")), float(w.get("b_mem", 0.0)))
+                    float(w.get("b_rt", 0.0)), _ptr(a.get("w_mem")), float(w.get("b_mem", 0.0)),
+                    _ptr(a.get("w_val")), float(w.get("b_val", 0.0)))
 
 
 class _ExtArgs:
-    """The optional parts of a call (shaped-reward state); keeps the arrays alive."""
+    """The optional parts of a call (shaped-reward state, log-probs, values); keeps the
+    arrays alive."""
 
     def __init__(self, cfg: dict, B: int, T: int, rt0=None, mem0=None):
-        self.out = {}
-        self.keep = []
-        self.s = None
+        self.out = {"logp_seq": np.zeros((T, B), np.float32)}
+        r = m = None
         if int(cfg.get("reward_mode", 0)) == 1:
             if rt0 is None or mem0 is None:
                 raise ValueError("the shaped reward needs rt0 and mem0")
             r, m = _f32(rt0).reshape(B), _f32(mem0).reshape(B)
-            self.out = {"rt_seq": np.zeros((T, B), np.float32), "mem_seq": np.zeros((T, B), np.float32)}
-            self.keep = [r, m]
-            self.s = _Ext(_ptr(r), _ptr(m), _ptr(self.out["rt_seq"]), _ptr(self.out["mem_seq"]))
+            self.out.update(rt_seq=np.zeros((T, B), np.float32), mem_seq=np.zeros((T, B), np.float32))
+        if int(cfg.get("value_head", 0)):
+            self.out["value_seq"] = np.zeros((T, B), np.float32)
+        self.keep = [r, m]
+        o = self.out
+        self.s = _Ext(_ptr(r), _ptr(m), _ptr(o.get("rt_seq")), _ptr(o.get("mem_seq")),
+                      _ptr(o["logp_seq"]), _ptr(o.get("value_seq")))
 
     def ref(self):
-        return None if self.s is None else C.byref(self.s)
+        return C.byref(self.s)
 
 
 # ---------------------------------------------------------------- building blocks
@@ -302,8 +314,34 @@ def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=No
                       _ptr(out["z_next"]), ext.ref())
     if rc != 0:
         raise ValueError(f"orc_step failed ({rc})")
-    if ext.out:
+    if "rt_seq" in ext.out:
         out["rt"], out["mem"] = ext.out["rt_seq"][0], ext.out["mem_seq"][0]
+    out["logp"] = ext.out["logp_seq"][0]
+    if "value_seq" in ext.out:
+        out["value"] = ext.out["value_seq"][0]
+    return out
+
+
+def returns(rewards, done, gamma: float, stop_at_done: bool = True, bootstrap=None,
+            episode_offset: int = 0, pop_size: int = 0, pop_group: int = 1) -> dict:
+    """Discounted returns G_t = r_t + gamma G_{t+1} of [T, B] rollouts (from bootstrap [B],
+    else 0; a done step ends the sum when stop_at_done) and, with a population, each
+    candidate's mean G_0 ("fitness")."""
+    lib = _load()
+    r = _f32(rewards)
+    T, B = r.shape
+    d = np.ascontiguousarray(done, dtype=np.uint8).reshape(T, B)
+    bs = None if bootstrap is None else _f32(bootstrap).reshape(B)
+    out = {"returns": np.zeros((T, B), np.float32)}
+    fit = None
+    if pop_size >= 1:
+        fit = np.zeros(pop_size, np.float64)
+        out["fitness"] = fit
+    rc = lib.orc_returns(B, T, float(gamma), int(bool(stop_at_done)), _ptr(r), _ptr(d), _ptr(bs),
+                         _ptr(out["returns"]), int(episode_offset), int(max(pop_size, 1)),
+                         int(pop_group), _ptr(fit))
+    if rc != 0:
+        raise ValueError(f"orc_returns failed ({rc})")
     return out
 
 

@@ -257,8 +257,9 @@ int orc_select_action(int A, const float *logits, const uint32_t *mask_words,
 /* Weights widened to fp64 (rounded to bf16 first in bf16 mode).             */
 /* ------------------------------------------------------------------------- */
 typedef struct {
-    double *W_lstm, *b_lstm, *W_mdn, *b_mdn, *w_rew, *w_done, *W_ctrl, *b_ctrl, *w_rt, *w_mem;
-    double b_rew, b_done, b_rt, b_mem;
+    double *W_lstm, *b_lstm, *W_mdn, *b_mdn, *w_rew, *w_done, *W_ctrl, *b_ctrl, *w_rt, *w_mem,
+        *w_val;
+    double b_rew, b_done, b_rt, b_mem, b_val;
 } wts64;
 
 static double *widen(const float *src, size_t n, int round_bf16)
@@ -273,7 +274,7 @@ static void free_wts(wts64 *v)
 {
     free(v->W_lstm); free(v->b_lstm); free(v->W_mdn); free(v->b_mdn);
     free(v->w_rew); free(v->w_done); free(v->W_ctrl); free(v->b_ctrl);
-    free(v->w_rt); free(v->w_mem);
+    free(v->w_rt); free(v->w_mem); free(v->w_val);
 }
 
 static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need_ctrl)
@@ -290,8 +291,17 @@ static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need
     v->b_rew = (double)w->b_rew;
     v->b_done = (double)w->b_done;
     if (need_ctrl) {
-        v->W_ctrl = widen(w->W_ctrl, (size_t)(Z + H) * A, rb);
-        v->b_ctrl = widen(w->b_ctrl, (size_t)A, 0);
+        const size_t P = cfg->pop_size > 1 ? (size_t)cfg->pop_size : 1;
+        v->W_ctrl = widen(w->W_ctrl, P * (Z + H) * A, rb);
+        v->b_ctrl = widen(w->b_ctrl, P * A, 0);
+    }
+    if (cfg->value_head) {
+        if (!w->w_val) {
+            free_wts(v);
+            return -1;
+        }
+        v->w_val = widen(w->w_val, (size_t)H, rb);
+        v->b_val = (double)w->b_val;
     }
     const int shaped = cfg->reward_mode == 1;
     if (shaped) {
@@ -305,7 +315,8 @@ static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need
         v->b_mem = (double)w->b_mem;
     }
     if (!v->W_lstm || !v->b_lstm || !v->W_mdn || !v->b_mdn || !v->w_rew || !v->w_done ||
-        (need_ctrl && (!v->W_ctrl || !v->b_ctrl)) || (shaped && (!v->w_rt || !v->w_mem))) {
+        (need_ctrl && (!v->W_ctrl || !v->b_ctrl)) || (shaped && (!v->w_rt || !v->w_mem)) ||
+        (cfg->value_head && !v->w_val)) {
         free_wts(v);
         return -1;
     }
@@ -324,6 +335,7 @@ static int check_cfg(const orc_cfg *c)
     if (c->z_dim <= 0 || c->a_dim <= 0 || c->h_dim <= 0 || c->k_mix <= 0 || c->k_mix > 64) return -1;
     if (!(c->mdn_tau >= 0.0) || !(c->ctrl_tau >= 0.0)) return -1;
     if (c->reward_mode != 0 && c->reward_mode != 1) return -1;
+    if (c->pop_size > 1 && c->pop_group < 1) return -1;
     return 0;
 }
 
@@ -406,7 +418,8 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
                         uint32_t s, double *z, double *h, double *c, double *rt, double *mem,
                         const uint32_t *mw, int a_use, const float *h_use, const uint8_t *k_use,
                         int32_t *action, float *ctrl_margin, float *reward, uint8_t *done,
-                        float *done_margin, float *mdn_out, uint8_t *comp, float *comp_margin)
+                        float *done_margin, float *mdn_out, uint8_t *comp, float *comp_margin,
+                        float *logp, float *value)
 {
     const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
     double *x = sb->x, *g = sb->g, *y = sb->y, *mdn = sb->mdn, *znew = sb->znew;
@@ -414,10 +427,12 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
     for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z[i]);
     for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
 
-    /* a1: controller logits, rounded to fp32 for the decision */
+    /* a1: controller logits of the episode's candidate, rounded to fp32 for the decision */
+    const size_t cand = cfg->pop_size > 1 ? (size_t)((e / (uint64_t)cfg->pop_group) % (uint64_t)cfg->pop_size) : 0;
+    const double *Wc = v->W_ctrl + cand * (size_t)(Z + H) * A, *bc = v->b_ctrl + cand * (size_t)A;
     for (int j = 0; j < A; ++j) {
-        double l = v->b_ctrl[j];
-        for (int i = 0; i < Z + H; ++i) l += x[i] * v->W_ctrl[(size_t)i * A + j];
+        double l = bc[j];
+        for (int i = 0; i < Z + H; ++i) l += x[i] * Wc[(size_t)i * A + j];
         lg[j] = (float)l;
     }
     /* a2: mask + select */
@@ -432,6 +447,19 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
     *action = a;
     if (ctrl_margin) *ctrl_margin = (float)cm;
     if (a_use >= -1) a = a_use;
+    /* log pi(a | z, h) of the action taken, pi = softmax(l / ctrl_tau) over the valid actions */
+    if (logp) {
+        double lp = 0.0;
+        if (a >= 0 && cfg->ctrl_tau > 0.0) {
+            double lmax = -INFINITY, S = 0.0;
+            for (int j = 0; j < A; ++j)
+                if ((!mw || bit_set(mw, j)) && (double)lg[j] > lmax) lmax = (double)lg[j];
+            for (int j = 0; j < A; ++j)
+                if (!mw || bit_set(mw, j)) S += exp(((double)lg[j] - lmax) / cfg->ctrl_tau);
+            lp = ((double)lg[a] - lmax) / cfg->ctrl_tau - log(S);
+        }
+        *logp = (float)lp;
+    }
 
     /* a3 + a4 */
     lstm_step(cfg, v, x, a, g, c, h);
@@ -453,6 +481,11 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
         *mem = mem_new;
     }
     *reward = (float)r;
+    if (value) {
+        double vv = v->b_val;
+        for (int i = 0; i < H; ++i) vv += y[i] * v->w_val[i];
+        *value = (float)vv;
+    }
     float dlf = (float)dl;
     if (done_margin) *done_margin = fabsf(dlf);
     int is_noop = cfg->noop_terminates && a == A - 1;
@@ -523,8 +556,12 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
     for (int t = 0; t < T; ++t) {
         const uint32_t s = t0 + (uint32_t)t;
         const size_t tb = (size_t)t * B + b;
+        float *lp_out = ext && ext->logp_seq ? ext->logp_seq + tb : NULL;
+        float *v_out = ext && ext->value_seq && cfg->value_head ? ext->value_seq + tb : NULL;
         if (frozen) {
             actions[tb] = -1; rewards[tb] = 0.0f; done[tb] = 1;
+            if (lp_out) *lp_out = 0.0f;
+            if (v_out) *v_out = 0.0f;
             if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = 0.0f;
             if (comp_seq) for (int d = 0; d < Z; ++d) comp_seq[tb * Z + d] = 255;
             if (ctrl_margin) ctrl_margin[tb] = INF_F;
@@ -537,7 +574,7 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
                                   done_margin ? &done_margin[tb] : NULL,
                                   mdn_seq ? mdn_seq + tb * M : NULL,
                                   comp_seq ? comp_seq + tb * Z : NULL,
-                                  comp_margin ? comp_margin + tb * Z : NULL);
+                                  comp_margin ? comp_margin + tb * Z : NULL, lp_out, v_out);
         }
         for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
         if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
@@ -621,8 +658,12 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
         for (int i = 0; i < Z; ++i) zs[i] = z[(size_t)b * Z + i];
         for (int i = 0; i < H; ++i) { hs[i] = h[(size_t)b * H + i]; cs[i] = c[(size_t)b * H + i]; }
         double rt = shaped ? (double)ext->rt0[b] : 0.0, mem = shaped ? (double)ext->mem0[b] : 0.0;
+        float *lp_out = ext && ext->logp_seq ? ext->logp_seq + b : NULL;
+        float *v_out = ext && ext->value_seq && cfg->value_head ? ext->value_seq + b : NULL;
         if (frozen && frozen[b]) {
             action[b] = -1; ctrl_margin[b] = INF_F; reward[b] = 0.0f; done[b] = 1;
+            if (lp_out) *lp_out = 0.0f;
+            if (v_out) *v_out = 0.0f;
             done_margin[b] = INF_F;
             for (int m = 0; m < M; ++m) mdn_out[(size_t)b * M + m] = 0.0f;
             for (int d = 0; d < Z; ++d) {
@@ -636,7 +677,7 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
                          k_use ? k_use + (size_t)b * Z : NULL,
                          &action[b], &ctrl_margin[b], &reward[b], &done[b], &done_margin[b],
                          mdn_out + (size_t)b * M, comp + (size_t)b * Z,
-                         comp_margin + (size_t)b * Z);
+                         comp_margin + (size_t)b * Z, lp_out, v_out);
         }
         for (int i = 0; i < Z; ++i) z_next[(size_t)b * Z + i] = (float)zs[i];
         for (int i = 0; i < H; ++i) {
@@ -649,6 +690,41 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
     }
     free_wts(&v);
     return bad ? -2 : 0;
+}
+
+int orc_returns(int B, int T, double gamma, int stop_at_done, const float *rewards,
+                const uint8_t *done, const float *bootstrap, float *returns,
+                uint64_t episode_offset, int P, int E, double *fitness)
+{
+    if (B < 0 || T < 0 || !rewards || !done || !returns) return -1;
+    if (fitness && (P < 1 || E < 1)) return -1;
+    double *g0 = malloc(sizeof(double) * (B > 0 ? B : 1));
+    if (!g0) return -2;
+    for (int b = 0; b < B; ++b) {
+        double G = bootstrap ? (double)bootstrap[b] : 0.0;
+        for (int t = T - 1; t >= 0; --t) {
+            const size_t tb = (size_t)t * B + b;
+            if (stop_at_done && done[tb]) G = 0.0;
+            G = (double)rewards[tb] + gamma * G;
+            returns[tb] = (float)G;
+        }
+        g0[b] = T > 0 ? G : (bootstrap ? (double)bootstrap[b] : 0.0);
+    }
+    if (fitness) {
+        for (int g = 0; g < P; ++g) {
+            double sum = 0.0;
+            long n = 0;
+            for (int b = 0; b < B; ++b) {
+                const uint64_t e = episode_offset + (uint64_t)b;
+                if ((int)((e / (uint64_t)E) % (uint64_t)P) != g) continue;
+                sum += g0[b];
+                ++n;
+            }
+            fitness[g] = n ? sum / (double)n : 0.0;
+        }
+    }
+    free(g0);
+    return 0;
 }
 
 static int nll_sequence(const orc_cfg *cfg, const wts64 *v, int n, int N, int T,

@@ -45,6 +45,12 @@ typedef struct {
      * (Eq. 1 is alpha = 1, beta = 0)                                       */
     int reward_mode;
     double reward_alpha, reward_beta, invalid_reward;
+    /* controller population (Sec. 3.4, CMA-ES over controller weights):
+     * pop_size P candidates; global episode e acts with candidate
+     * (e / pop_group) mod P.  P <= 1: one controller.                     */
+    int pop_size, pop_group;
+    /* value head V(h') = w_val . h' + b_val (1 = on)                        */
+    int value_head;
 } orc_cfg;
 
 typedef struct {
@@ -56,12 +62,14 @@ typedef struct {
     float b_rew;
     const float *w_done;  /* [H]                                             */
     float b_done;
-    const float *W_ctrl;  /* [Z+H, A]                                        */
-    const float *b_ctrl;  /* [A]                                             */
+    const float *W_ctrl;  /* [P, Z+H, A]  (P = max(pop_size, 1))             */
+    const float *b_ctrl;  /* [P, A]                                          */
     const float *w_rt;    /* [H] runtime head (reward_mode 1), else NULL     */
     float b_rt;
     const float *w_mem;   /* [H] memory-access head (reward_mode 1)          */
     float b_mem;
+    const float *w_val;   /* [H] value head (value_head 1), else NULL        */
+    float b_val;
 } orc_weights;
 
 /* Inputs and outputs of the optional parts of a rollout (NULL = not used).
@@ -71,6 +79,10 @@ typedef struct {
 typedef struct {
     const float *rt0, *mem0;
     float *rt_seq, *mem_seq;
+    /* logp_seq [T,B]: log pi(a_t | z_t, h_t) of the action taken under the
+     * controller's masked softmax at temperature ctrl_tau (0 when ctrl_tau
+     * is 0 or no action was valid); value_seq [T,B]: V(h_{t+1}) (value_head). */
+    float *logp_seq, *value_seq;
 } orc_ext;
 
 /* ---- building blocks (exported so tests can pin each one) ---------------- */
@@ -120,6 +132,16 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
              int32_t *action, float *ctrl_margin, float *h_out, float *c_out, float *mdn_out,
              float *reward, uint8_t *done, float *done_margin, uint8_t *comp,
              float *comp_margin, float *z_next, const orc_ext *ext);
+
+/* Discounted returns of B rollouts of T steps (Sec. 3.1 objective):
+ * G_t = r_t + gamma G_{t+1}, from G_T = bootstrap[b] (NULL: 0).  With
+ * stop_at_done, a step with done_t = 1 ends the sum (G_t = r_t).  returns
+ * [T,B] out.  If fitness is non-NULL, fitness[g] (g < P) is the mean G_0
+ * over the call's episodes of candidate g ((episode_offset + b) / E mod P),
+ * 0 for a candidate with no episode. */
+int orc_returns(int B, int T, double gamma, int stop_at_done, const float *rewards,
+                const uint8_t *done, const float *bootstrap, float *returns,
+                uint64_t episode_offset, int P, int E, double *fitness);
 
 int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
                 const float *z_seq, const int32_t *actions, const int32_t *lengths,

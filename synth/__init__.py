@@ -50,7 +50,7 @@ WORKLOADS = {
 
 _STREAM = {"W_lstm": 1, "b_lstm": 2, "W_mdn": 3, "b_mdn": 4, "w_rew": 5, "b_rew": 6,
            "w_done": 7, "b_done": 8, "W_ctrl": 9, "b_ctrl": 10, "w_rt": 11, "b_rt": 12,
-           "w_mem": 13, "b_mem": 14,
+           "w_mem": 13, "b_mem": 14, "W_pop": 15, "b_pop": 16, "w_val": 17, "b_val": 18,
            "z0": 20, "mask": 21, "zseq": 22, "actions": 23, "lengths": 24, "rt0": 25, "mem0": 26}
 
 
@@ -75,7 +75,9 @@ def model_config(name: str, **over) -> dict:
                ctrl_tau=w.get("ctrl_tau", 1.0), done_terminates=w.get("done_terminates", 0),
                noop_terminates=w.get("noop_terminates", 0), seed=w.get("seed", 0),
                reward_mode=w.get("reward_mode", 0), reward_alpha=w.get("reward_alpha", 0.8),
-               reward_beta=w.get("reward_beta", 0.2), invalid_reward=w.get("invalid_reward", -100.0))
+               reward_beta=w.get("reward_beta", 0.2), invalid_reward=w.get("invalid_reward", -100.0),
+               pop_size=w.get("pop_size", 0), pop_group=w.get("pop_group", 1),
+               value_head=w.get("value_head", 0))
     return cfg
 
 
@@ -85,12 +87,23 @@ def weights(cfg: dict, seed: int = 0, std: float = 0.05) -> dict:
     shapes = {"W_lstm": (Z + A + H, 4 * H), "b_lstm": (4 * H,), "W_mdn": (H, 3 * K * Z),
               "b_mdn": (3 * K * Z,), "w_rew": (H,), "b_rew": (), "w_done": (H,), "b_done": (),
               "W_ctrl": (Z + H, A), "b_ctrl": (A,), "w_rt": (H,), "b_rt": (), "w_mem": (H,),
-              "b_mem": ()}
+              "b_mem": (), "w_val": (H,), "b_val": ()}
     out = {}
     for name, shp in shapes.items():
         v = _rng(seed, _STREAM[name]).standard_normal(shp, dtype=np.float32) * np.float32(std)
         out[name] = float(v) if shp == () else np.ascontiguousarray(v, dtype=np.float32)
     return out
+
+
+def population(cfg: dict, P: int, seed: int = 0, std: float = 0.05):
+    """(W_ctrl [P, Z+H, A], b_ctrl [P, A]): P controller candidates, each ~ N(0, std^2)
+    from a stream of its own (one generation of a controller search)."""
+    Z, A, H = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"]
+    W = np.stack([_rng(seed, _STREAM["W_pop"], g).standard_normal((Z + H, A), dtype=np.float32)
+                  for g in range(P)]) * np.float32(std)
+    b = np.stack([_rng(seed, _STREAM["b_pop"], g).standard_normal(A, dtype=np.float32)
+                  for g in range(P)]) * np.float32(std)
+    return np.ascontiguousarray(W, np.float32), np.ascontiguousarray(b, np.float32)
 
 
 def shaping_state(B: int, seed: int = 0, shard: int = 0):

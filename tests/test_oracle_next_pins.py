@@ -112,3 +112,124 @@ def test_step_carries_the_predictions(orc):
         s = orc.step(cfg, w, np.arange(B), t, o["z"][t], h, c, mask=mk[t], rt=rp, mem=mp)
         assert np.array_equal(s["reward"], o["rewards"][t])
         assert np.array_equal(s["rt"], o["rt_seq"][t]) and np.array_equal(s["mem"], o["mem_seq"][t])
+
+
+# ----------------------------------------------------------------------------- population (Sec. 3.4)
+def test_population_equals_single_controller_runs(orc):
+    """Episode e acts with candidate (e / E) mod P: a population rollout equals, episode by
+    episode, a one-controller rollout with that candidate's weights."""
+    Z, A, H, K, B, T, P, E = 4, 12, 16, 2, 11, 5, 3, 2
+    cfg = _cfg(Z, A, H, K, reward_mode=0, ctrl_sample=1, ctrl_tau=0.9, pop_size=P, pop_group=E)
+    w = synth.weights(cfg, seed=52, std=0.4)
+    Wp, bp = synth.population(cfg, P, seed=52, std=0.4)
+    wp = dict(w, W_ctrl=Wp, b_ctrl=bp)
+    z0 = synth.z0(B, Z, seed=52)
+    mk = synth.mask(T, B, A, 0.6, seed=52)
+    off = 5
+    o = orc.rollout(cfg, wp, z0, mk, T, episode_offset=off, want_seq=True)
+    single = dict(cfg, pop_size=0)
+    seen = set()
+    for b in range(B):
+        g = ((off + b) // E) % P
+        seen.add(g)
+        one = orc.rollout(single, dict(w, W_ctrl=Wp[g], b_ctrl=bp[g]), z0[b:b + 1], mk[:, b:b + 1], T,
+                          episode_offset=off + b, want_seq=True)
+        for k in ("actions", "z", "rewards", "logp_seq", "h_seq"):
+            assert np.array_equal(o[k][:, b], one[k][:, 0]), (k, b)
+    assert seen == set(range(P))
+
+
+# ----------------------------------------------------------------------------- log-prob, value
+def test_logp_matches_torch_categorical(orc):
+    """logp_seq = log softmax(l / tau)[a] over the valid actions (torch Categorical on the
+    logits rebuilt from the rollout's own state)."""
+    import torch
+    Z, A, H, K, B, T = 5, 14, 16, 2, 6, 5
+    for sample, tau in ((1, 0.7), (0, 1.3)):
+        cfg = _cfg(Z, A, H, K, reward_mode=0, ctrl_sample=sample, ctrl_tau=tau)
+        w = synth.weights(cfg, seed=53, std=0.5)
+        z0 = synth.z0(B, Z, seed=53)
+        mk = synth.mask(T, B, A, 0.5, seed=53)
+        mk[1, 2] = 0
+        o = orc.rollout(cfg, w, z0, mk, T, want_seq=True)
+        for t in range(T):
+            h = np.zeros((B, H)) if t == 0 else o["h_seq"][t - 1].astype(np.float64)
+            lg = (np.concatenate([o["z"][t].astype(np.float64), h], 1) @ w["W_ctrl"].astype(np.float64)
+                  + w["b_ctrl"]).astype(np.float32).astype(np.float64)
+            valid = np.unpackbits(mk[t].view(np.uint8), axis=1, bitorder="little")[:, :A].astype(bool)
+            for b in range(B):
+                a = int(o["actions"][t, b])
+                if a < 0:
+                    assert o["logp_seq"][t, b] == 0.0
+                    continue
+                d = torch.distributions.Categorical(
+                    logits=torch.from_numpy(np.where(valid[b], lg[b] / tau, -np.inf)))
+                assert o["logp_seq"][t, b] == pytest.approx(float(d.log_prob(torch.tensor(a))), abs=2e-6)
+
+
+def test_logp_normalises_over_valid_actions(orc):
+    """Forcing each valid action in turn, exp(logp) sums to 1 (and tau = 0 gives 0)."""
+    Z, A, H, K, B = 4, 9, 12, 2, 5
+    cfg = _cfg(Z, A, H, K, reward_mode=0, ctrl_sample=1, ctrl_tau=0.6)
+    w = synth.weights(cfg, seed=54, std=0.6)
+    rng = np.random.default_rng(54)
+    z = rng.standard_normal((B, Z)).astype(np.float32)
+    h = (0.5 * rng.standard_normal((B, H))).astype(np.float32)
+    c = np.zeros((B, H), np.float32)
+    mk = synth.mask(1, B, A, 0.6, seed=54)[0]
+    valid = np.unpackbits(mk.view(np.uint8), axis=1, bitorder="little")[:, :A].astype(bool)
+    total = np.zeros(B)
+    for j in range(A):
+        s = orc.step(cfg, w, np.arange(B), 0, z, h, c, mask=mk, a_use=np.full(B, j))
+        total += np.where(valid[:, j], np.exp(s["logp"].astype(np.float64)), 0.0)
+    np.testing.assert_allclose(total[valid.any(1)], 1.0, atol=1e-5)
+    s0 = orc.step(dict(cfg, ctrl_tau=0.0), w, np.arange(B), 0, z, h, c, mask=mk)
+    assert np.all(s0["logp"] == 0.0)
+
+
+def test_value_head_is_linear_in_h(orc):
+    Z, A, H, K, B, T = 4, 8, 16, 2, 5, 4
+    cfg = _cfg(Z, A, H, K, reward_mode=0, value_head=1, done_terminates=1)
+    w = synth.weights(cfg, seed=55, std=0.4)
+    z0 = synth.z0(B, Z, seed=55)
+    o = orc.rollout(cfg, w, z0, None, T, want_seq=True)
+    ref = o["h_seq"].astype(np.float64) @ w["w_val"].astype(np.float64) + w["b_val"]
+    live = np.ones((T, B), bool)
+    live[1:] = np.cumsum(o["done"], 0)[:-1] == 0
+    np.testing.assert_allclose(o["value_seq"][live], ref[live], atol=1e-6)
+    assert np.all(o["value_seq"][~live] == 0)
+
+
+# ----------------------------------------------------------------------------- returns, fitness
+def test_returns_closed_forms(orc):
+    T, B, gamma = 6, 4, 0.9
+    r = np.full((T, B), 2.0, np.float32)
+    d = np.zeros((T, B), np.uint8)
+    boot = np.array([0.0, 1.0, -3.0, 10.0], np.float32)
+    out = orc.returns(r, d, gamma, bootstrap=boot)["returns"]
+    for t in range(T):
+        n = T - t
+        ref = 2.0 * (1 - gamma**n) / (1 - gamma) + gamma**n * boot.astype(np.float64)
+        np.testing.assert_allclose(out[t], ref, rtol=1e-6)
+    # a done step ends the sum: G_t = r_t there, and nothing after it leaks back
+    d[2, 1] = 1
+    r2 = r.copy()
+    r2[3:, 1] = 1000.0
+    out2 = orc.returns(r2, d, gamma, bootstrap=boot)["returns"]
+    assert out2[2, 1] == np.float32(2.0)
+    assert out2[0, 1] == pytest.approx(2.0 + gamma * 2.0 + gamma**2 * 2.0, rel=1e-6)
+    # without stop_at_done the done flag is ignored
+    out3 = orc.returns(r2, d, gamma, stop_at_done=False)["returns"]
+    assert out3[2, 1] > 100
+
+
+def test_fitness_is_mean_return_per_candidate(orc):
+    T, B, P, E, off = 3, 13, 3, 2, 7
+    rng = np.random.default_rng(56)
+    r = rng.standard_normal((T, B)).astype(np.float32)
+    d = np.zeros((T, B), np.uint8)
+    out = orc.returns(r, d, 0.5, episode_offset=off, pop_size=P, pop_group=E)
+    g0 = out["returns"][0].astype(np.float64)
+    for g in range(P):
+        sel = [b for b in range(B) if ((off + b) // E) % P == g]
+        assert out["fitness"][g] == pytest.approx(g0[sel].mean(), rel=1e-6)
