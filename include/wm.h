@@ -109,6 +109,10 @@ typedef struct {
     int reward_mode;                  /* WM_REWARD_HEAD or WM_REWARD_SHAPED         */
     float reward_alpha, reward_beta;
     float invalid_reward;
+    int value_head;                   /* 1: a value head V(h') = w_val . h' + b_val
+                                         (a critic on the world model's state, for
+                                         PPO-style training); stepwise and tensor
+                                         families                                   */
 } wm_config;
 
 enum { WM_REWARD_HEAD = 0, WM_REWARD_SHAPED = 1 };
@@ -130,6 +134,8 @@ typedef struct {
     float b_rt;
     const float *w_mem;   /* [H] predicted memory-access head (WM_REWARD_SHAPED)  */
     float b_mem;
+    const float *w_val;   /* [H] value head (value_head only)                    */
+    float b_val;
 } wm_weights;
 
 typedef struct wm_handle wm_handle;
@@ -157,6 +163,11 @@ typedef struct {
                                     entering the call (resume: the last rt_seq / mem_seq) */
     float *rt_seq, *mem_seq;     /* [T,B]   optional: RT_t, M_t after each step (frozen:
                                     repeated)                                          */
+    float *logp_seq;             /* [T,B]   optional: log pi(a_t | z_t, h_t) of the action
+                                    taken, pi = softmax(l / ctrl_tau) over the valid
+                                    actions (Sec. 3.4); 0 if ctrl_tau = 0, no action was
+                                    valid, or the episode is frozen                    */
+    float *value_seq;            /* [T,B]   optional (value_head): V(h_{t+1}); 0 if frozen */
 } wm_rollout_io;
 
 /* Creates a world model on the current CUDA device from the weights of the
@@ -223,6 +234,30 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
 #define WM_NOALLOC_SCRATCH_BYTES (16u << 20)
 wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned long long episode_offset,
                              unsigned int t0, const wm_rollout_io *io, void *cuda_stream);
+
+/* Replaces the controller with a population of P candidates (Sec. 3.4: CMA-ES
+ * searches over the controller's weights, evaluating each candidate by its
+ * return in the world model).  Global episode e = episode_offset + b acts with
+ * candidate (e / E) mod P, so a generation of P candidates x E episodes is one
+ * wm_rollout of P*E episodes.  W_ctrl [P, Z+H, A] and b_ctrl [P, A] are host
+ * fp32 arrays in the layout of wm_weights, copied and packed (P = 1 restores a
+ * single controller).  The tensor-core family takes a population when E and
+ * the call's episode_offset are multiples of 256 (its row tiles then belong to
+ * one candidate); AUTO picks another family otherwise, and the fused family
+ * takes none.  WM_ERR_INVALID_ARG for P < 1, E < 1 or NULL arrays. */
+wm_status wm_set_controllers(wm_handle *h, int P, int E, const float *W_ctrl, const float *b_ctrl);
+
+/* Discounted returns of a rollout (the objective of Sec. 3.1, discount gamma):
+ * G_t = r_t + gamma G_{t+1}, from G_T = bootstrap[b] (NULL: 0); with
+ * stop_at_done a step with done = 1 ends the sum (G_t = r_t).
+ *   rewards, done [T,B] as wm_rollout wrote them; returns [T,B] out;
+ *   fitness [P] optional out: each candidate's mean G_0 over this call's
+ *   episodes (candidate of episode b: (episode_offset + b) / E mod P, the
+ *   handle's population), summed in episode order (deterministic).
+ * Arrays may be host or device memory, as for wm_rollout. */
+wm_status wm_returns(wm_handle *h, int B, int T, unsigned long long episode_offset, float gamma,
+                     int stop_at_done, const float *rewards, const uint8_t *done,
+                     const float *bootstrap, float *returns, float *fitness, void *cuda_stream);
 
 /* Synchronises the device and returns the first device-side error since the
  * last wm_sync (WM_ERR_TIMEOUT if a bounded wait gave up), then clears it. */

@@ -233,18 +233,20 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
         for (size_t m = 0; m < M; ++m) Wh[i * (M + NR) + m] = wv(w->W_mdn[i * M + m]);
         Wh[i * (M + NR) + M] = wv(w->w_rew[i]);
         Wh[i * (M + NR) + M + 1] = wv(w->w_done[i]);
-        if (NR == 4) {
+        if (c.reward_mode == WM_REWARD_SHAPED) {
             Wh[i * (M + NR) + M + 2] = wv(w->w_rt[i]);
             Wh[i * (M + NR) + M + 3] = wv(w->w_mem[i]);
         }
+        if (c.value_head) Wh[i * (M + NR) + M + NR - 1] = wv(w->w_val[i]);
     }
     for (size_t m = 0; m < M; ++m) bh[m] = w->b_mdn[m];
     bh[M] = w->b_rew;
     bh[M + 1] = w->b_done;
-    if (NR == 4) {
+    if (c.reward_mode == WM_REWARD_SHAPED) {
         bh[M + 2] = w->b_rt;
         bh[M + 3] = w->b_mem;
     }
+    if (c.value_head) bh[M + NR - 1] = w->b_val;
     cudaError_t e;
     if ((e = upload(&h->step.Wg, Wg)) != cudaSuccess) return e;
     if ((e = upload(&h->step.Wa, Wa)) != cudaSuccess) return e;
@@ -255,13 +257,20 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
 
 // AUTO: the fused single-launch family for batches that fit one wave of clusters,
 // the tensor-core family for large bf16 batches, the stepwise family otherwise.
-int pick_path(const wm_handle *h, int B) {
+// fused_ok / tc_ok: whether this call's options allow those families.
+int pick_path(const wm_handle *h, int B, bool fused_ok = true, bool tc_ok = true) {
     const int p = h->cfg.path;
     if (p != WM_PATH_AUTO) return p;
-    if (wm_fused_supported(h, B) && B <= 2048) return WM_PATH_FUSED;
-    if (wm_tc_supported(h) && B >= 256) return WM_PATH_TENSOR;
-    if (wm_fused_supported(h, B)) return WM_PATH_FUSED;
+    const bool fu = fused_ok && wm_fused_supported(h, B), tc = tc_ok && wm_tc_supported(h);
+    if (fu && B <= 2048) return WM_PATH_FUSED;
+    if (tc && B >= 256) return WM_PATH_TENSOR;
+    if (fu) return WM_PATH_FUSED;
     return WM_PATH_STEPWISE;
+}
+
+template <class T>
+std::vector<T> host_vec(const T *p, size_t n) {
+    return p ? std::vector<T>(p, p + n) : std::vector<T>();
 }
 
 }  // namespace
@@ -276,11 +285,31 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) 
         !w->W_ctrl || !w->b_ctrl)
         return WM_ERR_INVALID_ARG;
     if (cfg->reward_mode == WM_REWARD_SHAPED && (!w->w_rt || !w->w_mem)) return WM_ERR_INVALID_ARG;
+    if (cfg->value_head && !w->w_val) return WM_ERR_INVALID_ARG;
     wm_handle *h = new (std::nothrow) wm_handle();
     if (!h) return WM_ERR_OOM;
     h->cfg = *cfg;
     h->M = 3 * cfg->k_mix * cfg->z_dim;
-    h->NR = cfg->reward_mode == WM_REWARD_SHAPED ? 4 : 2;
+    h->NR = 2 + (cfg->reward_mode == WM_REWARD_SHAPED ? 2 : 0) + (cfg->value_head ? 1 : 0);
+    {
+        const size_t Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, M = h->M;
+        wm_host_weights &hw = h->host;
+        hw.W_lstm = host_vec(w->W_lstm, (Z + A + H) * 4 * H);
+        hw.b_lstm = host_vec(w->b_lstm, 4 * H);
+        hw.W_mdn = host_vec(w->W_mdn, H * M);
+        hw.b_mdn = host_vec(w->b_mdn, M);
+        hw.w_rew = host_vec(w->w_rew, H);
+        hw.w_done = host_vec(w->w_done, H);
+        hw.W_ctrl = host_vec(w->W_ctrl, (Z + H) * A);
+        hw.b_ctrl = host_vec(w->b_ctrl, A);
+        if (cfg->reward_mode == WM_REWARD_SHAPED) {
+            hw.w_rt = host_vec(w->w_rt, H);
+            hw.w_mem = host_vec(w->w_mem, H);
+        }
+        if (cfg->value_head) hw.w_val = host_vec(w->w_val, H);
+        hw.b_rew = w->b_rew; hw.b_done = w->b_done; hw.b_rt = w->b_rt; hw.b_mem = w->b_mem;
+        hw.b_val = w->b_val;
+    }
     memset(&h->step, 0, sizeof(h->step));
     memset(&h->fused, 0, sizeof(h->fused));
     memset(&h->tc, 0, sizeof(h->tc));
@@ -312,6 +341,8 @@ void wm_destroy(wm_handle *h) {
     cudaFree(h->step.bg);
     cudaFree(h->step.Wh);
     cudaFree(h->step.bh);
+    cudaFree(h->step.Wp);
+    cudaFree(h->step.bp);
     wm_fused_free(h);
     wm_tc_free(h);
     cudaFree(h->ws);
@@ -465,6 +496,8 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     st.add((void **)&a.c_seq, io->c_seq, t * b * H * 4, true, STEP_OUT, b * H * 4);
     st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true, STEP_OUT, b * M * 4);
     st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true, STEP_OUT, b * Z);
+    st.add((void **)&a.logp_seq, io->logp_seq, t * b * 4, true, STEP_OUT, b * 4);
+    if (c.value_head) st.add((void **)&a.value_seq, io->value_seq, t * b * 4, true, STEP_OUT, b * 4);
     if (shaped) {
         st.add((void **)&a.rt0, io->rt0, b * 4, false);
         st.add((void **)&a.mem0, io->mem0, b * 4, false);
@@ -472,11 +505,15 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
         st.add((void **)&a.mem_seq, io->mem_seq, t * b * 4, true, STEP_OUT, b * 4);
     }
 
-    int path = pick_path(h, B);
-    if (path == WM_PATH_FUSED && !wm_fused_supported(h, B))
-        return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
-    if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
-        return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
+    // the fused family writes no log-probs or values and has one controller; the tensor
+    // family needs a population's candidates aligned to its 256-row tiles
+    const bool fused_ok = !io->logp_seq && !(c.value_head && io->value_seq) && h->P == 1;
+    const bool tc_ok = wm_tc_call_ok(h, episode_offset) != 0;
+    int path = pick_path(h, B, fused_ok, tc_ok);
+    if (path == WM_PATH_FUSED && !(fused_ok && wm_fused_supported(h, B)))
+        return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch / outputs");
+    if (path == WM_PATH_TENSOR && !(tc_ok && wm_tc_supported(h)))
+        return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model / call");
 
     size_t need = path == WM_PATH_STEPWISE ? wm_step_rollout_ws(h, B) : path == WM_PATH_TENSOR ? wm_tc_ws(h, B) : 0;
     if (need) {
@@ -495,7 +532,80 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     if (e != cudaSuccess) return cuda_fail(h, e, "rollout launch");
     h->last_path = path;
     if (path == WM_PATH_STEPWISE)
-        h->last_launches = B == 0 ? 0 : 1 + 4 * T + ((a.h_final || a.c_final) ? 1 : 0);
+        h->last_launches = B == 0 ? 0 : 1 + (h->P > 1 ? 5 : 4) * T + ((a.h_final || a.c_final) ? 1 : 0);
+    if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
+    return WM_OK;
+}
+
+wm_status wm_set_controllers(wm_handle *h, int P, int E, const float *W_ctrl, const float *b_ctrl) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->err.clear();
+    if (P < 1 || E < 1 || !W_ctrl || !b_ctrl) return fail(h, WM_ERR_INVALID_ARG, "P, E >= 1 and arrays required");
+    const wm_config &c = h->cfg;
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, KX = Z + H, N1 = 4 * H + A;
+    cudaError_t e = cudaSetDevice(h->device);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+    e = cudaDeviceSynchronize();  // earlier calls may still read the controller weights
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaDeviceSynchronize");
+    const bool rb = c.precision == WM_BF16;
+    auto wv = [&](float x) { return rb ? bf16_round_host(x) : x; };
+    // stepwise: candidate 0 in the controller columns of the combined GEMM matrix, and all
+    // candidates in Wp / bp when there is more than one
+    std::vector<float> w0(KX * A);
+    for (size_t i = 0; i < KX * A; ++i) w0[i] = wv(W_ctrl[i]);
+    e = cudaMemcpy2D(h->step.Wg + 4 * H, N1 * 4, w0.data(), A * 4, A * 4, KX, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(h->step.bg + 4 * H, b_ctrl, A * 4, cudaMemcpyHostToDevice);
+    cudaFree(h->step.Wp);
+    cudaFree(h->step.bp);
+    h->step.Wp = h->step.bp = nullptr;
+    if (e == cudaSuccess && P > 1) {
+        std::vector<float> wp((size_t)P * KX * A), bpv(b_ctrl, b_ctrl + (size_t)P * A);
+        for (size_t i = 0; i < wp.size(); ++i) wp[i] = wv(W_ctrl[i]);
+        e = upload(&h->step.Wp, wp);
+        if (e == cudaSuccess) e = upload(&h->step.bp, bpv);
+    }
+    if (e == cudaSuccess && h->tc.ok) e = wm_tc_set_controllers(h, P, W_ctrl, b_ctrl);
+    // the fused family packs the controller into its per-rank images: repack them
+    if (e == cudaSuccess && P == 1) {
+        h->host.W_ctrl.assign(W_ctrl, W_ctrl + KX * A);
+        h->host.b_ctrl.assign(b_ctrl, b_ctrl + A);
+        wm_fused_free(h);
+        const wm_weights hv = h->host.view();
+        e = wm_fused_pack(h, &hv);
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "wm_set_controllers");
+    h->P = P;
+    h->E = E;
+    return WM_OK;
+}
+
+wm_status wm_returns(wm_handle *h, int B, int T, unsigned long long episode_offset, float gamma,
+                     int stop_at_done, const float *rewards, const uint8_t *done, const float *bootstrap,
+                     float *returns, float *fitness, void *cuda_stream) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->err.clear();
+    if (B < 0 || T < 0 || B > (1 << 22)) return fail(h, WM_ERR_INVALID_ARG, "B must be in [0, 2^22], T >= 0");
+    if (B > 0 && T > 0 && (!rewards || !done || !returns))
+        return fail(h, WM_ERR_INVALID_ARG, "rewards, done and returns are required");
+    if (!(gamma >= 0.f && gamma <= 1.f)) return fail(h, WM_ERR_INVALID_ARG, "gamma must be in [0, 1]");
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    cudaError_t e = cudaSetDevice(h->device);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+    const size_t b = (size_t)B, t = (size_t)T;
+    const float *r = rewards, *bs = bootstrap;
+    const uint8_t *d = done;
+    float *ret = returns, *fit = fitness;
+    Stager st;
+    st.add((void **)&r, rewards, t * b * 4, false);
+    st.add((void **)&d, done, t * b, false);
+    st.add((void **)&bs, bootstrap, b * 4, false);
+    st.add((void **)&ret, returns, t * b * 4, true);
+    st.add((void **)&fit, fitness, (size_t)h->P * 4, true);
+    e = grow(&h->ws, &h->ws_bytes, wm_returns_ws(h, B));
+    if (e != cudaSuccess) return cuda_fail(h, e, "workspace");
+    if ((e = st.begin(h, T, false, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    e = wm_returns_launch(h, B, T, episode_offset, gamma, stop_at_done, r, d, bs, ret, fit, h->ws, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "returns launch");
     if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
     return WM_OK;
 }

@@ -37,6 +37,8 @@ struct wm_rollout_dev {
     uint8_t *comp_seq;
     const float *rt0, *mem0;   // shaped reward: predictions entering the call
     float *rt_seq, *mem_seq;   // shaped reward: predictions after each step (optional)
+    float *logp_seq;           // log-prob of the action taken (optional)
+    float *value_seq;          // value head V(h_{t+1}) (optional)
 };
 
 // Device pointers of one teacher-forced scoring call.
@@ -53,8 +55,10 @@ struct wm_step_weights {
     float *Wg;   // [Z+H, 4H+A]  rows z | h; cols gates i|f|g|o then controller
     float *Wa;   // [A, 4H]      action rows of the gate matrix
     float *bg;   // [4H+A]       gate bias then controller bias
-    float *Wh;   // [H, M+NR]    mixture head, reward, done (+ runtime, memory when shaped)
+    float *Wh;   // [H, M+NR]    mixture head, reward, done (+ runtime, memory) (+ value)
     float *bh;   // [M+NR]
+    float *Wp;   // [P, Z+H, A]  controller candidates (P > 1 only; else in Wg)
+    float *bp;   // [P, A]
 };
 
 // Weights of the fused single-launch family: per cluster size (slot 0: 16 CTAs,
@@ -69,7 +73,7 @@ struct wm_fused_weights {
 
 // Weights of the tensor-core family (bf16, K-major; orders in wm_tensor.cu).
 struct wm_tc_weights {
-    void *wc, *wg, *wa, *wh;  // W_c^T [A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
+    void *wc, *wg, *wa, *wh;  // W_c^T [P*A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
     float *bc, *bg, *bh;
     int dims_per_tile, n_head_tiles, rd_tile, rd_col;  // reward, done (, runtime, memory) columns
     int sms;
@@ -90,11 +94,30 @@ struct wm_timer {
     long long launches[WM_KERNEL_CLASSES] = {};
 };
 
+// A canonical host copy of the weights (the layouts of wm_weights).
+struct wm_host_weights {
+    std::vector<float> W_lstm, b_lstm, W_mdn, b_mdn, w_rew, w_done, W_ctrl, b_ctrl, w_rt, w_mem, w_val;
+    float b_rew = 0.f, b_done = 0.f, b_rt = 0.f, b_mem = 0.f, b_val = 0.f;
+    wm_weights view() const {
+        auto p = [](const std::vector<float> &v) { return v.empty() ? nullptr : v.data(); };
+        wm_weights w{};
+        w.W_lstm = p(W_lstm); w.b_lstm = p(b_lstm); w.W_mdn = p(W_mdn); w.b_mdn = p(b_mdn);
+        w.w_rew = p(w_rew); w.b_rew = b_rew; w.w_done = p(w_done); w.b_done = b_done;
+        w.W_ctrl = p(W_ctrl); w.b_ctrl = p(b_ctrl); w.w_rt = p(w_rt); w.b_rt = b_rt;
+        w.w_mem = p(w_mem); w.b_mem = b_mem; w.w_val = p(w_val); w.b_val = b_val;
+        return w;
+    }
+};
+
 struct wm_handle {
     wm_config cfg;
     int device;
     int M;                       // 3 K Z
-    int NR;                      // head columns after the mixture: reward, done (+ runtime, memory)
+    int NR;                      // head columns after the mixture: reward, done (+ runtime,
+                                 // memory when shaped) (+ value when value_head), in that order
+    int P = 1, E = 1;            // controller population: candidate of episode e = (e / E) mod P
+    wm_host_weights host;        // canonical host copy (repacks the fused family's images
+                                 // when the controller changes)
     wm_step_weights step;
     wm_fused_weights fused;
     wm_tc_weights tc;
@@ -134,6 +157,16 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w);
 void wm_tc_free(wm_handle *h);
 cudaError_t wm_tc_rollout(const wm_handle *h, const wm_rollout_dev &a, void *ws, cudaStream_t s);
 cudaError_t wm_tc_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s);
+cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, const float *b_ctrl);
+// whether the tensor family can run a rollout call starting at this episode (population tiles)
+int wm_tc_call_ok(const wm_handle *h, unsigned long long episode_offset);
+
+// ---- discounted returns (wm_returns.cu) ----------------------------------------
+cudaError_t wm_returns_launch(const wm_handle *h, int B, int T, unsigned long long ep0, float gamma,
+                              int stop_at_done, const float *rewards, const uint8_t *done,
+                              const float *bootstrap, float *returns, float *fitness, void *ws,
+                              cudaStream_t s);
+size_t wm_returns_ws(const wm_handle *h, int B);
 
 // ---- stepwise family (wm_step.cu) -------------------------------------------
 size_t wm_step_rollout_ws(const wm_handle *h, int B);

@@ -83,7 +83,8 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
                           io->rewards, io->done, io->h_final, io->c_final, io->h_seq, io->c_seq,
                           io->mdn_seq, io->comp_seq, shaped ? io->rt0 : nullptr,
                           shaped ? io->mem0 : nullptr, shaped ? io->rt_seq : nullptr,
-                          shaped ? io->mem_seq : nullptr};
+                          shaped ? io->mem_seq : nullptr, io->logp_seq,
+                          h->cfg.value_head ? io->value_seq : nullptr};
     for (const void *p : ptrs)
         if (!device_accessible(p))
             return fail(h, WM_ERR_INVALID_ARG,
@@ -103,9 +104,11 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
     if (shaped) {
         a.rt0 = io->rt0; a.mem0 = io->mem0; a.rt_seq = io->rt_seq; a.mem_seq = io->mem_seq;
     }
+    a.logp_seq = io->logp_seq;
+    a.value_seq = h->cfg.value_head ? io->value_seq : nullptr;
     e = wm_step_rollout(h, a, scratch, (cudaStream_t)cuda_stream);
     if (e != cudaSuccess) return fail(h, WM_ERR_CUDA, "wm_rollout_noalloc launch failed");
     h->last_path = WM_PATH_STEPWISE;
-    h->last_launches = B == 0 ? 0 : 1 + 4 * T + ((a.h_final || a.c_final) ? 1 : 0);
+    h->last_launches = B == 0 ? 0 : 1 + (h->P > 1 ? 5 : 4) * T + ((a.h_final || a.c_final) ? 1 : 0);
     return WM_OK;
 }

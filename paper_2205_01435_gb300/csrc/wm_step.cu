@@ -120,14 +120,55 @@ struct StepParams {
     float alpha, beta, invalid_reward;
     float *rt, *mem;
     float *rt_seq, *mem_seq;
+    // controller population: episode e acts with candidate (e / E) mod P (Wp, bp when P > 1)
+    int P, E;
+    const float *Wp, *bp;
+    float *logp_seq;      // log pi(a_t | z_t, h_t) of the action taken (optional)
+    float *value_seq;     // value head, heads column value_col (optional)
+    int value_col;
 };
 
 __device__ __forceinline__ bool action_valid(const uint32_t *mw, int j) {
     return !mw || ((mw[j >> 5] >> (j & 31)) & 1u);
 }
 
-// a2 on one warp: masked argmax (lowest index on ties) or a tempered draw.
-__device__ int select_action_warp(const StepParams &p, int b) {
+// a1 for a controller population: the logits of each episode's candidate into the
+// controller columns of G.  One block per episode, the input [z_t; h_t] staged in
+// shared memory (bf16-rounded on the bf16 path), one column per thread.
+template <bool ROUND>
+__global__ void __launch_bounds__(128) k_ctrl_pop(StepParams p, const float *__restrict__ z) {
+    extern __shared__ float xs[];
+    const int b = blockIdx.x, Z = p.Z, H = p.H, A = p.A, KX = Z + H;
+    for (int i = threadIdx.x; i < KX; i += blockDim.x) {
+        float v = i < Z ? z[(size_t)b * Z + i] : p.h[(size_t)b * H + (i - Z)];
+        xs[i] = ROUND ? round_bf16(v) : v;
+    }
+    __syncthreads();
+    const size_t cand = (size_t)(((p.ep0 + b) / (unsigned long long)p.E) % (unsigned long long)p.P);
+    const float *W = p.Wp + cand * KX * A, *bias = p.bp + cand * A;
+    float *out = const_cast<float *>(p.G) + (size_t)b * p.ldg + 4 * H;
+    for (int j = threadIdx.x; j < A; j += blockDim.x) {
+        float acc = 0.f;
+        for (int i = 0; i < KX; ++i) acc = fmaf(xs[i], W[(size_t)i * A + j], acc);
+        out[j] = acc + bias[j];
+    }
+}
+
+// log pi(a) under softmax(l / tau) over the valid actions (one warp; every lane returns it)
+__device__ float action_logp_warp(const StepParams &p, const float *l, const uint32_t *mw, int a, float lmax) {
+    const int lane = threadIdx.x & 31;
+    const float tau = p.ctrl_tau;
+    float S = 0.f;
+    for (int j = lane; j < p.A; j += 32)
+        if (action_valid(mw, j)) S += expf((l[j] - lmax) / tau);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
+    return (l[a] - lmax) / tau - logf(S);
+}
+
+// a2 on one warp: masked argmax (lowest index on ties) or a tempered draw.  With
+// p.logp_seq, *logp receives log pi(a) of the chosen action (0 if none or tau = 0).
+__device__ int select_action_warp(const StepParams &p, int b, float *logp) {
     const int lane = threadIdx.x & 31;
     const float *l = p.G + (long)b * p.ldg + 4 * p.H;
     const int A = p.A, W = (A + 31) >> 5;
@@ -146,7 +187,12 @@ __device__ int select_action_warp(const StepParams &p, int b) {
         bool take = oi >= 0 && (bi < 0 || ov > bv || (ov == bv && oi < bi));
         if (take) { bv = ov; bi = oi; }
     }
-    if (bi < 0 || !p.ctrl_sample || !(p.ctrl_tau > 0.f)) return bi;
+    *logp = 0.f;
+    if (bi < 0) return bi;
+    if (!p.ctrl_sample || !(p.ctrl_tau > 0.f)) {
+        if (p.logp_seq && p.ctrl_tau > 0.f) *logp = action_logp_warp(p, l, mw, bi, bv);
+        return bi;
+    }
 
     const float tau = p.ctrl_tau;
     float S = 0.f;
@@ -171,9 +217,14 @@ __device__ int select_action_warp(const StepParams &p, int b) {
         unsigned hit = __ballot_sync(0xffffffffu, ok && target < cum);
         unsigned okm = __ballot_sync(0xffffffffu, ok);
         if (okm) last = j0 + 31 - __clz(okm);
-        if (hit) return j0 + __ffs(hit) - 1;
+        if (hit) {
+            const int a = j0 + __ffs(hit) - 1;
+            if (p.logp_seq) *logp = (l[a] - bv) / tau - logf(S);
+            return a;
+        }
         run += __shfl_sync(0xffffffffu, sc, 31);
     }
+    if (p.logp_seq && last >= 0) *logp = (l[last] - bv) / tau - logf(S);
     return last;
 }
 
@@ -183,6 +234,7 @@ __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
     const bool fz = p.frozen[b] != 0;
     if (threadIdx.x < 32) {
         int a;
+        float lp = 0.f;
         if (fz) {
             a = -1;
         } else if (p.teacher) {
@@ -190,11 +242,12 @@ __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
             if (a >= p.A) report_status(p.status, WM_ERR_INVALID_ARG);
             if (a >= p.A || a < 0) a = -1;
         } else {
-            a = select_action_warp(p, b);
+            a = select_action_warp(p, b, &lp);
         }
         if (threadIdx.x == 0) {
             s_a = a;
             if (!p.teacher) p.act_out[(size_t)p.t * p.B + b] = a;
+            if (!p.teacher && p.logp_seq) p.logp_seq[(size_t)p.t * p.B + b] = lp;
         }
     }
     __syncthreads();
@@ -347,6 +400,7 @@ __global__ void __launch_bounds__(128) k_sample(StepParams p) {
         }
         if (shaped && p.rt_seq) p.rt_seq[tb] = p.rt[b];
         if (shaped && p.mem_seq) p.mem_seq[tb] = p.mem[b];
+        if (p.value_seq) p.value_seq[tb] = fz ? 0.f : row[p.value_col];
     }
 }
 
@@ -456,6 +510,9 @@ StepParams base_params(const wm_handle *hd, int B, int T, const StepWs &w) {
     p.reward_mode = c.reward_mode;
     p.alpha = c.reward_alpha; p.beta = c.reward_beta; p.invalid_reward = c.invalid_reward;
     p.rt = w.rt; p.mem = w.mem;
+    p.P = hd->P; p.E = hd->E;
+    p.Wp = hd->step.Wp; p.bp = hd->step.bp;
+    p.value_col = hd->M + hd->NR - 1;
     return p;
 }
 
@@ -486,14 +543,23 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
     p.h_seq = a.h_seq; p.c_seq = a.c_seq;
     p.rewards = a.rewards; p.done = a.done; p.mdn_seq = a.mdn_seq; p.comp_seq = a.comp_seq;
     p.rt_seq = a.rt_seq; p.mem_seq = a.mem_seq;
+    p.logp_seq = a.logp_seq;
+    p.value_seq = c.value_head ? a.value_seq : nullptr;
     const int NH = hd->M + hd->NR;  // head GEMM columns
+    const bool pop = hd->P > 1;     // controller logits per candidate, in k_ctrl_pop
     for (int t = 0; t < T; ++t) {
         p.t = t;
         p.step = a.t0 + (uint32_t)t;
         p.z_cur = a.z_out + (size_t)t * B * Z;
         p.z_next = a.z_out + (size_t)(t + 1) * B * Z;
-        launch_gemm(hd, round, B, 4 * H + A, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A, hd->step.bg,
-                    w.G, 4L * H + A, s);
+        launch_gemm(hd, round, B, pop ? 4 * H : 4 * H + A, Z, H, p.z_cur, Z, w.h, H, hd->step.Wg, 4L * H + A,
+                    hd->step.bg, w.G, 4L * H + A, s);
+        if (pop) {
+            wm_ktime kt(hd, WM_KERNEL_STEP_GEMM, s);
+            const size_t sm = (size_t)(Z + H) * 4;
+            if (round) k_ctrl_pop<true><<<B, 128, sm, s>>>(p, p.z_cur);
+            else k_ctrl_pop<false><<<B, 128, sm, s>>>(p, p.z_cur);
+        }
         {
             wm_ktime kt(hd, WM_KERNEL_STEP_CELL, s);
             k_select_cell<<<B, 256, 0, s>>>(p);

@@ -126,6 +126,10 @@ struct GemmGrid {
     int m_tiles, n_tiles, k_steps;
     int a_col0;   // first K column of A (the heads read X from column Z)
     int *status;
+    // B-operand rows per 256-row tile (controller population): tile m reads the B rows of
+    // candidate ((ep0 + 256 m) / pop_E) mod pop_P, which start at row candidate * pop_rows
+    unsigned long long ep0;
+    int pop_P, pop_E, pop_rows;
 };
 
 // ---------------------------------------------------------------------------
@@ -166,6 +170,12 @@ struct StepIO {
     float alpha, beta, invalid_reward;
     const float *rt0, *mem0;
     float *rt, *mem, *rt_seq, *mem_seq;
+    // controller population: episode e acts with candidate (e / pop_E) mod pop_P; b_ctrl is
+    // [pop_P, A] (a 256-row tile belongs to one candidate)
+    int pop_P, pop_E;
+    float *logp_seq;                // log pi(a_t | z_t, h_t) of the action taken (optional)
+    float *value_seq;               // value head at head column rd_col + nr - 1 (optional)
+    int nr;                         // head columns from rd_col: reward, done (, rt, mem) (, value)
 };
 
 // Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
@@ -217,14 +227,17 @@ struct EpiCtrl {
     static constexpr uint32_t QUAD_STAGE = 0;
     static constexpr int MAX_A = 512, NCH = MAX_A / 4 / 16;  // chunks per column group, at most
     static constexpr uint32_t RED_FLOATS = 4 * 4 * 32 * 2;
-    static constexpr uint32_t RED_BYTES = (RED_FLOATS + MAX_A) * 4;  // reductions | bias
+    // reductions | the bias, one copy per lane quadrant (a population's tiles change it)
+    static constexpr uint32_t RED_BYTES = (RED_FLOATS + 4 * MAX_A) * 4;
     struct Pre {
         uint32_t bits[NCH];  // the chunk's 16 mask bits (0 for rows that do not act)
         bool live;           // a row of the batch whose episode is not frozen
     };
-    // once per CTA, by all 512 epilogue threads (e = 0..511), before the first tile
+    // once per CTA, by all 512 epilogue threads (e = 0..511), before the first tile: the
+    // bias of a single controller into every quadrant's copy
     static __device__ void init(const StepIO &p, EpiCtx &x, int e) {
-        for (int i = e; i < p.A; i += 32 * EPI_WARPS) x.red[RED_FLOATS + i] = p.b_ctrl[i];
+        if (p.pop_P > 1) return;
+        for (int i = e; i < 4 * p.A; i += 32 * EPI_WARPS) x.red[RED_FLOATS + (i / p.A) * MAX_A + i % p.A] = p.b_ctrl[i % p.A];
     }
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
     static __device__ void pre(const StepIO &p, int m, int, EpiCtx &x, Pre &q) {
@@ -236,6 +249,14 @@ struct EpiCtrl {
         for (int k = 0; k < NCH; ++k) {
             const int c0 = c_lo + 16 * k;
             q.bits[k] = (!q.live || 16 * k >= CW) ? 0u : mw ? (mw[c0 >> 5] >> (c0 & 31)) & 0xFFFFu : 0xFFFFu;
+        }
+        if (p.pop_P > 1) {  // the tile's candidate's bias into the quadrant's copy (the previous
+                            // tile's readers are past its closing barrier)
+            const unsigned long long cand = ((p.ep0 + (unsigned long long)m * BM) / (unsigned long long)p.pop_E) %
+                                            (unsigned long long)p.pop_P;
+            const float *bc = p.b_ctrl + cand * p.A;
+            float *bq = x.red + RED_FLOATS + x.quad * MAX_A;
+            for (int i = x.cg * 32 + x.lane; i < A; i += 128) bq[i] = bc[i];
         }
     }
     // logits of chunk k (accumulator + bias)
@@ -267,7 +288,8 @@ struct EpiCtrl {
         const int b = m * BM + x.row;
         const bool valid = b < p.B, live = q.live;
         const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
-        const float *bs = x.red + RED_FLOATS;
+        const float *bs = x.red + RED_FLOATS + x.quad * MAX_A;
+        if (p.pop_P > 1) x.sync();  // the quadrant's bias copy (pre) is complete
         // pass 1: masked argmax over this group's columns (lowest index on ties): per chunk,
         // the maximum of the valid logits, then the lowest valid column that attains it
         int a = -1, last_v = -1;
@@ -306,7 +328,10 @@ struct EpiCtrl {
             const int i = __float_as_int(o[1]);
             if (i >= 0 && (ga < 0 || o[0] > gbv)) { gbv = o[0]; ga = i; }
         }
-        if (p.ctrl_sample && p.ctrl_tau > 0.f) {  // uniform over the warp
+        const bool sampled = p.ctrl_sample && p.ctrl_tau > 0.f;         // uniform over the warp
+        const bool want_lp = p.logp_seq != nullptr && p.ctrl_tau > 0.f;  // log pi(a) requested
+        float logp = 0.f;
+        if (sampled || want_lp) {
             const bool draw = live && ga >= 0;
             // weight of logit v: exp((v - max) / tau) = 2^(v * s - max * s), s = log2(e) / tau;
             // a masked column's weight is forced to +0 (its logit may exceed the maximum)
@@ -339,61 +364,83 @@ struct EpiCtrl {
                 total += o[0];
                 glast = max(glast, __float_as_int(o[1]));
             }
-            const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x) : 0.f;
-            const float target = u * total;
-            const bool mine = draw && target >= prefix && target < prefix + S;
-            // the chunk holding the drawn point (the group's last chunk with a valid
-            // action if rounding carries the running sum past the target)
-            int kc = -1, klast = -1;
-            float base = prefix;
+            const float itau = 1.f / p.ctrl_tau, log_total = logf(total);
+            if (!sampled) {
+                logp = draw ? -log_total : 0.f;  // the argmax: its logit is the maximum
+            } else {
+                const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x) : 0.f;
+                const float target = u * total;
+                // the group holding the drawn point; if rounding puts the target at or past the
+                // total, the group holding the last valid action
+                const bool mine = draw && ((target >= prefix && target < prefix + S) ||
+                                           (target >= total && last_v == glast));
+                // the chunk holding the drawn point (the group's last chunk with a valid
+                // action if rounding carries the running sum past the target)
+                int kc = -1, klast = -1;
+                float base = prefix;
 #pragma unroll
-            for (int k = 0; k < NCH; ++k) {
-                if (k >= nch || !mine) continue;
-                if (q.bits[k]) klast = k;
-                if (kc < 0) {
-                    if (target < base + cs[k]) kc = k;
-                    else base += cs[k];
+                for (int k = 0; k < NCH; ++k) {
+                    if (k >= nch || !mine) continue;
+                    if (q.bits[k]) klast = k;
+                    if (kc < 0) {
+                        if (target < base + cs[k]) kc = k;
+                        else base += cs[k];
+                    }
+                }
+                if (mine && kc < 0) {
+                    kc = klast;
+                    base = prefix;
+                    for (int k = 0; k < NCH; ++k)
+                        if (k < klast) base += cs[k];
+                }
+                // pass 3: only chunks some row of the warp needs
+                int chosen = -1;
+                float lv = 0.f;  // the chosen column's logit
+#pragma unroll
+                for (int k = 0; k < NCH; ++k) {
+                    if (k >= nch) break;
+                    if (!__any_sync(0xffffffffu, kc == k)) continue;
+                    float v[16];
+                    chunk(tacc, bs, c_lo + 16 * k, v);
+                    if (kc != k) continue;
+                    const uint32_t bits = q.bits[k];
+                    float cum = base;
+                    uint32_t hit = 0u;  // valid columns at which the running sum has passed the target
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        cum += __uint_as_float(__float_as_uint(ex2_approx(fmaf(v[j], sc, off))) & lane_mask(bits, j));
+                        hit |= (target < cum ? 1u : 0u) << j;
+                    }
+                    hit &= bits;
+                    // the first such column; rounding: the chunk's last valid action
+                    const int jj = hit ? __ffs(hit) - 1 : (bits ? 31 - __clz(bits) : -1);
+                    chosen = jj >= 0 ? c_lo + 16 * k + jj : -1;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) lv = j == jj ? v[j] : lv;
+                }
+                x.sync();  // everyone has read the sum partials
+                my[0] = lv;
+                my[1] = __int_as_float(chosen);
+                x.sync();
+                int pick = -1;
+                float lvp = 0.f;
+                for (int g = 0; g < 4; ++g) {
+                    const int c = __float_as_int(x.slot(g)[1]);
+                    if (c > pick) { pick = c; lvp = x.slot(g)[0]; }
+                }
+                if (draw) {
+                    ga = pick >= 0 ? pick : glast;  // rounding past the last valid action
+                    logp = pick >= 0 ? (lvp - gbv) * itau - log_total : 0.f;
                 }
             }
-            if (mine && kc < 0) {
-                kc = klast;
-                base = prefix;
-                for (int k = 0; k < NCH; ++k)
-                    if (k < klast) base += cs[k];
-            }
-            // pass 3: only chunks some row of the warp needs
-            int chosen = -1;
-#pragma unroll
-            for (int k = 0; k < NCH; ++k) {
-                if (k >= nch) break;
-                if (!__any_sync(0xffffffffu, kc == k)) continue;
-                float v[16];
-                chunk(tacc, bs, c_lo + 16 * k, v);
-                if (kc != k) continue;
-                const uint32_t bits = q.bits[k];
-                float cum = base;
-                uint32_t hit = 0u;  // valid columns at which the running sum has passed the target
-#pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    cum += __uint_as_float(__float_as_uint(ex2_approx(fmaf(v[j], sc, off))) & lane_mask(bits, j));
-                    hit |= (target < cum ? 1u : 0u) << j;
-                }
-                hit &= bits;
-                // the first such column; rounding: the chunk's last valid action
-                chosen = hit ? c_lo + 16 * k + __ffs(hit) - 1 : (bits ? c_lo + 16 * k + 31 - __clz(bits) : -1);
-            }
-            x.sync();  // everyone has read the sum partials
-            my[1] = __int_as_float(chosen);
-            x.sync();
-            int pick = -1;
-            for (int g = 0; g < 4; ++g) pick = max(pick, __float_as_int(x.slot(g)[1]));
-            if (draw) ga = pick >= 0 ? pick : glast;  // rounding past the last valid action
         }
         x.sync();  // the scratch is reused by the next tile
         if (!valid || x.cg != 0) return;
         if (!live) ga = -1;
         p.act[b] = ga;
-        p.actions[(size_t)p.t * p.B + b] = ga;
+        const size_t tb = (size_t)p.t * p.B + b;
+        p.actions[tb] = ga;
+        if (p.logp_seq) p.logp_seq[tb] = ga >= 0 ? logp : 0.f;
     }
 };
 
@@ -785,7 +832,12 @@ struct EpiHeads {
             if (shaped)
                 asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
                              : "=r"(q[0]), "=r"(q[1]) : "r"(tacc + p.rd_col + 2));
+            uint32_t vr = 0u;
+            if (p.value_seq)  // uniform
+                asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];"
+                             : "=r"(vr) : "r"(tacc + p.rd_col + p.nr - 1));
             tc::tmem_ld_wait();
+            const float vq = __uint_as_float(vr);
             if (!p.teacher && valid && x.cg == 0) {
                 float rew = __uint_as_float(r[0]) + bh[p.rd_col];
                 const float dl = __uint_as_float(r[1]) + bh[p.rd_col + 1];
@@ -802,6 +854,7 @@ struct EpiHeads {
                     if (p.rt_seq) p.rt_seq[tb] = p.rt[b];
                     if (p.mem_seq) p.mem_seq[tb] = p.mem[b];
                 }
+                if (p.value_seq) p.value_seq[tb] = fz ? 0.f : vq + bh[p.rd_col + p.nr - 1];
                 p.rewards[tb] = fz ? 0.f : rew;
                 p.done[tb] = (fz || dl > 0.f || noop) ? 1 : 0;
                 p.fz_next[b] = (fz || (p.done_terminates && dl > 0.f) || noop) ? 1 : 0;
@@ -887,6 +940,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             uint32_t phase = 0;
             for (int tile = pair; tile < ntiles; tile += npairs) {
                 const int m = tile / g.n_tiles, n = tile % g.n_tiles;
+                const int brow = g.pop_P > 1 ? (int)(((g.ep0 + (unsigned long long)m * (2 * BM)) /
+                                                      (unsigned long long)g.pop_E) % (unsigned long long)g.pop_P) * g.pop_rows
+                                             : 0;
                 for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
                     const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;  // k-steps in this stage
                     const uint32_t full_ldr = tc::map_rank(full_b(stage), 0);
@@ -899,8 +955,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                         tma_load_2sm(sa, &tmA, g.a_col0 + ks * BK, (2 * m + (int)rank) * BM, full_ldr);
 #pragma unroll
                         for (int s = 0; s < NSUB; ++s)
-                            tma_load_2sm(sa + A_BYTES + s * B_SUB, &tmB, ks * BK, n * TILE_N + s * BN + (int)rank * BNH,
-                                         full_ldr);
+                            tma_load_2sm(sa + A_BYTES + s * B_SUB, &tmB, ks * BK,
+                                         brow + n * TILE_N + s * BN + (int)rank * BNH, full_ldr);
                     }
                     if (s_abort) break;
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -1230,13 +1286,17 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         }
         bh[rr] = w->b_rew;
         bh[rr + 1] = w->b_done;
-        if (h->NR == 4) {
+        if (c.reward_mode == WM_REWARD_SHAPED) {
             for (int i = 0; i < H; ++i) {
                 wh[(rr + 2) * H + i] = bf(w->w_rt[i]);
                 wh[(rr + 3) * H + i] = bf(w->w_mem[i]);
             }
             bh[rr + 2] = w->b_rt;
             bh[rr + 3] = w->b_mem;
+        }
+        if (c.value_head) {
+            for (int i = 0; i < H; ++i) wh[(rr + h->NR - 1) * H + i] = bf(w->w_val[i]);
+            bh[rr + h->NR - 1] = w->b_val;
         }
     }
     cudaError_t e;
@@ -1257,6 +1317,31 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
     cudaDeviceGetAttribute(&T.sms, cudaDevAttrMultiProcessorCount, dev);
     T.ok = 1;
     return cudaSuccess;
+}
+
+int wm_tc_call_ok(const wm_handle *h, unsigned long long episode_offset) {
+    // a 256-row tile must not straddle two candidates of a population
+    return h->P <= 1 || (h->E % 256 == 0 && episode_offset % 256 == 0);
+}
+
+cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, const float *b_ctrl) {
+    wm_tc_weights &T = h->tc;
+    const wm_config &c = h->cfg;
+    const int A = c.a_dim, KX = c.z_dim + c.h_dim;
+    std::vector<__nv_bfloat16> wc((size_t)P * A * KX);
+    for (int g = 0; g < P; ++g)
+        for (int a = 0; a < A; ++a)
+            for (int k = 0; k < KX; ++k)
+                wc[((size_t)g * A + a) * KX + k] = __float2bfloat16_rn(W_ctrl[((size_t)g * KX + k) * A + a]);
+    cudaFree(T.wc);
+    cudaFree(T.bc);
+    T.wc = nullptr;
+    T.bc = nullptr;
+    cudaError_t e = cudaMalloc(&T.wc, wc.size() * 2);
+    if (e == cudaSuccess) e = cudaMemcpy(T.wc, wc.data(), wc.size() * 2, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMalloc((void **)&T.bc, (size_t)P * A * 4);
+    if (e == cudaSuccess) e = cudaMemcpy(T.bc, b_ctrl, (size_t)P * A * 4, cudaMemcpyHostToDevice);
+    return e;
 }
 
 void wm_tc_free(wm_handle *h) {
@@ -1295,6 +1380,12 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     if (!teacher && c.reward_mode == WM_REWARD_SHAPED) {
         io.rt0 = ra->rt0; io.mem0 = ra->mem0; io.rt_seq = ra->rt_seq; io.mem_seq = ra->mem_seq;
     }
+    io.pop_P = h->P; io.pop_E = h->E;
+    io.nr = h->NR;
+    if (!teacher) {
+        io.logp_seq = ra->logp_seq;
+        io.value_seq = c.value_head ? ra->value_seq : nullptr;
+    }
     if (teacher) {
         io.act_in = na->actions; io.z_seq = na->z_seq; io.lengths = na->lengths;
         io.h_seq = na->h_seq; io.c_seq = na->c_seq; io.mdn_seq = na->mdn_seq;
@@ -1326,7 +1417,7 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     if (!make_map(&mx[0], w.x[0], B, KX, BM) || !make_map(&mx[1], w.x[1], B, KX, BM) ||
         !make_map(&mxs[0], w.x[0], B, KX, 32) || !make_map(&mxs[1], w.x[1], B, KX, 32) ||
         !make_map(&mc, w.c, B, H, 32, true) ||
-        !make_map(&mwc, T.wc, A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 128) ||
+        !make_map(&mwc, T.wc, (uint64_t)h->P * A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 128) ||
         !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE / 2))
         return cudaErrorInvalidValue;
     const int m_tiles = (B + 2 * BM - 1) / (2 * BM);  // 256-row tiles, one per CTA pair
@@ -1341,7 +1432,8 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         io.x_next = w.x[(t + 1) & 1];
         io.fz_cur = w.fz[t & 1];
         io.fz_next = w.fz[(t + 1) & 1];
-        const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status};
+        // the controller's weight rows: the tile's candidate's, when there is a population
+        const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status, teacher ? 0ull : ra->ep0, h->P, h->E, A};
         if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
         if (!teacher) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);

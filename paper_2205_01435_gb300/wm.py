@@ -6,7 +6,7 @@ no CPU fallback: if ``libwm.so`` is missing, importing the binding fails.
 
 Names mirror the C entry points: ``wm_create``, ``wm_rollout``, ``wm_mdn_nll``,
 ``wm_sync``, ``wm_destroy``, ``wm_last_error``, ``wm_last_path``, ``wm_last_launches``,
-``wm_set_timing``, ``wm_kernel_time``.  The
+``wm_set_timing``, ``wm_kernel_time``, ``wm_set_controllers``, ``wm_returns``.  The
 ``WorldModel`` class wraps them for convenience.
 """
 from __future__ import annotations
@@ -38,7 +38,7 @@ class wm_config(C.Structure):
                 ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_float), ("done_terminates", C.c_int),
                 ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int),
                 ("fused_cluster", C.c_int), ("reward_mode", C.c_int), ("reward_alpha", C.c_float),
-                ("reward_beta", C.c_float), ("invalid_reward", C.c_float)]
+                ("reward_beta", C.c_float), ("invalid_reward", C.c_float), ("value_head", C.c_int)]
 
 
 class wm_weights(C.Structure):
@@ -46,13 +46,15 @@ class wm_weights(C.Structure):
                 ("b_mdn", C.c_void_p), ("w_rew", C.c_void_p), ("b_rew", C.c_float),
                 ("w_done", C.c_void_p), ("b_done", C.c_float), ("W_ctrl", C.c_void_p),
                 ("b_ctrl", C.c_void_p), ("w_rt", C.c_void_p), ("b_rt", C.c_float),
-                ("w_mem", C.c_void_p), ("b_mem", C.c_float)]
+                ("w_mem", C.c_void_p), ("b_mem", C.c_float), ("w_val", C.c_void_p),
+                ("b_val", C.c_float)]
 
 
 class wm_rollout_io(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "z0", "h0", "c0", "done0", "mask", "z_out", "actions", "rewards", "done", "h_final",
-        "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq", "rt0", "mem0", "rt_seq", "mem_seq")]
+        "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq", "rt0", "mem0", "rt_seq", "mem_seq",
+        "logp_seq", "value_seq")]
 
 
 def _load():
@@ -69,6 +71,10 @@ def _load():
     lib.wm_rollout_noalloc.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_uint,
                                        C.POINTER(wm_rollout_io), P]
     lib.wm_rollout_noalloc.restype = C.c_int
+    lib.wm_set_controllers.argtypes = [P, C.c_int, C.c_int, P, P]
+    lib.wm_set_controllers.restype = C.c_int
+    lib.wm_returns.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_float, C.c_int, P, P, P, P, P, P]
+    lib.wm_returns.restype = C.c_int
     lib.wm_mdn_nll.argtypes = [P, C.c_int, C.c_int] + [P] * 7 + [P]
     lib.wm_mdn_nll.restype = C.c_int
     lib.wm_sync.argtypes = [P]
@@ -123,15 +129,17 @@ def wm_create(cfg: dict, weights: dict):
                   PATHS[cfg.get("path", "auto")] if isinstance(cfg.get("path", "auto"), str)
                   else int(cfg["path"]), int(cfg.get("fused_cluster", 0)),
                   int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
-                  float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)))
+                  float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)),
+                  int(cfg.get("value_head", 0)))
     keep = {k: torch.as_tensor(weights[k], dtype=torch.float32).contiguous().cpu()
             for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl",
-                      "w_rt", "w_mem") if weights.get(k) is not None}
+                      "w_rt", "w_mem", "w_val") if weights.get(k) is not None}
     w = wm_weights(_ptr(keep["W_lstm"]), _ptr(keep["b_lstm"]), _ptr(keep["W_mdn"]),
                    _ptr(keep["b_mdn"]), _ptr(keep["w_rew"]), float(weights["b_rew"]),
                    _ptr(keep["w_done"]), float(weights["b_done"]), _ptr(keep["W_ctrl"]),
                    _ptr(keep["b_ctrl"]), _ptr(keep.get("w_rt")), float(weights.get("b_rt", 0.0)),
-                   _ptr(keep.get("w_mem")), float(weights.get("b_mem", 0.0)))
+                   _ptr(keep.get("w_mem")), float(weights.get("b_mem", 0.0)), _ptr(keep.get("w_val")),
+                   float(weights.get("b_val", 0.0)))
     h = C.c_void_p()
     st = _lib.wm_create(C.byref(c), C.byref(w), C.byref(h))
     if st != WM_OK:
@@ -158,6 +166,21 @@ def wm_mdn_nll(h, N: int, T: int, z_seq, actions, lengths, nll, h_seq=None, c_se
     _check(h, _lib.wm_mdn_nll(h, N, T, _ptr(z_seq), _ptr(actions), _ptr(lengths), _ptr(nll),
                               _ptr(h_seq), _ptr(c_seq), _ptr(mdn_seq), C.c_void_p(stream)),
            "wm_mdn_nll")
+
+
+def wm_set_controllers(h, W_ctrl, b_ctrl, pop_group: int):
+    """wm_set_controllers: P = W_ctrl.shape[0] candidates (host fp32 [P, Z+H, A], [P, A])."""
+    W = torch.as_tensor(W_ctrl, dtype=torch.float32).contiguous().cpu()
+    b = torch.as_tensor(b_ctrl, dtype=torch.float32).contiguous().cpu()
+    _check(h, _lib.wm_set_controllers(h, int(W.shape[0]), int(pop_group), _ptr(W), _ptr(b)),
+           "wm_set_controllers")
+
+
+def wm_returns(h, B: int, T: int, episode_offset: int, gamma: float, stop_at_done: bool, rewards,
+               done, bootstrap, returns, fitness=None, stream: int = 0):
+    _check(h, _lib.wm_returns(h, B, T, episode_offset, float(gamma), int(bool(stop_at_done)),
+                              _ptr(rewards), _ptr(done), _ptr(bootstrap), _ptr(returns),
+                              _ptr(fitness), C.c_void_p(stream)), "wm_returns")
 
 
 def wm_sync(h):
@@ -225,9 +248,10 @@ class WorldModel:
     def rollout(self, z0: torch.Tensor, T: int, mask: torch.Tensor | None = None,
                 episode_offset: int = 0, t0: int = 0, h0=None, c0=None, done0=None,
                 want_final: bool = True, want_seq: bool = False, out: dict | None = None,
-                stream=None, rt0=None, mem0=None) -> dict:
+                stream=None, rt0=None, mem0=None, want_logp: bool = False) -> dict:
         """wm_rollout on B = z0.shape[0] episodes; returns the output tensors (device of z0).
-        With the shaped reward, rt0 / mem0 are required and rt_seq / mem_seq are returned."""
+        With the shaped reward, rt0 / mem0 are required and rt_seq / mem_seq are returned;
+        want_logp adds logp_seq, and a value head adds value_seq."""
         B = int(z0.shape[0])
         o = dict(out or {})
         for name, shape, dt in (("z", (T + 1, B, self.Z), torch.float32),
@@ -248,11 +272,16 @@ class WorldModel:
         if int(self.cfg.get("reward_mode", 0)) == 1:
             o.setdefault("rt_seq", self._alloc(z0, (T, B), torch.float32))
             o.setdefault("mem_seq", self._alloc(z0, (T, B), torch.float32))
+        if want_logp:
+            o.setdefault("logp_seq", self._alloc(z0, (T, B), torch.float32))
+        if int(self.cfg.get("value_head", 0)):
+            o.setdefault("value_seq", self._alloc(z0, (T, B), torch.float32))
         io = {"z0": z0, "h0": h0, "c0": c0, "done0": done0, "mask": mask, "z_out": o["z"],
               "actions": o["actions"], "rewards": o["rewards"], "done": o["done"],
               "h_final": o.get("h_final"), "c_final": o.get("c_final"), "h_seq": o.get("h_seq"),
               "c_seq": o.get("c_seq"), "mdn_seq": o.get("mdn_seq"), "comp_seq": o.get("comp_seq"),
-              "rt0": rt0, "mem0": mem0, "rt_seq": o.get("rt_seq"), "mem_seq": o.get("mem_seq")}
+              "rt0": rt0, "mem0": mem0, "rt_seq": o.get("rt_seq"), "mem_seq": o.get("mem_seq"),
+              "logp_seq": o.get("logp_seq"), "value_seq": o.get("value_seq")}
         with torch.cuda.device(self.device):
             wm_rollout(self.h, B, T, episode_offset, t0, io, self._stream(stream))
         return o
@@ -269,6 +298,26 @@ class WorldModel:
         with torch.cuda.device(self.device):
             wm_mdn_nll(self.h, N, T, z_seq, actions, lengths, o["nll"], o.get("h_seq"),
                        o.get("c_seq"), o.get("mdn_seq"), self._stream(stream))
+        return o
+
+    def set_controllers(self, W_ctrl, b_ctrl, pop_group: int = 1):
+        """A population of W_ctrl.shape[0] controllers; episode e acts with candidate
+        (e / pop_group) mod P."""
+        with torch.cuda.device(self.device):
+            wm_set_controllers(self.h, W_ctrl, b_ctrl, pop_group)
+        self.P = int(torch.as_tensor(W_ctrl).shape[0])
+
+    def returns(self, rewards: torch.Tensor, done: torch.Tensor, gamma: float,
+                stop_at_done: bool = True, bootstrap=None, episode_offset: int = 0,
+                want_fitness: bool = False, stream=None) -> dict:
+        """wm_returns: discounted returns [T, B] (and each candidate's mean G_0)."""
+        T, B = int(rewards.shape[0]), int(rewards.shape[1])
+        o = {"returns": self._alloc(rewards, (T, B), torch.float32)}
+        if want_fitness:
+            o["fitness"] = self._alloc(rewards, (getattr(self, "P", 1),), torch.float32)
+        with torch.cuda.device(self.device):
+            wm_returns(self.h, B, T, episode_offset, gamma, stop_at_done, rewards, done, bootstrap,
+                       o["returns"], o.get("fitness"), self._stream(stream))
         return o
 
     def sync(self):

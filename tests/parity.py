@@ -75,6 +75,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
     c = np.zeros((B, H), np.float32) if c0 is None else np.asarray(c0, np.float32)
     frozen = np.zeros(B, bool) if done0 is None else np.asarray(done0).astype(bool)
     shaped = int(cfg.get("reward_mode", 0)) == 1
+    g_lp = np_(g["logp_seq"]) if g.get("logp_seq") is not None else None
+    g_v = np_(g["value_seq"]) if g.get("value_seq") is not None else None
     if shaped:
         rt, mem = np.asarray(rt0, np.float32), np.asarray(mem0, np.float32)
         g_rt, g_mem = np_(g["rt_seq"]), np_(g["mem_seq"])
@@ -105,6 +107,10 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                     ("reward", gr[t], s["reward"]), ("z", gz[t + 1], s["z_next"])]
             if shaped:
                 vals += [("rt", g_rt[t], s["rt"]), ("mem", g_mem[t], s["mem"])]
+            if g_lp is not None:
+                vals.append(("logp", g_lp[t], s["logp"]))
+            if g_v is not None:
+                vals.append(("value", g_v[t], s["value"]))
             for key, gv, ov in vals:
                 e = np.abs(gv.astype(np.float64) - ov.astype(np.float64))
                 e = e.reshape(B, -1).max(axis=1) if e.ndim > 1 else e
@@ -125,6 +131,10 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                 assert np.all(gm[t, fz] == 0), where
                 if shaped:
                     assert np.array_equal(g_rt[t, fz], rt[fz]) and np.array_equal(g_mem[t, fz], mem[fz]), where
+                if g_lp is not None:
+                    assert np.all(g_lp[t, fz] == 0), where
+                if g_v is not None:
+                    assert np.all(g_v[t, fz] == 0), where
                 st["frozen_steps"] += len(fz)
             # decisions: equal, or excused by the oracle's own margin
             nl = int(live.sum())

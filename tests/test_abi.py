@@ -39,7 +39,8 @@ def test_binding_loads_and_mirrors_names():
     import paper_2205_01435_gb300 as pkg
     wm = pkg.load()
     for n in ("wm_create", "wm_rollout", "wm_mdn_nll", "wm_sync", "wm_destroy", "wm_last_path",
-              "wm_last_launches", "wm_rollout_noalloc", "wm_set_timing", "wm_kernel_time"):
+              "wm_last_launches", "wm_rollout_noalloc", "wm_set_timing", "wm_kernel_time",
+              "wm_set_controllers", "wm_returns"):
         assert callable(getattr(wm, n))
 
 
@@ -60,7 +61,8 @@ def test_invalid_config_rejected_on_host():
     cfg = synth.model_config("tiny_fp32")
     w = synth.weights(cfg)
     for bad in (dict(z_dim=0), dict(k_mix=0), dict(k_mix=33), dict(mdn_tau=-1.0),
-                dict(ctrl_tau=-0.5), dict(h_dim=-4), dict(precision_code=7)):
+                dict(ctrl_tau=-0.5), dict(h_dim=-4), dict(precision_code=7), dict(reward_mode=5),
+                dict(reward_mode=1, w_missing="w_rt"), dict(value_head=1, w_missing="w_val")):
         c = dict(cfg)
         if "precision_code" in bad:
             c["precision"] = "fp8"
@@ -75,9 +77,12 @@ def test_invalid_config_rejected_on_host():
                                keep["b_ctrl"].ctypes.data)
             assert wm._lib.wm_create(C.byref(c2), C.byref(ws), C.byref(h)) == wm.WM_ERR_INVALID_ARG
             continue
+        ww = dict(w)
+        if "w_missing" in bad:
+            ww[bad.pop("w_missing")] = None
         c.update(bad)
         with pytest.raises(wm.WMError) as ei:
-            wm.wm_create(c, w)
+            wm.wm_create(c, ww)
         assert ei.value.status == wm.WM_ERR_INVALID_ARG
 
 
@@ -87,5 +92,7 @@ def test_null_handle_calls_are_rejected():
     assert wm._lib.wm_rollout(None, 1, 1, 0, 0, None, None) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_mdn_nll(None, 1, 1, *([None] * 8)) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_sync(None) == wm.WM_ERR_INVALID_ARG
+    assert wm._lib.wm_set_controllers(None, 1, 1, None, None) == wm.WM_ERR_INVALID_ARG
+    assert wm._lib.wm_returns(None, 1, 1, 0, 0.9, 1, *([None] * 6)) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_last_error(None) == b"null handle"
     wm._lib.wm_destroy(None)  # no-op

@@ -480,3 +480,82 @@ def test_shaped_reward_against_oracle(wm, orc, path, name, flags):
                   rt0=a["rt_seq"][2].contiguous(), mem0=a["mem_seq"][2].contiguous(), want_seq=True)
     for k in ("rewards", "rt_seq", "mem_seq", "actions"):
         assert torch.equal(torch.cat([a[k], b[k]]), g[k]), k
+
+
+# ------------------------------------------------------------------ population, log-probs, values, returns
+@pytest.mark.parametrize("path,name,P,E,off,flags", [
+    ("tensor", "small_bf16", 3, 256, 512, dict(ctrl_sample=1, ctrl_tau=0.8)),
+    ("tensor", "mid_bf16", 2, 256, 0, dict(done_terminates=1)),
+    ("stepwise", "tiny_fp32", 3, 5, 7, dict(ctrl_sample=1, ctrl_tau=1.2)),
+    ("auto", "small_bf16", 4, 100, 0, dict()),  # E not a multiple of 256: not the tensor family
+])
+def test_population_logp_value_against_oracle(wm, orc, path, name, P, E, off, flags):
+    """A population of controllers (episode e -> candidate (e / E) mod P), the log-prob of
+    each action taken and the value head, step-anchored against the oracle."""
+    cfg = dict(synth.model_config(name), value_head=1, **flags)
+    w = synth.weights(cfg, seed=14)
+    Wp, bp = synth.population(cfg, P, seed=14)
+    B, T = (768, 5) if name != "tiny_fp32" else (16, 10)
+    z0 = synth.z0(B, cfg["z_dim"], seed=14)
+    mask = synth.mask(T, B, cfg["a_dim"], synth.WORKLOADS[name]["mask_density"], seed=14)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    m.set_controllers(Wp, bp, pop_group=E)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=off, want_seq=True, want_logp=True)
+    torch.cuda.synchronize()
+    if path != "auto":
+        assert m.last_path == path
+    else:
+        assert m.last_path == "stepwise"
+    ocfg = dict(cfg, pop_size=P, pop_group=E)
+    r = check_rollout(g, ocfg, dict(w, W_ctrl=Wp, b_ctrl=bp), z0, mask, episodes=off + np.arange(B),
+                      orc=orc)
+    print("population", path, name, P, E, r)
+    # every candidate acted
+    cands = ((off + np.arange(B)) // E) % P
+    assert len(set(cands.tolist())) == P
+    # back to a single controller: the call matches the base model again
+    m.set_controllers(w["W_ctrl"][None], w["b_ctrl"][None], pop_group=1)
+    g1 = m.rollout(_cuda(z0[:300]), 3, mask=_cuda(mask[:3, :300]), want_seq=True, want_logp=True)
+    check_rollout(g1, cfg, w, z0[:300], mask[:3, :300], orc=orc)
+
+
+def test_fused_family_takes_a_new_single_controller(wm, orc):
+    """wm_set_controllers with P = 1 repacks the fused family's images."""
+    cfg = synth.model_config("small_bf16")
+    w = synth.weights(cfg, seed=15)
+    Wp, bp = synth.population(cfg, 1, seed=16)
+    B, T = 200, 4
+    z0 = synth.z0(B, cfg["z_dim"], seed=15)
+    mask = synth.mask(T, B, cfg["a_dim"], 0.3, seed=15)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    m.set_controllers(Wp, bp)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    check_rollout(g, cfg, dict(w, W_ctrl=Wp[0], b_ctrl=bp[0]), z0, mask, orc=orc)
+    with pytest.raises(wm.WMError):  # the fused family writes no log-probs
+        m.rollout(_cuda(z0), T, mask=_cuda(mask), want_logp=True)
+
+
+@pytest.mark.parametrize("host", [False, True])
+def test_returns_and_fitness_match_oracle(wm, orc, host):
+    """wm_returns: G_t = r_t + gamma G_{t+1} (done ends the sum), bit for bit the oracle's
+    fp64 recursion; fitness = each candidate's mean G_0."""
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("mid_bf16", B=1000, T=30)
+    P, E, off = 5, 7, 3
+    m = wm.WorldModel(dict(cfg, value_head=1), w)
+    Wp, bp = synth.population(cfg, P, seed=17)
+    m.set_controllers(Wp, bp, pop_group=E)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=off)
+    gamma = float(np.float32(0.97))
+    boot = torch.randn(B, device="cuda")
+    args = (g["rewards"], g["done"], gamma)
+    if host:
+        args = (g["rewards"].cpu(), g["done"].cpu(), gamma)
+        boot = boot.cpu()
+    res = m.returns(*args, bootstrap=boot, episode_offset=off, want_fitness=True)
+    torch.cuda.synchronize()
+    o = orc.returns(np_(g["rewards"]), np_(g["done"]), gamma, stop_at_done=True, bootstrap=np_(boot),
+                    episode_offset=off, pop_size=P, pop_group=E)
+    assert np.array_equal(np_(res["returns"]), o["returns"])
+    np.testing.assert_allclose(np_(res["fitness"]), o["fitness"], rtol=1e-6)
