@@ -201,11 +201,13 @@ def dist_env():
     return ws, rank, local
 
 
-def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps):
+def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps, shaping=None):
     """The same rollout through the C ABI with pinned HOST arrays: copies are timed.
     env_steps: the (episode, step) pairs one call counts over all ranks."""
     import torch
 
+    sh = {} if shaping is None else {"rt0": torch.from_numpy(shaping[0]).pin_memory(),
+                                     "mem0": torch.from_numpy(shaping[1]).pin_memory()}
     zh = torch.from_numpy(z0).pin_memory()
     mh = torch.from_numpy(mask).pin_memory()
     hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
@@ -213,17 +215,17 @@ def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps
             "rewards": torch.empty((T, B), pin_memory=True),
             "done": torch.empty((T, B), dtype=torch.uint8, pin_memory=True)}
     for _ in range(2):
-        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout, **sh)
     torch.cuda.synchronize()
     e2e_t = []
     for i in range(args.steps):
         flush.fill_(float(i))
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout)
+        model.rollout(zh, T, mask=mh, episode_offset=ep0, want_final=False, out=hout, **sh)
         e2e_t.append(time.perf_counter() - t0)
     e2e_value = env_steps / max_over_ranks(sum(e2e_t) / len(e2e_t), ws, dev)
-    h2d = zh.numel() * 4 + mh.numel() * 4
+    h2d = zh.numel() * 4 + mh.numel() * 4 + sum(v.numel() * 4 for v in sh.values())
     d2h = sum(v.numel() * v.element_size() for v in hout.values())
 
     return e2e_value, h2d, d2h
@@ -355,10 +357,24 @@ def run_ours(args) -> None:
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=args.batch, shard=rank)
     if args.path:
         cfg["path"] = args.path
+    shaping = None
+    if args.reward == "shaped":
+        cfg["reward_mode"] = 1
+        shaping = synth.shaping_state(B, shard=rank)
+    P = args.population
+    if P:
+        if B % P or (B // P) % 256:
+            raise SystemExit("--population: B / P must be a multiple of 256")
+        cfg["value_head"] = 1
     model = wm.WorldModel(cfg, w, device=local)
+    if P:
+        Wp, bp = synth.population(cfg, P)
+        model.set_controllers(Wp, bp, pop_group=B // P)
     dev = torch.device("cuda", local)
     zc = torch.from_numpy(z0).to(dev)
     mc = torch.from_numpy(mask).to(dev)
+    sh_dev = {} if shaping is None else {"rt0": torch.from_numpy(shaping[0]).to(dev),
+                                         "mem0": torch.from_numpy(shaping[1]).to(dev)}
     ep0 = rank * B
     out = {"z": torch.empty((T + 1, B, cfg["z_dim"]), device=dev),
            "actions": torch.empty((T, B), dtype=torch.int32, device=dev),
@@ -367,15 +383,27 @@ def run_ours(args) -> None:
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
 
+    if P:  # a generation of a controller search: log-probs, values, returns and fitness too
+        out["logp_seq"] = torch.empty((T, B), device=dev)
+        out["value_seq"] = torch.empty((T, B), device=dev)
+        ret = {"returns": torch.empty((T, B), device=dev)}
+
     def step():
-        return model.rollout(zc, T, mask=mc, episode_offset=ep0, want_final=False, out=out,
-                             stream=stream)
+        r = model.rollout(zc, T, mask=mc, episode_offset=ep0, want_final=False, out=out,
+                          stream=stream, **sh_dev)
+        n = model.last_launches
+        if P:
+            ret.update(model.returns(out["rewards"], out["done"], 0.99, bootstrap=out["value_seq"][T - 1],
+                                     episode_offset=ep0, want_fitness=True, stream=stream))
+            n += model.last_launches
+        step.launches = n
+        return r
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
     path_name = model.last_path
-    launches = model.last_launches
+    launches = step.launches
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -416,7 +444,7 @@ def run_ours(args) -> None:
         e2e_value, h2d, d2h = None, 0, 0
     else:
         e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg,
-                                          env_steps)
+                                          env_steps, shaping)
 
     # roofline of the dominant kernel: its algorithmic FLOPs per launch over its own
     # event-timed average launch duration inside the timed region
@@ -453,11 +481,18 @@ def run_ours(args) -> None:
             "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if cfg["precision"] == "bf16" else "f32",
             "data": "synthetic (seeded: weights N(0,0.05^2), z0 N(0,1), Bernoulli masks)",
-            "config": {"workload": name if args.batch is None else f"{name} with B overridden",
+            "config": {"workload": (name + ("+shaped_reward" if shaping is not None else "")
+                                    + (f"+population{P}" if P else ""))
+                       if args.batch is None else f"{name} with B overridden",
                        "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
                        "H": cfg["h_dim"], "K": cfg["k_mix"],
                        "mask_density": synth.WORKLOADS[name]["mask_density"],
                        "precision": cfg["precision"], "kernel_path": path_name,
+                       "reward": "Eq. 2 on predicted runtime / memory heads (alpha 0.8, beta 0.2, "
+                                 "-100 invalid)" if shaping is not None else "linear reward head",
+                       "population": None if not P else
+                       f"{P} controller candidates x {B // P} episodes; log-probs, value head, "
+                       "discounted returns (gamma 0.99) and per-candidate fitness in the step",
                        "l2": "flushed between timed steps (512 MiB write)",
                        "parallelism": f"episodes sharded over {ws} GPU(s), no collective"},
             "e2e": None if e2e_value is None else
@@ -468,7 +503,7 @@ def run_ours(args) -> None:
     if live is not None:
         line["live_steps"] = live  # value counts live pairs; frozen pairs are executed too
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes)
+        line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes, shaped=shaping is not None)
     if rank == 0:
         print(json.dumps(line), flush=True)
     model.close()
@@ -494,7 +529,8 @@ def counted_steps(cfg: dict, done) -> int:
     return int((~ended).sum())
 
 
-def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) -> dict:
+def cpu_baseline(name: str, episodes: int | None, threads: int | None = None,
+                 shaped: bool = False) -> dict:
     """The oracle on the host cores (all of them), plus a one-thread figure on a tenth of the
     sample (episodes are independent, so throughput per episode-step is comparable)."""
     import oracle
@@ -502,12 +538,18 @@ def cpu_baseline(name: str, episodes: int | None, threads: int | None = None) ->
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name)
     n = min(episodes or oracle_episodes(name, 2e11), B)
     threads = threads or os.cpu_count() or 1
+    sh = {}
+    if shaped:
+        cfg["reward_mode"] = 1
+        rt0, mem0 = synth.shaping_state(n)
+        sh = {"rt0": rt0, "mem0": mem0}
     t0 = time.perf_counter()
-    o = oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads)
+    o = oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads, **sh)
     dt = time.perf_counter() - t0
     n1 = max(1, n // 10)
+    sh1 = {k: v[:n1] for k, v in sh.items()}
     t1 = time.perf_counter()
-    o1 = oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1)
+    o1 = oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1, **sh1)
     dt1 = time.perf_counter() - t1
     return {"value": round(counted_steps(cfg, o["done"]) / dt, 2), "unit": "env-steps/s",
             "cores": threads,
@@ -593,6 +635,13 @@ def main():
     ap.add_argument("--precision", choices=["fp32", "bf16"], default=None,
                     help="nll workload only: fp32 or bf16 path (default bf16)")
     ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
+    ap.add_argument("--population", type=int, default=0,
+                    help="P controller candidates (B / P episodes each): each step is one "
+                         "generation's evaluation (rollout with log-probs and values, returns, "
+                         "fitness)")
+    ap.add_argument("--reward", choices=["head", "shaped"], default="head",
+                    help="rollout reward: the linear head, or Eq. 2 on the predicted runtime / "
+                         "memory heads (Sec. 3.1.4)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer leg (profiling runs)")
     ap.add_argument("--batch", type=int, default=None,
