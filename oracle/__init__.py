@@ -49,7 +49,7 @@ class _Cfg(C.Structure):
                 ("seed", C.c_uint64), ("nthreads", C.c_int), ("reward_mode", C.c_int),
                 ("reward_alpha", C.c_double), ("reward_beta", C.c_double),
                 ("invalid_reward", C.c_double), ("pop_size", C.c_int), ("pop_group", C.c_int),
-                ("value_head", C.c_int)]
+                ("value_head", C.c_int), ("n_xfers", C.c_int)]
 
 
 class _W(C.Structure):
@@ -63,7 +63,9 @@ class _W(C.Structure):
 
 class _Ext(C.Structure):
     _fields_ = [("rt0", C.c_void_p), ("mem0", C.c_void_p), ("rt_seq", C.c_void_p),
-                ("mem_seq", C.c_void_p), ("logp_seq", C.c_void_p), ("value_seq", C.c_void_p)]
+                ("mem_seq", C.c_void_p), ("logp_seq", C.c_void_p), ("value_seq", C.c_void_p),
+                ("loc_mask", C.c_void_p), ("loc_seq", C.c_void_p), ("loc_margin", C.c_void_p),
+                ("loc_use", C.c_void_p)]
 
 
 def _load():
@@ -118,7 +120,7 @@ def _cfg(cfg: dict, nthreads: int) -> _Cfg:
                 int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
                 float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)),
                 int(cfg.get("pop_size", 0)), int(cfg.get("pop_group", 1)),
-                int(cfg.get("value_head", 0)))
+                int(cfg.get("value_head", 0)), int(cfg.get("n_xfers", 0)))
 
 
 class _Weights:
@@ -140,8 +142,17 @@ class _ExtArgs:
     """The optional parts of a call (shaped-reward state, log-probs, values); keeps the
     arrays alive."""
 
-    def __init__(self, cfg: dict, B: int, T: int, rt0=None, mem0=None):
+    def __init__(self, cfg: dict, B: int, T: int, rt0=None, mem0=None, loc_mask=None, loc_use=None):
         self.out = {"logp_seq": np.zeros((T, B), np.float32)}
+        NX = int(cfg.get("n_xfers", 0))
+        lm = lu = None
+        if NX > 0:
+            WL = (int(cfg["a_dim"]) - NX + 31) // 32
+            if loc_mask is not None:
+                lm = np.ascontiguousarray(loc_mask, dtype=np.uint32).reshape(T, B, NX, WL)
+            if loc_use is not None:
+                lu = np.ascontiguousarray(loc_use, dtype=np.int32).reshape(B)
+            self.out.update(loc_seq=np.zeros((T, B), np.int32), loc_margin=np.zeros((T, B), np.float32))
         r = m = None
         if int(cfg.get("reward_mode", 0)) == 1:
             if rt0 is None or mem0 is None:
@@ -150,10 +161,11 @@ class _ExtArgs:
             self.out.update(rt_seq=np.zeros((T, B), np.float32), mem_seq=np.zeros((T, B), np.float32))
         if int(cfg.get("value_head", 0)):
             self.out["value_seq"] = np.zeros((T, B), np.float32)
-        self.keep = [r, m]
+        self.keep = [r, m, lm, lu]
         o = self.out
         self.s = _Ext(_ptr(r), _ptr(m), _ptr(o.get("rt_seq")), _ptr(o.get("mem_seq")),
-                      _ptr(o["logp_seq"]), _ptr(o.get("value_seq")))
+                      _ptr(o["logp_seq"]), _ptr(o.get("value_seq")), _ptr(lm),
+                      _ptr(o.get("loc_seq")), _ptr(o.get("loc_margin")), _ptr(lu))
 
     def ref(self):
         return C.byref(self.s)
@@ -238,7 +250,7 @@ def select_action(logits, mask_words=None, ctrl_sample: int = 0, ctrl_tau: float
 # ---------------------------------------------------------------- the path
 def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset: int = 0,
             t0: int = 0, h0=None, c0=None, done0=None, want_seq: bool = False,
-            nthreads: int = 1, rt0=None, mem0=None) -> dict:
+            nthreads: int = 1, rt0=None, mem0=None, loc_mask=None) -> dict:
     """Free-running dream rollout of B = len(z0) episodes for T steps (a1..a8).
     With the shaped reward (reward_mode 1), rt0 / mem0 [B] are the predictions of the
     current graphs and the result carries rt_seq / mem_seq [T, B]."""
@@ -264,7 +276,7 @@ def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset:
                    comp_seq=np.zeros((T, B, Z), np.uint8))
     w = _Weights(weights)
     cs = _cfg(cfg, nthreads)
-    ext = _ExtArgs(cfg, B, T, rt0, mem0)
+    ext = _ExtArgs(cfg, B, T, rt0, mem0, loc_mask)
     out.update(ext.out)
     rc = lib.orc_rollout(C.byref(cs), C.byref(w.s), B, T, int(episode_offset), int(t0),
                          _ptr(z0), _ptr(h0), _ptr(c0), _ptr(d0), _ptr(mk),
@@ -279,7 +291,8 @@ def rollout(cfg: dict, weights: dict, z0, mask=None, T: int = 1, episode_offset:
 
 
 def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=None, mask=None,
-         a_use=None, h_use=None, k_use=None, nthreads: int = 1, rt=None, mem=None) -> dict:
+         a_use=None, h_use=None, k_use=None, nthreads: int = 1, rt=None, mem=None,
+         loc_mask=None, loc_use=None) -> dict:
     """One dream step (a1..a8) of B = len(episodes) episodes started from the state
     (z [B,Z], h [B,H], c [B,H], frozen [B]); episodes are global Philox indices.
     a_use / h_use / k_use replace what flows downstream of the action, h' and
@@ -305,7 +318,7 @@ def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=No
            "z_next": np.zeros((B, Z), np.float32)}
     w = _Weights(weights)
     cs = _cfg(cfg, nthreads)
-    ext = _ExtArgs(cfg, B, 1, rt, mem)
+    ext = _ExtArgs(cfg, B, 1, rt, mem, loc_mask, loc_use)
     rc = lib.orc_step(C.byref(cs), C.byref(w.s), B, _ptr(ep), int(step_index) & 0xFFFFFFFF,
                       _ptr(z), _ptr(h), _ptr(c), _ptr(fz), _ptr(mk), _ptr(au), _ptr(hu), _ptr(ku),
                       _ptr(out["action"]), _ptr(out["ctrl_margin"]), _ptr(out["h"]), _ptr(out["c"]),
@@ -317,6 +330,8 @@ def step(cfg: dict, weights: dict, episodes, step_index: int, z, h, c, frozen=No
     if "rt_seq" in ext.out:
         out["rt"], out["mem"] = ext.out["rt_seq"][0], ext.out["mem_seq"][0]
     out["logp"] = ext.out["logp_seq"][0]
+    if "loc_seq" in ext.out:
+        out["loc"], out["loc_margin"] = ext.out["loc_seq"][0], ext.out["loc_margin"][0]
     if "value_seq" in ext.out:
         out["value"] = ext.out["value_seq"][0]
     return out

@@ -336,11 +336,13 @@ static int check_cfg(const orc_cfg *c)
     if (!(c->mdn_tau >= 0.0) || !(c->ctrl_tau >= 0.0)) return -1;
     if (c->reward_mode != 0 && c->reward_mode != 1) return -1;
     if (c->pop_size > 1 && c->pop_group < 1) return -1;
+    if (c->n_xfers < 0 || c->n_xfers >= c->a_dim) return -1;
     return 0;
 }
 
-/* a3 + a4: one LSTM step for one episode.  x = [op(z); op(h)] of length Z+H. */
-static void lstm_step(const orc_cfg *cfg, const wts64 *v, const double *x, int a,
+/* a3 + a4: one LSTM step for one episode.  x = [op(z); op(h)] of length Z+H; a, a2 are
+ * the one-hot action rows taken (-1: none). */
+static void lstm_step(const orc_cfg *cfg, const wts64 *v, const double *x, int a, int a2,
                       double *gates, double *c, double *h)
 {
     const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, N4 = 4 * H;
@@ -348,6 +350,7 @@ static void lstm_step(const orc_cfg *cfg, const wts64 *v, const double *x, int a
         double g = v->b_lstm[n];
         for (int i = 0; i < Z; ++i) g += x[i] * v->W_lstm[(size_t)i * N4 + n];
         if (a >= 0) g += v->W_lstm[(size_t)(Z + a) * N4 + n];
+        if (a2 >= 0) g += v->W_lstm[(size_t)(Z + a2) * N4 + n];
         for (int i = 0; i < H; ++i) g += x[Z + i] * v->W_lstm[(size_t)(Z + A + i) * N4 + n];
         gates[n] = g;
     }
@@ -419,7 +422,8 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
                         const uint32_t *mw, int a_use, const float *h_use, const uint8_t *k_use,
                         int32_t *action, float *ctrl_margin, float *reward, uint8_t *done,
                         float *done_margin, float *mdn_out, uint8_t *comp, float *comp_margin,
-                        float *logp, float *value)
+                        float *logp, float *value, const uint32_t *lmw, int l_use, int32_t *loc_out,
+                        float *loc_margin)
 {
     const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix;
     double *x = sb->x, *g = sb->g, *y = sb->y, *mdn = sb->mdn, *znew = sb->znew;
@@ -443,26 +447,51 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
         u_ctrl = orc_uniform(r4[0]);
     }
     double cm;
-    int a = orc_select_action(A, lg, mw, cfg->ctrl_sample, cfg->ctrl_tau, u_ctrl, &cm);
+    /* hierarchical (Sec. 3.1.3): the xfer among the first NX logits, then the location
+     * among the other L under the chosen xfer's location mask; flat: one choice of A */
+    const int NX = cfg->n_xfers, hier = NX > 0, L = A - NX, WL = (L + 31) / 32;
+    const int noop = hier ? NX - 1 : A - 1;
+    int a = orc_select_action(hier ? NX : A, lg, mw, cfg->ctrl_sample, cfg->ctrl_tau, u_ctrl, &cm);
+    int loc = -1;
+    double lm = INFINITY;
+    if (hier && a >= 0 && a != noop) {
+        double u_loc = 0.0;
+        if (cfg->ctrl_sample && cfg->ctrl_tau > 0.0) {
+            uint32_t r4[4];
+            orc_draw(cfg->seed, e, s, 2u, 0u, r4);
+            u_loc = orc_uniform(r4[1]);
+        }
+        loc = orc_select_action(L, lg + NX, lmw ? lmw + (size_t)a * WL : NULL, cfg->ctrl_sample,
+                                cfg->ctrl_tau, u_loc, &lm);
+    }
     *action = a;
     if (ctrl_margin) *ctrl_margin = (float)cm;
+    if (loc_out) *loc_out = loc;
+    if (loc_margin) *loc_margin = (float)lm;
     if (a_use >= -1) a = a_use;
-    /* log pi(a | z, h) of the action taken, pi = softmax(l / ctrl_tau) over the valid actions */
+    if (hier && l_use >= -1) loc = l_use;
+    if (hier && (a < 0 || a == noop)) loc = -1;
+    /* log pi of the action taken, pi = softmax(l / ctrl_tau) over the valid actions; for a
+     * hierarchical action log pi(xfer) + log pi(location | xfer) */
     if (logp) {
         double lp = 0.0;
-        if (a >= 0 && cfg->ctrl_tau > 0.0) {
+        for (int part = 0; part < (hier ? 2 : 1); ++part) {
+            const int choice = part ? loc : a;
+            const int n0 = part ? NX : 0, n = hier ? (part ? L : NX) : A;
+            const uint32_t *pm = part ? (lmw ? lmw + (size_t)a * WL : NULL) : mw;
+            if (choice < 0 || !(cfg->ctrl_tau > 0.0)) continue;
             double lmax = -INFINITY, S = 0.0;
-            for (int j = 0; j < A; ++j)
-                if ((!mw || bit_set(mw, j)) && (double)lg[j] > lmax) lmax = (double)lg[j];
-            for (int j = 0; j < A; ++j)
-                if (!mw || bit_set(mw, j)) S += exp(((double)lg[j] - lmax) / cfg->ctrl_tau);
-            lp = ((double)lg[a] - lmax) / cfg->ctrl_tau - log(S);
+            for (int j = 0; j < n; ++j)
+                if ((!pm || bit_set(pm, j)) && (double)lg[n0 + j] > lmax) lmax = (double)lg[n0 + j];
+            for (int j = 0; j < n; ++j)
+                if (!pm || bit_set(pm, j)) S += exp(((double)lg[n0 + j] - lmax) / cfg->ctrl_tau);
+            lp += ((double)lg[n0 + choice] - lmax) / cfg->ctrl_tau - log(S);
         }
         *logp = (float)lp;
     }
 
     /* a3 + a4 */
-    lstm_step(cfg, v, x, a, g, c, h);
+    lstm_step(cfg, v, x, a, loc >= 0 ? NX + loc : -1, g, c, h);
 
     /* a5: heads on op(h') */
     for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h_use ? (double)h_use[i] : h[i]);
@@ -475,8 +504,9 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
         for (int i = 0; i < H; ++i) { rt_new += y[i] * v->w_rt[i]; mem_new += y[i] * v->w_mem[i]; }
         rt_new = (double)(float)rt_new;   /* predictions are carried in fp32 */
         mem_new = (double)(float)mem_new;
-        r = a >= 0 ? cfg->reward_alpha * (*rt - rt_new) + cfg->reward_beta * (*mem - mem_new)
-                   : cfg->invalid_reward;
+        const int valid = a >= 0 && (!hier || a == noop || loc >= 0);
+        r = valid ? cfg->reward_alpha * (*rt - rt_new) + cfg->reward_beta * (*mem - mem_new)
+                  : cfg->invalid_reward;
         *rt = rt_new;
         *mem = mem_new;
     }
@@ -488,7 +518,7 @@ static int step_episode(const orc_cfg *cfg, const wts64 *v, step_buf *sb, uint64
     }
     float dlf = (float)dl;
     if (done_margin) *done_margin = fabsf(dlf);
-    int is_noop = cfg->noop_terminates && a == A - 1;
+    int is_noop = cfg->noop_terminates && a == noop;
     *done = (uint8_t)((dlf > 0.0f) || is_noop);
 
     /* a6 + a7: per-dim mixture sample */
@@ -558,10 +588,16 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
         const size_t tb = (size_t)t * B + b;
         float *lp_out = ext && ext->logp_seq ? ext->logp_seq + tb : NULL;
         float *v_out = ext && ext->value_seq && cfg->value_head ? ext->value_seq + tb : NULL;
+        const int NX = cfg->n_xfers, WL = (A - NX + 31) / 32;
+        const uint32_t *lmw = NX > 0 && ext && ext->loc_mask ? ext->loc_mask + tb * NX * WL : NULL;
+        int32_t *loc_out = NX > 0 && ext && ext->loc_seq ? ext->loc_seq + tb : NULL;
+        float *lm_out = NX > 0 && ext && ext->loc_margin ? ext->loc_margin + tb : NULL;
         if (frozen) {
             actions[tb] = -1; rewards[tb] = 0.0f; done[tb] = 1;
             if (lp_out) *lp_out = 0.0f;
             if (v_out) *v_out = 0.0f;
+            if (loc_out) *loc_out = -1;
+            if (lm_out) *lm_out = INF_F;
             if (mdn_seq) for (int m = 0; m < M; ++m) mdn_seq[tb * M + m] = 0.0f;
             if (comp_seq) for (int d = 0; d < Z; ++d) comp_seq[tb * Z + d] = 255;
             if (ctrl_margin) ctrl_margin[tb] = INF_F;
@@ -574,7 +610,8 @@ static int rollout_episode(const orc_cfg *cfg, const wts64 *v, int b, int B, int
                                   done_margin ? &done_margin[tb] : NULL,
                                   mdn_seq ? mdn_seq + tb * M : NULL,
                                   comp_seq ? comp_seq + tb * Z : NULL,
-                                  comp_margin ? comp_margin + tb * Z : NULL, lp_out, v_out);
+                                  comp_margin ? comp_margin + tb * Z : NULL, lp_out, v_out, lmw, -2,
+                                  loc_out, lm_out);
         }
         for (int i = 0; i < Z; ++i) z_out[((size_t)(t + 1) * B + b) * Z + i] = (float)z[i];
         if (h_seq) for (int i = 0; i < H; ++i) h_seq[tb * H + i] = (float)h[i];
@@ -660,10 +697,17 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
         double rt = shaped ? (double)ext->rt0[b] : 0.0, mem = shaped ? (double)ext->mem0[b] : 0.0;
         float *lp_out = ext && ext->logp_seq ? ext->logp_seq + b : NULL;
         float *v_out = ext && ext->value_seq && cfg->value_head ? ext->value_seq + b : NULL;
+        const int NX = cfg->n_xfers, WL = (A - NX + 31) / 32;
+        const uint32_t *lmw = NX > 0 && ext && ext->loc_mask ? ext->loc_mask + (size_t)b * NX * WL : NULL;
+        int32_t *loc_out = NX > 0 && ext && ext->loc_seq ? ext->loc_seq + b : NULL;
+        float *lm_out = NX > 0 && ext && ext->loc_margin ? ext->loc_margin + b : NULL;
+        const int l_use = NX > 0 && ext && ext->loc_use ? ext->loc_use[b] : -2;
         if (frozen && frozen[b]) {
             action[b] = -1; ctrl_margin[b] = INF_F; reward[b] = 0.0f; done[b] = 1;
             if (lp_out) *lp_out = 0.0f;
             if (v_out) *v_out = 0.0f;
+            if (loc_out) *loc_out = -1;
+            if (lm_out) *lm_out = INF_F;
             done_margin[b] = INF_F;
             for (int m = 0; m < M; ++m) mdn_out[(size_t)b * M + m] = 0.0f;
             for (int d = 0; d < Z; ++d) {
@@ -677,7 +721,7 @@ int orc_step(const orc_cfg *cfg, const orc_weights *w, int B, const uint64_t *ep
                          k_use ? k_use + (size_t)b * Z : NULL,
                          &action[b], &ctrl_margin[b], &reward[b], &done[b], &done_margin[b],
                          mdn_out + (size_t)b * M, comp + (size_t)b * Z,
-                         comp_margin + (size_t)b * Z, lp_out, v_out);
+                         comp_margin + (size_t)b * Z, lp_out, v_out, lmw, l_use, loc_out, lm_out);
         }
         for (int i = 0; i < Z; ++i) z_next[(size_t)b * Z + i] = (float)zs[i];
         for (int i = 0; i < H; ++i) {
@@ -744,7 +788,7 @@ static int nll_sequence(const orc_cfg *cfg, const wts64 *v, int n, int N, int T,
         const size_t tn = (size_t)t * N + n;
         for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z_seq[tn * Z + i]);
         for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
-        lstm_step(cfg, v, x, actions[tn], g, c, h);
+        lstm_step(cfg, v, x, actions[tn], -1, g, c, h);
         for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h[i]);
         mdn_head(cfg, v, y, mdn);
         if (h_seq) for (int i = 0; i < H; ++i) h_seq[tn * H + i] = (float)h[i];

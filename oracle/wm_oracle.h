@@ -51,6 +51,13 @@ typedef struct {
     int pop_size, pop_group;
     /* value head V(h') = w_val . h' + b_val (1 = on)                        */
     int value_head;
+    /* hierarchical action (Sec. 3.1.3): n_xfers = NX > 0 splits the a_dim
+     * controller outputs into NX xfer logits (the last one, NX - 1, is the
+     * NO-OP) and L = a_dim - NX location logits; the xfer is chosen under the
+     * step's xfer mask (bits 0..NX-1 of the mask words), then the location
+     * under that xfer's location mask; the LSTM input is onehot(xfer) ||
+     * onehot(location) (action rows xfer and NX + location).  0 = flat.     */
+    int n_xfers;
 } orc_cfg;
 
 typedef struct {
@@ -83,6 +90,13 @@ typedef struct {
      * controller's masked softmax at temperature ctrl_tau (0 when ctrl_tau
      * is 0 or no action was valid); value_seq [T,B]: V(h_{t+1}) (value_head). */
     float *logp_seq, *value_seq;
+    /* hierarchical action: loc_mask [T,B,NX,ceil(L/32)] (NULL = all valid);
+     * loc_seq [T,B] the location taken (-1: none, e.g. NO-OP); loc_margin
+     * [T,B] the location decision's margin (infinite when there is none). */
+    const uint32_t *loc_mask;
+    int32_t *loc_seq;
+    float *loc_margin;
+    const int32_t *loc_use;   /* orc_step only: [B] location override (< -1: none) */
 } orc_ext;
 
 /* ---- building blocks (exported so tests can pin each one) ---------------- */

@@ -51,6 +51,7 @@ WORKLOADS = {
 _STREAM = {"W_lstm": 1, "b_lstm": 2, "W_mdn": 3, "b_mdn": 4, "w_rew": 5, "b_rew": 6,
            "w_done": 7, "b_done": 8, "W_ctrl": 9, "b_ctrl": 10, "w_rt": 11, "b_rt": 12,
            "w_mem": 13, "b_mem": 14, "W_pop": 15, "b_pop": 16, "w_val": 17, "b_val": 18,
+           "hier": 27,
            "z0": 20, "mask": 21, "zseq": 22, "actions": 23, "lengths": 24, "rt0": 25, "mem0": 26}
 
 
@@ -77,7 +78,7 @@ def model_config(name: str, **over) -> dict:
                reward_mode=w.get("reward_mode", 0), reward_alpha=w.get("reward_alpha", 0.8),
                reward_beta=w.get("reward_beta", 0.2), invalid_reward=w.get("invalid_reward", -100.0),
                pop_size=w.get("pop_size", 0), pop_group=w.get("pop_group", 1),
-               value_head=w.get("value_head", 0))
+               value_head=w.get("value_head", 0), n_xfers=w.get("n_xfers", 0))
     return cfg
 
 
@@ -140,6 +141,29 @@ def mask(T: int, B: int, A: int, density: float, seed: int = 0, shard: int = 0) 
         r = _shard_rng(seed, _STREAM["mask"], t, shard)
         out[t] = pack_mask(r.random((B, A), dtype=np.float32) < thr)
     return out
+
+
+def hier_masks(T: int, B: int, NX: int, L: int, density: float, seed: int = 0, shard: int = 0):
+    """Masks of the hierarchical action (Sec. 3.1.3): (xfer mask [T, B, ceil((NX+L)/32)],
+    location masks [T, B, NX, ceil(L/32)]).  Each (step, episode, xfer) has a count of valid
+    locations, a prefix of the L location slots (the environment lists a graph's locations
+    first and marks the rest of the slots invalid): 0 with probability 1 - density, else
+    uniform on [1, L].  An xfer is valid iff it has a location; the NO-OP (xfer NX - 1)
+    is always valid and has none."""
+    A = NX + L
+    W, WL = (A + 31) // 32, (L + 31) // 32
+    xm = np.empty((T, B, W), dtype=np.uint32)
+    lm = np.empty((T, B, NX, WL), dtype=np.uint32)
+    for t in range(T):
+        r = _shard_rng(seed, _STREAM["hier"], t, shard)
+        n = r.integers(1, L + 1, size=(B, NX), dtype=np.int32)
+        n = np.where(r.random((B, NX), dtype=np.float32) < np.float32(density), n, 0)
+        n[:, NX - 1] = 0
+        valid_x = n > 0
+        valid_x[:, NX - 1] = True
+        xm[t] = pack_mask(np.concatenate([valid_x, np.zeros((B, L), bool)], axis=1))
+        lm[t] = pack_mask(np.arange(L)[None, None, :] < n[:, :, None])
+    return xm, lm
 
 
 def teacher_inputs(N: int, T: int, Z: int, A: int, seed: int = 0, ragged: bool = False):

@@ -233,3 +233,148 @@ def test_fitness_is_mean_return_per_candidate(orc):
     for g in range(P):
         sel = [b for b in range(B) if ((off + b) // E) % P == g]
         assert out["fitness"][g] == pytest.approx(g0[sel].mean(), rel=1e-6)
+
+
+# ----------------------------------------------------------------------------- hierarchical action (Sec. 3.1.3)
+def _hier_case(seed=57, **kw):
+    NX, L = 6, 11
+    Z, A, H, K, B, T = 4, NX + L, 16, 2, 9, 6
+    kw.setdefault("reward_mode", 0)
+    cfg = _cfg(Z, A, H, K, n_xfers=NX, **kw)
+    w = synth.weights(cfg, seed=seed, std=0.5)
+    z0 = synth.z0(B, Z, seed=seed)
+    xm, lm = synth.hier_masks(T, B, NX, L, 0.6, seed=seed)
+    return cfg, w, z0, xm, lm, NX, L, B, T
+
+
+def test_hier_argmax_is_two_masked_argmaxes(orc):
+    """Argmax mode: the xfer is the masked argmax of the first NX logits, the location the
+    masked argmax of the other L under the chosen xfer's location mask (numpy, on logits
+    rebuilt from the rollout's own state); NO-OP takes no location."""
+    cfg, w, z0, xm, lm, NX, L, B, T = _hier_case()
+    o = orc.rollout(cfg, w, z0, xm, T, want_seq=True, loc_mask=lm)
+    Z, H = cfg["z_dim"], cfg["h_dim"]
+    checked = 0
+    for t in range(T):
+        h = np.zeros((B, H)) if t == 0 else o["h_seq"][t - 1].astype(np.float64)
+        lg = (np.concatenate([o["z"][t].astype(np.float64), h], 1) @ w["W_ctrl"].astype(np.float64)
+              + w["b_ctrl"]).astype(np.float32)
+        vx = np.unpackbits(xm[t].view(np.uint8), axis=1, bitorder="little")[:, :NX].astype(bool)
+        for b in range(B):
+            x = int(o["actions"][t, b])
+            assert x == int(np.argmax(np.where(vx[b], lg[b, :NX], -np.inf)))
+            loc = int(o["loc_seq"][t, b])
+            if x == NX - 1:
+                assert loc == -1
+                continue
+            vl = np.unpackbits(lm[t, b, x].view(np.uint8), bitorder="little")[:L].astype(bool)
+            assert vl.any() and vl[loc]
+            assert loc == int(np.argmax(np.where(vl, lg[b, NX:], -np.inf)))
+            checked += 1
+    assert checked > B * T // 3
+
+
+def test_hier_lstm_takes_both_rows(orc):
+    """h' = LSTMCell([z, onehot(xfer), onehot(location)], (h, c)) with the action rows of
+    W_lstm (torch, forced choices)."""
+    import torch
+    cfg, w, z0, xm, lm, NX, L, B, T = _hier_case()
+    Z, A, H = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"]
+    rng = np.random.default_rng(58)
+    h = (0.5 * rng.standard_normal((B, H))).astype(np.float32)
+    c = (0.5 * rng.standard_normal((B, H))).astype(np.float32)
+    xs = rng.integers(0, NX - 1, B).astype(np.int32)
+    ls = rng.integers(0, L, B).astype(np.int32)
+    ls[2] = -1
+    s = orc.step(cfg, w, np.arange(B), 0, z0, h, c, mask=xm[0], loc_mask=lm[0], a_use=xs, loc_use=ls)
+    cell = torch.nn.LSTMCell(Z + A, H, dtype=torch.float64)
+    Wl = torch.from_numpy(w["W_lstm"]).double()
+    with torch.no_grad():
+        cell.weight_ih.copy_(Wl[:Z + A].T)
+        cell.weight_hh.copy_(Wl[Z + A:].T)
+        cell.bias_ih.copy_(torch.from_numpy(w["b_lstm"]).double())
+        cell.bias_hh.zero_()
+        oh = torch.zeros(B, A, dtype=torch.float64)
+        oh[np.arange(B), xs] = 1.0
+        ok = ls >= 0
+        oh[np.nonzero(ok)[0], NX + ls[ok]] = 1.0
+        hr, cr = cell(torch.cat([torch.from_numpy(z0).double(), oh], 1),
+                      (torch.from_numpy(h).double(), torch.from_numpy(c).double()))
+    np.testing.assert_allclose(s["h"], hr.numpy(), atol=2e-6)
+    np.testing.assert_allclose(s["c"], cr.numpy(), atol=2e-6)
+
+
+def test_hier_logp_normalises_over_joint_actions(orc):
+    """exp(logp) summed over every valid (xfer, location) pair and the NO-OP is 1."""
+    cfg, w, z0, xm, lm, NX, L, B, T = _hier_case(ctrl_sample=1, ctrl_tau=0.8)
+    rng = np.random.default_rng(59)
+    h = (0.5 * rng.standard_normal((B, 16))).astype(np.float32)
+    c = np.zeros((B, 16), np.float32)
+    vx = np.unpackbits(xm[0].view(np.uint8), axis=1, bitorder="little")[:, :NX].astype(bool)
+    total = np.zeros(B)
+    for x in range(NX):
+        for loc in ([-1] if x == NX - 1 else range(L)):
+            s = orc.step(cfg, w, np.arange(B), 0, z0, h, c, mask=xm[0], loc_mask=lm[0],
+                         a_use=np.full(B, x), loc_use=np.full(B, loc))
+            ok = vx[:, x].copy()
+            if loc >= 0:
+                ok &= np.array([bool((lm[0, b, x, loc // 32] >> (loc % 32)) & 1) for b in range(B)])
+            total += np.where(ok, np.exp(s["logp"].astype(np.float64)), 0.0)
+    np.testing.assert_allclose(total, 1.0, atol=1e-5)
+
+
+def test_hier_sampled_frequencies(orc):
+    """Sampled mode: over many episodes (independent Philox streams) from one state, the
+    (xfer, location) frequencies follow pi(xfer) pi(location | xfer) (chi-square)."""
+    from scipy import stats
+    NX, L = 4, 5
+    Z, A, H, K, B = 3, NX + L, 8, 2, 6000
+    cfg = _cfg(Z, A, H, K, reward_mode=0, n_xfers=NX, ctrl_sample=1, ctrl_tau=1.0)
+    w = synth.weights(cfg, seed=60, std=0.6)
+    z = np.tile(synth.z0(1, Z, seed=60), (B, 1))
+    h = np.zeros((B, H), np.float32)
+    xm = synth.pack_mask(np.tile(np.array([[1, 0, 1, 1] + [0] * L], bool), (B, 1)))
+    locs = np.zeros((NX, L), bool)
+    locs[0, :3] = True
+    locs[2, :5] = True
+    lm = np.tile(synth.pack_mask(locs)[None], (B, 1, 1))
+    s = orc.step(cfg, w, np.arange(B), 0, z, h, h, mask=xm, loc_mask=lm)
+    lg = (np.concatenate([z[0].astype(np.float64), h[0]]) @ w["W_ctrl"].astype(np.float64)
+          + w["b_ctrl"]).astype(np.float32).astype(np.float64)
+    px = np.where([1, 0, 1, 1], np.exp(lg[:NX]), 0.0)
+    px /= px.sum()
+    cells, probs = [], []
+    for x in (0, 2):
+        pl = np.where(locs[x], np.exp(lg[NX:]), 0.0)
+        pl /= pl.sum()
+        for loc in np.nonzero(locs[x])[0]:
+            cells.append((x, loc))
+            probs.append(px[x] * pl[loc])
+    cells.append((3, -1))
+    probs.append(px[3])
+    counts = [int(np.sum((s["action"] == x) & (s["loc"] == loc))) for x, loc in cells]
+    assert sum(counts) == B
+    assert stats.chisquare(counts, np.array(probs) * B).pvalue > 1e-4
+
+
+def test_hier_noop_terminates_and_invalid(orc):
+    cfg, w, z0, xm, lm, NX, L, B, T = _hier_case(noop_terminates=1, reward_mode=1)
+    w["b_ctrl"][:] = 0
+    w["W_ctrl"][:] = 0
+    w["b_ctrl"][NX - 1] = 5.0  # NO-OP wins wherever it is valid
+    rt0, mem0 = synth.shaping_state(B, seed=57)
+    o = orc.rollout(cfg, w, z0, xm, T, want_seq=True, loc_mask=lm, rt0=rt0, mem0=mem0)
+    assert np.all(o["actions"][0] == NX - 1) and np.all(o["loc_seq"][0] == -1)
+    assert np.all(o["done"] == 1) and np.all(o["actions"][1:] == -1)
+    assert np.all(o["rewards"][0] != -100.0)  # the NO-OP is a valid action
+    # an xfer whose location mask is empty: the location is -1, the action invalid (-100)
+    cfg2 = dict(cfg, noop_terminates=0)
+    w2 = dict(w, b_ctrl=np.zeros(NX + L, np.float32))
+    w2["b_ctrl"][0] = 5.0
+    xm2 = xm.copy()
+    xm2[:] = 1  # xfer 0 valid everywhere ...
+    lm2 = lm.copy()
+    lm2[:, :, 0, :] = 0  # ... but with no location
+    o2 = orc.rollout(cfg2, w2, z0, xm2, T, want_seq=True, loc_mask=lm2, rt0=rt0, mem0=mem0)
+    assert np.all(o2["actions"] == 0) and np.all(o2["loc_seq"] == -1)
+    assert np.all(o2["rewards"] == np.float32(-100.0))
