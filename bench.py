@@ -201,13 +201,16 @@ def dist_env():
     return ws, rank, local
 
 
-def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps, shaping=None):
+def measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg, env_steps, shaping=None,
+                loc_mask=None):
     """The same rollout through the C ABI with pinned HOST arrays: copies are timed.
     env_steps: the (episode, step) pairs one call counts over all ranks."""
     import torch
 
     sh = {} if shaping is None else {"rt0": torch.from_numpy(shaping[0]).pin_memory(),
                                      "mem0": torch.from_numpy(shaping[1]).pin_memory()}
+    if loc_mask is not None:
+        sh["loc_mask"] = torch.from_numpy(loc_mask).pin_memory()
     zh = torch.from_numpy(z0).pin_memory()
     mh = torch.from_numpy(mask).pin_memory()
     hout = {"z": torch.empty((T + 1, B, cfg["z_dim"]), pin_memory=True),
@@ -361,6 +364,11 @@ def run_ours(args) -> None:
     if args.reward == "shaped":
         cfg["reward_mode"] = 1
         shaping = synth.shaping_state(B, shard=rank)
+    if args.xfers:  # hierarchical action: NX xfers (with the NO-OP) x L = A - NX locations
+        NX = args.xfers
+        cfg["n_xfers"] = NX
+        mask, loc_mask = synth.hier_masks(T, B, NX, cfg["a_dim"] - NX,
+                                          synth.WORKLOADS[name]["mask_density"], shard=rank)
     P = args.population
     if P:
         if B % P or (B // P) % 256:
@@ -375,6 +383,8 @@ def run_ours(args) -> None:
     mc = torch.from_numpy(mask).to(dev)
     sh_dev = {} if shaping is None else {"rt0": torch.from_numpy(shaping[0]).to(dev),
                                          "mem0": torch.from_numpy(shaping[1]).to(dev)}
+    if args.xfers:
+        sh_dev["loc_mask"] = torch.from_numpy(loc_mask).to(dev)
     ep0 = rank * B
     out = {"z": torch.empty((T + 1, B, cfg["z_dim"]), device=dev),
            "actions": torch.empty((T, B), dtype=torch.int32, device=dev),
@@ -444,7 +454,7 @@ def run_ours(args) -> None:
         e2e_value, h2d, d2h = None, 0, 0
     else:
         e2e_value, h2d, d2h = measure_e2e(model, z0, mask, T, ep0, args, flush, dev, ws, B, cfg,
-                                          env_steps, shaping)
+                                          env_steps, shaping, loc_mask if args.xfers else None)
 
     # roofline of the dominant kernel: its algorithmic FLOPs per launch over its own
     # event-timed average launch duration inside the timed region
@@ -482,7 +492,8 @@ def run_ours(args) -> None:
             "vs_baseline": None, "dtype": "bf16" if cfg["precision"] == "bf16" else "f32",
             "data": "synthetic (seeded: weights N(0,0.05^2), z0 N(0,1), Bernoulli masks)",
             "config": {"workload": (name + ("+shaped_reward" if shaping is not None else "")
-                                    + (f"+population{P}" if P else ""))
+                                    + (f"+population{P}" if P else "")
+                                    + (f"+hierarchical{args.xfers}" if args.xfers else ""))
                        if args.batch is None else f"{name} with B overridden",
                        "B": B, "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"],
                        "H": cfg["h_dim"], "K": cfg["k_mix"],
@@ -490,6 +501,9 @@ def run_ours(args) -> None:
                        "precision": cfg["precision"], "kernel_path": path_name,
                        "reward": "Eq. 2 on predicted runtime / memory heads (alpha 0.8, beta 0.2, "
                                  "-100 invalid)" if shaping is not None else "linear reward head",
+                       "action": "flat" if not args.xfers else
+                       f"hierarchical: {args.xfers} xfers (incl. NO-OP) x {cfg['a_dim'] - args.xfers} "
+                       "location slots (Sec. 3.1.3)",
                        "population": None if not P else
                        f"{P} controller candidates x {B // P} episodes; log-probs, value head, "
                        "discounted returns (gamma 0.99) and per-candidate fitness in the step",
@@ -635,6 +649,9 @@ def main():
     ap.add_argument("--precision", choices=["fp32", "bf16"], default=None,
                     help="nll workload only: fp32 or bf16 path (default bf16)")
     ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
+    ap.add_argument("--xfers", type=int, default=0,
+                    help="hierarchical action: NX xfers (the last is the NO-OP) and A - NX "
+                         "location slots (Sec. 3.1.3)")
     ap.add_argument("--population", type=int, default=0,
                     help="P controller candidates (B / P episodes each): each step is one "
                          "generation's evaluation (rollout with log-probs and values, returns, "

@@ -113,6 +113,18 @@ typedef struct {
                                          (a critic on the world model's state, for
                                          PPO-style training); stepwise and tensor
                                          families                                   */
+    /* Hierarchical action (Sec. 3.1.3): n_xfers = NX > 0 splits the A controller
+     * outputs into NX xfer logits (xfer NX-1 is the NO-OP) and L = A - NX location
+     * logits.  The xfer is chosen among the valid ones (bits 0..NX-1 of the step's
+     * mask words), then the location among the valid ones of the chosen xfer's
+     * location mask (io.loc_mask); a tempered draw takes the controller uniform's
+     * word 0 for the xfer and word 1 for the location.  The NO-OP takes no
+     * location (and ends the episode with noop_terminates); an xfer with no valid
+     * location gives location -1, an invalid action.  The LSTM input is
+     * onehot(xfer) || onehot(location): action rows xfer and NX + location of
+     * W_lstm.  0 = one flat action of A.  Stepwise and tensor-core families;
+     * rollouts only (wm_mdn_nll returns WM_ERR_UNSUPPORTED).                  */
+    int n_xfers;
 } wm_config;
 
 enum { WM_REWARD_HEAD = 0, WM_REWARD_SHAPED = 1 };
@@ -168,6 +180,11 @@ typedef struct {
                                     actions (Sec. 3.4); 0 if ctrl_tau = 0, no action was
                                     valid, or the episode is frozen                    */
     float *value_seq;            /* [T,B]   optional (value_head): V(h_{t+1}); 0 if frozen */
+    /* hierarchical action (n_xfers > 0) only: */
+    const uint32_t *loc_mask;    /* [T,B,NX,ceil(L/32)] or NULL = all valid: bit j of
+                                    xfer x's words set = location j valid for x       */
+    int32_t *loc_actions;        /* [T,B]   optional: the location taken (-1: none;
+                                    `actions` holds the xfer)                         */
 } wm_rollout_io;
 
 /* Creates a world model on the current CUDA device from the weights of the
@@ -189,7 +206,7 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *weights, wm_handle *
 wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offset,
                      unsigned int t0, const wm_rollout_io *io, void *cuda_stream);
 
-/* Teacher-forced scoring (a9): runs the LSTM over the given latents and
+/* Teacher-forced scoring (a9) of a flat-action model: runs the LSTM over the given latents and
  * actions from h = c = 0 and returns the per-sequence mixture NLL in nats.
  *   z_seq   [T+1,N,Z] latents; step t reads z_seq[t] and scores z_seq[t+1]
  *   actions [T,N]     in [0,A) or negative for no action row

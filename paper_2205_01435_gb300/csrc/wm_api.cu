@@ -211,7 +211,8 @@ bool valid_cfg(const wm_config *c) {
            c->ctrl_tau >= 0.f && c->path >= WM_PATH_AUTO && c->path <= WM_PATH_TENSOR &&
            c->z_dim <= 4096 && c->a_dim <= 65536 && c->h_dim <= 16384 &&
            (c->fused_cluster == 0 || c->fused_cluster == 8 || c->fused_cluster == 16) &&
-           (c->reward_mode == WM_REWARD_HEAD || c->reward_mode == WM_REWARD_SHAPED);
+           (c->reward_mode == WM_REWARD_HEAD || c->reward_mode == WM_REWARD_SHAPED) &&
+           c->n_xfers >= 0 && c->n_xfers < c->a_dim;
 }
 
 cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
@@ -497,6 +498,11 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
     st.add((void **)&a.mdn_seq, io->mdn_seq, t * b * M * 4, true, STEP_OUT, b * M * 4);
     st.add((void **)&a.comp_seq, io->comp_seq, t * b * Z, true, STEP_OUT, b * Z);
     st.add((void **)&a.logp_seq, io->logp_seq, t * b * 4, true, STEP_OUT, b * 4);
+    if (c.n_xfers > 0) {
+        const size_t WL = (A - c.n_xfers + 31) / 32, NX = c.n_xfers;
+        st.add((void **)&a.loc_mask, io->loc_mask, t * b * NX * WL * 4, false, STEP_IN, b * NX * WL * 4);
+        st.add((void **)&a.loc_actions, io->loc_actions, t * b * 4, true, STEP_OUT, b * 4);
+    }
     if (c.value_head) st.add((void **)&a.value_seq, io->value_seq, t * b * 4, true, STEP_OUT, b * 4);
     if (shaped) {
         st.add((void **)&a.rt0, io->rt0, b * 4, false);
@@ -507,7 +513,7 @@ wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offs
 
     // the fused family writes no log-probs or values and has one controller; the tensor
     // family needs a population's candidates aligned to its 256-row tiles
-    const bool fused_ok = !io->logp_seq && !(c.value_head && io->value_seq) && h->P == 1;
+    const bool fused_ok = !io->logp_seq && !(c.value_head && io->value_seq) && h->P == 1 && c.n_xfers == 0;
     const bool tc_ok = wm_tc_call_ok(h, episode_offset) != 0;
     int path = pick_path(h, B, fused_ok, tc_ok);
     if (path == WM_PATH_FUSED && !(fused_ok && wm_fused_supported(h, B)))
@@ -619,6 +625,8 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
     if (N > 0 && (!z_seq || !nll || (T > 0 && !actions)))
         return fail(h, WM_ERR_INVALID_ARG, "z_seq, actions and nll are required");
     const wm_config &c = h->cfg;
+    if (c.n_xfers > 0)
+        return fail(h, WM_ERR_UNSUPPORTED, "teacher-forced scoring takes flat-action models only");
     const size_t Z = c.z_dim, H = c.h_dim, M = h->M, n = (size_t)N, t = (size_t)T;
     if (actions && is_host_ptr(actions))
         for (size_t i = 0; i < n * t; ++i)

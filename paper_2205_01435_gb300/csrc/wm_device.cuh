@@ -79,6 +79,94 @@ __device__ __forceinline__ float uniform_for_dim(unsigned long long seed, unsign
     return to_uniform(u32x4_get(v, d & 3));
 }
 
+// Bit j of a mask row (null: every action valid).
+__device__ __forceinline__ bool action_valid(const uint32_t *mw, int j) {
+    return !mw || ((mw[j >> 5] >> (j & 31)) & 1u);
+}
+
+// One warp's controller choice over n logits (Sec. 3.4, masks of Sec. 3.1.3).
+struct WarpSelect {
+    bool sample;                     // tempered draw (else masked argmax)
+    float tau;                       // controller temperature
+    bool want_lp;                    // compute the log-prob of the choice
+    unsigned long long seed, episode;
+    uint32_t step;
+};
+
+// log pi(a) under softmax(l / tau) over the valid of n actions (every lane returns it)
+__device__ inline float warp_logp(const float *l, int n, const uint32_t *mw, int a, float lmax, float tau) {
+    const int lane = threadIdx.x & 31;
+    float S = 0.f;
+    for (int j = lane; j < n; j += 32)
+        if (action_valid(mw, j)) S += expf((l[j] - lmax) / tau);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
+    return (l[a] - lmax) / tau - logf(S);
+}
+
+// Masked argmax (lowest index on ties) or a tempered draw by inverse CDF with word `word` of
+// the controller's Philox block, over the n logits l with mask words mw (or null).  Returns
+// the choice (-1: nothing valid); with want_lp, *logp receives its log-prob under
+// softmax(l / tau) over the valid actions (0 if none, or tau = 0).  Called by a full warp.
+__device__ inline int warp_select(const WarpSelect &s, const float *l, int n, const uint32_t *mw, int word,
+                                  float *logp) {
+    const int lane = threadIdx.x & 31;
+    const int A = n;
+    float bv = -INFINITY;
+    int bi = -1;
+    for (int j = lane; j < A; j += 32) {
+        if (!action_valid(mw, j)) continue;
+        float v = l[j];
+        if (bi < 0 || v > bv) { bv = v; bi = j; }
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+        float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+        int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+        bool take = oi >= 0 && (bi < 0 || ov > bv || (ov == bv && oi < bi));
+        if (take) { bv = ov; bi = oi; }
+    }
+    *logp = 0.f;
+    if (bi < 0) return bi;
+    if (!s.sample) {
+        if (s.want_lp && s.tau > 0.f) *logp = warp_logp(l, A, mw, bi, bv, s.tau);
+        return bi;
+    }
+    const float tau = s.tau;
+    float S = 0.f;
+    for (int j = lane; j < A; j += 32)
+        if (action_valid(mw, j)) S += expf((l[j] - bv) / tau);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
+    const u32x4 rc = rng_draw(s.seed, s.episode, s.step, RNG_CONTROLLER, 0);
+    const float u = to_uniform(word ? rc.y : rc.x);
+    const float target = u * S;
+    float run = 0.f;
+    int last = -1;
+    for (int j0 = 0; j0 < A; j0 += 32) {
+        int j = j0 + lane;
+        bool ok = j < A && action_valid(mw, j);
+        float sc = ok ? expf((l[j] - bv) / tau) : 0.f;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            float o = __shfl_up_sync(0xffffffffu, sc, off);
+            if (lane >= off) sc += o;
+        }
+        float cum = run + sc;
+        unsigned hit = __ballot_sync(0xffffffffu, ok && target < cum);
+        unsigned okm = __ballot_sync(0xffffffffu, ok);
+        if (okm) last = j0 + 31 - __clz(okm);
+        if (hit) {
+            const int a = j0 + __ffs(hit) - 1;
+            if (s.want_lp) *logp = (l[a] - bv) / tau - logf(S);
+            return a;
+        }
+        run += __shfl_sync(0xffffffffu, sc, 31);
+    }
+    if (s.want_lp && last >= 0) *logp = (l[last] - bv) / tau - logf(S);
+    return last;
+}
+
 // Records a device-side error in the status word unless one is already recorded
 // (wm_sync returns the first).
 __device__ __forceinline__ void report_status(int *status, int code) {

@@ -39,6 +39,8 @@ struct wm_rollout_dev {
     float *rt_seq, *mem_seq;   // shaped reward: predictions after each step (optional)
     float *logp_seq;           // log-prob of the action taken (optional)
     float *value_seq;          // value head V(h_{t+1}) (optional)
+    const uint32_t *loc_mask;  // hierarchical action: [T, B, NX, WL] location masks (or null)
+    int32_t *loc_actions;      // hierarchical action: the location taken (optional)
 };
 
 // Device pointers of one teacher-forced scoring call.

@@ -84,7 +84,9 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
                           io->mdn_seq, io->comp_seq, shaped ? io->rt0 : nullptr,
                           shaped ? io->mem0 : nullptr, shaped ? io->rt_seq : nullptr,
                           shaped ? io->mem_seq : nullptr, io->logp_seq,
-                          h->cfg.value_head ? io->value_seq : nullptr};
+                          h->cfg.value_head ? io->value_seq : nullptr,
+                          h->cfg.n_xfers > 0 ? io->loc_mask : nullptr,
+                          h->cfg.n_xfers > 0 ? io->loc_actions : nullptr};
     for (const void *p : ptrs)
         if (!device_accessible(p))
             return fail(h, WM_ERR_INVALID_ARG,
@@ -106,6 +108,10 @@ extern "C" wm_status wm_rollout_noalloc(wm_handle *h, int B, int T, unsigned lon
     }
     a.logp_seq = io->logp_seq;
     a.value_seq = h->cfg.value_head ? io->value_seq : nullptr;
+    if (h->cfg.n_xfers > 0) {
+        a.loc_mask = io->loc_mask;
+        a.loc_actions = io->loc_actions;
+    }
     e = wm_step_rollout(h, a, scratch, (cudaStream_t)cuda_stream);
     if (e != cudaSuccess) return fail(h, WM_ERR_CUDA, "wm_rollout_noalloc launch failed");
     h->last_path = WM_PATH_STEPWISE;

@@ -126,11 +126,12 @@ struct StepParams {
     float *logp_seq;      // log pi(a_t | z_t, h_t) of the action taken (optional)
     float *value_seq;     // value head, heads column value_col (optional)
     int value_col;
+    // hierarchical action: n_xfers xfer logits, then A - n_xfers location logits
+    int n_xfers;
+    const uint32_t *loc_mask;  // [T, B, NX, WL] or null
+    int32_t *loc_out;          // [T, B] the location taken (optional)
+    int32_t *loc_cur;          // [B] this step's location (workspace)
 };
-
-__device__ __forceinline__ bool action_valid(const uint32_t *mw, int j) {
-    return !mw || ((mw[j >> 5] >> (j & 31)) & 1u);
-}
 
 // a1 for a controller population: the logits of each episode's candidate into the
 // controller columns of G.  One block per episode, the input [z_t; h_t] staged in
@@ -154,86 +155,46 @@ __global__ void __launch_bounds__(128) k_ctrl_pop(StepParams p, const float *__r
     }
 }
 
-// log pi(a) under softmax(l / tau) over the valid actions (one warp; every lane returns it)
-__device__ float action_logp_warp(const StepParams &p, const float *l, const uint32_t *mw, int a, float lmax) {
-    const int lane = threadIdx.x & 31;
-    const float tau = p.ctrl_tau;
-    float S = 0.f;
-    for (int j = lane; j < p.A; j += 32)
-        if (action_valid(mw, j)) S += expf((l[j] - lmax) / tau);
-#pragma unroll
-    for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
-    return (l[a] - lmax) / tau - logf(S);
+// a2 on one warp over the n logits l: the shared masked argmax / tempered draw.
+__device__ int select_warp(const StepParams &p, const float *l, int n, const uint32_t *mw, int b, int word,
+                           float *logp) {
+    WarpSelect ws;
+    ws.sample = p.ctrl_sample && p.ctrl_tau > 0.f;
+    ws.tau = p.ctrl_tau;
+    ws.want_lp = p.logp_seq != nullptr;
+    ws.seed = p.seed;
+    ws.episode = p.ep0 + b;
+    ws.step = p.step;
+    return warp_select(ws, l, n, mw, word, logp);
 }
 
-// a2 on one warp: masked argmax (lowest index on ties) or a tempered draw.  With
-// p.logp_seq, *logp receives log pi(a) of the chosen action (0 if none or tau = 0).
-__device__ int select_action_warp(const StepParams &p, int b, float *logp) {
-    const int lane = threadIdx.x & 31;
+// The step's action: one flat choice of A, or (Sec. 3.1.3) the xfer among the first NX
+// logits, then the location among the other L under the chosen xfer's location mask.
+// Returns the action (the xfer); *loc receives the location (-1: none), *logp the log-prob
+// of the whole action.
+__device__ int select_action_warp(const StepParams &p, int b, int *loc, float *logp) {
     const float *l = p.G + (long)b * p.ldg + 4 * p.H;
-    const int A = p.A, W = (A + 31) >> 5;
+    const int A = p.A, W = (A + 31) >> 5, NX = p.n_xfers;
     const uint32_t *mw = p.mask ? p.mask + ((size_t)p.t * p.B + b) * W : nullptr;
-    float bv = -INFINITY;
-    int bi = -1;
-    for (int j = lane; j < A; j += 32) {
-        if (!action_valid(mw, j)) continue;
-        float v = l[j];
-        if (bi < 0 || v > bv) { bv = v; bi = j; }
+    *loc = -1;
+    if (NX == 0) return select_warp(p, l, A, mw, b, 0, logp);
+    const int L = A - NX, WL = (L + 31) >> 5;
+    const int x = select_warp(p, l, NX, mw, b, 0, logp);
+    if (x >= 0 && x != NX - 1) {
+        const uint32_t *lmw = p.loc_mask ? p.loc_mask + (((size_t)p.t * p.B + b) * NX + x) * WL : nullptr;
+        float lpl = 0.f;
+        *loc = select_warp(p, l + NX, L, lmw, b, 1, &lpl);
+        *logp += lpl;
     }
-#pragma unroll
-    for (int off = 16; off; off >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        bool take = oi >= 0 && (bi < 0 || ov > bv || (ov == bv && oi < bi));
-        if (take) { bv = ov; bi = oi; }
-    }
-    *logp = 0.f;
-    if (bi < 0) return bi;
-    if (!p.ctrl_sample || !(p.ctrl_tau > 0.f)) {
-        if (p.logp_seq && p.ctrl_tau > 0.f) *logp = action_logp_warp(p, l, mw, bi, bv);
-        return bi;
-    }
-
-    const float tau = p.ctrl_tau;
-    float S = 0.f;
-    for (int j = lane; j < A; j += 32)
-        if (action_valid(mw, j)) S += expf((l[j] - bv) / tau);
-#pragma unroll
-    for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
-    const float u = to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x);
-    const float target = u * S;
-    float run = 0.f;
-    int last = -1;
-    for (int j0 = 0; j0 < A; j0 += 32) {
-        int j = j0 + lane;
-        bool ok = j < A && action_valid(mw, j);
-        float sc = ok ? expf((l[j] - bv) / tau) : 0.f;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            float o = __shfl_up_sync(0xffffffffu, sc, off);
-            if (lane >= off) sc += o;
-        }
-        float cum = run + sc;
-        unsigned hit = __ballot_sync(0xffffffffu, ok && target < cum);
-        unsigned okm = __ballot_sync(0xffffffffu, ok);
-        if (okm) last = j0 + 31 - __clz(okm);
-        if (hit) {
-            const int a = j0 + __ffs(hit) - 1;
-            if (p.logp_seq) *logp = (l[a] - bv) / tau - logf(S);
-            return a;
-        }
-        run += __shfl_sync(0xffffffffu, sc, 31);
-    }
-    if (p.logp_seq && last >= 0) *logp = (l[last] - bv) / tau - logf(S);
-    return last;
+    return x;
 }
 
 __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
     const int b = blockIdx.x;
-    __shared__ int s_a;
+    __shared__ int s_a, s_a2;
     const bool fz = p.frozen[b] != 0;
     if (threadIdx.x < 32) {
-        int a;
+        int a, loc = -1;
         float lp = 0.f;
         if (fz) {
             a = -1;
@@ -242,18 +203,24 @@ __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
             if (a >= p.A) report_status(p.status, WM_ERR_INVALID_ARG);
             if (a >= p.A || a < 0) a = -1;
         } else {
-            a = select_action_warp(p, b, &lp);
+            a = select_action_warp(p, b, &loc, &lp);
         }
         if (threadIdx.x == 0) {
             s_a = a;
+            s_a2 = loc >= 0 ? p.n_xfers + loc : -1;  // the location's action row
             if (!p.teacher) p.act_out[(size_t)p.t * p.B + b] = a;
             if (!p.teacher && p.logp_seq) p.logp_seq[(size_t)p.t * p.B + b] = lp;
+            if (p.n_xfers > 0 && !p.teacher) {
+                p.loc_cur[b] = loc;
+                if (p.loc_out) p.loc_out[(size_t)p.t * p.B + b] = loc;
+            }
         }
     }
     __syncthreads();
-    const int a = s_a, H = p.H;
+    const int a = s_a, a2 = s_a2, H = p.H;
     const float *g = p.G + (long)b * p.ldg;
     const float *wa = a >= 0 ? p.Wa + (size_t)a * 4 * H : nullptr;
+    const float *wa2 = a2 >= 0 ? p.Wa + (size_t)a2 * 4 * H : nullptr;
     for (int u = threadIdx.x; u < H; u += blockDim.x) {
         const size_t i = (size_t)b * H + u;
         float hv, cv;
@@ -263,6 +230,7 @@ __global__ void __launch_bounds__(256) k_select_cell(StepParams p) {
         } else {
             float gi = g[u], gf = g[H + u], gg = g[2 * H + u], go = g[3 * H + u];
             if (wa) { gi += wa[u]; gf += wa[H + u]; gg += wa[2 * H + u]; go += wa[3 * H + u]; }
+            if (wa2) { gi += wa2[u]; gf += wa2[H + u]; gg += wa2[2 * H + u]; go += wa2[3 * H + u]; }
             cv = sigmoidf_(gf) * p.c[i] + sigmoidf_(gi) * tanhf(gg);
             hv = sigmoidf_(go) * tanhf(cv);
             p.c[i] = cv;
@@ -387,10 +355,13 @@ __global__ void __launch_bounds__(128) k_sample(StepParams p) {
             float r = row[M];
             const float dl = row[M + 1];
             const int a = p.act_out[tb];
-            const bool noop = p.noop_terminates && a == p.A - 1;
+            const int noop_a = p.n_xfers > 0 ? p.n_xfers - 1 : p.A - 1;
+            const bool noop = p.noop_terminates && a == noop_a;
             if (shaped) {  // Eq. 2 on the predictions entering and leaving the step
                 const float rt = row[M + 2], mem = row[M + 3];
-                r = a >= 0 ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
+                // valid: an action was taken (and, for an xfer, a location)
+                const bool ok = a >= 0 && (p.n_xfers == 0 || a == noop_a || p.loc_cur[b] >= 0);
+                r = ok ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
                 p.rt[b] = rt;
                 p.mem[b] = mem;
             }
@@ -442,6 +413,7 @@ inline size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
 struct StepWs {
     float *G, *heads, *h, *c;
     float *rt, *mem;  // shaped reward: each episode's last predictions
+    int32_t *loc;     // hierarchical action: the step's location
     uint8_t *frozen;
     double *nll_acc;
 };
@@ -453,7 +425,8 @@ size_t step_ws_bytes(const wm_handle *hd, int B, bool teacher) {
     s += align_up((size_t)B * (4 * H + A) * 4);
     s += align_up((size_t)B * (M + NR) * 4);
     s += 2 * align_up((size_t)B * H * 4);
-    if (NR == 4) s += 2 * align_up((size_t)B * 4);
+    if (c.reward_mode == WM_REWARD_SHAPED) s += 2 * align_up((size_t)B * 4);
+    s += align_up((size_t)B * 4);
     s += align_up((size_t)B);
     if (teacher) s += align_up((size_t)B * 8);
     return s;
@@ -468,10 +441,11 @@ StepWs carve(const wm_handle *hd, int B, void *ws, bool teacher) {
     w.heads = (float *)p; p += align_up((size_t)B * (M + NR) * 4);
     w.h = (float *)p; p += align_up((size_t)B * H * 4);
     w.c = (float *)p; p += align_up((size_t)B * H * 4);
-    if (NR == 4) {
+    if (c.reward_mode == WM_REWARD_SHAPED) {
         w.rt = (float *)p; p += align_up((size_t)B * 4);
         w.mem = (float *)p; p += align_up((size_t)B * 4);
     }
+    w.loc = (int32_t *)p; p += align_up((size_t)B * 4);
     w.frozen = (uint8_t *)p; p += align_up((size_t)B);
     w.nll_acc = teacher ? (double *)p : nullptr;
     return w;
@@ -513,6 +487,8 @@ StepParams base_params(const wm_handle *hd, int B, int T, const StepWs &w) {
     p.P = hd->P; p.E = hd->E;
     p.Wp = hd->step.Wp; p.bp = hd->step.bp;
     p.value_col = hd->M + hd->NR - 1;
+    p.n_xfers = c.n_xfers;
+    p.loc_cur = w.loc;
     return p;
 }
 
@@ -545,6 +521,8 @@ cudaError_t wm_step_rollout(const wm_handle *hd, const wm_rollout_dev &a, void *
     p.rt_seq = a.rt_seq; p.mem_seq = a.mem_seq;
     p.logp_seq = a.logp_seq;
     p.value_seq = c.value_head ? a.value_seq : nullptr;
+    p.loc_mask = a.loc_mask;
+    p.loc_out = a.loc_actions;
     const int NH = hd->M + hd->NR;  // head GEMM columns
     const bool pop = hd->P > 1;     // controller logits per candidate, in k_ctrl_pop
     for (int t = 0; t < T; ++t) {

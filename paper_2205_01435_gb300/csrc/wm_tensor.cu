@@ -176,6 +176,14 @@ struct StepIO {
     float *logp_seq;                // log pi(a_t | z_t, h_t) of the action taken (optional)
     float *value_seq;               // value head at head column rd_col + nr - 1 (optional)
     int nr;                         // head columns from rd_col: reward, done (, rt, mem) (, value)
+    // hierarchical action (n_xfers > 0): the controller GEMM writes its logits, a selection
+    // kernel picks the xfer (act) and the location, whose action row n_xfers + location is
+    // act2 (-1: none)
+    int n_xfers;
+    float *logits;                  // [B, A]
+    const uint32_t *loc_mask;       // [T, B, NX, WL] or null
+    int32_t *loc_actions;           // [T, B] optional
+    int32_t *act2;                  // [B]
 };
 
 // Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
@@ -445,6 +453,81 @@ struct EpiCtrl {
 };
 
 
+// ---- controller logits epilogue (hierarchical actions): every live row's A logits plus
+// its candidate's bias to a [B, A] buffer; the two-stage choice is made by k_tc_select.
+// Column group g stores its A/4 columns, 16 at a time (64 contiguous bytes per row).
+struct EpiLogits {
+    static constexpr bool TMA_STAGE = false;
+    static constexpr uint32_t QUAD_STAGE = 0;
+    static constexpr uint32_t RED_BYTES = 0;
+    struct Pre {};
+    static __device__ void init(const StepIO &, EpiCtx &, int) {}
+    static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
+    static __device__ void pre(const StepIO &, int, int, EpiCtx &, Pre &) {}
+    static __device__ void run(const StepIO &p, uint32_t tacc, int m, int, EpiCtx &x, const Pre &, int, int) {
+        const int b = m * BM + x.row;
+        const bool store = b < p.B && !p.fz_cur[b < p.B ? b : 0];  // frozen rows choose nothing
+        const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
+        const unsigned long long cand =
+            p.pop_P > 1 ? ((p.ep0 + (unsigned long long)m * BM) / (unsigned long long)p.pop_E) % (unsigned long long)p.pop_P
+                        : 0ull;
+        const float *bias = p.b_ctrl + cand * p.A;
+        float *out = p.logits + (size_t)(b < p.B ? b : 0) * p.A;
+        for (int k = 0; k < nch; ++k) {  // every lane issues the (warp-collective) TMEM loads
+            const int c0 = c_lo + 16 * k;
+            uint32_t r[16];
+            TC_LD16(tacc + c0, r);
+            tc::tmem_ld_wait();
+            if (!store) continue;
+            const float4 *b4 = reinterpret_cast<const float4 *>(bias + c0);
+            float4 *o4 = reinterpret_cast<float4 *>(out + c0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float4 t = b4[i];
+                o4[i] = make_float4(__uint_as_float(r[4 * i]) + t.x, __uint_as_float(r[4 * i + 1]) + t.y,
+                                    __uint_as_float(r[4 * i + 2]) + t.z, __uint_as_float(r[4 * i + 3]) + t.w);
+            }
+        }
+    }
+};
+
+// The hierarchical choice (Sec. 3.1.3) from the stored logits, one warp per episode: the
+// xfer among the first NX under the xfer mask, then (unless it is the NO-OP) the location
+// among the other L under that xfer's location mask.
+__global__ void __launch_bounds__(256) k_tc_select(StepIO p) {
+    const int warp = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (warp >= p.B) return;
+    const int b = warp, A = p.A, NX = p.n_xfers, L = A - NX, W = (A + 31) >> 5, WL = (L + 31) >> 5;
+    const size_t tb = (size_t)p.t * p.B + b;
+    int x = -1, loc = -1;
+    float lp = 0.f;
+    if (!p.fz_cur[b]) {
+        WarpSelect ws;
+        ws.sample = p.ctrl_sample && p.ctrl_tau > 0.f;
+        ws.tau = p.ctrl_tau;
+        ws.want_lp = p.logp_seq != nullptr;
+        ws.seed = p.seed;
+        ws.episode = p.ep0 + b;
+        ws.step = p.step;
+        const float *l = p.logits + (size_t)b * A;
+        const uint32_t *mw = p.mask ? p.mask + tb * W : nullptr;
+        x = warp_select(ws, l, NX, mw, 0, &lp);
+        if (x >= 0 && x != NX - 1) {
+            const uint32_t *lmw = p.loc_mask ? p.loc_mask + (tb * NX + x) * WL : nullptr;
+            float lpl = 0.f;
+            loc = warp_select(ws, l + NX, L, lmw, 1, &lpl);
+            lp += lpl;
+        }
+    }
+    if (lane == 0) {
+        p.act[b] = x;
+        p.act2[b] = loc >= 0 ? NX + loc : -1;
+        p.actions[tb] = x;
+        if (p.loc_actions) p.loc_actions[tb] = loc;
+        if (p.logp_seq) p.logp_seq[tb] = lp;
+    }
+}
+
 // ---- gate epilogue: 64 units per tile, columns [i | f | g | o] x 64; 16 units per group
 // The quadrant's c rows (32 x 64 fp32) and h' rows (32 x 64 bf16) go through
 // shared memory in the 128-byte-swizzled layout of TMA boxes 128 bytes wide,
@@ -454,8 +537,10 @@ struct EpiCtrl {
 // the stores have read the slab.  (Separate in- and out-slabs, refilled
 // mid-tile, measured slower: the extra quadrant barrier costs more than the
 // load latency it hides.)  The cell is formed gate by gate over the thread's 16
-// units, so that each gate's W_a segment is one 256-bit load.
-struct EpiGates {
+// units, so that each gate's W_a segment is one 256-bit load.  TWO: a hierarchical action
+// adds a second action row (the location's) to every gate.
+template <bool TWO>
+struct EpiGatesT {
     static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
     static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
     static constexpr uint32_t QUAD_STAGE = C_SLAB + X_SLAB;  // c (in place) | h' out
@@ -474,9 +559,10 @@ struct EpiGates {
     }
 
     struct Pre {
-        uint32_t wi[8], wg[8];  // the W_a row segments of gates i and g (16 units, bf16)
-        int a;                  // the action (-1: none)
-        bool fz;                // frozen episode
+        uint32_t wi[8], wg[8];    // the W_a row segments of gates i and g (16 units, bf16)
+        uint32_t wi2[8], wg2[8];  // TWO: the second action row's
+        int a, a2;                // the action rows (-1: none)
+        bool fz;                  // frozen episode
     };
     static __device__ void init(const StepIO &, EpiCtx &, int) {}
     // one gate's W_a segment for the thread's 16 units: a single 32-byte sector, read with
@@ -508,10 +594,18 @@ struct EpiGates {
         pr.a = (a >= 0 && !pr.fz) ? a : -1;
         ld_wa(p, pr.a, n, x.cg, 0, pr.wi);
         ld_wa(p, pr.a, n, x.cg, 2, pr.wg);
+        if (TWO) {
+            const int a2 = p.act2[bb];
+            pr.a2 = (a2 >= 0 && !pr.fz) ? a2 : -1;
+            ld_wa(p, pr.a2, n, x.cg, 0, pr.wi2);
+            ld_wa(p, pr.a2, n, x.cg, 2, pr.wg2);
+        }
     }
     // pre-activations of one gate for the thread's 16 units: accumulator + bias + W_a[a]
+    // (+ W_a[a2] when TWO)
     static __device__ __forceinline__ void gate_pre(uint32_t tacc, const float *bg, int gate, int ut,
-                                                    const uint32_t (&w)[8], float (&g)[16]) {
+                                                    const uint32_t (&w)[8], const uint32_t (&w2)[8],
+                                                    float (&g)[16]) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {  // 8 columns per TMEM load: fewer registers held
             uint32_t r[8];
@@ -528,6 +622,11 @@ struct EpiGates {
                     const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&w[k / 2]);
                     g[k] = __uint_as_float(r[4 * i + 2 * e]) + bv[2 * e] + __low2float(v2);
                     g[k + 1] = __uint_as_float(r[4 * i + 2 * e + 1]) + bv[2 * e + 1] + __high2float(v2);
+                    if (TWO) {
+                        const __nv_bfloat162 u2 = *reinterpret_cast<const __nv_bfloat162 *>(&w2[k / 2]);
+                        g[k] += __low2float(u2);
+                        g[k + 1] += __high2float(u2);
+                    }
                 }
             }
         }
@@ -542,9 +641,13 @@ struct EpiGates {
         const bool fz = pr.fz;
         const int ut = 16 * q, u0 = 64 * n + ut;  // the thread's first unit: in the tile, in H
         // gates f and o: loaded while i and g are computed
-        uint32_t wf[8], wo[8];
+        uint32_t wf[8], wo[8], wf2[8], wo2[8];
         ld_wa(p, pr.a, n, q, 1, wf);
         ld_wa(p, pr.a, n, q, 3, wo);
+        if (TWO) {
+            ld_wa(p, pr.a2, n, q, 1, wf2);
+            ld_wa(p, pr.a2, n, q, 3, wo2);
+        }
         const float *bg = p.b_gate + 256 * n + 16 * q;
         const bool store_h32 = valid && !fz && (p.h32_mode == 2 || (p.h32_mode == 1 && p.t == p.T - 1));
         unsigned char *cs = x.stage, *xs = x.stage + C_SLAB;
@@ -555,10 +658,10 @@ struct EpiGates {
         float cv[16], hv[16];
         {  // hv = sigma(i) * tanh(g), one gate's pre-activations live at a time
             float g[16];
-            gate_pre(tacc, bg, 0, ut, pr.wi, g);
+            gate_pre(tacc, bg, 0, ut, pr.wi, pr.wi2, g);
 #pragma unroll
             for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]);
-            gate_pre(tacc, bg, 2, ut, pr.wg, g);
+            gate_pre(tacc, bg, 2, ut, pr.wg, pr.wg2, g);
 #pragma unroll
             for (int j = 0; j < 16; ++j) hv[j] *= tanh_hw(g[j]);
         }
@@ -570,12 +673,12 @@ struct EpiGates {
         }
         {
             float g[16];
-            gate_pre(tacc, bg, 1, ut, wf, g);
+            gate_pre(tacc, bg, 1, ut, wf, wf2, g);
             if (!fz) {
 #pragma unroll
                 for (int j = 0; j < 16; ++j) cv[j] = sigmoid_hw(g[j]) * cv[j] + hv[j];
             }
-            gate_pre(tacc, bg, 3, ut, wo, g);
+            gate_pre(tacc, bg, 3, ut, wo, wo2, g);
 #pragma unroll
             for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]) * tanh_hw(cv[j]);
         }
@@ -630,6 +733,9 @@ struct EpiGates {
         }
     }
 };
+
+using EpiGates = EpiGatesT<false>;
+using EpiGates2 = EpiGatesT<true>;
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
 // Before the accumulator wait, the quadrant's 128 threads make the tile's random draws:
@@ -842,12 +948,15 @@ struct EpiHeads {
                 float rew = __uint_as_float(r[0]) + bh[p.rd_col];
                 const float dl = __uint_as_float(r[1]) + bh[p.rd_col + 1];
                 const int a = p.act[b];
-                const bool noop = p.noop_terminates && a == p.A - 1;
+                const int noop_a = p.n_xfers > 0 ? p.n_xfers - 1 : p.A - 1;
+                const bool noop = p.noop_terminates && a == noop_a;
                 if (shaped) {
                     if (!fz) {  // Eq. 2 on the predictions entering and leaving the step
                         const float rt = __uint_as_float(q[0]) + bh[p.rd_col + 2];
                         const float mem = __uint_as_float(q[1]) + bh[p.rd_col + 3];
-                        rew = a >= 0 ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
+                        // valid: an action was taken (and, for an xfer, a location)
+                        const bool ok = a >= 0 && (p.n_xfers == 0 || a == noop_a || p.act2[b] >= 0);
+                        rew = ok ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
                         p.rt[b] = rt;
                         p.mem[b] = mem;
                     }
@@ -1192,6 +1301,8 @@ inline size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
 struct TcWs {
     __nv_bfloat16 *x[2];
     float *c, *h32, *nll_part, *rt, *mem;
+    float *logits;   // hierarchical action: [B, A]
+    int32_t *act2;   // hierarchical action: the location's action row
     int32_t *act;
     uint8_t *fz[2];
 };
@@ -1208,6 +1319,10 @@ TcWs carve_ws(const wm_handle *h, int B, void *ws) {
     for (int i = 0; i < 2; ++i) { w.fz[i] = (uint8_t *)p; p += a256((size_t)B); }
     w.rt = (float *)p; p += a256((size_t)B * 4);
     w.mem = (float *)p; p += a256((size_t)B * 4);
+    if (c.n_xfers > 0) {
+        w.logits = (float *)p; p += a256((size_t)B * c.a_dim * 4);
+        w.act2 = (int32_t *)p; p += a256((size_t)B * 4);
+    }
     w.nll_part = (float *)p;
     return w;
 }
@@ -1223,7 +1338,8 @@ size_t wm_tc_ws(const wm_handle *h, int B) {
     const wm_config &c = h->cfg;
     const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
     return 2 * a256((size_t)B * KX * 2) + 2 * a256((size_t)B * H * 4) + a256((size_t)B * 4) + 2 * a256(B) +
-           2 * a256((size_t)B * 4) + a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256;
+           2 * a256((size_t)B * 4) + a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256 +
+           (c.n_xfers > 0 ? a256((size_t)B * c.a_dim * 4) + a256((size_t)B * 4) : 0);
 }
 
 cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
@@ -1382,6 +1498,14 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     }
     io.pop_P = h->P; io.pop_E = h->E;
     io.nr = h->NR;
+    const bool hier = !teacher && c.n_xfers > 0;
+    io.n_xfers = hier ? c.n_xfers : 0;
+    io.logits = w.logits;
+    io.act2 = w.act2;
+    if (hier) {
+        io.loc_mask = ra->loc_mask;
+        io.loc_actions = ra->loc_actions;
+    }
     if (!teacher) {
         io.logp_seq = ra->logp_seq;
         io.value_seq = c.value_head ? ra->value_seq : nullptr;
@@ -1435,18 +1559,33 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         // the controller's weight rows: the tile's candidate's, when there is a population
         const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status, teacher ? 0ull : ra->ep0, h->P, h->E, A};
         if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
-        if (!teacher) {
+        if (!teacher && !hier) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
             if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
             else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
             else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
             ++launches;
             if (e != cudaSuccess) break;
+        } else if (hier) {  // the logits, then the two-stage choice (Sec. 3.1.3)
+            {
+                wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
+                if (A > 256) e = launch_gemm<256, 2, 2, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+                else if (A > 128) e = launch_gemm<256, 1, 3, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+                else e = launch_gemm<128, 1, 3, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+            }
+            ++launches;
+            if (e != cudaSuccess) break;
+            {
+                wm_ktime kt(h, WM_KERNEL_AUX, s);
+                k_tc_select<<<(unsigned)(((size_t)B * 32 + 255) / 256), 256, 0, s>>>(io);
+            }
+            ++launches;
         }
         const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
         {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
-            e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
+            if (hier) e = launch_gemm<256, 1, 2, EpiGates2, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
+            else e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
         }
         ++launches;
         if (e != cudaSuccess) break;

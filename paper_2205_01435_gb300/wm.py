@@ -38,7 +38,8 @@ class wm_config(C.Structure):
                 ("ctrl_sample", C.c_int), ("ctrl_tau", C.c_float), ("done_terminates", C.c_int),
                 ("noop_terminates", C.c_int), ("seed", C.c_ulonglong), ("path", C.c_int),
                 ("fused_cluster", C.c_int), ("reward_mode", C.c_int), ("reward_alpha", C.c_float),
-                ("reward_beta", C.c_float), ("invalid_reward", C.c_float), ("value_head", C.c_int)]
+                ("reward_beta", C.c_float), ("invalid_reward", C.c_float), ("value_head", C.c_int),
+                ("n_xfers", C.c_int)]
 
 
 class wm_weights(C.Structure):
@@ -54,7 +55,7 @@ class wm_rollout_io(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "z0", "h0", "c0", "done0", "mask", "z_out", "actions", "rewards", "done", "h_final",
         "c_final", "h_seq", "c_seq", "mdn_seq", "comp_seq", "rt0", "mem0", "rt_seq", "mem_seq",
-        "logp_seq", "value_seq")]
+        "logp_seq", "value_seq", "loc_mask", "loc_actions")]
 
 
 def _load():
@@ -130,7 +131,7 @@ def wm_create(cfg: dict, weights: dict):
                   else int(cfg["path"]), int(cfg.get("fused_cluster", 0)),
                   int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
                   float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)),
-                  int(cfg.get("value_head", 0)))
+                  int(cfg.get("value_head", 0)), int(cfg.get("n_xfers", 0)))
     keep = {k: torch.as_tensor(weights[k], dtype=torch.float32).contiguous().cpu()
             for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn", "w_rew", "w_done", "W_ctrl", "b_ctrl",
                       "w_rt", "w_mem", "w_val") if weights.get(k) is not None}
@@ -248,7 +249,7 @@ class WorldModel:
     def rollout(self, z0: torch.Tensor, T: int, mask: torch.Tensor | None = None,
                 episode_offset: int = 0, t0: int = 0, h0=None, c0=None, done0=None,
                 want_final: bool = True, want_seq: bool = False, out: dict | None = None,
-                stream=None, rt0=None, mem0=None, want_logp: bool = False) -> dict:
+                stream=None, rt0=None, mem0=None, want_logp: bool = False, loc_mask=None) -> dict:
         """wm_rollout on B = z0.shape[0] episodes; returns the output tensors (device of z0).
         With the shaped reward, rt0 / mem0 are required and rt_seq / mem_seq are returned;
         want_logp adds logp_seq, and a value head adds value_seq."""
@@ -276,12 +277,15 @@ class WorldModel:
             o.setdefault("logp_seq", self._alloc(z0, (T, B), torch.float32))
         if int(self.cfg.get("value_head", 0)):
             o.setdefault("value_seq", self._alloc(z0, (T, B), torch.float32))
+        if int(self.cfg.get("n_xfers", 0)) > 0:
+            o.setdefault("loc_actions", self._alloc(z0, (T, B), torch.int32))
         io = {"z0": z0, "h0": h0, "c0": c0, "done0": done0, "mask": mask, "z_out": o["z"],
               "actions": o["actions"], "rewards": o["rewards"], "done": o["done"],
               "h_final": o.get("h_final"), "c_final": o.get("c_final"), "h_seq": o.get("h_seq"),
               "c_seq": o.get("c_seq"), "mdn_seq": o.get("mdn_seq"), "comp_seq": o.get("comp_seq"),
               "rt0": rt0, "mem0": mem0, "rt_seq": o.get("rt_seq"), "mem_seq": o.get("mem_seq"),
-              "logp_seq": o.get("logp_seq"), "value_seq": o.get("value_seq")}
+              "logp_seq": o.get("logp_seq"), "value_seq": o.get("value_seq"), "loc_mask": loc_mask,
+              "loc_actions": o.get("loc_actions")}
         with torch.cuda.device(self.device):
             wm_rollout(self.h, B, T, episode_offset, t0, io, self._stream(stream))
         return o

@@ -49,7 +49,7 @@ def np_(x):
 
 def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=None, t0: int = 0,
                   h0=None, c0=None, done0=None, orc=None, nthreads: int = NT, rt0=None,
-                  mem0=None) -> dict:
+                  mem0=None, loc_mask=None) -> dict:
     """Step-anchored parity of a GPU rollout of B episodes.
 
     g: the GPU's outputs with their per-step sequences (z, actions, rewards, done,
@@ -57,7 +57,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
     checked episodes.  z0, mask [T, B, W], h0, c0, done0: the inputs of those
     episodes.  episodes: their global Philox indices (default 0..B-1); t0: the
     global index of step 0.  With the shaped reward, rt0 / mem0 are the predictions
-    entering the call and g carries rt_seq / mem_seq."""
+    entering the call and g carries rt_seq / mem_seq; with a hierarchical action, loc_mask
+    [T, B, NX, WL] are the location masks and g carries loc_actions."""
     if orc is None:
         import oracle as orc
     prec = cfg.get("precision", "fp32")
@@ -76,6 +77,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
     frozen = np.zeros(B, bool) if done0 is None else np.asarray(done0).astype(bool)
     shaped = int(cfg.get("reward_mode", 0)) == 1
     g_lp = np_(g["logp_seq"]) if g.get("logp_seq") is not None else None
+    hier = int(cfg.get("n_xfers", 0)) > 0
+    g_loc = np_(g["loc_actions"]) if hier else None
     g_v = np_(g["value_seq"]) if g.get("value_seq") is not None else None
     if shaped:
         rt, mem = np.asarray(rt0, np.float32), np.asarray(mem0, np.float32)
@@ -96,6 +99,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
         mk = None if mask is None else np.asarray(mask)[t]
         for ri, (rcfg, rtol) in enumerate(refs):
             sk = dict(rt=rt, mem=mem) if shaped else {}
+            if hier:
+                sk.update(loc_use=g_loc[t], loc_mask=None if loc_mask is None else np.asarray(loc_mask)[t])
             s = orc.step(rcfg, weights, ep, t0 + t, gz[t], h, c, frozen=frozen, mask=mk,
                          a_use=ga[t], h_use=gh[t], k_use=gk[t], nthreads=nthreads, **sk)
             if ri == 0:
@@ -135,6 +140,8 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                     assert np.all(g_lp[t, fz] == 0), where
                 if g_v is not None:
                     assert np.all(g_v[t, fz] == 0), where
+                if hier:
+                    assert np.all(g_loc[t, fz] == -1), where
                 st["frozen_steps"] += len(fz)
             # decisions: equal, or excused by the oracle's own margin
             nl = int(live.sum())
@@ -145,6 +152,12 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
                 assert m < ctrl_thr, (f"action {where} episode {ep[b]}: gpu {ga[t, b]} oracle "
                                       f"{s['action'][b]} margin {m}")
                 flip("action", m)
+            if hier:  # the location: a second decision (counted with the action's draws)
+                for b in np.nonzero(live & (g_loc[t] != s["loc"]))[0]:
+                    m = s["loc_margin"][b]
+                    assert m < ctrl_thr, (f"location {where} episode {ep[b]}: gpu {g_loc[t, b]} "
+                                          f"oracle {s['loc'][b]} margin {m}")
+                    flip("action", m)
             for b in np.nonzero(live & (gd[t] != s["done"]))[0]:
                 m = s["done_margin"][b]
                 assert m < DONE_GAP, (f"done {where} episode {ep[b]}: gpu {gd[t, b]} oracle "
@@ -163,7 +176,7 @@ def check_rollout(g: dict, cfg: dict, weights: dict, z0, mask=None, episodes=Non
         if cfg.get("done_terminates"):
             frozen = frozen | (gd[t] == 1)
         if cfg.get("noop_terminates"):
-            frozen = frozen | (ga[t] == A - 1)
+            frozen = frozen | (ga[t] == (int(cfg["n_xfers"]) - 1 if hier else A - 1))
     if T > 0 and g.get("h_final") is not None:
         for key, gv in (("h_final", g["h_final"]), ("c_final", g["c_final"])):
             e = float(np.abs(np_(gv).astype(np.float64)

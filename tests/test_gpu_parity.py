@@ -559,3 +559,47 @@ def test_returns_and_fitness_match_oracle(wm, orc, host):
                     episode_offset=off, pop_size=P, pop_group=E)
     assert np.array_equal(np_(res["returns"]), o["returns"])
     np.testing.assert_allclose(np_(res["fitness"]), o["fitness"], rtol=1e-6)
+
+
+# ------------------------------------------------------------------ hierarchical (xfer, location) action
+@pytest.mark.parametrize("path,name,NX,flags", [
+    ("stepwise", "tiny_fp32", 16, dict(ctrl_sample=1, ctrl_tau=0.9, noop_terminates=1)),
+    ("tensor", "small_bf16", 32, dict(ctrl_sample=1, ctrl_tau=1.0)),
+    # 55 transformations + NO-OP and the paper's 200 location slots
+    ("tensor", "mid_bf16", 56, dict(done_terminates=1, noop_terminates=1, reward_mode=1)),
+    ("tensor", "large_bf16", 112, dict(value_head=1)),
+    ("auto", "small_bf16", 32, dict()),
+])
+def test_hierarchical_action_against_oracle(wm, orc, path, name, NX, flags):
+    """Sec. 3.1.3: the xfer under the xfer mask, then the location under that xfer's location
+    mask; the LSTM takes both one-hot rows.  Step-anchored against the oracle; AUTO never
+    routes it to the fused family, and teacher-forced scoring declines it."""
+    cfg = dict(synth.model_config(name), n_xfers=NX, **flags)
+    w = synth.weights(cfg, seed=18)
+    A = cfg["a_dim"]
+    B, T = (16, 10) if name == "tiny_fp32" else (600, 5)
+    z0 = synth.z0(B, cfg["z_dim"], seed=18)
+    xm, lm = synth.hier_masks(T, B, NX, A - NX, 0.5, seed=18)
+    sh = {}
+    if cfg.get("reward_mode"):
+        rt0, mem0 = synth.shaping_state(B, seed=18)
+        sh = dict(rt0=rt0, mem0=mem0)
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(xm), loc_mask=_cuda(lm), episode_offset=33, t0=2,
+                  want_seq=True, want_logp=True, **{k: _cuda(v) for k, v in sh.items()})
+    torch.cuda.synchronize()
+    assert m.last_path != "fused" and (path == "auto" or m.last_path == path)
+    r = check_rollout(g, cfg, w, z0, xm, episodes=33 + np.arange(B), t0=2, loc_mask=lm, orc=orc, **sh)
+    print("hierarchical", path, name, NX, flags, r)
+    locs = np_(g["loc_actions"])
+    assert (locs >= 0).any() and (np_(g["actions"]) == NX - 1).any() or name == "large_bf16"
+    if path == "tensor" and name == "small_bf16":
+        # host arrays (the location masks staged per step) give the same bits
+        hz, hx, hl = (torch.from_numpy(a).pin_memory() for a in (z0, xm, lm))
+        gh = m.rollout(hz, T, mask=hx, loc_mask=hl, episode_offset=33, t0=2, want_seq=True, want_logp=True)
+        for k in ("actions", "loc_actions", "z", "rewards", "logp_seq"):
+            assert torch.equal(gh[k], g[k].cpu()), k
+    zs, acts, _ = synth.teacher_inputs(4, 3, cfg["z_dim"], A)
+    with pytest.raises(wm.WMError) as ei:
+        m.mdn_nll(_cuda(zs), _cuda(acts))
+    assert ei.value.status == wm.WM_ERR_UNSUPPORTED

@@ -30,7 +30,14 @@ def _case(orc, precision="fp32", **flags):
         kw.update(rt0=rt0, mem0=mem0)
         ck.update(rt0=rt0, mem0=mem0)
         keys += ("rt_seq", "mem_seq")
+    if cfg.get("n_xfers"):
+        mask, lm = synth.hier_masks(T, B, cfg["n_xfers"], 20 - cfg["n_xfers"], 0.6, seed=41)
+        kw.update(loc_mask=lm)
+        ck.update(loc_mask=lm)
     o = orc.rollout(cfg, w, z0, mask, T, want_seq=True, **kw)
+    if cfg.get("n_xfers"):
+        o["loc_actions"] = o["loc_seq"]
+        keys += ("loc_actions",)
     g = {k: o[k].copy() for k in keys}
     return cfg, w, z0, mask, g, o, ck
 
@@ -38,7 +45,9 @@ def _case(orc, precision="fp32", **flags):
 @pytest.mark.parametrize("precision,flags", [("fp32", {}), ("bf16", {}),
                                              ("fp32", dict(done_terminates=1, noop_terminates=1)),
                                              ("fp32", dict(ctrl_sample=1, ctrl_tau=0.8)),
-                                             ("bf16", dict(reward_mode=1, done_terminates=1))])
+                                             ("bf16", dict(reward_mode=1, done_terminates=1)),
+                                             ("fp32", dict(n_xfers=7, noop_terminates=1, ctrl_sample=1,
+                                                           ctrl_tau=0.9))])
 def test_oracle_trajectory_passes_without_flips(orc, precision, flags):
     cfg, w, z0, mask, g, o, ck = _case(orc, precision, **flags)
     r = check_rollout(g, cfg, w, z0, mask, **ck)
