@@ -49,7 +49,7 @@ class _Cfg(C.Structure):
                 ("seed", C.c_uint64), ("nthreads", C.c_int), ("reward_mode", C.c_int),
                 ("reward_alpha", C.c_double), ("reward_beta", C.c_double),
                 ("invalid_reward", C.c_double), ("pop_size", C.c_int), ("pop_group", C.c_int),
-                ("value_head", C.c_int), ("n_xfers", C.c_int)]
+                ("value_head", C.c_int), ("n_xfers", C.c_int), ("state64", C.c_int)]
 
 
 class _W(C.Structure):
@@ -96,6 +96,8 @@ def _load():
             lib.orc_returns.argtypes = [C.c_int, C.c_int, C.c_double, C.c_int, P, P, P, P,
                                         C.c_uint64, C.c_int, C.c_int, P]
             lib.orc_returns.restype = C.c_int
+            lib.orc_mdn_nll_grad.argtypes = [P, P, C.c_int, C.c_int] + [P] * 8
+            lib.orc_mdn_nll_grad.restype = C.c_int
             lib.orc_mdn_nll.argtypes = [P, P, C.c_int, C.c_int] + [P] * 7
             lib.orc_mdn_nll.restype = C.c_int
             _lib = lib
@@ -120,7 +122,8 @@ def _cfg(cfg: dict, nthreads: int) -> _Cfg:
                 int(cfg.get("reward_mode", 0)), float(cfg.get("reward_alpha", 0.8)),
                 float(cfg.get("reward_beta", 0.2)), float(cfg.get("invalid_reward", -100.0)),
                 int(cfg.get("pop_size", 0)), int(cfg.get("pop_group", 1)),
-                int(cfg.get("value_head", 0)), int(cfg.get("n_xfers", 0)))
+                int(cfg.get("value_head", 0)), int(cfg.get("n_xfers", 0)),
+                int(cfg.get("state64", 0)))
 
 
 class _Weights:
@@ -357,6 +360,28 @@ def returns(rewards, done, gamma: float, stop_at_done: bool = True, bootstrap=No
                          int(pop_group), _ptr(fit))
     if rc != 0:
         raise ValueError(f"orc_returns failed ({rc})")
+    return out
+
+
+def mdn_nll_grad(cfg: dict, weights: dict, z_seq, actions, lengths=None, nthreads: int = 1) -> dict:
+    """Gradient of sum_n NLL_n with respect to W_lstm, b_lstm, W_mdn, b_mdn (BPTT, fp64),
+    plus the per-sequence NLL."""
+    lib = _load()
+    Z, A, H, K = (int(cfg[k]) for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
+    z_seq = _f32(z_seq)
+    T, N = z_seq.shape[0] - 1, z_seq.shape[1]
+    act = np.ascontiguousarray(actions, dtype=np.int32).reshape(T, N)
+    ln = None if lengths is None else np.ascontiguousarray(lengths, dtype=np.int32).reshape(N)
+    M = 3 * K * Z
+    out = {"nll": np.zeros(N), "W_lstm": np.zeros((Z + A + H, 4 * H)), "b_lstm": np.zeros(4 * H),
+           "W_mdn": np.zeros((H, M)), "b_mdn": np.zeros(M)}
+    w = _Weights(weights)
+    cs = _cfg(cfg, nthreads)
+    rc = lib.orc_mdn_nll_grad(C.byref(cs), C.byref(w.s), N, T, _ptr(z_seq), _ptr(act), _ptr(ln),
+                              _ptr(out["nll"]), _ptr(out["W_lstm"]), _ptr(out["b_lstm"]),
+                              _ptr(out["W_mdn"]), _ptr(out["b_mdn"]))
+    if rc != 0:
+        raise ValueError(f"orc_mdn_nll_grad failed ({rc})")
     return out
 
 

@@ -323,11 +323,13 @@ static int load_wts(const orc_cfg *cfg, const orc_weights *w, wts64 *v, int need
     return 0;
 }
 
-/* GEMM A-operand: bf16-rounded through fp32 in bf16 mode, else fp32 value. */
+/* GEMM A-operand: bf16-rounded through fp32 in bf16 mode, else fp32 value (unrounded
+ * with state64, the smooth fp64 model the gradient pins differentiate). */
 static double opnd(const orc_cfg *cfg, double v)
 {
     float f = (float)v;
-    return cfg->bf16 ? (double)orc_bf16(f) : (double)f;
+    if (cfg->bf16) return (double)orc_bf16(f);
+    return cfg->state64 ? v : (double)f;
 }
 
 static int check_cfg(const orc_cfg *c)
@@ -356,10 +358,11 @@ static void lstm_step(const orc_cfg *cfg, const wts64 *v, const double *x, int a
     }
     orc_lstm_cell(H, gates, c, c, h);
     /* the recurrent state is carried in fp32 between steps */
-    for (int u = 0; u < H; ++u) {
-        c[u] = (double)(float)c[u];
-        h[u] = (double)(float)h[u];
-    }
+    if (!cfg->state64)
+        for (int u = 0; u < H; ++u) {
+            c[u] = (double)(float)c[u];
+            h[u] = (double)(float)h[u];
+        }
 }
 
 /* a5: MDN head outputs on y = op(h'). */
@@ -804,6 +807,173 @@ static int nll_sequence(const orc_cfg *cfg, const wts64 *v, int n, int N, int T,
     nll[n] = total;
     free(h); free(c); free(x); free(g); free(y); free(mdn);
     return 0;
+}
+
+/* d NLL / d [logit | mu | log sigma] of one latent dim's mixture (K components) at
+ * target x, with responsibilities g_k = pi_k N_k / sum_j pi_j N_j:
+ *   d/d logit_k = pi_k - g_k,  d/d mu_k = -g_k (x - mu_k) / sigma_k^2,
+ *   d/d log sigma_k = g_k (1 - ((x - mu_k) / sigma_k)^2).  Returns the NLL. */
+static double mixture_nll_grad_1d(int K, const double *lg, const double *mu, const double *ls, double x,
+                                  double *dlg, double *dmu, double *dls)
+{
+    double lmax = -INFINITY, s = 0.0, terms[64], tmax = -INFINITY, acc = 0.0;
+    for (int k = 0; k < K; ++k) if (lg[k] > lmax) lmax = lg[k];
+    for (int k = 0; k < K; ++k) s += exp(lg[k] - lmax);
+    const double logz = lmax + log(s);
+    for (int k = 0; k < K; ++k) {
+        const double zs = (x - mu[k]) * exp(-ls[k]);
+        terms[k] = (lg[k] - logz) - 0.5 * zs * zs - ls[k] - 0.5 * log(2.0 * M_PI);
+        if (terms[k] > tmax) tmax = terms[k];
+    }
+    for (int k = 0; k < K; ++k) acc += exp(terms[k] - tmax);
+    const double lse = tmax + log(acc);
+    for (int k = 0; k < K; ++k) {
+        const double pi = exp(lg[k] - logz), gam = exp(terms[k] - lse);
+        const double zs = (x - mu[k]) * exp(-ls[k]);
+        dlg[k] = pi - gam;
+        dmu[k] = -gam * zs * exp(-ls[k]);
+        dls[k] = gam * (1.0 - zs * zs);
+    }
+    return -lse;
+}
+
+/* BPTT of one sequence; gradients are added to the per-thread accumulators. */
+static int grad_sequence(const orc_cfg *cfg, const wts64 *v, int n, int N, int T, const float *z_seq,
+                         const int32_t *actions, int len, double *nll_out, double *gW, double *gb,
+                         double *gWm, double *gbm)
+{
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, K = cfg->k_mix, M = 3 * K * Z;
+    const int KX = Z + H, N4 = 4 * H;
+    /* forward, keeping every step's operands, gate activations, cell and head outputs */
+    double *X = malloc(sizeof(double) * (size_t)T * KX), *act = malloc(sizeof(double) * (size_t)T * N4);
+    double *C = malloc(sizeof(double) * (size_t)(T + 1) * H), *Y = malloc(sizeof(double) * (size_t)T * H);
+    double *MD = malloc(sizeof(double) * (size_t)T * M), *h = calloc((size_t)H, sizeof(double));
+    double *g = malloc(sizeof(double) * N4), *dmd = malloc(sizeof(double) * M);
+    double *dh = malloc(sizeof(double) * H), *dhn = calloc((size_t)H, sizeof(double));
+    double *dcn = calloc((size_t)H, sizeof(double)), *dG = malloc(sizeof(double) * N4);
+    if (!X || !act || !C || !Y || !MD || !h || !g || !dmd || !dh || !dhn || !dcn || !dG) {
+        free(X); free(act); free(C); free(Y); free(MD); free(h); free(g); free(dmd); free(dh);
+        free(dhn); free(dcn); free(dG);
+        return -1;
+    }
+    for (int u = 0; u < H; ++u) C[u] = 0.0;  /* c_0 */
+    double total = 0.0;
+    for (int t = 0; t < T; ++t) {
+        const size_t tn = (size_t)t * N + n;
+        double *x = X + (size_t)t * KX, *c = C + (size_t)(t + 1) * H;
+        for (int i = 0; i < Z; ++i) x[i] = opnd(cfg, z_seq[tn * Z + i]);
+        for (int i = 0; i < H; ++i) x[Z + i] = opnd(cfg, h[i]);
+        for (int u = 0; u < H; ++u) c[u] = C[(size_t)t * H + u];
+        lstm_step(cfg, v, x, actions[tn], -1, g, c, h);
+        double *ac = act + (size_t)t * N4;
+        for (int u = 0; u < H; ++u) {  /* i, f, g, o from the pre-activations */
+            ac[u] = 1.0 / (1.0 + exp(-g[u]));
+            ac[H + u] = 1.0 / (1.0 + exp(-g[H + u]));
+            ac[2 * H + u] = tanh(g[2 * H + u]);
+            ac[3 * H + u] = 1.0 / (1.0 + exp(-g[3 * H + u]));
+        }
+        double *y = Y + (size_t)t * H, *md = MD + (size_t)t * M;
+        for (int i = 0; i < H; ++i) y[i] = opnd(cfg, h[i]);
+        mdn_head(cfg, v, y, md);
+    }
+    /* backward through time */
+    for (int t = T - 1; t >= 0; --t) {
+        const size_t tn = (size_t)t * N + n;
+        const double *md = MD + (size_t)t * M, *y = Y + (size_t)t * H, *x = X + (size_t)t * KX;
+        const double *ac = act + (size_t)t * N4, *c = C + (size_t)(t + 1) * H, *cp = C + (size_t)t * H;
+        for (int m = 0; m < M; ++m) dmd[m] = 0.0;
+        if (t < len) {
+            const float *target = z_seq + ((size_t)(t + 1) * N + n) * Z;
+            for (int d = 0; d < Z; ++d)
+                total += mixture_nll_grad_1d(K, md + d * K, md + K * Z + d * K, md + 2 * K * Z + d * K,
+                                             (double)target[d], dmd + d * K, dmd + K * Z + d * K,
+                                             dmd + 2 * K * Z + d * K);
+        }
+        /* heads: mdn = W_mdn^T y + b_mdn */
+        for (int i = 0; i < H; ++i) {
+            double s = 0.0;
+            for (int m = 0; m < M; ++m) {
+                gWm[(size_t)i * M + m] += y[i] * dmd[m];
+                s += v->W_mdn[(size_t)i * M + m] * dmd[m];
+            }
+            dh[i] = s + dhn[i];
+        }
+        for (int m = 0; m < M; ++m) gbm[m] += dmd[m];
+        /* cell: c = f c_prev + i g, h = o tanh(c) */
+        for (int u = 0; u < H; ++u) {
+            const double ig = ac[u], fg = ac[H + u], gg = ac[2 * H + u], og = ac[3 * H + u];
+            const double tc = tanh(c[u]);
+            const double dc = dh[u] * og * (1.0 - tc * tc) + dcn[u];
+            dG[u] = dc * gg * ig * (1.0 - ig);
+            dG[H + u] = dc * cp[u] * fg * (1.0 - fg);
+            dG[2 * H + u] = dc * ig * (1.0 - gg * gg);
+            dG[3 * H + u] = dh[u] * tc * og * (1.0 - og);
+            dcn[u] = dc * fg;
+        }
+        /* gates: G = W^T [x_z; onehot(a); x_h] + b */
+        const int a = actions[tn];
+        for (int k = 0; k < N4; ++k) gb[k] += dG[k];
+        for (int i = 0; i < Z; ++i)
+            for (int k = 0; k < N4; ++k) gW[(size_t)i * N4 + k] += x[i] * dG[k];
+        if (a >= 0)
+            for (int k = 0; k < N4; ++k) gW[(size_t)(Z + a) * N4 + k] += dG[k];
+        for (int i = 0; i < H; ++i) {
+            double s = 0.0;
+            for (int k = 0; k < N4; ++k) {
+                gW[(size_t)(Z + A + i) * N4 + k] += x[Z + i] * dG[k];
+                s += v->W_lstm[(size_t)(Z + A + i) * N4 + k] * dG[k];
+            }
+            dhn[i] = s;
+        }
+    }
+    if (nll_out) nll_out[n] = total;
+    free(X); free(act); free(C); free(Y); free(MD); free(h); free(g); free(dmd); free(dh);
+    free(dhn); free(dcn); free(dG);
+    return 0;
+}
+
+int orc_mdn_nll_grad(const orc_cfg *cfg, const orc_weights *w, int N, int T,
+                     const float *z_seq, const int32_t *actions, const int32_t *lengths,
+                     double *nll, double *gW_lstm, double *gb_lstm, double *gW_mdn,
+                     double *gb_mdn)
+{
+    if (check_cfg(cfg) || N < 0 || T < 0 || !z_seq || !actions || !gW_lstm || !gb_lstm ||
+        !gW_mdn || !gb_mdn)
+        return -1;
+    for (size_t i = 0; i < (size_t)N * T; ++i)
+        if (actions[i] >= cfg->a_dim) return -1;
+    if (lengths)
+        for (int n = 0; n < N; ++n)
+            if (lengths[n] < 0 || lengths[n] > T) return -1;
+    const int Z = cfg->z_dim, A = cfg->a_dim, H = cfg->h_dim, M = 3 * cfg->k_mix * Z;
+    const size_t nW = (size_t)(Z + A + H) * 4 * H, nb = (size_t)4 * H, nWm = (size_t)H * M;
+    const size_t per = nW + nb + nWm + (size_t)M;
+    wts64 v;
+    if (load_wts(cfg, w, &v, 0)) return -2;
+    int nt = cfg->nthreads > 0 ? cfg->nthreads : 1;
+    if (nt > N && N > 0) nt = N;
+    if (nt < 1) nt = 1;
+    /* one accumulator per thread; sequence n goes to thread n % nt, partials summed in
+     * thread order (deterministic for a given thread count) */
+    double *acc = calloc((size_t)nt * per, sizeof(double));
+    if (!acc) { free_wts(&v); return -2; }
+    int bad = 0;
+#pragma omp parallel for schedule(static, 1) num_threads(nt) reduction(| : bad)
+    for (int r = 0; r < nt; ++r) {
+        double *a = acc + (size_t)r * per;
+        for (int n = r; n < N; n += nt) {
+            const int len = lengths ? lengths[n] : T;
+            bad |= grad_sequence(cfg, &v, n, N, T, z_seq, actions, len, nll, a, a + nW, a + nW + nb,
+                                 a + nW + nb + nWm) ? 1 : 0;
+        }
+    }
+    for (size_t i = 0; i < nW; ++i) { double s = 0; for (int r = 0; r < nt; ++r) s += acc[(size_t)r * per + i]; gW_lstm[i] = s; }
+    for (size_t i = 0; i < nb; ++i) { double s = 0; for (int r = 0; r < nt; ++r) s += acc[(size_t)r * per + nW + i]; gb_lstm[i] = s; }
+    for (size_t i = 0; i < nWm; ++i) { double s = 0; for (int r = 0; r < nt; ++r) s += acc[(size_t)r * per + nW + nb + i]; gW_mdn[i] = s; }
+    for (size_t i = 0; i < (size_t)M; ++i) { double s = 0; for (int r = 0; r < nt; ++r) s += acc[(size_t)r * per + nW + nb + nWm + i]; gb_mdn[i] = s; }
+    free(acc);
+    free_wts(&v);
+    return bad ? -2 : 0;
 }
 
 int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,

@@ -58,6 +58,10 @@ typedef struct {
      * under that xfer's location mask; the LSTM input is onehot(xfer) ||
      * onehot(location) (action rows xfer and NX + location).  0 = flat.     */
     int n_xfers;
+    /* 1: carry the recurrent state, and take the fp32 path's GEMM operands,
+     * in fp64 instead of rounding them to fp32 (a smooth model for the
+     * finite-difference and autograd pins of the gradients only)           */
+    int state64;
 } orc_cfg;
 
 typedef struct {
@@ -160,6 +164,19 @@ int orc_returns(int B, int T, double gamma, int stop_at_done, const float *rewar
 int orc_mdn_nll(const orc_cfg *cfg, const orc_weights *w, int N, int T,
                 const float *z_seq, const int32_t *actions, const int32_t *lengths,
                 double *nll, float *h_seq, float *c_seq, float *mdn_seq);
+
+/* Gradient of the teacher-forced loss sum_n NLL_n (the world model's training
+ * objective, Sec. 4.7; trained by backpropagation, Sec. 3.3.2) with respect to
+ * the MDN-RNN's parameters, by backpropagation through time: the mixture
+ * NLL's gradient at each counted step, back through the heads and the LSTM.
+ * Same inputs as orc_mdn_nll (flat actions).  Outputs (overwritten, fp64):
+ * nll [N] (may be NULL), gW_lstm [Z+A+H, 4H], gb_lstm [4H], gW_mdn [H, 3KZ],
+ * gb_mdn [3KZ].  With bf16 operand rounding (cfg->bf16) the rounding is
+ * treated as the identity in the backward pass. */
+int orc_mdn_nll_grad(const orc_cfg *cfg, const orc_weights *w, int N, int T,
+                     const float *z_seq, const int32_t *actions, const int32_t *lengths,
+                     double *nll, double *gW_lstm, double *gb_lstm, double *gW_mdn,
+                     double *gb_mdn);
 
 #ifdef __cplusplus
 }

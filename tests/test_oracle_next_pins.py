@@ -378,3 +378,100 @@ def test_hier_noop_terminates_and_invalid(orc):
     o2 = orc.rollout(cfg2, w2, z0, xm2, T, want_seq=True, loc_mask=lm2, rt0=rt0, mem0=mem0)
     assert np.all(o2["actions"] == 0) and np.all(o2["loc_seq"] == -1)
     assert np.all(o2["rewards"] == np.float32(-100.0))
+
+
+# ----------------------------------------------------------------------------- BPTT gradient (Sec. 3.3.2, Sec. 4.7)
+def _grad_case(seed=61, precision="fp32", **kw):
+    Z, A, H, K, N, T = 3, 5, 6, 2, 4, 5
+    cfg = _cfg(Z, A, H, K, reward_mode=0, precision=precision, **kw)
+    w = synth.weights(cfg, seed=seed, std=0.4)
+    zs, acts, lens = synth.teacher_inputs(N, T, Z, A, seed=seed, ragged=True)
+    acts[1, 2] = -1
+    lens[0] = T
+    return cfg, w, zs, acts, lens
+
+
+def test_grad_matches_central_differences(orc):
+    """Every parameter block against central differences of sum_n NLL_n (state carried in
+    fp64, so the loss is smooth to the last bit; the step is the fp32 weights' own)."""
+    cfg, w, zs, acts, lens = _grad_case(state64=1)
+    g = orc.mdn_nll_grad(cfg, w, zs, acts, lens)
+    loss = lambda ww: orc.mdn_nll(cfg, ww, zs, acts, lengths=lens)["nll"].sum()
+    assert np.allclose(g["nll"], orc.mdn_nll(cfg, w, zs, acts, lengths=lens)["nll"], rtol=1e-12)
+    rng = np.random.default_rng(61)
+    Z, A = cfg["z_dim"], cfg["a_dim"]
+    picks = {"W_lstm": [(0, 3), (Z + 1, 7), (Z + acts[0, 1], 2), (Z + A + 2, 20), (Z + A + 5, 23)],
+             "b_lstm": [(5,), (12,), (19,)], "W_mdn": [(0, 0), (3, 11), (5, 17)], "b_mdn": [(2,), (9,), (16,)]}
+    for name, idxs in picks.items():
+        for idx in idxs:
+            wp, wm = {k: (np.array(v, copy=True) if isinstance(v, np.ndarray) else v) for k, v in w.items()}, \
+                     {k: (np.array(v, copy=True) if isinstance(v, np.ndarray) else v) for k, v in w.items()}
+            x0 = float(w[name][idx])
+            xp, xm = np.float32(x0 + 1e-3), np.float32(x0 - 1e-3)
+            wp[name][idx], wm[name][idx] = xp, xm
+            fd = (loss(wp) - loss(wm)) / (float(xp) - float(xm))
+            assert g[name][idx] == pytest.approx(fd, rel=2e-5, abs=2e-7), (name, idx, g[name][idx], fd)
+
+
+def _torch_loss(cfg, w, zs, acts, lens, bf16=False):
+    """sum_n NLL_n in torch fp64 (LSTMCell + MixtureSameFamily), for autograd; bf16 rounds the
+    weights and the GEMM operands with a straight-through gradient."""
+    import torch
+    from torch.distributions import Categorical, MixtureSameFamily, Normal
+    Z, A, H, K = (cfg[k] for k in ("z_dim", "a_dim", "h_dim", "k_mix"))
+    rnd = (lambda x: x + (x.to(torch.bfloat16).double() - x).detach()) if bf16 else (lambda x: x)
+    wr = (lambda a: torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).double()) if bf16 else \
+         (lambda a: torch.from_numpy(np.asarray(a, np.float32)).double())
+    P = {"W_lstm": wr(w["W_lstm"]).requires_grad_(), "b_lstm": torch.from_numpy(w["b_lstm"]).double().requires_grad_(),
+         "W_mdn": wr(w["W_mdn"]).requires_grad_(), "b_mdn": torch.from_numpy(w["b_mdn"]).double().requires_grad_()}
+    T, N = acts.shape
+    h = torch.zeros(N, H, dtype=torch.float64)
+    c = torch.zeros(N, H, dtype=torch.float64)
+    total = 0.0
+    for t in range(T):
+        x = torch.cat([rnd(torch.from_numpy(zs[t]).double()), rnd(h)], 1)
+        Wz, Wa, Wh = P["W_lstm"][:Z], P["W_lstm"][Z:Z + A], P["W_lstm"][Z + A:]
+        oh = torch.zeros(N, A, dtype=torch.float64)
+        ok = acts[t] >= 0
+        oh[np.nonzero(ok)[0], acts[t][ok]] = 1.0
+        G = x[:, :Z] @ Wz + oh @ Wa + x[:, Z:] @ Wh + P["b_lstm"]
+        i, f, g, o = G[:, :H].sigmoid(), G[:, H:2 * H].sigmoid(), G[:, 2 * H:3 * H].tanh(), G[:, 3 * H:].sigmoid()
+        c = f * c + i * g
+        h = o * c.tanh()
+        md = (rnd(h) @ P["W_mdn"] + P["b_mdn"]).view(N, 3, Z, K)
+        mix = MixtureSameFamily(Categorical(logits=md[:, 0]), Normal(md[:, 1], md[:, 2].exp()))
+        lp = mix.log_prob(torch.from_numpy(zs[t + 1]).double()).sum(1)
+        total = total - (lp * torch.from_numpy((t < lens).astype(np.float64))).sum()
+    total.backward()
+    return total, P
+
+
+@pytest.mark.parametrize("precision", ["fp32", "bf16"])
+def test_grad_matches_torch_autograd(orc, precision):
+    """fp32: torch autograd through LSTMCell-style gates and MixtureSameFamily (fp64, state
+    in fp64); bf16: the same with bf16 weights and straight-through operand rounding."""
+    Z, A, H, K, N, T = 5, 7, 12, 3, 6, 6
+    cfg = _cfg(Z, A, H, K, reward_mode=0, precision=precision, state64=1)
+    w = synth.weights(cfg, seed=62, std=0.4)
+    zs, acts, lens = synth.teacher_inputs(N, T, Z, A, seed=62, ragged=True)
+    acts[2, 3] = -1
+    g = orc.mdn_nll_grad(cfg, w, zs, acts, lens, nthreads=3)
+    total, P = _torch_loss(cfg, w, zs, acts, lens, bf16=(precision == "bf16"))
+    assert g["nll"].sum() == pytest.approx(float(total), rel=1e-10)
+    for k in P:
+        np.testing.assert_allclose(g[k], P[k].grad.numpy(), rtol=1e-8, atol=1e-10, err_msg=k)
+
+
+def test_grad_is_additive_over_sequences(orc):
+    """The gradient of a batch is the sum of its sequences' gradients (any split)."""
+    cfg, w, zs, acts, lens = _grad_case(seed=63)
+    full = orc.mdn_nll_grad(cfg, w, zs, acts, lens, nthreads=2)
+    a = orc.mdn_nll_grad(cfg, w, zs[:, :1], acts[:, :1], lens[:1])
+    b = orc.mdn_nll_grad(cfg, w, zs[:, 1:], acts[:, 1:], lens[1:])
+    for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn"):
+        np.testing.assert_allclose(full[k], a[k] + b[k], rtol=1e-12, atol=1e-15)
+    # padding: a zero-length sequence contributes nothing
+    l0 = lens.copy()
+    l0[:] = 0
+    z = orc.mdn_nll_grad(cfg, w, zs, acts, l0)
+    assert all(np.all(z[k] == 0) for k in ("W_lstm", "b_lstm", "W_mdn", "b_mdn"))
