@@ -223,6 +223,34 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
                      const int32_t *lengths, float *nll, float *h_seq, float *c_seq,
                      float *mdn_seq, void *cuda_stream);
 
+/* Gradients of the world model's training loss.  Output arrays (device or host
+ * memory, overwritten, fp32) in the canonical layouts of wm_weights. */
+typedef struct {
+    float *W_lstm;   /* [Z+A+H, 4H] required */
+    float *b_lstm;   /* [4H]        required */
+    float *W_mdn;    /* [H, 3KZ]    required */
+    float *b_mdn;    /* [3KZ]       required */
+} wm_grads;
+
+/* The world model's training step (Sec. 3.3.2: the MDN-RNN is trained by
+ * backpropagation on minibatches of rollouts; Sec. 4.7: its loss is the
+ * mixture log-likelihood): the teacher-forced loss sum_n NLL_n of wm_mdn_nll
+ * and its gradient with respect to W_lstm, b_lstm, W_mdn and b_mdn, by
+ * backpropagation through time.  Inputs as wm_mdn_nll (flat-action models);
+ * nll [N] is optional.  The reward, done, runtime, memory and value heads are
+ * not in the loss.  On the bf16 path the operand rounding is treated as the
+ * identity in the backward pass, and the backward's GEMM operands are bf16
+ * (fp32 accumulation); the fp32 path computes in fp32.  The forward runs on the
+ * kernel family wm_mdn_nll would pick; the batched GEMMs of the backward
+ * (gate activations over all N*T rows, the heads' and the recurrent input
+ * gradients, the weight gradients) are cuBLAS calls, the rest (the mixture
+ * NLL's gradient, the cell's backward step, the action-row and bias sums) are
+ * the library's kernels.  Deterministic: every reduction has a fixed order.
+ * Returns WM_ERR_UNSUPPORTED for hierarchical models. */
+wm_status wm_mdn_nll_backward(wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                              const int32_t *lengths, float *nll, const wm_grads *grads,
+                              void *cuda_stream);
+
 /* wm_rollout without any device allocation.  The paper has no counterpart:
  * this entry point exists for callers that cannot call cudaMalloc/cudaFree
  * while they run -- work issued during CUDA stream capture, real-time loops
@@ -306,7 +334,9 @@ enum {
     WM_KERNEL_TC_GATES = 5,     /* tensor: gate GEMM with the LSTM cell            */
     WM_KERNEL_TC_HEADS = 6,     /* tensor: head GEMM with sampling or NLL          */
     WM_KERNEL_AUX = 7,          /* state set-up, finishing copies, reductions      */
-    WM_KERNEL_CLASSES = 8
+    WM_KERNEL_BW = 8,           /* training step: the library's backward kernels    */
+    WM_KERNEL_BW_GEMM = 9,      /* training step: its cuBLAS GEMMs                  */
+    WM_KERNEL_CLASSES = 10
 };
 
 /* enable != 0 turns timing on and clears the totals; 0 turns it off (events

@@ -346,6 +346,7 @@ void wm_destroy(wm_handle *h) {
     cudaFree(h->step.bp);
     wm_fused_free(h);
     wm_tc_free(h);
+    wm_bw_free(h);
     cudaFree(h->ws);
     cudaFree(h->stage);
     cudaFree(h->status);
@@ -612,6 +613,78 @@ wm_status wm_returns(wm_handle *h, int B, int T, unsigned long long episode_offs
     if ((e = st.begin(h, T, false, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
     e = wm_returns_launch(h, B, T, episode_offset, gamma, stop_at_done, r, d, bs, ret, fit, h->ws, s);
     if (e != cudaSuccess) return cuda_fail(h, e, "returns launch");
+    if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
+    return WM_OK;
+}
+
+wm_status wm_mdn_nll_backward(wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                              const int32_t *lengths, float *nll, const wm_grads *grads, void *cuda_stream) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->err.clear();
+    const wm_config &c = h->cfg;
+    if (c.n_xfers > 0) return fail(h, WM_ERR_UNSUPPORTED, "the training step takes flat-action models only");
+    if (N < 0 || T < 0 || N > (1 << 22)) return fail(h, WM_ERR_INVALID_ARG, "N must be in [0, 2^22], T >= 0");
+    if (!grads || !grads->W_lstm || !grads->b_lstm || !grads->W_mdn || !grads->b_mdn)
+        return fail(h, WM_ERR_INVALID_ARG, "all four gradient arrays are required");
+    if (N > 0 && T > 0 && (!z_seq || !actions)) return fail(h, WM_ERR_INVALID_ARG, "z_seq and actions are required");
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, n = (size_t)N, t = (size_t)T;
+    if (actions && is_host_ptr(actions))
+        for (size_t i = 0; i < n * t; ++i)
+            if (actions[i] >= c.a_dim) return fail(h, WM_ERR_INVALID_ARG, "action index >= A");
+    if (lengths && is_host_ptr(lengths))
+        for (size_t i = 0; i < n; ++i)
+            if (lengths[i] < 0 || lengths[i] > T) return fail(h, WM_ERR_INVALID_ARG, "length outside [0, T]");
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    cudaError_t e = cudaSetDevice(h->device);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+    if ((e = wm_bw_prepare(h)) != cudaSuccess) return cuda_fail(h, e, "training-step set-up (cuBLAS)");
+
+    const float *zs = z_seq;
+    const int32_t *ac = actions, *ln = lengths;
+    float *nl = nll;
+    wm_grads g = *grads;
+    Stager st;
+    st.add((void **)&zs, z_seq, (t + 1) * n * Z * 4, false);
+    st.add((void **)&ac, actions, t * n * 4, false);
+    st.add((void **)&ln, lengths, n * 4, false);
+    st.add((void **)&nl, nll, n * 4, true);
+    st.add((void **)&g.W_lstm, grads->W_lstm, (Z + A + H) * 4 * H * 4, true);
+    st.add((void **)&g.b_lstm, grads->b_lstm, 4 * H * 4, true);
+    st.add((void **)&g.W_mdn, grads->W_mdn, H * M * 4, true);
+    st.add((void **)&g.b_mdn, grads->b_mdn, M * 4, true);
+
+    // the forward: the teacher-forced pass, keeping h, c and the head outputs of every row
+    const int path = pick_path(h, N);
+    if (path == WM_PATH_FUSED && !wm_fused_supported(h, N))
+        return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
+    if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
+        return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
+    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N)
+                                                                                      : wm_step_nll_ws(h, N);
+    if ((e = grow(&h->ws, &h->ws_bytes, need)) != cudaSuccess) return cuda_fail(h, e, "workspace");
+    if ((e = grow(&h->bws, &h->bws_bytes, wm_bw_ws(h, N, T))) != cudaSuccess)
+        return cuda_fail(h, e, "training-step workspace");
+    if ((e = st.begin(h, T, false, s)) != cudaSuccess) return cuda_fail(h, e, "staging inputs");
+    wm_nll_dev a{};
+    a.N = N; a.T = T; a.z_seq = zs; a.actions = ac; a.lengths = ln;
+    float *nll_ws;
+    void *tail;
+    wm_bw_carve(h, N, T, h->bws, &a.h_seq, &a.c_seq, &a.mdn_seq, &nll_ws, &tail);
+    a.nll = nl ? nl : nll_ws;
+    int fwd_launches = 0;
+    if (N > 0 && T > 0) {
+        if (path == WM_PATH_FUSED) e = wm_fused_nll(h, a, h->ws, s);
+        else if (path == WM_PATH_TENSOR) e = wm_tc_nll(h, a, h->ws, s);
+        else e = wm_step_nll(h, a, h->ws, s);
+        if (e != cudaSuccess) return cuda_fail(h, e, "training-step forward");
+        fwd_launches = path == WM_PATH_STEPWISE ? 2 + 4 * T : h->last_launches;
+    } else if (nl && N > 0) {
+        if ((e = cudaMemsetAsync(nl, 0, n * 4, s)) != cudaSuccess) return cuda_fail(h, e, "nll");
+    }
+    h->last_path = path;
+    h->last_launches = fwd_launches;
+    e = wm_bw_launch(h, N, T, zs, ac, ln, g, a.h_seq, a.c_seq, a.mdn_seq, tail, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "training-step backward");
     if ((e = st.end(s)) != cudaSuccess) return cuda_fail(h, e, "staging outputs");
     return WM_OK;
 }

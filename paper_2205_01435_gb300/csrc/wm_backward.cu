@@ -1,0 +1,391 @@
+// wm_backward.cu -- wm_mdn_nll_backward: the world model's training step, the gradient
+// of the teacher-forced mixture NLL (Sec. 4.7) by backpropagation through time
+// (Sec. 3.3.2).
+//
+// Rows are (step, sequence) pairs r = t N + n, time-major like every [T, N, ...] array of
+// the library.  Everything that does not depend on the recurrence is batched over all
+// N T rows:
+//   forward      the teacher-forced pass of the kernel family wm_mdn_nll picks, keeping
+//                h_t, c_t and the head outputs of every row
+//   X, Y         the GEMM operands of every row, X = [op(z_t); op(h_{t-1})], Y = op(h_t)
+//   gates        G = X W_zh (one GEMM) + b + W_a[a_t], then sigma / tanh  (k_bw_gates)
+//   dMD          d NLL / d [logit | mu | log sigma] of every counted row     (k_bw_mdn)
+//   dY           dMD W_mdn^T (one GEMM): the heads' share of d loss / d h_t
+// then the recurrence, t = T-1 .. 0:
+//   dG_t         the cell's backward step from dY_t + dH and the carried dc  (k_bw_cell)
+//   dH           dG_t W_h^T (one GEMM on N rows): d loss / d h_{t-1}
+// and the weight gradients, batched again:
+//   dW_z, dW_h   X^T dG (two GEMMs writing the z and h rows of the output)
+//   dW_a         per action, the sum of the dG rows that took it          (k_bw_arows)
+//   dW_mdn       Y^T dMD (one GEMM);  db_lstm, db_mdn  column sums          (k_bw_colsum)
+// The plain GEMMs are cuBLAS calls (bf16 operands and fp32 accumulation on the bf16 path,
+// fp32 without reduced-precision shortcuts on the fp32 path); the rest are the kernels
+// below.  Every reduction has a fixed order, so results are bit-reproducible.
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "wm_internal.h"
+
+namespace {
+
+constexpr int CHUNKS = 16;  // row chunks of the two-level reductions
+
+template <class T> __device__ __forceinline__ T to_op(float v);
+template <> __device__ __forceinline__ float to_op<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 to_op<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// X [NT, Z+H] = [z_t | h_{t-1}] and Y [NT, H] = h_t, in the GEMM operand type (bf16: RNE,
+// the forward's operand rounding)
+template <class T>
+__global__ void k_bw_build(int N, int TT, int Z, int H, const float *__restrict__ z_seq,
+                           const float *__restrict__ hs, T *__restrict__ X, T *__restrict__ Y) {
+    const int KX = Z + H;
+    const size_t NT = (size_t)N * TT, nx = NT * KX;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nx; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = i / KX, k = i % KX;
+        float v;
+        if (k < (size_t)Z) v = z_seq[r * Z + k];
+        else v = r >= (size_t)N ? hs[(r - N) * H + (k - Z)] : 0.f;  // h_{-1} = 0
+        X[i] = to_op<T>(v);
+    }
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < NT * H; i += (size_t)gridDim.x * blockDim.x)
+        Y[i] = to_op<T>(hs[i]);
+}
+
+// gate pre-activations + bias + the action row -> i, f, g, o (in place)
+__global__ void k_bw_gates(size_t NT, int N, int H, int A, float *__restrict__ G, const int32_t *__restrict__ act,
+                           const float *__restrict__ Wa, const float *__restrict__ bias) {
+    const int H4 = 4 * H;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < NT * H4; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = i / H4;
+        const int col = (int)(i % H4);
+        int a = act[r];
+        float v = G[i] + bias[col];
+        if (a >= 0 && a < A) v += Wa[(size_t)a * H4 + col];
+        G[i] = col / H == 2 ? tanhf(v) : 1.f / (1.f + expf(-v));
+    }
+}
+
+// d NLL / d [logit | mu | log sigma] of one row's latent dim d (0 past the row's length)
+template <class T>
+__global__ void k_bw_mdn(int N, int TT, int Z, int K, const float *__restrict__ md, const float *__restrict__ z_seq,
+                         const int32_t *__restrict__ lengths, float *__restrict__ dmd, T *__restrict__ dmd_op) {
+    const int KZ = K * Z, M = 3 * KZ;
+    const size_t NT = (size_t)N * TT;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < NT * Z; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = i / Z;
+        const int d = (int)(i % Z), t = (int)(r / N), n = (int)(r % N);
+        int len = lengths ? lengths[n] : TT;
+        len = len < 0 ? 0 : (len > TT ? TT : len);
+        const float *row = md + r * M;
+        float *out = dmd + r * M;
+        T *oop = dmd_op + r * M;
+        if (t >= len) {
+            for (int k = 0; k < K; ++k)
+                for (int p = 0; p < 3; ++p) {
+                    out[p * KZ + d * K + k] = 0.f;
+                    oop[p * KZ + d * K + k] = to_op<T>(0.f);
+                }
+            continue;
+        }
+        const float x = z_seq[(r + N) * Z + d];  // the target z_{t+1}
+        const float *lg = row + d * K, *mu = row + KZ + d * K, *ls = row + 2 * KZ + d * K;
+        float lmax = -INFINITY, s = 0.f, term[32], tmax = -INFINITY, acc = 0.f;
+        for (int k = 0; k < K; ++k) lmax = fmaxf(lmax, lg[k]);
+        for (int k = 0; k < K; ++k) s += expf(lg[k] - lmax);
+        const float logz = lmax + logf(s);
+        for (int k = 0; k < K; ++k) {
+            const float zs = (x - mu[k]) * expf(-ls[k]);
+            term[k] = (lg[k] - logz) - 0.5f * zs * zs - ls[k] - 0.91893853320467274178f;
+            tmax = fmaxf(tmax, term[k]);
+        }
+        for (int k = 0; k < K; ++k) acc += expf(term[k] - tmax);
+        const float lse = tmax + logf(acc);
+        for (int k = 0; k < K; ++k) {
+            const float pi = expf(lg[k] - logz), gam = expf(term[k] - lse);
+            const float is = expf(-ls[k]), zs = (x - mu[k]) * is;
+            const float v0 = pi - gam, v1 = -gam * zs * is, v2 = gam * (1.f - zs * zs);
+            out[d * K + k] = v0;
+            out[KZ + d * K + k] = v1;
+            out[2 * KZ + d * K + k] = v2;
+            oop[d * K + k] = to_op<T>(v0);
+            oop[KZ + d * K + k] = to_op<T>(v1);
+            oop[2 * KZ + d * K + k] = to_op<T>(v2);
+        }
+    }
+}
+
+// The cell's backward step at t for N rows: dh = dY_t + dH (from step t + 1), and
+//   dc = dh o (1 - tanh^2 c_t) + dc_carried;  dG = [dc g i(1-i) | dc c_{t-1} f(1-f) |
+//   dc i (1-g^2) | dh tanh(c_t) o(1-o)];  dc_carried <- dc f.
+template <class T>
+__global__ void k_bw_cell(int N, int H, int t, int first, const float *__restrict__ act, const float *__restrict__ cs,
+                          const float *__restrict__ dY, const float *__restrict__ dH, float *__restrict__ dC,
+                          float *__restrict__ dG, T *__restrict__ dG_op) {
+    const size_t base = (size_t)t * N;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)N * H; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t n = i / H;
+        const int u = (int)(i % H);
+        const size_t r = base + n;
+        const float *a = act + r * 4 * H;
+        const float ig = a[u], fg = a[H + u], gg = a[2 * H + u], og = a[3 * H + u];
+        const float c = cs[r * H + u], cp = t > 0 ? cs[(r - N) * H + u] : 0.f;
+        const float dh = dY[r * H + u] + (first ? 0.f : dH[i]);
+        const float tc = tanhf(c);
+        const float dc = dh * og * (1.f - tc * tc) + (first ? 0.f : dC[i]);
+        const float g0 = dc * gg * ig * (1.f - ig), g1 = dc * cp * fg * (1.f - fg);
+        const float g2 = dc * ig * (1.f - gg * gg), g3 = dh * tc * og * (1.f - og);
+        float *o = dG + r * 4 * H;
+        T *oo = dG_op + r * 4 * H;
+        o[u] = g0; o[H + u] = g1; o[2 * H + u] = g2; o[3 * H + u] = g3;
+        oo[u] = to_op<T>(g0); oo[H + u] = to_op<T>(g1); oo[2 * H + u] = to_op<T>(g2); oo[3 * H + u] = to_op<T>(g3);
+        dC[i] = dc * fg;
+    }
+}
+
+// Column sums of a [R, C] matrix, two levels: chunk c of the rows into part[c][C], then
+// the CHUNKS partials in order.  One thread per column, rows in order (fixed sum order).
+__global__ void k_bw_colsum(size_t R, int C, const float *__restrict__ in, float *__restrict__ part) {
+    const int col = blockIdx.x * blockDim.x + threadIdx.x, c = blockIdx.y;
+    if (col >= C) return;
+    const size_t r0 = R * c / CHUNKS, r1 = R * (c + 1) / CHUNKS;
+    double s = 0.0;
+    for (size_t r = r0; r < r1; ++r) s += in[r * C + col];
+    part[(size_t)c * C + col] = (float)s;
+}
+__global__ void k_bw_colsum_fin(int C, const float *__restrict__ part, float *__restrict__ out) {
+    const int col = blockIdx.x * blockDim.x + threadIdx.x;
+    if (col >= C) return;
+    double s = 0.0;
+    for (int c = 0; c < CHUNKS; ++c) s += part[(size_t)c * C + col];
+    out[col] = (float)s;
+}
+
+// The action rows of dW_lstm: block (a, c) sums, in row order, the dG rows of chunk c whose
+// action is a, into part[c][a][4H]; then the CHUNKS partials in order.
+__global__ void k_bw_arows(size_t R, int A, int H4, const int32_t *__restrict__ act, const float *__restrict__ dG,
+                           float *__restrict__ part) {
+    const int a = blockIdx.x, c = blockIdx.y;
+    const size_t r0 = R * c / CHUNKS, r1 = R * (c + 1) / CHUNKS;
+    for (int col0 = 0; col0 < H4; col0 += blockDim.x * 4) {
+        float s[4] = {0.f, 0.f, 0.f, 0.f};
+        const int col = col0 + 4 * threadIdx.x;
+        for (size_t r = r0; r < r1; ++r) {
+            if (act[r] != a) continue;  // uniform over the block
+            if (col < H4)
+                for (int j = 0; j < 4; ++j)
+                    if (col + j < H4) s[j] += dG[r * H4 + col + j];
+        }
+        for (int j = 0; j < 4; ++j)
+            if (col + j < H4) part[((size_t)c * A + a) * H4 + col + j] = s[j];
+    }
+}
+__global__ void k_bw_arows_fin(int A, int H4, const float *__restrict__ part, float *__restrict__ out) {
+    const size_t n = (size_t)A * H4;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+        float s = 0.f;
+        for (int c = 0; c < CHUNKS; ++c) s += part[(size_t)c * n + i];
+        out[i] = s;
+    }
+}
+
+// bf16 copies of the weights the backward's GEMMs read (bf16 path): W_zh [Z+H, 4H] and
+// W_mdn [H, M] from the stepwise family's (already bf16-rounded) fp32 matrices
+__global__ void k_bw_cast(size_t rows, int cols, const float *__restrict__ src, long lds, __nv_bfloat16 *__restrict__ dst) {
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < rows * cols; i += (size_t)gridDim.x * blockDim.x)
+        dst[i] = __float2bfloat16_rn(src[(i / cols) * lds + i % cols]);
+}
+
+int grid_of(size_t n) {
+    size_t g = (n + 255) / 256;
+    if (g > 8192) g = 8192;
+    return g < 1 ? 1 : (int)g;
+}
+
+inline size_t al(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Row-major GEMM on cuBLAS: C[m][n] = sum_k A(m,k) B(k,n), A(m,k) = ta ? A[k lda + m] :
+// A[m lda + k], B(k,n) = tb ? B[n ldb + k] : B[k ldb + n].  (cuBLAS is column-major: it
+// computes C^T = B^T A^T.)
+cublasStatus_t gemm(cublasHandle_t hb, bool bf16, bool ta, bool tb, int m, int n, int k, const void *A, long lda,
+                    const void *B, long ldb, float *C, long ldc) {
+    const float one = 1.f, zero = 0.f;
+    const cudaDataType_t dt = bf16 ? CUDA_R_16BF : CUDA_R_32F;
+    return cublasGemmEx(hb, tb ? CUBLAS_OP_T : CUBLAS_OP_N, ta ? CUBLAS_OP_T : CUBLAS_OP_N, n, m, k, &one, B, dt,
+                        (int)ldb, A, dt, (int)lda, &zero, C, CUDA_R_32F, (int)ldc,
+                        bf16 ? CUBLAS_COMPUTE_32F : CUBLAS_COMPUTE_32F_PEDANTIC, CUBLAS_GEMM_DEFAULT);
+}
+
+cudaError_t cublas_err(cublasStatus_t st) {
+    return st == CUBLAS_STATUS_SUCCESS ? cudaSuccess
+                                       : st == CUBLAS_STATUS_ALLOC_FAILED ? cudaErrorMemoryAllocation
+                                                                          : cudaErrorUnknown;
+}
+
+}  // namespace
+
+// The forward's outputs at the front of the backward's workspace, then its own buffers.
+void wm_bw_carve(const wm_handle *h, int N, int T, void *base, float **hs, float **cs, float **md, float **nll,
+                 void **tail) {
+    const size_t NT = (size_t)N * T, H = h->cfg.h_dim, M = h->M;
+    char *p = (char *)base;
+    *hs = (float *)p; p += al(NT * H * 4);
+    *cs = (float *)p; p += al(NT * H * 4);
+    *md = (float *)p; p += al(NT * M * 4);
+    *nll = (float *)p; p += al((size_t)N * 4);
+    *tail = p;
+}
+
+size_t wm_bw_ws(const wm_handle *h, int N, int T) {
+    const wm_config &c = h->cfg;
+    const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, KX = Z + H, H4 = 4 * H;
+    const size_t NT = (size_t)N * T, es = c.precision == WM_BF16 ? 2 : 4;
+    const size_t part_cols = H4 > M ? H4 : M;
+    return al(NT * H * 4) * 2 + al(NT * M * 4) + al((size_t)N * 4)             // h, c, head outputs, nll
+           + al(NT * KX * es) + al(NT * H * es)                                // X, Y
+           + al(NT * H4 * 4)                                                   // gate activations
+           + al(NT * M * 4) + al(NT * M * es)                                  // dMD
+           + al(NT * H * 4)                                                    // dY
+           + al(NT * H4 * 4) + al(NT * H4 * es)                                // dG
+           + 2 * al((size_t)N * H * 4)                                         // dH, dc
+           + al((size_t)CHUNKS * part_cols * 4) + al((size_t)CHUNKS * A * H4 * 4) + 256;
+}
+
+cudaError_t wm_bw_prepare(wm_handle *h) {
+    if (!h->cublas) {
+        cublasHandle_t hb;
+        cublasStatus_t st = cublasCreate(&hb);
+        if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+        h->cublas = hb;
+    }
+    const wm_config &c = h->cfg;
+    if (c.precision == WM_BF16 && !h->bw_wzh) {
+        const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, KX = Z + H;
+        cudaError_t e = cudaMalloc(&h->bw_wzh, KX * 4 * H * 2);
+        if (e == cudaSuccess) e = cudaMalloc(&h->bw_wm, H * M * 2);
+        if (e != cudaSuccess) return e;
+        k_bw_cast<<<grid_of(KX * 4 * H), 256>>>(KX, 4 * (int)H, h->step.Wg, (long)(4 * H + A), (__nv_bfloat16 *)h->bw_wzh);
+        k_bw_cast<<<grid_of(H * M), 256>>>(H, (int)M, h->step.Wh, (long)(M + h->NR), (__nv_bfloat16 *)h->bw_wm);
+        e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaGetLastError();
+}
+
+void wm_bw_free(wm_handle *h) {
+    if (h->cublas) cublasDestroy((cublasHandle_t)h->cublas);
+    cudaFree(h->bw_wzh);
+    cudaFree(h->bw_wm);
+    cudaFree(h->bws);
+    h->cublas = h->bw_wzh = h->bw_wm = h->bws = nullptr;
+    h->bws_bytes = 0;
+}
+
+template <class T>
+static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq, const int32_t *actions,
+                          const int32_t *lengths, const wm_grads &g, const float *hs, const float *cs,
+                          const float *md, char *p, cudaStream_t s) {
+    const wm_config &c = h->cfg;
+    const bool bf = c.precision == WM_BF16;
+    const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M, KX = Z + H, H4 = 4 * H;
+    const size_t NT = (size_t)N * TT;
+    cublasHandle_t hb = (cublasHandle_t)h->cublas;
+    cublasStatus_t st = cublasSetStream(hb, s);
+    if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+    T *X = (T *)p; p += al(NT * KX * sizeof(T));
+    T *Y = (T *)p; p += al(NT * H * sizeof(T));
+    float *G = (float *)p; p += al(NT * H4 * 4);
+    float *dMD = (float *)p; p += al(NT * M * 4);
+    T *dMDo = (T *)p; p += al(NT * M * sizeof(T));
+    float *dY = (float *)p; p += al(NT * H * 4);
+    float *dG = (float *)p; p += al(NT * H4 * 4);
+    T *dGo = (T *)p; p += al(NT * H4 * sizeof(T));
+    float *dH = (float *)p; p += al((size_t)N * H * 4);
+    float *dC = (float *)p; p += al((size_t)N * H * 4);
+    float *part = (float *)p; p += al((size_t)CHUNKS * (H4 > M ? H4 : M) * 4);
+    float *apart = (float *)p;
+    // weights of the GEMMs: W_zh = the z and h rows of the gate matrix, W_mdn, W_h = W_zh's h rows
+    const void *Wzh = bf ? (const void *)h->bw_wzh : (const void *)h->step.Wg;
+    const long ldw = bf ? H4 : H4 + A;
+    const void *Wm = bf ? (const void *)h->bw_wm : (const void *)h->step.Wh;
+    const long ldm = bf ? M : M + h->NR;
+    const void *Wh = bf ? (const void *)((const __nv_bfloat16 *)h->bw_wzh + (size_t)Z * H4)
+                        : (const void *)(h->step.Wg + (size_t)Z * (H4 + A));
+    int launches = 0;
+    {
+        wm_ktime kt(h, WM_KERNEL_BW, s);
+        k_bw_build<T><<<grid_of(NT * KX), 256, 0, s>>>(N, TT, Z, H, z_seq, hs, X, Y);
+        ++launches;
+    }
+    {
+        wm_ktime kt(h, WM_KERNEL_BW_GEMM, s);
+        st = gemm(hb, bf, false, false, (int)NT, H4, KX, X, KX, Wzh, ldw, G, H4);
+        ++launches;
+    }
+    if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+    {
+        wm_ktime kt(h, WM_KERNEL_BW, s);
+        k_bw_gates<<<grid_of(NT * H4), 256, 0, s>>>(NT, N, H, A, G, actions, h->step.Wa, h->step.bg);
+        k_bw_mdn<T><<<grid_of(NT * Z), 256, 0, s>>>(N, TT, Z, c.k_mix, md, z_seq, lengths, dMD, dMDo);
+        launches += 2;
+    }
+    {
+        wm_ktime kt(h, WM_KERNEL_BW_GEMM, s);
+        st = gemm(hb, bf, false, true, (int)NT, H, M, dMDo, M, Wm, ldm, dY, H);
+        ++launches;
+    }
+    if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+    for (int t = TT - 1; t >= 0; --t) {
+        {
+            wm_ktime kt(h, WM_KERNEL_BW, s);
+            k_bw_cell<T><<<grid_of((size_t)N * H), 256, 0, s>>>(N, H, t, t == TT - 1, G, cs, dY, dH, dC, dG, dGo);
+            ++launches;
+        }
+        if (t > 0) {
+            wm_ktime kt(h, WM_KERNEL_BW_GEMM, s);
+            st = gemm(hb, bf, false, true, N, H, H4, dGo + (size_t)t * N * H4, H4, Wh, ldw, dH, H);
+            ++launches;
+            if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+        }
+    }
+    {
+        wm_ktime kt(h, WM_KERNEL_BW_GEMM, s);
+        // z rows and h rows of dW_lstm: X^T dG, straight into the output's row blocks
+        st = gemm(hb, bf, true, false, Z, H4, (int)NT, X, KX, dGo, H4, g.W_lstm, H4);
+        if (st == CUBLAS_STATUS_SUCCESS)
+            st = gemm(hb, bf, true, false, H, H4, (int)NT, X + Z, KX, dGo, H4, g.W_lstm + (size_t)(Z + A) * H4, H4);
+        if (st == CUBLAS_STATUS_SUCCESS) st = gemm(hb, bf, true, false, H, M, (int)NT, Y, H, dMDo, M, g.W_mdn, M);
+        launches += 3;
+    }
+    if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
+    {
+        wm_ktime kt(h, WM_KERNEL_BW, s);
+        k_bw_arows<<<dim3(A, CHUNKS), 256, 0, s>>>(NT, A, H4, actions, dG, apart);
+        k_bw_arows_fin<<<grid_of((size_t)A * H4), 256, 0, s>>>(A, H4, apart, g.W_lstm + (size_t)Z * H4);
+        k_bw_colsum<<<dim3((H4 + 255) / 256, CHUNKS), 256, 0, s>>>(NT, H4, dG, part);
+        k_bw_colsum_fin<<<(H4 + 255) / 256, 256, 0, s>>>(H4, part, g.b_lstm);
+        k_bw_colsum<<<dim3((M + 255) / 256, CHUNKS), 256, 0, s>>>(NT, M, dMD, part);
+        k_bw_colsum_fin<<<(M + 255) / 256, 256, 0, s>>>(M, part, g.b_mdn);
+        launches += 6;
+    }
+    h->last_launches += launches;
+    return cudaGetLastError();
+}
+
+cudaError_t wm_bw_launch(const wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                         const int32_t *lengths, const wm_grads &g, const float *hs, const float *cs,
+                         const float *md, void *tail, cudaStream_t s) {
+    if (N == 0 || T == 0) {  // no rows: every gradient is 0
+        const wm_config &c = h->cfg;
+        const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim, M = h->M;
+        cudaError_t e = cudaMemsetAsync(g.W_lstm, 0, (Z + A + H) * 4 * H * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(g.b_lstm, 0, 4 * H * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(g.W_mdn, 0, H * M * 4, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(g.b_mdn, 0, M * 4, s);
+        return e;
+    }
+    if (h->cfg.precision == WM_BF16)
+        return bw_run<__nv_bfloat16>(h, N, T, z_seq, actions, lengths, g, hs, cs, md, (char *)tail, s);
+    return bw_run<float>(h, N, T, z_seq, actions, lengths, g, hs, cs, md, (char *)tail, s);
+}

@@ -134,6 +134,12 @@ struct wm_handle {
     mutable int last_launches = 0;   // kernels launched by the last call
     mutable wm_timer timer;
     std::string err;
+    // the training step (wm_backward.cu): cuBLAS handle, bf16 copies of its GEMMs' weights,
+    // and its workspace (all created on first use)
+    void *cublas = nullptr;
+    void *bw_wzh = nullptr, *bw_wm = nullptr;
+    void *bws = nullptr;
+    size_t bws_bytes = 0;
 };
 
 // Brackets the kernel launches of its scope with CUDA events on stream s when
@@ -162,6 +168,16 @@ cudaError_t wm_tc_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStr
 cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, const float *b_ctrl);
 // whether the tensor family can run a rollout call starting at this episode (population tiles)
 int wm_tc_call_ok(const wm_handle *h, unsigned long long episode_offset);
+
+// ---- the training step (wm_backward.cu) -----------------------------------------
+size_t wm_bw_ws(const wm_handle *h, int N, int T);
+void wm_bw_carve(const wm_handle *h, int N, int T, void *base, float **hs, float **cs, float **md, float **nll,
+                 void **tail);
+cudaError_t wm_bw_prepare(wm_handle *h);
+void wm_bw_free(wm_handle *h);
+cudaError_t wm_bw_launch(const wm_handle *h, int N, int T, const float *z_seq, const int32_t *actions,
+                         const int32_t *lengths, const wm_grads &g, const float *hs, const float *cs,
+                         const float *md, void *tail, cudaStream_t s);
 
 // ---- discounted returns (wm_returns.cu) ----------------------------------------
 cudaError_t wm_returns_launch(const wm_handle *h, int B, int T, unsigned long long ep0, float gamma,

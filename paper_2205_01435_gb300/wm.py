@@ -23,7 +23,7 @@ WM_FP32, WM_BF16 = 0, 1
 PATHS = {"auto": 0, "stepwise": 1, "fused": 2, "tensor": 3}
 PATH_NAMES = {v: k for k, v in PATHS.items()}
 KERNEL_CLASSES = ("step_gemm", "step_cell", "step_sample", "fused", "tc_ctrl", "tc_gates",
-                  "tc_heads", "aux")  # WM_KERNEL_* in order
+                  "tc_heads", "aux", "bw", "bw_gemm")  # WM_KERNEL_* in order
 
 
 class WMError(RuntimeError):
@@ -58,6 +58,10 @@ class wm_rollout_io(C.Structure):
         "logp_seq", "value_seq", "loc_mask", "loc_actions")]
 
 
+class wm_grads(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("W_lstm", "b_lstm", "W_mdn", "b_mdn")]
+
+
 def _load():
     if not os.path.exists(_LIB_PATH):
         raise ImportError(f"{_LIB_PATH} is missing: build it with "
@@ -76,6 +80,8 @@ def _load():
     lib.wm_set_controllers.restype = C.c_int
     lib.wm_returns.argtypes = [P, C.c_int, C.c_int, C.c_ulonglong, C.c_float, C.c_int, P, P, P, P, P, P]
     lib.wm_returns.restype = C.c_int
+    lib.wm_mdn_nll_backward.argtypes = [P, C.c_int, C.c_int, P, P, P, P, C.POINTER(wm_grads), P]
+    lib.wm_mdn_nll_backward.restype = C.c_int
     lib.wm_mdn_nll.argtypes = [P, C.c_int, C.c_int] + [P] * 7 + [P]
     lib.wm_mdn_nll.restype = C.c_int
     lib.wm_sync.argtypes = [P]
@@ -182,6 +188,12 @@ def wm_returns(h, B: int, T: int, episode_offset: int, gamma: float, stop_at_don
     _check(h, _lib.wm_returns(h, B, T, episode_offset, float(gamma), int(bool(stop_at_done)),
                               _ptr(rewards), _ptr(done), _ptr(bootstrap), _ptr(returns),
                               _ptr(fitness), C.c_void_p(stream)), "wm_returns")
+
+
+def wm_mdn_nll_backward(h, N: int, T: int, z_seq, actions, lengths, nll, grads: dict, stream: int = 0):
+    g = wm_grads(*[_ptr(grads.get(n)) for n, _ in wm_grads._fields_])
+    _check(h, _lib.wm_mdn_nll_backward(h, N, T, _ptr(z_seq), _ptr(actions), _ptr(lengths), _ptr(nll),
+                                       C.byref(g), C.c_void_p(stream)), "wm_mdn_nll_backward")
 
 
 def wm_sync(h):
@@ -322,6 +334,22 @@ class WorldModel:
         with torch.cuda.device(self.device):
             wm_returns(self.h, B, T, episode_offset, gamma, stop_at_done, rewards, done, bootstrap,
                        o["returns"], o.get("fitness"), self._stream(stream))
+        return o
+
+    def mdn_nll_backward(self, z_seq: torch.Tensor, actions: torch.Tensor, lengths=None,
+                         stream=None) -> dict:
+        """wm_mdn_nll_backward: the per-sequence NLL and the gradient of their sum with respect
+        to W_lstm, b_lstm, W_mdn, b_mdn (arrays on z_seq's device)."""
+        T = int(z_seq.shape[0]) - 1
+        N = int(z_seq.shape[1])
+        Z, A, H, M = self.Z, self.A, self.H, self.M
+        o = {"nll": self._alloc(z_seq, (N,), torch.float32),
+             "W_lstm": self._alloc(z_seq, (Z + A + H, 4 * H), torch.float32),
+             "b_lstm": self._alloc(z_seq, (4 * H,), torch.float32),
+             "W_mdn": self._alloc(z_seq, (H, M), torch.float32),
+             "b_mdn": self._alloc(z_seq, (M,), torch.float32)}
+        with torch.cuda.device(self.device):
+            wm_mdn_nll_backward(self.h, N, T, z_seq, actions, lengths, o["nll"], o, self._stream(stream))
         return o
 
     def sync(self):

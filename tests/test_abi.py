@@ -40,7 +40,7 @@ def test_binding_loads_and_mirrors_names():
     wm = pkg.load()
     for n in ("wm_create", "wm_rollout", "wm_mdn_nll", "wm_sync", "wm_destroy", "wm_last_path",
               "wm_last_launches", "wm_rollout_noalloc", "wm_set_timing", "wm_kernel_time",
-              "wm_set_controllers", "wm_returns"):
+              "wm_set_controllers", "wm_returns", "wm_mdn_nll_backward"):
         assert callable(getattr(wm, n))
 
 
@@ -94,5 +94,6 @@ def test_null_handle_calls_are_rejected():
     assert wm._lib.wm_sync(None) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_set_controllers(None, 1, 1, None, None) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_returns(None, 1, 1, 0, 0.9, 1, *([None] * 6)) == wm.WM_ERR_INVALID_ARG
+    assert wm._lib.wm_mdn_nll_backward(None, 1, 1, None, None, None, None, None, None) == wm.WM_ERR_INVALID_ARG
     assert wm._lib.wm_last_error(None) == b"null handle"
     wm._lib.wm_destroy(None)  # no-op

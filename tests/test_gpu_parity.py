@@ -603,3 +603,75 @@ def test_hierarchical_action_against_oracle(wm, orc, path, name, NX, flags):
     with pytest.raises(wm.WMError) as ei:
         m.mdn_nll(_cuda(zs), _cuda(acts))
     assert ei.value.status == wm.WM_ERR_UNSUPPORTED
+
+
+# ------------------------------------------------------------------ the training step (BPTT)
+GRAD_KEYS = ("W_lstm", "b_lstm", "W_mdn", "b_mdn")
+# relative Frobenius error of each gradient block: fp32 ~ 100 fp32 roundoffs; bf16 ~ 4 bf16
+# roundoffs (2^-9 each: the backward's GEMM operands are rounded to bf16 once)
+GRAD_TOL = {"fp32": 1e-5, "bf16": 1e-2}
+
+
+def _grad_err(g, o):
+    out = {}
+    for k in GRAD_KEYS:
+        a, b = np_(g[k]).astype(np.float64), np.asarray(o[k], np.float64)
+        out[k] = float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+    return out
+
+
+@pytest.mark.parametrize("name,prec,path,N,T", [("tiny_fp32", "fp32", "stepwise", 37, 9),
+                                                ("small_bf16", "bf16", "auto", 64, 12),
+                                                ("nll", "bf16", "tensor", 300, 10),
+                                                ("nll", "fp32", "stepwise", 64, 16)])
+def test_training_step_gradient_against_oracle(wm, orc, name, prec, path, N, T):
+    """wm_mdn_nll_backward against the oracle's fp64 BPTT, ragged lengths and no-action rows."""
+    cfg = dict(synth.model_config(name), precision=prec)
+    if name == "tiny_fp32":
+        cfg.update(z_dim=7, a_dim=45, h_dim=40, k_mix=3)
+    w = synth.weights(cfg, seed=19)
+    zs, acts, lens = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=19, ragged=True)
+    acts[1, ::5] = -1
+    lens[0], lens[1] = 0, T
+    m = wm.WorldModel(dict(cfg, path=path), w)
+    g = m.mdn_nll_backward(_cuda(zs), _cuda(acts), lengths=_cuda(lens))
+    torch.cuda.synchronize()
+    o = orc.mdn_nll_grad(cfg, w, zs, acts, lens, nthreads=NT)
+    err = _grad_err(g, o)
+    print("gradient", name, prec, m.last_path, err)
+    for k, e in err.items():
+        assert e <= GRAD_TOL[prec], (k, e)
+    rel = np.abs(np_(g["nll"]) - o["nll"]) / np.maximum(np.abs(o["nll"]), 1e-12)
+    assert np.all(rel[o["nll"] != 0] <= 1e-3) and np.all(np_(g["nll"])[o["nll"] == 0] == 0)
+    # deterministic, and host arrays give the same bits
+    g2 = m.mdn_nll_backward(_cuda(zs), _cuda(acts), lengths=_cuda(lens))
+    gh = m.mdn_nll_backward(torch.from_numpy(zs), torch.from_numpy(acts), lengths=torch.from_numpy(lens))
+    for k in GRAD_KEYS + ("nll",):
+        assert torch.equal(g[k], g2[k]) and torch.equal(g[k].cpu(), gh[k]), k
+
+
+def test_training_step_full_size(wm, orc):
+    """The nll workload at full size (512 sequences x 128 steps, bf16, tensor forward): the
+    gradient is additive over sequences (two halves sum to the whole), and 16 sequences
+    against the oracle."""
+    cfg = dict(synth.model_config("nll"), precision="bf16")
+    w = synth.weights(cfg, seed=20)
+    N, T = 512, 128
+    zs, acts, lens = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=20, ragged=True)
+    m = wm.WorldModel(dict(cfg, path="tensor"), w)
+    zc, ac, lc = _cuda(zs), _cuda(acts), _cuda(lens)
+    full = m.mdn_nll_backward(zc, ac, lengths=lc)
+    a = m.mdn_nll_backward(zc[:, :256].contiguous(), ac[:, :256].contiguous(), lengths=lc[:256].contiguous())
+    b = m.mdn_nll_backward(zc[:, 256:].contiguous(), ac[:, 256:].contiguous(), lengths=lc[256:].contiguous())
+    torch.cuda.synchronize()
+    assert m.last_path == "tensor"
+    err = _grad_err(full, {k: np_(a[k]).astype(np.float64) + np_(b[k]) for k in GRAD_KEYS})
+    print("additivity", err)
+    for k, e in err.items():
+        assert e <= 1e-5, (k, e)  # the same bf16 products, summed in another order
+    sub = m.mdn_nll_backward(zc[:, :16].contiguous(), ac[:, :16].contiguous(), lengths=lc[:16].contiguous())
+    o = orc.mdn_nll_grad(cfg, w, zs[:, :16], acts[:, :16], lens[:16], nthreads=NT)
+    err = _grad_err(sub, o)
+    print("full-T subset vs oracle", err)
+    for k, e in err.items():
+        assert e <= GRAD_TOL["bf16"], (k, e)
