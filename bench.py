@@ -344,6 +344,108 @@ def run_nll(args) -> None:
     model.close()
 
 
+def train_flops_per_step(cfg: dict) -> float:
+    """Algorithmic FLOPs of one (sequence, step) of the training step: the forward's gates and
+    head, then the backward's gate recompute, dY = dMD W_mdn^T, the recurrent dG W_h^T and
+    the weight gradients X^T dG and Y^T dMD."""
+    Z, H, K = cfg["z_dim"], cfg["h_dim"], cfg["k_mix"]
+    KX, M = Z + H, 3 * K * Z
+    fwd = 2.0 * (KX * 4 * H + H * (M + 2))
+    bwd = 2.0 * (KX * 4 * H + M * H + 4 * H * H + KX * 4 * H + H * M)
+    return fwd + bwd
+
+
+def run_train(args) -> None:
+    """The world model's training step (wm_mdn_nll_backward) on the nll workload: loss and
+    gradient of 512 sequences x 128 steps, in scored (sequence, step) pairs per second."""
+    import torch
+
+    import paper_2205_01435_gb300 as pkg
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    wm = pkg.load()
+    cfg = synth.model_config("nll", precision=args.precision or "bf16")
+    if args.path:
+        cfg["path"] = args.path
+    w = synth.weights(cfg)
+    zs, acts = nll_inputs(cfg, rank)
+    T, N = acts.shape
+    model = wm.WorldModel(cfg, w, device=local)
+    dev = torch.device("cuda", local)
+    zc, ac = torch.from_numpy(zs).to(dev), torch.from_numpy(acts).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    for _ in range(args.warmup):
+        model.mdn_nll_backward(zc, ac, stream=stream)
+    torch.cuda.synchronize()
+    path_name, launches = model.last_path, model.last_launches
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            ev[i][0].record(stream)
+            model.mdn_nll_backward(zc, ac, stream=stream)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+    kt = kernel_timing_pass(model, lambda: model.mdn_nll_backward(zc, ac, stream=stream), flush, stream,
+                            args.steps)
+    ms_per_step = max_over_ranks(sum(a.elapsed_time(b) for a, b in ev), ws, dev) / args.steps
+    value = N * T * ws / (ms_per_step / 1e3)
+    zh, ah = torch.from_numpy(zs).pin_memory(), torch.from_numpy(acts).pin_memory()
+    model.mdn_nll_backward(zh, ah)
+    e2e_t = []
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        model.mdn_nll_backward(zh, ah)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_value = N * T * ws / max_over_ranks(sum(e2e_t) / len(e2e_t), ws, dev)
+    peaks = load_peaks()
+    all_ms = sum(v[0] for v in kt.values())
+    call_fl = train_flops_per_step(cfg) * N * T
+    bf = cfg["precision"] == "bf16"
+    peak = peaks["bf16_tflops"] if bf else fp32_simt_peak_tflops()
+    achieved = call_fl / (ms_per_step / 1e3) / 1e12
+    Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
+    grad_bytes = 4 * ((Z + A + H) * 4 * H + 4 * H + H * 3 * K * Z + 3 * K * Z)
+    roof = {"bound": "tensor" if bf else "alu", "achieved": round(achieved, 3), "peak": round(peak, 1),
+            "unit": "TFLOP/s", "frac": round(achieved / peak, 5), "traffic": None,
+            "peak_source": (peaks["source"] + " bf16 burst") if bf else
+            "derived: 152 SM x 128 fp32 FMA x 2 FLOP x 2.07 GHz",
+            "kernel": "whole training step (forward + BPTT)", "algorithmic_flops_per_step": call_fl,
+            "kernel_shares": {k: round(v[0] / all_ms, 4) for k, v in sorted(kt.items())}}
+    line = {"metric": "world-model training steps: scored (sequence, step) pairs/s (wm_mdn_nll_backward)",
+            "value": round(value, 1), "unit": "scored-steps/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if bf else "f32",
+            "data": "synthetic (seeded: weights N(0,0.05^2), z ~ N(0,1), actions uniform)",
+            "config": {"workload": f"nll_{cfg['precision']}_train", "N": N, "T": T, "z": Z, "A": A, "H": H,
+                       "K": K, "kernel_path": path_name, "l2": "flushed between timed steps (512 MiB write)",
+                       "parallelism": f"sequences sharded over {ws} GPU(s), no collective"},
+            "e2e": {"value": round(e2e_value, 1), "unit": "scored-steps/s",
+                    "h2d_bytes_per_step": zh.numel() * 4 + ah.numel() * 4,
+                    "d2h_bytes_per_step": N * 4 + grad_bytes},
+            "gpu_launches": launches * args.steps, "roofline": roof, "clocks": clk.summary()}
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        import oracle
+        n = max(4, min(N, args.cpu_episodes or 16))
+        threads = os.cpu_count() or 1
+        t0 = time.perf_counter()
+        oracle.mdn_nll_grad(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": round(n * T / dt, 2), "unit": "scored-steps/s", "cores": threads,
+                                "kind": "oracle", "sample": f"{n} of {N} sequences x {T} steps, loss and "
+                                                            f"gradient, {threads} threads, {dt:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+
+
 def run_ours(args) -> None:
     import torch
     import torch.distributed as dist
@@ -585,25 +687,28 @@ def run_reference(args) -> None:
         w = synth.weights(cfg)
         zs, acts = nll_inputs(cfg)
         T, N = acts.shape
-        n = max(8, min(N, args.ref_episodes or N // 16))
+        n = max(8, min(N, args.ref_episodes or (N // 64 if args.train else N // 16)))
         threads = os.cpu_count() or 1
+        fn = oracle.mdn_nll_grad if args.train else oracle.mdn_nll
         for _ in range(args.warmup):
-            oracle.mdn_nll(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+            fn(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
         times = []
         for _ in range(args.steps):
             t0 = time.perf_counter()
-            oracle.mdn_nll(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
+            fn(cfg, w, zs[:, :n], acts[:, :n], nthreads=threads)
             times.append(time.perf_counter() - t0)
         per = sum(times) / len(times)
         value = n * T / per
-        line = {"impl": "reference", "metric": "teacher-forced scored steps/s (wm_mdn_nll)",
+        metric = ("world-model training steps: scored (sequence, step) pairs/s (wm_mdn_nll_backward)"
+                  if args.train else "teacher-forced scored steps/s (wm_mdn_nll)")
+        line = {"impl": "reference", "metric": metric,
                 "value": round(value, 2), "unit": "scored-steps/s", "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": round(per * 1e3, 3), "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None,
                 "dtype": "f64 (bf16 operand emulation)" if cfg["precision"] == "bf16" else "f64",
                 "data": "synthetic (seeded: weights N(0,0.05^2), z ~ N(0,1), actions uniform)",
-                "config": {"workload": f"nll_{cfg['precision']}", "N": N, "T": T, "z": cfg["z_dim"],
-                           "A": cfg["a_dim"], "H": cfg["h_dim"], "K": cfg["k_mix"]},
+                "config": {"workload": f"nll_{cfg['precision']}" + ("_train" if args.train else ""), "N": N,
+                           "T": T, "z": cfg["z_dim"], "A": cfg["a_dim"], "H": cfg["h_dim"], "K": cfg["k_mix"]},
                 "cpu_baseline": {"value": round(value, 2), "unit": "scored-steps/s", "cores": threads,
                                  "kind": "oracle", "sample": f"{n} of {N} sequences x {T} steps, {threads} threads"},
                 "e2e": {"value": round(value, 2), "unit": "scored-steps/s", "h2d_bytes_per_step": 0,
@@ -649,6 +754,8 @@ def main():
     ap.add_argument("--precision", choices=["fp32", "bf16"], default=None,
                     help="nll workload only: fp32 or bf16 path (default bf16)")
     ap.add_argument("--path", choices=["auto", "stepwise", "fused", "tensor"], default=None)
+    ap.add_argument("--train", action="store_true",
+                    help="nll workload: time the training step (loss and BPTT gradient)")
     ap.add_argument("--xfers", type=int, default=0,
                     help="hierarchical action: NX xfers (the last is the NO-OP) and A - NX "
                          "location slots (Sec. 3.1.3)")
@@ -672,6 +779,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "nll" and args.train:
+        run_train(args)
     elif args.workload == "nll":
         run_nll(args)
     else:
