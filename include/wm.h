@@ -304,6 +304,20 @@ wm_status wm_returns(wm_handle *h, int B, int T, unsigned long long episode_offs
                      int stop_at_done, const float *rewards, const uint8_t *done,
                      const float *bootstrap, float *returns, float *fitness, void *cuda_stream);
 
+/* Failure injection for tests of the timeout path.  The paper has no
+ * counterpart: every wait inside the fused and tensor-core kernels is bounded,
+ * and this lets a test make one of them run out without faulting or hanging the
+ * GPU.  With polls > 0, the next wm_rollout or wm_mdn_nll call that runs the
+ * fused or the tensor-core family makes its first kernel launch wait, before
+ * that kernel issues any MMA or copy, on a barrier that nothing completes, for
+ * at most `polls` polls.  The wait then gives up the way a real bounded wait
+ * does: the kernel records WM_ERR_TIMEOUT in the status word, skips its work and
+ * frees what it holds, and the next wm_sync returns WM_ERR_TIMEOUT (and clears
+ * it).  The outputs of that call are undefined; later calls are unaffected.
+ * One shot: the call that consumes the setting clears it, and polls = 0 clears
+ * it without a call.  The stepwise family has no waits and ignores it. */
+wm_status wm_inject_wait_timeout(wm_handle *h, unsigned int polls);
+
 /* Synchronises the device and returns the first device-side error since the
  * last wm_sync (WM_ERR_TIMEOUT if a bounded wait gave up), then clears it. */
 wm_status wm_sync(wm_handle *h);

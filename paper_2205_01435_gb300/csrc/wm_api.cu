@@ -440,6 +440,12 @@ wm_status wm_kernel_time(wm_handle *h, int kernel_class, double *total_ms, long 
     return WM_OK;
 }
 
+wm_status wm_inject_wait_timeout(wm_handle *h, unsigned int polls) {
+    if (!h) return WM_ERR_INVALID_ARG;
+    h->test_wait = polls;
+    return WM_OK;
+}
+
 const char *wm_last_error(const wm_handle *h) { return h ? h->err.c_str() : "null handle"; }
 
 int wm_last_path(const wm_handle *h) { return h ? h->last_path : 0; }

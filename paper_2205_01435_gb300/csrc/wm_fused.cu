@@ -133,6 +133,9 @@ struct FusedParams {
     const int32_t *act_in, *lengths;
     float *nll_part;  // [Z, B]: one partial per latent dim
     int *status;
+    // failure injection (wm_inject_wait_timeout): > 0 makes the kernel wait, before it issues
+    // any MMA or copy of its own, on a barrier that nothing completes, at most this many polls
+    uint32_t test_wait;
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -177,8 +180,9 @@ template <class S>
 __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     constexpr int CL = S::CL, UG = S::UG, ZD = S::ZD, KM = S::KM;
     extern __shared__ __align__(1024) unsigned char smem[];
-    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in, 5 W_a/W2 buffer
-    __shared__ __align__(8) uint64_t mbar[6];
+    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in, 5 W_a/W2 buffer,
+    // 6 never completed (the injected wait)
+    __shared__ __align__(8) uint64_t mbar[7];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     __shared__ float s_done_logit[TILE];
@@ -208,7 +212,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     const uint32_t WA_BYTES = (uint32_t)A * S::WA_STRIDE, W2_BYTES = (uint32_t)S::N2 * H * 2;
     const uint32_t mb = tc::smem_u32(&mbar[0]);
     const uint32_t MB_MMA1 = mb, MB_MMA2 = mb + 8, MB_PART = mb + 16, MB_H = mb + 24, MB_Z = mb + 32,
-                   MB_W = mb + 40;
+                   MB_W = mb + 40, MB_NEVER = mb + 48;
     const unsigned char *img = p.img + rank * p.img_stride;
     const uint32_t buf_u32 = tc::smem_u32(sBuf);
 
@@ -243,7 +247,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         frozen = live && p.done0 && p.done0[b] != 0;
     }
     if (tid == 0) {
-        for (int i = 0; i < 6; ++i) tc::mbar_init(mb + 8 * i, 1);
+        for (int i = 0; i < 7; ++i) tc::mbar_init(mb + 8 * i, 1);
         tc::fence_mbar_init();
         // arm the exchange barriers for step 0; start the first W_a load
         tc::mbar_arrive_expect_tx(MB_PART, (CL - 1) * PART_BYTES);
@@ -304,7 +308,26 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     uint32_t mword = 0xFFFFFFFFu;
     if (!p.teacher && grp == 0 && p.mask && live && p.T > 0) mword = __ldg(p.mask + (size_t)b * W + (a0 >> 5));
 
-    if (issuer) {  // MMA1 of step 0
+    // Injected wait (tests of the timeout path): one thread of every CTA waits on a barrier
+    // that nothing completes, after the prologue's W_a load has landed and before any MMA or
+    // exchange, so nothing of this kernel is in flight when it gives up.  Every CTA of the
+    // cluster gives up the same way, records WM_ERR_TIMEOUT and skips all T steps; no CTA
+    // then sends anything into another, and all of them still meet at the final cluster
+    // barrier and free their TMEM.
+    int t_end = p.T;
+    if (p.test_wait) {
+        if (tid == 0) {
+            tc::mbar_wait_bounded(MB_W, 0, WAIT_POLLS);
+            if (!tc::mbar_wait_bounded(MB_NEVER, 0, p.test_wait)) {
+                s_abort = 1;
+                atomicExch(p.status, (int)WM_ERR_TIMEOUT);
+            }
+        }
+        __syncthreads();
+        if (s_abort) t_end = 0;
+    }
+
+    if (issuer && t_end > 0) {  // MMA1 of step 0
         tc::fence_after_sync();
         mma1(Z / 16, K1 / 16, false);
         mma1(0, Z / 16, true);
@@ -312,7 +335,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     }
     __syncwarp();  // the MMA warp reconverges before the next aligned barrier
 
-    for (int t = 0; t < p.T; ++t) {
+    for (int t = 0; t < t_end; ++t) {
         const uint32_t step = p.t0 + (uint32_t)t;
         const size_t tb = (size_t)t * p.B + b;
         const uint32_t parity = (uint32_t)t & 1u;
@@ -877,6 +900,8 @@ cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaSt
     p.z_out = a.z_out; p.actions = a.actions; p.rewards = a.rewards; p.done = a.done;
     p.h_final = a.h_final; p.c_final = a.c_final; p.h_seq = a.h_seq; p.c_seq = a.c_seq;
     p.mdn_seq = a.mdn_seq; p.comp_seq = a.comp_seq;
+    p.test_wait = h->test_wait;
+    h->test_wait = 0;
     cudaError_t e;
     {
         wm_ktime kt(h, WM_KERNEL_FUSED, s);
@@ -899,6 +924,8 @@ cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cuda
     p.z_seq = a.z_seq; p.act_in = a.actions; p.lengths = a.lengths;
     p.h_seq = a.h_seq; p.c_seq = a.c_seq; p.mdn_seq = a.mdn_seq;
     p.nll_part = (float *)ws;
+    p.test_wait = h->test_wait;
+    h->test_wait = 0;
     cudaError_t e;
     {
         wm_ktime kt(h, WM_KERNEL_FUSED, s);

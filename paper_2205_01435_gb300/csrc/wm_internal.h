@@ -130,6 +130,8 @@ struct wm_handle {
     cudaStream_t copy_in = nullptr, copy_out = nullptr;  // per-step staging copies (lazy)
     std::vector<cudaEvent_t> events;                       // per-step staging events (grows)
     int *status = nullptr;       // device status word (WM_ERR_TIMEOUT etc.)
+    mutable uint32_t test_wait = 0;  // wm_inject_wait_timeout: polls of the next call's injected
+                                     // wait (consumed by that call's first fused / GEMM launch)
     int last_path = 0;
     mutable int last_launches = 0;   // kernels launched by the last call
     mutable wm_timer timer;

@@ -130,6 +130,9 @@ struct GemmGrid {
     // candidate ((ep0 + 256 m) / pop_E) mod pop_P, which start at row candidate * pop_rows
     unsigned long long ep0;
     int pop_P, pop_E, pop_rows;
+    // failure injection (wm_inject_wait_timeout): > 0 makes the kernel wait, before it issues
+    // any MMA or copy, on a barrier that nothing completes, at most this many polls
+    uint32_t test_wait;
 };
 
 // ---------------------------------------------------------------------------
@@ -591,12 +594,12 @@ struct EpiGatesT {
             if (a >= p.A && b < p.B && n == 0 && x.cg == 0) report_status(x.status, WM_ERR_INVALID_ARG);
             if (a < 0 || a >= p.A) a = -1;
         }
-        pr.a = (a >= 0 && !pr.fz) ? a : -1;
+        pr.a = (a >= 0 && a < p.A && !pr.fz) ? a : -1;
         ld_wa(p, pr.a, n, x.cg, 0, pr.wi);
         ld_wa(p, pr.a, n, x.cg, 2, pr.wg);
         if (TWO) {
             const int a2 = p.act2[bb];
-            pr.a2 = (a2 >= 0 && !pr.fz) ? a2 : -1;
+            pr.a2 = (a2 >= 0 && a2 < p.A && !pr.fz) ? a2 : -1;
             ld_wa(p, pr.a2, n, x.cg, 0, pr.wi2);
             ld_wa(p, pr.a2, n, x.cg, 2, pr.wg2);
         }
@@ -1005,7 +1008,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     static_assert(BN % 16 == 0 && BNH % 8 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4];
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4],
+        bar_never;
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1023,6 +1027,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             tc::mbar_init(tc::smem_u32(&bar_acce[a]), 2 * EPI_WARPS);  // the leader's: both CTAs' warps
         }
         for (int q = 0; q < 4; ++q) tc::mbar_init(tc::smem_u32(&bar_stage[q]), 1);
+        tc::mbar_init(tc::smem_u32(&bar_never), 1);
         tc::fence_mbar_init();
         s_abort = 0;
     }
@@ -1035,7 +1040,19 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // the previous kernel of the stream; every read of its outputs comes after this wait.
     // (It returns at once for a launch without programmatic serialization.)
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    const int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
+    int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
+    // Injected wait (tests of the timeout path): one thread of each CTA waits on a barrier
+    // that nothing completes, before any MMA or copy is issued.  Both CTAs of every pair give
+    // up the same way, record WM_ERR_TIMEOUT and take no tile, so nothing is in flight; the
+    // set-up's TMEM is still freed at the end.
+    if (g.test_wait) {
+        if (tid == 0 && !tc::mbar_wait_bounded(tc::smem_u32(&bar_never), 0, g.test_wait)) {
+            s_abort = 1;
+            atomicExch(g.status, (int)WM_ERR_TIMEOUT);
+        }
+        __syncthreads();
+        if (s_abort) ntiles = 0;
+    }
     auto wait = [&](uint32_t bar, uint32_t parity) {
         if (!s_abort && !tc::mbar_wait_bounded(bar, parity, POLLS)) {
             s_abort = 1;
@@ -1198,6 +1215,9 @@ __global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const floa
     }
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)p.B; i += (size_t)gridDim.x * blockDim.x) {
         fz0[i] = fz1[i] = done0 ? (done0[i] != 0) : 0;
+        // no action until a controller epilogue chooses one (a launch that gave up chooses none)
+        p.act[i] = -1;
+        if (p.act2) p.act2[i] = -1;
         if (p.rt0) {
             p.rt[i] = p.rt0[i];
             p.mem[i] = p.mem0[i];
@@ -1557,7 +1577,14 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         io.fz_cur = w.fz[t & 1];
         io.fz_next = w.fz[(t + 1) & 1];
         // the controller's weight rows: the tile's candidate's, when there is a population
-        const GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status, teacher ? 0ull : ra->ep0, h->P, h->E, A};
+        GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status, teacher ? 0ull : ra->ep0, h->P, h->E, A};
+        // an injected wait (wm_inject_wait_timeout) goes to the call's first GEMM launch
+        uint32_t test_wait = 0;
+        if (t == 0) {
+            test_wait = h->test_wait;
+            h->test_wait = 0;
+        }
+        if (!teacher) g1.test_wait = test_wait;
         if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
         if (!teacher && !hier) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
@@ -1581,7 +1608,8 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
             }
             ++launches;
         }
-        const GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
+        GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
+        if (teacher) g2.test_wait = test_wait;
         {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
             if (hier) e = launch_gemm<256, 1, 2, EpiGates2, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);

@@ -84,6 +84,8 @@ def _load():
     lib.wm_mdn_nll_backward.restype = C.c_int
     lib.wm_mdn_nll.argtypes = [P, C.c_int, C.c_int] + [P] * 7 + [P]
     lib.wm_mdn_nll.restype = C.c_int
+    lib.wm_inject_wait_timeout.argtypes = [P, C.c_uint]
+    lib.wm_inject_wait_timeout.restype = C.c_int
     lib.wm_sync.argtypes = [P]
     lib.wm_sync.restype = C.c_int
     lib.wm_last_error.argtypes = [P]
@@ -194,6 +196,10 @@ def wm_mdn_nll_backward(h, N: int, T: int, z_seq, actions, lengths, nll, grads: 
     g = wm_grads(*[_ptr(grads.get(n)) for n, _ in wm_grads._fields_])
     _check(h, _lib.wm_mdn_nll_backward(h, N, T, _ptr(z_seq), _ptr(actions), _ptr(lengths), _ptr(nll),
                                        C.byref(g), C.c_void_p(stream)), "wm_mdn_nll_backward")
+
+
+def wm_inject_wait_timeout(h, polls: int):
+    _check(h, _lib.wm_inject_wait_timeout(h, int(polls)), "wm_inject_wait_timeout")
 
 
 def wm_sync(h):
@@ -354,6 +360,11 @@ class WorldModel:
 
     def sync(self):
         wm_sync(self.h)
+
+    def inject_wait_timeout(self, polls: int):
+        """Make the next fused / tensor-core call's first kernel give up on a wait that
+        nothing completes, after at most `polls` polls (tests of the timeout path)."""
+        wm_inject_wait_timeout(self.h, polls)
 
     @property
     def last_path(self) -> str:
