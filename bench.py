@@ -307,6 +307,9 @@ def run_nll(args) -> None:
     achieved = fl / (dom_ms / dom_n / 1e3) / 1e12
     if cfg["precision"] == "bf16" and dom in ("fused", "tc_gates", "tc_heads"):
         bound, peak, psrc = "tensor", peaks["bf16_tflops"], peaks["source"] + " bf16 burst"
+    elif dom in ("tc_gates", "tc_heads"):  # fp32 on the tensor cores: three bf16 passes
+        bound, peak = "tensor", peaks["bf16_tflops"] / 3
+        psrc = peaks["source"] + " bf16 burst / 3 (fp32 products as three bf16 passes)"
     else:
         bound, peak, psrc = "alu", fp32_simt_peak_tflops(), "derived: 152 SM x 128 fp32 FMA x 2 FLOP x 2.07 GHz"
     kname, ksrc = KERNELS[dom]
@@ -566,6 +569,11 @@ def run_ours(args) -> None:
     dom_ms, dom_n = timed[dom]
     launch_ms = dom_ms / dom_n
     fl = kernel_flops(dom, cfg, B, T, dom_n)
+    # the tensor family compacts the live episodes of a single controller before every step:
+    # its GEMMs compute live rows only, so their algorithmic work is the live fraction's
+    compacted = live is not None and path_name == "tensor" and not P
+    if compacted:
+        fl *= live["live_fraction"]
     achieved = fl / (launch_ms / 1e3) / 1e12
     unit = "TFLOP/s"
     if cfg["precision"] == "bf16" and dom in ("fused", "tc_ctrl", "tc_gates", "tc_heads"):
@@ -575,6 +583,9 @@ def run_ours(args) -> None:
         burst = dom == "fused"
         peak = peaks["bf16_tflops"] if burst else peaks["bf16_tflops_sustained"]
         peak_source = f"{peaks['source']} bf16 {'burst' if burst else 'sustained'}"
+    elif dom in ("tc_ctrl", "tc_gates", "tc_heads"):  # fp32 on the tensor cores: three bf16 passes
+        bound, peak = "tensor", peaks["bf16_tflops_sustained"] / 3
+        peak_source = f"{peaks['source']} bf16 sustained / 3 (fp32 products as three bf16 passes)"
     else:
         bound, peak = "alu", fp32_simt_peak_tflops()
         peak_source = "derived: 152 SM x 128 fp32 FMA x 2 FLOP x 2.07 GHz"
@@ -617,7 +628,10 @@ def run_ours(args) -> None:
             "gpu_launches": launches * args.steps,
             "roofline": roof, "clocks": clk.summary()}
     if live is not None:
-        line["live_steps"] = live  # value counts live pairs; frozen pairs are executed too
+        # value counts live pairs; the tensor family computes only those (compaction), the
+        # other families also execute the frozen pairs
+        live["frozen_pairs_executed"] = not compacted
+        line["live_steps"] = live
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(name, args.cpu_episodes, shaped=shaping is not None)
     if rank == 0:

@@ -36,9 +36,13 @@
  * A uniform is (x >> 8) * 2^-24.  Results therefore do not depend on how the
  * episodes are split across calls or devices.
  *
- * Precision: WM_FP32 computes in fp32.  WM_BF16 rounds every weight matrix to
- * bf16 (RNE) at wm_create and rounds the GEMM operands [z_t; h_t] and h' to
- * bf16; biases, accumulation, nonlinearities, state and sampling stay fp32.
+ * Precision: WM_FP32 gives fp32-accurate results: the stepwise family computes
+ * in fp32; the tensor-core family computes each contraction as three bf16
+ * products of operands split into bf16 hi and lo parts (x = hi + lo), with fp32
+ * accumulation (about 3e-6 relative error), and everything else in fp32.
+ * WM_BF16 rounds every weight matrix to bf16 (RNE) at wm_create and rounds the
+ * GEMM operands [z_t; h_t] and h' to bf16; biases, accumulation,
+ * nonlinearities, state and sampling stay fp32.
  *
  * Memory: every array argument below may be device memory (cudaMalloc'd,
  * managed) or host memory (pinned or pageable); the library tells them apart
@@ -202,7 +206,17 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *weights, wm_handle *
  * keyed to Philox as episode_offset + b and its steps as t0 + t, so a rollout
  * split over calls (resume: pass z_out[T], h_final, c_final, done[T-1]) or over
  * devices (shard: episode_offset) reproduces the unsplit one bit for bit.
- * B = 0 or T = 0 are valid (T = 0 only copies z0 to z_out[0]). */
+ * B = 0 or T = 0 are valid (T = 0 only copies z0 to z_out[0]).
+ *
+ * Models whose episodes end (done_terminates or noop_terminates) with one
+ * controller: the tensor-core family packs the live episodes into the first
+ * rows before every step and computes only those; a frozen episode's outputs
+ * are written without computing it.  Once every episode has ended the call
+ * issues no further step.  To notice that in time it keeps at most 4 steps in
+ * flight, so it returns when its last step has been issued, a few steps before
+ * the device has finished (not when per-step staging of host arrays or stream
+ * capture is in use: then every step is issued).  Results are the same bit for
+ * bit however far the host got. */
 wm_status wm_rollout(wm_handle *h, int B, int T, unsigned long long episode_offset,
                      unsigned int t0, const wm_rollout_io *io, void *cuda_stream);
 
@@ -240,7 +254,8 @@ typedef struct {
  * nll [N] is optional.  The reward, done, runtime, memory and value heads are
  * not in the loss.  On the bf16 path the operand rounding is treated as the
  * identity in the backward pass, and the backward's GEMM operands are bf16
- * (fp32 accumulation); the fp32 path computes in fp32.  The forward runs on the
+ * (fp32 accumulation); on the fp32 path the backward's GEMMs are fp32 and the
+ * forward is fp32-accurate (see Precision above).  The forward runs on the
  * kernel family wm_mdn_nll would pick; the batched GEMMs of the backward
  * (gate activations over all N*T rows, the heads' and the recurrent input
  * gradients, the weight gradients) are cuBLAS calls, the rest (the mixture

@@ -158,6 +158,7 @@ struct Stager : wm_step_stage {
         }
         return cudaSuccess;
     }
+    bool stepping() const override { return stepped; }
     cudaError_t after_init(cudaStream_t s) override {
         if (!stepped) return cudaSuccess;
         cudaError_t e = cudaEventRecord(ev[1], s);
@@ -665,7 +666,7 @@ wm_status wm_mdn_nll_backward(wm_handle *h, int N, int T, const float *z_seq, co
         return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
     if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
         return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
-    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N)
+    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N, T)
                                                                                       : wm_step_nll_ws(h, N);
     if ((e = grow(&h->ws, &h->ws_bytes, need)) != cudaSuccess) return cuda_fail(h, e, "workspace");
     if ((e = grow(&h->bws, &h->bws_bytes, wm_bw_ws(h, N, T))) != cudaSuccess)
@@ -733,7 +734,7 @@ wm_status wm_mdn_nll(wm_handle *h, int N, int T, const float *z_seq, const int32
         return fail(h, WM_ERR_UNSUPPORTED, "the fused family does not take this model / batch");
     if (path == WM_PATH_TENSOR && !wm_tc_supported(h))
         return fail(h, WM_ERR_UNSUPPORTED, "the tensor family does not take this model");
-    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N)
+    size_t need = path == WM_PATH_FUSED ? wm_fused_nll_ws(h, N) : path == WM_PATH_TENSOR ? wm_tc_ws(h, N, T)
                                                                                       : wm_step_nll_ws(h, N);
     e = grow(&h->ws, &h->ws_bytes, need);
     if (e != cudaSuccess) return cuda_fail(h, e, "workspace");

@@ -18,6 +18,7 @@ struct wm_step_stage {
     virtual cudaError_t after_init(cudaStream_t s) = 0;        // the init kernel is enqueued
     virtual cudaError_t before_step(int t, cudaStream_t s) = 0;  // before step t's first launch
     virtual cudaError_t after_step(int t, cudaStream_t s) = 0;   // after step t's last launch
+    virtual bool stepping() const = 0;  // whether outputs leave step by step (after_step copies)
     virtual ~wm_step_stage() {}
 };
 
@@ -76,6 +77,8 @@ struct wm_fused_weights {
 // Weights of the tensor-core family (bf16, K-major; orders in wm_tensor.cu).
 struct wm_tc_weights {
     void *wc, *wg, *wa, *wh;  // W_c^T [P*A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
+    // fp32 path: the weights are the bf16 sums hi + lo; these are the lo parts (else null)
+    void *wc_lo, *wg_lo, *wa_lo, *wh_lo;
     float *bc, *bg, *bh;
     int dims_per_tile, n_head_tiles, rd_tile, rd_col;  // reward, done (, runtime, memory) columns
     int sms;
@@ -130,6 +133,12 @@ struct wm_handle {
     cudaStream_t copy_in = nullptr, copy_out = nullptr;  // per-step staging copies (lazy)
     std::vector<cudaEvent_t> events;                       // per-step staging events (grows)
     int *status = nullptr;       // device status word (WM_ERR_TIMEOUT etc.)
+    // tensor family, compacted rollouts: a host-mapped word the compaction kernel sets to the
+    // call's sequence number once no episode is live, so that the host stops issuing steps
+    mutable int *dead_host = nullptr;
+    mutable int *dead_dev = nullptr;
+    mutable int call_seq = 0;
+    mutable std::vector<cudaEvent_t> step_events;  // the early stop's step events (lazy)
     mutable uint32_t test_wait = 0;  // wm_inject_wait_timeout: polls of the next call's injected
                                      // wait (consumed by that call's first fused / GEMM launch)
     int last_path = 0;
@@ -162,7 +171,9 @@ class wm_ktime {
 
 // ---- tensor-core family (wm_tensor.cu) ----------------------------------------
 int wm_tc_supported(const wm_handle *h);
-size_t wm_tc_ws(const wm_handle *h, int B);
+// workspace of a call of B rows; T_teacher >= 0: teacher-forced scoring of T_teacher steps
+// (its operand rows of all T_teacher + 1 frames), -1: a rollout
+size_t wm_tc_ws(const wm_handle *h, int B, int T_teacher = -1);
 cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w);
 void wm_tc_free(wm_handle *h);
 cudaError_t wm_tc_rollout(const wm_handle *h, const wm_rollout_dev &a, void *ws, cudaStream_t s);

@@ -29,6 +29,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <vector>
 
 #include "tc_ptx.cuh"
@@ -133,6 +134,9 @@ struct GemmGrid {
     // failure injection (wm_inject_wait_timeout): > 0 makes the kernel wait, before it issues
     // any MMA or copy, on a barrier that nothing completes, at most this many polls
     uint32_t test_wait;
+    // compacted live episodes: the rows to compute are *n_rows (written by the previous
+    // kernel), not m_tiles * 256
+    const int *n_rows;
 };
 
 // ---------------------------------------------------------------------------
@@ -146,6 +150,7 @@ struct StepIO {
     float ctrl_tau, mdn_tau;
     // state
     __nv_bfloat16 *x_cur, *x_next;  // [B, Z+H]
+    __nv_bfloat16 *x_next_lo;       // fp32 path: the lo parts of x_next (else null)
     float *c, *h32;                 // [B, H]
     int32_t *act;                   // [B] the step's action
     const uint8_t *fz_cur;
@@ -153,12 +158,17 @@ struct StepIO {
     // weights (packed orders, see wm_tc_pack)
     const float *b_ctrl, *b_gate, *b_head;
     const __nv_bfloat16 *wa;        // [A, 4H] gate-tile column order
+    const __nv_bfloat16 *wa_lo;     // fp32 path: the lo parts of wa
     // head tiles
     int dims_per_tile, rd_tile, rd_col;  // reward / done columns: tile, first column
     // inputs / outputs
     const uint32_t *mask;           // [T, B, W] or null
     const int32_t *act_in;          // teacher: [T, B]
     const float *z_seq;             // teacher: [T+1, B, Z]
+    // teacher: the head epilogue's targets, row e scores z_tgt[e]; nseq > 0: the rows are all
+    // (step, sequence) pairs e = t nseq + n of a batched head GEMM (else the rows of step t)
+    const float *z_tgt;
+    int nseq;
     const int32_t *lengths;
     float *z_out;                   // [T+1, B, Z]
     int32_t *actions;
@@ -187,6 +197,14 @@ struct StepIO {
     const uint32_t *loc_mask;       // [T, B, NX, WL] or null
     int32_t *loc_actions;           // [T, B] optional
     int32_t *act2;                  // [B]
+    // Compaction of the live episodes (rollouts whose episodes end): the step's GEMMs run
+    // over the *n_rows live rows only, and row r holds episode rows[r].  Row-keyed: the
+    // operands x, c, h32 and act, act2, logits, fz_cur, fz_next; episode-keyed: every [T, B]
+    // input and output, rt, mem and the Philox counters.  Null: row b is episode b of B.
+    const int32_t *rows;
+    const int *n_rows;
+    __device__ int live_rows() const { return n_rows ? *(volatile const int *)n_rows : B; }
+    __device__ int ep_of(int r) const { return rows ? rows[r] : r; }
 };
 
 // Epilogue thread layout: 16 warps; warp w reads TMEM lanes 32*(w%4).. (the rows of
@@ -204,7 +222,7 @@ struct EpiCtx {
     bool leader;        // lane 0 of the quadrant's first warp: issues the quadrant's TMA copies
     bool pending;       // leader: a prefetch not yet waited for (parity pending_phase)
     uint32_t pending_phase;
-    const CUtensorMap *tm_c, *tm_xs;
+    const CUtensorMap *tm_c, *tm_xs, *tm_xs2;  // c; X_next (and its lo part, fp32 path)
     int *abort_flag, *status;
     __device__ void sync() const { asm volatile("bar.sync %0, 128;" :: "r"(1 + quad) : "memory"); }
     __device__ float *slot(int g) const { return red + ((quad * 4 + g) * 32 + lane) * 2; }
@@ -243,6 +261,8 @@ struct EpiCtrl {
     struct Pre {
         uint32_t bits[NCH];  // the chunk's 16 mask bits (0 for rows that do not act)
         bool live;           // a row of the batch whose episode is not frozen
+        bool valid;          // a row of the batch
+        int e;               // its episode
     };
     // once per CTA, by all 512 epilogue threads (e = 0..511), before the first tile: the
     // bias of a single controller into every quadrant's copy
@@ -253,9 +273,11 @@ struct EpiCtrl {
     static __device__ void prefetch(const StepIO &, int, int, EpiCtx &) {}
     static __device__ void pre(const StepIO &p, int m, int, EpiCtx &x, Pre &q) {
         const int b = m * BM + x.row;
-        q.live = b < p.B && !p.fz_cur[b];
+        q.valid = b < p.live_rows();
+        q.live = q.valid && !p.fz_cur[b];
+        q.e = q.valid ? p.ep_of(b) : 0;
         const int A = p.A, W = (A + 31) >> 5, CW = A / 4, c_lo = x.cg * CW;
-        const uint32_t *mw = (q.live && p.mask) ? p.mask + ((size_t)p.t * p.B + b) * W : nullptr;
+        const uint32_t *mw = (q.live && p.mask) ? p.mask + ((size_t)p.t * p.B + q.e) * W : nullptr;
 #pragma unroll
         for (int k = 0; k < NCH; ++k) {
             const int c0 = c_lo + 16 * k;
@@ -297,7 +319,7 @@ struct EpiCtrl {
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &q, int, int) {
         (void)n;
         const int b = m * BM + x.row;
-        const bool valid = b < p.B, live = q.live;
+        const bool valid = q.valid, live = q.live;
         const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
         const float *bs = x.red + RED_FLOATS + x.quad * MAX_A;
         if (p.pop_P > 1) x.sync();  // the quadrant's bias copy (pre) is complete
@@ -379,7 +401,7 @@ struct EpiCtrl {
             if (!sampled) {
                 logp = draw ? -log_total : 0.f;  // the argmax: its logit is the maximum
             } else {
-                const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + b, p.step, RNG_CONTROLLER, 0).x) : 0.f;
+                const float u = draw ? to_uniform(rng_draw(p.seed, p.ep0 + q.e, p.step, RNG_CONTROLLER, 0).x) : 0.f;
                 const float target = u * total;
                 // the group holding the drawn point; if rounding puts the target at or past the
                 // total, the group holding the last valid action
@@ -449,7 +471,7 @@ struct EpiCtrl {
         if (!valid || x.cg != 0) return;
         if (!live) ga = -1;
         p.act[b] = ga;
-        const size_t tb = (size_t)p.t * p.B + b;
+        const size_t tb = (size_t)p.t * p.B + q.e;
         p.actions[tb] = ga;
         if (p.logp_seq) p.logp_seq[tb] = ga >= 0 ? logp : 0.f;
     }
@@ -469,7 +491,8 @@ struct EpiLogits {
     static __device__ void pre(const StepIO &, int, int, EpiCtx &, Pre &) {}
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int, EpiCtx &x, const Pre &, int, int) {
         const int b = m * BM + x.row;
-        const bool store = b < p.B && !p.fz_cur[b < p.B ? b : 0];  // frozen rows choose nothing
+        const int nrows = p.live_rows();
+        const bool store = b < nrows && !p.fz_cur[b < nrows ? b : 0];  // frozen rows choose nothing
         const int CW = p.A / 4, c_lo = x.cg * CW, nch = CW / 16;  // nch is warp-uniform
         const unsigned long long cand =
             p.pop_P > 1 ? ((p.ep0 + (unsigned long long)m * BM) / (unsigned long long)p.pop_E) % (unsigned long long)p.pop_P
@@ -499,9 +522,10 @@ struct EpiLogits {
 // among the other L under that xfer's location mask.
 __global__ void __launch_bounds__(256) k_tc_select(StepIO p) {
     const int warp = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-    if (warp >= p.B) return;
+    if (warp >= p.live_rows()) return;
     const int b = warp, A = p.A, NX = p.n_xfers, L = A - NX, W = (A + 31) >> 5, WL = (L + 31) >> 5;
-    const size_t tb = (size_t)p.t * p.B + b;
+    const int e = p.ep_of(b);
+    const size_t tb = (size_t)p.t * p.B + e;
     int x = -1, loc = -1;
     float lp = 0.f;
     if (!p.fz_cur[b]) {
@@ -510,7 +534,7 @@ __global__ void __launch_bounds__(256) k_tc_select(StepIO p) {
         ws.tau = p.ctrl_tau;
         ws.want_lp = p.logp_seq != nullptr;
         ws.seed = p.seed;
-        ws.episode = p.ep0 + b;
+        ws.episode = p.ep0 + e;
         ws.step = p.step;
         const float *l = p.logits + (size_t)b * A;
         const uint32_t *mw = p.mask ? p.mask + tb * W : nullptr;
@@ -542,11 +566,16 @@ __global__ void __launch_bounds__(256) k_tc_select(StepIO p) {
 // load latency it hides.)  The cell is formed gate by gate over the thread's 16
 // units, so that each gate's W_a segment is one 256-bit load.  TWO: a hierarchical action
 // adds a second action row (the location's) to every gate.
-template <bool TWO>
+// MODE 0: one action row, bf16 path.  MODE 1: two action rows (hierarchical action).
+// MODE 2: the fp32 path: the action row is gathered as its bf16 hi and lo parts (the two-row
+// machinery with the same action), the nonlinearities are the accurate ones, and h' is
+// stored as bf16 hi and lo parts.
+template <int MODE>
 struct EpiGatesT {
+    static constexpr bool TWO = MODE != 0, F32 = MODE == 2;
     static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
     static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
-    static constexpr uint32_t QUAD_STAGE = C_SLAB + X_SLAB;  // c (in place) | h' out
+    static constexpr uint32_t QUAD_STAGE = C_SLAB + (F32 ? 2 : 1) * X_SLAB;  // c (in place) | h' out (| h' lo)
     static constexpr bool TMA_STAGE = true;
     static constexpr uint32_t RED_BYTES = 0;
 
@@ -563,21 +592,23 @@ struct EpiGatesT {
 
     struct Pre {
         uint32_t wi[8], wg[8];    // the W_a row segments of gates i and g (16 units, bf16)
-        uint32_t wi2[8], wg2[8];  // TWO: the second action row's
+        uint32_t wi2[8], wg2[8];  // TWO: the second action row's (F32: the lo parts)
         int a, a2;                // the action rows (-1: none)
         bool fz;                  // frozen episode
+        int e;                    // the row's episode
     };
     static __device__ void init(const StepIO &, EpiCtx &, int) {}
     // one gate's W_a segment for the thread's 16 units: a single 32-byte sector, read with
     // one 256-bit load (half the L1 wavefronts of two 16-byte loads: each lane reads
     // another row, so every load instruction touches 32 lines)
-    static __device__ __forceinline__ void ld_wa(const StepIO &p, int a, int n, int q, int gate, uint32_t (&w)[8]) {
+    static __device__ __forceinline__ void ld_wa(const StepIO &p, int a, int n, int q, int gate, uint32_t (&w)[8],
+                                                 bool lo = false) {
         if (a < 0) {
 #pragma unroll
             for (int i = 0; i < 8; ++i) w[i] = 0u;
             return;
         }
-        const __nv_bfloat16 *src = p.wa + (size_t)a * 4 * p.H + 256 * n + 64 * gate + 16 * q;
+        const __nv_bfloat16 *src = (lo ? p.wa_lo : p.wa) + (size_t)a * 4 * p.H + 256 * n + 64 * gate + 16 * q;
         asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
                      : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
                      : "l"(src));
@@ -586,24 +617,34 @@ struct EpiGatesT {
     // (L2 gathers), so that their latency overlaps the mainloop
     static __device__ void pre(const StepIO &p, int m, int n, EpiCtx &x, Pre &pr) {
         const int b = m * BM + x.row;
-        const int bb = b < p.B ? b : 0;
+        const bool valid = b < p.live_rows();
+        const int bb = valid ? b : 0;
         pr.fz = p.fz_cur[bb] != 0;
+        pr.e = p.ep_of(bb);
         int a = p.act[bb];
         if (p.teacher) {
-            a = p.act_in[(size_t)p.t * p.B + bb];
-            if (a >= p.A && b < p.B && n == 0 && x.cg == 0) report_status(x.status, WM_ERR_INVALID_ARG);
+            a = p.act_in[(size_t)p.t * p.B + pr.e];
+            if (a >= p.A && valid && n == 0 && x.cg == 0) report_status(x.status, WM_ERR_INVALID_ARG);
             if (a < 0 || a >= p.A) a = -1;
         }
         pr.a = (a >= 0 && a < p.A && !pr.fz) ? a : -1;
         ld_wa(p, pr.a, n, x.cg, 0, pr.wi);
         ld_wa(p, pr.a, n, x.cg, 2, pr.wg);
         if (TWO) {
-            const int a2 = p.act2[bb];
-            pr.a2 = (a2 >= 0 && a2 < p.A && !pr.fz) ? a2 : -1;
-            ld_wa(p, pr.a2, n, x.cg, 0, pr.wi2);
-            ld_wa(p, pr.a2, n, x.cg, 2, pr.wg2);
+            if (F32) {
+                pr.a2 = pr.a;
+            } else {
+                const int a2 = p.act2[bb];
+                pr.a2 = (a2 >= 0 && a2 < p.A && !pr.fz) ? a2 : -1;
+            }
+            ld_wa(p, pr.a2, n, x.cg, 0, pr.wi2, F32);
+            ld_wa(p, pr.a2, n, x.cg, 2, pr.wg2, F32);
         }
     }
+    // the cell's nonlinearities: the hardware tanh on the bf16 path; accurate ones on the
+    // fp32 path (tanh.approx's relative error, about 2^-11, is above its tolerance)
+    static __device__ __forceinline__ float sig_(float x) { return F32 ? fmaf(0.5f, tanhf(0.5f * x), 0.5f) : sigmoid_hw(x); }
+    static __device__ __forceinline__ float tanh_(float x) { return F32 ? tanhf(x) : tanh_hw(x); }
     // pre-activations of one gate for the thread's 16 units: accumulator + bias + W_a[a]
     // (+ W_a[a2] when TWO)
     static __device__ __forceinline__ void gate_pre(uint32_t tacc, const float *bg, int gate, int ut,
@@ -638,8 +679,8 @@ struct EpiGatesT {
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &pr, int next_m,
                                int next_n) {
         const int b = m * BM + x.row;
-        const bool valid = b < p.B;
-        const int bb = valid ? b : 0;  // rows past B compute on row 0; TMA stores clip them
+        const bool valid = b < p.live_rows();
+        const int bb = valid ? b : 0;  // rows past the batch compute on row 0; TMA stores clip them
         const int H = p.H, r = x.lane, q = x.cg;
         const bool fz = pr.fz;
         const int ut = 16 * q, u0 = 64 * n + ut;  // the thread's first unit: in the tile, in H
@@ -648,8 +689,8 @@ struct EpiGatesT {
         ld_wa(p, pr.a, n, q, 1, wf);
         ld_wa(p, pr.a, n, q, 3, wo);
         if (TWO) {
-            ld_wa(p, pr.a2, n, q, 1, wf2);
-            ld_wa(p, pr.a2, n, q, 3, wo2);
+            ld_wa(p, pr.a2, n, q, 1, wf2, F32);
+            ld_wa(p, pr.a2, n, q, 3, wo2, F32);
         }
         const float *bg = p.b_gate + 256 * n + 16 * q;
         const bool store_h32 = valid && !fz && (p.h32_mode == 2 || (p.h32_mode == 1 && p.t == p.T - 1));
@@ -663,10 +704,10 @@ struct EpiGatesT {
             float g[16];
             gate_pre(tacc, bg, 0, ut, pr.wi, pr.wi2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]);
+            for (int j = 0; j < 16; ++j) hv[j] = sig_(g[j]);
             gate_pre(tacc, bg, 2, ut, pr.wg, pr.wg2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] *= tanh_hw(g[j]);
+            for (int j = 0; j < 16; ++j) hv[j] *= tanh_(g[j]);
         }
         x.wait_stage();  // the quadrant's c rows have landed
 #pragma unroll
@@ -679,11 +720,11 @@ struct EpiGatesT {
             gate_pre(tacc, bg, 1, ut, wf, wf2, g);
             if (!fz) {
 #pragma unroll
-                for (int j = 0; j < 16; ++j) cv[j] = sigmoid_hw(g[j]) * cv[j] + hv[j];
+                for (int j = 0; j < 16; ++j) cv[j] = sig_(g[j]) * cv[j] + hv[j];
             }
             gate_pre(tacc, bg, 3, ut, wo, wo2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] = sigmoid_hw(g[j]) * tanh_hw(cv[j]);
+            for (int j = 0; j < 16; ++j) hv[j] = sig_(g[j]) * tanh_(cv[j]);
         }
         if (fz) {  // frozen: h is the carried one
             const float4 *h4 = reinterpret_cast<const float4 *>(p.h32 + (size_t)bb * H + u0);
@@ -706,6 +747,16 @@ struct EpiGatesT {
                 pk[j] = *reinterpret_cast<uint32_t *>(&v);
             }
             *reinterpret_cast<uint4 *>(xs + sw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            if (F32) {  // the lo parts, h' - bf16(h')
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float a0 = hv[8 * i + 2 * j], a1 = hv[8 * i + 2 * j + 1];
+                    __nv_bfloat162 hi2 = *reinterpret_cast<__nv_bfloat162 *>(&pk[j]);
+                    __nv_bfloat162 v = __floats2bfloat162_rn(a0 - __low2float(hi2), a1 - __high2float(hi2));
+                    pk[j] = *reinterpret_cast<uint32_t *>(&v);
+                }
+                *reinterpret_cast<uint4 *>(xs + X_SLAB + sw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            }
         }
         if (store_h32) {
             float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)b * H + u0);
@@ -713,7 +764,7 @@ struct EpiGatesT {
             for (int i = 0; i < 4; ++i) h4[i] = make_float4(hv[4 * i], hv[4 * i + 1], hv[4 * i + 2], hv[4 * i + 3]);
         }
         if (valid) {
-            const size_t o = ((size_t)p.t * p.B + b) * H + u0;
+            const size_t o = ((size_t)p.t * p.B + pr.e) * H + u0;
             if (p.h_seq)
                 for (int j = 0; j < 16; ++j) p.h_seq[o + j] = hv[j];
             if (p.c_seq)
@@ -729,6 +780,7 @@ struct EpiGatesT {
                 tma_store_2d(x.tm_c, 64 * n, y, x.stage_u);
                 tma_store_2d(x.tm_c, 64 * n + 32, y, x.stage_u + 4096);
                 tma_store_2d(x.tm_xs, p.Z + 64 * n, y, x.stage_u + C_SLAB);
+                if (F32) tma_store_2d(x.tm_xs2, p.Z + 64 * n, y, x.stage_u + C_SLAB + X_SLAB);
                 bulk_commit();
                 bulk_wait_read();  // the slab may be refilled
             }
@@ -737,8 +789,9 @@ struct EpiGatesT {
     }
 };
 
-using EpiGates = EpiGatesT<false>;
-using EpiGates2 = EpiGatesT<true>;
+using EpiGates = EpiGatesT<0>;
+using EpiGates2 = EpiGatesT<1>;
+using EpiGates32 = EpiGatesT<2>;
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
 // Before the accumulator wait, the quadrant's 128 threads make the tile's random draws:
@@ -770,9 +823,9 @@ struct EpiHeads {
         for (int i = x.cg * 32 + x.lane; i < HEAD_TILE; i += 128) bq[i] = bh[i];
         // the row's draws for the tile's dims (a5, a7): Philox blocks of 4 dims
         const int b0 = m * BM + x.row;
-        const int b = b0 < p.B ? b0 : 0;
+        const int b = b0 < p.live_rows() ? b0 : 0;
         if (p.teacher || !(p.mdn_tau > 0.f) || p.fz_cur[b]) return;
-        const unsigned long long ep = p.ep0 + b;
+        const unsigned long long ep = p.ep0 + p.ep_of(b);
         const int d0 = n * p.dims_per_tile, nd = min(p.dims_per_tile, p.Z - d0);
         float *es = reinterpret_cast<float *>(x.stage), *us = reinterpret_cast<float *>(x.stage + US_OFF);
         for (int blk = (d0 >> 2) + x.cg; 4 * blk < d0 + nd; blk += 4) {
@@ -792,12 +845,14 @@ struct EpiHeads {
     }
     static __device__ void run(const StepIO &p, uint32_t tacc, int m, int n, EpiCtx &x, const Pre &, int, int) {
         const int b0 = m * BM + x.row;
-        const bool valid = b0 < p.B;
-        const int b = valid ? b0 : 0;  // rows past B compute on row 0 and store nothing
+        const int nrows = p.live_rows();
+        const bool valid = b0 < nrows;
+        const int b = valid ? b0 : 0;  // rows past the batch compute on row 0 and store nothing
+        const int e = p.ep_of(b);     // the row's episode
         const int Z = p.Z, K = p.K, KZ = K * Z, M = 3 * KZ, KX = Z + p.H;
         const int DS = (3 * K + 7) & ~7;  // columns per latent dim (8-aligned TMEM loads)
-        const bool fz = p.fz_cur[b] != 0;
-        const size_t tb = (size_t)p.t * p.B + b;
+        const bool fz = !p.teacher && p.fz_cur[b] != 0;
+        const size_t tb = (size_t)p.t * p.B + e;
         const int d0 = n * p.dims_per_tile;
         const int nd = min(p.dims_per_tile, Z - d0);
         const float *bh = reinterpret_cast<const float *>(x.stage + BIAS_OFF);  // the tile's bias
@@ -855,7 +910,7 @@ struct EpiHeads {
                 }
                 float zn;
                 if (p.teacher) {
-                    const float xv = p.z_seq[((size_t)(p.t + 1) * p.B + b) * Z + d];
+                    const float xv = p.z_tgt[(size_t)e * Z + d];
                     float mx = -INFINITY;
 #pragma unroll
                     for (int k = 0; k < 8; ++k) if (k < K) mx = fmaxf(mx, lg[k]);
@@ -928,10 +983,13 @@ struct EpiHeads {
             }
         }
         if (p.teacher && valid) {
-            const int len = p.lengths ? p.lengths[b] : p.T;
-            if (p.t == 0 && n == 0 && x.cg == 0 && (len < 0 || len > p.T))
+            const int sq = p.nseq ? e % p.nseq : e, tt = p.nseq ? e / p.nseq : p.t;  // sequence, step
+            const int len = p.lengths ? p.lengths[sq] : p.T;
+            if (tt == 0 && n == 0 && x.cg == 0 && (len < 0 || len > p.T))
                 report_status(x.status, WM_ERR_INVALID_ARG);
-            if (p.t < len) p.nll_part[((size_t)n * 4 + x.cg) * p.B + b] += nll;
+            float *part = p.nll_part + ((size_t)n * 4 + x.cg) * p.B + e;
+            if (p.nseq) *part = tt < len ? nll : 0.f;  // one row per (step, sequence)
+            else if (tt < len) *part += nll;
         }
         if (n == p.rd_tile) {
             const bool shaped = p.reward_mode == WM_REWARD_SHAPED;  // uniform
@@ -959,12 +1017,12 @@ struct EpiHeads {
                         const float mem = __uint_as_float(q[1]) + bh[p.rd_col + 3];
                         // valid: an action was taken (and, for an xfer, a location)
                         const bool ok = a >= 0 && (p.n_xfers == 0 || a == noop_a || p.act2[b] >= 0);
-                        rew = ok ? p.alpha * (p.rt[b] - rt) + p.beta * (p.mem[b] - mem) : p.invalid_reward;
-                        p.rt[b] = rt;
-                        p.mem[b] = mem;
+                        rew = ok ? p.alpha * (p.rt[e] - rt) + p.beta * (p.mem[e] - mem) : p.invalid_reward;
+                        p.rt[e] = rt;
+                        p.mem[e] = mem;
                     }
-                    if (p.rt_seq) p.rt_seq[tb] = p.rt[b];
-                    if (p.mem_seq) p.mem_seq[tb] = p.mem[b];
+                    if (p.rt_seq) p.rt_seq[tb] = p.rt[e];
+                    if (p.mem_seq) p.mem_seq[tb] = p.mem[e];
                 }
                 if (p.value_seq) p.value_seq[tb] = fz ? 0.f : vq + bh[p.rd_col + p.nr - 1];
                 p.rewards[tb] = fz ? 0.f : rew;
@@ -974,13 +1032,17 @@ struct EpiHeads {
         }
         // the quadrant's 32 x nd block of z', stored row-major by its 128 threads
         x.sync();
-        const int y0 = m * BM + 32 * x.quad, nrow = min(32, p.B - y0);
-        for (int e = x.cg * 32 + x.lane; e < nrow * nd; e += 128) {
-            const int rr = e / nd, i = e - rr * nd;
+        const int y0 = m * BM + 32 * x.quad, nrow = min(32, nrows - y0);
+        for (int j = x.cg * 32 + x.lane; j < nrow * nd; j += 128) {
+            const int rr = j / nd, i = j - rr * nd;
             const size_t bb = (size_t)(y0 + rr);
             const float zn = zs[rr * ZS_PITCH + i];
-            if (!p.teacher) p.z_out[((size_t)(p.t + 1) * p.B + bb) * Z + d0 + i] = zn;
-            p.x_next[bb * KX + d0 + i] = __float2bfloat16_rn(zn);
+            if (!p.teacher) p.z_out[((size_t)(p.t + 1) * p.B + p.ep_of((int)bb)) * Z + d0 + i] = zn;
+            if (p.x_next) {  // (a batched scoring GEMM has no next operand: the frames are staged)
+                const __nv_bfloat16 zh = __float2bfloat16_rn(zn);
+                p.x_next[bb * KX + d0 + i] = zh;
+                if (p.x_next_lo) p.x_next_lo[bb * KX + d0 + i] = __float2bfloat16_rn(zn - __bfloat162float(zh));
+            }
         }
         x.sync();  // the staging may be rewritten by the next tile
     }
@@ -995,17 +1057,29 @@ struct EpiHeads {
 // MMA thread waits for a stage once, issues all its MMAs back to back and commits once, to
 // the stage's "empty" barrier: any wait or commit on the issuing thread lets the tensor
 // pipe drain, and a pair's multicast commit costs more than one k-step's MMAs can hide.
-template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
+// NP = 3: the fp32 path.  Each fp32 operand is split into bf16 parts x = x_hi + x_lo (x_hi =
+// bf16(x), x_lo = bf16(x - x_hi)), and the accumulator takes three passes over K: A_hi B_hi,
+// A_hi B_lo (tmB2) and A_lo B_hi (tmA2).  The dropped A_lo B_lo term and the parts'
+// residuals are below 2^-16 of each product.
+template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1, int NP = 1>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmXs, GemmGrid g,
-              StepIO io) {
+              const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmXs,
+              const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
+              const __grid_constant__ CUtensorMap tmXs2, GemmGrid g, StepIO io) {
     constexpr int TILE_N = BN * NSUB, BNH = BN / 2;
     constexpr uint32_t A_BYTES = BM * BK * 2, B_SUB = BNH * BK * 2, B_BYTES = B_SUB * NSUB;
     constexpr uint32_t KSTEP_BYTES = A_BYTES + B_BYTES, STAGE_BYTES = KPS * KSTEP_BYTES;  // per CTA
     constexpr int NACC = TILE_N <= 256 ? 2 : 1;
     constexpr uint32_t ACC_COLS = 256;
     static_assert(BN % 16 == 0 && BNH % 8 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
+    // Compacted live episodes: a pair with no tile this step leaves before its set-up (both
+    // CTAs read the same row count, written by the previous kernel).
+    if (g.n_rows) {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        const int mt = (*(volatile const int *)g.n_rows + 2 * BM - 1) / (2 * BM);
+        if ((int)(blockIdx.x >> 1) >= mt * g.n_tiles) return;
+    }
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4],
@@ -1040,7 +1114,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // the previous kernel of the stream; every read of its outputs comes after this wait.
     // (It returns at once for a launch without programmatic serialization.)
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    int ntiles = g.m_tiles * g.n_tiles;  // m_tiles counts 256-row tiles
+    int m_tiles = g.m_tiles;  // 256-row tiles
+    if (g.n_rows) m_tiles = (*(volatile const int *)g.n_rows + 2 * BM - 1) / (2 * BM);
+    int ntiles = m_tiles * g.n_tiles;
+    const int ksteps = NP * g.k_steps;  // k-steps per tile over all passes
     // Injected wait (tests of the timeout path): one thread of each CTA waits on a barrier
     // that nothing completes, before any MMA or copy is issued.  Both CTAs of every pair give
     // up the same way, record WM_ERR_TIMEOUT and take no tile, so nothing is in flight; the
@@ -1069,19 +1146,26 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 const int brow = g.pop_P > 1 ? (int)(((g.ep0 + (unsigned long long)m * (2 * BM)) /
                                                       (unsigned long long)g.pop_E) % (unsigned long long)g.pop_P) * g.pop_rows
                                              : 0;
-                for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
-                    const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;  // k-steps in this stage
+                for (int ks0 = 0; ks0 < ksteps; ks0 += KPS) {
+                    const int nk = ksteps - ks0 < KPS ? ksteps - ks0 : KPS;  // k-steps in this stage
                     const uint32_t full_ldr = tc::map_rank(full_b(stage), 0);
                     wait(empty_b(stage), phase ^ 1u);  // the stage's previous MMAs are done
                     if (s_abort) break;
                     for (int h = 0; h < nk; ++h) {
-                        const int ks = ks0 + h;
+                        int ks = ks0 + h;
+                        const CUtensorMap *ma = &tmA, *mb = &tmB;
+                        if (NP > 1) {  // pass 0: A_hi B_hi, 1: A_hi B_lo, 2: A_lo B_hi
+                            const int pass = ks / g.k_steps;
+                            ks -= pass * g.k_steps;
+                            if (pass == 1) mb = &tmB2;
+                            if (pass == 2) ma = &tmA2;
+                        }
                         const uint32_t sa = smem_u + stage * STAGE_BYTES + h * KSTEP_BYTES;
                         if (h == 0 && rank == 0) tc::mbar_arrive_expect_tx(full_b(stage), 2 * nk * KSTEP_BYTES);
-                        tma_load_2sm(sa, &tmA, g.a_col0 + ks * BK, (2 * m + (int)rank) * BM, full_ldr);
+                        tma_load_2sm(sa, ma, g.a_col0 + ks * BK, (2 * m + (int)rank) * BM, full_ldr);
 #pragma unroll
                         for (int s = 0; s < NSUB; ++s)
-                            tma_load_2sm(sa + A_BYTES + s * B_SUB, &tmB, ks * BK,
+                            tma_load_2sm(sa + A_BYTES + s * B_SUB, mb, ks * BK,
                                          brow + n * TILE_N + s * BN + (int)rank * BNH, full_ldr);
                     }
                     if (s_abort) break;
@@ -1098,8 +1182,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 wait(tc::smem_u32(&bar_acce[acc]), acc_phase ^ 1u);
                 tc::fence_after_sync();
                 const uint32_t dcol = tm + acc * ACC_COLS;
-                for (int ks0 = 0; ks0 < g.k_steps; ks0 += KPS) {
-                    const int nk = g.k_steps - ks0 < KPS ? g.k_steps - ks0 : KPS;
+                for (int ks0 = 0; ks0 < ksteps; ks0 += KPS) {
+                    const int nk = ksteps - ks0 < KPS ? ksteps - ks0 : KPS;
                     wait(full_b(stage), phase);
                     if (s_abort) break;
                     tc::fence_after_sync();
@@ -1148,6 +1232,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x.pending_phase = 0;
         x.tm_c = &tmC;
         x.tm_xs = &tmXs;
+        x.tm_xs2 = &tmXs2;
         x.abort_flag = &s_abort;
         x.status = g.status;
         int acc = 0;
@@ -1196,7 +1281,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
 // ---------------------------------------------------------------------------
 __global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const float *c0, const uint8_t *done0,
-                          __nv_bfloat16 *x0, uint8_t *fz0, uint8_t *fz1, int n_head_tiles) {
+                          __nv_bfloat16 *x0, __nv_bfloat16 *x0_lo, uint8_t *fz0, uint8_t *fz1, int n_head_tiles,
+                          int *dstep, int *cnt) {
+    if (cnt && blockIdx.x == 0 && threadIdx.x < 4) cnt[threadIdx.x] = 0;
     const int KX = p.Z + p.H;
     const size_t nx = (size_t)p.B * KX;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nx; i += (size_t)gridDim.x * blockDim.x) {
@@ -1204,7 +1291,9 @@ __global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const floa
         float v;
         if (k < (size_t)p.Z) v = p.teacher ? p.z_seq[b * p.Z + k] : z0[b * p.Z + k];
         else v = h0 ? h0[b * p.H + (k - p.Z)] : 0.f;
-        x0[i] = __float2bfloat16_rn(v);
+        const __nv_bfloat16 vh = __float2bfloat16_rn(v);
+        x0[i] = vh;
+        if (x0_lo) x0_lo[i] = __float2bfloat16_rn(v - __bfloat162float(vh));
         if (k >= (size_t)p.Z) {
             const size_t j = b * p.H + (k - p.Z);
             p.h32[j] = h0 ? h0[j] : 0.f;
@@ -1218,6 +1307,7 @@ __global__ void k_tc_init(StepIO p, const float *z0, const float *h0, const floa
         // no action until a controller epilogue chooses one (a launch that gave up chooses none)
         p.act[i] = -1;
         if (p.act2) p.act2[i] = -1;
+        if (dstep) dstep[i] = p.T;
         if (p.rt0) {
             p.rt[i] = p.rt0[i];
             p.mem[i] = p.mem0[i];
@@ -1240,6 +1330,271 @@ __global__ void k_tc_finish(int B, int H, const float *h32, const float *c, floa
             for (int t = 0; t < n_parts; ++t) s += (double)nll_part[(size_t)t * B + i];
             nll[i] = (float)s;
         }
+}
+
+// ---------------------------------------------------------------------------
+// Batched teacher-forced scoring: the operand rows of all T + 1 frames are staged at once
+// (frame f, sequence n at row f N + n: z part from z_seq; the h part of frame f + 1 is
+// written by step f's gate epilogue), the recurrence runs one gate GEMM per step, and one
+// head GEMM then scores all N T (step, sequence) rows.
+__global__ void k_tc_frames(int N, int T, int Z, int KX, const float *__restrict__ z_seq,
+                            __nv_bfloat16 *__restrict__ x, __nv_bfloat16 *__restrict__ x_lo) {
+    const size_t n = (size_t)T * N * Z;  // frames 1..T (frame 0 is the init kernel's)
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = (size_t)N + i / Z, k = i % Z;  // operand row, z column
+        const float v = z_seq[r * Z + k];
+        const __nv_bfloat16 vh = __float2bfloat16_rn(v);
+        x[r * KX + k] = vh;
+        if (x_lo) x_lo[r * KX + k] = __float2bfloat16_rn(v - __bfloat162float(vh));
+    }
+}
+
+// nll[n] = sum over the head tiles' partials and the steps of sequence n (uncounted steps
+// hold 0), in a fixed order
+__global__ void k_tc_nll_reduce(int N, int T, int parts, const float *__restrict__ part, float *__restrict__ nll) {
+    for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < N; n += gridDim.x * blockDim.x) {
+        double s = 0.0;
+        for (int j = 0; j < parts; ++j)
+            for (int t = 0; t < T; ++t) s += (double)part[((size_t)j * T + t) * N + n];
+        nll[n] = (float)s;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Compaction of the live episodes (rollouts whose episodes end: done head or NO-OP).
+// Before step t's GEMMs, k_tc_compact packs the rows whose episode is still live after
+// step t-1 into the first rows of the operand buffers, so that the three GEMMs of step t
+// compute live episodes only, and writes step t's outputs of every frozen episode (the
+// ones the GEMMs no longer see).  A row's arithmetic does not depend on its position in a
+// tile, so the order in which blocks claim their output rows (an atomic per block) changes
+// no result.  One block per 256 rows of step t-1, one warp per row copy.
+struct CompactIO {
+    int B, Z, H, KX, M, t;
+    const int32_t *rows_in;           // [B] row -> episode at step t-1 (null: row b is episode b)
+    const int *n_in;                  // rows of step t-1 (null: B)
+    const uint8_t *dies;              // [B] row-keyed: the episode ended at step t-1 (at t = 0: done0)
+    const __nv_bfloat16 *x_in;        // [B, KX] operands after step t-1
+    __nv_bfloat16 *x_out;             // [B, KX] compacted
+    const __nv_bfloat16 *x_in_lo;     // fp32 path: the lo parts (else null)
+    __nv_bfloat16 *x_out_lo;
+    const float *c_in, *h32;          // [B, H] row-keyed c, h after step t-1
+    float *c_out;                     // [B, H] compacted c
+    int32_t *rows_out;                // [B] row -> episode at step t
+    int *n_out;                       // rows of step t (zero on entry)
+    int *n_clear;                     // set to zero: the counter of step t + 1
+    int T;
+    int fill;                         // write the frozen episodes' step-t outputs now (else one
+                                      // kernel writes every step's after the last step)
+    int *dstep;                       // [B] first step at which the episode is frozen (T: never)
+    int *dead_flag;                   // host-mapped: set to call_id once no episode is live
+    int call_id;
+    const int *n_prev2;               // rows of step t-2 (null at t < 2)
+    float *hfin, *cfin;               // [B, H] an ended episode's h, c
+    const float *rt, *mem;            // [B] carried predictions (shaped reward)
+    float *z_out;                     // step t's outputs of frozen episodes
+    int32_t *actions;
+    float *rewards;
+    uint8_t *done;
+    float *h_seq, *c_seq, *mdn_seq;
+    uint8_t *comp_seq;
+    float *logp_seq, *value_seq, *rt_seq, *mem_seq;
+    int32_t *loc_actions;
+};
+
+// Element k of frozen episode e's step-t outputs (k < fill_elems): z repeated (and component
+// 255), h and c repeated, mixture outputs 0, then the scalars (no action, reward 0, done).
+__device__ __forceinline__ int fill_elems(const CompactIO &q) {
+    return q.Z + ((q.h_seq || q.c_seq) ? q.H : 0) + (q.mdn_seq ? q.M : 0) + 1;
+}
+__device__ void fill_elem(const CompactIO &q, int e, int k, const float *hs, const float *cs) {
+    const size_t tb = (size_t)q.t * q.B + e;
+    if (k < q.Z) {
+        q.z_out[(tb + q.B) * q.Z + k] = q.z_out[tb * q.Z + k];
+        if (q.comp_seq) q.comp_seq[tb * q.Z + k] = 255;
+        return;
+    }
+    k -= q.Z;
+    if (q.h_seq || q.c_seq) {
+        if (k < q.H) {
+            if (q.h_seq) q.h_seq[tb * q.H + k] = hs[k];
+            if (q.c_seq) q.c_seq[tb * q.H + k] = cs[k];
+            return;
+        }
+        k -= q.H;
+    }
+    if (q.mdn_seq) {
+        if (k < q.M) {
+            q.mdn_seq[tb * q.M + k] = 0.f;
+            return;
+        }
+    }
+    q.actions[tb] = -1;
+    q.rewards[tb] = 0.f;
+    q.done[tb] = 1;
+    if (q.logp_seq) q.logp_seq[tb] = 0.f;
+    if (q.value_seq) q.value_seq[tb] = 0.f;
+    if (q.rt_seq) q.rt_seq[tb] = q.rt[e];
+    if (q.mem_seq) q.mem_seq[tb] = q.mem[e];
+    if (q.loc_actions) q.loc_actions[tb] = -1;
+}
+
+constexpr int CROWS = 16;         // rows of step t-1 per block
+constexpr int CTHREADS = 128;
+
+// Every phase is flattened over the block's (or the grid's) threads, so that many
+// independent 16-byte copies are in flight: a warp walking rows one by one is bound by
+// memory latency, not bandwidth.
+__global__ void __launch_bounds__(CTHREADS) k_tc_compact(CompactIO q) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // the previous step's outputs are complete
+    __shared__ int s_pos[CROWS], s_e[CROWS], s_base;
+    const int tid = (int)threadIdx.x;
+    const int n_in = q.n_in ? *(volatile const int *)q.n_in : q.B;
+    const int r0 = (int)blockIdx.x * CROWS;
+    if (r0 < n_in) {  // block-uniform
+        const int nrow = min(CROWS, n_in - r0);
+        if (tid < 32) {  // one warp claims the block's output rows
+            const int r = r0 + tid;
+            const bool in = tid < nrow;
+            const bool keep = in && !(q.dies && q.dies[r]);
+            const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+            int base = 0;
+            if (tid == 0 && bal) base = atomicAdd(q.n_out, __popc(bal));
+            base = __shfl_sync(0xffffffffu, base, 0);
+            if (in) {
+                const int e = q.rows_in ? q.rows_in[r] : r;
+                s_e[tid] = e;
+                s_pos[tid] = keep ? base + __popc(bal & ((1u << tid) - 1u)) : -1;
+                if (keep) q.rows_out[s_pos[tid]] = e;
+                else q.dstep[e] = q.t;
+            }
+        }
+        __syncthreads();
+        // survivors: the operand row and c to their new row; ended episodes: h, c recorded
+        const int XC = q.KX / 8, CC = q.H / 4;  // 16-byte chunks per row
+        const int XL = q.x_in_lo ? XC : 0;       // the operand's lo parts (fp32 path)
+        const int per = max(XC + XL + CC, 2 * CC);
+        const uint4 *__restrict__ xi = reinterpret_cast<const uint4 *>(q.x_in);
+        uint4 *__restrict__ xo = reinterpret_cast<uint4 *>(q.x_out);
+        const uint4 *__restrict__ ci = reinterpret_cast<const uint4 *>(q.c_in);
+        const uint4 *__restrict__ hi = reinterpret_cast<const uint4 *>(q.h32);
+        uint4 *__restrict__ co = reinterpret_cast<uint4 *>(q.c_out);
+        uint4 *__restrict__ hf = reinterpret_cast<uint4 *>(q.hfin);
+        uint4 *__restrict__ cf = reinterpret_cast<uint4 *>(q.cfin);
+#pragma unroll 4
+        for (int i = tid; i < nrow * per; i += CTHREADS) {
+            const int j = i / per, k = i - j * per;
+            const size_t rr = (size_t)(r0 + j);
+            const int pos = s_pos[j];
+            if (pos >= 0) {
+                if (k < XC) xo[(size_t)pos * XC + k] = xi[rr * XC + k];
+                else if (k < XC + XL)
+                    reinterpret_cast<uint4 *>(q.x_out_lo)[(size_t)pos * XC + k - XC] =
+                        reinterpret_cast<const uint4 *>(q.x_in_lo)[rr * XC + k - XC];
+                else if (k < XC + XL + CC) co[(size_t)pos * CC + k - XC - XL] = ci[rr * CC + k - XC - XL];
+            } else {
+                const size_t e = (size_t)s_e[j];
+                if (k < CC) hf[e * CC + k] = hi[rr * CC + k];
+                else if (k < 2 * CC) cf[e * CC + k - CC] = ci[rr * CC + k - CC];
+            }
+        }
+        // the ended episodes' step-t outputs, from their rows
+        const int fe = q.fill ? fill_elems(q) : 0;
+        for (int i = tid; i < nrow * fe; i += CTHREADS) {
+            const int j = i / fe, k = i - j * fe;
+            if (s_pos[j] >= 0) continue;
+            const size_t rr = (size_t)(r0 + j);
+            fill_elem(q, s_e[j], k, q.h32 + rr * q.H, q.c_in + rr * q.H);
+        }
+    }
+    // episodes frozen before this step's compaction stay frozen: their step-t outputs, over
+    // the whole grid (an episode ending now reads dstep as T or t: either way it is not here)
+    if (q.fill && q.t > 0) {
+        const int fe = fill_elems(q);
+        const size_t n = (size_t)q.B * fe, stride = (size_t)gridDim.x * CTHREADS;
+        for (size_t i = (size_t)blockIdx.x * CTHREADS + tid; i < n; i += stride) {
+            const int e = (int)(i / fe), k = (int)(i - (size_t)e * fe);
+            if (q.dstep[e] >= q.t) continue;
+            fill_elem(q, e, k, q.hfin + (size_t)e * q.H, q.cfin + (size_t)e * q.H);
+        }
+    }
+    if (blockIdx.x == 0 && tid == 0) {
+        *q.n_clear = 0;
+        // every episode has ended (reported once, at the first step that sees it): the host
+        // may stop issuing steps
+        if (n_in == 0 && q.dead_flag && (!q.n_prev2 || *(volatile const int *)q.n_prev2 != 0))
+            *(volatile int *)q.dead_flag = q.call_id;
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Every frozen episode's outputs of every step from the one at which it froze, after the
+// last step (calls whose outputs are not staged step by step).  One warp per episode: each
+// lane reads its z (and h, c) values once and writes them to every frozen step.
+__global__ void k_tc_fill_frozen(CompactIO q) {
+    const int lane = threadIdx.x & 31;
+    const int nw = (int)((gridDim.x * blockDim.x) >> 5);
+    for (int e = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); e < q.B; e += nw) {
+        const int d = q.dstep[e];
+        if (d >= q.T) continue;  // warp-uniform
+        const size_t B = (size_t)q.B;
+        for (int k = lane; k < q.Z; k += 32) {
+            const float v = q.z_out[((size_t)d * B + e) * q.Z + k];  // z of the step it froze at
+            for (int t = d; t < q.T; ++t) {
+                const size_t tb = (size_t)t * B + e;
+                q.z_out[(tb + B) * q.Z + k] = v;
+                if (q.comp_seq) q.comp_seq[tb * q.Z + k] = 255;
+            }
+        }
+        if (q.h_seq || q.c_seq)
+            for (int k = lane; k < q.H; k += 32) {
+                const float hv = q.hfin[(size_t)e * q.H + k], cv = q.cfin[(size_t)e * q.H + k];
+                for (int t = d; t < q.T; ++t) {
+                    const size_t tb = (size_t)t * B + e;
+                    if (q.h_seq) q.h_seq[tb * q.H + k] = hv;
+                    if (q.c_seq) q.c_seq[tb * q.H + k] = cv;
+                }
+            }
+        if (q.mdn_seq)
+            for (int k = lane; k < q.M; k += 32)
+                for (int t = d; t < q.T; ++t) q.mdn_seq[((size_t)t * B + e) * q.M + k] = 0.f;
+        const float rt = q.rt_seq ? q.rt[e] : 0.f, mem = q.mem_seq ? q.mem[e] : 0.f;
+        for (int t = d + lane; t < q.T; t += 32) {  // the scalars, a step per lane
+            const size_t tb = (size_t)t * B + e;
+            q.actions[tb] = -1;
+            q.rewards[tb] = 0.f;
+            q.done[tb] = 1;
+            if (q.logp_seq) q.logp_seq[tb] = 0.f;
+            if (q.value_seq) q.value_seq[tb] = 0.f;
+            if (q.rt_seq) q.rt_seq[tb] = rt;
+            if (q.mem_seq) q.mem_seq[tb] = mem;
+            if (q.loc_actions) q.loc_actions[tb] = -1;
+        }
+    }
+}
+
+// h_final, c_final after a compacted rollout: the last step's rows, and the recorded state
+// of the episodes frozen before it
+__global__ void k_tc_finish_compact(int B, int H, int T, const int *dstep, const int32_t *rows, const int *n_rows,
+                                    const float *h32, const float *c, const float *hfin, const float *cfin,
+                                    float *h_final, float *c_final) {
+    const int warp = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    const int nw = (int)((gridDim.x * blockDim.x) >> 5);
+    const int n = *n_rows;
+    // (the caller's arrays need only 4-byte alignment: element-wise copies)
+    for (int r = warp; r < n; r += nw) {
+        const int e = rows[r];
+        for (int i = lane; i < H; i += 32) {
+            if (h_final) h_final[(size_t)e * H + i] = h32[(size_t)r * H + i];
+            if (c_final) c_final[(size_t)e * H + i] = c[(size_t)r * H + i];
+        }
+    }
+    for (int e = warp; e < B; e += nw) {
+        if (dstep[e] >= T) continue;  // live at the last step: one of its rows
+        for (int i = lane; i < H; i += 32) {
+            if (h_final) h_final[(size_t)e * H + i] = hfin[(size_t)e * H + i];
+            if (c_final) c_final[(size_t)e * H + i] = cfin[(size_t)e * H + i];
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -1281,12 +1636,17 @@ size_t gemm_smem() {
            4 * (size_t)Epi::QUAD_STAGE + Epi::RED_BYTES;
 }
 
-template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
-cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
-                        const CUtensorMap &mxs, GemmGrid g, const StepIO &io, int sms, cudaStream_t s,
-                        bool pdl) {
+// The operand maps of one GEMM: A (and its lo part), B (and its lo part); the fp32 path's
+// second maps are unused on the bf16 path (NP = 1).
+struct OpMaps {
+    const CUtensorMap *a, *b, *a2, *b2;
+};
+
+template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1, int NP = 1>
+cudaError_t launch_gemm(const OpMaps &op, const CUtensorMap &mc, const CUtensorMap &mxs, const CUtensorMap &mxs2,
+                        GemmGrid g, const StepIO &io, int sms, cudaStream_t s, bool pdl) {
     const size_t smem = gemm_smem<BN, NSUB, STAGES, Epi, KPS>();
-    auto kern = k_tc_gemm<BN, NSUB, STAGES, Epi, KPS>;
+    auto kern = k_tc_gemm<BN, NSUB, STAGES, Epi, KPS, NP>;
     cudaLaunchConfig_t lc = {};
     cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1313,26 +1673,40 @@ cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUte
     const int tiles = g.m_tiles * g.n_tiles;
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     lc.gridDim = dim3(2 * pairs);
-    return cudaLaunchKernelEx(&lc, kern, ma, mb, mc, mxs, g, io);
+    return cudaLaunchKernelEx(&lc, kern, *op.a, *op.b, mc, mxs, *op.a2, *op.b2, mxs2, g, io);
 }
 
 inline size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct TcWs {
     __nv_bfloat16 *x[2];
+    __nv_bfloat16 *x_lo[2];  // fp32 path: the lo parts of x
     float *c, *h32, *nll_part, *rt, *mem;
     float *logits;   // hierarchical action: [B, A]
     int32_t *act2;   // hierarchical action: the location's action row
     int32_t *act;
     uint8_t *fz[2];
+    // compaction of live episodes (models whose episodes end)
+    float *c2, *hfin, *cfin;
+    int32_t *rows[2];
+    int *cnt;        // [4] ring of per-step row counts
+    int *dstep;      // [B] first step at which each episode is frozen
+    // batched teacher-forced scoring
+    __nv_bfloat16 *xall, *xall_lo;  // [(T+1) B, KX] the operand rows of every frame
+    float *part;                    // [4 head tiles, T B] per-(step, sequence) partials
 };
 
-TcWs carve_ws(const wm_handle *h, int B, void *ws) {
+// models whose episodes can end get the compaction buffers (and use them when P = 1)
+inline bool can_compact(const wm_config &c) { return c.done_terminates || c.noop_terminates; }
+
+TcWs carve_ws(const wm_handle *h, int B, void *ws, int T_teacher = -1) {
     const wm_config &c = h->cfg;
     const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
     char *p = (char *)ws;
     TcWs w{};
     for (int i = 0; i < 2; ++i) { w.x[i] = (__nv_bfloat16 *)p; p += a256((size_t)B * KX * 2); }
+    if (c.precision == WM_FP32)
+        for (int i = 0; i < 2; ++i) { w.x_lo[i] = (__nv_bfloat16 *)p; p += a256((size_t)B * KX * 2); }
     w.c = (float *)p; p += a256((size_t)B * H * 4);
     w.h32 = (float *)p; p += a256((size_t)B * H * 4);
     w.act = (int32_t *)p; p += a256((size_t)B * 4);
@@ -1343,7 +1717,22 @@ TcWs carve_ws(const wm_handle *h, int B, void *ws) {
         w.logits = (float *)p; p += a256((size_t)B * c.a_dim * 4);
         w.act2 = (int32_t *)p; p += a256((size_t)B * 4);
     }
+    if (can_compact(c)) {
+        w.c2 = (float *)p; p += a256((size_t)B * H * 4);
+        w.hfin = (float *)p; p += a256((size_t)B * H * 4);
+        w.cfin = (float *)p; p += a256((size_t)B * H * 4);
+        for (int i = 0; i < 2; ++i) { w.rows[i] = (int32_t *)p; p += a256((size_t)B * 4); }
+        w.cnt = (int *)p; p += 256;
+        w.dstep = (int *)p; p += a256((size_t)B * 4);
+    }
     w.nll_part = (float *)p;
+    p += a256((size_t)4 * h->tc.n_head_tiles * B * 4);
+    if (T_teacher >= 0) {  // scoring: frame 0 is written by the init kernel even when T = 0
+        const size_t rows = (size_t)(T_teacher + 1) * B;
+        w.xall = (__nv_bfloat16 *)p; p += a256(rows * KX * 2);
+        if (c.precision == WM_FP32) { w.xall_lo = (__nv_bfloat16 *)p; p += a256(rows * KX * 2); }
+        w.part = (float *)p;
+    }
     return w;
 }
 
@@ -1354,12 +1743,18 @@ TcWs carve_ws(const wm_handle *h, int B, void *ws) {
 
 int wm_tc_supported(const wm_handle *h) { return h->tc.ok; }
 
-size_t wm_tc_ws(const wm_handle *h, int B) {
+size_t wm_tc_ws(const wm_handle *h, int B, int T_teacher) {
     const wm_config &c = h->cfg;
     const size_t KX = (size_t)c.z_dim + c.h_dim, H = c.h_dim;
-    return 2 * a256((size_t)B * KX * 2) + 2 * a256((size_t)B * H * 4) + a256((size_t)B * 4) + 2 * a256(B) +
+    const size_t rows = T_teacher >= 0 ? (size_t)(T_teacher + 1) * B : 0;
+    const size_t teach = T_teacher >= 0 ? (c.precision == WM_FP32 ? 2 : 1) * a256(rows * KX * 2) +
+                                              a256((size_t)4 * h->tc.n_head_tiles * T_teacher * B * 4)
+                                        : 0;
+    return teach + 2 * a256((size_t)B * KX * 2) + 2 * a256((size_t)B * H * 4) + a256((size_t)B * 4) + 2 * a256(B) +
            2 * a256((size_t)B * 4) + a256((size_t)4 * h->tc.n_head_tiles * B * 4) + 256 +
-           (c.n_xfers > 0 ? a256((size_t)B * c.a_dim * 4) + a256((size_t)B * 4) : 0);
+           (c.n_xfers > 0 ? a256((size_t)B * c.a_dim * 4) + a256((size_t)B * 4) : 0) +
+           (can_compact(c) ? 3 * a256((size_t)B * H * 4) + 3 * a256((size_t)B * 4) + 256 : 0) +
+           (c.precision == WM_FP32 ? 2 * a256((size_t)B * KX * 2) : 0);
 }
 
 cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
@@ -1367,7 +1762,10 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
     wm_tc_weights &T = h->tc;
     memset(&T, 0, sizeof(T));
     const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, K = c.k_mix, KX = Z + H;
-    if (c.precision != WM_BF16 || H % 64 != 0 || A % 64 != 0 || (A > 256 && A != 512) || K > 8 || Z % 8 != 0 ||
+    // fp32 models: the split path (flat actions only: the gate epilogue's second-row slots
+    // carry the action row's lo part)
+    const bool f32 = c.precision == WM_FP32;
+    if ((f32 && c.n_xfers > 0) || H % 64 != 0 || A % 64 != 0 || (A > 256 && A != 512) || K > 8 || Z % 8 != 0 ||
         !get_encode())
         return cudaSuccess;
     const int DS = (3 * K + 7) & ~7;  // head columns per latent dim
@@ -1441,6 +1839,50 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         if (r == cudaSuccess) r = cudaMemcpy(*dst, src, bytes, cudaMemcpyHostToDevice);
         return r;
     };
+    if (f32) {  // the lo parts: bf16(w - hi), from the same canonical values
+        auto lo_of = [&](std::vector<__nv_bfloat16> &hi, auto canon) {
+            std::vector<__nv_bfloat16> lo(hi.size());
+            for (size_t i = 0; i < hi.size(); ++i) lo[i] = bf(canon(i) - __bfloat162float(hi[i]));
+            return lo;
+        };
+        auto wc_lo = lo_of(wc, [&](size_t i) { const size_t a = i / KX, k = i % KX; return w->W_ctrl[k * A + a]; });
+        auto wg_lo = lo_of(wg, [&](size_t i) {
+            const size_t n = i / KX, k = i % KX;
+            const size_t j = n / 256, gate = (n % 256) / 64, u = n % 64, col = gate * H + 64 * j + u;
+            const size_t src = k < (size_t)Z ? k : k + A;
+            return w->W_lstm[src * 4 * H + col];
+        });
+        auto wa_lo = lo_of(wa, [&](size_t i) {
+            const size_t a = i / (4 * H), n = i % (4 * H);
+            const size_t j = n / 256, gate = (n % 256) / 64, u = n % 64, col = gate * H + 64 * j + u;
+            return w->W_lstm[(Z + a) * 4 * H + col];
+        });
+        std::vector<float> whf(wh.size(), 0.f);  // canonical values of the packed head rows
+        for (int d = 0; d < Z; ++d)
+            for (int part = 0; part < 3; ++part)
+                for (int k = 0; k < K; ++k) {
+                    const size_t row = (size_t)(d / dpt) * HEAD_TILE + DS * (d % dpt) + 3 * k + part;
+                    const size_t col = (size_t)part * K * Z + (size_t)d * K + k;
+                    for (int i = 0; i < H; ++i) whf[row * H + i] = w->W_mdn[(size_t)i * M + col];
+                }
+        {
+            const size_t rr = (size_t)rd_tile * HEAD_TILE + rd_col;
+            for (int i = 0; i < H; ++i) {
+                whf[rr * H + i] = w->w_rew[i];
+                whf[(rr + 1) * H + i] = w->w_done[i];
+                if (c.reward_mode == WM_REWARD_SHAPED) {
+                    whf[(rr + 2) * H + i] = w->w_rt[i];
+                    whf[(rr + 3) * H + i] = w->w_mem[i];
+                }
+                if (c.value_head) whf[(rr + h->NR - 1) * H + i] = w->w_val[i];
+            }
+        }
+        auto wh_lo = lo_of(wh, [&](size_t i) { return whf[i]; });
+        if ((e = up(&T.wc_lo, wc_lo.data(), wc_lo.size() * 2)) != cudaSuccess) return e;
+        if ((e = up(&T.wg_lo, wg_lo.data(), wg_lo.size() * 2)) != cudaSuccess) return e;
+        if ((e = up(&T.wa_lo, wa_lo.data(), wa_lo.size() * 2)) != cudaSuccess) return e;
+        if ((e = up(&T.wh_lo, wh_lo.data(), wh_lo.size() * 2)) != cudaSuccess) return e;
+    }
     if ((e = up(&T.wc, wc.data(), wc.size() * 2)) != cudaSuccess) return e;
     if ((e = up(&T.wg, wg.data(), wg.size() * 2)) != cudaSuccess) return e;
     if ((e = up(&T.wa, wa.data(), wa.size() * 2)) != cudaSuccess) return e;
@@ -1464,17 +1906,26 @@ cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, cons
     wm_tc_weights &T = h->tc;
     const wm_config &c = h->cfg;
     const int A = c.a_dim, KX = c.z_dim + c.h_dim;
-    std::vector<__nv_bfloat16> wc((size_t)P * A * KX);
+    const bool f32 = c.precision == WM_FP32;
+    std::vector<__nv_bfloat16> wc((size_t)P * A * KX), wcl(f32 ? wc.size() : 0);
     for (int g = 0; g < P; ++g)
         for (int a = 0; a < A; ++a)
-            for (int k = 0; k < KX; ++k)
-                wc[((size_t)g * A + a) * KX + k] = __float2bfloat16_rn(W_ctrl[((size_t)g * KX + k) * A + a]);
+            for (int k = 0; k < KX; ++k) {
+                const size_t i = ((size_t)g * A + a) * KX + k;
+                const float v = W_ctrl[((size_t)g * KX + k) * A + a];
+                wc[i] = __float2bfloat16_rn(v);
+                if (f32) wcl[i] = __float2bfloat16_rn(v - __bfloat162float(wc[i]));
+            }
     cudaFree(T.wc);
+    cudaFree(T.wc_lo);
     cudaFree(T.bc);
     T.wc = nullptr;
+    T.wc_lo = nullptr;
     T.bc = nullptr;
     cudaError_t e = cudaMalloc(&T.wc, wc.size() * 2);
     if (e == cudaSuccess) e = cudaMemcpy(T.wc, wc.data(), wc.size() * 2, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && f32) e = cudaMalloc(&T.wc_lo, wcl.size() * 2);
+    if (e == cudaSuccess && f32) e = cudaMemcpy(T.wc_lo, wcl.data(), wcl.size() * 2, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMalloc((void **)&T.bc, (size_t)P * A * 4);
     if (e == cudaSuccess) e = cudaMemcpy(T.bc, b_ctrl, (size_t)P * A * 4, cudaMemcpyHostToDevice);
     return e;
@@ -1483,6 +1934,11 @@ cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, cons
 void wm_tc_free(wm_handle *h) {
     wm_tc_weights &T = h->tc;
     cudaFree(T.wc); cudaFree(T.wg); cudaFree(T.wa); cudaFree(T.wh);
+    cudaFree(T.wc_lo); cudaFree(T.wg_lo); cudaFree(T.wa_lo); cudaFree(T.wh_lo);
+    if (h->dead_host) cudaFreeHost(h->dead_host);
+    h->dead_host = h->dead_dev = nullptr;
+    for (cudaEvent_t ev : h->step_events) cudaEventDestroy(ev);
+    h->step_events.clear();
     cudaFree(T.bc); cudaFree(T.bg); cudaFree(T.bh);
     memset(&T, 0, sizeof(T));
 }
@@ -1495,7 +1951,7 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     const int B = teacher ? na->N : ra->B, Tn = teacher ? na->T : ra->T;
     const int Z = c.z_dim, A = c.a_dim, H = c.h_dim, KX = Z + H;
     if (B == 0) { h->last_launches = 0; return cudaSuccess; }
-    TcWs w = carve_ws(h, B, ws);
+    TcWs w = carve_ws(h, B, ws, teacher ? Tn : -1);
     StepIO io{};
     io.B = B; io.Z = Z; io.A = A; io.H = H; io.K = c.k_mix; io.T = Tn;
     io.seed = c.seed; io.teacher = teacher;
@@ -1541,12 +1997,18 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     }
     int launches = 0;
     const int init_grid = 1024;
+    // Rollouts whose episodes end compact their live episodes before every step (one
+    // controller per call: a population's tiles must stay whole).
+    const bool compact = !teacher && can_compact(c) && h->P <= 1 && Tn > 0;
     io.fz_cur = w.fz[0];
     {
         wm_ktime kt(h, WM_KERNEL_AUX, s);
         k_tc_init<<<init_grid, 256, 0, s>>>(io, teacher ? nullptr : ra->z0, teacher ? nullptr : ra->h0,
-                                            teacher ? nullptr : ra->c0, teacher ? nullptr : ra->done0, w.x[0],
-                                            w.fz[0], w.fz[1], T.n_head_tiles);
+                                            teacher ? nullptr : ra->c0,
+                                            (teacher || compact) ? nullptr : ra->done0,
+                                            teacher ? w.xall : w.x[0], teacher ? w.xall_lo : w.x_lo[0], w.fz[0], w.fz[1],
+                                            T.n_head_tiles, compact ? w.dstep : nullptr,
+                                            compact ? w.cnt : nullptr);
     }
     ++launches;
     wm_step_stage *hooks = teacher ? nullptr : ra->stage;  // per-step staging of host arrays
@@ -1554,30 +2016,205 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         cudaError_t he = hooks->after_init(s);
         if (he != cudaSuccess) return he;
     }
-    CUtensorMap mx[2], mxs[2], mwc, mwg, mwh, mc;
+    const bool f32 = c.precision == WM_FP32;  // the split path: second operand maps and lo outputs
+    CUtensorMap mx[2], mxs[2], mwc, mwg, mwh, mc, mc2, mxl[2], mxsl[2], mwcl, mwgl, mwhl;
     // B-operand boxes are half an instantiated BN (each CTA of a pair loads half the rows;
     // rows past A read as zero)
     const uint32_t ctrl_box = A > 128 ? 128u : 64u;
     if (!make_map(&mx[0], w.x[0], B, KX, BM) || !make_map(&mx[1], w.x[1], B, KX, BM) ||
         !make_map(&mxs[0], w.x[0], B, KX, 32) || !make_map(&mxs[1], w.x[1], B, KX, 32) ||
-        !make_map(&mc, w.c, B, H, 32, true) ||
+        !make_map(&mc, w.c, B, H, 32, true) || (compact && !make_map(&mc2, w.c2, B, H, 32, true)) ||
         !make_map(&mwc, T.wc, (uint64_t)h->P * A, KX, ctrl_box) || !make_map(&mwg, T.wg, 4 * H, KX, 128) ||
         !make_map(&mwh, T.wh, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE / 2))
         return cudaErrorInvalidValue;
+    if (f32) {
+        if (!make_map(&mxl[0], w.x_lo[0], B, KX, BM) || !make_map(&mxl[1], w.x_lo[1], B, KX, BM) ||
+            !make_map(&mxsl[0], w.x_lo[0], B, KX, 32) || !make_map(&mxsl[1], w.x_lo[1], B, KX, 32) ||
+            !make_map(&mwcl, T.wc_lo, (uint64_t)h->P * A, KX, ctrl_box) || !make_map(&mwgl, T.wg_lo, 4 * H, KX, 128) ||
+            !make_map(&mwhl, T.wh_lo, (uint64_t)T.n_head_tiles * HEAD_TILE, H, HEAD_TILE / 2))
+            return cudaErrorInvalidValue;
+    } else {  // unused by the bf16 kernels
+        mxl[0] = mx[0]; mxl[1] = mx[1]; mxsl[0] = mxs[0]; mxsl[1] = mxs[1];
+        mwcl = mwc; mwgl = mwg; mwhl = mwh;
+    }
+    io.wa_lo = (const __nv_bfloat16 *)T.wa_lo;
     const int m_tiles = (B + 2 * BM - 1) / (2 * BM);  // 256-row tiles, one per CTA pair
     // Programmatic dependent launch hides the ~4 us between consecutive launches (a fifth of
     // a call at B = 8192), but made the long launches of B = 65536 3% slower: on below 32768.
     const bool pdl = B < 32768;
+    if (teacher) {  // batched scoring: the recurrence step by step, then one head GEMM
+        const size_t fr = (size_t)B * KX;  // elements of one frame of operand rows
+        cudaError_t e = cudaSuccess;
+        if (Tn > 0) {
+            wm_ktime kt(h, WM_KERNEL_AUX, s);
+            k_tc_frames<<<init_grid, 256, 0, s>>>(B, Tn, Z, KX, na->z_seq, w.xall, w.xall_lo);
+            ++launches;
+        }
+        io.x_cur = io.x_next = io.x_next_lo = nullptr;
+        for (int t = 0; t < Tn && e == cudaSuccess; ++t) {
+            io.t = t;
+            io.step = (uint32_t)t;
+            // this step's operand rows (frame t) and where h' goes (frame t + 1)
+            CUtensorMap ma, mal, ms, msl;
+            if (!make_map(&ma, w.xall + t * fr, B, KX, BM) || !make_map(&ms, w.xall + (t + 1) * fr, B, KX, 32))
+                return cudaErrorInvalidValue;
+            if (f32) {
+                if (!make_map(&mal, w.xall_lo + t * fr, B, KX, BM) || !make_map(&msl, w.xall_lo + (t + 1) * fr, B, KX, 32))
+                    return cudaErrorInvalidValue;
+            } else {
+                mal = ma;
+                msl = ms;
+            }
+            GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
+            if (t == 0) {  // an injected wait (wm_inject_wait_timeout) goes to the first GEMM
+                g2.test_wait = h->test_wait;
+                h->test_wait = 0;
+            }
+            const OpMaps opg{&ma, &mwg, &mal, &mwgl};
+            {
+                wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
+                if (f32) e = launch_gemm<256, 1, 2, EpiGates32, 2, 3>(opg, mc, ms, msl, g2, io, T.sms, s, pdl);
+                else e = launch_gemm<256, 1, 2, EpiGates, 2>(opg, mc, ms, ms, g2, io, T.sms, s, pdl);
+            }
+            ++launches;
+        }
+        if (e != cudaSuccess) return e;
+        const int parts = 4 * T.n_head_tiles;
+        if (Tn > 0) {  // every (step, sequence) row: h_{t+1} of frame t + 1 against z_{t+1}
+            CUtensorMap mh, mhl;
+            const int rows = B * Tn;
+            if (!make_map(&mh, w.xall + fr, (uint64_t)rows, KX, BM)) return cudaErrorInvalidValue;
+            if (f32) {
+                if (!make_map(&mhl, w.xall_lo + fr, (uint64_t)rows, KX, BM)) return cudaErrorInvalidValue;
+            } else {
+                mhl = mh;
+            }
+            StepIO hio = io;
+            hio.B = rows;
+            hio.t = 0;
+            hio.nseq = B;
+            hio.z_tgt = na->z_seq + (size_t)B * Z;
+            hio.nll_part = w.part;
+            const GemmGrid g3{(rows + 2 * BM - 1) / (2 * BM), T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
+            const OpMaps oph{&mh, &mwh, &mhl, &mwhl};
+            wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
+            if (f32) e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2, 3>(oph, mc, mc, mc, g3, hio, T.sms, s, pdl);
+            else e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(oph, mc, mc, mc, g3, hio, T.sms, s, pdl);
+            ++launches;
+            if (e != cudaSuccess) return e;
+        }
+        {
+            wm_ktime kt(h, WM_KERNEL_AUX, s);
+            k_tc_nll_reduce<<<(B + 255) / 256, 256, 0, s>>>(B, Tn, parts, w.part, na->nll);
+        }
+        ++launches;
+        h->last_launches = launches;
+        return cudaGetLastError();
+    }
+    float *cbuf[2] = {w.c, w.c2};
+    const bool staged = hooks && hooks->stepping();  // host outputs copied step by step
+    CompactIO q{};  // compaction: the fields that do not change from step to step
+    // Early stop: once every episode has ended, the remaining steps would only launch empty
+    // kernels; the compaction kernel then sets a host-mapped word to this call's number and
+    // the host issues no further step.  To see it in time, the host keeps at most LOOKAHEAD
+    // steps in flight (it waits for step t - LOOKAHEAD before issuing step t), so such a call
+    // returns once its last step is issued, a few steps before the device finishes.  Where
+    // the host stops depends on timing; the results do not.  Not with per-step staging or
+    // during stream capture.
+    constexpr int LOOKAHEAD = 4;
+    bool early = false;
+    if (compact && !staged) {
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(s, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone) {
+            if (!h->dead_host && cudaHostAlloc((void **)&h->dead_host, sizeof(int), cudaHostAllocMapped) == cudaSuccess) {
+                *h->dead_host = 0;
+                if (cudaHostGetDevicePointer((void **)&h->dead_dev, h->dead_host, 0) != cudaSuccess) {
+                    cudaFreeHost(h->dead_host);
+                    h->dead_host = h->dead_dev = nullptr;
+                }
+            }
+            while (h->step_events.size() < (size_t)LOOKAHEAD) {
+                cudaEvent_t ev = nullptr;
+                if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) break;
+                h->step_events.push_back(ev);
+            }
+            cudaGetLastError();
+            early = h->dead_dev != nullptr && h->step_events.size() >= (size_t)LOOKAHEAD;
+        }
+    }
+    if (compact) {
+        q.dead_flag = early ? h->dead_dev : nullptr;
+        q.call_id = ++h->call_seq;
+        q.B = B; q.Z = Z; q.H = H; q.KX = KX; q.M = 3 * c.k_mix * Z; q.T = Tn;
+        q.fill = staged;  // staged outputs leave step by step: fill each step's
+        q.dstep = w.dstep; q.h32 = w.h32;
+        q.hfin = w.hfin; q.cfin = w.cfin; q.rt = w.rt; q.mem = w.mem;
+        q.z_out = ra->z_out; q.actions = ra->actions; q.rewards = ra->rewards; q.done = ra->done;
+        q.h_seq = ra->h_seq; q.c_seq = ra->c_seq; q.mdn_seq = ra->mdn_seq; q.comp_seq = ra->comp_seq;
+        q.logp_seq = io.logp_seq; q.value_seq = io.value_seq; q.rt_seq = io.rt_seq; q.mem_seq = io.mem_seq;
+        q.loc_actions = io.loc_actions;
+    }
     cudaError_t e = cudaSuccess;
+    int t_end = Tn;  // steps issued
     for (int t = 0; t < Tn && e == cudaSuccess; ++t) {
+        if (early && t >= LOOKAHEAD) {
+            if ((e = cudaEventSynchronize(h->step_events[t % LOOKAHEAD])) != cudaSuccess) break;
+            if (*(volatile int *)h->dead_host == q.call_id) {
+                t_end = t;
+                break;
+            }
+        }
         io.t = t;
         io.step = teacher ? (uint32_t)t : ra->t0 + (uint32_t)t;
-        io.x_cur = w.x[t & 1];
-        io.x_next = w.x[(t + 1) & 1];
-        io.fz_cur = w.fz[t & 1];
-        io.fz_next = w.fz[(t + 1) & 1];
+        // operands: X ping-pongs between the two buffers; when compacting, the live rows are
+        // packed from x[0] (written by the previous step) into x[1] (this step's operand), and
+        // this step writes x[0] again; c alternates between its two buffers
+        const int xa = compact ? 1 : (t & 1), xn = compact ? 0 : ((t + 1) & 1);
+        io.x_cur = w.x[xa];
+        io.x_next = w.x[xn];
+        io.x_next_lo = w.x_lo[xn];
+        io.fz_cur = w.fz[compact ? 0 : (t & 1)];
+        io.fz_next = w.fz[compact ? 1 : ((t + 1) & 1)];
+        const CUtensorMap &mC = (compact && ((t + 1) & 1)) ? mc2 : mc;
+        if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
+        if (compact) {
+            q.t = t;
+            q.rows_in = t ? w.rows[(t - 1) & 1] : nullptr;
+            q.n_in = t ? w.cnt + ((t - 1) & 3) : nullptr;
+            q.dies = t ? w.fz[1] : ra->done0;
+            q.x_in = w.x[0]; q.x_out = w.x[1];
+            q.x_in_lo = w.x_lo[0]; q.x_out_lo = w.x_lo[1];
+            q.c_in = cbuf[t & 1]; q.c_out = cbuf[(t + 1) & 1];
+            q.rows_out = w.rows[t & 1]; q.n_out = w.cnt + (t & 3); q.n_clear = w.cnt + ((t + 1) & 3);
+            q.n_prev2 = t >= 2 ? w.cnt + ((t - 2) & 3) : nullptr;
+            io.rows = w.rows[t & 1];
+            io.n_rows = w.cnt + (t & 3);
+            io.c = cbuf[(t + 1) & 1];
+            cudaLaunchConfig_t lc = {};
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            at[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+            {  // a block per CROWS rows, and enough threads for the frozen episodes' outputs
+                const size_t fe = q.fill ? (size_t)Z + ((q.h_seq || q.c_seq) ? H : 0) + (q.mdn_seq ? q.M : 0) + 1 : 0;
+                const size_t rows_blocks = ((size_t)B + CROWS - 1) / CROWS;
+                const size_t fill_blocks = std::min<size_t>(((size_t)B * fe + 4 * CTHREADS - 1) / (4 * CTHREADS),
+                                                            (size_t)16 * T.sms);
+                lc.gridDim = dim3((unsigned)std::max(rows_blocks, fill_blocks));
+            }
+            lc.blockDim = dim3(CTHREADS);
+            lc.stream = s;
+            lc.attrs = at;
+            lc.numAttrs = 1;
+            {
+                wm_ktime kt(h, WM_KERNEL_AUX, s);
+                e = cudaLaunchKernelEx(&lc, k_tc_compact, q);
+            }
+            ++launches;
+            if (e != cudaSuccess) break;
+        }
         // the controller's weight rows: the tile's candidate's, when there is a population
         GemmGrid g1{m_tiles, 1, (KX + BK - 1) / BK, 0, h->status, teacher ? 0ull : ra->ep0, h->P, h->E, A};
+        g1.n_rows = io.n_rows;
         // an injected wait (wm_inject_wait_timeout) goes to the call's first GEMM launch
         uint32_t test_wait = 0;
         if (t == 0) {
@@ -1585,20 +2222,27 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
             h->test_wait = 0;
         }
         if (!teacher) g1.test_wait = test_wait;
-        if (hooks && (e = hooks->before_step(t, s)) != cudaSuccess) break;
+        const OpMaps opc{&mx[xa], &mwc, &mxl[xa], &mwcl}, opg{&mx[xa], &mwg, &mxl[xa], &mwgl},
+            oph{&mx[xn], &mwh, &mxl[xn], &mwhl};
         if (!teacher && !hier) {
             wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
-            if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
-            else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
-            else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+            if (f32) {
+                if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2, 3>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2, 3>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else e = launch_gemm<128, 1, 3, EpiCtrl, 2, 3>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+            } else {
+                if (A > 256) e = launch_gemm<256, 2, 2, EpiCtrl, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else if (A > 128) e = launch_gemm<256, 1, 3, EpiCtrl, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else e = launch_gemm<128, 1, 3, EpiCtrl, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+            }
             ++launches;
             if (e != cudaSuccess) break;
-        } else if (hier) {  // the logits, then the two-stage choice (Sec. 3.1.3)
+        } else if (hier) {  // the logits, then the two-stage choice (Sec. 3.1.3); bf16 models only
             {
                 wm_ktime kt(h, WM_KERNEL_TC_CTRL, s);
-                if (A > 256) e = launch_gemm<256, 2, 2, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
-                else if (A > 128) e = launch_gemm<256, 1, 3, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
-                else e = launch_gemm<128, 1, 3, EpiLogits, 2>(mx[t & 1], mwc, mc, mc, g1, io, T.sms, s, pdl);
+                if (A > 256) e = launch_gemm<256, 2, 2, EpiLogits, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else if (A > 128) e = launch_gemm<256, 1, 3, EpiLogits, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
+                else e = launch_gemm<128, 1, 3, EpiLogits, 2>(opc, mc, mc, mc, g1, io, T.sms, s, pdl);
             }
             ++launches;
             if (e != cudaSuccess) break;
@@ -1609,30 +2253,49 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
             ++launches;
         }
         GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
+        g2.n_rows = io.n_rows;
         if (teacher) g2.test_wait = test_wait;
         {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
-            if (hier) e = launch_gemm<256, 1, 2, EpiGates2, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
-            else e = launch_gemm<256, 1, 2, EpiGates, 2>(mx[t & 1], mwg, mc, mxs[(t + 1) & 1], g2, io, T.sms, s, pdl);
+            if (f32) e = launch_gemm<256, 1, 2, EpiGates32, 2, 3>(opg, mC, mxs[xn], mxsl[xn], g2, io, T.sms, s, pdl);
+            else if (hier) e = launch_gemm<256, 1, 2, EpiGates2, 2>(opg, mC, mxs[xn], mxs[xn], g2, io, T.sms, s, pdl);
+            else e = launch_gemm<256, 1, 2, EpiGates, 2>(opg, mC, mxs[xn], mxs[xn], g2, io, T.sms, s, pdl);
         }
         ++launches;
         if (e != cudaSuccess) break;
-        const GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
+        GemmGrid g3{m_tiles, T.n_head_tiles, (H + BK - 1) / BK, Z, h->status};
+        g3.n_rows = io.n_rows;
         {
             wm_ktime kt(h, WM_KERNEL_TC_HEADS, s);
-            e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(mx[(t + 1) & 1], mwh, mc, mc, g3, io, T.sms, s, pdl);
+            if (f32) e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2, 3>(oph, mc, mc, mc, g3, io, T.sms, s, pdl);
+            else e = launch_gemm<HEAD_TILE, 1, 3, EpiHeads, 2>(oph, mc, mc, mc, g3, io, T.sms, s, pdl);
         }
         ++launches;
         if (e == cudaSuccess && hooks) e = hooks->after_step(t, s);
+        if (e == cudaSuccess && early) e = cudaEventRecord(h->step_events[t % LOOKAHEAD], s);
     }
     if (e != cudaSuccess) return e;
-    {
+    if (compact) {
+        if (!q.fill) {
+            wm_ktime kt(h, WM_KERNEL_AUX, s);
+            k_tc_fill_frozen<<<16 * T.sms, 256, 0, s>>>(q);
+            ++launches;
+        }
+        if (ra->h_final || ra->c_final) {
+            wm_ktime kt(h, WM_KERNEL_AUX, s);
+            const int tl = t_end - 1;  // the last issued step
+            k_tc_finish_compact<<<init_grid, 256, 0, s>>>(B, H, Tn, w.dstep, w.rows[tl & 1], w.cnt + (tl & 3),
+                                                          w.h32, cbuf[Tn & 1], w.hfin, w.cfin, ra->h_final,
+                                                          ra->c_final);
+            ++launches;
+        }
+    } else {
         wm_ktime kt(h, WM_KERNEL_AUX, s);
         k_tc_finish<<<init_grid, 256, 0, s>>>(B, H, w.h32, w.c, teacher ? nullptr : ra->h_final,
                                               teacher ? nullptr : ra->c_final, w.nll_part, 4 * T.n_head_tiles,
                                               teacher ? na->nll : nullptr);
+        ++launches;
     }
-    ++launches;
     h->last_launches = launches;
     return cudaGetLastError();
 }

@@ -82,12 +82,14 @@ def test_teacher_forced_ragged_lengths_and_no_action(wm, orc):
 
 
 # ------------------------------------------------------------------ free-running rollouts
-@pytest.mark.parametrize("path", PATHS_SMALL)
+@pytest.mark.parametrize("path", PATHS_SMALL + ["tensor"])
 def test_rollout_tiny_full(wm, orc, path):
     cfg, w, z0, mask, B, T = synth.rollout_inputs("tiny_fp32")
     m = wm.WorldModel(dict(cfg, path=path), w)
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
     torch.cuda.synchronize()
+    if path == "tensor":
+        assert m.last_path == "tensor"
     r = check_rollout(g, cfg, w, z0, mask, orc=orc)
     assert r["compared"] == B * T
     # the fp32 path also follows the oracle's own free-running trajectory
@@ -278,11 +280,12 @@ def test_sharding_is_bit_exact(wm, name):
         assert torch.equal(torch.cat([lo[k], hi[k]], 1), full[k]), k
 
 
-@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
-def test_resume_is_bit_exact(wm, name):
+@pytest.mark.parametrize("name,path", [("tiny_fp32", "auto"), ("small_bf16", "auto"),
+                                       ("small_bf16", "tensor")])  # tensor: compacted live episodes
+def test_resume_is_bit_exact(wm, name, path):
     cfg, w, z0, mask, B, T = synth.rollout_inputs(name, T=10)
     cfg["done_terminates"] = 1
-    m = wm.WorldModel(cfg, w)
+    m = wm.WorldModel(dict(cfg, path=path), w)
     zc, mc = _cuda(z0), _cuda(mask)
     full = m.rollout(zc, T, mask=mc)
     a = m.rollout(zc, 4, mask=mc[:4].contiguous())
@@ -294,11 +297,13 @@ def test_resume_is_bit_exact(wm, name):
 
 
 @pytest.mark.parametrize("kind", ["pinned", "pageable"])
-@pytest.mark.parametrize("path,B,T,seq", [("auto", None, 6, False),   # fused: copied whole around the call
-                                          ("tensor", 700, 6, True),   # per-step staging, every output kind
-                                          ("tensor", 700, 1, False)])  # one step: copied whole
-def test_host_buffers_match_device_buffers(wm, kind, path, B, T, seq):
+@pytest.mark.parametrize("path,B,T,seq,done", [("auto", None, 6, False, 0),  # fused: copied whole around the call
+                                               ("tensor", 700, 6, True, 0),   # per-step staging, every output kind
+                                               ("tensor", 700, 6, True, 1),   # ... with compacted live episodes
+                                               ("tensor", 700, 1, False, 0)])  # one step: copied whole
+def test_host_buffers_match_device_buffers(wm, kind, path, B, T, seq, done):
     cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=B, T=T)
+    cfg["done_terminates"] = done
     m = wm.WorldModel(dict(cfg, path=path), w)
     dev = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=seq)
     zh, mh = torch.from_numpy(z0), torch.from_numpy(mask)
@@ -379,7 +384,12 @@ def test_fused_matches_stepwise_closely(wm):
                                         ("small_bf16", dict(a_dim=192, ctrl_sample=1, ctrl_tau=0.8)),
                                         ("small_bf16", dict(a_dim=64)),
                                         # an odd number of k-steps in the head GEMM (H / 64 = 5)
-                                        ("small_bf16", dict(h_dim=320))])
+                                        ("small_bf16", dict(h_dim=320)),
+                                        # fp32: three bf16 passes over K (hi/lo split operands)
+                                        ("tiny_fp32", dict()),
+                                        ("tiny_fp32", dict(ctrl_sample=1, ctrl_tau=0.8, done_terminates=1,
+                                                           noop_terminates=1, mdn_tau=0.7)),
+                                        ("mid_bf16", dict(precision="fp32", k_mix=5))])
 def test_tensor_against_oracle(wm, orc, name, flags):
     """Two row tiles (the second partly filled), resumed state, offsets, flags."""
     cfg = dict(synth.model_config(name), **flags)
@@ -403,7 +413,8 @@ def test_tensor_against_oracle(wm, orc, name, flags):
 
 
 @pytest.mark.parametrize("name,prec,N,T", [("mid_bf16", None, 300, 9), ("nll", "bf16", 512, 128),
-                                           ("large_bf16", None, 130, 5)])
+                                           ("large_bf16", None, 130, 5), ("nll", "fp32", 512, 128),
+                                           ("tiny_fp32", None, 300, 20)])
 def test_tensor_teacher_forced(wm, orc, name, prec, N, T):
     cfg = synth.model_config(name)
     if prec:
@@ -623,7 +634,8 @@ def _grad_err(g, o):
 @pytest.mark.parametrize("name,prec,path,N,T", [("tiny_fp32", "fp32", "stepwise", 37, 9),
                                                 ("small_bf16", "bf16", "auto", 64, 12),
                                                 ("nll", "bf16", "tensor", 300, 10),
-                                                ("nll", "fp32", "stepwise", 64, 16)])
+                                                ("nll", "fp32", "stepwise", 64, 16),
+                                                ("nll", "fp32", "tensor", 300, 10)])
 def test_training_step_gradient_against_oracle(wm, orc, name, prec, path, N, T):
     """wm_mdn_nll_backward against the oracle's fp64 BPTT, ragged lengths and no-action rows."""
     cfg = dict(synth.model_config(name), precision=prec)
@@ -675,3 +687,29 @@ def test_training_step_full_size(wm, orc):
     print("full-T subset vs oracle", err)
     for k, e in err.items():
         assert e <= GRAD_TOL["bf16"], (k, e)
+
+
+def test_tensor_compaction_when_every_episode_ends_early(wm, orc):
+    """Compacted rollouts whose episodes all end within the first steps: the host may stop
+    issuing steps once the device reports no live episode (when it does depends on timing),
+    and every later step's outputs are the frozen ones.  Two calls in a row: the second must
+    not see the first's report."""
+    cfg = dict(synth.model_config("mid_bf16"), done_terminates=1)
+    w = synth.weights(cfg, seed=12)
+    w["b_done"] = np.float32(3.0)  # done logits well above 0: almost every episode ends at once
+    B, T = 300, 40
+    z0 = synth.z0(B, cfg["z_dim"], seed=12)
+    mask = synth.mask(T, B, cfg["a_dim"], 0.2, seed=12)
+    done0 = (np.arange(B) % 7 == 3).astype(np.uint8)
+    m = wm.WorldModel(dict(cfg, path="tensor"), w)
+    outs = []
+    for _ in range(2):
+        g = m.rollout(_cuda(z0), T, mask=_cuda(mask), done0=_cuda(done0), want_seq=True)
+        m.sync()
+        assert m.last_path == "tensor"
+        outs.append(g)
+    r = check_rollout(outs[0], cfg, w, z0, mask, done0=done0, orc=orc)
+    assert r["frozen_steps"] > 0.9 * B * T, r
+    for k in ("z", "actions", "rewards", "done", "h_seq", "c_seq", "mdn_seq", "comp_seq", "h_final",
+              "c_final"):
+        assert torch.equal(outs[0][k], outs[1][k]), k
