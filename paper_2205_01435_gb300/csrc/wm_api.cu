@@ -258,14 +258,15 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
 }
 
 // AUTO: the fused single-launch family for batches that fit one wave of clusters,
-// the tensor-core family for large bf16 batches, the stepwise family otherwise.
-// fused_ok / tc_ok: whether this call's options allow those families.
+// the tensor-core family for large bf16 batches and for fp32 models of any batch (its
+// three-pass split beat the fp32 SIMT family 2x even at B = 16), the stepwise family
+// otherwise.  fused_ok / tc_ok: whether this call's options allow those families.
 int pick_path(const wm_handle *h, int B, bool fused_ok = true, bool tc_ok = true) {
     const int p = h->cfg.path;
     if (p != WM_PATH_AUTO) return p;
     const bool fu = fused_ok && wm_fused_supported(h, B), tc = tc_ok && wm_tc_supported(h);
     if (fu && B <= 2048) return WM_PATH_FUSED;
-    if (tc && B >= 256) return WM_PATH_TENSOR;
+    if (tc && (B >= 256 || h->cfg.precision == WM_FP32)) return WM_PATH_TENSOR;
     if (fu) return WM_PATH_FUSED;
     return WM_PATH_STEPWISE;
 }

@@ -1350,13 +1350,18 @@ __global__ void k_tc_frames(int N, int T, int Z, int KX, const float *__restrict
 }
 
 // nll[n] = sum over the head tiles' partials and the steps of sequence n (uncounted steps
-// hold 0), in a fixed order
+// hold 0).  A warp per sequence: lane l adds the partials l, l + 32, ... of the sequence's
+// parts x T values in fp64, then a shuffle tree of fixed shape combines the lanes, so the
+// order, and the result, is the same every time.
 __global__ void k_tc_nll_reduce(int N, int T, int parts, const float *__restrict__ part, float *__restrict__ nll) {
-    for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < N; n += gridDim.x * blockDim.x) {
+    const int lane = threadIdx.x & 31, nw = (int)((gridDim.x * blockDim.x) >> 5);
+    const int total = parts * T;
+    for (int n = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); n < N; n += nw) {
         double s = 0.0;
-        for (int j = 0; j < parts; ++j)
-            for (int t = 0; t < T; ++t) s += (double)part[((size_t)j * T + t) * N + n];
-        nll[n] = (float)s;
+        for (int i = lane; i < total; i += 32) s += (double)part[(size_t)i * N + n];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
+        if (lane == 0) nll[n] = (float)s;
     }
 }
 
@@ -1438,72 +1443,81 @@ __device__ void fill_elem(const CompactIO &q, int e, int k, const float *hs, con
     if (q.loc_actions) q.loc_actions[tb] = -1;
 }
 
-constexpr int CROWS = 16;         // rows of step t-1 per block
-constexpr int CTHREADS = 128;
+constexpr int CROWS = 8;          // rows of step t-1 per block: a warp per row
+constexpr int CTHREADS = 32 * CROWS;
 
-// Every phase is flattened over the block's (or the grid's) threads, so that many
-// independent 16-byte copies are in flight: a warp walking rows one by one is bound by
-// memory latency, not bandwidth.
+// A row's 16-byte chunks [0, n) from src to dst, by one warp: each lane loads up to 8 chunks
+// before it stores any, so that the loads are in flight together (a load-then-store per
+// chunk waits out the memory latency once per chunk).
+__device__ __forceinline__ void warp_copy16(const uint4 *__restrict__ src, uint4 *__restrict__ dst, int n, int lane) {
+    for (int base = 0; base < n; base += 256) {
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int k = base + 32 * u + lane;
+            if (k < n) v[u] = src[k];
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int k = base + 32 * u + lane;
+            if (k < n) dst[k] = v[u];
+        }
+    }
+}
+
+// Phase A (rows of step t-1, a warp per row): survivors' operand row (and its lo part) and c
+// to their new row; ended episodes' h and c recorded, and, when outputs are staged step by
+// step, their step-t outputs written.  Phase B (the whole grid): when staged, the step-t
+// outputs of the episodes frozen before.
 __global__ void __launch_bounds__(CTHREADS) k_tc_compact(CompactIO q) {
     asm volatile("griddepcontrol.wait;" ::: "memory");  // the previous step's outputs are complete
-    __shared__ int s_pos[CROWS], s_e[CROWS], s_base;
-    const int tid = (int)threadIdx.x;
+    __shared__ int s_pos[CROWS], s_e[CROWS];
+    const int tid = (int)threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n_in = q.n_in ? *(volatile const int *)q.n_in : q.B;
     const int r0 = (int)blockIdx.x * CROWS;
     if (r0 < n_in) {  // block-uniform
         const int nrow = min(CROWS, n_in - r0);
-        if (tid < 32) {  // one warp claims the block's output rows
-            const int r = r0 + tid;
-            const bool in = tid < nrow;
+        if (warp == 0) {  // the block claims its output rows with one atomic
+            const int r = r0 + lane;
+            const bool in = lane < nrow;
             const bool keep = in && !(q.dies && q.dies[r]);
             const uint32_t bal = __ballot_sync(0xffffffffu, keep);
             int base = 0;
-            if (tid == 0 && bal) base = atomicAdd(q.n_out, __popc(bal));
+            if (lane == 0 && bal) base = atomicAdd(q.n_out, __popc(bal));
             base = __shfl_sync(0xffffffffu, base, 0);
             if (in) {
                 const int e = q.rows_in ? q.rows_in[r] : r;
-                s_e[tid] = e;
-                s_pos[tid] = keep ? base + __popc(bal & ((1u << tid) - 1u)) : -1;
-                if (keep) q.rows_out[s_pos[tid]] = e;
+                const int pos = keep ? base + __popc(bal & ((1u << lane) - 1u)) : -1;
+                s_e[lane] = e;
+                s_pos[lane] = pos;
+                if (keep) q.rows_out[pos] = e;
                 else q.dstep[e] = q.t;
             }
         }
         __syncthreads();
-        // survivors: the operand row and c to their new row; ended episodes: h, c recorded
         const int XC = q.KX / 8, CC = q.H / 4;  // 16-byte chunks per row
-        const int XL = q.x_in_lo ? XC : 0;       // the operand's lo parts (fp32 path)
-        const int per = max(XC + XL + CC, 2 * CC);
-        const uint4 *__restrict__ xi = reinterpret_cast<const uint4 *>(q.x_in);
-        uint4 *__restrict__ xo = reinterpret_cast<uint4 *>(q.x_out);
-        const uint4 *__restrict__ ci = reinterpret_cast<const uint4 *>(q.c_in);
-        const uint4 *__restrict__ hi = reinterpret_cast<const uint4 *>(q.h32);
-        uint4 *__restrict__ co = reinterpret_cast<uint4 *>(q.c_out);
-        uint4 *__restrict__ hf = reinterpret_cast<uint4 *>(q.hfin);
-        uint4 *__restrict__ cf = reinterpret_cast<uint4 *>(q.cfin);
-#pragma unroll 4
-        for (int i = tid; i < nrow * per; i += CTHREADS) {
-            const int j = i / per, k = i - j * per;
-            const size_t rr = (size_t)(r0 + j);
-            const int pos = s_pos[j];
+        if (warp < nrow) {
+            const size_t rr = (size_t)(r0 + warp);
+            const int pos = s_pos[warp];
+            const uint4 *ci = reinterpret_cast<const uint4 *>(q.c_in) + rr * CC;
             if (pos >= 0) {
-                if (k < XC) xo[(size_t)pos * XC + k] = xi[rr * XC + k];
-                else if (k < XC + XL)
-                    reinterpret_cast<uint4 *>(q.x_out_lo)[(size_t)pos * XC + k - XC] =
-                        reinterpret_cast<const uint4 *>(q.x_in_lo)[rr * XC + k - XC];
-                else if (k < XC + XL + CC) co[(size_t)pos * CC + k - XC - XL] = ci[rr * CC + k - XC - XL];
+                warp_copy16(reinterpret_cast<const uint4 *>(q.x_in) + rr * XC,
+                            reinterpret_cast<uint4 *>(q.x_out) + (size_t)pos * XC, XC, lane);
+                if (q.x_in_lo)
+                    warp_copy16(reinterpret_cast<const uint4 *>(q.x_in_lo) + rr * XC,
+                                reinterpret_cast<uint4 *>(q.x_out_lo) + (size_t)pos * XC, XC, lane);
+                warp_copy16(ci, reinterpret_cast<uint4 *>(q.c_out) + (size_t)pos * CC, CC, lane);
             } else {
-                const size_t e = (size_t)s_e[j];
-                if (k < CC) hf[e * CC + k] = hi[rr * CC + k];
-                else if (k < 2 * CC) cf[e * CC + k - CC] = ci[rr * CC + k - CC];
+                const size_t e = (size_t)s_e[warp];
+                warp_copy16(reinterpret_cast<const uint4 *>(q.h32) + rr * CC, reinterpret_cast<uint4 *>(q.hfin) + e * CC,
+                            CC, lane);
+                warp_copy16(ci, reinterpret_cast<uint4 *>(q.cfin) + e * CC, CC, lane);
+                if (q.fill) {  // its step-t outputs, from its row
+                    const int fe = fill_elems(q);
+                    for (int k = lane; k < fe; k += 32)
+                        fill_elem(q, (int)e, k, q.h32 + rr * q.H, q.c_in + rr * q.H);
+                }
             }
-        }
-        // the ended episodes' step-t outputs, from their rows
-        const int fe = q.fill ? fill_elems(q) : 0;
-        for (int i = tid; i < nrow * fe; i += CTHREADS) {
-            const int j = i / fe, k = i - j * fe;
-            if (s_pos[j] >= 0) continue;
-            const size_t rr = (size_t)(r0 + j);
-            fill_elem(q, s_e[j], k, q.h32 + rr * q.H, q.c_in + rr * q.H);
         }
     }
     // episodes frozen before this step's compaction stay frozen: their step-t outputs, over
@@ -2105,7 +2119,7 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         }
         {
             wm_ktime kt(h, WM_KERNEL_AUX, s);
-            k_tc_nll_reduce<<<(B + 255) / 256, 256, 0, s>>>(B, Tn, parts, w.part, na->nll);
+            k_tc_nll_reduce<<<(B + 7) / 8, 256, 0, s>>>(B, Tn, parts, w.part, na->nll);
         }
         ++launches;
         h->last_launches = launches;
