@@ -180,9 +180,9 @@ template <class S>
 __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     constexpr int CL = S::CL, UG = S::UG, ZD = S::ZD, KM = S::KM;
     extern __shared__ __align__(1024) unsigned char smem[];
-    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in, 5 W_a/W2 buffer,
-    // 6 never completed (the injected wait)
-    __shared__ __align__(8) uint64_t mbar[7];
+    // mbarriers: 0 MMA1 done, 1 MMA2 done, 2 partials in, 3 h' in, 4 z' in, 5 W_a in the
+    // buffer, 6 never completed (the injected wait), 7 W2 in the buffer (compute threads)
+    __shared__ __align__(8) uint64_t mbar[8];
     __shared__ uint32_t tmem_base;
     __shared__ int s_abort;
     __shared__ float s_done_logit[TILE];
@@ -212,7 +212,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     const uint32_t WA_BYTES = (uint32_t)A * S::WA_STRIDE, W2_BYTES = (uint32_t)S::N2 * H * 2;
     const uint32_t mb = tc::smem_u32(&mbar[0]);
     const uint32_t MB_MMA1 = mb, MB_MMA2 = mb + 8, MB_PART = mb + 16, MB_H = mb + 24, MB_Z = mb + 32,
-                   MB_W = mb + 40, MB_NEVER = mb + 48;
+                   MB_W = mb + 40, MB_NEVER = mb + 48, MB_W2 = mb + 56;
     const unsigned char *img = p.img + rank * p.img_stride;
     const uint32_t buf_u32 = tc::smem_u32(sBuf);
 
@@ -248,6 +248,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
     }
     if (tid == 0) {
         for (int i = 0; i < 7; ++i) tc::mbar_init(mb + 8 * i, 1);
+        tc::mbar_init(MB_W2, NT);  // every compute thread arrives once its part of W2 is stored
         tc::fence_mbar_init();
         // arm the exchange barriers for step 0; start the first W_a load
         tc::mbar_arrive_expect_tx(MB_PART, (CL - 1) * PART_BYTES);
@@ -359,14 +360,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         if (grp == 0 && !mma_warp) {
             uint64_t rec = 0xFFFFFFFF00000000ull;  // index -1: nothing valid here
             if (!p.teacher) {
-                const uint32_t *r = rc;
-                // local masked argmax over this rank's actions (lowest index on ties)
+                // local masked argmax over this rank's actions (lowest index on ties); the
+                // loop runs over the padded column count so that every register index is
+                // static (a runtime bound put rc[] in local memory)
                 float bv = -INFINITY;
                 int bi = -1;
-                for (int j = 0; j < p.AC; ++j) {
+#pragma unroll
+                for (int j = 0; j < S::NA; ++j) {
                     const int a = a0 + j;
-                    const bool ok = (mword >> (a & 31)) & 1u;
-                    const float v = __uint_as_float(r[j]) + sB1[S::NG + j];
+                    const bool ok = j < p.AC && ((mword >> (a & 31)) & 1u);
+                    const float v = __uint_as_float(rc[j]) + sB1[S::NG + j];
                     if (ok && (bi < 0 || v > bv)) { bv = v; bi = a; }
                 }
                 rec = ((uint64_t)(uint32_t)bi << 32) | __float_as_uint(bv);
@@ -405,7 +408,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         if (!p.teacher && rank == 0 && grp == 0 && live) p.actions[tb] = a;
 
         // ---------------- LSTM cell (a3, a4): UG units per thread -------------
-        wait_bar(MB_W, 0);  // W_a is in the buffer
+        wait_bar(MB_W, parity);  // W_a is in the buffer (one load per step)
         {
             const float *bb = sB1 + 4 * UG * grp;
             const uint4 *src = reinterpret_cast<const uint4 *>(sBuf + (size_t)(a >= 0 ? a : 0) * S::WA_STRIDE +
@@ -450,13 +453,28 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         }  // !mma_warp
         tc::fence_proxy_async_smem();
         __syncthreads();  // every W_a read and h' write of this CTA is done
-        if (issuer) {      // W2 replaces W_a in the buffer while h' travels
-            tc::mbar_arrive_expect_tx(MB_W, W2_BYTES);
-            tc::bulk_load_global(buf_u32, img + g.iw2, W2_BYTES, MB_W);
-        }
-        __syncwarp();
         const uint32_t hblk = x_u32 + tc::kmajor_offset(0, Z + rank * S::U, TILE);
         push_to_peers<CL>(hblk, H_BYTES, MB_H, rank, warp, lane, NT / 32);
+        // W2 replaces W_a in the buffer while h' travels.  The compute threads copy it (L2 ->
+        // registers -> shared memory): the TMA engine, which moves every exchange, is left to
+        // the h' slices (with W2 in its queue too, MMA2 waited for both).
+        if (!mma_warp) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(img + g.iw2);
+            uint4 *dst = reinterpret_cast<uint4 *>(sBuf);
+            constexpr int PER = (int)(S::N2 * 256 * 2 / 16 / NT);  // 16-byte chunks per thread (H = 256)
+            static_assert(PER >= 1 && PER <= 8, "W2 chunks per thread");
+            if ((int)(W2_BYTES / 16) == PER * NT) {
+                uint4 v[PER];
+#pragma unroll
+                for (int i = 0; i < PER; ++i) v[i] = __ldg(src + tid + i * NT);
+#pragma unroll
+                for (int i = 0; i < PER; ++i) dst[tid + i * NT] = v[i];
+            } else {
+                for (int i = tid; i < (int)(W2_BYTES / 16); i += NT) dst[i] = __ldg(src + i);
+            }
+            tc::fence_proxy_async_smem();  // generic stores -> the MMA's reads
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(MB_W2) : "memory");
+        }
         if (live) {
             const size_t o = tb * H + rank * S::U + u0;
             if (p.h_seq)
@@ -474,7 +492,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
         // ---------------- MMA2: heads (a5); then the h part of the next MMA1 ---
         if (issuer) {
             wait_one(MB_H, parity);  // h' of every rank is in X
-            wait_one(MB_W, 1);       // W2 is in the buffer
+            wait_one(MB_W2, parity);  // W2 is in the buffer
             if (!s_abort) {
                 tc::fence_after_sync();
                 uint64_t da = dX0 + ((uint64_t)Z * 256u >> 4), db = dW20;  // X_h: Z/8 k-blocks in
@@ -535,8 +553,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
             } else if (frozen) {
                 zn = zs;
             } else if (!(p.mdn_tau > 0.f)) {
-                for (int k = 1; k < KM; ++k) if (lg[k] > lg[kc]) kc = k;
-                zn = mu[kc];
+                float best = lg[0];
+                zn = mu[0];
+#pragma unroll
+                for (int k = 1; k < KM; ++k)
+                    if (lg[k] > best) { best = lg[k]; kc = k; zn = mu[k]; }
             } else {
                 const float tau = p.mdn_tau;
                 float m = -INFINITY;
@@ -545,14 +566,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_fused(FusedParams p) {
                 float pk[KM], s = 0.f;
                 for (int k = 0; k < KM; ++k) { pk[k] = __expf(lg[k] * itau - m); s += pk[k]; }
                 const float u = u_dim, is = __fdividef(1.f, s);
-                kc = KM - 1;
+                // first k with u < C_k (else K-1), and its mu and log sigma by selects: every
+                // register index static (mu[kc] with a runtime kc put hv[] in local memory)
                 float cum = 0.f;
+                uint32_t hit = 0u;
+#pragma unroll
                 for (int k = 0; k < KM - 1; ++k) {
                     cum += pk[k] * is;
-                    if (u < cum) { kc = k; break; }
+                    hit |= (u < cum ? 1u : 0u) << k;
+                }
+                kc = hit ? __ffs(hit) - 1 : KM - 1;
+                float muc = mu[0], lsc = ls[0];
+#pragma unroll
+                for (int k = 1; k < KM; ++k) {
+                    muc = k == kc ? mu[k] : muc;
+                    lsc = k == kc ? ls[k] : lsc;
                 }
                 const float scale = p.sigma_sqrt_tau ? sqrtf(tau) : 1.f;
-                zn = mu[kc] + __expf(ls[kc]) * scale * eps_dim;
+                zn = muc + __expf(lsc) * scale * eps_dim;
             }
         }
         // ---------------- z' exchange, then the z part of the next MMA1 ------

@@ -1073,13 +1073,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     constexpr int NACC = TILE_N <= 256 ? 2 : 1;
     constexpr uint32_t ACC_COLS = 256;
     static_assert(BN % 16 == 0 && BNH % 8 == 0 && BN <= 256 && TILE_N <= 512, "tile shape");
-    // Compacted live episodes: a pair with no tile this step leaves before its set-up (both
-    // CTAs read the same row count, written by the previous kernel).
-    if (g.n_rows) {
-        asm volatile("griddepcontrol.wait;" ::: "memory");
-        const int mt = (*(volatile const int *)g.n_rows + 2 * BM - 1) / (2 * BM);
-        if ((int)(blockIdx.x >> 1) >= mt * g.n_tiles) return;
-    }
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_accf[2], bar_acce[2], bar_stage[4],
