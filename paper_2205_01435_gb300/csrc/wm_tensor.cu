@@ -570,29 +570,36 @@ __global__ void __launch_bounds__(256) k_tc_select(StepIO p) {
 // MODE 2: the fp32 path: the action row is gathered as its bf16 hi and lo parts (the two-row
 // machinery with the same action), the nonlinearities are the accurate ones, and h' is
 // stored as bf16 hi and lo parts.
-template <int MODE>
+// UNITS: hidden units per tile (64: a 256-column tile; 32: a 128-column tile, for calls with
+// few row tiles, where twice the tiles keep twice the CTA pairs busy and each tile's
+// epilogue is half as long).  Each thread of a quadrant's 4 column groups takes UT units.
+template <int MODE, int UNITS = 64>
 struct EpiGatesT {
     static constexpr bool TWO = MODE != 0, F32 = MODE == 2;
-    static constexpr uint32_t C_SLAB = 32 * 64 * 4;  // two boxes of 32 fp32 x 32 rows
-    static constexpr uint32_t X_SLAB = 32 * 64 * 2;  // one box of 64 bf16 x 32 rows
+    static constexpr int UT = UNITS / 4, WW = UT / 2;  // units per thread, W_a words per gate
+    static_assert(UNITS == 64 || UNITS == 32, "gate tile of 64 or 32 units");
+    static constexpr uint32_t C_SLAB = 32 * UNITS * 4;  // UNITS / 32 boxes of 32 fp32 x 32 rows
+    static constexpr uint32_t X_SLAB = 32 * UNITS * 2;  // one box of UNITS bf16 x 32 rows
     static constexpr uint32_t QUAD_STAGE = C_SLAB + (F32 ? 2 : 1) * X_SLAB;  // c (in place) | h' out (| h' lo)
     static constexpr bool TMA_STAGE = true;
     static constexpr uint32_t RED_BYTES = 0;
 
     // byte offset of (row r, 16-byte chunk j) in a 128-byte-swizzled box
     static __device__ __forceinline__ uint32_t sw(int r, int j) { return r * 128 + ((j ^ (r & 7)) << 4); }
+    // the h' slab: a 128-byte-swizzled box of 64 units, or a plain 64-byte-row box of 32
+    static __device__ __forceinline__ uint32_t xsw(int r, int j) { return UNITS == 64 ? sw(r, j) : r * 64 + (j << 4); }
 
     // leader of a quadrant: TMA load of the c rows of 128-row block m, unit tile n
     static __device__ void prefetch(const StepIO &, int m, int n, EpiCtx &x) {
         x.note_prefetch();
         tc::mbar_arrive_expect_tx(x.stage_bar, C_SLAB);
-        for (int bx = 0; bx < 2; ++bx)
-            tma_load_2d(x.stage_u + bx * 4096, x.tm_c, 64 * n + 32 * bx, m * BM + 32 * x.quad, x.stage_bar);
+        for (int bx = 0; bx < UNITS / 32; ++bx)
+            tma_load_2d(x.stage_u + bx * 4096, x.tm_c, UNITS * n + 32 * bx, m * BM + 32 * x.quad, x.stage_bar);
     }
 
     struct Pre {
-        uint32_t wi[8], wg[8];    // the W_a row segments of gates i and g (16 units, bf16)
-        uint32_t wi2[8], wg2[8];  // TWO: the second action row's (F32: the lo parts)
+        uint32_t wi[WW], wg[WW];    // the W_a row segments of gates i and g (UT units, bf16)
+        uint32_t wi2[WW], wg2[WW];  // TWO: the second action row's (F32: the lo parts)
         int a, a2;                // the action rows (-1: none)
         bool fz;                  // frozen episode
         int e;                    // the row's episode
@@ -601,17 +608,22 @@ struct EpiGatesT {
     // one gate's W_a segment for the thread's 16 units: a single 32-byte sector, read with
     // one 256-bit load (half the L1 wavefronts of two 16-byte loads: each lane reads
     // another row, so every load instruction touches 32 lines)
-    static __device__ __forceinline__ void ld_wa(const StepIO &p, int a, int n, int q, int gate, uint32_t (&w)[8],
+    static __device__ __forceinline__ void ld_wa(const StepIO &p, int a, int n, int q, int gate, uint32_t (&w)[WW],
                                                  bool lo = false) {
         if (a < 0) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) w[i] = 0u;
+            for (int i = 0; i < WW; ++i) w[i] = 0u;
             return;
         }
-        const __nv_bfloat16 *src = (lo ? p.wa_lo : p.wa) + (size_t)a * 4 * p.H + 256 * n + 64 * gate + 16 * q;
-        asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-                     : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
-                     : "l"(src));
+        const __nv_bfloat16 *src =
+            (lo ? p.wa_lo : p.wa) + (size_t)a * 4 * p.H + 4 * UNITS * n + UNITS * gate + UT * q;
+        if constexpr (WW == 8)
+            asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                         : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+                         : "l"(src));
+        else
+            asm volatile("ld.global.nc.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]) : "l"(src));
     }
     // before the accumulator wait: the row's action and the W_a segments of gates i and g
     // (L2 gathers), so that their latency overlaps the mainloop
@@ -648,21 +660,21 @@ struct EpiGatesT {
     // pre-activations of one gate for the thread's 16 units: accumulator + bias + W_a[a]
     // (+ W_a[a2] when TWO)
     static __device__ __forceinline__ void gate_pre(uint32_t tacc, const float *bg, int gate, int ut,
-                                                    const uint32_t (&w)[8], const uint32_t (&w2)[8],
-                                                    float (&g)[16]) {
+                                                    const uint32_t (&w)[WW], const uint32_t (&w2)[WW],
+                                                    float (&g)[UT]) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {  // 8 columns per TMEM load: fewer registers held
+        for (int h = 0; h < UT / 8; ++h) {  // 8 columns per TMEM load: fewer registers held
             uint32_t r[8];
-            TC_LD8(tacc + 64 * gate + ut + 8 * h, r);
+            TC_LD8(tacc + UNITS * gate + ut + 8 * h, r);
             tc::tmem_ld_wait();
             // the bias is read after the wait (an L1 hit), so that it is not held across it
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
-                const float4 t = *reinterpret_cast<const float4 *>(bg + 64 * gate + 8 * h + 4 * i);
+                const float4 t = *reinterpret_cast<const float4 *>(bg + UNITS * gate + 8 * h + 4 * i);
                 const float bv[4] = {t.x, t.y, t.z, t.w};
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
-                    const int k = 8 * h + 4 * i + 2 * e;  // unit (column) index in 0..15
+                    const int k = 8 * h + 4 * i + 2 * e;  // unit (column) index in 0..UT-1
                     const __nv_bfloat162 v2 = *reinterpret_cast<const __nv_bfloat162 *>(&w[k / 2]);
                     g[k] = __uint_as_float(r[4 * i + 2 * e]) + bv[2 * e] + __low2float(v2);
                     g[k + 1] = __uint_as_float(r[4 * i + 2 * e + 1]) + bv[2 * e + 1] + __high2float(v2);
@@ -683,70 +695,70 @@ struct EpiGatesT {
         const int bb = valid ? b : 0;  // rows past the batch compute on row 0; TMA stores clip them
         const int H = p.H, r = x.lane, q = x.cg;
         const bool fz = pr.fz;
-        const int ut = 16 * q, u0 = 64 * n + ut;  // the thread's first unit: in the tile, in H
+        const int ut = UT * q, u0 = UNITS * n + ut;  // the thread's first unit: in the tile, in H
         // gates f and o: loaded while i and g are computed
-        uint32_t wf[8], wo[8], wf2[8], wo2[8];
+        uint32_t wf[WW], wo[WW], wf2[WW], wo2[WW];
         ld_wa(p, pr.a, n, q, 1, wf);
         ld_wa(p, pr.a, n, q, 3, wo);
         if (TWO) {
             ld_wa(p, pr.a2, n, q, 1, wf2, F32);
             ld_wa(p, pr.a2, n, q, 3, wo2, F32);
         }
-        const float *bg = p.b_gate + 256 * n + 16 * q;
+        const float *bg = p.b_gate + 4 * UNITS * n + UT * q;
         const bool store_h32 = valid && !fz && (p.h32_mode == 2 || (p.h32_mode == 1 && p.t == p.T - 1));
         unsigned char *cs = x.stage, *xs = x.stage + C_SLAB;
-        // the thread's 16 c values: 4 chunks of the swizzled box that holds units ut..ut+15
+        // the thread's UT c values: UT / 4 chunks of the swizzled box that holds units ut..
         const uint32_t cbox = (ut >> 5) * 4096, cch = (ut & 31) >> 2;
         // Every lane forms all four gates: the TMEM loads are warp-collective, and the rows
         // of a warp may be frozen or not; a frozen row keeps its c and its carried h.
-        float cv[16], hv[16];
+        float cv[UT], hv[UT];
         {  // hv = sigma(i) * tanh(g), one gate's pre-activations live at a time
-            float g[16];
+            float g[UT];
             gate_pre(tacc, bg, 0, ut, pr.wi, pr.wi2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] = sig_(g[j]);
+            for (int j = 0; j < UT; ++j) hv[j] = sig_(g[j]);
             gate_pre(tacc, bg, 2, ut, pr.wg, pr.wg2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] *= tanh_(g[j]);
+            for (int j = 0; j < UT; ++j) hv[j] *= tanh_(g[j]);
         }
         x.wait_stage();  // the quadrant's c rows have landed
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < UT / 4; ++i) {
             const float4 t = *reinterpret_cast<const float4 *>(cs + cbox + sw(r, cch + i));
             cv[4 * i] = t.x; cv[4 * i + 1] = t.y; cv[4 * i + 2] = t.z; cv[4 * i + 3] = t.w;
         }
         {
-            float g[16];
+            float g[UT];
             gate_pre(tacc, bg, 1, ut, wf, wf2, g);
             if (!fz) {
 #pragma unroll
-                for (int j = 0; j < 16; ++j) cv[j] = sig_(g[j]) * cv[j] + hv[j];
+                for (int j = 0; j < UT; ++j) cv[j] = sig_(g[j]) * cv[j] + hv[j];
             }
             gate_pre(tacc, bg, 3, ut, wo, wo2, g);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) hv[j] = sig_(g[j]) * tanh_(cv[j]);
+            for (int j = 0; j < UT; ++j) hv[j] = sig_(g[j]) * tanh_(cv[j]);
         }
         if (fz) {  // frozen: h is the carried one
             const float4 *h4 = reinterpret_cast<const float4 *>(p.h32 + (size_t)bb * H + u0);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
+            for (int i = 0; i < UT / 4; ++i) {
                 const float4 t = h4[i];
                 hv[4 * i] = t.x; hv[4 * i + 1] = t.y; hv[4 * i + 2] = t.z; hv[4 * i + 3] = t.w;
             }
         }
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
+        for (int i = 0; i < UT / 4; ++i)
             *reinterpret_cast<float4 *>(cs + cbox + sw(r, cch + i)) =
                 make_float4(cv[4 * i], cv[4 * i + 1], cv[4 * i + 2], cv[4 * i + 3]);
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < UT / 8; ++i) {
             uint32_t pk[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 __nv_bfloat162 v = __floats2bfloat162_rn(hv[8 * i + 2 * j], hv[8 * i + 2 * j + 1]);
                 pk[j] = *reinterpret_cast<uint32_t *>(&v);
             }
-            *reinterpret_cast<uint4 *>(xs + sw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4 *>(xs + xsw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
             if (F32) {  // the lo parts, h' - bf16(h')
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
@@ -755,20 +767,20 @@ struct EpiGatesT {
                     __nv_bfloat162 v = __floats2bfloat162_rn(a0 - __low2float(hi2), a1 - __high2float(hi2));
                     pk[j] = *reinterpret_cast<uint32_t *>(&v);
                 }
-                *reinterpret_cast<uint4 *>(xs + X_SLAB + sw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                *reinterpret_cast<uint4 *>(xs + X_SLAB + xsw(r, (ut >> 3) + i)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
             }
         }
         if (store_h32) {
             float4 *h4 = reinterpret_cast<float4 *>(p.h32 + (size_t)b * H + u0);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) h4[i] = make_float4(hv[4 * i], hv[4 * i + 1], hv[4 * i + 2], hv[4 * i + 3]);
+            for (int i = 0; i < UT / 4; ++i) h4[i] = make_float4(hv[4 * i], hv[4 * i + 1], hv[4 * i + 2], hv[4 * i + 3]);
         }
         if (valid) {
             const size_t o = ((size_t)p.t * p.B + pr.e) * H + u0;
             if (p.h_seq)
-                for (int j = 0; j < 16; ++j) p.h_seq[o + j] = hv[j];
+                for (int j = 0; j < UT; ++j) p.h_seq[o + j] = hv[j];
             if (p.c_seq)
-                for (int j = 0; j < 16; ++j) p.c_seq[o + j] = cv[j];
+                for (int j = 0; j < UT; ++j) p.c_seq[o + j] = cv[j];
         }
         // the slab's generic-proxy reads and writes are ordered before the TMA (async-proxy)
         // stores and the refill by this fence and the barrier
@@ -777,10 +789,9 @@ struct EpiGatesT {
         if (x.leader) {
             const int y = m * BM + 32 * x.quad;
             if (y < p.B) {  // rows past B are clipped by the stores; a slab wholly past B is skipped
-                tma_store_2d(x.tm_c, 64 * n, y, x.stage_u);
-                tma_store_2d(x.tm_c, 64 * n + 32, y, x.stage_u + 4096);
-                tma_store_2d(x.tm_xs, p.Z + 64 * n, y, x.stage_u + C_SLAB);
-                if (F32) tma_store_2d(x.tm_xs2, p.Z + 64 * n, y, x.stage_u + C_SLAB + X_SLAB);
+                for (int bx = 0; bx < UNITS / 32; ++bx) tma_store_2d(x.tm_c, UNITS * n + 32 * bx, y, x.stage_u + 4096 * bx);
+                tma_store_2d(x.tm_xs, p.Z + UNITS * n, y, x.stage_u + C_SLAB);
+                if (F32) tma_store_2d(x.tm_xs2, p.Z + UNITS * n, y, x.stage_u + C_SLAB + X_SLAB);
                 bulk_commit();
                 bulk_wait_read();  // the slab may be refilled
             }
@@ -792,6 +803,7 @@ struct EpiGatesT {
 using EpiGates = EpiGatesT<0>;
 using EpiGates2 = EpiGatesT<1>;
 using EpiGates32 = EpiGatesT<2>;
+using EpiGatesN = EpiGatesT<0, 32>;  // 128-column tiles (few row tiles)
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
 // Before the accumulator wait, the quadrant's 128 threads make the tile's random draws:
@@ -1636,6 +1648,18 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, ui
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same over bf16 with a box of 32 columns (64 bytes) x 32 rows, unswizzled: the h' slab
+// of a 128-column gate tile.
+bool make_map_x32(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols) {
+    encode_fn_t enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {cols, rows}, strides[1] = {cols * 2};
+    cuuint32_t box[2] = {32, 32}, es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN, int NSUB, int STAGES, class Epi, int KPS = 1>
 size_t gemm_smem() {
     // per CTA: its A rows and half of each B slice per k-step
@@ -1890,6 +1914,23 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         if ((e = up(&T.wa_lo, wa_lo.data(), wa_lo.size() * 2)) != cudaSuccess) return e;
         if ((e = up(&T.wh_lo, wh_lo.data(), wh_lo.size() * 2)) != cudaSuccess) return e;
     }
+    if (!f32) {  // 128-column gate tiles: row n = 128 j + 32 gate + u <-> column gate H + 32 j + u
+        std::vector<__nv_bfloat16> wgn((size_t)4 * H * KX), wan((size_t)A * 4 * H);
+        std::vector<float> bgn(4 * H);
+        for (int n = 0; n < 4 * H; ++n) {
+            const int j = n / 128, gate = (n % 128) / 32, u = n % 32;
+            const size_t col = (size_t)gate * H + 32 * j + u;
+            for (int k = 0; k < KX; ++k) {
+                const size_t src = k < Z ? k : k + A;
+                wgn[(size_t)n * KX + k] = bf(w->W_lstm[src * 4 * H + col]);
+            }
+            bgn[n] = w->b_lstm[col];
+            for (int a = 0; a < A; ++a) wan[(size_t)a * 4 * H + n] = bf(w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
+        }
+        if ((e = up(&T.wg_n, wgn.data(), wgn.size() * 2)) != cudaSuccess) return e;
+        if ((e = up(&T.wa_n, wan.data(), wan.size() * 2)) != cudaSuccess) return e;
+        if ((e = up((void **)&T.bg_n, bgn.data(), bgn.size() * 4)) != cudaSuccess) return e;
+    }
     if ((e = up(&T.wc, wc.data(), wc.size() * 2)) != cudaSuccess) return e;
     if ((e = up(&T.wg, wg.data(), wg.size() * 2)) != cudaSuccess) return e;
     if ((e = up(&T.wa, wa.data(), wa.size() * 2)) != cudaSuccess) return e;
@@ -1942,6 +1983,7 @@ void wm_tc_free(wm_handle *h) {
     wm_tc_weights &T = h->tc;
     cudaFree(T.wc); cudaFree(T.wg); cudaFree(T.wa); cudaFree(T.wh);
     cudaFree(T.wc_lo); cudaFree(T.wg_lo); cudaFree(T.wa_lo); cudaFree(T.wh_lo);
+    cudaFree(T.wg_n); cudaFree(T.wa_n); cudaFree(T.bg_n);
     if (h->dead_host) cudaFreeHost(h->dead_host);
     h->dead_host = h->dead_dev = nullptr;
     for (cudaEvent_t ev : h->step_events) cudaEventDestroy(ev);
@@ -2049,6 +2091,15 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     // Programmatic dependent launch hides the ~4 us between consecutive launches (a fifth of
     // a call at B = 8192), but made the long launches of B = 65536 3% slower: on below 32768.
     const bool pdl = B < 32768;
+    // 128-column gate tiles when 256-column ones would leave most CTA pairs idle: few row
+    // tiles, or compacted live rows (bf16, flat actions)
+    const int pairs = T.sms / 2;
+    const bool narrow = !f32 && !hier && T.wg_n && (compact || teacher || m_tiles * (H / 64) < pairs);
+    CUtensorMap mwgn, mxsn[2];
+    if (narrow && (!make_map(&mwgn, T.wg_n, 4 * H, KX, 64) || !make_map_x32(&mxsn[0], w.x[0], B, KX) ||
+                   !make_map_x32(&mxsn[1], w.x[1], B, KX)))
+        return cudaErrorInvalidValue;
+    StepIO gio_n;  // the gate launches' parameters with the 128-column packing
     if (teacher) {  // batched scoring: the recurrence step by step, then one head GEMM
         const size_t fr = (size_t)B * KX;  // elements of one frame of operand rows
         cudaError_t e = cudaSuccess;
@@ -2078,7 +2129,18 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
                 h->test_wait = 0;
             }
             const OpMaps opg{&ma, &mwg, &mal, &mwgl};
-            {
+            if (narrow) {
+                CUtensorMap msn;
+                if (!make_map_x32(&msn, w.xall + (t + 1) * fr, B, KX)) return cudaErrorInvalidValue;
+                gio_n = io;
+                gio_n.wa = (const __nv_bfloat16 *)T.wa_n;
+                gio_n.b_gate = T.bg_n;
+                GemmGrid g2n = g2;
+                g2n.n_tiles = H / 32;
+                const OpMaps opn{&ma, &mwgn, &ma, &mwgn};
+                wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
+                e = launch_gemm<128, 1, 3, EpiGatesN, 2>(opn, mc, msn, msn, g2n, gio_n, T.sms, s, pdl);
+            } else {
                 wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
                 if (f32) e = launch_gemm<256, 1, 2, EpiGates32, 2, 3>(opg, mc, ms, msl, g2, io, T.sms, s, pdl);
                 else e = launch_gemm<256, 1, 2, EpiGates, 2>(opg, mc, ms, ms, g2, io, T.sms, s, pdl);
@@ -2262,7 +2324,16 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
         GemmGrid g2{m_tiles, H / 64, (KX + BK - 1) / BK, 0, h->status};
         g2.n_rows = io.n_rows;
         if (teacher) g2.test_wait = test_wait;
-        {
+        if (narrow) {
+            gio_n = io;
+            gio_n.wa = (const __nv_bfloat16 *)T.wa_n;
+            gio_n.b_gate = T.bg_n;
+            GemmGrid g2n = g2;
+            g2n.n_tiles = H / 32;
+            const OpMaps opn{&mx[xa], &mwgn, &mx[xa], &mwgn};
+            wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
+            e = launch_gemm<128, 1, 3, EpiGatesN, 2>(opn, mC, mxsn[xn], mxsn[xn], g2n, gio_n, T.sms, s, pdl);
+        } else {
             wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
             if (f32) e = launch_gemm<256, 1, 2, EpiGates32, 2, 3>(opg, mC, mxs[xn], mxsl[xn], g2, io, T.sms, s, pdl);
             else if (hier) e = launch_gemm<256, 1, 2, EpiGates2, 2>(opg, mC, mxs[xn], mxs[xn], g2, io, T.sms, s, pdl);
