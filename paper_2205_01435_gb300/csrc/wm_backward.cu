@@ -37,33 +37,44 @@ template <> __device__ __forceinline__ __nv_bfloat16 to_op<__nv_bfloat16>(float 
 
 // X [NT, Z+H] = [z_t | h_{t-1}] and Y [NT, H] = h_t, in the GEMM operand type (bf16: RNE,
 // the forward's operand rounding)
+// (a block per row at a time, the row's columns over its threads: no 64-bit divisions)
 template <class T>
 __global__ void k_bw_build(int N, int TT, int Z, int H, const float *__restrict__ z_seq,
                            const float *__restrict__ hs, T *__restrict__ X, T *__restrict__ Y) {
     const int KX = Z + H;
-    const size_t NT = (size_t)N * TT, nx = NT * KX;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nx; i += (size_t)gridDim.x * blockDim.x) {
-        const size_t r = i / KX, k = i % KX;
-        float v;
-        if (k < (size_t)Z) v = z_seq[r * Z + k];
-        else v = r >= (size_t)N ? hs[(r - N) * H + (k - Z)] : 0.f;  // h_{-1} = 0
-        X[i] = to_op<T>(v);
+    const size_t NT = (size_t)N * TT;
+    for (size_t r = blockIdx.x; r < NT; r += gridDim.x) {
+        const float *hp = r >= (size_t)N ? hs + (r - N) * H : nullptr;  // h_{-1} = 0
+        for (int k = threadIdx.x; k < KX; k += blockDim.x) {
+            const float v = k < Z ? z_seq[r * Z + k] : (hp ? hp[k - Z] : 0.f);
+            X[r * KX + k] = to_op<T>(v);
+        }
+        for (int k = threadIdx.x; k < H; k += blockDim.x) Y[r * H + k] = to_op<T>(hs[r * H + k]);
     }
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < NT * H; i += (size_t)gridDim.x * blockDim.x)
-        Y[i] = to_op<T>(hs[i]);
 }
 
-// gate pre-activations + bias + the action row -> i, f, g, o (in place)
+// gate pre-activations + bias + the action row -> i, f, g, o (in place); a block per row at
+// a time, four columns per thread
 __global__ void k_bw_gates(size_t NT, int N, int H, int A, float *__restrict__ G, const int32_t *__restrict__ act,
                            const float *__restrict__ Wa, const float *__restrict__ bias) {
     const int H4 = 4 * H;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < NT * H4; i += (size_t)gridDim.x * blockDim.x) {
-        const size_t r = i / H4;
-        const int col = (int)(i % H4);
-        int a = act[r];
-        float v = G[i] + bias[col];
-        if (a >= 0 && a < A) v += Wa[(size_t)a * H4 + col];
-        G[i] = col / H == 2 ? tanhf(v) : 1.f / (1.f + expf(-v));
+    for (size_t r = blockIdx.x; r < NT; r += gridDim.x) {
+        const int a = act[r];
+        const float *wa = (a >= 0 && a < A) ? Wa + (size_t)a * H4 : nullptr;
+        float4 *g4 = reinterpret_cast<float4 *>(G + r * H4);
+        for (int c4 = threadIdx.x; c4 < H4 / 4; c4 += blockDim.x) {
+            const int col = 4 * c4;
+            float4 v = g4[c4];
+            float x[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float u = x[j] + bias[col + j];
+                if (wa) u += wa[col + j];
+                const bool cand = col + j >= 2 * H && col + j < 3 * H;  // the g gate: tanh
+                x[j] = cand ? tanhf(u) : 1.f / (1.f + expf(-u));
+            }
+            g4[c4] = make_float4(x[0], x[1], x[2], x[3]);
+        }
     }
 }
 
@@ -144,35 +155,89 @@ __global__ void k_bw_cell(int N, int H, int t, int first, const float *__restric
     }
 }
 
-// Column sums of a [R, C] matrix, two levels: chunk c of the rows into part[c][C], then
-// the CHUNKS partials in order.  One thread per column, rows in order (fixed sum order).
+// Column sums of a [R, C] matrix, two levels: chunk c of the rows (COLSUM_CHUNKS of them)
+// into part[c][C], then the chunks' partials in order.  One thread per column, rows in
+// order, a compensated (Kahan) fp32 sum: the error stays near one rounding whatever R,
+// and the order, so the result, is fixed.
+constexpr int COLSUM_CHUNKS = 64;
 __global__ void k_bw_colsum(size_t R, int C, const float *__restrict__ in, float *__restrict__ part) {
     const int col = blockIdx.x * blockDim.x + threadIdx.x, c = blockIdx.y;
     if (col >= C) return;
-    const size_t r0 = R * c / CHUNKS, r1 = R * (c + 1) / CHUNKS;
-    double s = 0.0;
-    for (size_t r = r0; r < r1; ++r) s += in[r * C + col];
-    part[(size_t)c * C + col] = (float)s;
+    const size_t r0 = R * c / COLSUM_CHUNKS, r1 = R * (c + 1) / COLSUM_CHUNKS;
+    float s = 0.f, comp = 0.f;
+    for (size_t r = r0; r < r1; ++r) {
+        const float y = in[r * C + col] - comp;
+        const float t = s + y;
+        comp = (t - s) - y;
+        s = t;
+    }
+    part[(size_t)c * C + col] = s;
 }
 __global__ void k_bw_colsum_fin(int C, const float *__restrict__ part, float *__restrict__ out) {
     const int col = blockIdx.x * blockDim.x + threadIdx.x;
     if (col >= C) return;
     double s = 0.0;
-    for (int c = 0; c < CHUNKS; ++c) s += part[(size_t)c * C + col];
+    for (int c = 0; c < COLSUM_CHUNKS; ++c) s += part[(size_t)c * C + col];
     out[col] = (float)s;
 }
 
-// The action rows of dW_lstm: block (a, c) sums, in row order, the dG rows of chunk c whose
-// action is a, into part[c][a][4H]; then the CHUNKS partials in order.
-__global__ void k_bw_arows(size_t R, int A, int H4, const int32_t *__restrict__ act, const float *__restrict__ dG,
-                           float *__restrict__ part) {
-    const int a = blockIdx.x, c = blockIdx.y;
+// The action rows of dW_lstm: dW_a[a] = sum of the dG rows whose action is a.  Each row
+// chunk is first sorted stably by action (k_bw_rowsort: one block per chunk, rows taken in
+// order by one warp 32 at a time, each lane's place among the lanes with the same action
+// from a match mask), then block (a, c) sums, in row order, only the rows of chunk c with
+// action a, into part[c][a][4H]; then the CHUNKS partials in order.
+__global__ void k_bw_rowsort(size_t R, int A, const int32_t *__restrict__ act, int32_t *__restrict__ srows,
+                             int32_t *__restrict__ soff) {
+    extern __shared__ int s_cnt[];  // [A] counts, then running cursors
+    const int c = blockIdx.x;
     const size_t r0 = R * c / CHUNKS, r1 = R * (c + 1) / CHUNKS;
+    for (int a = threadIdx.x; a < A; a += blockDim.x) s_cnt[a] = 0;
+    __syncthreads();
+    for (size_t r = r0 + threadIdx.x; r < r1; r += blockDim.x) {
+        const int a = act[r];
+        if (a >= 0 && a < A) atomicAdd(&s_cnt[a], 1);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {  // exclusive offsets within the chunk
+        int run = 0;
+        int32_t *off = soff + (size_t)c * (A + 1);
+        for (int a = 0; a < A; ++a) {
+            const int n = s_cnt[a];
+            off[a] = run;
+            s_cnt[a] = run;
+            run += n;
+        }
+        off[A] = run;
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        for (size_t b = r0; b < r1; b += 32) {
+            const size_t r = b + lane;
+            const int a = r < r1 ? act[r] : -1;
+            const bool ok = a >= 0 && a < A;
+            const uint32_t same = __match_any_sync(0xffffffffu, ok ? a : -1);
+            const int rank = __popc(same & ((1u << lane) - 1u));
+            int pos = 0;
+            if (ok) pos = s_cnt[a] + rank;
+            __syncwarp();
+            if (ok && rank == 0) s_cnt[a] += __popc(same);  // the lowest lane of each action
+            __syncwarp();
+            if (ok) srows[r0 + pos] = (int32_t)r;
+        }
+    }
+}
+__global__ void k_bw_arows(size_t R, int A, int H4, const int32_t *__restrict__ srows,
+                           const int32_t *__restrict__ soff, const float *__restrict__ dG, float *__restrict__ part) {
+    const int a = blockIdx.x, c = blockIdx.y;
+    const size_t r0 = R * c / CHUNKS;
+    const int32_t *off = soff + (size_t)c * (A + 1);
+    const int i0 = off[a], i1 = off[a + 1];
     for (int col0 = 0; col0 < H4; col0 += blockDim.x * 4) {
         float s[4] = {0.f, 0.f, 0.f, 0.f};
         const int col = col0 + 4 * threadIdx.x;
-        for (size_t r = r0; r < r1; ++r) {
-            if (act[r] != a) continue;  // uniform over the block
+        for (int i = i0; i < i1; ++i) {
+            const size_t r = (size_t)srows[r0 + i];
             if (col < H4)
                 for (int j = 0; j < 4; ++j)
                     if (col + j < H4) s[j] += dG[r * H4 + col + j];
@@ -249,7 +314,8 @@ size_t wm_bw_ws(const wm_handle *h, int N, int T) {
            + al(NT * H * 4)                                                    // dY
            + al(NT * H4 * 4) + al(NT * H4 * es)                                // dG
            + 2 * al((size_t)N * H * 4)                                         // dH, dc
-           + al((size_t)CHUNKS * part_cols * 4) + al((size_t)CHUNKS * A * H4 * 4) + 256;
+           + al((size_t)COLSUM_CHUNKS * part_cols * 4) + al((size_t)CHUNKS * A * H4 * 4)  // partials
+           + al(NT * 4) + al((size_t)CHUNKS * (A + 1) * 4) + 256;                  // rows sorted by action
 }
 
 cudaError_t wm_bw_prepare(wm_handle *h) {
@@ -303,8 +369,10 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     T *dGo = (T *)p; p += al(NT * H4 * sizeof(T));
     float *dH = (float *)p; p += al((size_t)N * H * 4);
     float *dC = (float *)p; p += al((size_t)N * H * 4);
-    float *part = (float *)p; p += al((size_t)CHUNKS * (H4 > M ? H4 : M) * 4);
-    float *apart = (float *)p;
+    float *part = (float *)p; p += al((size_t)COLSUM_CHUNKS * (H4 > M ? H4 : M) * 4);
+    float *apart = (float *)p; p += al((size_t)CHUNKS * A * H4 * 4);
+    int32_t *srows = (int32_t *)p; p += al(NT * 4);
+    int32_t *soff = (int32_t *)p;
     // weights of the GEMMs: W_zh = the z and h rows of the gate matrix, W_mdn, W_h = W_zh's h rows
     const void *Wzh = bf ? (const void *)h->bw_wzh : (const void *)h->step.Wg;
     const long ldw = bf ? H4 : H4 + A;
@@ -315,7 +383,7 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     int launches = 0;
     {
         wm_ktime kt(h, WM_KERNEL_BW, s);
-        k_bw_build<T><<<grid_of(NT * KX), 256, 0, s>>>(N, TT, Z, H, z_seq, hs, X, Y);
+        k_bw_build<T><<<(unsigned)(NT < 8192 ? NT : 8192), 256, 0, s>>>(N, TT, Z, H, z_seq, hs, X, Y);
         ++launches;
     }
     {
@@ -326,7 +394,7 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
     {
         wm_ktime kt(h, WM_KERNEL_BW, s);
-        k_bw_gates<<<grid_of(NT * H4), 256, 0, s>>>(NT, N, H, A, G, actions, h->step.Wa, h->step.bg);
+        k_bw_gates<<<(unsigned)(NT < 8192 ? NT : 8192), 256, 0, s>>>(NT, N, H, A, G, actions, h->step.Wa, h->step.bg);
         k_bw_mdn<T><<<grid_of(NT * Z), 256, 0, s>>>(N, TT, Z, c.k_mix, md, z_seq, lengths, dMD, dMDo);
         launches += 2;
     }
@@ -361,13 +429,14 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
     {
         wm_ktime kt(h, WM_KERNEL_BW, s);
-        k_bw_arows<<<dim3(A, CHUNKS), 256, 0, s>>>(NT, A, H4, actions, dG, apart);
+        k_bw_rowsort<<<CHUNKS, 256, (size_t)A * 4, s>>>(NT, A, actions, srows, soff);
+        k_bw_arows<<<dim3(A, CHUNKS), 256, 0, s>>>(NT, A, H4, srows, soff, dG, apart);
         k_bw_arows_fin<<<grid_of((size_t)A * H4), 256, 0, s>>>(A, H4, apart, g.W_lstm + (size_t)Z * H4);
-        k_bw_colsum<<<dim3((H4 + 255) / 256, CHUNKS), 256, 0, s>>>(NT, H4, dG, part);
+        k_bw_colsum<<<dim3((H4 + 255) / 256, COLSUM_CHUNKS), 256, 0, s>>>(NT, H4, dG, part);
         k_bw_colsum_fin<<<(H4 + 255) / 256, 256, 0, s>>>(H4, part, g.b_lstm);
-        k_bw_colsum<<<dim3((M + 255) / 256, CHUNKS), 256, 0, s>>>(NT, M, dMD, part);
+        k_bw_colsum<<<dim3((M + 255) / 256, COLSUM_CHUNKS), 256, 0, s>>>(NT, M, dMD, part);
         k_bw_colsum_fin<<<(M + 255) / 256, 256, 0, s>>>(M, part, g.b_mdn);
-        launches += 6;
+        launches += 7;
     }
     h->last_launches += launches;
     return cudaGetLastError();
