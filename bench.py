@@ -69,6 +69,7 @@ def fp32_simt_peak_tflops() -> float:
 
 # kernel class -> (kernel as the profiler names it, source file)
 KERNELS = {"fused": ("k_fused", "wm_fused.cu"),
+           "fused_small": ("k_small", "wm_small.cu"),
            "tc_ctrl": ("k_tc_gemm<EpiCtrl>", "wm_tensor.cu"),
            "tc_gates": ("k_tc_gemm<EpiGates>", "wm_tensor.cu"),
            "tc_heads": ("k_tc_gemm<EpiHeads>", "wm_tensor.cu"),
@@ -92,7 +93,7 @@ def nll_inputs(cfg: dict, rank: int = 0):
 def kernel_flops(cls: str, cfg: dict, B: int, T: int, launches: int) -> float:
     """Algorithmic FLOPs of one launch of a kernel class (its contraction)."""
     Z, A, H, K = cfg["z_dim"], cfg["a_dim"], cfg["h_dim"], cfg["k_mix"]
-    if cls == "fused":
+    if cls in ("fused", "fused_small"):
         return (nll_flops_per_step(cfg) if cfg.get("teacher") else flops_per_env_step(cfg)) * B * T
     if cls == "tc_ctrl":
         return 2.0 * B * (Z + H) * A

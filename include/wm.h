@@ -87,7 +87,17 @@ typedef enum {
 enum { WM_FP32 = 0, WM_BF16 = 1 };
 
 /* Kernel family.  AUTO picks by batch size and model size; the others force
- * one (WM_ERR_UNSUPPORTED if it cannot run the model). */
+ * one (WM_ERR_UNSUPPORTED if it cannot run the model).
+ *   STEPWISE  four SIMT launches per step; every model and option.
+ *   FUSED     one launch for all T steps, in two members: a tcgen05 kernel for
+ *             bf16 models with Z = 32, H = 256, K = 5, masked argmax and the
+ *             linear reward head (one cluster per 128 episodes), and a small-batch
+ *             fp32 SIMT kernel for the other models whose weights fit a cluster's
+ *             shared memory (one cluster per 16 episodes; either precision,
+ *             controller and reward), taken while the batch needs at most 4 waves
+ *             of clusters.  Neither writes log-probs or values, takes a population
+ *             or a hierarchical action.
+ *   TENSOR    three tcgen05 GEMM launches per step (H % 64 == 0, A % 64 == 0). */
 enum { WM_PATH_AUTO = 0, WM_PATH_STEPWISE = 1, WM_PATH_FUSED = 2, WM_PATH_TENSOR = 3 };
 
 typedef struct {
@@ -101,15 +111,17 @@ typedef struct {
     int noop_terminates;              /* action A-1 (NO-OP, Sec. 3.1.3) freezes it */
     unsigned long long seed;          /* Philox key                                */
     int path;                         /* WM_PATH_*                                 */
-    int fused_cluster;                /* fused family: CTAs per cluster, 8 or 16;
-                                         0 = choose per call (fewest waves)        */
+    int fused_cluster;                /* fused family, tcgen05 member: CTAs per
+                                         cluster, 8 or 16; 0 = choose per call
+                                         (fewest waves)                             */
     /* Reward (Sec. 3.1.4).  WM_REWARD_HEAD: r_t = w_rew . h' + b_rew.
      * WM_REWARD_SHAPED: two more linear heads on h' predict the graph's runtime
      * RT and memory accesses M, and r_t = alpha (RT_{t-1} - RT_t) +
      * beta (M_{t-1} - M_t) (Eq. 2; Eq. 1 is alpha = 1, beta = 0) when an action
      * was taken, invalid_reward when none was (a = -1).  Sec. 4.3 found
      * alpha = 0.8, beta = 0.2 best; Eq. 1 / 2 give -100 for an invalid action.
-     * The stepwise and tensor-core families take it; the fused family does not. */
+     * The stepwise and tensor-core families and the fused family's small-batch
+     * member take it; the fused family's tcgen05 member does not. */
     int reward_mode;                  /* WM_REWARD_HEAD or WM_REWARD_SHAPED         */
     float reward_alpha, reward_beta;
     float invalid_reward;
@@ -365,7 +377,8 @@ enum {
     WM_KERNEL_AUX = 7,          /* state set-up, finishing copies, reductions      */
     WM_KERNEL_BW = 8,           /* training step: the library's backward kernels    */
     WM_KERNEL_BW_GEMM = 9,      /* training step: its cuBLAS GEMMs                  */
-    WM_KERNEL_CLASSES = 10
+    WM_KERNEL_FUSED_SMALL = 10, /* fused, small-batch member: the single kernel     */
+    WM_KERNEL_CLASSES = 11
 };
 
 /* enable != 0 turns timing on and clears the totals; 0 turns it off (events

@@ -257,10 +257,12 @@ cudaError_t pack_step(wm_handle *h, const wm_weights *w) {
     return upload(&h->step.bh, bh);
 }
 
-// AUTO: the fused single-launch family for batches that fit one wave of clusters,
-// the tensor-core family for large bf16 batches and for fp32 models of any batch (its
-// three-pass split beat the fp32 SIMT family 2x even at B = 16), the stepwise family
-// otherwise.  fused_ok / tc_ok: whether this call's options allow those families.
+// AUTO: the fused single-launch family when one of its members takes the model and the
+// batch (its tcgen05 member up to B = 2048; its small-batch member while the batch needs at
+// most 4 waves of 16-episode clusters), else the tensor-core family for large bf16 batches
+// and for fp32 models of any batch (its three-pass split beat the stepwise fp32 SIMT family
+// 2x even at B = 16), the stepwise family otherwise.  fused_ok / tc_ok: whether this call's
+// options allow those families.
 int pick_path(const wm_handle *h, int B, bool fused_ok = true, bool tc_ok = true) {
     const int p = h->cfg.path;
     if (p != WM_PATH_AUTO) return p;
@@ -315,11 +317,13 @@ wm_status wm_create(const wm_config *cfg, const wm_weights *w, wm_handle **out) 
     }
     memset(&h->step, 0, sizeof(h->step));
     memset(&h->fused, 0, sizeof(h->fused));
+    memset(&h->small, 0, sizeof(h->small));
     memset(&h->tc, 0, sizeof(h->tc));
     cudaError_t e = cudaGetDevice(&h->device);
     if (e == cudaSuccess) e = pack_step(h, w);
     h->fused.force_cluster = cfg->fused_cluster;
     if (e == cudaSuccess) e = wm_fused_pack(h, w);
+    if (e == cudaSuccess) e = wm_small_prepare(h);
     if (e == cudaSuccess) e = wm_tc_pack(h, w);
     if (e == cudaSuccess) e = cudaMalloc((void **)&h->status, sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(h->status, 0, sizeof(int));

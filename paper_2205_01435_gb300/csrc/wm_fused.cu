@@ -47,6 +47,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <mutex>
 #include <vector>
 
 #include "tc_ptx.cuh"
@@ -783,6 +784,23 @@ void *pack_images(const wm_config &c, const wm_weights *w, size_t *img_bytes, cu
     return d;
 }
 
+// Raises k_fused<S>'s dynamic shared-memory limit on the current device to at least `bytes`,
+// never lowering it: the geometry depends on A, and handles of other models may launch the
+// same instantiation with more.
+template <class S>
+cudaError_t smem_at_least(size_t bytes) {
+    static std::mutex mu;
+    static size_t cur[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lk(mu);
+    if (dev >= 0 && dev < 64 && bytes <= cur[dev]) return cudaSuccess;
+    e = cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess && dev >= 0 && dev < 64) cur[dev] = bytes;
+    return e;
+}
+
 // How many clusters of shape S can be resident at once (0 if none).
 template <class S>
 int max_clusters(const wm_config &c) {
@@ -791,7 +809,7 @@ int max_clusters(const wm_config &c) {
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if ((size_t)optin < g.smem + 2048) return 0;
-    if (cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem) != cudaSuccess ||
+    if (smem_at_least<S>(g.smem) != cudaSuccess ||
         (S::CL > 8 && cudaFuncSetAttribute(k_fused<S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
                           cudaSuccess)) {
         cudaGetLastError();
@@ -836,6 +854,8 @@ cudaError_t launch_fused(const wm_handle *h, int slot, FusedParams &p, cudaStrea
     p.img_stride = h->fused.img_bytes[slot];
     p.AC = p.A / S::CL;
     p.status = h->status;
+    const cudaError_t e = smem_at_least<S>(g.smem);
+    if (e != cudaSuccess) return e;
     return cudaLaunchKernelEx(&lc, k_fused<S>, p);
 }
 
@@ -867,14 +887,17 @@ FusedParams base_params(const wm_handle *h, int B, int T) {
 }  // namespace
 
 // ---------------------------------------------------------------------------
-int wm_fused_supported(const wm_handle *h, int B) {
-    (void)B;
+// Whether the tcgen05 member takes the model: bf16, its shapes, masked argmax and the linear
+// reward head.  The family's other member (wm_small.cu) takes small batches of the rest.
+static int tc_member(const wm_handle *h) {
     const wm_config &c = h->cfg;
     if (!h->fused.ok) return 0;
     if (c.ctrl_sample && c.ctrl_tau > 0.f) return 0;  // masked argmax only
     if (c.reward_mode != WM_REWARD_HEAD) return 0;    // the linear reward head only
     return 1;
 }
+
+int wm_fused_supported(const wm_handle *h, int B) { return tc_member(h) || wm_small_supported(h, B); }
 
 cudaError_t wm_fused_pack(wm_handle *h, const wm_weights *w) {
     const wm_config &c = h->cfg;
@@ -902,6 +925,7 @@ void wm_fused_free(wm_handle *h) {
 int wm_fused_cluster_size(const wm_handle *h, int B) { return choose_slot(h, B) == 0 ? S16::CL : S8::CL; }
 
 cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaStream_t s) {
+    if (!tc_member(h)) return wm_small_rollout(h, a, s);
     if (a.B == 0) { h->last_launches = 0; return cudaSuccess; }
     // z_out[0] = z0
     const size_t nz = (size_t)a.B * h->cfg.z_dim;
@@ -945,6 +969,7 @@ cudaError_t wm_fused_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaSt
 size_t wm_fused_nll_ws(const wm_handle *h, int N) { return (size_t)h->cfg.z_dim * N * 4 + 256; }
 
 cudaError_t wm_fused_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStream_t s) {
+    if (!tc_member(h)) return wm_small_nll(h, a, s);
     if (a.N == 0) { h->last_launches = 0; return cudaSuccess; }
     if (a.T == 0) {
         h->last_launches = 0;

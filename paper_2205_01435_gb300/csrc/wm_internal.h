@@ -74,6 +74,15 @@ struct wm_fused_weights {
     int ok;                // 1 if the model fits this family
 };
 
+// The fused family's small-batch member (wm_small.cu): it reads the stepwise weights;
+// this records the cluster size chosen for the model and its shared-memory geometry.
+struct wm_small_cfg {
+    int ok;                  // 1 if the model's per-CTA columns fit a cluster's shared memory
+    int cl;                  // CTAs per cluster (1, 2, 4, 8 or 16)
+    int max_clusters_eb[3];  // clusters resident at once, per tile size (16, 8, 4 episodes)
+    alignas(8) unsigned char geo[3][256];  // wm_small.cu's geometry record per tile size
+};
+
 // Weights of the tensor-core family (bf16, K-major; orders in wm_tensor.cu).
 struct wm_tc_weights {
     void *wc, *wg, *wa, *wh;  // W_c^T [P*A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
@@ -129,6 +138,7 @@ struct wm_handle {
                                  // when the controller changes)
     wm_step_weights step;
     wm_fused_weights fused;
+    wm_small_cfg small;
     wm_tc_weights tc;
     void *ws = nullptr;          // workspace (grows on demand)
     size_t ws_bytes = 0;
@@ -185,6 +195,13 @@ cudaError_t wm_tc_nll(const wm_handle *h, const wm_nll_dev &a, void *ws, cudaStr
 cudaError_t wm_tc_set_controllers(wm_handle *h, int P, const float *W_ctrl, const float *b_ctrl);
 // whether the tensor family can run a rollout call starting at this episode (population tiles)
 int wm_tc_call_ok(const wm_handle *h, unsigned long long episode_offset);
+
+// ---- the fused family's small-batch member (wm_small.cu) ----------------------
+cudaError_t wm_small_prepare(wm_handle *h);
+int wm_small_supported(const wm_handle *h, int B);
+int wm_small_cluster_size(const wm_handle *h);
+cudaError_t wm_small_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaStream_t s);
+cudaError_t wm_small_nll(const wm_handle *h, const wm_nll_dev &a, cudaStream_t s);
 
 // ---- the training step (wm_backward.cu) -----------------------------------------
 size_t wm_bw_ws(const wm_handle *h, int N, int T);

@@ -23,7 +23,7 @@ WM_FP32, WM_BF16 = 0, 1
 PATHS = {"auto": 0, "stepwise": 1, "fused": 2, "tensor": 3}
 PATH_NAMES = {v: k for k, v in PATHS.items()}
 KERNEL_CLASSES = ("step_gemm", "step_cell", "step_sample", "fused", "tc_ctrl", "tc_gates",
-                  "tc_heads", "aux", "bw", "bw_gemm")  # WM_KERNEL_* in order
+                  "tc_heads", "aux", "bw", "bw_gemm", "fused_small")  # WM_KERNEL_* in order
 
 
 class WMError(RuntimeError):

@@ -202,11 +202,12 @@ def test_empty_and_zero_length(wm):
     assert n["nll"].numel() == 0
 
 
-@pytest.mark.parametrize("path", ["fused", "tensor"])
-def test_empty_and_zero_length_on_each_family(wm, path):
-    """B = 0, T = 0 (state passes through unchanged) and N = 0 / T = 0 scoring on the
-    fused and tensor-core families, which the small tiny_fp32 case above does not reach."""
-    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=40, T=3)
+@pytest.mark.parametrize("path,name", [("fused", "small_bf16"), ("fused", "tiny_fp32"),
+                                       ("tensor", "small_bf16")])
+def test_empty_and_zero_length_on_each_family(wm, path, name):
+    """B = 0, T = 0 (state passes through unchanged) and N = 0 / T = 0 scoring on both
+    members of the fused family and on the tensor-core family."""
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=40, T=3)
     m = wm.WorldModel(dict(cfg, path=path), w)
     g = m.rollout(_cuda(z0[:0]), T, mask=_cuda(mask[:, :0]))
     torch.cuda.synchronize()
@@ -238,12 +239,13 @@ def test_invalid_arguments(wm):
         m.mdn_nll(torch.from_numpy(zs), torch.from_numpy(acts))  # host actions are checked
 
 
-@pytest.mark.parametrize("path", ["stepwise", "fused", "tensor"])
-def test_device_teacher_inputs_out_of_range_are_reported(wm, orc, path):
+@pytest.mark.parametrize("path,name", [("stepwise", "small_bf16"), ("fused", "small_bf16"),
+                                       ("fused", "tiny_fp32"), ("tensor", "small_bf16")])
+def test_device_teacher_inputs_out_of_range_are_reported(wm, orc, path, name):
     """On device arrays an action >= A or a length outside [0, T] is found by the kernels:
     wm_sync reports WM_ERR_INVALID_ARG once, the action counts as no action, the length is
     clamped, and the next call runs clean."""
-    cfg = synth.model_config("small_bf16")
+    cfg = synth.model_config(name)
     w = synth.weights(cfg, seed=12)
     N, T = 40, 5
     zs, acts, _ = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=12)
@@ -261,7 +263,7 @@ def test_device_teacher_inputs_out_of_range_are_reported(wm, orc, path):
         assert m.last_path == path
         fixed_a = np.where(a2 >= cfg["a_dim"], -1, a2)
         o = orc.mdn_nll(cfg, w, zs, fixed_a, lengths=np.clip(lens, 0, T))
-        check_teacher({"nll": g["nll"]}, o, "bf16")
+        check_teacher({"nll": g["nll"]}, o, cfg["precision"])
         m.mdn_nll(_cuda(zs), _cuda(acts))
         m.sync()  # the status was cleared
 
@@ -374,6 +376,87 @@ def test_fused_matches_stepwise_closely(wm):
     assert ok.mean() > 0.95, ok.mean()
 
 
+# ------------------------------------------------------------------ the fused family's small-batch member
+SMALL_CASES = [
+    ("fp32", dict()),
+    ("fp32", dict(done_terminates=1, noop_terminates=1)),
+    ("fp32", dict(ctrl_sample=1, ctrl_tau=0.7, mdn_tau=0.5, sigma_sqrt_tau=1)),
+    ("fp32", dict(mdn_tau=0.0)),
+    ("fp32", dict(reward_mode=1, done_terminates=1)),
+    ("bf16", dict(ctrl_sample=1, ctrl_tau=1.0)),  # bf16, a controller the tcgen05 member does not take
+]
+
+
+@pytest.mark.parametrize("prec,flags", SMALL_CASES)
+def test_fused_small_against_oracle(wm, orc, prec, flags):
+    """The single-launch fp32 SIMT member on the tiny model: 13 clusters of 16 episodes (the
+    last one partly filled), resumed state, frozen episodes, offsets, every flag; one launch."""
+    cfg = dict(synth.model_config("tiny_fp32"), precision=prec, **flags)
+    w = synth.weights(cfg, seed=21)
+    B, T = 200, 9
+    z0 = synth.z0(B, cfg["z_dim"], seed=21)
+    mask = synth.mask(T, B, cfg["a_dim"], 0.5, seed=21)
+    mask[3, 17] = 0  # no valid action for one episode at one step
+    rng = np.random.default_rng(21)
+    h0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    c0 = (0.3 * rng.standard_normal((B, cfg["h_dim"]))).astype(np.float32)
+    done0 = (np.arange(B) % 37 == 0).astype(np.uint8)
+    extra, okw = {}, {}
+    if flags.get("reward_mode") == 1:
+        rt0, mem0 = synth.shaping_state(B, seed=21)
+        extra = dict(rt0=_cuda(rt0), mem0=_cuda(mem0))
+        okw = dict(rt0=rt0, mem0=mem0)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=91, t0=5, h0=_cuda(h0), c0=_cuda(c0),
+                  done0=_cuda(done0), want_seq=True, **extra)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused" and m.last_launches == 1
+    assert int(g["actions"][3, 17]) == -1 or bool(done0[17])
+    r = check_rollout(g, cfg, w, z0, mask, episodes=91 + np.arange(B), t0=5, h0=h0, c0=c0,
+                      done0=done0, orc=orc, **okw)
+    assert r["compared"] + r["frozen_steps"] == B * T
+    print("fused small", prec, flags, r)
+    # AUTO takes the same member for this batch: the same bits
+    ga = wm.WorldModel(dict(cfg, path="auto"), w).rollout(
+        _cuda(z0), T, mask=_cuda(mask), episode_offset=91, t0=5, h0=_cuda(h0), c0=_cuda(c0),
+        done0=_cuda(done0), **extra)
+    for k in ("z", "actions", "rewards", "done"):
+        assert torch.equal(ga[k], g[k]), k
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_fused_small_teacher_forced_ragged(wm, orc, prec):
+    """Scoring on the small-batch member: ragged lengths, no-action steps, a partial tile."""
+    cfg = dict(synth.model_config("tiny_fp32"), precision=prec, ctrl_sample=1)
+    w = synth.weights(cfg, seed=22)
+    zs, acts, lens = synth.teacher_inputs(45, 13, cfg["z_dim"], cfg["a_dim"], seed=22, ragged=True)
+    acts[4, ::3] = -1
+    lens[0], lens[1] = 0, 13
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused" and m.last_launches == 1
+    o = orc.mdn_nll(cfg, w, zs, acts, lengths=lens, want_seq=True, nthreads=NT)
+    check_teacher({k: np_(v) for k, v in g.items()}, o, prec)
+
+
+def test_fused_small_odd_shapes(wm, orc):
+    """A model whose sizes divide nothing (Z=7, A=45, H=40, K=3): ranks own ragged slices of
+    units, actions and dims, and some own none."""
+    cfg = dict(synth.model_config("tiny_fp32"), z_dim=7, a_dim=45, h_dim=40, k_mix=3,
+               done_terminates=1, noop_terminates=1, ctrl_sample=1, ctrl_tau=0.9)
+    w = synth.weights(cfg, seed=23, std=0.3)
+    B, T = 53, 11
+    z0 = synth.z0(B, 7, seed=23)
+    mask = synth.mask(T, B, 45, 0.4, seed=23)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=5, want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    r = check_rollout(g, cfg, w, z0, mask, episodes=5 + np.arange(B), orc=orc)
+    assert r["compared"] + r["frozen_steps"] == B * T
+
+
 # ------------------------------------------------------------------ the tensor-core family
 @pytest.mark.parametrize("name,flags", [("mid_bf16", dict()), ("large_bf16", dict()),
                                         ("small_bf16", dict(mdn_tau=0.0)),
@@ -461,7 +544,7 @@ def test_tensor_full_batch_is_deterministic(wm, name, T, B, flags):
                                              ("stepwise", "mid_bf16", dict(reward_alpha=1.0, reward_beta=0.0))])
 def test_shaped_reward_against_oracle(wm, orc, path, name, flags):
     """Eq. 2 on the predicted runtime / memory heads, with an invalid step (-100), resumed
-    state, offsets and frozen episodes; AUTO never routes it to the fused family."""
+    state, offsets and frozen episodes."""
     cfg = dict(synth.model_config(name), reward_mode=1, **flags)
     w = synth.weights(cfg, seed=13)
     B, T = (16, 12) if name == "tiny_fp32" else (200, 6)
@@ -477,7 +560,7 @@ def test_shaped_reward_against_oracle(wm, orc, path, name, flags):
     g = m.rollout(_cuda(z0), T, mask=_cuda(mask), episode_offset=55, t0=4, h0=_cuda(h0), c0=_cuda(c0),
                   done0=_cuda(done0), rt0=_cuda(rt0), mem0=_cuda(mem0), want_seq=True)
     torch.cuda.synchronize()
-    assert m.last_path != "fused" and (path == "auto" or m.last_path == path)
+    assert path == "auto" or m.last_path == path  # AUTO: the fused family's small-batch member
     assert int(g["actions"][0, 9]) == -1 and float(g["rewards"][0, 9]) == -100.0
     r = check_rollout(g, cfg, w, z0, mask, episodes=55 + np.arange(B), t0=4, h0=h0, c0=c0,
                       done0=done0, orc=orc, rt0=rt0, mem0=mem0)

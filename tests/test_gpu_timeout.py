@@ -38,9 +38,10 @@ def _expect_timeout(wm, m):
     m.sync()  # the status word was cleared
 
 
-@pytest.mark.parametrize("path,B,T", [("fused", 256, 4), ("tensor", 300, 3)])
-def test_rollout_wait_runs_out_then_recovers(wm, orc, path, B, T):
-    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=B, T=T)
+@pytest.mark.parametrize("name,path,B,T", [("small_bf16", "fused", 256, 4), ("tiny_fp32", "fused", 40, 4),
+                                            ("small_bf16", "tensor", 300, 3)])
+def test_rollout_wait_runs_out_then_recovers(wm, orc, name, path, B, T):
+    cfg, w, z0, mask, B, T = synth.rollout_inputs(name, B=B, T=T)
     m = wm.WorldModel(dict(cfg, path=path), w)
     zc, mc = _cuda(z0), _cuda(mask)
     m.inject_wait_timeout(POLLS)
@@ -62,9 +63,10 @@ def test_rollout_wait_runs_out_then_recovers(wm, orc, path, B, T):
     m.close()
 
 
-@pytest.mark.parametrize("path", ["fused", "tensor"])
-def test_scoring_wait_runs_out_then_recovers(wm, orc, path):
-    cfg = synth.model_config("small_bf16")
+@pytest.mark.parametrize("name,path", [("small_bf16", "fused"), ("tiny_fp32", "fused"),
+                                       ("small_bf16", "tensor")])
+def test_scoring_wait_runs_out_then_recovers(wm, orc, name, path):
+    cfg = synth.model_config(name)
     w = synth.weights(cfg)
     N, T = 200, 5
     zs, acts, _ = synth.teacher_inputs(N, T, cfg["z_dim"], cfg["a_dim"], seed=5)
@@ -76,7 +78,7 @@ def test_scoring_wait_runs_out_then_recovers(wm, orc, path):
     g = m.mdn_nll(_cuda(zs), _cuda(acts), want_seq=True)
     m.sync()
     o = orc.mdn_nll(cfg, w, zs, acts, want_seq=True)
-    check_teacher({k: v.cpu().numpy() for k, v in g.items()}, o, "bf16")
+    check_teacher({k: v.cpu().numpy() for k, v in g.items()}, o, cfg["precision"])
     m.close()
 
 

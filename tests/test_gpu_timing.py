@@ -11,6 +11,7 @@ pytestmark = pytest.mark.gpu
 CASES = [  # workload, path, B, T, classes the call must launch
     ("tiny_fp32", "stepwise", 16, 5, {"step_gemm", "step_cell", "step_sample", "aux"}),
     ("small_bf16", "fused", 256, 6, {"fused", "aux"}),
+    ("tiny_fp32", "fused", 16, 5, {"fused_small"}),
     ("mid_bf16", "tensor", 384, 4, {"tc_ctrl", "tc_gates", "tc_heads", "aux"}),
 ]
 
