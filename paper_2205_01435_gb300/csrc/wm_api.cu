@@ -351,6 +351,7 @@ void wm_destroy(wm_handle *h) {
     cudaFree(h->step.Wp);
     cudaFree(h->step.bp);
     wm_fused_free(h);
+    wm_small_free(h);
     wm_tc_free(h);
     wm_bw_free(h);
     cudaFree(h->ws);
@@ -591,6 +592,7 @@ wm_status wm_set_controllers(wm_handle *h, int P, int E, const float *W_ctrl, co
         wm_fused_free(h);
         const wm_weights hv = h->host.view();
         e = wm_fused_pack(h, &hv);
+        if (e == cudaSuccess) e = wm_small_repack(h);
     }
     if (e != cudaSuccess) return cuda_fail(h, e, "wm_set_controllers");
     h->P = P;

@@ -81,6 +81,8 @@ struct wm_small_cfg {
     int cl;                  // CTAs per cluster (1, 2, 4, 8 or 16)
     int max_clusters_eb[3];  // clusters resident at once, per tile size (16, 8, 4 episodes)
     alignas(8) unsigned char geo[3][256];  // wm_small.cu's geometry record per tile size
+    void *img;               // per-rank weight images (the shared-memory layout), cl of them
+    size_t img_stride;       // bytes between two ranks' images
 };
 
 // Weights of the tensor-core family (bf16, K-major; orders in wm_tensor.cu).
@@ -198,6 +200,8 @@ int wm_tc_call_ok(const wm_handle *h, unsigned long long episode_offset);
 
 // ---- the fused family's small-batch member (wm_small.cu) ----------------------
 cudaError_t wm_small_prepare(wm_handle *h);
+cudaError_t wm_small_repack(wm_handle *h);  // after the stepwise weights changed
+void wm_small_free(wm_handle *h);
 int wm_small_supported(const wm_handle *h, int B);
 int wm_small_cluster_size(const wm_handle *h);
 cudaError_t wm_small_rollout(const wm_handle *h, const wm_rollout_dev &a, cudaStream_t s);

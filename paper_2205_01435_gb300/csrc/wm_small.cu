@@ -64,7 +64,8 @@ struct Tile {
 // Shared-memory geometry of one CTA (offsets in floats, each a multiple of 4).
 struct Geo {
     int EB, XS, CL, KX, U, AC, DZ, G4, NC1, NC1P, NC2, NC2P, AP, W, nthreads;
-    int w1, wa, b1, w2, b2, xt, lg, g1, hd, cs, hs, zs, nl, pu, pe, mk, sc, ep;
+    int w1, b1, wa, w2, b2, xt, lg, g1, hd, cs, hs, zs, nl, pu, pe, mk, sc, ep;
+    int wpart1, wend;  // the weight image: [0, wpart1) W1 and b1, [wpart1, wend) W_a, W2, b2
     size_t smem;
 };
 
@@ -99,10 +100,12 @@ Geo geometry(int Z, int A, int H, int K, int NR, int CL, int EB, int XS, int S1,
         return at;
     };
     g.w1 = take((long)g.KX * g.NC1P);
-    g.wa = take((long)A * g.G4);
     g.b1 = take(g.NC1P);
+    g.wpart1 = o;
+    g.wa = take((long)A * g.G4);
     g.w2 = take((long)H * g.NC2P);
     g.b2 = take(g.NC2P);
+    g.wend = o;
     g.xt = take(2L * g.KX * XS);
     g.lg = take((long)g.AP * XS);
     g.g1 = take((long)EB * g.G4);
@@ -144,8 +147,10 @@ struct SmallParams {
     int sigma_sqrt_tau, done_terminates, noop_terminates;
     int shaped;
     float alpha, beta, invalid_reward;
-    // weights in the stepwise family's layouts (wm_internal.h)
-    const float *Wg, *Wa, *bg, *Wh, *bh;
+    // this model's per-rank weight images (the shared-memory layout of [0, wend)), one per
+    // cluster rank, img_stride bytes apart
+    const unsigned char *img;
+    size_t img_stride;
     // rollout
     const float *z0, *h0, *c0;
     const uint8_t *done0;
@@ -176,41 +181,10 @@ __device__ __forceinline__ double ld_cluster_f64(uint32_t caddr) {
 __device__ __forceinline__ void cp4(void *dst, const void *src) {
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" :: "r"(tc::smem_u32(dst)), "l"(src) : "memory");
 }
-__device__ __forceinline__ void cp16(void *dst, const void *src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(tc::smem_u32(dst)), "l"(src) : "memory");
-}
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 // waits until at most N of this thread's committed groups are still in flight
 template <int N>
 __device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory"); }
-
-// dst[k * ldd + c] = src[k * lds + col(c)] for rows k < R and columns c < ldd (0 where
-// col(c) < 0), as asynchronous copies: 16 bytes where four columns are contiguous and aligned
-// in the source, else 4.  Lanes take column groups (their maps computed once), warps rows.
-template <class ColFn>
-__device__ __forceinline__ void load_cols(float *dst, int ldd, const float *src, int lds, int R, ColFn col) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    for (int c0 = 4 * lane; c0 < ldd; c0 += 128) {
-        int cl[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) cl[q] = col(c0 + q);
-        const bool vec = cl[0] >= 0 && (cl[0] & 3) == 0 && (lds & 3) == 0 && cl[1] == cl[0] + 1 &&
-                         cl[2] == cl[0] + 2 && cl[3] == cl[0] + 3;
-        for (int k = warp; k < R; k += nw) {
-            float *d = dst + (size_t)k * ldd + c0;
-            const float *sr = src + (size_t)k * lds;
-            if (vec) {
-                cp16(d, sr + cl[0]);
-            } else {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    if (cl[q] >= 0) cp4(d + q, sr + cl[q]);
-                    else d[q] = 0.f;
-                }
-            }
-        }
-    }
-}
 
 // The gate nonlinearities from the exponential: sigma(x) = 1 / (1 + e^-x), tanh(x) =
 // 2 sigma(2x) - 1.  With the exp2-based exponential (relative error ~1e-7 at the gates'
@@ -249,9 +223,13 @@ __device__ __forceinline__ void step_sync(int CL) {
     else __syncthreads();
 }
 
-// Copies n4 16-byte words at src (this CTA's shared memory) to the same offset in every
-// other CTA of the cluster.
-__device__ __forceinline__ void to_peers(const float *src, int n4, int CL, int r) {
+constexpr uint32_t WAIT_POLLS = 1u << 26;  // bound of every wait on a peer's data
+
+// Copies n4 16-byte words at src (this CTA's shared memory) to the same offset in every other
+// CTA of the cluster with st.async: each store counts its 16 bytes on the receiver's mbarrier
+// `mbar` (the same offset in every CTA), so that the receiver waits for the bytes, not on a
+// cluster-wide barrier, and the sender issues no fence.
+__device__ __forceinline__ void to_peers(const float *src, int n4, int CL, int r, uint32_t mbar) {
     if (CL <= 1 || n4 <= 0) return;
     const uint32_t sa = tc::smem_u32(src);
     const int tot = n4 * (CL - 1);
@@ -260,8 +238,44 @@ __device__ __forceinline__ void to_peers(const float *src, int n4, int CL, int r
         const int j = i - q * n4;
         q += q >= r;
         const uint4 v = reinterpret_cast<const uint4 *>(src)[j];
-        tc::st_cluster_v4(tc::map_rank(sa + 16u * (uint32_t)j, (uint32_t)q), v);
+        const uint32_t dst = tc::map_rank(sa + 16u * (uint32_t)j, (uint32_t)q), mb = tc::map_rank(mbar, (uint32_t)q);
+        asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];"
+                     :: "r"(dst), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(mb) : "memory");
     }
+}
+
+// Waits (bounded) until phase `parity` of this CTA's mbarrier completes (the bulk copies it
+// counts have landed); thread 0 polls, the CTA barrier hands data and outcome to every thread.
+__device__ __forceinline__ bool wait_local(uint32_t mbar, uint32_t parity, int *flag) {
+    if (threadIdx.x == 0) *flag = tc::mbar_wait_bounded(mbar, parity, WAIT_POLLS) ? 1 : 0;
+    __syncthreads();
+    return *flag != 0;
+}
+
+// Waits (bounded) until phase `parity` of this CTA's mbarrier completes, i.e. every peer's
+// bytes of this exchange have landed.  Thread 0 polls with cluster-scope acquire; the CTA
+// barrier then hands the data, and the outcome, to every thread.  Returns false on expiry
+// (the same answer in every thread).
+__device__ __forceinline__ bool wait_peers(int CL, uint32_t mbar, uint32_t parity, int *flag) {
+    if (CL <= 1) {
+        __syncthreads();
+        return true;
+    }
+    if (threadIdx.x == 0) {
+        bool ok = false;
+        for (uint32_t i = 0; i < WAIT_POLLS && !ok; ++i) {
+            uint32_t done;
+            asm volatile(
+                "{\n\t.reg .pred p;\n\t"
+                "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+                "selp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(done) : "r"(mbar), "r"(parity) : "memory");
+            ok = done != 0;
+        }
+        *flag = ok ? 1 : 0;
+    }
+    __syncthreads();
+    return *flag != 0;
 }
 
 // One butterfly level over the lanes xor `o` of a group: the lane with bit o set keeps the
@@ -286,15 +300,16 @@ struct Fold {
 
 // The 4 x 4 tile (episodes e0 .. e0+3, columns c0 .. c0+3) of sum_k X^T[k][e] W[k][c],
 // k < K, on a group of S lanes (lane s takes k = s, s + S, ...), reduced over the group by a
-// butterfly: lane s returns in v[j] the sum of output Fold<S>::out(s, j), o = 4 i + jj
+// butterfly: lane s returns as value j the sum of output Fold<S>::out(s, j), o = 4 i + jj
 // meaning episode e0 + i, column c0 + jj (with S = 32 both lanes of a pair hold it).  Every
 // lane of the warp must call it (the reduction shuffles); lanes with on = false contribute
 // zeros.  Each output's sum is formed in the same order whatever the tile's position, so an
 // episode's results do not depend on the batch it is in.  The products are paired into
-// f32x2 FMAs (two fp32 FMAs, each rounded once, as fmaf).
+// f32x2 FMAs (two fp32 FMAs, each rounded once, as fmaf).  Out of line: both products call
+// the one copy, which keeps the step's code within the instruction cache.
 template <int S, int XS>
-__device__ __forceinline__ void tile_dot(const float *__restrict__ xt, const float *__restrict__ w, int ldw,
-                                         int K, int e0, int c0, int s, bool on, float *v) {
+__device__ __noinline__ float2 tile_dot(const float *__restrict__ xt, const float *__restrict__ w, int ldw, int K,
+                                        int e0, int c0, int s, bool on) {
     unsigned long long acc2[8];  // (episode pair, column): acc2[2 c + p] = episodes e0 + 2p, e0 + 2p + 1
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc2[j] = 0ull;
@@ -343,8 +358,7 @@ __device__ __forceinline__ void tile_dot(const float *__restrict__ xt, const flo
         fold<4>(acc, (s & 2) != 0, 2);
         fold<2>(acc, (s & 1) != 0, 1);
     }
-#pragma unroll
-    for (int j = 0; j < Fold<S>::NV; ++j) v[j] = acc[j];
+    return make_float2(acc[0], Fold<S>::NV > 1 ? acc[1] : 0.f);
 }
 
 // Global column of step.Wg [Z+H, 4H+A] behind local column c of W1 (-1: padding).
@@ -373,6 +387,43 @@ __device__ __forceinline__ int col2(const Geo &g, int c, int r, int Z, int K, in
 
 __device__ __forceinline__ int clampi(int x, int lo, int hi) { return x < lo ? lo : (x > hi ? hi : x); }
 
+// The tempered draw of the controller (Sec. 3.4) for one episode, on a full warp: the logits
+// col[j * ld] are copied into the contiguous row `row`, then the shared warp selection draws.
+__device__ __noinline__ int select_sampled(const float *col, int ld, float *row, int A, const uint32_t *mw,
+                                           float tau, unsigned long long seed, unsigned long long episode,
+                                           uint32_t step) {
+    const int lane = threadIdx.x & 31;
+    for (int j = lane; j < A; j += 32) row[j] = col[j * ld];
+    __syncwarp();
+    WarpSelect ws;
+    ws.sample = true;
+    ws.tau = tau;
+    ws.want_lp = false;
+    ws.seed = seed;
+    ws.episode = episode;
+    ws.step = step;
+    float lp;
+    return warp_select(ws, row, A, mw, 0, &lp);
+}
+
+// -log sum_k pi_k N(x; mu_k, sigma_k) of one latent dim on a full warp, lane k holding
+// component k's logit lgv, mean muv and log sigma lsv (lanes >= K: lgv = -inf): pi the softmax
+// of the logits, log sigma used directly, a log-sum-exp over the logits and one over the
+// components (a9, the loss of Sec. 4.7).
+__device__ __noinline__ float nll_dim(float lgv, float muv, float lsv, float x, bool kv) {
+    const float m = warp_max(lgv);
+    const float lse = m + logf(warp_sum(kv ? expf(lgv - m) : 0.f));
+    const float zk = (x - muv) * expf(-lsv);
+    const float lp = kv ? (lgv - lse) - 0.5f * zk * zk - lsv - 0.91893853320467274178f : -INFINITY;
+    const float tmax = warp_max(lp);
+    return -(tmax + logf(warp_sum(kv ? expf(lp - tmax) : 0.f)));
+}
+
+// The step's Philox numbers of one latent dim: the component uniform and the Gaussian draw.
+__device__ __noinline__ float2 draw_dim(unsigned long long seed, unsigned long long ep, uint32_t step, int d) {
+    return make_float2(uniform_for_dim(seed, ep, step, d), normal_for_dim(seed, ep, step, d));
+}
+
 template <int EB>
 __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant__ SmallParams p) {
     using TL = Tile<EB>;
@@ -385,29 +436,44 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
     const int Z = p.Z, A = p.A, H = p.H, K = p.K, KX = g.KX, U = g.U, G4 = g.G4, DZ = g.DZ, W = g.W;
     const int u0 = r * U, a0 = r * g.AC, d0 = r * DZ;
     const int nu = clampi(H - u0, 0, U), na = clampi(A - a0, 0, g.AC), nd = clampi(Z - d0, 0, DZ);
-    const int B = p.B, T = p.T, M = p.M, KZ = K * Z, ldg = 4 * H + A, ldh = M + p.NR;
+    const int B = p.B, T = p.T, M = p.M, KZ = K * Z;
     const bool teacher = p.teacher != 0, draw = !teacher && p.mdn_tau > 0.f;
     float *w1 = sm + g.w1, *wa = sm + g.wa, *b1 = sm + g.b1, *w2 = sm + g.w2, *b2 = sm + g.b2;
     float *xt = sm + g.xt, *lg = sm + g.lg, *g1 = sm + g.g1, *hd = sm + g.hd;
     float *cs = sm + g.cs, *hs = sm + g.hs, *zs = sm + g.zs, *nl = sm + g.nl, *sc = sm + g.sc;
     float *pu = sm + g.pu, *pe = sm + g.pe;
     uint32_t *mk = reinterpret_cast<uint32_t *>(sm + g.mk);
+    // the three exchanges' mbarriers (logits, h', z') and the wait outcome word
+    __shared__ __align__(8) unsigned long long xbar[3];
+    __shared__ int wflag;
+    const uint32_t MB_LG = tc::smem_u32(&xbar[0]), MB_H = tc::smem_u32(&xbar[1]), MB_Z = tc::smem_u32(&xbar[2]);
     int *act = reinterpret_cast<int *>(sm + g.ep), *frz = act + EB, *frzn = act + 2 * EB, *len = act + 3 * EB;
     float *rts = sm + g.ep + 4 * EB, *mems = rts + EB;
     double *nacc = reinterpret_cast<double *>(sm + g.ep + 6 * EB);  // 8-byte aligned: g.ep % 4 == 0
     auto rnd = [&](float v) { return p.round ? round_bf16(v) : v; };
     const int nsd = EB * DZ;  // (episode, dim) items of the rank
 
-    // ---- weights of this CTA's columns (once per call): asynchronous copies, all in flight at
-    // once; group 0 holds W1 and b1 (the first product's), group 1 the rest (needed later)
-    load_cols(w1, g.NC1P, p.Wg, ldg, KX, [&](int c) { return col1(g, c, r, H, A); });
-    load_cols(b1, g.NC1P, p.bg, 0, 1, [&](int c) { return col1(g, c, r, H, A); });
-    cp_commit();
-    load_cols(wa, G4, p.Wa, 4 * H, A, [&](int c) { return col1(g, c, r, H, A); });
-    load_cols(w2, g.NC2P, p.Wh, ldh, H, [&](int c) { return col2(g, c, r, Z, K, M); });
-    load_cols(b2, g.NC2P, p.bh, 0, 1, [&](int c) { return col2(g, c, r, Z, K, M); });
-    cp_commit();
-    // step 0's mask words (group 2); step t + 1's are fetched during step t
+    // ---- weights of this CTA's columns (once per call): the rank's packed image, by bulk copies
+    // on the TMA engine; part 0 (W1, b1) is waited for before the first product, part 1 (W_a,
+    // W2, b2) before the first cell
+    __shared__ __align__(8) unsigned long long wbar[2];
+    if (tid == 0) {
+        tc::mbar_init(tc::smem_u32(&wbar[0]), 1);
+        tc::mbar_init(tc::smem_u32(&wbar[1]), 1);
+        tc::fence_mbar_init();
+        const unsigned char *src = p.img + (size_t)r * p.img_stride;
+        const uint32_t base = tc::smem_u32(sm);
+        const uint32_t lim[3] = {0u, (uint32_t)g.wpart1 * 4u, (uint32_t)g.wend * 4u};
+        for (int part = 0; part < 2; ++part) {
+            const uint32_t mb = tc::smem_u32(&wbar[part]);
+            tc::mbar_arrive_expect_tx(mb, lim[part + 1] - lim[part]);
+            for (uint32_t off = lim[part]; off < lim[part + 1]; off += 32768u) {
+                const uint32_t n = lim[part + 1] - off < 32768u ? lim[part + 1] - off : 32768u;
+                tc::bulk_load_global(base + off, src + off, n, mb);
+            }
+        }
+    }
+    // step 0's mask words; step t + 1's are fetched during step t
     if (!teacher && p.mask && T > 0)
         for (int i = tid; i < EB * W; i += nt) {
             const int e = i / W;
@@ -455,7 +521,19 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         mems[e] = p.shaped && e < nv ? p.mem0[b] : 0.f;
         nacc[e] = 0.0;
     }
-    cp_wait<2>();  // this thread's W1 copies have landed (the barriers below publish them)
+    cp_wait<0>();  // step 0's mask words have landed (the barriers below publish them)
+    // bytes each exchange brings from the peers (their slices differ at ragged edges)
+    uint32_t in_lg = 0, in_h = 0, in_z = 0;
+    for (int q = 0; q < CL; ++q)
+        if (q != r) {
+            in_lg += (uint32_t)clampi(A - q * g.AC, 0, g.AC) * XS * 4;
+            in_h += (uint32_t)clampi(H - q * U, 0, U) * XS * 4;
+            in_z += (uint32_t)clampi(Z - q * DZ, 0, DZ) * XS * 4;
+        }
+    if (tid == 0) {
+        for (int i = 0; i < 3; ++i) tc::mbar_init(tc::smem_u32(&xbar[i]), 1);
+        tc::fence_mbar_init();
+    }
     // the injected wait: a barrier nothing completes, polled at most test_wait times; every
     // CTA gives up the same way, so the abort is uniform across the cluster
     bool abort = false;
@@ -473,13 +551,26 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         }
         abort = true;
     }
-    __syncthreads();
-    step_sync(CL);  // every CTA of the cluster is running and initialised
+    bool w_rest = false;  // whether the second weight part has been waited for
+    if (!wait_local(tc::smem_u32(&wbar[0]), 0, &wflag)) {  // W1, b1
+        if (tid == 0) report_status(p.status, WM_ERR_TIMEOUT);
+        abort = true;
+    }
+    step_sync(CL);  // every CTA of the cluster is running, its mbarriers initialised
 
     const int CG1 = (g.NC1 + 3) / 4, CG2 = (g.NC2 + 3) / 4;
     for (int t = 0; t < T && !abort; ++t) {
         float *xc = xt + (t & 1) * KX * XS, *xn = xt + ((t + 1) & 1) * KX * XS;
         const uint32_t step = p.t0 + (uint32_t)t;
+        // this step's incoming bytes on each exchange's mbarrier (phase t); every peer's bytes of
+        // phase t - 1 have been waited for, and a peer sends phase t's only after this CTA's
+        // own sends of phase t - 1, so no phase can receive early
+        const bool zx = t + 1 < T;  // the last step sends no z'
+        if (tid == 0 && CL > 1) {
+            tc::mbar_arrive_expect_tx(MB_LG, in_lg);
+            tc::mbar_arrive_expect_tx(MB_H, in_h);
+            if (zx) tc::mbar_arrive_expect_tx(MB_Z, in_z);
+        }
         // the next step's mask words, in flight for a whole step (double buffer)
         uint32_t *mkc = mk + (t & 1) * EB * W;
         if (!teacher && p.mask && t + 1 < T) {
@@ -497,8 +588,8 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 const int ti = base + gid;
                 const bool on = ti < tiles;
                 const int eg = on ? ti % EG : 0, cg = on ? ti / EG : 0;
-                float v[Fold<S1>::NV];
-                tile_dot<S1, XS>(xc, w1, g.NC1P, KX, 4 * eg, 4 * cg, s, on, v);
+                const float2 v2 = tile_dot<S1, XS>(xc, w1, g.NC1P, KX, 4 * eg, 4 * cg, s, on);
+                const float v[2] = {v2.x, v2.y};
                 if (on && Fold<S1>::writer(s)) {
 #pragma unroll
                     for (int j = 0; j < Fold<S1>::NV; ++j) {
@@ -510,11 +601,15 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 }
             }
         }
-        cp_wait<1>();  // all but the newest group: this step's mask words (and, at t = 0, the weights)
+        cp_wait<1>();  // all but the newest group: this step's mask words
         __syncthreads();
         // 2. the rank's logit rows to every CTA
-        to_peers(lg + a0 * XS, na * XS / 4, CL, r);
-        step_sync(CL);
+        to_peers(lg + a0 * XS, na * XS / 4, CL, r, MB_LG);
+        if (!wait_peers(CL, MB_LG, t & 1, &wflag)) {
+            if (tid == 0) report_status(p.status, WM_ERR_TIMEOUT);
+            abort = true;
+            break;
+        }
         // 3. the action of each episode (a2), the same in every CTA
         if (warp < EB) {
             const int e = warp;
@@ -541,18 +636,8 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                     warp_argmax(bv, bi);
                     a = bi;
                 } else {
-                    float *row = sc + e * g.AP;
-                    for (int j = lane; j < A; j += 32) row[j] = lg[j * XS + e];
-                    __syncwarp();
-                    WarpSelect ws;
-                    ws.sample = true;
-                    ws.tau = p.ctrl_tau;
-                    ws.want_lp = false;
-                    ws.seed = p.seed;
-                    ws.episode = p.ep0 + b;
-                    ws.step = step;
-                    float lp;
-                    a = warp_select(ws, row, A, p.mask ? mkc + e * W : nullptr, 0, &lp);
+                    a = select_sampled(lg + e, XS, sc + e * g.AP, A, p.mask ? mkc + e * W : nullptr, p.ctrl_tau,
+                                       p.seed, p.ep0 + b, step);
                 }
             }
             if (lane == 0) {
@@ -560,7 +645,16 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 if (!teacher && r == 0 && e < nv) p.actions[(size_t)t * B + b] = a;
             }
         }
-        __syncthreads();
+        if (t == 0) {  // the rest of the weights (W_a, W2, b2)
+            w_rest = true;
+            if (!wait_local(tc::smem_u32(&wbar[1]), 0, &wflag)) {
+                if (tid == 0) report_status(p.status, WM_ERR_TIMEOUT);
+                abort = true;
+                break;
+            }
+        } else {
+            __syncthreads();
+        }
         // 4. the cell for the rank's units (a3, a4); h' into every CTA's next frame.  Threads
         // past the cell's draw the step's Philox numbers for the rank's dims meanwhile.
         for (int i = tid; i < EB * U; i += nt) {
@@ -594,12 +688,17 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
             for (int i = nt - 1 - tid; i >= 0 && i < nsd; i += nt) {
                 const int e = i / DZ, d = d0 + (i - e * DZ);
                 if (e >= nv || d >= Z || frz[e]) continue;
-                pu[i] = uniform_for_dim(p.seed, p.ep0 + b0 + e, step, d);
-                pe[i] = normal_for_dim(p.seed, p.ep0 + b0 + e, step, d);
+                const float2 ue = draw_dim(p.seed, p.ep0 + b0 + e, step, d);
+                pu[i] = ue.x;
+                pe[i] = ue.y;
             }
         __syncthreads();
-        to_peers(xn + (Z + u0) * XS, nu * XS / 4, CL, r);
-        step_sync(CL);
+        to_peers(xn + (Z + u0) * XS, nu * XS / 4, CL, r, MB_H);
+        if (!wait_peers(CL, MB_H, t & 1, &wflag)) {
+            if (tid == 0) report_status(p.status, WM_ERR_TIMEOUT);
+            abort = true;
+            break;
+        }
         // 5. the rank's head columns (a5)
         {
             const int ng = nt / S2, tiles = EG * CG2, gid = tid / S2, s = tid % S2;
@@ -607,8 +706,8 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 const int ti = base + gid;
                 const bool on = ti < tiles;
                 const int eg = on ? ti % EG : 0, cg = on ? ti / EG : 0;
-                float v[Fold<S2>::NV];
-                tile_dot<S2, XS>(xn + Z * XS, w2, g.NC2P, H, 4 * eg, 4 * cg, s, on, v);
+                const float2 v2 = tile_dot<S2, XS>(xn + Z * XS, w2, g.NC2P, H, 4 * eg, 4 * cg, s, on);
+                const float v[2] = {v2.x, v2.y};
                 if (on && Fold<S2>::writer(s)) {
 #pragma unroll
                     for (int j = 0; j < Fold<S2>::NV; ++j) {
@@ -642,17 +741,10 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 ms[2 * KZ + d * K + lane] = fz ? 0.f : lsv;
             }
             if (teacher) {
-                // -log sum_k pi_k N(x; mu_k, sigma_k): pi the softmax of the logits, log sigma
-                // direct, a log-sum-exp over the logits and one over the components
                 const float x = p.z_seq[((size_t)(t + 1) * B + b) * Z + d];
-                const float m = warp_max(lgv);
-                const float lse = m + logf(warp_sum(kv ? expf(lgv - m) : 0.f));
-                const float zk = (x - muv) * expf(-lsv);
-                const float lp = kv ? (lgv - lse) - 0.5f * zk * zk - lsv - 0.91893853320467274178f : -INFINITY;
-                const float tmax = warp_max(lp);
-                const float acc = warp_sum(kv ? expf(lp - tmax) : 0.f);
+                const float nll = nll_dim(lgv, muv, lsv, x, kv);
                 if (lane == 0) {
-                    nl[it] = -(tmax + logf(acc));
+                    nl[it] = nll;
                     xn[d * XS + e] = rnd(x);
                 }
                 continue;
@@ -740,11 +832,22 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 frz[e] = frzn[e];
             }
         }
-        to_peers(xn + d0 * XS, nd * XS / 4, CL, r);
-        step_sync(CL);
+        if (zx) {
+            to_peers(xn + d0 * XS, nd * XS / 4, CL, r, MB_Z);
+            if (!wait_peers(CL, MB_Z, t & 1, &wflag)) {
+                if (tid == 0) report_status(p.status, WM_ERR_TIMEOUT);
+                abort = true;
+                break;
+            }
+        }
     }
 
-    // ---- end of the call
+    // ---- end of the call.  Nothing of this CTA's may still be in flight into its shared memory:
+    // the second weight part (if no step waited for it) and the mask prefetches.
+    if (!w_rest) wait_local(tc::smem_u32(&wbar[1]), 0, &wflag);
+    cp_wait<0>();
+    // every CTA's last writes (the NLL partials) are visible cluster-wide
+    step_sync(CL);
     if (!abort && !teacher)
         for (int i = tid; i < EB * U; i += nt) {
             const int e = i / U, u = u0 + (i - e * U);
@@ -761,6 +864,35 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         p.nll[(size_t)b0 + tid] = (float)s;
     }
     step_sync(CL);  // no CTA leaves while a peer may still read its shared memory
+}
+
+// Packs rank blockIdx.x's weight image: the shared-memory layout [0, wend) of Geo, from the
+// stepwise family's weights (zeros in the padding columns).
+__global__ void k_small_pack(const Geo g, int Z, int A, int H, int K, int M, int NR, const float *__restrict__ Wg,
+                             const float *__restrict__ Wa, const float *__restrict__ bg, const float *__restrict__ Wh,
+                             const float *__restrict__ bh, float *img, size_t stride) {
+    const int r = blockIdx.x, ldg = 4 * H + A, ldh = M + NR;
+    float *o = img + (size_t)r * stride;
+    for (int i = threadIdx.x; i < g.KX * g.NC1P; i += blockDim.x) {
+        const int k = i / g.NC1P, col = col1(g, i - k * g.NC1P, r, H, A);
+        o[g.w1 + i] = col >= 0 ? Wg[(size_t)k * ldg + col] : 0.f;
+    }
+    for (int c = threadIdx.x; c < g.NC1P; c += blockDim.x) {
+        const int col = col1(g, c, r, H, A);
+        o[g.b1 + c] = col >= 0 ? bg[col] : 0.f;
+    }
+    for (int i = threadIdx.x; i < A * g.G4; i += blockDim.x) {
+        const int a = i / g.G4, col = col1(g, i - a * g.G4, r, H, A);
+        o[g.wa + i] = col >= 0 ? Wa[(size_t)a * 4 * H + col] : 0.f;
+    }
+    for (int i = threadIdx.x; i < H * g.NC2P; i += blockDim.x) {
+        const int k = i / g.NC2P, col = col2(g, i - k * g.NC2P, r, Z, K, M);
+        o[g.w2 + i] = col >= 0 ? Wh[(size_t)k * ldh + col] : 0.f;
+    }
+    for (int c = threadIdx.x; c < g.NC2P; c += blockDim.x) {
+        const int col = col2(g, c, r, Z, K, M);
+        o[g.b2 + c] = col >= 0 ? bh[col] : 0.f;
+    }
 }
 
 __global__ void k_small_copy(size_t n, const float *src, float *dst) {
@@ -841,7 +973,8 @@ SmallParams base(const wm_handle *h, int B, int T, int slot) {
     p.noop_terminates = c.noop_terminates;
     p.shaped = c.reward_mode == WM_REWARD_SHAPED;
     p.alpha = c.reward_alpha; p.beta = c.reward_beta; p.invalid_reward = c.invalid_reward;
-    p.Wg = h->step.Wg; p.Wa = h->step.Wa; p.bg = h->step.bg; p.Wh = h->step.Wh; p.bh = h->step.bh;
+    p.img = (const unsigned char *)h->small.img;
+    p.img_stride = h->small.img_stride;
     p.status = h->status;
     p.test_wait = h->test_wait;
     h->test_wait = 0;
@@ -908,8 +1041,29 @@ cudaError_t wm_small_prepare(wm_handle *h) {
         h->small.max_clusters_eb[i] = n[i];
     }
     h->small.cl = best.CL;
+    h->small.img_stride = ((size_t)best.wend * 4 + 255) & ~(size_t)255;
+    cudaError_t e = cudaMalloc(&h->small.img, h->small.img_stride * best.CL);
+    if (e != cudaSuccess) return e;
+    if ((e = wm_small_repack(h)) != cudaSuccess) return e;
     h->small.ok = 1;
     return cudaSuccess;
+}
+
+cudaError_t wm_small_repack(wm_handle *h) {
+    if (!h->small.img) return cudaSuccess;
+    const wm_config &c = h->cfg;
+    Geo g;
+    memcpy(&g, h->small.geo[0], sizeof(Geo));
+    k_small_pack<<<g.CL, 256>>>(g, c.z_dim, c.a_dim, c.h_dim, c.k_mix, h->M, h->NR, h->step.Wg, h->step.Wa,
+                                h->step.bg, h->step.Wh, h->step.bh, (float *)h->small.img, h->small.img_stride / 4);
+    cudaError_t e = cudaGetLastError();
+    return e != cudaSuccess ? e : cudaDeviceSynchronize();
+}
+
+void wm_small_free(wm_handle *h) {
+    cudaFree(h->small.img);
+    h->small.img = nullptr;
+    h->small.ok = 0;
 }
 
 int wm_small_supported(const wm_handle *h, int B) {
