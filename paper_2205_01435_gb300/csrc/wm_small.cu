@@ -33,6 +33,7 @@
 //      rows go to every CTA's next frame; cluster barrier
 // Every thread of every CTA runs the same sequence of cluster barriers, and the kernel
 // has no other waits but the injected test wait (bounded), so it cannot hang on a peer.
+#include <limits.h>
 #include <math.h>
 #include <string.h>
 
@@ -114,8 +115,8 @@ Geo geometry(int Z, int A, int H, int K, int NR, int CL, int EB, int XS, int S1,
     g.hs = take((long)EB * g.U);
     g.zs = take((long)EB * g.DZ);
     g.nl = take((long)EB * g.DZ);
-    g.pu = take((long)EB * g.DZ);
-    g.pe = take((long)EB * g.DZ);
+    g.pu = take(2L * EB * g.DZ);  // the step's Philox uniforms and normals, two steps (double buffer)
+    g.pe = take(2L * EB * g.DZ);
     g.mk = take(2L * EB * g.W);  // two steps' mask words (double buffer)
     g.sc = take((long)EB * g.AP);
     g.ep = take(8L * EB);  // act, frozen, frozen next, length (int); rt, mem; NLL (double)
@@ -144,6 +145,7 @@ struct SmallParams {
     uint32_t t0;
     int ctrl_sample;
     float ctrl_tau, mdn_tau;
+    float inv_tau, sigma_scale;  // 1 / mdn_tau; sqrt(mdn_tau) with sigma_sqrt_tau, else 1
     int sigma_sqrt_tau, done_terminates, noop_terminates;
     int shaped;
     float alpha, beta, invalid_reward;
@@ -203,18 +205,19 @@ __device__ __forceinline__ float warp_sum(float v) {
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
-// (value, index) argmax over the lanes, lowest index on ties; index -1 means none
-__device__ __forceinline__ void warp_argmax(float &v, int &i) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-        if (oi >= 0 && (i < 0 || ov > v || (ov == v && oi < i))) {
-            v = ov;
-            i = oi;
-        }
-    }
+// A signed-integer key with the order of the float (for the warp's integer max reduction).
+__device__ __forceinline__ int ord_key(float v) {
+    const int i = __float_as_int(v);
+    return i >= 0 ? i : i ^ 0x7fffffff;
 }
+
+// Index of the largest of the lanes' keys (lowest index on ties) by two warp reductions;
+// idx = INT_MAX: the lane has none.  Returns INT_MAX if no lane has one.
+__device__ __forceinline__ int redux_argmax(int key, int idx) {
+    const int kmax = __reduce_max_sync(0xffffffffu, idx != INT_MAX ? key : INT_MIN);
+    return __reduce_min_sync(0xffffffffu, (idx != INT_MAX && key == kmax) ? idx : INT_MAX);
+}
+
 
 // The cluster barrier (release / acquire: the DSMEM stores before it are visible after it),
 // or the CTA barrier for a cluster of one.
@@ -452,6 +455,8 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
     double *nacc = reinterpret_cast<double *>(sm + g.ep + 6 * EB);  // 8-byte aligned: g.ep % 4 == 0
     auto rnd = [&](float v) { return p.round ? round_bf16(v) : v; };
     const int nsd = EB * DZ;  // (episode, dim) items of the rank
+    int KP = 1;               // lanes of the mixture reductions: K rounded up to a power of 2
+    while (KP < K) KP <<= 1;
 
     // ---- weights of this CTA's columns (once per call): the rank's packed image, by bulk copies
     // on the TMA engine; part 0 (W1, b1) is waited for before the first product, part 1 (W_a,
@@ -473,6 +478,15 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
             }
         }
     }
+    // step 0's Philox numbers (step t + 1's are drawn during step t's sampling)
+    if (draw && T > 0)
+        for (int i = tid; i < nsd; i += nt) {
+            const int e = i / DZ, d = d0 + (i - e * DZ);
+            if (e >= nv || d >= Z) continue;
+            const float2 ue = draw_dim(p.seed, p.ep0 + b0 + e, p.t0, d);
+            pu[i] = ue.x;
+            pe[i] = ue.y;
+        }
     // step 0's mask words; step t + 1's are fetched during step t
     if (!teacher && p.mask && T > 0)
         for (int i = tid; i < EB * W; i += nt) {
@@ -623,18 +637,17 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 } else if (!(p.ctrl_sample && p.ctrl_tau > 0.f)) {
                     // masked argmax, lowest index on ties
                     const uint32_t *mw = p.mask ? mkc + e * W : nullptr;
-                    float bv = -INFINITY;
-                    int bi = -1;
+                    int key = INT_MIN, bj = INT_MAX;
                     for (int j = lane; j < A; j += 32) {
                         if (mw && !((mw[j >> 5] >> (j & 31)) & 1u)) continue;
-                        const float v = lg[j * XS + e];
-                        if (bi < 0 || v > bv) {
-                            bv = v;
-                            bi = j;
+                        const int k = ord_key(lg[j * XS + e]);
+                        if (bj == INT_MAX || k > key) {
+                            key = k;
+                            bj = j;
                         }
                     }
-                    warp_argmax(bv, bi);
-                    a = bi;
+                    const int am = redux_argmax(key, bj);
+                    a = am == INT_MAX ? -1 : am;
                 } else {
                     a = select_sampled(lg + e, XS, sc + e * g.AP, A, p.mask ? mkc + e * W : nullptr, p.ctrl_tau,
                                        p.seed, p.ep0 + b, step);
@@ -655,8 +668,7 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         } else {
             __syncthreads();
         }
-        // 4. the cell for the rank's units (a3, a4); h' into every CTA's next frame.  Threads
-        // past the cell's draw the step's Philox numbers for the rank's dims meanwhile.
+        // 4. the cell for the rank's units (a3, a4); h' into every CTA's next frame
         for (int i = tid; i < EB * U; i += nt) {
             const int e = i / U, uu = i - e * U, u = u0 + uu;
             if (u >= H) continue;
@@ -684,14 +696,6 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 if (p.c_seq) p.c_seq[o] = cv;
             }
         }
-        if (draw)
-            for (int i = nt - 1 - tid; i >= 0 && i < nsd; i += nt) {
-                const int e = i / DZ, d = d0 + (i - e * DZ);
-                if (e >= nv || d >= Z || frz[e]) continue;
-                const float2 ue = draw_dim(p.seed, p.ep0 + b0 + e, step, d);
-                pu[i] = ue.x;
-                pe[i] = ue.y;
-            }
         __syncthreads();
         to_peers(xn + (Z + u0) * XS, nu * XS / 4, CL, r, MB_H);
         if (!wait_peers(CL, MB_H, t & 1, &wflag)) {
@@ -721,6 +725,16 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         // 6. the rank's dims: the next latent (a6, a7) or the NLL (a9); z' into the next frame.
         // One warp per (episode, dim) item, lane k holding mixture component k (K <= 32).
         const int KD = K * DZ, X0 = 3 * KD;
+        const float *puc = pu + (t & 1) * nsd, *pec = pe + (t & 1) * nsd;
+        // the next step's Philox numbers, on the warps past the items (counted from the top)
+        if (draw && t + 1 < T)
+            for (int i = nt - 1 - tid; i >= 0 && i < nsd; i += nt) {
+                const int e = i / DZ, d = d0 + (i - e * DZ);
+                if (e >= nv || d >= Z) continue;
+                const float2 ue = draw_dim(p.seed, p.ep0 + b0 + e, step + 1u, d);
+                pu[((t + 1) & 1) * nsd + i] = ue.x;
+                pe[((t + 1) & 1) * nsd + i] = ue.y;
+            }
         for (int it = warp; it < nsd; it += nw) {
             const int e = it / DZ, dd = it - e * DZ, d = d0 + dd;
             if (d >= Z) continue;
@@ -755,28 +769,27 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 z = zs[it];
                 kc = 255;
             } else if (!draw) {
-                float bv = lgv;
-                int bi = kv ? lane : -1;
-                warp_argmax(bv, bi);
-                kc = bi;
+                kc = redux_argmax(ord_key(lgv), kv ? lane : INT_MAX);  // lowest component on ties
                 z = __shfl_sync(0xffffffffu, muv, kc);
             } else {
-                // component by inverse CDF of softmax(logits / tau), then z ~ N(mu, sigma^2)
-                const float tau = p.mdn_tau;
-                const float q = kv ? lgv / tau : -INFINITY;
-                const float m = warp_max(q);
-                const float ev = kv ? expf(q - m) : 0.f;
-                float cum = ev / warp_sum(ev);
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
+                // component by inverse CDF of softmax(logits / tau): the first k < K - 1 whose
+                // cumulative weight exceeds u (u S against the unnormalised sums), then
+                // z ~ N(mu, sigma^2).  The reductions and the prefix sum run over the KP lanes
+                // of the components only.
+                const float q = kv ? lgv * p.inv_tau : -INFINITY;
+                float m = q;
+                for (int o = KP >> 1; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+                const float ev = kv ? __expf(q - m) : 0.f;
+                float S = ev, cum = ev;
+                for (int o = KP >> 1; o; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
+                for (int o = 1; o < KP; o <<= 1) {
                     const float up = __shfl_up_sync(0xffffffffu, cum, o);
                     if (lane >= o) cum += up;
                 }
-                const unsigned hit = __ballot_sync(0xffffffffu, lane < K - 1 && pu[it] < cum);
+                const unsigned hit = __ballot_sync(0xffffffffu, lane < K - 1 && puc[it] * S < cum);
                 kc = hit ? __ffs(hit) - 1 : K - 1;
                 const float mk_ = __shfl_sync(0xffffffffu, muv, kc), lk = __shfl_sync(0xffffffffu, lsv, kc);
-                const float scale = p.sigma_sqrt_tau ? sqrtf(tau) : 1.f;
-                z = mk_ + expf(lk) * scale * pe[it];
+                z = mk_ + __expf(lk) * p.sigma_scale * pec[it];
             }
             if (lane == 0) {
                 if (!fz) zs[it] = z;
@@ -969,6 +982,8 @@ SmallParams base(const wm_handle *h, int B, int T, int slot) {
     p.round = c.precision == WM_BF16;
     p.seed = c.seed;
     p.ctrl_sample = c.ctrl_sample; p.ctrl_tau = c.ctrl_tau; p.mdn_tau = c.mdn_tau;
+    p.inv_tau = c.mdn_tau > 0.f ? 1.f / c.mdn_tau : 0.f;
+    p.sigma_scale = c.sigma_sqrt_tau && c.mdn_tau > 0.f ? sqrtf(c.mdn_tau) : 1.f;
     p.sigma_sqrt_tau = c.sigma_sqrt_tau; p.done_terminates = c.done_terminates;
     p.noop_terminates = c.noop_terminates;
     p.shaped = c.reward_mode == WM_REWARD_SHAPED;
