@@ -94,29 +94,30 @@ struct WarpSelect {
 };
 
 // log pi(a) under softmax(l / tau) over the valid of n actions (every lane returns it)
-__device__ inline float warp_logp(const float *l, int n, const uint32_t *mw, int a, float lmax, float tau) {
+__device__ inline float warp_logp(const float *l, int n, const uint32_t *mw, int a, float lmax, float tau,
+                                  int ld = 1) {
     const int lane = threadIdx.x & 31;
     float S = 0.f;
     for (int j = lane; j < n; j += 32)
-        if (action_valid(mw, j)) S += expf((l[j] - lmax) / tau);
+        if (action_valid(mw, j)) S += expf((l[j * ld] - lmax) / tau);
 #pragma unroll
     for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
-    return (l[a] - lmax) / tau - logf(S);
+    return (l[a * ld] - lmax) / tau - logf(S);
 }
 
 // Masked argmax (lowest index on ties) or a tempered draw by inverse CDF with word `word` of
-// the controller's Philox block, over the n logits l with mask words mw (or null).  Returns
+// the controller's Philox block, over the n logits l[j * ld] with mask words mw (or null).  Returns
 // the choice (-1: nothing valid); with want_lp, *logp receives its log-prob under
 // softmax(l / tau) over the valid actions (0 if none, or tau = 0).  Called by a full warp.
 __device__ inline int warp_select(const WarpSelect &s, const float *l, int n, const uint32_t *mw, int word,
-                                  float *logp) {
+                                  float *logp, int ld = 1) {
     const int lane = threadIdx.x & 31;
     const int A = n;
     float bv = -INFINITY;
     int bi = -1;
     for (int j = lane; j < A; j += 32) {
         if (!action_valid(mw, j)) continue;
-        float v = l[j];
+        float v = l[j * ld];
         if (bi < 0 || v > bv) { bv = v; bi = j; }
     }
 #pragma unroll
@@ -129,13 +130,13 @@ __device__ inline int warp_select(const WarpSelect &s, const float *l, int n, co
     *logp = 0.f;
     if (bi < 0) return bi;
     if (!s.sample) {
-        if (s.want_lp && s.tau > 0.f) *logp = warp_logp(l, A, mw, bi, bv, s.tau);
+        if (s.want_lp && s.tau > 0.f) *logp = warp_logp(l, A, mw, bi, bv, s.tau, ld);
         return bi;
     }
     const float tau = s.tau;
     float S = 0.f;
     for (int j = lane; j < A; j += 32)
-        if (action_valid(mw, j)) S += expf((l[j] - bv) / tau);
+        if (action_valid(mw, j)) S += expf((l[j * ld] - bv) / tau);
 #pragma unroll
     for (int off = 16; off; off >>= 1) S += __shfl_xor_sync(0xffffffffu, S, off);
     const u32x4 rc = rng_draw(s.seed, s.episode, s.step, RNG_CONTROLLER, 0);
@@ -146,7 +147,7 @@ __device__ inline int warp_select(const WarpSelect &s, const float *l, int n, co
     for (int j0 = 0; j0 < A; j0 += 32) {
         int j = j0 + lane;
         bool ok = j < A && action_valid(mw, j);
-        float sc = ok ? expf((l[j] - bv) / tau) : 0.f;
+        float sc = ok ? expf((l[j * ld] - bv) / tau) : 0.f;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
             float o = __shfl_up_sync(0xffffffffu, sc, off);
@@ -158,12 +159,12 @@ __device__ inline int warp_select(const WarpSelect &s, const float *l, int n, co
         if (okm) last = j0 + 31 - __clz(okm);
         if (hit) {
             const int a = j0 + __ffs(hit) - 1;
-            if (s.want_lp) *logp = (l[a] - bv) / tau - logf(S);
+            if (s.want_lp) *logp = (l[a * ld] - bv) / tau - logf(S);
             return a;
         }
         run += __shfl_sync(0xffffffffu, sc, 31);
     }
-    if (s.want_lp && last >= 0) *logp = (l[last] - bv) / tau - logf(S);
+    if (s.want_lp && last >= 0) *logp = (l[last * ld] - bv) / tau - logf(S);
     return last;
 }
 

@@ -65,7 +65,7 @@ struct Tile {
 // Shared-memory geometry of one CTA (offsets in floats, each a multiple of 4).
 struct Geo {
     int EB, XS, CL, KX, U, AC, DZ, G4, NC1, NC1P, NC2, NC2P, AP, W, nthreads;
-    int w1, b1, wa, w2, b2, xt, lg, g1, hd, cs, hs, zs, nl, pu, pe, mk, sc, ep;
+    int w1, b1, wa, w2, b2, xt, lg, g1, hd, cs, hs, zs, nl, pu, pe, mk, ep;
     int wpart1, wend;  // the weight image: [0, wpart1) W1 and b1, [wpart1, wend) W_a, W2, b2
     size_t smem;
 };
@@ -118,7 +118,6 @@ Geo geometry(int Z, int A, int H, int K, int NR, int CL, int EB, int XS, int S1,
     g.pu = take(2L * EB * g.DZ);  // the step's Philox uniforms and normals, two steps (double buffer)
     g.pe = take(2L * EB * g.DZ);
     g.mk = take(2L * EB * g.W);  // two steps' mask words (double buffer)
-    g.sc = take((long)EB * g.AP);
     g.ep = take(8L * EB);  // act, frozen, frozen next, length (int); rt, mem; NLL (double)
     g.smem = (size_t)o * 4;
     const int eg = EB / 4;
@@ -390,14 +389,10 @@ __device__ __forceinline__ int col2(const Geo &g, int c, int r, int Z, int K, in
 
 __device__ __forceinline__ int clampi(int x, int lo, int hi) { return x < lo ? lo : (x > hi ? hi : x); }
 
-// The tempered draw of the controller (Sec. 3.4) for one episode, on a full warp: the logits
-// col[j * ld] are copied into the contiguous row `row`, then the shared warp selection draws.
-__device__ __noinline__ int select_sampled(const float *col, int ld, float *row, int A, const uint32_t *mw,
-                                           float tau, unsigned long long seed, unsigned long long episode,
-                                           uint32_t step) {
-    const int lane = threadIdx.x & 31;
-    for (int j = lane; j < A; j += 32) row[j] = col[j * ld];
-    __syncwarp();
+// The tempered draw of the controller (Sec. 3.4) for one episode, on a full warp, over the
+// logits col[j * ld] (the shared warp selection).
+__device__ __noinline__ int select_sampled(const float *col, int ld, int A, const uint32_t *mw, float tau,
+                                           unsigned long long seed, unsigned long long episode, uint32_t step) {
     WarpSelect ws;
     ws.sample = true;
     ws.tau = tau;
@@ -406,7 +401,7 @@ __device__ __noinline__ int select_sampled(const float *col, int ld, float *row,
     ws.episode = episode;
     ws.step = step;
     float lp;
-    return warp_select(ws, row, A, mw, 0, &lp);
+    return warp_select(ws, col, A, mw, 0, &lp, ld);
 }
 
 // -log sum_k pi_k N(x; mu_k, sigma_k) of one latent dim on a full warp, lane k holding
@@ -443,7 +438,7 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
     const bool teacher = p.teacher != 0, draw = !teacher && p.mdn_tau > 0.f;
     float *w1 = sm + g.w1, *wa = sm + g.wa, *b1 = sm + g.b1, *w2 = sm + g.w2, *b2 = sm + g.b2;
     float *xt = sm + g.xt, *lg = sm + g.lg, *g1 = sm + g.g1, *hd = sm + g.hd;
-    float *cs = sm + g.cs, *hs = sm + g.hs, *zs = sm + g.zs, *nl = sm + g.nl, *sc = sm + g.sc;
+    float *cs = sm + g.cs, *hs = sm + g.hs, *zs = sm + g.zs, *nl = sm + g.nl;
     float *pu = sm + g.pu, *pe = sm + g.pe;
     uint32_t *mk = reinterpret_cast<uint32_t *>(sm + g.mk);
     // the three exchanges' mbarriers (logits, h', z') and the wait outcome word
@@ -649,8 +644,8 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                     const int am = redux_argmax(key, bj);
                     a = am == INT_MAX ? -1 : am;
                 } else {
-                    a = select_sampled(lg + e, XS, sc + e * g.AP, A, p.mask ? mkc + e * W : nullptr, p.ctrl_tau,
-                                       p.seed, p.ep0 + b, step);
+                    a = select_sampled(lg + e, XS, A, p.mask ? mkc + e * W : nullptr, p.ctrl_tau, p.seed, p.ep0 + b,
+                                       step);
                 }
             }
             if (lane == 0) {
