@@ -542,6 +542,10 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
     if (tid == 0) {
         for (int i = 0; i < 3; ++i) tc::mbar_init(tc::smem_u32(&xbar[i]), 1);
         tc::fence_mbar_init();
+        if (CL > 1 && T > 0) {  // phase 0 of the logits and h' exchanges (z': in step 0)
+            tc::mbar_arrive_expect_tx(MB_LG, in_lg);
+            tc::mbar_arrive_expect_tx(MB_H, in_h);
+        }
     }
     // the injected wait: a barrier nothing completes, polled at most test_wait times; every
     // CTA gives up the same way, so the abort is uniform across the cluster
@@ -571,25 +575,17 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
     for (int t = 0; t < T && !abort; ++t) {
         float *xc = xt + (t & 1) * KX * XS, *xn = xt + ((t + 1) & 1) * KX * XS;
         const uint32_t step = p.t0 + (uint32_t)t;
-        // this step's incoming bytes on each exchange's mbarrier (phase t); every peer's bytes of
-        // phase t - 1 have been waited for, and a peer sends phase t's only after this CTA's
-        // own sends of phase t - 1, so no phase can receive early
+        // Each exchange's mbarrier completes one phase per step.  The arrive that sets a phase's
+        // expected bytes is made by the CTA's last thread (in a phase where its warp is idle),
+        // after the mbarrier's previous phase has completed: the logits' for step t + 1 during
+        // the cell of step t, the h' one during the head product, the z' one during the
+        // selection.  Peers' bytes may land before the arrive (the transaction count goes
+        // negative meanwhile); they cannot land before the previous phase completed, since a
+        // peer sends step t + 1's data only after it has this CTA's data of step t, which this
+        // CTA sends after reading its own of step t.
         const bool zx = t + 1 < T;  // the last step sends no z'
-        if (tid == 0 && CL > 1) {
-            tc::mbar_arrive_expect_tx(MB_LG, in_lg);
-            tc::mbar_arrive_expect_tx(MB_H, in_h);
-            if (zx) tc::mbar_arrive_expect_tx(MB_Z, in_z);
-        }
-        // the next step's mask words, in flight for a whole step (double buffer)
-        uint32_t *mkc = mk + (t & 1) * EB * W;
-        if (!teacher && p.mask && t + 1 < T) {
-            uint32_t *mkn = mk + ((t + 1) & 1) * EB * W;
-            for (int i = tid; i < EB * W; i += nt) {
-                const int e = i / W;
-                if (e < nv) cp4(mkn + i, p.mask + ((size_t)(t + 1) * B + b0 + e) * W + (i - e * W));
-            }
-        }
-        cp_commit();
+        const bool last_thread = tid == nt - 1 && CL > 1;
+        uint32_t *mkc = mk + (t & 1) * EB * W;  // this step's mask words (double buffer)
         // 1. gate pre-activations and logits of the rank's columns
         {
             const int ng = nt / S1, tiles = EG * CG1, gid = tid / S1, s = tid % S1;
@@ -610,7 +606,7 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
                 }
             }
         }
-        cp_wait<1>();  // all but the newest group: this step's mask words
+        cp_wait<0>();  // this step's mask words (fetched during the previous step)
         __syncthreads();
         // 2. the rank's logit rows to every CTA
         to_peers(lg + a0 * XS, na * XS / 4, CL, r, MB_LG);
@@ -620,6 +616,7 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
             break;
         }
         // 3. the action of each episode (a2), the same in every CTA
+        if (last_thread && zx) tc::mbar_arrive_expect_tx(MB_Z, in_z);  // phase t of the z' exchange
         if (warp < EB) {
             const int e = warp;
             const size_t b = (size_t)b0 + e;
@@ -663,7 +660,18 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
         } else {
             __syncthreads();
         }
-        // 4. the cell for the rank's units (a3, a4); h' into every CTA's next frame
+        // 4. the cell for the rank's units (a3, a4); h' into every CTA's next frame.  The last
+        // warp meanwhile fetches the next step's mask words (the other buffer, last read by the
+        // previous step's selection).
+        if (last_thread && t + 1 < T) tc::mbar_arrive_expect_tx(MB_LG, in_lg);  // phase t + 1
+        if (warp == nw - 1 && !teacher && p.mask && t + 1 < T) {
+            uint32_t *mkn = mk + ((t + 1) & 1) * EB * W;
+            for (int i = lane; i < EB * W; i += 32) {
+                const int e = i / W;
+                if (e < nv) cp4(mkn + i, p.mask + ((size_t)(t + 1) * B + b0 + e) * W + (i - e * W));
+            }
+            cp_commit();
+        }
         for (int i = tid; i < EB * U; i += nt) {
             const int e = i / U, uu = i - e * U, u = u0 + uu;
             if (u >= H) continue;
@@ -699,6 +707,7 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
             break;
         }
         // 5. the rank's head columns (a5)
+        if (last_thread && t + 1 < T) tc::mbar_arrive_expect_tx(MB_H, in_h);  // phase t + 1
         {
             const int ng = nt / S2, tiles = EG * CG2, gid = tid / S2, s = tid % S2;
             for (int base = 0; base < tiles; base += ng) {
