@@ -1,14 +1,14 @@
 // wm_small.cu -- the fused family's small-batch member: one launch runs all T dream steps
-// in fp32 SIMT arithmetic, one thread-block cluster per tile of 16 episodes, with the
-// model's weights resident in the cluster's shared memory.
+// in fp32 SIMT arithmetic, one thread-block cluster per tile of EB = 4, 8 or 16 episodes,
+// with the model's weights resident in the cluster's shared memory.
 //
 // It serves the models the tcgen05 member (wm_fused.cu) does not take -- the fp32 path
 // (Sec. 3.3.2's MDN-RNN evaluated in fp32) and bf16 models of other shapes, with either
 // controller (Sec. 3.4: masked argmax or tempered draw) and either reward (Sec. 3.1.4:
-// the linear head or Eq. 2) -- when the batch is small: a few waves of 16-episode tiles.
-// A tile of 16 rows is far below the M = 128 of a tensor-core MMA, and the step is bound
-// by its chain of dependent phases, so the products run on the FMA pipes: fp32 operands
-// (bf16-rounded ones for a bf16 model), fp32 accumulation (paired f32x2 FMAs).
+// the linear head or Eq. 2) -- when the batch is small: at most 4 waves of 16-episode
+// tiles.  A tile of 16 rows is far below the M = 128 of a tensor-core MMA, and the step is
+// bound by its chain of dependent phases, so the products run on the FMA pipes: fp32
+// operands (bf16-rounded ones for a bf16 model), fp32 accumulation (paired f32x2 FMAs).
 //
 // Layout of the work.  CTA r of a cluster of CL owns
 //   hidden units [r U, r U + U)                  -> 4U gate columns      (a3, a4)
@@ -16,23 +16,23 @@
 //   latent dims [r DZ, r DZ + DZ)                -> their 3K mixture columns (a5 - a7)
 // and computes the NR reward / done (/ runtime, memory) columns itself, so every CTA
 // decides reward, done and freezing for every episode of the tile without an exchange
-// (its inputs, h', are the same bits in every CTA).  Every CTA holds the operand
-// X = [z_t | h_t] of the tile transposed, X^T [k][episode] (rows of 16 + 4 floats, the
-// pad keeping the k-split lanes on distinct banks), in two frames: step t reads frame
-// t & 1 and fills the other.  Step t:
-//   1. its gate and controller columns: X W1 + b1, a 4 x 4 register tile per group of 8
-//      lanes that split k, reduced over the 8 lanes by a butterfly that leaves each lane
-//      two of the 16 sums
-//   2. its logit rows go to every CTA (DSMEM stores); cluster barrier
+// (its inputs, h', are the same bits in every CTA).  Its weight columns are packed once per
+// model into an image in the shared-memory layout and loaded per call by bulk copies.  Every
+// CTA holds the operand X = [z_t | h_t] of the tile transposed, X^T [k][episode] (rows of EB
+// plus a pad that keeps the k-split lanes on distinct banks), in two frames: step t reads
+// frame t & 1 and fills the other.  Step t:
+//   1. its gate and controller columns: X W1 + b1, a 4 x 4 register tile per group of S1
+//      lanes that split k, reduced over the group by a butterfly
+//   2. its logit rows go to every CTA
 //   3. one warp per episode: masked argmax / tempered draw over all A logits (every CTA
 //      reaches the same action, so it needs no exchange)                   (a2)
-//   4. the cell for its units; its h' rows go to every CTA's next frame; cluster barrier
-//   5. its head columns: h' W2 + b2 (16 lanes split k)
-//   6. its dims: temperature softmax, inverse-CDF component and Gaussian draw (or, when
-//      scoring, the per-dim mixture NLL); reward, done and freezing per episode; its z'
-//      rows go to every CTA's next frame; cluster barrier
-// Every thread of every CTA runs the same sequence of cluster barriers, and the kernel
-// has no other waits but the injected test wait (bounded), so it cannot hang on a peer.
+//   4. the cell for its units; its h' rows go to every CTA's next frame
+//   5. its head columns: h' W2 + b2 (S2 lanes split k)
+//   6. one warp per (episode, dim) of its dims: temperature softmax, inverse-CDF component
+//      and Gaussian draw (or, when scoring, the dim's mixture NLL); reward, done and
+//      freezing per episode; its z' rows go to every CTA's next frame
+// Exchanges are st.async DSMEM stores counted on the receivers' mbarriers; each wait is
+// bounded, and a CTA that gives up records WM_ERR_TIMEOUT and leaves the step loop.
 #include <limits.h>
 #include <math.h>
 #include <string.h>

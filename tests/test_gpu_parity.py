@@ -457,6 +457,43 @@ def test_fused_small_odd_shapes(wm, orc):
     assert r["compared"] + r["frozen_steps"] == B * T
 
 
+def test_fused_small_bf16_sampled_controller(wm, orc):
+    """The small bf16 model with a tempered-draw controller, which the tcgen05 member does not
+    take: the fused family runs it on the small-batch member (bf16-rounded operands)."""
+    cfg, w, z0, mask, B, T = synth.rollout_inputs("small_bf16", B=100, T=10)
+    cfg.update(ctrl_sample=1, ctrl_tau=0.9)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused" and m.last_launches == 1
+    r = check_rollout(g, cfg, w, z0, mask, orc=orc)
+    assert r["compared"] == B * T
+
+
+def test_fused_small_at_the_wave_limit(wm, orc):
+    """The largest batch AUTO gives the small-batch member (at most 4 waves of 16-episode
+    clusters, several tiles per SM over the call): parity on a spread of its episodes."""
+    cfg, w, z0, mask, _, T = synth.rollout_inputs("tiny_fp32", B=1, T=6)
+    m = wm.WorldModel(dict(cfg, path="auto"), w)
+    nmax = None
+    for B in range(16 * 64, 0, -16):  # find the limit by asking for the path
+        zb = synth.z0(B, cfg["z_dim"], seed=31)
+        mb = synth.mask(T, B, cfg["a_dim"], 0.5, seed=31)
+        m.rollout(_cuda(zb), 1, mask=_cuda(mb[:1]))
+        if m.last_path == "fused":
+            nmax = B
+            break
+    assert nmax is not None and nmax >= 16 * 4, nmax
+    z0 = synth.z0(nmax, cfg["z_dim"], seed=31)
+    mask = synth.mask(T, nmax, cfg["a_dim"], 0.5, seed=31)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    idx = _spread(nmax, 40)
+    r = check_rollout(_sub(g, idx), cfg, w, z0[idx], mask[:, idx], episodes=idx, orc=orc)
+    assert r["compared"] == len(idx) * T
+
+
 # ------------------------------------------------------------------ the tensor-core family
 @pytest.mark.parametrize("name,flags", [("mid_bf16", dict()), ("large_bf16", dict()),
                                         ("small_bf16", dict(mdn_tau=0.0)),
