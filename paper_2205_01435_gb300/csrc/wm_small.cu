@@ -526,8 +526,9 @@ __global__ void __launch_bounds__(MAX_THREADS, 1) k_small(const __grid_constant_
             if (r == 0 && (L < 0 || L > T)) report_status(p.status, WM_ERR_INVALID_ARG);
         }
         len[e] = L;
-        rts[e] = p.shaped && e < nv ? p.rt0[b] : 0.f;
-        mems[e] = p.shaped && e < nv ? p.mem0[b] : 0.f;
+        const bool sh = p.shaped && !teacher && e < nv;  // scoring takes no runtime / memory state
+        rts[e] = sh ? p.rt0[b] : 0.f;
+        mems[e] = sh ? p.mem0[b] : 0.f;
         nacc[e] = 0.0;
     }
     cp_wait<0>();  // step 0's mask words have landed (the barriers below publish them)

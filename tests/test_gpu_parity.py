@@ -440,6 +440,20 @@ def test_fused_small_teacher_forced_ragged(wm, orc, prec):
     check_teacher({k: np_(v) for k, v in g.items()}, o, prec)
 
 
+def test_fused_small_scores_a_shaped_reward_model(wm, orc):
+    """Scoring ignores the reward heads: a model with the runtime / memory heads of Eq. 2 scores
+    on the small-batch member (no runtime / memory inputs) as on the stepwise family."""
+    cfg = dict(synth.model_config("tiny_fp32"), reward_mode=1)
+    w = synth.weights(cfg, seed=24)
+    zs, acts, lens = synth.teacher_inputs(21, 6, cfg["z_dim"], cfg["a_dim"], seed=24, ragged=True)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    o = orc.mdn_nll(cfg, w, zs, acts, lengths=lens, want_seq=True)
+    check_teacher({k: np_(v) for k, v in g.items()}, o, "fp32")
+
+
 def test_fused_small_odd_shapes(wm, orc):
     """A model whose sizes divide nothing (Z=7, A=45, H=40, K=3): ranks own ragged slices of
     units, actions and dims, and some own none."""
@@ -752,6 +766,7 @@ def _grad_err(g, o):
 
 
 @pytest.mark.parametrize("name,prec,path,N,T", [("tiny_fp32", "fp32", "stepwise", 37, 9),
+                                                ("tiny_fp32", "fp32", "fused", 37, 9),  # small-batch member's forward
                                                 ("small_bf16", "bf16", "auto", 64, 12),
                                                 ("nll", "bf16", "tensor", 300, 10),
                                                 ("nll", "fp32", "stepwise", 64, 16),
