@@ -272,14 +272,20 @@ inline size_t al(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // Row-major GEMM on cuBLAS: C[m][n] = sum_k A(m,k) B(k,n), A(m,k) = ta ? A[k lda + m] :
 // A[m lda + k], B(k,n) = tb ? B[n ldb + k] : B[k ldb + n].  (cuBLAS is column-major: it
-// computes C^T = B^T A^T.)
+// computes C^T = B^T A^T.)  bf16 operands accumulate in fp32; fp32 operands take cuBLAS's
+// fp32 emulation on the tensor cores (each operand split into three bf16 parts, fp32-accurate
+// products), or plain fp32 where the library does not offer it.
 cublasStatus_t gemm(cublasHandle_t hb, bool bf16, bool ta, bool tb, int m, int n, int k, const void *A, long lda,
                     const void *B, long ldb, float *C, long ldc) {
     const float one = 1.f, zero = 0.f;
     const cudaDataType_t dt = bf16 ? CUDA_R_16BF : CUDA_R_32F;
-    return cublasGemmEx(hb, tb ? CUBLAS_OP_T : CUBLAS_OP_N, ta ? CUBLAS_OP_T : CUBLAS_OP_N, n, m, k, &one, B, dt,
-                        (int)ldb, A, dt, (int)lda, &zero, C, CUDA_R_32F, (int)ldc,
-                        bf16 ? CUBLAS_COMPUTE_32F : CUBLAS_COMPUTE_32F_PEDANTIC, CUBLAS_GEMM_DEFAULT);
+    auto run = [&](cublasComputeType_t ct) {
+        return cublasGemmEx(hb, tb ? CUBLAS_OP_T : CUBLAS_OP_N, ta ? CUBLAS_OP_T : CUBLAS_OP_N, n, m, k, &one, B, dt,
+                            (int)ldb, A, dt, (int)lda, &zero, C, CUDA_R_32F, (int)ldc, ct, CUBLAS_GEMM_DEFAULT);
+    };
+    if (bf16) return run(CUBLAS_COMPUTE_32F);
+    const cublasStatus_t st = run(CUBLAS_COMPUTE_32F_EMULATED_16BFX9);
+    return st == CUBLAS_STATUS_NOT_SUPPORTED ? run(CUBLAS_COMPUTE_32F_PEDANTIC) : st;
 }
 
 cudaError_t cublas_err(cublasStatus_t st) {
