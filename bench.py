@@ -677,20 +677,26 @@ def cpu_baseline(name: str, episodes: int | None, threads: int | None = None,
         cfg["reward_mode"] = 1
         rt0, mem0 = synth.shaping_state(n)
         sh = {"rt0": rt0, "mem0": mem0}
-    t0 = time.perf_counter()
-    o = oracle.rollout(cfg, w, z0[:n], mask[:, :n], T, nthreads=threads, **sh)
-    dt = time.perf_counter() - t0
+    def timed(nn, nthreads, shs):
+        """The sample's rollout, repeated until about 2 s have passed (a whole small workload
+        takes milliseconds): (outputs, seconds per repetition, repetitions)."""
+        reps, t0 = 0, time.perf_counter()
+        while True:
+            out = oracle.rollout(cfg, w, z0[:nn], mask[:, :nn], T, nthreads=nthreads, **shs)
+            reps += 1
+            dt = time.perf_counter() - t0
+            if dt >= 2.0 or reps >= 1000:
+                return out, dt / reps, reps
+
+    o, dt, reps = timed(n, threads, sh)
     n1 = max(1, n // 10)
-    sh1 = {k: v[:n1] for k, v in sh.items()}
-    t1 = time.perf_counter()
-    o1 = oracle.rollout(cfg, w, z0[:n1], mask[:, :n1], T, nthreads=1, **sh1)
-    dt1 = time.perf_counter() - t1
+    o1, dt1, reps1 = timed(n1, 1, {k: v[:n1] for k, v in sh.items()})
     return {"value": round(counted_steps(cfg, o["done"]) / dt, 2), "unit": "env-steps/s",
             "cores": threads,
             "kind": "oracle", "sample": f"{n} of {B} episodes x {T} steps of {name}, "
-                                        f"{threads} threads, {dt:.1f} s",
+                                        f"{threads} threads, {dt:.3g} s per repetition x {reps}",
             "value_1thread": round(counted_steps(cfg, o1["done"]) / dt1, 2),
-            "sample_1thread": f"{n1} episodes x {T} steps, 1 thread, {dt1:.1f} s"}
+            "sample_1thread": f"{n1} episodes x {T} steps, 1 thread, {dt1:.3g} s per repetition x {reps1}"}
 
 
 def run_reference(args) -> None:
