@@ -454,6 +454,29 @@ def test_fused_small_scores_a_shaped_reward_model(wm, orc):
     check_teacher({k: np_(v) for k, v in g.items()}, o, "fp32")
 
 
+@pytest.mark.parametrize("K,tau", [(1, 1.0), (32, 1.0), (32, 0.0), (7, 0.4)])
+def test_fused_small_mixture_sizes(wm, orc, K, tau):
+    """The mixture's warp reductions over K component lanes at the edges: one component (no
+    reduction level), a full warp of 32, an odd K; argmax (tau = 0) and tempered draws."""
+    cfg = dict(synth.model_config("tiny_fp32"), z_dim=6, a_dim=40, h_dim=48, k_mix=K, mdn_tau=tau,
+               done_terminates=1)
+    w = synth.weights(cfg, seed=25, std=0.2)
+    B, T = 21, 7
+    z0 = synth.z0(B, 6, seed=25)
+    mask = synth.mask(T, B, 40, 0.5, seed=25)
+    m = wm.WorldModel(dict(cfg, path="fused"), w)
+    g = m.rollout(_cuda(z0), T, mask=_cuda(mask), want_seq=True)
+    torch.cuda.synchronize()
+    assert m.last_path == "fused"
+    r = check_rollout(g, cfg, w, z0, mask, orc=orc)
+    assert r["compared"] + r["frozen_steps"] == B * T
+    zs, acts, lens = synth.teacher_inputs(B, T, 6, 40, seed=25, ragged=True)
+    gn = m.mdn_nll(_cuda(zs), _cuda(acts), lengths=_cuda(lens), want_seq=True)
+    torch.cuda.synchronize()
+    o = orc.mdn_nll(cfg, w, zs, acts, lengths=lens, want_seq=True)
+    check_teacher({k: np_(v) for k, v in gn.items()}, o, "fp32")
+
+
 def test_fused_small_odd_shapes(wm, orc):
     """A model whose sizes divide nothing (Z=7, A=45, H=40, K=3): ranks own ragged slices of
     units, actions and dims, and some own none."""
