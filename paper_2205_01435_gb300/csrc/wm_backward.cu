@@ -330,6 +330,11 @@ cudaError_t wm_bw_prepare(wm_handle *h) {
         cublasStatus_t st = cublasCreate(&hb);
         if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
         h->cublas = hb;
+        // fp32 GEMMs: the emulation whenever the library has it, and without the scans and
+        // patches for infinities and NaNs (every operand here is finite: activations, their
+        // gradients and the weights); where the library lacks either setting, its default
+        cublasSetEmulationStrategy(hb, CUBLAS_EMULATION_STRATEGY_EAGER);
+        cublasSetEmulationSpecialValuesSupport(hb, CUDA_EMULATION_SPECIAL_VALUES_SUPPORT_NONE);
     }
     const wm_config &c = h->cfg;
     if (c.precision == WM_BF16 && !h->bw_wzh) {
