@@ -347,6 +347,15 @@ cudaError_t wm_bw_prepare(wm_handle *h) {
         e = cudaDeviceSynchronize();
         if (e != cudaSuccess) return e;
     }
+    if (c.precision != WM_BF16 && !h->bw_wm) {
+        // W_mdn without the reward and done columns: the step layout's row stride M + NR is not a
+        // multiple of 16 bytes, which keeps cuBLAS off the tensor cores for dY = dMD W_mdn^T
+        const size_t H = c.h_dim, M = h->M;
+        cudaError_t e = cudaMalloc(&h->bw_wm, H * M * 4);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2D(h->bw_wm, M * 4, h->step.Wh, (M + h->NR) * 4, M * 4, H, cudaMemcpyDeviceToDevice);
+        if (e != cudaSuccess) return e;
+    }
     return cudaGetLastError();
 }
 
@@ -387,8 +396,8 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     // weights of the GEMMs: W_zh = the z and h rows of the gate matrix, W_mdn, W_h = W_zh's h rows
     const void *Wzh = bf ? (const void *)h->bw_wzh : (const void *)h->step.Wg;
     const long ldw = bf ? H4 : H4 + A;
-    const void *Wm = bf ? (const void *)h->bw_wm : (const void *)h->step.Wh;
-    const long ldm = bf ? M : M + h->NR;
+    const void *Wm = h->bw_wm;
+    const long ldm = M;
     const void *Wh = bf ? (const void *)((const __nv_bfloat16 *)h->bw_wzh + (size_t)Z * H4)
                         : (const void *)(h->step.Wg + (size_t)Z * (H4 + A));
     int launches = 0;

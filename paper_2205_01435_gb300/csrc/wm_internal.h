@@ -161,8 +161,9 @@ struct wm_handle {
     mutable int last_launches = 0;   // kernels launched by the last call
     mutable wm_timer timer;
     std::string err;
-    // the training step (wm_backward.cu): cuBLAS handle, bf16 copies of its GEMMs' weights,
-    // and its workspace (all created on first use)
+    // the training step (wm_backward.cu): cuBLAS handle, copies of its GEMMs' weights (bf16 for
+    // the bf16 path; W_mdn packed without the reward and done columns for the fp32 path), and its
+    // workspace (all created on first use)
     void *cublas = nullptr;
     void *bw_wzh = nullptr, *bw_wm = nullptr;
     void *bws = nullptr;
