@@ -22,9 +22,9 @@ had run on its own:
 To keep every value comparable after an excused flip, the replay takes the
 GPU's decisions downstream of the oracle's own: its action row into the LSTM,
 its h' into the heads (the second state point inside a step) and its
-components into z_{t+1}.  The oracle still reports, and is judged on, its own
-decisions.  The teacher-forced check compares the GPU's whole chain with the
-oracle's directly.
+components into z_{t+1}.  The oracle still reports its own decisions, and each
+GPU decision is checked against them.  The teacher-forced check compares the
+GPU's whole chain with the oracle's directly.
 """
 from __future__ import annotations
 
