@@ -266,11 +266,14 @@ typedef struct {
  * nll [N] is optional.  The reward, done, runtime, memory and value heads are
  * not in the loss.  On the bf16 path the operand rounding is treated as the
  * identity in the backward pass, and the backward's GEMM operands are bf16
- * (fp32 accumulation); on the fp32 path the backward's GEMMs are fp32-accurate
- * (cuBLAS's fp32 emulation on the tensor cores, each operand split into three
- * bf16 parts; plain fp32 where the library lacks it), for finite inputs and
- * weights (non-finite values are not propagated as IEEE arithmetic would), and
- * the forward is fp32-accurate (see Precision above).  The forward runs on the
+ * (fp32 accumulation); on the fp32 path the backward's batched GEMMs are
+ * fp32-accurate (cuBLAS's fp32 emulation on the tensor cores, each operand
+ * split into three bf16 parts; plain fp32 where the library lacks it), the
+ * recurrence's dH = dG_t W_h^T takes each operand as two bf16 parts and
+ * accumulates the three products hi.hi + hi.lo + lo.hi in fp32 (each product
+ * within a few 2^-18 of the fp32 one), all for finite inputs and weights
+ * (non-finite values are not propagated as IEEE arithmetic would), and the
+ * forward is fp32-accurate (see Precision above).  The forward runs on the
  * kernel family wm_mdn_nll would pick; the batched GEMMs of the backward
  * (gate activations over all N*T rows, the heads' and the recurrent input
  * gradients, the weight gradients) are cuBLAS calls, the rest (the mixture

@@ -18,9 +18,10 @@
 //   dW_z, dW_h   X^T dG (two GEMMs writing the z and h rows of the output)
 //   dW_a         per action, the sum of the dG rows that took it          (k_bw_arows)
 //   dW_mdn       Y^T dMD (one GEMM);  db_lstm, db_mdn  column sums          (k_bw_colsum)
-// The plain GEMMs are cuBLAS calls (bf16 operands and fp32 accumulation on the bf16 path,
-// fp32 without reduced-precision shortcuts on the fp32 path); the rest are the kernels
-// below.  Every reduction has a fixed order, so results are bit-reproducible.
+// The plain GEMMs are cuBLAS calls (bf16 operands and fp32 accumulation on the bf16 path;
+// on the fp32 path the library's fp32 emulation, and for the recurrence's dH one bf16 GEMM
+// over the operands' hi and lo parts, see k_bw_split3); the rest are the kernels below.
+// Every reduction has a fixed order, so results are bit-reproducible.
 #include <cublas_v2.h>
 #include <cuda_bf16.h>
 #include <math.h>
@@ -133,7 +134,7 @@ __global__ void k_bw_mdn(int N, int TT, int Z, int K, const float *__restrict__ 
 template <class T>
 __global__ void k_bw_cell(int N, int H, int t, int first, const float *__restrict__ act, const float *__restrict__ cs,
                           const float *__restrict__ dY, const float *__restrict__ dH, float *__restrict__ dC,
-                          float *__restrict__ dG, T *__restrict__ dG_op) {
+                          float *__restrict__ dG, T *__restrict__ dG_op, __nv_bfloat16 *__restrict__ dG3) {
     const size_t base = (size_t)t * N;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)N * H; i += (size_t)gridDim.x * blockDim.x) {
         const size_t n = i / H;
@@ -151,6 +152,17 @@ __global__ void k_bw_cell(int N, int H, int t, int first, const float *__restric
         T *oo = dG_op + r * 4 * H;
         o[u] = g0; o[H + u] = g1; o[2 * H + u] = g2; o[3 * H + u] = g3;
         oo[u] = to_op<T>(g0); oo[H + u] = to_op<T>(g1); oo[2 * H + u] = to_op<T>(g2); oo[3 * H + u] = to_op<T>(g3);
+        if (dG3) {  // this step's row as [hi | hi | lo] for the three-product recurrence GEMM
+            __nv_bfloat16 *q = dG3 + n * 12 * H;
+            const float gv[4] = {g0, g1, g2, g3};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const __nv_bfloat16 hi = __float2bfloat16_rn(gv[j]);
+                q[j * H + u] = hi;
+                q[4 * H + j * H + u] = hi;
+                q[8 * H + j * H + u] = __float2bfloat16_rn(gv[j] - __bfloat162float(hi));
+            }
+        }
         dC[i] = dc * fg;
     }
 }
@@ -262,6 +274,24 @@ __global__ void k_bw_cast(size_t rows, int cols, const float *__restrict__ src, 
         dst[i] = __float2bfloat16_rn(src[(i / cols) * lds + i % cols]);
 }
 
+// W_h [H, 4H] (the h rows of the gate matrix) as bf16 rows [hi | lo | hi], hi = bf16(w),
+// lo = bf16(w - hi): against a [hi | hi | lo] row of dG the K = 12H contraction is
+// hi.hi + hi.lo + lo.hi, the fp32 product up to the dropped lo.lo term and the parts'
+// residuals (a few 2^-18 of each product)
+__global__ void k_bw_split3(size_t rows, int cols, const float *__restrict__ src, long lds,
+                            __nv_bfloat16 *__restrict__ dst) {
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < rows * cols; i += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = i / cols;
+        const int k = (int)(i % cols);
+        const float w = src[r * lds + k];
+        const __nv_bfloat16 hi = __float2bfloat16_rn(w), lo = __float2bfloat16_rn(w - __bfloat162float(hi));
+        __nv_bfloat16 *d = dst + r * 3 * cols;
+        d[k] = hi;
+        d[cols + k] = lo;
+        d[2 * cols + k] = hi;
+    }
+}
+
 int grid_of(size_t n) {
     size_t g = (n + 255) / 256;
     if (g > 8192) g = 8192;
@@ -321,7 +351,8 @@ size_t wm_bw_ws(const wm_handle *h, int N, int T) {
            + al(NT * H4 * 4) + al(NT * H4 * es)                                // dG
            + 2 * al((size_t)N * H * 4)                                         // dH, dc
            + al((size_t)COLSUM_CHUNKS * part_cols * 4) + al((size_t)CHUNKS * A * H4 * 4)  // partials
-           + al(NT * 4) + al((size_t)CHUNKS * (A + 1) * 4) + 256;                  // rows sorted by action
+           + al(NT * 4) + al((size_t)CHUNKS * (A + 1) * 4)                       // rows sorted by action
+           + (es == 4 ? al((size_t)N * 3 * H4 * 2) : 0) + 256;                   // fp32: dG_t as bf16 parts
 }
 
 cudaError_t wm_bw_prepare(wm_handle *h) {
@@ -347,6 +378,15 @@ cudaError_t wm_bw_prepare(wm_handle *h) {
         e = cudaDeviceSynchronize();
         if (e != cudaSuccess) return e;
     }
+    if (c.precision != WM_BF16 && !h->bw_w3) {
+        const size_t Z = c.z_dim, A = c.a_dim, H = c.h_dim;
+        cudaError_t e = cudaMalloc(&h->bw_w3, H * 12 * H * 2);
+        if (e != cudaSuccess) return e;
+        k_bw_split3<<<grid_of(H * 4 * H), 256>>>(H, 4 * (int)H, h->step.Wg + Z * (4 * H + A), (long)(4 * H + A),
+                                                 (__nv_bfloat16 *)h->bw_w3);
+        e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return e;
+    }
     if (c.precision != WM_BF16 && !h->bw_wm) {
         // W_mdn without the reward and done columns: the step layout's row stride M + NR is not a
         // multiple of 16 bytes, which keeps cuBLAS off the tensor cores for dY = dMD W_mdn^T
@@ -363,8 +403,9 @@ void wm_bw_free(wm_handle *h) {
     if (h->cublas) cublasDestroy((cublasHandle_t)h->cublas);
     cudaFree(h->bw_wzh);
     cudaFree(h->bw_wm);
+    cudaFree(h->bw_w3);
     cudaFree(h->bws);
-    h->cublas = h->bw_wzh = h->bw_wm = h->bws = nullptr;
+    h->cublas = h->bw_wzh = h->bw_wm = h->bw_w3 = h->bws = nullptr;
     h->bws_bytes = 0;
 }
 
@@ -392,7 +433,8 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     float *part = (float *)p; p += al((size_t)COLSUM_CHUNKS * (H4 > M ? H4 : M) * 4);
     float *apart = (float *)p; p += al((size_t)CHUNKS * A * H4 * 4);
     int32_t *srows = (int32_t *)p; p += al(NT * 4);
-    int32_t *soff = (int32_t *)p;
+    int32_t *soff = (int32_t *)p; p += al((size_t)CHUNKS * (A + 1) * 4);
+    __nv_bfloat16 *dG3 = bf ? nullptr : (__nv_bfloat16 *)p;  // fp32: dG_t as [hi | hi | lo]
     // weights of the GEMMs: W_zh = the z and h rows of the gate matrix, W_mdn, W_h = W_zh's h rows
     const void *Wzh = bf ? (const void *)h->bw_wzh : (const void *)h->step.Wg;
     const long ldw = bf ? H4 : H4 + A;
@@ -427,12 +469,15 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     for (int t = TT - 1; t >= 0; --t) {
         {
             wm_ktime kt(h, WM_KERNEL_BW, s);
-            k_bw_cell<T><<<grid_of((size_t)N * H), 256, 0, s>>>(N, H, t, t == TT - 1, G, cs, dY, dH, dC, dG, dGo);
+            k_bw_cell<T><<<grid_of((size_t)N * H), 256, 0, s>>>(N, H, t, t == TT - 1, G, cs, dY, dH, dC, dG, dGo,
+                                                                  t > 0 ? dG3 : nullptr);
             ++launches;
         }
         if (t > 0) {
             wm_ktime kt(h, WM_KERNEL_BW_GEMM, s);
-            st = gemm(hb, bf, false, true, N, H, H4, dGo + (size_t)t * N * H4, H4, Wh, ldw, dH, H);
+            // fp32: bf16 operands over K = 12H (three products, fp32 accumulation)
+            st = bf ? gemm(hb, true, false, true, N, H, H4, dGo + (size_t)t * N * H4, H4, Wh, ldw, dH, H)
+                    : gemm(hb, true, false, true, N, H, 3 * H4, dG3, 3 * H4, h->bw_w3, 3 * H4, dH, H);
             ++launches;
             if (st != CUBLAS_STATUS_SUCCESS) return cublas_err(st);
         }

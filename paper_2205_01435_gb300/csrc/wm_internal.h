@@ -166,6 +166,7 @@ struct wm_handle {
     // workspace (all created on first use)
     void *cublas = nullptr;
     void *bw_wzh = nullptr, *bw_wm = nullptr;
+    void *bw_w3 = nullptr;  // fp32 path: W_h as bf16 rows [hi | lo | hi] for the recurrence GEMM
     void *bws = nullptr;
     size_t bws_bytes = 0;
 };
