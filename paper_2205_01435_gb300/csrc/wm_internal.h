@@ -90,9 +90,10 @@ struct wm_tc_weights {
     void *wc, *wg, *wa, *wh;  // W_c^T [P*A, Z+H], W_g^T [4H, Z+H], W_a [A, 4H], W_h^T [tiles*240, H]
     // fp32 path: the weights are the bf16 sums hi + lo; these are the lo parts (else null)
     void *wc_lo, *wg_lo, *wa_lo, *wh_lo;
-    // bf16 models: the gate weights, action rows and bias packed again for 128-column tiles
-    // (32 units x i|f|g|o per tile), for calls with few row tiles
+    // the gate weights, action rows and bias packed again for 128-column tiles (32 units x
+    // i|f|g|o per tile), for calls with few row tiles; the fp32 path's lo parts of the first two
     void *wg_n, *wa_n;
+    void *wg_n_lo, *wa_n_lo;
     float *bg_n;
     float *bc, *bg, *bh;
     int dims_per_tile, n_head_tiles, rd_tile, rd_col;  // reward, done (, runtime, memory) columns

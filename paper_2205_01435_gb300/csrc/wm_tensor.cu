@@ -804,6 +804,7 @@ using EpiGates = EpiGatesT<0>;
 using EpiGates2 = EpiGatesT<1>;
 using EpiGates32 = EpiGatesT<2>;
 using EpiGatesN = EpiGatesT<0, 32>;  // 128-column tiles (few row tiles)
+using EpiGates32N = EpiGatesT<2, 32>;  // the same, fp32 path (teacher-forced scoring)
 
 // ---- head epilogue: dims_per_tile latent dims, DS columns each; reward / done -----
 // Before the accumulator wait, the quadrant's 128 threads make the tile's random draws:
@@ -1914,22 +1915,35 @@ cudaError_t wm_tc_pack(wm_handle *h, const wm_weights *w) {
         if ((e = up(&T.wa_lo, wa_lo.data(), wa_lo.size() * 2)) != cudaSuccess) return e;
         if ((e = up(&T.wh_lo, wh_lo.data(), wh_lo.size() * 2)) != cudaSuccess) return e;
     }
-    if (!f32) {  // 128-column gate tiles: row n = 128 j + 32 gate + u <-> column gate H + 32 j + u
+    {  // 128-column gate tiles: row n = 128 j + 32 gate + u <-> column gate H + 32 j + u
         std::vector<__nv_bfloat16> wgn((size_t)4 * H * KX), wan((size_t)A * 4 * H);
+        std::vector<__nv_bfloat16> wgnl(f32 ? wgn.size() : 0), wanl(f32 ? wan.size() : 0);
         std::vector<float> bgn(4 * H);
+        auto lo = [&](float v, __nv_bfloat16 hi) { return bf(v - __bfloat162float(hi)); };
         for (int n = 0; n < 4 * H; ++n) {
             const int j = n / 128, gate = (n % 128) / 32, u = n % 32;
             const size_t col = (size_t)gate * H + 32 * j + u;
             for (int k = 0; k < KX; ++k) {
-                const size_t src = k < Z ? k : k + A;
-                wgn[(size_t)n * KX + k] = bf(w->W_lstm[src * 4 * H + col]);
+                const size_t src = k < Z ? k : k + A, i = (size_t)n * KX + k;
+                const float v = w->W_lstm[src * 4 * H + col];
+                wgn[i] = bf(v);
+                if (f32) wgnl[i] = lo(v, wgn[i]);
             }
             bgn[n] = w->b_lstm[col];
-            for (int a = 0; a < A; ++a) wan[(size_t)a * 4 * H + n] = bf(w->W_lstm[(size_t)(Z + a) * 4 * H + col]);
+            for (int a = 0; a < A; ++a) {
+                const size_t i = (size_t)a * 4 * H + n;
+                const float v = w->W_lstm[(size_t)(Z + a) * 4 * H + col];
+                wan[i] = bf(v);
+                if (f32) wanl[i] = lo(v, wan[i]);
+            }
         }
         if ((e = up(&T.wg_n, wgn.data(), wgn.size() * 2)) != cudaSuccess) return e;
         if ((e = up(&T.wa_n, wan.data(), wan.size() * 2)) != cudaSuccess) return e;
         if ((e = up((void **)&T.bg_n, bgn.data(), bgn.size() * 4)) != cudaSuccess) return e;
+        if (f32) {
+            if ((e = up(&T.wg_n_lo, wgnl.data(), wgnl.size() * 2)) != cudaSuccess) return e;
+            if ((e = up(&T.wa_n_lo, wanl.data(), wanl.size() * 2)) != cudaSuccess) return e;
+        }
     }
     if ((e = up(&T.wc, wc.data(), wc.size() * 2)) != cudaSuccess) return e;
     if ((e = up(&T.wg, wg.data(), wg.size() * 2)) != cudaSuccess) return e;
@@ -1983,7 +1997,7 @@ void wm_tc_free(wm_handle *h) {
     wm_tc_weights &T = h->tc;
     cudaFree(T.wc); cudaFree(T.wg); cudaFree(T.wa); cudaFree(T.wh);
     cudaFree(T.wc_lo); cudaFree(T.wg_lo); cudaFree(T.wa_lo); cudaFree(T.wh_lo);
-    cudaFree(T.wg_n); cudaFree(T.wa_n); cudaFree(T.bg_n);
+    cudaFree(T.wg_n); cudaFree(T.wa_n); cudaFree(T.bg_n); cudaFree(T.wg_n_lo); cudaFree(T.wa_n_lo);
     if (h->dead_host) cudaFreeHost(h->dead_host);
     h->dead_host = h->dead_dev = nullptr;
     for (cudaEvent_t ev : h->step_events) cudaEventDestroy(ev);
@@ -2092,13 +2106,15 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
     // a call at B = 8192), but made the long launches of B = 65536 3% slower: on below 32768.
     const bool pdl = B < 32768;
     // 128-column gate tiles when 256-column ones would leave most CTA pairs idle: few row
-    // tiles, or compacted live rows (bf16, flat actions)
+    // tiles, or compacted live rows (bf16, flat actions); on the fp32 path, scoring
     const int pairs = T.sms / 2;
-    const bool narrow = !f32 && !hier && T.wg_n && (compact || teacher || m_tiles * (H / 64) < pairs);
-    CUtensorMap mwgn, mxsn[2];
+    const bool narrow = !hier && T.wg_n &&
+                        (f32 ? teacher && T.wg_n_lo : (compact || teacher || m_tiles * (H / 64) < pairs));
+    CUtensorMap mwgn, mwgnl, mxsn[2];
     if (narrow && (!make_map(&mwgn, T.wg_n, 4 * H, KX, 64) || !make_map_x32(&mxsn[0], w.x[0], B, KX) ||
                    !make_map_x32(&mxsn[1], w.x[1], B, KX)))
         return cudaErrorInvalidValue;
+    if (narrow && f32 && !make_map(&mwgnl, T.wg_n_lo, 4 * H, KX, 64)) return cudaErrorInvalidValue;
     StepIO gio_n;  // the gate launches' parameters with the 128-column packing
     if (teacher) {  // batched scoring: the recurrence step by step, then one head GEMM
         const size_t fr = (size_t)B * KX;  // elements of one frame of operand rows
@@ -2130,16 +2146,23 @@ static cudaError_t tc_run(const wm_handle *h, int teacher, const wm_rollout_dev 
             }
             const OpMaps opg{&ma, &mwg, &mal, &mwgl};
             if (narrow) {
-                CUtensorMap msn;
+                CUtensorMap msn, msnl;
                 if (!make_map_x32(&msn, w.xall + (t + 1) * fr, B, KX)) return cudaErrorInvalidValue;
+                if (f32 && !make_map_x32(&msnl, w.xall_lo + (t + 1) * fr, B, KX)) return cudaErrorInvalidValue;
                 gio_n = io;
                 gio_n.wa = (const __nv_bfloat16 *)T.wa_n;
                 gio_n.b_gate = T.bg_n;
                 GemmGrid g2n = g2;
                 g2n.n_tiles = H / 32;
-                const OpMaps opn{&ma, &mwgn, &ma, &mwgn};
                 wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
-                e = launch_gemm<128, 1, 3, EpiGatesN, 2>(opn, mc, msn, msn, g2n, gio_n, T.sms, s, pdl);
+                if (f32) {
+                    gio_n.wa_lo = (const __nv_bfloat16 *)T.wa_n_lo;
+                    const OpMaps opn{&ma, &mwgn, &mal, &mwgnl};
+                    e = launch_gemm<128, 1, 3, EpiGates32N, 2, 3>(opn, mc, msn, msnl, g2n, gio_n, T.sms, s, pdl);
+                } else {
+                    const OpMaps opn{&ma, &mwgn, &ma, &mwgn};
+                    e = launch_gemm<128, 1, 3, EpiGatesN, 2>(opn, mc, msn, msn, g2n, gio_n, T.sms, s, pdl);
+                }
             } else {
                 wm_ktime kt(h, WM_KERNEL_TC_GATES, s);
                 if (f32) e = launch_gemm<256, 1, 2, EpiGates32, 2, 3>(opg, mc, ms, msl, g2, io, T.sms, s, pdl);
