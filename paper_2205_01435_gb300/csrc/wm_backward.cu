@@ -136,9 +136,10 @@ __global__ void k_bw_cell(int N, int H, int t, int first, const float *__restric
                           const float *__restrict__ dY, const float *__restrict__ dH, float *__restrict__ dC,
                           float *__restrict__ dG, T *__restrict__ dG_op, __nv_bfloat16 *__restrict__ dG3) {
     const size_t base = (size_t)t * N;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)N * H; i += (size_t)gridDim.x * blockDim.x) {
-        const size_t n = i / H;
-        const int u = (int)(i % H);
+    const int u = blockIdx.x * blockDim.x + threadIdx.x;  // unit; rows n over the grid's y
+    if (u >= H) return;
+    for (size_t n = blockIdx.y; n < (size_t)N; n += gridDim.y) {
+        const size_t i = n * H + u;
         const size_t r = base + n;
         const float *a = act + r * 4 * H;
         const float ig = a[u], fg = a[H + u], gg = a[2 * H + u], og = a[3 * H + u];
@@ -469,8 +470,8 @@ static cudaError_t bw_run(const wm_handle *h, int N, int TT, const float *z_seq,
     for (int t = TT - 1; t >= 0; --t) {
         {
             wm_ktime kt(h, WM_KERNEL_BW, s);
-            k_bw_cell<T><<<grid_of((size_t)N * H), 256, 0, s>>>(N, H, t, t == TT - 1, G, cs, dY, dH, dC, dG, dGo,
-                                                                  t > 0 ? dG3 : nullptr);
+            const dim3 grid((unsigned)((H + 255) / 256), (unsigned)(N < 65535 ? N : 65535));
+            k_bw_cell<T><<<grid, 256, 0, s>>>(N, H, t, t == TT - 1, G, cs, dY, dH, dC, dG, dGo, t > 0 ? dG3 : nullptr);
             ++launches;
         }
         if (t > 0) {
