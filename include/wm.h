@@ -271,7 +271,7 @@ typedef struct {
  * split into three bf16 parts; plain fp32 where the library lacks it), the
  * recurrence's dH = dG_t W_h^T takes each operand as two bf16 parts and
  * accumulates the three products hi.hi + hi.lo + lo.hi in fp32 (each product
- * within a few 2^-18 of the fp32 one), all for finite inputs and weights
+ * within 3 * 2^-16 of the fp32 one at worst), all for finite inputs and weights
  * (non-finite values are not propagated as IEEE arithmetic would), and the
  * forward is fp32-accurate (see Precision above).  The forward runs on the
  * kernel family wm_mdn_nll would pick; the batched GEMMs of the backward

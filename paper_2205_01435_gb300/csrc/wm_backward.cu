@@ -278,7 +278,7 @@ __global__ void k_bw_cast(size_t rows, int cols, const float *__restrict__ src, 
 // W_h [H, 4H] (the h rows of the gate matrix) as bf16 rows [hi | lo | hi], hi = bf16(w),
 // lo = bf16(w - hi): against a [hi | hi | lo] row of dG the K = 12H contraction is
 // hi.hi + hi.lo + lo.hi, the fp32 product up to the dropped lo.lo term and the parts'
-// residuals (a few 2^-18 of each product)
+// residuals (at most about 3 * 2^-16 of each product: bf16's unit roundoff is 2^-8)
 __global__ void k_bw_split3(size_t rows, int cols, const float *__restrict__ src, long lds,
                             __nv_bfloat16 *__restrict__ dst) {
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < rows * cols; i += (size_t)gridDim.x * blockDim.x) {
