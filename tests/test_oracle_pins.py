@@ -222,6 +222,44 @@ def test_lstm_zero_weights_closed_form(orc):
     assert np.all(out["rewards"] == 0.0) and np.all(out["done"] == 0)
 
 
+def test_zero_weight_rollout_with_mask_offset_and_resume(orc):
+    """The same closed form over a whole call with a mask, an episode offset, a resumed step
+    and a seed: every step's action is the lowest valid index of that step's mask row (equal
+    logits, ties to the lowest index), and z_{t+1} is the episode's own normals for its
+    absolute step (counter: episode_offset + b, t0 + t; block d / 4, pair (d mod 4) / 2),
+    whatever component is drawn (uniform weights, mu = 0, sigma = 1)."""
+    Z, A, H, K, B, T = 6, 40, 8, 3, 5, 6
+    off, t0, seed = 1000, 17, 9
+    cfg = _cfg(Z, A, H, K, seed=seed)
+    w = _zero_weights(Z, A, H, K)
+    rng = np.random.default_rng(5)
+    valid = rng.random((T, B, A)) < 0.15
+    valid[..., A - 1] |= ~valid.any(axis=-1)  # at least one valid action per (t, b)
+    valid[2, 1, :] = False
+    valid[2, 1, 37] = True  # the only valid action sits in the second mask word
+    mask = synth.pack_mask(valid)
+    c0 = rng.standard_normal((B, H)).astype(np.float32)
+    h0 = rng.standard_normal((B, H)).astype(np.float32)
+    z0 = rng.standard_normal((B, Z)).astype(np.float32)
+    out = orc.rollout(cfg, w, z0, mask, T, episode_offset=off, t0=t0, h0=h0, c0=c0, want_seq=True)
+    np.testing.assert_array_equal(out["actions"], valid.argmax(axis=-1))
+    assert out["actions"][2, 1] == 37
+    for t in range(T):
+        ct = c0.astype(np.float64) * 2.0 ** -(t + 1)
+        np.testing.assert_allclose(out["c_seq"][t], ct, rtol=1e-6, atol=0)
+        np.testing.assert_allclose(out["h_seq"][t], 0.5 * np.tanh(ct), rtol=1e-6, atol=1e-12)
+        for b in range(B):
+            want = []
+            for d in range(Z):
+                r = orc.draw(seed, off + b, t0 + t, 1, d // 4)
+                pair = (d % 4) // 2
+                e0, e1 = orc.box_muller(int(r[2 * pair]), int(r[2 * pair + 1]))
+                want.append(e0 if d % 2 == 0 else e1)
+            np.testing.assert_allclose(out["z"][t + 1, b], want, rtol=1e-6, atol=1e-7)
+    np.testing.assert_array_equal(out["z"][0], z0)
+    assert np.all(out["rewards"] == 0.0) and np.all(out["done"] == 0)
+
+
 # ----------------------------------------------------------------------------- heads (a5)
 @pytest.mark.parametrize("precision", ["fp32", "bf16"])
 def test_mdn_head_matches_torch_linear(orc, precision):
